@@ -1,0 +1,380 @@
+"""MoECa oracle: a plain, slow CPU statement of the branch-cached MoE layer.
+
+TEST INFRASTRUCTURE.  Only the tests, the package smoke check and the CPU
+baseline leg of the benchmark may import this module.  It shares no code with
+the CUDA path.
+
+Arithmetic is float64 (numpy).  Where floating point decides an integer -- the
+top-k expert choice and the recompute/reuse decision -- the decision is taken
+on values rounded to float32, the precision the GPU decides in; the other
+quantities stay float64.  Matrix products use numpy's matmul as a library step.
+
+Each function names the passage of the paper it follows:
+  Eq. 5 / Eq. 6   routed (and shared) MoE-FFN output, residual form
+  Eq. 7           routing set B_i^t and branch cache C_i^{t0}
+  Sec. 4.1        full-computation vs cache steps, synchronized update rule
+  Eq. 8           branch-level combine with current gate weights
+  Sec. 4.2, Eq. 9 branch matching, score s = w + l1*Delta + l2*o, s > tau
+  Eq. 10          EMA spatial activation statistic C_{e,i}
+  Eq. 11          spatial response entropy H_e and its normalisation
+  Eq. 12          expert-aware threshold tau_e = tau0 (1 + alpha (2 Hbar_e - 1))
+
+Readings where the paper is silent (each is a switch in ``Params``):
+  * gate weights: softmax over all E experts, top-k, then renormalised over
+    the k picks (``renorm_topk``);
+  * top-k order p: descending logit, ties to the lower expert id;
+  * ||h|| in o is the L2 norm over D of the unweighted cached branch output,
+    the sum runs over the token's k cached routed slots, o = 0 if it is 0;
+  * Hbar_e = H_e / ln T over all T token rows ("log_t"); an expert with an
+    all-zero statistic, or T = 1, gets Hbar = 0.5; "minmax" rescales
+    H across the layer's experts instead;
+  * C starts at 0 and is updated on every step, refresh steps included;
+  * an unmatched branch takes a cache slot whose expert is no longer routed,
+    in ascending p -> ascending q order; on a full-computation step slot = p;
+  * a reused slot keeps its cached weight w^{t0} ("keep") or takes w^t
+    ("overwrite");
+  * shared experts are recomputed on full-computation steps and for tokens
+    with a non-empty recompute set ("sync"), or always ("always");
+  * GELU is the tanh form ("tanh") or the erf form ("erf"); experts have no bias.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+_TINY = 1e-30
+
+
+@dataclass
+class Params:
+    """Hyper-parameters of MoECa (Eq. 9, Eq. 10, Eq. 12, Sec. 5.1) and readings."""
+
+    top_k: int
+    lambda1: float = 1.0
+    lambda2: float = 0.5
+    tau0: float = 0.8
+    alpha: float = 0.6
+    beta: float = 0.65
+    refresh_period: int = 0
+    renorm_topk: bool = True
+    entropy_norm: str = "log_t"        # or "minmax"
+    shared_policy: str = "sync"        # or "always"
+    reused_meta_policy: str = "keep"   # or "overwrite"
+    gelu: str = "tanh"                 # or "erf"
+
+
+# ---------------------------------------------------------------------------
+# Expert FFN (Eq. 5 / Eq. 6)
+# ---------------------------------------------------------------------------
+
+def gelu(z: np.ndarray, form: str = "tanh") -> np.ndarray:
+    """GELU; the tanh form is the DiT convention, the erf form is exact GELU."""
+    z = np.asarray(z, dtype=np.float64)
+    if form == "tanh":
+        return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
+    if form == "erf":
+        from scipy.special import erf
+        return 0.5 * z * (1.0 + erf(z / math.sqrt(2.0)))
+    raise ValueError(form)
+
+
+def expert_ffn(u_rows: np.ndarray, w1: np.ndarray, w2: np.ndarray, form: str) -> np.ndarray:
+    """FFN_e(u) = W2_e GELU(W1_e u) for each row of ``u_rows``.
+
+    w1 is [F, D] and w2 is [D, F] (rows are output features).
+    """
+    u = np.asarray(u_rows, dtype=np.float64)
+    hmid = gelu(u @ np.asarray(w1, np.float64).T, form)
+    return hmid @ np.asarray(w2, np.float64).T
+
+
+# ---------------------------------------------------------------------------
+# Routing (Eq. 7)
+# ---------------------------------------------------------------------------
+
+def router_logits(u: np.ndarray, w_gate: np.ndarray, b_gate=None) -> np.ndarray:
+    """Gate logits u W_g^T (+ b), float64, [T, E]."""
+    z = np.asarray(u, np.float64) @ np.asarray(w_gate, np.float64).T
+    if b_gate is not None:
+        z = z + np.asarray(b_gate, np.float64)[None, :]
+    return z
+
+
+def route(u, w_gate, b_gate, k: int, renorm: bool):
+    """Top-k routing set B_i^t = {(e_p, w_p)}, p = 1..k (Eq. 7).
+
+    Returns (e [T,k] int32, w [T,k] float64, near [T] float64) where ``near``
+    is the smallest gap between adjacent ranks 1..k+1 of the float32 logits,
+    relative to the token's largest |logit| (how close the choice is to a tie).
+    """
+    z = router_logits(u, w_gate, b_gate)
+    T, E = z.shape
+    if not (1 <= k <= E):
+        raise ValueError("top_k must be in [1, E]")
+    z32 = z.astype(np.float32)
+    # Descending float32 logit; the stable sort keeps ties in ascending expert id.
+    order = np.argsort(-z32, axis=1, kind="stable")
+    e_sel = order[:, :k].astype(np.int32)
+    zmax = z.max(axis=1, keepdims=True)
+    p_all = np.exp(z - zmax)
+    p_all /= p_all.sum(axis=1, keepdims=True)
+    w = np.take_along_axis(p_all, e_sel.astype(np.int64), axis=1)
+    if renorm:
+        w = w / w.sum(axis=1, keepdims=True)
+    ranks = min(k + 1, E)
+    zs = np.take_along_axis(z32.astype(np.float64), order[:, :ranks], axis=1)
+    scale = np.maximum(np.abs(z32).max(axis=1).astype(np.float64), _TINY)
+    if ranks > 1:
+        near = (zs[:, :-1] - zs[:, 1:]).min(axis=1) / scale
+    else:
+        near = np.full(T, np.inf)
+    return e_sel, w, near
+
+
+# ---------------------------------------------------------------------------
+# Expert-aware adaptive threshold (Eq. 10 - Eq. 12)
+# ---------------------------------------------------------------------------
+
+def ema_update(C: np.ndarray, e_sel: np.ndarray, beta: float) -> np.ndarray:
+    """C_{e,i} <- beta C_{e,i} + (1 - beta) 1[e in B_i]   (Eq. 10).  C is [E, T]."""
+    E, T = C.shape
+    ind = np.zeros((E, T), dtype=np.float64)
+    for i in range(T):
+        for e in e_sel[i]:
+            ind[int(e), i] = 1.0
+    return beta * np.asarray(C, np.float64) + (1.0 - beta) * ind
+
+
+def spatial_entropy(C: np.ndarray) -> np.ndarray:
+    """H_e = -sum_i P_e(i) log P_e(i), P_e(i) = C_{e,i} / sum_j C_{e,j}  (Eq. 11).
+
+    Terms with P = 0 contribute 0.  Experts with an all-zero row get NaN.
+    """
+    C = np.asarray(C, np.float64)
+    E, T = C.shape
+    H = np.full(E, np.nan)
+    for e in range(E):
+        S = C[e].sum()
+        if S <= 0.0:
+            continue
+        P = C[e] / S
+        nz = P > 0.0
+        H[e] = -np.sum(P[nz] * np.log(P[nz]))
+    return H
+
+
+def normalized_entropy(C: np.ndarray, mode: str = "log_t") -> np.ndarray:
+    """Hbar_e in [0, 1] (Eq. 11 normalisation); see the module readings."""
+    E, T = C.shape
+    H = spatial_entropy(C)
+    live = ~np.isnan(H)
+    Hbar = np.full(E, 0.5)
+    if mode == "log_t":
+        if T > 1:
+            Hbar[live] = np.clip(H[live] / math.log(T), 0.0, 1.0)
+    elif mode == "minmax":
+        if live.any():
+            lo, hi = H[live].min(), H[live].max()
+            if hi > lo:
+                Hbar[live] = (H[live] - lo) / (hi - lo)
+    else:
+        raise ValueError(mode)
+    return Hbar
+
+
+def expert_threshold(Hbar: np.ndarray, tau0: float, alpha: float) -> np.ndarray:
+    """tau_e = tau0 (1 + alpha (2 Hbar_e - 1))   (Eq. 12)."""
+    return tau0 * (1.0 + alpha * (2.0 * np.asarray(Hbar, np.float64) - 1.0))
+
+
+# ---------------------------------------------------------------------------
+# Branch matching, scoring and the recompute set (Sec. 4.2, Eq. 9)
+# ---------------------------------------------------------------------------
+
+def historical_contribution(cache_norm: np.ndarray) -> np.ndarray:
+    """o_{i,q} = ||h_{i,q}|| / sum_j ||h_{i,j}||  (Eq. 9); 0 where the sum is 0."""
+    n = np.asarray(cache_norm, np.float64)
+    s = n.sum(axis=1, keepdims=True)
+    return np.where(s > 0.0, n / np.where(s > 0.0, s, 1.0), 0.0)
+
+
+def select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, lambda1, lambda2,
+                    refresh: bool):
+    """Partition B_i^t into the recompute set R_i^t and the reuse set.
+
+    Returns a dict of [T, k] arrays:
+      recompute (bool), slot (int32: cache slot that holds branch p after the
+      step), matched (bool), score (float64, NaN if unmatched) and margin
+      (|s - tau| / |tau|, inf where no threshold decides).
+    """
+    e_cur = np.asarray(e_cur)
+    T, k = e_cur.shape
+    recompute = np.ones((T, k), dtype=bool)
+    slot = np.tile(np.arange(k, dtype=np.int32), (T, 1))
+    matched = np.zeros((T, k), dtype=bool)
+    score = np.full((T, k), np.nan)
+    margin = np.full((T, k), np.inf)
+    if refresh:
+        return dict(recompute=recompute, slot=slot, matched=matched, score=score, margin=margin)
+    o = historical_contribution(cache_norm)
+    tau = np.asarray(tau, np.float64)
+    for i in range(T):
+        q_of = [-1] * k
+        for p in range(k):
+            e = int(e_cur[i, p])
+            hits = [q for q in range(k) if int(cache_e[i, q]) == e]
+            if not hits:
+                continue          # unmatched: no cached state for this expert
+            q = hits[0]
+            q_of[p] = q
+            matched[i, p] = True
+            w = float(w_cur[i, p])
+            delta = abs(w - float(cache_w[i, q]))
+            s = w + lambda1 * delta + lambda2 * float(o[i, q])
+            score[i, p] = s
+            t = float(tau[e])
+            recompute[i, p] = bool(np.float32(s) > np.float32(t))
+            if math.isfinite(t):
+                margin[i, p] = abs(s - t) / max(abs(t), _TINY)
+        # Matched branches keep their slot; unmatched ones take the freed slots.
+        free = [q for q in range(k) if q not in q_of]
+        unmatched = [p for p in range(k) if q_of[p] < 0]
+        for p in range(k):
+            if q_of[p] >= 0:
+                slot[i, p] = q_of[p]
+        for p, q in zip(unmatched, free):
+            slot[i, p] = q
+    return dict(recompute=recompute, slot=slot, matched=matched, score=score, margin=margin)
+
+
+# ---------------------------------------------------------------------------
+# Layer state and one step of a layer
+# ---------------------------------------------------------------------------
+
+@dataclass
+class LayerState:
+    """Per-layer cache (Eq. 7) and EMA statistic (Eq. 10) for T token rows."""
+
+    cache_e: np.ndarray        # [T, k] int32   e_{i,q}^{t0}
+    cache_w: np.ndarray        # [T, k] float64 w_{i,q}^{t0}
+    cache_norm: np.ndarray     # [T, k] float64 ||h_{i,q}^{t0}||
+    cache_h: np.ndarray        # [T, k, D] float64 h_{i,q}^{t0}
+    shared_h: np.ndarray | None  # [T, D] float64, shared-expert output
+    C: np.ndarray              # [E, T] float64 C_{e,i}
+    valid: bool = False
+
+    @staticmethod
+    def empty(T: int, D: int, E: int, k: int, n_shared: int) -> "LayerState":
+        return LayerState(
+            cache_e=np.full((T, k), -1, np.int32), cache_w=np.zeros((T, k)),
+            cache_norm=np.zeros((T, k)), cache_h=np.zeros((T, k, D)),
+            shared_h=np.zeros((T, D)) if n_shared else None, C=np.zeros((E, T)), valid=False)
+
+    def copy(self) -> "LayerState":
+        return LayerState(self.cache_e.copy(), self.cache_w.copy(), self.cache_norm.copy(),
+                          self.cache_h.copy(), None if self.shared_h is None else self.shared_h.copy(),
+                          self.C.copy(), self.valid)
+
+
+def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, refresh: bool):
+    """One MoE layer at one denoising step; returns (out [T, D], new state, info).
+
+    Order of work: route (Eq. 7) -> EMA (Eq. 10) -> entropy and tau (Eq. 11-12)
+    -> match, score, decide (Eq. 9) -> recompute R (Eq. 5) -> shared experts
+    under the synchronized rule (Sec. 4.1) -> combine with current gate weights
+    (Eq. 8) plus the residual (Eq. 5 / 6) -> refresh the cached norms.
+    """
+    u = np.asarray(u, np.float64)
+    T, D = u.shape
+    k = prm.top_k
+    e_cur, w_cur, near = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
+    C = ema_update(state.C, e_cur, prm.beta)
+    Hbar = normalized_entropy(C, prm.entropy_norm)
+    tau = expert_threshold(Hbar, prm.tau0, prm.alpha)
+    sel = select_branches(e_cur, w_cur, state.cache_e, state.cache_w, state.cache_norm, tau,
+                          prm.lambda1, prm.lambda2, refresh)
+    new = state.copy()
+    new.C = C
+    rec, slot = sel["recompute"], sel["slot"]
+    # Recompute the branches of R, one expert's rows at a time.
+    for e in np.unique(e_cur[rec]):
+        rows = np.argwhere(rec & (e_cur == e))
+        h = expert_ffn(u[rows[:, 0]], weights["w1"][e], weights["w2"][e], prm.gelu)
+        for (i, p), hv in zip(rows, h):
+            q = slot[i, p]
+            new.cache_h[i, q] = hv
+            new.cache_e[i, q] = e
+            new.cache_w[i, q] = w_cur[i, p]
+    if prm.reused_meta_policy == "overwrite":
+        for i, p in np.argwhere(~rec):
+            new.cache_w[i, slot[i, p]] = w_cur[i, p]
+    token_any = rec.any(axis=1)
+    ws1 = weights.get("ws1")
+    if ws1 is not None and len(ws1):
+        if refresh or prm.shared_policy == "always":
+            rows = np.arange(T)
+        else:
+            rows = np.nonzero(token_any)[0]
+        if len(rows):
+            acc = np.zeros((len(rows), D))
+            for s in range(len(ws1)):
+                acc += expert_ffn(u[rows], ws1[s], weights["ws2"][s], prm.gelu)
+            new.shared_h[rows] = acc
+    # Eq. 8: every current branch p reads slot(p), fresh or cached, with w^t.
+    y = np.zeros((T, D))
+    for p in range(k):
+        y += w_cur[:, p:p + 1] * new.cache_h[np.arange(T), slot[:, p]]
+    if new.shared_h is not None:
+        y += new.shared_h
+    out = u + y
+    new.cache_norm = np.sqrt(np.sum(new.cache_h ** 2, axis=2))
+    new.valid = True
+    info = dict(e=e_cur, w=w_cur, near_route=near, C=C, Hbar=Hbar, tau=tau,
+                token_any=token_any, refresh=refresh, **sel)
+    return out, new, info
+
+
+def stats_of(info: dict) -> dict:
+    """Branch counts of one layer step (Fig. 8's reuse-over-match ratio inputs)."""
+    rec, matched = info["recompute"], info["matched"]
+    return dict(branches=int(rec.size), matched=int(matched.sum()),
+                recomputed=int(rec.sum()), reused=int((~rec).sum()),
+                tokens_fully_reused=int((~info["token_any"]).sum()))
+
+
+class Stack:
+    """A stack of L MoE layers run over denoising steps (Sec. 4.1 schedule).
+
+    A step is a full-computation step when it is forced, when the caches are
+    not valid or the token count changed, or when ``refresh_period`` N > 0
+    divides the step index; otherwise it is a cache step.
+    """
+
+    def __init__(self, layers: list, prm: Params, hidden: int, n_experts: int, n_shared: int = 0):
+        self.layers = layers
+        self.prm = prm
+        self.D, self.E, self.S = hidden, n_experts, n_shared
+        self.states = None
+        self.T = None
+
+    def is_refresh(self, step_index: int, n_tokens: int, force: bool = False) -> bool:
+        N = self.prm.refresh_period
+        return bool(force or self.states is None or n_tokens != self.T
+                    or not all(s.valid for s in self.states)
+                    or (N > 0 and step_index % N == 0))
+
+    def step(self, x: np.ndarray, step_index: int, force: bool = False):
+        x = np.asarray(x, np.float64)
+        T = x.shape[0]
+        refresh = self.is_refresh(step_index, T, force)
+        if self.states is None or T != self.T:
+            self.states = [LayerState.empty(T, self.D, self.E, self.prm.top_k, self.S)
+                           for _ in self.layers]
+            self.T = T
+        infos = []
+        for l, w in enumerate(self.layers):
+            x, self.states[l], info = layer_step(self.states[l], x, w, self.prm, refresh)
+            infos.append(info)
+        return x, infos

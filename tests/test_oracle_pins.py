@@ -1,0 +1,266 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a closed form,
+a special case, an invariant of the definitions, a textbook formulation written
+independently (dense einsum MoE), or exact reuse.  The brute-force and
+hand-worked fixture pins live in their own files.
+"""
+import math
+
+import numpy as np
+import pytest
+
+from oracle import moeca_oracle as O
+from paper_2606_15615_gb300.workloads import tiny_layer
+
+
+def _softmax_rows(z):
+    z = z - z.max(axis=1, keepdims=True)
+    ez = np.exp(z)
+    return ez / ez.sum(axis=1, keepdims=True)
+
+
+def _gelu_tanh(z):
+    return 0.5 * z * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (z + 0.044715 * z ** 3)))
+
+
+def textbook_moe(u, w, k):
+    """Eq. 5 / Eq. 6 as a dense computation: every expert on every token, then gated.
+
+    Independent of the oracle: einsum over all experts, top-k by lexsort.
+    """
+    u = u.astype(np.float64)
+    z = np.einsum("td,ed->te", u, w["w_gate"].astype(np.float64))
+    if w.get("b_gate") is not None:
+        z = z + w["b_gate"][None, :]
+    T, E = z.shape
+    z32 = z.astype(np.float32)
+    gate = np.zeros((T, E))
+    probs = _softmax_rows(z)
+    for t in range(T):
+        order = np.lexsort((np.arange(E), -z32[t]))[:k]
+        g = probs[t, order] / probs[t, order].sum()
+        gate[t, order] = g
+    hid = _gelu_tanh(np.einsum("td,efd->tef", u, w["w1"].astype(np.float64)))
+    outs = np.einsum("tef,edf->ted", hid, w["w2"].astype(np.float64))
+    y = np.einsum("te,ted->td", gate, outs)
+    if w.get("ws1") is not None:
+        hs = _gelu_tanh(np.einsum("td,sfd->tsf", u, w["ws1"].astype(np.float64)))
+        y = y + np.einsum("tsf,sdf->td", hs, w["ws2"].astype(np.float64))
+    return u + y
+
+
+# --- Routing (Eq. 7) --------------------------------------------------------
+
+def test_topk_weights_renormalised_sum_to_one():
+    w, x, _ = tiny_layer(1, T=64, D=16, E=8, k=3, F=8, bias=True)
+    e, wt, _ = O.route(x, w["w_gate"], w["b_gate"], 3, renorm=True)
+    np.testing.assert_allclose(wt.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+    assert (wt[:, :-1] >= wt[:, 1:] - 1e-15).all(), "branches are ordered by descending weight"
+    for row in e:
+        assert len(set(row.tolist())) == 3
+
+
+def test_topk_without_renorm_keeps_softmax_ratios():
+    # Softmax fixes w_p / w_p' = exp(z_p - z_p') and sum over all E of p = 1.
+    w, x, _ = tiny_layer(2, T=32, D=12, E=6, k=2, F=4)
+    e, wt, _ = O.route(x, w["w_gate"], None, 2, renorm=False)
+    z = x.astype(np.float64) @ w["w_gate"].astype(np.float64).T
+    for t in range(32):
+        np.testing.assert_allclose(wt[t, 0] / wt[t, 1], math.exp(z[t, e[t, 0]] - z[t, e[t, 1]]), rtol=1e-12)
+        assert wt[t].sum() < 1.0
+    np.testing.assert_allclose(O.route(x, w["w_gate"], None, 6, renorm=False)[1].sum(axis=1), 1.0, atol=1e-12)
+
+
+def test_topk_ties_go_to_lower_expert_id():
+    wg = np.array([[1.0, 0.0], [1.0, 0.0], [0.5, 0.0], [1.0, 0.0]])
+    e, wt, near = O.route(np.array([[2.0, 1.0]]), wg, None, 2, renorm=True)
+    assert e.tolist() == [[0, 1]]
+    np.testing.assert_allclose(wt, [[0.5, 0.5]])
+    assert near[0] == 0.0
+
+
+# --- EMA, entropy, threshold (Eq. 10-12) ------------------------------------
+
+@pytest.mark.parametrize("beta", [0.45, 0.65, 0.85])
+def test_ema_closed_form(beta):
+    # Routed for n steps from C = 0: C = 1 - beta^n; then unrouted m steps: times beta^m.
+    C = np.zeros((2, 1))
+    for n in range(1, 9):
+        C = O.ema_update(C, np.array([[0]]), beta)
+        assert C[0, 0] == pytest.approx(1.0 - beta ** n, rel=1e-12)
+        assert C[1, 0] == 0.0
+    for m in range(1, 5):
+        C = O.ema_update(C, np.array([[1]]), beta)
+        assert C[0, 0] == pytest.approx((1.0 - beta ** 8) * beta ** m, rel=1e-12)
+        assert C[1, 0] == pytest.approx(1.0 - beta ** m, rel=1e-12)
+
+
+def test_threshold_special_cases():
+    T = 16
+    uniform = np.full((1, T), 0.3)
+    onehot = np.zeros((1, T)); onehot[0, 5] = 0.9
+    rng = np.random.default_rng(0)
+    rand = rng.random((3, T))
+    for tau0, alpha in [(0.8, 0.6), (0.65, 0.3), (1.0, 0.9)]:
+        assert O.expert_threshold(O.normalized_entropy(uniform), tau0, alpha)[0] == pytest.approx(tau0 * (1 + alpha))
+        assert O.expert_threshold(O.normalized_entropy(onehot), tau0, alpha)[0] == pytest.approx(tau0 * (1 - alpha))
+        np.testing.assert_allclose(O.expert_threshold(O.normalized_entropy(rand), tau0, 0.0), tau0)
+    Hbar = O.normalized_entropy(rand)
+    assert ((Hbar > 0) & (Hbar < 1)).all()
+
+
+def test_entropy_two_point_and_scale_invariance():
+    # Mass split evenly over m positions gives H = ln m, whatever the scale of C.
+    for m in (1, 2, 3, 7):
+        C = np.zeros((1, 10)); C[0, :m] = 0.123
+        assert O.spatial_entropy(C)[0] == pytest.approx(math.log(m), abs=1e-12)
+        assert O.spatial_entropy(5.0 * C)[0] == pytest.approx(math.log(m), abs=1e-12)
+
+
+def test_entropy_minmax_mode():
+    C = np.array([[1.0, 0, 0, 0], [1.0, 1.0, 0, 0], [1.0, 1.0, 1.0, 1.0], [0, 0, 0, 0]])
+    np.testing.assert_allclose(O.normalized_entropy(C, "minmax"), [0.0, 0.5, 1.0, 0.5])
+
+
+# --- Scoring and selection (Eq. 9) ------------------------------------------
+
+def test_historical_contribution_sums_to_one():
+    n = np.abs(np.random.default_rng(3).standard_normal((50, 4)))
+    n[7] = 0.0
+    o = O.historical_contribution(n)
+    np.testing.assert_allclose(np.delete(o, 7, axis=0).sum(axis=1), 1.0, atol=1e-12)
+    assert (o[7] == 0).all()
+
+
+def _run(layer_w, prm, xs, n_shared=0):
+    D = xs[0].shape[1]
+    E = layer_w["w_gate"].shape[0]
+    st = O.Stack([layer_w], prm, D, E, n_shared)
+    outs, infos = [], []
+    for t, x in enumerate(xs):
+        o, inf = st.step(x, t)
+        outs.append(o)
+        infos.append(inf[0])
+    return outs, infos, st
+
+
+def test_identical_input_matches_every_branch_with_zero_drift():
+    w, x, _ = tiny_layer(4, T=40, D=16, E=6, k=2, F=8)
+    prm = O.Params(top_k=2, tau0=0.8)
+    st = O.Stack([w], prm, 16, 6)
+    st.step(x, 0)
+    norms_before = st.states[0].cache_norm.copy()
+    _, infos = st.step(x, 1)
+    inf = infos[0]
+    assert inf["matched"].all()
+    o = O.historical_contribution(norms_before)[np.arange(40)[:, None], inf["slot"]]
+    # Same routing, so Delta = 0 and s = w + lambda2 * o.
+    np.testing.assert_allclose(inf["score"], inf["w"] + prm.lambda2 * o, rtol=1e-12)
+
+
+def test_reuse_disabled_equals_textbook_moe():
+    # tau0 = -inf recomputes every branch on every step: Eq. 5 at each step.
+    w, x0, rng = tiny_layer(5, T=48, D=16, E=5, k=2, F=12, bias=True)
+    prm = O.Params(top_k=2, tau0=-math.inf)
+    xs = [x0 + 0.1 * t * rng.standard_normal(x0.shape).astype(np.float32) for t in range(4)]
+    outs, infos, _ = _run(w, prm, xs)
+    for x, o, inf in zip(xs, outs, infos):
+        assert inf["recompute"].all()
+        np.testing.assert_allclose(o, textbook_moe(x, w, 2), rtol=1e-12, atol=1e-12)
+
+
+def test_reuse_disabled_with_shared_expert_equals_textbook_moe():
+    w, x0, rng = tiny_layer(6, T=32, D=8, E=4, k=2, F=6, n_shared=1)
+    prm = O.Params(top_k=2, tau0=-math.inf)
+    xs = [x0, x0 + 0.2 * rng.standard_normal(x0.shape).astype(np.float32)]
+    outs, _, _ = _run(w, prm, xs, n_shared=1)
+    for x, o in zip(xs, outs):
+        np.testing.assert_allclose(o, textbook_moe(x, w, 2), rtol=1e-12, atol=1e-12)
+
+
+def test_refresh_every_step_equals_textbook_moe():
+    w, x0, rng = tiny_layer(7, T=32, D=8, E=4, k=2, F=6)
+    prm = O.Params(top_k=2, tau0=10.0, refresh_period=1)
+    xs = [x0 + 0.3 * t * rng.standard_normal(x0.shape).astype(np.float32) for t in range(3)]
+    outs, infos, _ = _run(w, prm, xs)
+    for x, o, inf in zip(xs, outs, infos):
+        assert inf["refresh"]
+        np.testing.assert_allclose(o, textbook_moe(x, w, 2), rtol=1e-12, atol=1e-12)
+
+
+def test_everything_reused_returns_cached_output_exactly():
+    w, x, _ = tiny_layer(8, T=40, D=16, E=6, k=3, F=8, n_shared=1)
+    prm = O.Params(top_k=3, tau0=math.inf)
+    outs, infos, _ = _run(w, prm, [x, x, x], n_shared=1)
+    assert not infos[1]["recompute"].any() and not infos[2]["recompute"].any()
+    assert np.array_equal(outs[1], outs[0]) and np.array_equal(outs[2], outs[0])
+
+
+def test_slots_are_a_permutation_and_cache_holds_current_experts():
+    w, x0, rng = tiny_layer(9, T=64, D=16, E=8, k=3, F=8)
+    prm = O.Params(top_k=3, tau0=0.9)
+    xs = [x0 + 0.5 * t * rng.standard_normal(x0.shape).astype(np.float32) for t in range(5)]
+    outs, infos, st = _run(w, prm, xs)
+    saw_unmatched = saw_reuse = False
+    for inf in infos:
+        for i in range(64):
+            assert sorted(inf["slot"][i].tolist()) == [0, 1, 2]
+        saw_unmatched |= bool((~inf["matched"] & ~np.array(inf["refresh"])).any())
+        saw_reuse |= bool((~inf["recompute"]).any())
+    assert saw_unmatched and saw_reuse
+    last = infos[-1]
+    state = st.states[0]
+    for i in range(64):
+        for p in range(3):
+            assert state.cache_e[i, last["slot"][i, p]] == last["e"][i, p]
+
+
+def test_recomputed_branch_equals_fresh_ffn_and_reused_keeps_old_weight():
+    w, x0, rng = tiny_layer(10, T=64, D=16, E=6, k=2, F=8)
+    prm = O.Params(top_k=2, tau0=0.75)
+    xs = [x0, x0 + 0.05 * rng.standard_normal(x0.shape).astype(np.float32)]
+    outs, infos, st = _run(w, prm, xs)
+    inf, state = infos[1], st.states[0]
+    rec = inf["recompute"]
+    assert rec.any() and (~rec).any()
+    for i, p in np.argwhere(rec):
+        e = inf["e"][i, p]
+        h = O.gelu(xs[1][i].astype(np.float64) @ w["w1"][e].T.astype(np.float64)) @ w["w2"][e].T.astype(np.float64)
+        np.testing.assert_allclose(state.cache_h[i, inf["slot"][i, p]], h, rtol=1e-12)
+        assert state.cache_w[i, inf["slot"][i, p]] == inf["w"][i, p]
+    for i, p in np.argwhere(~rec):
+        q = inf["slot"][i, p]
+        assert state.cache_w[i, q] == infos[0]["w"][i, q]  # kept w^{t0}
+
+
+def test_shared_expert_follows_synchronized_rule():
+    w, x0, rng = tiny_layer(11, T=64, D=8, E=4, k=2, F=6, n_shared=1)
+    prm = O.Params(top_k=2, tau0=0.9)
+    x1 = x0 + 0.05 * rng.standard_normal(x0.shape).astype(np.float32)
+    outs, infos, st = _run(w, prm, [x0, x1], n_shared=1)
+    any1 = infos[1]["token_any"]
+    assert any1.any() and (~any1).any()
+    fresh = O.expert_ffn(x1.astype(np.float64), w["ws1"][0], w["ws2"][0], "tanh")
+    old = O.expert_ffn(x0.astype(np.float64), w["ws1"][0], w["ws2"][0], "tanh")
+    np.testing.assert_allclose(st.states[0].shared_h[any1], fresh[any1], rtol=1e-12)
+    np.testing.assert_allclose(st.states[0].shared_h[~any1], old[~any1], rtol=1e-12)
+
+
+def test_reused_meta_overwrite_policy():
+    w, x0, rng = tiny_layer(12, T=48, D=8, E=4, k=2, F=6)
+    prm = O.Params(top_k=2, tau0=0.9, reused_meta_policy="overwrite")
+    x1 = x0 + 0.05 * rng.standard_normal(x0.shape).astype(np.float32)
+    _, infos, st = _run(w, prm, [x0, x1])
+    inf = infos[1]
+    for i, p in np.argwhere(~inf["recompute"]):
+        assert st.states[0].cache_w[i, inf["slot"][i, p]] == inf["w"][i, p]
+
+
+def test_refresh_schedule():
+    w, x, _ = tiny_layer(13, T=8, D=8, E=4, k=2, F=4)
+    st = O.Stack([w], O.Params(top_k=2, refresh_period=3), 8, 4)
+    flags = [st.step(x, t)[1][0]["refresh"] for t in range(7)]
+    assert flags == [True, False, False, True, False, False, True]
+    assert st.step(x[:5], 7)[1][0]["refresh"], "a new token count forces a full step"
+    assert st.step(x[:5], 8, force=True)[1][0]["refresh"]
