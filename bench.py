@@ -1,0 +1,500 @@
+#!/usr/bin/env python3
+"""Benchmark of the GB300 branch-cached MoE layer stack (MoECa).
+
+A step is one denoising step of the whole stack (every layer: router, select,
+compact, grouped FFN x2, combine) over one batch of synthetic tokens.  The
+default workload is the 12-layer stack D 768, E 16, top-2, F 3072, T 2048
+(8 x 256 tokens) in bf16, driven along its seeded drift trajectory.  The
+headline value is tokens/s at the 60% branch-reuse point (tau0 calibrated on
+the GPU path itself); the same line carries the sweep over reuse 0/30/60/90%,
+end-to-end numbers with host buffers, a roofline entry for the dominant kernel,
+the oracle's CPU baseline, and the SM clocks sampled during the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank runs its own replica (the path shares nothing
+between GPUs); the time is the max over ranks and the value sums the tokens.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "branch-cached MoE layer tokens/s and effective TFLOP/s vs reuse ratio; % roofline"
+DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine"]
+
+
+# ---------------------------------------------------------------------------
+# ranks
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_group(world: int, backend: str):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    if not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def aggregate(elapsed_ms: float, tokens: int, dist, device=None):
+    """Max time and summed tokens over ranks (barrier-bracketed timing)."""
+    if dist is None:
+        return elapsed_ms, tokens
+    import torch
+    t = torch.tensor([elapsed_ms], dtype=torch.float64, device=device)
+    n = torch.tensor([float(tokens)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        import tempfile
+        fd, self.path = tempfile.mkstemp(prefix="moeca_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", self.gpu_id], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1])]
+        mx = [num(r[2]) for r in rows if num(r[2])]
+        pw = [num(r[3]) for r in rows if num(r[3])]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for r in rows for j in range(4) if r[5 + j].lower() == "active"})
+        load = [s for s, p in zip(sm, pw) if pw and p > 0.5 * max(pw)] or sm
+        return {"sm_mhz": statistics.median(load) if load else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def gpu_smi_id(dev_index: int) -> str:
+    import torch
+    try:
+        u = str(torch.cuda.get_device_properties(dev_index).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return str(dev_index)
+
+
+# ---------------------------------------------------------------------------
+# peaks, traffic
+# ---------------------------------------------------------------------------
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_source_sha(kind: str) -> str:
+    fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
+             "compact": "select.cu", "combine": "combine.cu"}[kind]
+    with open(os.path.join(ROOT, "paper_2606_15615_gb300", "csrc", fname), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def recorded_traffic(kind: str, workload: str, reuse_target: float):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel is unchanged."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    for e in d.get("entries", []):
+        if (e.get("kernel") == kind and e.get("workload") == workload
+                and abs(e.get("reuse_target", -1) - reuse_target) < 1e-6
+                and e.get("source_sha") == kernel_source_sha(kind)):
+            return e.get("dram_bytes_per_launch")
+    return None
+
+
+# ---------------------------------------------------------------------------
+# the GPU runner
+# ---------------------------------------------------------------------------
+
+class Runner:
+    def __init__(self, wl, device_index: int, n_steps: int):
+        import numpy as np
+        import torch
+        from paper_2606_15615_gb300 import build
+        build.build()
+        from paper_2606_15615_gb300 import moeca as M
+        from paper_2606_15615_gb300 import workloads as W
+        self.torch, self.M, self.W, self.np = torch, M, W, np
+        self.wl = wl
+        self.dev = torch.device("cuda", device_index)
+        torch.cuda.set_device(self.dev)
+        self.weights = [W.make_layer_weights_device(wl, l, self.dev) for l in range(wl.n_layers)]
+        cfg = M.moeca_config_default(
+            n_layers=wl.n_layers, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts, top_k=wl.top_k,
+            n_shared=wl.n_shared, max_tokens=wl.n_tokens,
+            dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period)
+        self.cfg = cfg
+        self.stack = M.Stack(cfg, self.weights, device=device_index)
+        dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+        self.dt = dt
+        xs = [torch.from_numpy(x) for x in W.trajectory(wl, n_steps)]
+        self.x_host = torch.stack(xs).to(dt).pin_memory()
+        self.x_dev = self.x_host.to(self.dev)
+        T, D = wl.n_tokens, wl.hidden
+        self.out = torch.empty((T, D), dtype=dt, device=self.dev)
+        self.in_buf = torch.empty((T, D), dtype=dt, device=self.dev)
+        self.out_host = torch.empty((T, D), dtype=dt).pin_memory()
+        self.stream = torch.cuda.current_stream(self.dev)
+
+    def _run(self, tau0, W_, K, kernel_timing=False, e2e=False):
+        torch, M = self.torch, self.M
+        h = self.stack.handle
+        M.moeca_reset(h)
+        M.moeca_set_kernel_timing(h, False)
+        sp = self.stream.cuda_stream
+        T = self.wl.n_tokens
+        for t in range(W_):
+            M.moeca_step(h, self.x_dev[t].data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
+        torch.cuda.synchronize(self.dev)
+        M.moeca_reset_stats(h)
+        if kernel_timing:
+            M.moeca_get_kernel_times(h, reset=True)
+            M.moeca_set_kernel_timing(h, True)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(self.stream)
+        for t in range(W_, W_ + K):
+            if e2e:
+                self.in_buf.copy_(self.x_host[t], non_blocking=True)
+                M.moeca_step(h, self.in_buf.data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
+                self.out_host.copy_(self.out, non_blocking=True)
+            else:
+                M.moeca_step(h, self.x_dev[t].data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
+        e1.record(self.stream)
+        torch.cuda.synchronize(self.dev)
+        ms = e0.elapsed_time(e1)
+        kt = None
+        if kernel_timing:
+            M.moeca_set_kernel_timing(h, False)
+            kt = M.moeca_get_kernel_times(h, reset=True)
+        st = M.moeca_get_stats(h)
+        return ms, st, kt
+
+    def reuse_of(self, st) -> float:
+        return st["reused"] / max(st["branches"], 1)
+
+    def calibrate(self, target: float, W_, K) -> tuple:
+        """tau0 whose reuse over the timed window is closest to ``target`` (bisection)."""
+        if target <= 0.0:
+            _, st, _ = self._run(-math.inf, W_, K)
+            return -math.inf, self.reuse_of(st)
+        lo, hi = 0.0, 4.0
+        _, st_hi, _ = self._run(hi, W_, K)
+        if self.reuse_of(st_hi) <= target:
+            return hi, self.reuse_of(st_hi)
+        best = (hi, self.reuse_of(st_hi))
+        for _ in range(14):
+            mid = 0.5 * (lo + hi)
+            _, st, _ = self._run(mid, W_, K)
+            r = self.reuse_of(st)
+            if abs(r - target) < abs(best[1] - target):
+                best = (mid, r)
+            if r < target:
+                lo = mid
+            else:
+                hi = mid
+        return best
+
+
+def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float):
+    """Algorithmic (bytes, flops) of one launch of a kernel kind for this workload."""
+    T, D, E, k, F, S = wl.n_tokens, wl.hidden, wl.n_experts, wl.top_k, wl.ffn, wl.n_shared
+    es = 2 if wl.dtype == "bf16" else 4
+    if kind == "router":
+        return T * D * es + E * D * es + T * E * 8 + T * k * 8, 2.0 * T * D * E
+    if kind == "select":
+        return T * k * (8 + 12 + 8 + 3) + T, 0.0
+    if kind == "compact":
+        return T * k * 6 + T + rows_per_launch * (4 + 2 * D * es), 0.0
+    if kind == "ffn1":
+        return active_groups * F * D * es + rows_per_launch * (D + F) * es, 2.0 * rows_per_launch * D * F
+    if kind == "ffn2":
+        return active_groups * F * D * es + rows_per_launch * (F + D) * es, 2.0 * rows_per_launch * D * F
+    if kind == "combine":
+        return T * D * es * (2 + k + S) + T * k * 9, 0.0
+    raise KeyError(kind)
+
+
+def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
+    """The oracle on this host's cores: full-T cache steps of layer 0, extrapolated to L layers."""
+    import numpy as np
+    from oracle import moeca_oracle as O
+    torch = runner.torch
+    w = {k: (None if v is None else v.float().cpu().numpy().astype(np.float64)) for k, v in runner.weights[0].items()}
+    if w["ws1"] is None:
+        w["ws1"] = w["ws2"] = None
+    prm = O.Params(top_k=wl.top_k, tau0=tau0 if math.isfinite(tau0) else tau0, refresh_period=wl.refresh_period)
+    st = O.Stack([w], prm, wl.hidden, wl.n_experts, wl.n_shared)
+    xs = runner.x_host.float().numpy()
+    st.step(xs[0], 0)
+    times = []
+    t_all = time.perf_counter()
+    for t in range(1, xs.shape[0]):
+        if wl.refresh_period and t % wl.refresh_period == 0:
+            st.step(xs[t], t)
+            continue
+        t0 = time.perf_counter()
+        st.step(xs[t], t)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_all > budget_s:
+            break
+    per_layer = statistics.mean(times)
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
+    except Exception:
+        cores = os.cpu_count()
+    return {"value": wl.n_tokens / (per_layer * wl.n_layers), "unit": "tokens/s", "cores": cores,
+            "kind": "oracle",
+            "sample": (f"{len(times)} cache steps of layer 0 at full T={wl.n_tokens} (tau0 of the headline point), "
+                       f"{per_layer * 1e3:.0f} ms per layer step, extrapolated to {wl.n_layers} layers; "
+                       f"numpy float64, host cores {os.cpu_count()}")}
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the oracle on host cores
+# ---------------------------------------------------------------------------
+
+def reference_arm(args, wl):
+    import numpy as np
+    from oracle import moeca_oracle as O
+    from paper_2606_15615_gb300 import workloads as W
+    rng_layers = min(wl.n_layers, 2)
+    ws = [W.make_layer_weights(wl, l) for l in range(rng_layers)]
+    xs = list(W.trajectory(wl, args.warmup + args.steps + 1))
+    prm = O.Params(top_k=wl.top_k, tau0=args.ref_tau0, refresh_period=wl.refresh_period)
+    stacks = [O.Stack([ws[l]], prm, wl.hidden, wl.n_experts, wl.n_shared) for l in range(rng_layers)]
+    for t in range(args.warmup):
+        stacks[t % rng_layers].step(xs[t], t)
+    times = []
+    for j in range(args.steps):
+        t = args.warmup + j
+        s = stacks[t % rng_layers]
+        t0 = time.perf_counter()
+        s.step(xs[t], t)
+        times.append(time.perf_counter() - t0)
+    per_layer = statistics.mean(times)
+    value = wl.n_tokens / (per_layer * wl.n_layers)
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * wl.n_layers * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "tau0": args.ref_tau0},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": (f"each step is one full-T layer step of the CPU oracle (layers 0-{rng_layers - 1} "
+                                    f"alternating, numpy weights), time extrapolated to {wl.n_layers} layers")},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+# ---------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--reuse", type=float, default=0.6, help="headline reuse target")
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--ref-tau0", type=float, default=0.8)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    from paper_2606_15615_gb300 import workloads as W
+    wl = W.workload(args.workload)
+    world, rank, local = dist_env()
+
+    if args.impl == "reference":
+        if rank == 0:
+            reference_arm(args, wl)
+        return
+
+    import torch
+    dist = init_group(world, "nccl")
+    runner = Runner(wl, local, args.warmup + args.steps)
+    dev = runner.dev
+    W_, K = args.warmup, args.steps
+    targets = [args.reuse] if args.no_sweep else sorted(set(wl.reuse_targets) | {args.reuse})
+    if wl.reuse_targets == (0.5,) and args.no_sweep is False:
+        targets = sorted(set(wl.reuse_targets) | {args.reuse})
+    sweep = []
+    head = None
+    pk, pk_src = peaks()
+    for tgt in targets:
+        tau0, achieved = runner.calibrate(tgt, W_, K)
+        is_head = abs(tgt - args.reuse) < 1e-9
+        sampler = None
+        if is_head and rank == 0:
+            sampler = ClockSampler(gpu_smi_id(local))
+            sampler.start()
+        reps = []
+        st = None
+        for _ in range(args.reps if is_head else 2):
+            if dist is not None:
+                dist.barrier()
+            torch.cuda.synchronize(dev)
+            ms, st, _ = runner._run(tau0, W_, K)
+            ms, tokens = aggregate(ms, wl.n_tokens * K, dist, dev)
+            reps.append(ms)
+        clocks = sampler.stop() if sampler else None
+        ms = statistics.median(reps)
+        tokens_all = wl.n_tokens * K * world
+        tps = tokens_all / (ms / 1e3)
+        executed = (st["recomputed"] + st["shared_recomputed"]) * 4.0 * wl.hidden * wl.ffn  # per rank, K steps
+        dense = wl.dense_flops_per_layer() * wl.n_layers * K
+        row = {"reuse_target": tgt, "reuse_achieved": round(runner.reuse_of(st), 4),
+               "tau0": None if not math.isfinite(tau0) else round(tau0, 5), "tokens_per_s": tps,
+               "ms_per_step": ms / K, "effective_tflops": dense * world / (ms / 1e3) / 1e12,
+               "executed_tflops": executed * world / (ms / 1e3) / 1e12}
+        sweep.append(row)
+        if is_head:
+            head = dict(row, clocks=clocks, stats=st, tau0_raw=tau0)
+
+    # Per-kernel CUDA-event durations on the launching stream, same steps as the headline.
+    _, st_k, kt = runner._run(head["tau0_raw"], W_, K, kernel_timing=True)
+    # End to end through the C ABI with host buffers.
+    if dist is not None:
+        dist.barrier()
+    e2e_ms, _, _ = runner._run(head["tau0_raw"], W_, K, e2e=True)
+    e2e_ms, _ = aggregate(e2e_ms, 0, dist, dev)
+    rows_per_launch = (st_k["recomputed"] + st_k["shared_recomputed"]) / (K * wl.n_layers)
+    kernels = {}
+    for kind in KINDS:
+        tot, n = kt[kind]
+        nb, nf = algorithmic(kind, wl, rows_per_launch, wl.n_experts + wl.n_shared)
+        avg = tot / max(n, 1)
+        kernels[kind] = {"launches": n, "avg_us": avg * 1e3, "share": tot / max(sum(v[0] for v in kt.values()), 1e-12),
+                         "alg_bytes": nb, "alg_flops": nf,
+                         "gbs": nb / (avg * 1e-3) / 1e9 if avg > 0 else None,
+                         "tflops": nf / (avg * 1e-3) / 1e12 if avg > 0 and nf else None}
+    dom = max(KINDS, key=lambda k_: kt[k_][0])
+    kd = kernels[dom]
+    ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+    if kd["alg_flops"] and kd["alg_flops"] / kd["alg_bytes"] > ridge:
+        roof = {"bound": "tensor", "achieved": kd["tflops"], "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": kd["gbs"], "peak": pk["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"] if roof["achieved"] else None
+    tr = recorded_traffic(dom, wl.name, args.reuse)
+    roof["traffic"] = tr
+    roof["kernel"] = dom
+    roof["peak_source"] = f"{pk_src} (MEASURED_PEAKS.json)" if pk_src == "measured" else "fallback"
+    roof["alg_bytes_per_launch"] = kd["alg_bytes"]
+    roof["alg_flops_per_launch"] = kd["alg_flops"]
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = cpu_oracle_baseline(wl, runner, head["tau0_raw"])
+    es = 2 if wl.dtype == "bf16" else 4
+    io_bytes = wl.n_tokens * wl.hidden * es
+    line = {
+        "metric": METRIC, "value": head["tokens_per_s"], "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W_, "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "tokens": wl.n_tokens, "hidden": wl.hidden, "experts": wl.n_experts,
+                   "shared_experts": wl.n_shared, "top_k": wl.top_k, "ffn": wl.ffn, "layers": wl.n_layers,
+                   "refresh_period": wl.refresh_period, "reuse_target": args.reuse,
+                   "reuse_achieved": head["reuse_achieved"], "tau0": head["tau0"],
+                   "effective_tflops": head["effective_tflops"], "executed_tflops": head["executed_tflops"],
+                   "timed": f"median of {args.reps} reps of {K} steps after {W_} warm-up steps (step 0 full)",
+                   "l2": "no flush: each step streams the active experts' weights "
+                         f"({wl.n_layers} x {2 * wl.n_experts * wl.hidden * wl.ffn * es / 1e6:.0f} MB) > 129 MB L2",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "e2e": {"value": wl.n_tokens * K * world / (e2e_ms / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes},
+        "gpu_launches": sum(kt[k_][1] for k_ in KINDS),
+        "clocks": head["clocks"],
+        "sweep": sweep,
+        "kernels": kernels,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    runner.stack.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,249 @@
+/*
+ * moeca.h -- C ABI of the GB300 branch-cached MoE layer stack (MoECa).
+ *
+ * One call of moeca_step() runs a stack of L DiT-MoE expert layers for one
+ * denoising step with branch-level feature reuse:
+ *   route (Eq. 7) -> EMA statistic, entropy, per-expert threshold (Eq. 10-12)
+ *   -> match each routed (token, expert) branch against the token's cached
+ *   branches, score it and decide recompute / reuse (Sec. 4.2, Eq. 9)
+ *   -> run the expert FFN only on recomputed branches (Eq. 5 / Eq. 6)
+ *   -> combine fresh and cached branch outputs with the current gate weights
+ *   and add the residual (Eq. 8) -> refresh the cached branch norms.
+ * Full-computation and cache steps alternate as in Sec. 4.1.
+ *
+ * Conventions
+ *  - All tensors are row-major.  "device" pointers are CUDA global memory of
+ *    the handle's device; "host" pointers are ordinary host memory.
+ *  - Weights and activation buffers are BORROWED: the caller owns them and
+ *    keeps them alive (weights for the handle's lifetime).  The library owns
+ *    every state and workspace buffer it allocates in moeca_create().
+ *  - Every function returns a moeca_status; none throws or aborts.  Kernels
+ *    never trap: a device-side problem (an index out of range, a bounded wait
+ *    that ran out) is written to a status word that the next moeca_step()
+ *    or moeca_get_stats() reports as MOECA_ERR_DEVICE_STATUS / _TIMEOUT.
+ *  - Calls that take a `stream` enqueue work on that cudaStream_t (NULL = the
+ *    legacy default stream) and return without waiting for the GPU.
+ *  - A handle is not thread-safe; use one handle per host thread.
+ */
+#ifndef MOECA_H_
+#define MOECA_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct moeca_handle moeca_handle; /* opaque, owned by the library */
+
+typedef enum {
+  MOECA_OK = 0,
+  MOECA_ERR_INVALID_ARG = -1,   /* bad pointer, size, alias or config value     */
+  MOECA_ERR_UNSUPPORTED = -2,   /* valid but not built (e.g. D not a multiple of 64 on bf16) */
+  MOECA_ERR_CUDA = -3,          /* a CUDA runtime call failed (see moeca_last_error) */
+  MOECA_ERR_OOM = -4,           /* device allocation failed                       */
+  MOECA_ERR_STATE = -5,         /* call not valid in the handle's state           */
+  MOECA_ERR_TIMEOUT = -6,       /* a bounded device wait ran out                  */
+  MOECA_ERR_DEVICE_STATUS = -7  /* a kernel flagged bad data (index out of range) */
+} moeca_status;
+
+typedef enum {
+  MOECA_F32 = 0,  /* fp32 storage, fp32 FFMA everywhere (debug-precision path)   */
+  MOECA_BF16 = 1  /* bf16 activations/weights/cache, fp32 accumulation and logic */
+} moeca_dtype;
+
+typedef enum {
+  MOECA_FFN_AUTO = 0, /* tcgen05 tensor-core grouped GEMM for bf16, SIMT for fp32 */
+  MOECA_FFN_SIMT = 1  /* CUDA-core grouped GEMM for both dtypes (cross-check path) */
+} moeca_ffn_impl;
+
+/* Shapes, hyper-parameters and the readings of points the paper leaves open. */
+typedef struct {
+  int32_t n_layers;    /* L >= 1                                                  */
+  int32_t hidden;      /* D: multiple of 8 (fp32: 4); bf16 tensor path: of 64     */
+  int32_t ffn;         /* F: expert FFN width; bf16 tensor path: multiple of 64   */
+  int32_t n_experts;   /* E routed experts, 1..64                                  */
+  int32_t top_k;       /* k, 1..8 and <= E                                         */
+  int32_t n_shared;    /* always-on shared experts (Eq. 6): 0 or 1, width F        */
+  int32_t max_tokens;  /* largest T = batch * tokens a step may carry (>= 1)      */
+  int32_t dtype;       /* moeca_dtype                                              */
+  float lambda1;       /* Eq. 9 weight of the temporal drift Delta                 */
+  float lambda2;       /* Eq. 9 weight of the historical contribution o            */
+  float tau0;          /* Eq. 12 base threshold (may be +-inf)                     */
+  float alpha;         /* Eq. 12 expert adaptation strength, [0, 1)                */
+  float beta;          /* Eq. 10 EMA decay, [0, 1)                                 */
+  int32_t refresh_period;     /* N: full-computation step when step % N == 0 (0: only step 0 / forced) */
+  int32_t renorm_topk;        /* 1: top-k gate weights renormalised to sum 1 (default) */
+  int32_t entropy_norm;       /* 0: Hbar = H / ln T (default); 1: min-max over the layer's experts */
+  int32_t shared_policy;      /* 0: shared expert recomputed iff the token's recompute set is
+                                 non-empty or the step is full (Sec. 4.1 sync rule, default); 1: always */
+  int32_t reused_meta_policy; /* 0: a reused slot keeps w^{t0} (default); 1: it takes w^t */
+  int32_t gelu_tanh;          /* 1: tanh-form GELU (default); 0: erf form */
+  int32_t ffn_impl;           /* moeca_ffn_impl */
+} moeca_config;
+
+/* Fill `cfg` with the defaults above and the paper's hyper-parameters
+ * (tau0 0.8, alpha 0.6, beta 0.65, Sec. 5.3; lambda1 1.0 and lambda2 0.5 are
+ * this library's choice: the paper does not print its values). */
+void moeca_config_default(moeca_config* cfg);
+
+/* Device pointers of one layer's weights (dtype of the config; bias fp32).
+ * Eq. 7 router and Eq. 5 / Eq. 6 experts; every matrix is "K-major":
+ *   w_gate [E, D], b_gate [E] fp32 or NULL,
+ *   w1 [E, F, D], w2 [E, D, F]  (FFN_e(u) = w2_e GELU(w1_e u), no bias),
+ *   ws1 [F, D], ws2 [D, F] for the shared expert (NULL when n_shared == 0).
+ * Base pointers must be 16-byte aligned. */
+typedef struct {
+  const void* w_gate;
+  const float* b_gate;
+  const void* w1;
+  const void* w2;
+  const void* ws1;
+  const void* ws2;
+} moeca_layer_weights;
+
+/* Per-step arguments. */
+typedef struct {
+  int32_t n_tokens;      /* T, 0..max_tokens; T = 0 is a no-op; a new T forces a full step */
+  int32_t step_index;    /* denoising step counter used by the refresh schedule             */
+  int32_t force_refresh; /* 1: make this a full-computation step (Sec. 4.1)                 */
+  float tau0_override;   /* NaN: use config tau0; otherwise the Eq. 12 base threshold now   */
+} moeca_step_args;
+
+/* Branch counters, cumulative since create / moeca_reset_stats (Fig. 8 inputs). */
+typedef struct {
+  int64_t layer_steps;          /* layer evaluations                                    */
+  int64_t refresh_layer_steps;  /* of which full-computation                            */
+  int64_t branches;             /* routed branches, T * k per layer step                */
+  int64_t cache_step_branches;  /* routed branches on cache steps                       */
+  int64_t matched;              /* cache-step branches whose expert is cached for the token */
+  int64_t recomputed;           /* branches recomputed (every branch on full steps)     */
+  int64_t reused;               /* branches served from the cache                       */
+  int64_t tokens_fully_reused;  /* cache-step tokens with an empty recompute set        */
+  int64_t shared_recomputed;    /* shared-expert rows recomputed                        */
+  int64_t near_margin_route;    /* tokens whose ranks 1..k+1 logits differ by < 1e-5 relative */
+  int64_t near_margin_score;    /* matched branches with |s - tau| < 1e-5 |tau|         */
+  int32_t device_status;        /* 0, or the first kernel status code seen              */
+  int32_t device_detail;        /* kernel-specific detail of that status                */
+} moeca_stats;
+
+/* Caller-owned DEVICE buffers for one layer's cached state, T rows each.
+ * Any pointer may be NULL in moeca_get_layer_state (that field is skipped);
+ * moeca_set_layer_state needs all of them (shared_h only when n_shared == 1).
+ *   cache_e [T, k] int32   cached expert ids e^{t0}        (Eq. 7)
+ *   cache_w [T, k] fp32    cached gate weights w^{t0}      (Eq. 7)
+ *   cache_norm [T, k] fp32 ||h^{t0}|| over D                (Eq. 9, o)
+ *   cache_h [T, k, D] dtype cached branch outputs h^{t0}    (Eq. 7)
+ *   shared_h [T, D] dtype  cached shared-expert output      (Eq. 6)
+ *   ema [T, E] fp32        C_{e,i} stored at [i * E + e]     (Eq. 10) */
+typedef struct {
+  int32_t* cache_e;
+  float* cache_w;
+  float* cache_norm;
+  void* cache_h;
+  void* shared_h;
+  float* ema;
+} moeca_layer_state;
+
+/* Caller-owned DEVICE buffers for what one layer computed on the last step.
+ * Any pointer may be NULL (skipped).  G = E + n_shared work groups.
+ *   route_e [T, k] int32, route_w [T, k] fp32   routing B_i^t (Eq. 7)
+ *   tau [E] fp32                                 thresholds (Eq. 12)
+ *   recompute [T, k] uint8, slot [T, k] int8     decision and cache slot of branch p
+ *   matched [T, k] uint8                         expert found in the token's cache
+ *   token_any [T] uint8                          recompute set non-empty (Sec. 4.1)
+ *   counts [G] int32, offsets [G + 1] int32      rows per expert group
+ *   list [offsets[G]] int32                      rows: token * k + slot (routed), token (shared)
+ *   layer_in [T, D] dtype                        the layer's input activations */
+typedef struct {
+  int32_t* route_e;
+  float* route_w;
+  float* tau;
+  uint8_t* recompute;
+  int8_t* slot;
+  uint8_t* matched;
+  uint8_t* token_any;
+  int32_t* counts;
+  int32_t* offsets;
+  int32_t* list;
+  void* layer_in;
+} moeca_layer_trace;
+
+/* Kernel kinds timed by moeca_set_kernel_timing(). */
+enum {
+  MOECA_K_ROUTER = 0,  /* gate logits, softmax, top-k, EMA, entropy -> tau  */
+  MOECA_K_SELECT = 1,  /* match, score, threshold, slots, group counts      */
+  MOECA_K_COMPACT = 2, /* per-expert row lists and row gather               */
+  MOECA_K_FFN1 = 3,    /* grouped GEMM X W1^T + GELU                        */
+  MOECA_K_FFN2 = 4,    /* grouped GEMM Hmid W2^T -> cache rows              */
+  MOECA_K_COMBINE = 5, /* Eq. 8 combine + residual + cached norms           */
+  MOECA_K_COUNT = 6
+};
+
+typedef struct {
+  double total_ms[MOECA_K_COUNT]; /* summed CUDA-event time per kernel kind */
+  int64_t launches[MOECA_K_COUNT];
+} moeca_kernel_times;
+
+/* Create a handle on CUDA device `device` and allocate its state (caches for
+ * max_tokens rows per layer) and workspace.  `layers` points to n_layers host
+ * structs of device weight pointers.  Errors: INVALID_ARG (NULL, a field out
+ * of range), UNSUPPORTED (shape the kernels do not take), OOM, CUDA.  On error
+ * *out is set to NULL and nothing is leaked. */
+moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* layers,
+                          int32_t device, moeca_handle** out);
+
+/* Run the stack for one denoising step on `stream`.  x_in [T, D] and
+ * x_out [T, D] are device buffers of the config dtype that must not overlap.
+ * The step is a full-computation step when forced, on the first step after
+ * create / reset, when T differs from the previous step, or when
+ * refresh_period > 0 divides step_index (Sec. 4.1); otherwise a cache step.
+ * Asynchronous: no host synchronisation inside.  Errors: INVALID_ARG,
+ * STATE (handle destroyed), DEVICE_STATUS / TIMEOUT (from an earlier kernel),
+ * CUDA (launch failure). */
+moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out,
+                        const moeca_step_args* args, void* stream);
+
+/* Copy the counters of `layer` (or the sum over layers for layer = -1) into
+ * *out.  Synchronises the device. */
+moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out);
+moeca_status moeca_reset_stats(moeca_handle* h);
+
+/* Copy one layer's cached state into caller device buffers (async on stream);
+ * *n_tokens receives the T the state holds (0 if none). */
+moeca_status moeca_get_layer_state(moeca_handle* h, int32_t layer, const moeca_layer_state* dst,
+                                   int32_t* n_tokens, void* stream);
+
+/* Load one layer's cached state from caller device buffers (async on stream)
+ * for n_tokens rows (1..max_tokens) and mark the caches valid, so the next
+ * step with that T is a cache step unless the schedule says otherwise.  Used to
+ * resume a trajectory and to teacher-force parity tests.  Every layer must
+ * hold the same T. */
+moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_layer_state* src,
+                                   int32_t n_tokens, void* stream);
+
+/* Copy what `layer` computed on the last step (see moeca_layer_trace). */
+moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_layer_trace* dst,
+                                   void* stream);
+
+/* Drop every cache and zero the EMA statistics; the next step is a full step. */
+moeca_status moeca_reset(moeca_handle* h);
+
+/* Record CUDA events around every kernel launch (enable = 1) and accumulate
+ * their durations; moeca_get_kernel_times() synchronises and reads them, and
+ * resets the sums when reset = 1. */
+moeca_status moeca_set_kernel_timing(moeca_handle* h, int32_t enable);
+moeca_status moeca_get_kernel_times(moeca_handle* h, moeca_kernel_times* out, int32_t reset);
+
+/* Free everything the handle owns.  NULL is accepted. */
+moeca_status moeca_destroy(moeca_handle* h);
+
+const char* moeca_status_string(moeca_status s);
+/* Message of the last error on this handle ("" if none); NULL handle: the
+ * last moeca_create() failure of this thread. */
+const char* moeca_last_error(const moeca_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MOECA_H_ */

@@ -278,27 +278,23 @@ class LayerState:
                           self.C.copy(), self.valid)
 
 
-def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, refresh: bool):
-    """One MoE layer at one denoising step; returns (out [T, D], new state, info).
+def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, slot, weights: dict,
+                          prm: Params, refresh: bool):
+    """Apply a recompute decision and form the layer output (Sec. 4.1, Eq. 5-8).
 
-    Order of work: route (Eq. 7) -> EMA (Eq. 10) -> entropy and tau (Eq. 11-12)
-    -> match, score, decide (Eq. 9) -> recompute R (Eq. 5) -> shared experts
-    under the synchronized rule (Sec. 4.1) -> combine with current gate weights
-    (Eq. 8) plus the residual (Eq. 5 / 6) -> refresh the cached norms.
+    Recomputes FFN_e(u_i) for the branches in R (rows of one expert together),
+    stores them in their cache slots with (e^t, w^t), recomputes shared experts
+    under the synchronized rule, combines every branch p from slot(p) with the
+    current weight w^t (Eq. 8), adds the residual and refreshes the cached
+    norms.  Returns (out [T, D], new state, token_any [T]).
     """
     u = np.asarray(u, np.float64)
     T, D = u.shape
     k = prm.top_k
-    e_cur, w_cur, near = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
-    C = ema_update(state.C, e_cur, prm.beta)
-    Hbar = normalized_entropy(C, prm.entropy_norm)
-    tau = expert_threshold(Hbar, prm.tau0, prm.alpha)
-    sel = select_branches(e_cur, w_cur, state.cache_e, state.cache_w, state.cache_norm, tau,
-                          prm.lambda1, prm.lambda2, refresh)
     new = state.copy()
-    new.C = C
-    rec, slot = sel["recompute"], sel["slot"]
-    # Recompute the branches of R, one expert's rows at a time.
+    e_cur = np.asarray(e_cur)
+    rec = np.asarray(rec, bool)
+    slot = np.asarray(slot)
     for e in np.unique(e_cur[rec]):
         rows = np.argwhere(rec & (e_cur == e))
         h = expert_ffn(u[rows[:, 0]], weights["w1"][e], weights["w2"][e], prm.gelu)
@@ -325,12 +321,35 @@ def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, ref
     # Eq. 8: every current branch p reads slot(p), fresh or cached, with w^t.
     y = np.zeros((T, D))
     for p in range(k):
-        y += w_cur[:, p:p + 1] * new.cache_h[np.arange(T), slot[:, p]]
+        y += np.asarray(w_cur, np.float64)[:, p:p + 1] * new.cache_h[np.arange(T), slot[:, p]]
     if new.shared_h is not None:
         y += new.shared_h
     out = u + y
     new.cache_norm = np.sqrt(np.sum(new.cache_h ** 2, axis=2))
     new.valid = True
+    return out, new, token_any
+
+
+def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, refresh: bool):
+    """One MoE layer at one denoising step; returns (out [T, D], new state, info).
+
+    Order of work: route (Eq. 7) -> EMA (Eq. 10) -> entropy and tau (Eq. 11-12)
+    -> match, score, decide (Eq. 9) -> recompute R (Eq. 5) -> shared experts
+    under the synchronized rule (Sec. 4.1) -> combine with current gate weights
+    (Eq. 8) plus the residual (Eq. 5 / 6) -> refresh the cached norms.
+    """
+    u = np.asarray(u, np.float64)
+    T, D = u.shape
+    k = prm.top_k
+    e_cur, w_cur, near = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
+    C = ema_update(state.C, e_cur, prm.beta)
+    Hbar = normalized_entropy(C, prm.entropy_norm)
+    tau = expert_threshold(Hbar, prm.tau0, prm.alpha)
+    sel = select_branches(e_cur, w_cur, state.cache_e, state.cache_w, state.cache_norm, tau,
+                          prm.lambda1, prm.lambda2, refresh)
+    out, new, token_any = recompute_and_combine(state, u, e_cur, w_cur, sel["recompute"], sel["slot"],
+                                                weights, prm, refresh)
+    new.C = C
     info = dict(e=e_cur, w=w_cur, near_route=near, C=C, Hbar=Hbar, tau=tau,
                 token_any=token_any, refresh=refresh, **sel)
     return out, new, info

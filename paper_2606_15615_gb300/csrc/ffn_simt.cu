@@ -1,0 +1,125 @@
+// CUDA-core grouped expert FFN over the compacted recompute rows.
+//
+// Phase 1: hmid[r, :] = GELU(xg[r, :] W1_g^T)      (first half of Eq. 5's FFN)
+// Phase 2: dst[list[r], :] = hmid[r, :] W2_g^T     (second half; rows land in
+//          the branch cache slot token*k+slot, or the shared-expert row)
+// Rows of group g are [offsets[g], offsets[g] + counts[g]).  The counts live
+// on the device, so the grid covers the worst case and each block finds its
+// (group, m-tile) from them; blocks past the last tile exit.  fp32 FFMA with
+// fp32 accumulation: the fp32 debug-precision path, and a cross-check of the
+// tensor-core kernel on bf16.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace moeca {
+namespace {
+
+constexpr int BM = 64, BN = 64, BK = 16;
+
+template <typename TI, int PHASE>
+__global__ void __launch_bounds__(256) ffn_simt_kernel(FfnArgs a) {
+  const int N = PHASE == 1 ? a.F : a.D;
+  const int K = PHASE == 1 ? a.D : a.F;
+  int mt = blockIdx.y, g = -1, m0 = 0;
+  for (int gg = 0; gg < a.G; ++gg) {
+    const int tiles = (a.counts[gg] + BM - 1) / BM;
+    if (mt < tiles) {
+      g = gg;
+      m0 = mt * BM;
+      break;
+    }
+    mt -= tiles;
+  }
+  if (g < 0) return;
+  const int rows = a.counts[g];
+  const int row0 = a.offsets[g];
+  const int n0 = blockIdx.x * BN;
+  const TI* A = static_cast<const TI*>(PHASE == 1 ? a.xg : a.hmid);
+  const TI* B;
+  if (g < a.E) {
+    B = static_cast<const TI*>(PHASE == 1 ? a.w1 : a.w2) + static_cast<size_t>(g) * a.F * a.D;
+  } else {
+    B = static_cast<const TI*>(PHASE == 1 ? a.ws1 : a.ws2);
+  }
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Bs[BK][BN + 4];
+  const int t = threadIdx.x;
+  const int ty = t / 16, tx = t % 16;
+  const int lr = t / 4, lk = (t % 4) * 4;
+  float acc[4][4];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += BK) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int kk = k0 + lk + j;
+      float av = 0.f, bv = 0.f;
+      if (m0 + lr < rows && kk < K)
+        av = Elem<TI>::to_f(A[static_cast<size_t>(row0 + m0 + lr) * K + kk]);
+      if (n0 + lr < N && kk < K)
+        bv = Elem<TI>::to_f(B[static_cast<size_t>(n0 + lr) * K + kk]);
+      As[lk + j][lr] = av;
+      Bs[lk + j][lr] = bv;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < BK; ++kk) {
+      float av[4], bv[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) av[r] = As[kk][ty * 4 + r];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) bv[c] = Bs[kk][tx * 4 + c];
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(av[r], bv[c], acc[r][c]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int m = m0 + ty * 4 + r;
+    if (m >= rows) continue;
+    const size_t row = static_cast<size_t>(row0 + m);
+    if (PHASE == 1) {
+      TI* H = static_cast<TI*>(a.hmid);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int n = n0 + tx * 4 + c;
+        if (n < N) H[row * a.F + n] = Elem<TI>::from_f(gelu_f(acc[r][c], a.gelu_tanh));
+      }
+    } else {
+      const int dr = a.list[row];
+      const int lim = g < a.E ? a.T * a.k : a.T;
+      if (dr < 0 || dr >= lim) {
+        report_status(a.status, kStatusBadIndex, 2000000 + static_cast<int>(row));
+        continue;
+      }
+      TI* dst = static_cast<TI*>(g < a.E ? a.cache_h : a.shared_h);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int n = n0 + tx * 4 + c;
+        if (n < N) dst[static_cast<size_t>(dr) * a.D + n] = Elem<TI>::from_f(acc[r][c]);
+      }
+    }
+  }
+}
+
+template <typename TI>
+cudaError_t launch_t(const FfnArgs& a, int phase, cudaStream_t s) {
+  const int N = phase == 1 ? a.F : a.D;
+  const dim3 grid((N + BN - 1) / BN, (a.max_rows + BM - 1) / BM + a.G);
+  if (phase == 1) ffn_simt_kernel<TI, 1><<<grid, 256, 0, s>>>(a);
+  else ffn_simt_kernel<TI, 2><<<grid, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s) {
+  return bf16 ? launch_t<__nv_bfloat16>(a, phase, s) : launch_t<float>(a, phase, s);
+}
+
+}  // namespace moeca

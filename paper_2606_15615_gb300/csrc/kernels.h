@@ -1,0 +1,128 @@
+// Internal launch interface between the host engine and the MoECa kernels.
+// Plain structs of device pointers and sizes; `bf16` selects the element type
+// (__nv_bfloat16 when true, float otherwise) of every activation, weight and
+// cached-output buffer.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace moeca {
+
+// Counters per layer, in this order (device uint64).
+enum StatIndex {
+  kStLayerSteps = 0, kStRefreshSteps, kStBranches, kStCacheBranches, kStMatched,
+  kStRecomputed, kStReused, kStTokensFullyReused, kStSharedRecomputed,
+  kStNearRoute, kStNearScore, kStCount
+};
+
+constexpr int kMaxExperts = 64;
+constexpr int kMaxTopK = 8;
+constexpr int kRouterTokensPerBlock = 16;   // 8 warps x 2 tokens
+constexpr int kSelectTokensPerBlock = 128;  // one token per thread
+
+// Eq. 7 router + Eq. 10 EMA + Eq. 11-12 threshold (finished by the last block).
+struct RouterArgs {
+  const void* x;        // [T, D]
+  const void* w_gate;   // [E, D]
+  const float* b_gate;  // [E] or null
+  int T, D, E, k;
+  int renorm;
+  float beta;
+  float tau0, alpha;
+  int entropy_norm;
+  int32_t* route_e;     // [T, k]
+  float* route_w;       // [T, k]
+  float* ema;           // [T, E]
+  float* partials;      // [gridDim.x, E, 2]   (sum C, sum C ln C) per block
+  unsigned* done;       // last-block ticket, left at 0
+  float* tau;           // [E]
+  unsigned long long* stats;
+};
+cudaError_t launch_router(const RouterArgs& a, bool bf16, cudaStream_t s);
+
+// Sec. 4.2 match / Eq. 9 score / threshold / slots + per-group counts (the
+// last block scans them into offsets).
+struct SelectArgs {
+  int T, k, E, G;       // G = E + n_shared
+  int refresh;
+  float lambda1, lambda2;
+  int reused_meta_policy, shared_policy, n_shared;
+  const int32_t* route_e;
+  const float* route_w;
+  const float* tau;
+  int32_t* cache_e;     // [T, k]  updated in place
+  float* cache_w;       // [T, k]  updated in place
+  const float* cache_norm;
+  uint8_t* recompute;   // [T, k]
+  int8_t* slot;         // [T, k]
+  uint8_t* matched;     // [T, k]
+  uint8_t* token_any;   // [T]
+  int32_t* block_counts;   // [nblk, G]
+  int32_t* block_offsets;  // [nblk, G]
+  int32_t* counts;         // [G]
+  int32_t* offsets;        // [G + 1]
+  unsigned* done;
+  unsigned long long* stats;
+  int* status;
+};
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t s);
+
+// Per-group row lists in ascending token order + gather of the rows' inputs.
+struct CompactArgs {
+  int T, k, E, G, D, n_shared;
+  int refresh, shared_policy;
+  const int32_t* route_e;
+  const uint8_t* recompute;
+  const int8_t* slot;
+  const uint8_t* token_any;
+  const int32_t* block_offsets;
+  const int32_t* offsets;
+  int32_t* list;        // [rows]
+  const void* x;        // [T, D]
+  void* xg;             // [rows, D] gathered inputs
+};
+cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s);
+
+// Grouped expert FFN over the compacted rows (Eq. 5 / Eq. 6 on R only).
+struct FfnArgs {
+  int G, E, D, F, k, T;
+  int max_rows;          // capacity of xg / hmid rows
+  const int32_t* counts;
+  const int32_t* offsets;
+  const int32_t* list;
+  const void* xg;        // [rows, D]
+  void* hmid;            // [rows, F]
+  const void* w1;        // [E, F, D]
+  const void* w2;        // [E, D, F]
+  const void* ws1;       // [F, D]   shared expert (group E) or null
+  const void* ws2;       // [D, F]
+  void* cache_h;         // [T*k, D]   destination rows of routed groups
+  void* shared_h;        // [T, D]     destination rows of the shared group
+  int gelu_tanh;
+  int* status;
+};
+cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s);
+
+// tcgen05 / TMA grouped GEMM (bf16 only).  Tensor maps are built once per
+// handle; `TcPlan` owns them.
+struct TcPlan;
+TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen);
+void tc_plan_destroy(TcPlan* p);
+cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s);
+
+// Eq. 8 combine + residual + cached branch norms.
+struct CombineArgs {
+  int T, D, k, n_shared;
+  const void* x;          // [T, D]
+  void* out;              // [T, D]
+  const void* cache_h;    // [T, k, D]
+  const void* shared_h;   // [T, D] or null
+  const float* route_w;   // [T, k]
+  const int8_t* slot;     // [T, k]
+  float* cache_norm;      // [T, k]
+  int* status;
+};
+cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);
+
+}  // namespace moeca

@@ -1,0 +1,602 @@
+// Host engine and C ABI of the branch-cached MoE layer stack (include/moeca.h).
+//
+// Per step and layer the engine enqueues, on the caller's stream and with no
+// host synchronisation:
+//   router (Eq. 7, Eq. 10-12) -> select (Sec. 4.2, Eq. 9) -> compact ->
+//   grouped FFN phase 1 and 2 over the recompute rows (Eq. 5 / Eq. 6) ->
+//   combine (Eq. 8) writing the next layer's input.
+// It decides full-computation vs cache steps (Sec. 4.1), owns every state and
+// workspace buffer, and reports errors as status codes.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "moeca.h"
+
+using namespace moeca;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+struct LayerBuf {
+  moeca_layer_weights w;
+  int32_t* cache_e = nullptr;
+  float* cache_w = nullptr;
+  float* cache_norm = nullptr;
+  void* cache_h = nullptr;
+  void* shared_h = nullptr;
+  float* ema = nullptr;
+  int32_t* route_e = nullptr;
+  float* route_w = nullptr;
+  float* tau = nullptr;
+  uint8_t* recompute = nullptr;
+  int8_t* slot = nullptr;
+  uint8_t* matched = nullptr;
+  uint8_t* token_any = nullptr;
+  int32_t* counts = nullptr;
+  int32_t* offsets = nullptr;
+  int32_t* list = nullptr;
+  unsigned long long* stats = nullptr;
+  TcPlan* tc = nullptr;
+  bool valid = false;
+};
+
+struct PendingTiming {
+  int kind;
+  cudaEvent_t start, stop;
+};
+
+}  // namespace
+
+struct moeca_handle {
+  moeca_config cfg{};
+  int device = 0;
+  bool bf16 = false;
+  size_t es = 4;
+  int G = 0;
+  int n_sms = 0;
+  int max_rows = 0;
+  std::vector<LayerBuf> layers;
+  float* partials = nullptr;
+  unsigned* done = nullptr;  // [0] router ticket, [1] select ticket
+  int32_t* block_counts = nullptr;
+  int32_t* block_offsets = nullptr;
+  void* xg = nullptr;
+  void* hmid = nullptr;
+  std::vector<void*> act;  // input of layer l (l >= 1)
+  int* status_host = nullptr;
+  int* status_dev = nullptr;
+  int state_T = 0;
+  const void* last_x_in = nullptr;
+  std::string last_error;
+  std::vector<void*> allocs;
+  bool timing = false;
+  std::vector<cudaEvent_t> event_pool;
+  std::vector<PendingTiming> pending;
+  double total_ms[MOECA_K_COUNT] = {};
+  int64_t launches[MOECA_K_COUNT] = {};
+};
+
+namespace {
+
+moeca_status fail(moeca_handle* h, moeca_status s, const std::string& msg) {
+  if (h) h->last_error = msg;
+  else g_create_error = msg;
+  return s;
+}
+
+moeca_status cuda_fail(moeca_handle* h, cudaError_t e, const char* what) {
+  return fail(h, MOECA_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+bool dev_alloc(moeca_handle* h, void** p, size_t bytes) {
+  if (bytes == 0) bytes = 16;
+  if (cudaMalloc(p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return false;
+  }
+  h->allocs.push_back(*p);
+  if (cudaMemset(*p, 0, bytes) != cudaSuccess) return false;
+  return true;
+}
+
+void free_all(moeca_handle* h) {
+  for (auto& L : h->layers)
+    if (L.tc) tc_plan_destroy(L.tc);
+  for (void* p : h->allocs) cudaFree(p);
+  h->allocs.clear();
+  if (h->status_host) cudaFreeHost(h->status_host);
+  h->status_host = nullptr;
+  for (auto ev : h->event_pool) cudaEventDestroy(ev);
+  for (auto& pt : h->pending) {
+    cudaEventDestroy(pt.start);
+    cudaEventDestroy(pt.stop);
+  }
+  h->event_pool.clear();
+  h->pending.clear();
+}
+
+cudaEvent_t take_event(moeca_handle* h) {
+  if (!h->event_pool.empty()) {
+    cudaEvent_t e = h->event_pool.back();
+    h->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Launch `fn` with optional CUDA events around it.
+template <typename Fn>
+cudaError_t timed(moeca_handle* h, int kind, cudaStream_t s, Fn&& fn) {
+  if (!h->timing) return fn();
+  PendingTiming pt{kind, take_event(h), take_event(h)};
+  cudaEventRecord(pt.start, s);
+  cudaError_t e = fn();
+  cudaEventRecord(pt.stop, s);
+  h->pending.push_back(pt);
+  return e;
+}
+
+moeca_status check_device_status(moeca_handle* h) {
+  volatile int* st = h->status_host;
+  const int code = st[0];
+  if (code == 0) return MOECA_OK;
+  char buf[160];
+  snprintf(buf, sizeof buf, "device status %d (detail %d) from an earlier kernel", code, st[1]);
+  return fail(h, code == kStatusWaitTimeout ? MOECA_ERR_TIMEOUT : MOECA_ERR_DEVICE_STATUS, buf);
+}
+
+bool overlaps(const void* a, const void* b, size_t n) {
+  const char* x = static_cast<const char*>(a);
+  const char* y = static_cast<const char*>(b);
+  return x < y + n && y < x + n;
+}
+
+}  // namespace
+
+extern "C" {
+
+void moeca_config_default(moeca_config* c) {
+  if (!c) return;
+  std::memset(c, 0, sizeof *c);
+  c->n_layers = 1;
+  c->n_shared = 0;
+  c->max_tokens = 1;
+  c->dtype = MOECA_BF16;
+  c->lambda1 = 1.0f;
+  c->lambda2 = 0.5f;
+  c->tau0 = 0.8f;
+  c->alpha = 0.6f;
+  c->beta = 0.65f;
+  c->refresh_period = 0;
+  c->renorm_topk = 1;
+  c->entropy_norm = 0;
+  c->shared_policy = 0;
+  c->reused_meta_policy = 0;
+  c->gelu_tanh = 1;
+  c->ffn_impl = MOECA_FFN_AUTO;
+}
+
+const char* moeca_status_string(moeca_status s) {
+  switch (s) {
+    case MOECA_OK: return "ok";
+    case MOECA_ERR_INVALID_ARG: return "invalid argument";
+    case MOECA_ERR_UNSUPPORTED: return "unsupported";
+    case MOECA_ERR_CUDA: return "CUDA error";
+    case MOECA_ERR_OOM: return "out of device memory";
+    case MOECA_ERR_STATE: return "invalid state";
+    case MOECA_ERR_TIMEOUT: return "device wait timed out";
+    case MOECA_ERR_DEVICE_STATUS: return "device status error";
+  }
+  return "unknown status";
+}
+
+const char* moeca_last_error(const moeca_handle* h) {
+  return h ? h->last_error.c_str() : g_create_error.c_str();
+}
+
+moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* layers,
+                          int32_t device, moeca_handle** out) {
+  g_create_error.clear();
+  if (!out) return fail(nullptr, MOECA_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (!cfg || !layers) return fail(nullptr, MOECA_ERR_INVALID_ARG, "cfg or layers is NULL");
+  const moeca_config& c = *cfg;
+  const bool bf16 = c.dtype == MOECA_BF16;
+  if (c.dtype != MOECA_F32 && c.dtype != MOECA_BF16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "dtype");
+  if (c.n_layers < 1 || c.hidden < 1 || c.ffn < 1 || c.max_tokens < 1)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_layers, hidden, ffn and max_tokens must be >= 1");
+  if (c.n_experts < 1 || c.n_experts > kMaxExperts)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_experts must be in [1, 64]");
+  if (c.top_k < 1 || c.top_k > kMaxTopK || c.top_k > c.n_experts)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "top_k must be in [1, min(8, n_experts)]");
+  if (c.n_shared != 0 && c.n_shared != 1) return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_shared must be 0 or 1");
+  if (!(c.alpha >= 0.f && c.alpha < 1.f) || !(c.beta >= 0.f && c.beta < 1.f))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "alpha and beta must be in [0, 1)");
+  if (std::isnan(c.tau0) || !std::isfinite(c.lambda1) || !std::isfinite(c.lambda2))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "tau0, lambda1, lambda2");
+  if (c.refresh_period < 0) return fail(nullptr, MOECA_ERR_INVALID_ARG, "refresh_period < 0");
+  if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
+  const int vec = bf16 ? 8 : 4;
+  if (c.hidden % vec) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "hidden must be a multiple of 8 (bf16) / 4 (fp32)");
+  const bool use_tc = bf16 && c.ffn_impl == MOECA_FFN_AUTO;
+  if (use_tc && (c.hidden % 64 || c.ffn % 64))
+    return fail(nullptr, MOECA_ERR_UNSUPPORTED, "the tensor-core FFN needs hidden and ffn multiples of 64");
+  const size_t es = bf16 ? 2 : 4;
+  const long long rows_ll = static_cast<long long>(c.max_tokens) * (c.top_k + c.n_shared);
+  if (rows_ll > (1LL << 30) || static_cast<long long>(c.max_tokens) * c.top_k > (1LL << 30))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "max_tokens too large");
+  for (int l = 0; l < c.n_layers; ++l) {
+    const moeca_layer_weights& w = layers[l];
+    if (!w.w_gate || !w.w1 || !w.w2) return fail(nullptr, MOECA_ERR_INVALID_ARG, "layer weight pointer is NULL");
+    if (c.n_shared && (!w.ws1 || !w.ws2)) return fail(nullptr, MOECA_ERR_INVALID_ARG, "shared expert weights are NULL");
+    const void* ps[] = {w.w_gate, w.w1, w.w2, w.ws1, w.ws2};
+    for (const void* p : ps)
+      if (reinterpret_cast<uintptr_t>(p) % 16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "weights must be 16-byte aligned");
+  }
+  int ndev = 0;
+  cudaError_t ce = cudaGetDeviceCount(&ndev);
+  if (ce != cudaSuccess) { cudaGetLastError(); return fail(nullptr, MOECA_ERR_CUDA, std::string("no CUDA device: ") + cudaGetErrorString(ce)); }
+  if (device < 0 || device >= ndev) return fail(nullptr, MOECA_ERR_INVALID_ARG, "device out of range");
+  if ((ce = cudaSetDevice(device)) != cudaSuccess) return fail(nullptr, MOECA_ERR_CUDA, cudaGetErrorString(ce));
+
+  moeca_handle* h = new (std::nothrow) moeca_handle();
+  if (!h) return fail(nullptr, MOECA_ERR_OOM, "host allocation failed");
+  h->cfg = c;
+  h->device = device;
+  h->bf16 = bf16;
+  h->es = es;
+  h->G = c.n_experts + c.n_shared;
+  h->max_rows = static_cast<int>(rows_ll);
+  cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, device);
+  const size_t T = c.max_tokens, k = c.top_k, D = c.hidden, E = c.n_experts, G = h->G, F = c.ffn;
+  bool ok = true;
+  auto A = [&](void** p, size_t bytes) { ok = ok && dev_alloc(h, p, bytes); };
+  h->layers.resize(c.n_layers);
+  for (int l = 0; l < c.n_layers && ok; ++l) {
+    LayerBuf& L = h->layers[l];
+    L.w = layers[l];
+    A((void**)&L.cache_e, T * k * 4);
+    A((void**)&L.cache_w, T * k * 4);
+    A((void**)&L.cache_norm, T * k * 4);
+    A(&L.cache_h, T * k * D * es);
+    if (c.n_shared) A(&L.shared_h, T * D * es);
+    A((void**)&L.ema, T * E * 4);
+    A((void**)&L.route_e, T * k * 4);
+    A((void**)&L.route_w, T * k * 4);
+    A((void**)&L.tau, E * 4);
+    A((void**)&L.recompute, T * k);
+    A((void**)&L.slot, T * k);
+    A((void**)&L.matched, T * k);
+    A((void**)&L.token_any, T);
+    A((void**)&L.counts, G * 4);
+    A((void**)&L.offsets, (G + 1) * 4);
+    A((void**)&L.list, static_cast<size_t>(h->max_rows) * 4);
+    A((void**)&L.stats, kStCount * 8);
+  }
+  const size_t nblk_router = (T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
+  const size_t nblk_sel = (T + kSelectTokensPerBlock - 1) / kSelectTokensPerBlock;
+  A((void**)&h->partials, nblk_router * E * 2 * 4);
+  A((void**)&h->done, 2 * 4);
+  A((void**)&h->block_counts, nblk_sel * G * 4);
+  A((void**)&h->block_offsets, nblk_sel * G * 4);
+  A(&h->xg, static_cast<size_t>(h->max_rows) * D * es);
+  A(&h->hmid, static_cast<size_t>(h->max_rows) * F * es);
+  h->act.assign(c.n_layers, nullptr);
+  for (int l = 1; l < c.n_layers && ok; ++l) A(&h->act[l], T * D * es);
+  if (!ok) {
+    free_all(h);
+    delete h;
+    return fail(nullptr, MOECA_ERR_OOM, "device allocation failed");
+  }
+  if ((ce = cudaHostAlloc((void**)&h->status_host, 4 * sizeof(int), cudaHostAllocMapped)) != cudaSuccess ||
+      (ce = cudaHostGetDevicePointer((void**)&h->status_dev, h->status_host, 0)) != cudaSuccess) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return fail(nullptr, MOECA_ERR_CUDA, std::string("status word: ") + cudaGetErrorString(ce));
+  }
+  std::memset(h->status_host, 0, 4 * sizeof(int));
+  if (use_tc) {
+    for (int l = 0; l < c.n_layers; ++l) {
+      LayerBuf& L = h->layers[l];
+      FfnArgs fa{};
+      fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = c.max_tokens;
+      fa.max_rows = h->max_rows;
+      fa.xg = h->xg; fa.hmid = h->hmid;
+      fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
+      char err[256] = {0};
+      L.tc = tc_plan_create(fa, h->n_sms, err, sizeof err);
+      if (!L.tc) {
+        free_all(h);
+        delete h;
+        return fail(nullptr, MOECA_ERR_CUDA, std::string("tensor-core plan: ") + err);
+      }
+    }
+  }
+  if ((ce = cudaDeviceSynchronize()) != cudaSuccess) {
+    free_all(h);
+    delete h;
+    return fail(nullptr, MOECA_ERR_CUDA, cudaGetErrorString(ce));
+  }
+  *out = h;
+  return MOECA_OK;
+}
+
+moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const moeca_step_args* args,
+                        void* stream) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  if (!args || !x_in || !x_out) return fail(h, MOECA_ERR_INVALID_ARG, "args, x_in or x_out is NULL");
+  const moeca_config& c = h->cfg;
+  const int T = args->n_tokens;
+  if (T < 0 || T > c.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of [0, max_tokens]");
+  moeca_status st = check_device_status(h);
+  if (st != MOECA_OK) return st;
+  if (T == 0) return MOECA_OK;
+  const size_t xbytes = static_cast<size_t>(T) * c.hidden * h->es;
+  if (overlaps(x_in, x_out, xbytes)) return fail(h, MOECA_ERR_INVALID_ARG, "x_in and x_out overlap");
+  if (reinterpret_cast<uintptr_t>(x_in) % 16 || reinterpret_cast<uintptr_t>(x_out) % 16)
+    return fail(h, MOECA_ERR_INVALID_ARG, "x_in and x_out must be 16-byte aligned");
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  bool all_valid = h->state_T == T;
+  for (auto& L : h->layers) all_valid = all_valid && L.valid;
+  const int N = c.refresh_period;
+  const bool refresh = args->force_refresh || !all_valid || (N > 0 && args->step_index % N == 0);
+  if (h->state_T != T) {
+    // A new token count starts a new trajectory: the EMA positions restart.
+    for (auto& L : h->layers) {
+      cudaError_t e = cudaMemsetAsync(L.ema, 0, static_cast<size_t>(c.max_tokens) * c.n_experts * 4, s);
+      if (e != cudaSuccess) return cuda_fail(h, e, "reset EMA");
+      L.valid = false;
+    }
+  }
+  const float tau0 = std::isnan(args->tau0_override) ? c.tau0 : args->tau0_override;
+  const bool use_tc = h->bf16 && c.ffn_impl == MOECA_FFN_AUTO;
+  cudaError_t e = cudaSuccess;
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerBuf& L = h->layers[l];
+    const void* in = l == 0 ? x_in : h->act[l];
+    void* out = l + 1 == c.n_layers ? x_out : h->act[l + 1];
+
+    RouterArgs ra{};
+    ra.x = in; ra.w_gate = L.w.w_gate; ra.b_gate = L.w.b_gate;
+    ra.T = T; ra.D = c.hidden; ra.E = c.n_experts; ra.k = c.top_k;
+    ra.renorm = c.renorm_topk; ra.beta = c.beta; ra.tau0 = tau0; ra.alpha = c.alpha;
+    ra.entropy_norm = c.entropy_norm;
+    ra.route_e = L.route_e; ra.route_w = L.route_w; ra.ema = L.ema;
+    ra.partials = h->partials; ra.done = h->done; ra.tau = L.tau; ra.stats = L.stats;
+    if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
+
+    SelectArgs sa{};
+    sa.T = T; sa.k = c.top_k; sa.E = c.n_experts; sa.G = h->G; sa.refresh = refresh;
+    sa.lambda1 = c.lambda1; sa.lambda2 = c.lambda2;
+    sa.reused_meta_policy = c.reused_meta_policy; sa.shared_policy = c.shared_policy; sa.n_shared = c.n_shared;
+    sa.route_e = L.route_e; sa.route_w = L.route_w; sa.tau = L.tau;
+    sa.cache_e = L.cache_e; sa.cache_w = L.cache_w; sa.cache_norm = L.cache_norm;
+    sa.recompute = L.recompute; sa.slot = L.slot; sa.matched = L.matched; sa.token_any = L.token_any;
+    sa.block_counts = h->block_counts; sa.block_offsets = h->block_offsets;
+    sa.counts = L.counts; sa.offsets = L.offsets; sa.done = h->done + 1;
+    sa.stats = L.stats; sa.status = h->status_dev;
+    if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
+
+    CompactArgs ca{};
+    ca.T = T; ca.k = c.top_k; ca.E = c.n_experts; ca.G = h->G; ca.D = c.hidden; ca.n_shared = c.n_shared;
+    ca.refresh = refresh; ca.shared_policy = c.shared_policy;
+    ca.route_e = L.route_e; ca.recompute = L.recompute; ca.slot = L.slot; ca.token_any = L.token_any;
+    ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
+    ca.x = in; ca.xg = h->xg;
+    if ((e = timed(h, MOECA_K_COMPACT, s, [&] { return launch_compact(ca, h->bf16, s); })) != cudaSuccess) break;
+
+    FfnArgs fa{};
+    fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;
+    fa.max_rows = T * (c.top_k + c.n_shared);
+    fa.counts = L.counts; fa.offsets = L.offsets; fa.list = L.list;
+    fa.xg = h->xg; fa.hmid = h->hmid;
+    fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
+    fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
+    for (int phase = 1; phase <= 2 && e == cudaSuccess; ++phase) {
+      const int kind = phase == 1 ? MOECA_K_FFN1 : MOECA_K_FFN2;
+      e = timed(h, kind, s, [&] {
+        return use_tc ? launch_ffn_tc(L.tc, fa, phase, s) : launch_ffn_simt(fa, h->bf16, phase, s);
+      });
+    }
+    if (e != cudaSuccess) break;
+
+    CombineArgs cb{};
+    cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
+    cb.x = in; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+    cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
+    if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
+    L.valid = true;
+  }
+  if (e != cudaSuccess) {
+    for (auto& L : h->layers) L.valid = false;
+    return cuda_fail(h, e, "kernel launch");
+  }
+  h->state_T = T;
+  h->last_x_in = x_in;
+  return MOECA_OK;
+}
+
+moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out) {
+  if (!h || !out) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  const int L = h->cfg.n_layers;
+  if (layer < -1 || layer >= L) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
+  cudaSetDevice(h->device);
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(h, e, "synchronize");
+  std::memset(out, 0, sizeof *out);
+  for (int l = 0; l < L; ++l) {
+    if (layer >= 0 && l != layer) continue;
+    unsigned long long v[kStCount];
+    if ((e = cudaMemcpy(v, h->layers[l].stats, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess)
+      return cuda_fail(h, e, "read stats");
+    out->layer_steps += v[kStLayerSteps];
+    out->refresh_layer_steps += v[kStRefreshSteps];
+    out->branches += v[kStBranches];
+    out->cache_step_branches += v[kStCacheBranches];
+    out->matched += v[kStMatched];
+    out->recomputed += v[kStRecomputed];
+    out->reused += v[kStReused];
+    out->tokens_fully_reused += v[kStTokensFullyReused];
+    out->shared_recomputed += v[kStSharedRecomputed];
+    out->near_margin_route += v[kStNearRoute];
+    out->near_margin_score += v[kStNearScore];
+  }
+  volatile int* st = h->status_host;
+  out->device_status = st[0];
+  out->device_detail = st[1];
+  return out->device_status ? check_device_status(h) : MOECA_OK;
+}
+
+moeca_status moeca_reset_stats(moeca_handle* h) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  cudaSetDevice(h->device);
+  for (auto& L : h->layers) {
+    cudaError_t e = cudaMemset(L.stats, 0, kStCount * 8);
+    if (e != cudaSuccess) return cuda_fail(h, e, "reset stats");
+  }
+  return MOECA_OK;
+}
+
+moeca_status moeca_get_layer_state(moeca_handle* h, int32_t layer, const moeca_layer_state* dst,
+                                   int32_t* n_tokens, void* stream) {
+  if (!h || !dst) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
+  const LayerBuf& L = h->layers[layer];
+  const size_t T = L.valid ? h->state_T : 0, k = h->cfg.top_k, D = h->cfg.hidden, E = h->cfg.n_experts;
+  if (n_tokens) *n_tokens = static_cast<int32_t>(T);
+  if (T == 0) return MOECA_OK;
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  struct { void* d; const void* s; size_t n; } cp[] = {
+      {dst->cache_e, L.cache_e, T * k * 4},      {dst->cache_w, L.cache_w, T * k * 4},
+      {dst->cache_norm, L.cache_norm, T * k * 4}, {dst->cache_h, L.cache_h, T * k * D * h->es},
+      {dst->shared_h, L.shared_h, T * D * h->es}, {dst->ema, L.ema, T * E * 4}};
+  for (auto& x : cp) {
+    if (!x.d || !x.s) continue;
+    cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "copy layer state");
+  }
+  return MOECA_OK;
+}
+
+moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_layer_state* src,
+                                   int32_t n_tokens, void* stream) {
+  if (!h || !src) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
+  if (n_tokens < 1 || n_tokens > h->cfg.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of range");
+  if (!src->cache_e || !src->cache_w || !src->cache_norm || !src->cache_h || !src->ema ||
+      (h->cfg.n_shared && !src->shared_h))
+    return fail(h, MOECA_ERR_INVALID_ARG, "every state buffer is required");
+  LayerBuf& L = h->layers[layer];
+  const size_t T = n_tokens, k = h->cfg.top_k, D = h->cfg.hidden, E = h->cfg.n_experts;
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  struct { void* d; const void* s; size_t n; } cp[] = {
+      {L.cache_e, src->cache_e, T * k * 4},      {L.cache_w, src->cache_w, T * k * 4},
+      {L.cache_norm, src->cache_norm, T * k * 4}, {L.cache_h, src->cache_h, T * k * D * h->es},
+      {L.shared_h, src->shared_h, T * D * h->es}, {L.ema, src->ema, T * E * 4}};
+  for (auto& x : cp) {
+    if (!x.d || !x.s) continue;
+    cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "load layer state");
+  }
+  if (h->state_T != n_tokens) {
+    for (auto& other : h->layers) other.valid = false;
+    h->state_T = n_tokens;
+  }
+  L.valid = true;
+  return MOECA_OK;
+}
+
+moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_layer_trace* dst,
+                                   void* stream) {
+  if (!h || !dst) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
+  const LayerBuf& L = h->layers[layer];
+  const size_t T = h->state_T, k = h->cfg.top_k, D = h->cfg.hidden, E = h->cfg.n_experts, G = h->G;
+  if (T == 0) return fail(h, MOECA_ERR_STATE, "no step has run");
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const void* in = layer == 0 ? h->last_x_in : h->act[layer];
+  struct { void* d; const void* s; size_t n; } cp[] = {
+      {dst->route_e, L.route_e, T * k * 4}, {dst->route_w, L.route_w, T * k * 4},
+      {dst->tau, L.tau, E * 4},             {dst->recompute, L.recompute, T * k},
+      {dst->slot, L.slot, T * k},           {dst->matched, L.matched, T * k},
+      {dst->token_any, L.token_any, T},     {dst->counts, L.counts, G * 4},
+      {dst->offsets, L.offsets, (G + 1) * 4},
+      {dst->list, L.list, T * (k + h->cfg.n_shared) * 4},
+      {dst->layer_in, in, T * D * h->es}};
+  for (auto& x : cp) {
+    if (!x.d || !x.s) continue;
+    cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "copy layer trace");
+  }
+  return MOECA_OK;
+}
+
+moeca_status moeca_reset(moeca_handle* h) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  cudaSetDevice(h->device);
+  for (auto& L : h->layers) {
+    L.valid = false;
+    cudaError_t e = cudaMemset(L.ema, 0, static_cast<size_t>(h->cfg.max_tokens) * h->cfg.n_experts * 4);
+    if (e != cudaSuccess) return cuda_fail(h, e, "reset EMA");
+  }
+  h->state_T = 0;
+  return MOECA_OK;
+}
+
+moeca_status moeca_set_kernel_timing(moeca_handle* h, int32_t enable) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  h->timing = enable != 0;
+  return MOECA_OK;
+}
+
+moeca_status moeca_get_kernel_times(moeca_handle* h, moeca_kernel_times* out, int32_t reset) {
+  if (!h || !out) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  cudaSetDevice(h->device);
+  for (auto& pt : h->pending) {
+    cudaError_t e = cudaEventSynchronize(pt.stop);
+    if (e != cudaSuccess) return cuda_fail(h, e, "event synchronize");
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, pt.start, pt.stop);
+    h->total_ms[pt.kind] += ms;
+    h->launches[pt.kind] += 1;
+    h->event_pool.push_back(pt.start);
+    h->event_pool.push_back(pt.stop);
+  }
+  h->pending.clear();
+  for (int i = 0; i < MOECA_K_COUNT; ++i) {
+    out->total_ms[i] = h->total_ms[i];
+    out->launches[i] = h->launches[i];
+    if (reset) {
+      h->total_ms[i] = 0.0;
+      h->launches[i] = 0;
+    }
+  }
+  return MOECA_OK;
+}
+
+moeca_status moeca_destroy(moeca_handle* h) {
+  if (!h) return MOECA_OK;
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  free_all(h);
+  delete h;
+  return MOECA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,227 @@
+// Router of the branch-cached MoE layer.
+//
+// Per token i (one warp): gate logits z = x_i W_g^T (+ b) with fp32
+// accumulation, softmax over the E experts, top-k by descending logit with
+// ties to the lower expert id, optional renormalisation of the k weights
+// (Eq. 7).  The same pass updates the EMA statistic
+//   C_{e,i} <- beta C_{e,i} + (1 - beta) 1[e in B_i]        (Eq. 10)
+// and accumulates per block S_e = sum_i C_{e,i} and U_e = sum_i C ln C, from
+// which the last block to finish derives the spatial entropy
+//   H_e = ln S_e - U_e / S_e  (= -sum_i P ln P with P = C / S, Eq. 11),
+// its normalisation and the expert threshold tau_e (Eq. 12).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace moeca {
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kTokensPerWarp = kRouterTokensPerBlock / kWarps;
+
+template <typename TI, int EMAX>
+__global__ void __launch_bounds__(kWarps * 32) router_kernel(RouterArgs a) {
+  constexpr int V = Elem<TI>::kVec;
+  constexpr int EPL = (EMAX + 31) / 32;  // EMA experts per lane
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const TI* __restrict__ x = static_cast<const TI*>(a.x);
+  const TI* __restrict__ wg = static_cast<const TI*>(a.w_gate);
+  const int E = a.E, k = a.k, nvec = a.D / V;
+
+  __shared__ float sm_S[kWarps][EMAX];
+  __shared__ float sm_U[kWarps][EMAX];
+  __shared__ int sm_near[kWarps];
+
+  float accS[EPL], accU[EPL];
+#pragma unroll
+  for (int j = 0; j < EPL; ++j) accS[j] = accU[j] = 0.f;
+  int near_count = 0;
+
+  for (int tt = 0; tt < kTokensPerWarp; ++tt) {
+    const int i = blockIdx.x * kRouterTokensPerBlock + warp * kTokensPerWarp + tt;
+    if (i >= a.T) break;  // warp-uniform
+    float z[EMAX];
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) z[e] = 0.f;
+    const TI* xr = x + static_cast<size_t>(i) * a.D;
+    for (int c = lane; c < nvec; c += 32) {
+      float xv[V];
+      load_vec(xr + c * V, xv);
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e) {
+        if (e < E) {
+          float wv[V];
+          load_vec(wg + static_cast<size_t>(e) * a.D + c * V, wv);
+#pragma unroll
+          for (int j = 0; j < V; ++j) z[e] = fmaf(xv[j], wv[j], z[e]);
+        }
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) {
+      if (e < E) {
+        z[e] = warp_sum(z[e]);
+        if (a.b_gate) z[e] += a.b_gate[e];
+      }
+    }
+    // Top-(k+1) by repeated argmax (every lane holds every logit).
+    unsigned long long taken = 0ull, topk_mask = 0ull;
+    int sel[kMaxTopK];
+    float selz[kMaxTopK + 1];
+    const int ranks = (k + 1 < E) ? k + 1 : E;
+    float zabs = 0.f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) zabs = fmaxf(zabs, fabsf(z[e]));
+#pragma unroll
+    for (int p = 0; p < kMaxTopK + 1; ++p) {
+      if (p < ranks) {
+        int be = -1;
+        float best = 0.f;
+#pragma unroll
+        for (int e = 0; e < EMAX; ++e) {
+          if (e < E && !((taken >> e) & 1ull) && (be < 0 || z[e] > best)) {
+            best = z[e];
+            be = e;
+          }
+        }
+        taken |= 1ull << be;
+        selz[p] = best;
+        if (p < k) {
+          sel[p] = be;
+          topk_mask |= 1ull << be;
+        }
+      }
+    }
+    // Softmax over all E from the top logit, then the k weights.
+    const float m = selz[0];
+    float denom = 0.f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) denom += expf(z[e] - m);
+    float w[kMaxTopK];
+    float wsum = 0.f;
+#pragma unroll
+    for (int p = 0; p < kMaxTopK; ++p) {
+      if (p < k) {
+        w[p] = expf(selz[p] - m) / denom;
+        wsum += w[p];
+      }
+    }
+    bool near = false;
+#pragma unroll
+    for (int p = 0; p < kMaxTopK; ++p)
+      if (p + 1 < ranks && (selz[p] - selz[p + 1]) < 1e-5f * zabs) near = true;
+    if (lane == 0 && near) ++near_count;
+#pragma unroll
+    for (int p = 0; p < kMaxTopK; ++p) {
+      if (p < k && lane == p) {
+        a.route_e[static_cast<size_t>(i) * k + p] = sel[p];
+        a.route_w[static_cast<size_t>(i) * k + p] = a.renorm ? w[p] / wsum : w[p];
+      }
+    }
+    // EMA statistic and entropy partial sums.
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+      const int e = lane + 32 * j;
+      if (e < E) {
+        float* cp = a.ema + static_cast<size_t>(i) * E + e;
+        const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
+        const float c = a.beta * (*cp) + (1.f - a.beta) * ind;
+        *cp = c;
+        accS[j] += c;
+        if (c > 0.f) accU[j] += c * logf(c);
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < EPL; ++j) {
+    const int e = lane + 32 * j;
+    if (e < EMAX) {
+      sm_S[warp][e] = accS[j];
+      sm_U[warp][e] = accU[j];
+    }
+  }
+  if (lane == 0) sm_near[warp] = near_count;
+  __syncthreads();
+  const int t = threadIdx.x;
+  if (t < E) {
+    float S = 0.f, U = 0.f;
+#pragma unroll
+    for (int w8 = 0; w8 < kWarps; ++w8) {
+      S += sm_S[w8][t];
+      U += sm_U[w8][t];
+    }
+    a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 0] = S;
+    a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 1] = U;
+  }
+  if (t == 0) {
+    int n = 0;
+    for (int w8 = 0; w8 < kWarps; ++w8) n += sm_near[w8];
+    if (n) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(n));
+  }
+  // The last block to arrive reduces all partials in block order.
+  __threadfence();
+  __syncthreads();
+  __shared__ unsigned ticket;
+  if (t == 0) ticket = atomicAdd(a.done, 1u);
+  __syncthreads();
+  if (ticket != gridDim.x - 1) return;
+  __threadfence();
+  __shared__ double sm_H[EMAX];
+  __shared__ int sm_live[EMAX];
+  __shared__ double sm_lo, sm_hi;
+  if (t < E) {
+    double S = 0.0, U = 0.0;
+    for (unsigned b = 0; b < gridDim.x; ++b) {
+      S += static_cast<double>(__ldcg(a.partials + (static_cast<size_t>(b) * E + t) * 2 + 0));
+      U += static_cast<double>(__ldcg(a.partials + (static_cast<size_t>(b) * E + t) * 2 + 1));
+    }
+    sm_live[t] = S > 0.0;
+    sm_H[t] = S > 0.0 ? log(S) - U / S : 0.0;
+  }
+  __syncthreads();
+  if (t == 0) {
+    double lo = 0.0, hi = 0.0;
+    bool any = false;
+    for (int e = 0; e < E; ++e) {
+      if (!sm_live[e]) continue;
+      if (!any || sm_H[e] < lo) lo = sm_H[e];
+      if (!any || sm_H[e] > hi) hi = sm_H[e];
+      any = true;
+    }
+    sm_lo = lo;
+    sm_hi = hi;
+    *a.done = 0u;
+  }
+  __syncthreads();
+  if (t < E) {
+    double hb = 0.5;
+    if (sm_live[t]) {
+      if (a.entropy_norm == 0) {
+        if (a.T > 1) hb = fmin(1.0, fmax(0.0, sm_H[t] / log(static_cast<double>(a.T))));
+      } else if (sm_hi > sm_lo) {
+        hb = (sm_H[t] - sm_lo) / (sm_hi - sm_lo);
+      }
+    }
+    a.tau[t] = a.tau0 * (1.0f + a.alpha * (2.0f * static_cast<float>(hb) - 1.0f));
+  }
+}
+
+template <typename TI>
+cudaError_t launch_t(const RouterArgs& a, cudaStream_t s) {
+  const int grid = (a.T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
+  const dim3 block(kWarps * 32);
+  if (a.E <= 8) router_kernel<TI, 8><<<grid, block, 0, s>>>(a);
+  else if (a.E <= 16) router_kernel<TI, 16><<<grid, block, 0, s>>>(a);
+  else if (a.E <= 32) router_kernel<TI, 32><<<grid, block, 0, s>>>(a);
+  else router_kernel<TI, 64><<<grid, block, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_router(const RouterArgs& a, bool bf16, cudaStream_t s) {
+  return bf16 ? launch_t<__nv_bfloat16>(a, s) : launch_t<float>(a, s);
+}
+
+}  // namespace moeca

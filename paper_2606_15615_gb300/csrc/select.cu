@@ -1,0 +1,329 @@
+// Branch selection and compaction of the branch-cached MoE layer.
+//
+// select_kernel, one token per thread (Sec. 4.2):
+//   * match each routed branch p against the token's cached branches by
+//     expert id; an unmatched branch is always recomputed;
+//   * score a matched branch  s = w_p + lambda1 |w_p - w_q^{t0}|
+//     + lambda2 ||h_q|| / sum_j ||h_j||   (Eq. 9)  and recompute iff s > tau_e;
+//   * matched branches keep their cache slot q(p); unmatched ones take the
+//     slots whose expert is no longer routed, ascending p -> ascending q;
+//     on a full-computation step every branch is recomputed with slot = p;
+//   * write the new cache metadata, token_any = (R_i non-empty, Sec. 4.1) and
+//     per-block counts of recomputed rows per expert group (warp ballots).
+// The last block scans the per-block counts into per-group row offsets.
+//
+// compact_kernel, same token blocks: ranks each recomputed row inside its
+// group in ascending token order (ballot + popc prefix), writes the row list
+// (token * k + slot for routed experts, token for the shared expert) and
+// gathers the rows' layer inputs into a contiguous buffer for the GEMMs.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace moeca {
+namespace {
+
+constexpr int kThreads = kSelectTokensPerBlock;
+constexpr int kWarps = kThreads / 32;
+constexpr int kMaxGroups = kMaxExperts + 1;
+
+__global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int i = blockIdx.x * kThreads + t;
+  const bool valid = i < a.T;
+  const int k = a.k, E = a.E, G = a.G;
+  int e[kMaxTopK];
+  bool rec[kMaxTopK];
+  bool any = false;
+  int n_matched = 0, n_rec = 0, n_near = 0;
+  bool bad = false;
+#pragma unroll
+  for (int p = 0; p < kMaxTopK; ++p) {
+    e[p] = -1;
+    rec[p] = false;
+  }
+  if (valid) {
+    const size_t base = static_cast<size_t>(i) * k;
+    float w[kMaxTopK];
+    int sl[kMaxTopK];
+    bool mat[kMaxTopK];
+#pragma unroll
+    for (int p = 0; p < kMaxTopK; ++p) {
+      if (p < k) {
+        e[p] = a.route_e[base + p];
+        w[p] = a.route_w[base + p];
+        if (e[p] < 0 || e[p] >= E) bad = true;
+      }
+      mat[p] = false;
+      sl[p] = p;
+    }
+    if (bad) {
+      report_status(a.status, kStatusBadIndex, 1000000 + i);
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) e[p] = -1;
+    } else if (a.refresh) {
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) rec[p] = p < k;
+    } else {
+      int ce[kMaxTopK];
+      float cw[kMaxTopK], cn[kMaxTopK];
+      float nsum = 0.f;
+#pragma unroll
+      for (int q = 0; q < kMaxTopK; ++q) {
+        if (q < k) {
+          ce[q] = a.cache_e[base + q];
+          cw[q] = a.cache_w[base + q];
+          cn[q] = a.cache_norm[base + q];
+          nsum += cn[q];
+        }
+      }
+      unsigned used = 0u;
+      int qof[kMaxTopK];
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        qof[p] = -1;
+        if (p < k) {
+#pragma unroll
+          for (int q = kMaxTopK - 1; q >= 0; --q)
+            if (q < k && ce[q] == e[p]) qof[p] = q;  // lowest matching slot
+          if (qof[p] >= 0) {
+            const int q = qof[p];
+            used |= 1u << q;
+            mat[p] = true;
+            ++n_matched;
+            float cwq = 0.f, cnq = 0.f;
+#pragma unroll
+            for (int qq = 0; qq < kMaxTopK; ++qq)
+              if (qq == q) { cwq = cw[qq]; cnq = cn[qq]; }
+            const float delta = fabsf(w[p] - cwq);
+            const float o = nsum > 0.f ? cnq / nsum : 0.f;
+            const float s = w[p] + a.lambda1 * delta + a.lambda2 * o;
+            const float tau = a.tau[e[p]];
+            rec[p] = s > tau;
+            if (isfinite(tau) && fabsf(s - tau) < 1e-5f * fabsf(tau)) ++n_near;
+          } else {
+            rec[p] = true;
+          }
+        }
+      }
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        if (p < k) {
+          if (qof[p] >= 0) {
+            sl[p] = qof[p];
+          } else {
+            int fq = 0;
+            while ((used >> fq) & 1u) ++fq;
+            used |= 1u << fq;
+            sl[p] = fq;
+          }
+        }
+      }
+    }
+    if (!bad) {
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        if (p < k) {
+          any |= rec[p];
+          n_rec += rec[p];
+          a.recompute[base + p] = rec[p];
+          a.slot[base + p] = static_cast<int8_t>(sl[p]);
+          a.matched[base + p] = mat[p];
+          if (rec[p]) {
+            a.cache_e[base + sl[p]] = e[p];
+            a.cache_w[base + sl[p]] = w[p];
+          } else if (a.reused_meta_policy) {
+            a.cache_w[base + sl[p]] = w[p];
+          }
+        }
+      }
+      a.token_any[i] = any;
+    }
+  }
+  const bool shared_row = valid && !bad && a.n_shared && (a.refresh || a.shared_policy || any);
+
+  // Rows per (warp, group) by ballot, then per block.
+  __shared__ int sm_wc[kWarps][kMaxGroups];
+  for (int g = 0; g < G; ++g) {
+    bool has = false;
+    if (g < E) {
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) has |= (rec[p] && e[p] == g);
+    } else {
+      has = shared_row;
+    }
+    const unsigned b = __ballot_sync(0xffffffffu, has);
+    if (lane == 0) sm_wc[warp][g] = __popc(b);
+  }
+  // Branch counters.
+  const int c_matched = warp_sum_i(n_matched);
+  const int c_rec = warp_sum_i(n_rec);
+  const int c_near = warp_sum_i(n_near);
+  const int c_full = warp_sum_i(valid && !bad && !any ? 1 : 0);
+  const int c_shared = warp_sum_i(shared_row ? 1 : 0);
+  __shared__ int sm_c[kWarps][5];
+  if (lane == 0) {
+    sm_c[warp][0] = c_matched;
+    sm_c[warp][1] = c_rec;
+    sm_c[warp][2] = c_near;
+    sm_c[warp][3] = c_full;
+    sm_c[warp][4] = c_shared;
+  }
+  __syncthreads();
+  for (int g = t; g < G; g += kThreads) {
+    int s = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) s += sm_wc[w][g];
+    a.block_counts[static_cast<size_t>(blockIdx.x) * G + g] = s;
+  }
+  if (t == 0) {
+    int tot[5] = {0, 0, 0, 0, 0};
+    for (int w = 0; w < kWarps; ++w)
+      for (int j = 0; j < 5; ++j) tot[j] += sm_c[w][j];
+    const int nb = min(kThreads, a.T - static_cast<int>(blockIdx.x) * kThreads);
+    unsigned long long* st = a.stats;
+    atomicAdd(st + kStRecomputed, static_cast<unsigned long long>(tot[1]));
+    atomicAdd(st + kStReused, static_cast<unsigned long long>(nb * k - tot[1]));
+    if (tot[4]) atomicAdd(st + kStSharedRecomputed, static_cast<unsigned long long>(tot[4]));
+    if (!a.refresh) {
+      atomicAdd(st + kStMatched, static_cast<unsigned long long>(tot[0]));
+      atomicAdd(st + kStTokensFullyReused, static_cast<unsigned long long>(tot[3]));
+      if (tot[2]) atomicAdd(st + kStNearScore, static_cast<unsigned long long>(tot[2]));
+    }
+    if (blockIdx.x == 0) {
+      const unsigned long long br = static_cast<unsigned long long>(a.T) * k;
+      atomicAdd(st + kStLayerSteps, 1ull);
+      atomicAdd(st + kStBranches, br);
+      if (a.refresh) atomicAdd(st + kStRefreshSteps, 1ull);
+      else atomicAdd(st + kStCacheBranches, br);
+    }
+  }
+  // The last block turns per-block counts into offsets.
+  __threadfence();
+  __syncthreads();
+  __shared__ unsigned ticket;
+  if (t == 0) ticket = atomicAdd(a.done, 1u);
+  __syncthreads();
+  if (ticket != gridDim.x - 1) return;
+  __threadfence();
+  __shared__ int sm_tot[kMaxGroups];
+  for (int g = t; g < G; g += kThreads) {
+    int run = 0;
+    for (unsigned b = 0; b < gridDim.x; ++b) {
+      const int c = __ldcg(a.block_counts + static_cast<size_t>(b) * G + g);
+      a.block_offsets[static_cast<size_t>(b) * G + g] = run;
+      run += c;
+    }
+    sm_tot[g] = run;
+    a.counts[g] = run;
+  }
+  __syncthreads();
+  if (t == 0) {
+    int off = 0;
+    for (int g = 0; g < G; ++g) {
+      a.offsets[g] = off;
+      off += sm_tot[g];
+    }
+    a.offsets[G] = off;
+    *a.done = 0u;
+  }
+}
+
+template <typename TI>
+__global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int i = blockIdx.x * kThreads + t;
+  const bool valid = i < a.T;
+  const int k = a.k, E = a.E, G = a.G;
+  int e[kMaxTopK], sl[kMaxTopK];
+  bool rec[kMaxTopK];
+  bool any = false;
+#pragma unroll
+  for (int p = 0; p < kMaxTopK; ++p) {
+    e[p] = -1;
+    sl[p] = 0;
+    rec[p] = false;
+    if (valid && p < k) {
+      const size_t b = static_cast<size_t>(i) * k + p;
+      rec[p] = a.recompute[b] != 0;
+      e[p] = a.route_e[b];
+      sl[p] = a.slot[b];
+      if (e[p] < 0 || e[p] >= E) rec[p] = false;  // flagged by select
+    }
+  }
+  if (valid) any = a.token_any[i] != 0;
+  const bool shared_row = valid && a.n_shared && (a.refresh || a.shared_policy || any);
+
+  __shared__ unsigned sm_bal[kWarps][kMaxGroups];
+  __shared__ int sm_pre[kWarps][kMaxGroups];
+  __shared__ int sm_rows[kThreads * (kMaxTopK + 1)][2];
+  __shared__ int sm_nrows;
+  if (t == 0) sm_nrows = 0;
+  for (int g = 0; g < G; ++g) {
+    bool has = false;
+    if (g < E) {
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) has |= (rec[p] && e[p] == g);
+    } else {
+      has = shared_row;
+    }
+    const unsigned b = __ballot_sync(0xffffffffu, has);
+    if (lane == 0) sm_bal[warp][g] = b;
+  }
+  __syncthreads();
+  for (int g = t; g < G; g += kThreads) {
+    int run = a.offsets[g] + a.block_offsets[static_cast<size_t>(blockIdx.x) * G + g];
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      sm_pre[w][g] = run;
+      run += __popc(sm_bal[w][g]);
+    }
+  }
+  __syncthreads();
+  const unsigned lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int p = 0; p < kMaxTopK; ++p) {
+    if (rec[p]) {
+      const int g = e[p];
+      const int pos = sm_pre[warp][g] + __popc(sm_bal[warp][g] & lt);
+      a.list[pos] = i * k + sl[p];
+      const int r = atomicAdd(&sm_nrows, 1);
+      sm_rows[r][0] = pos;
+      sm_rows[r][1] = i;
+    }
+  }
+  if (shared_row) {
+    const int pos = sm_pre[warp][E] + __popc(sm_bal[warp][E] & lt);
+    a.list[pos] = i;
+    const int r = atomicAdd(&sm_nrows, 1);
+    sm_rows[r][0] = pos;
+    sm_rows[r][1] = i;
+  }
+  __syncthreads();
+  // Gather the inputs of this block's rows, one warp per row, 16-byte vectors.
+  const int nv = a.D * static_cast<int>(sizeof(TI)) / 16;
+  const uint4* x = static_cast<const uint4*>(a.x);
+  uint4* xg = static_cast<uint4*>(a.xg);
+  const int n = sm_nrows;
+  for (int r = warp; r < n; r += kWarps) {
+    const size_t dst = static_cast<size_t>(sm_rows[r][0]) * nv;
+    const size_t src = static_cast<size_t>(sm_rows[r][1]) * nv;
+    for (int c = lane; c < nv; c += 32) xg[dst + c] = x[src + c];
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t s) {
+  const int grid = (a.T + kThreads - 1) / kThreads;
+  select_kernel<<<grid, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s) {
+  const int grid = (a.T + kThreads - 1) / kThreads;
+  if (bf16) compact_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(a);
+  else compact_kernel<float><<<grid, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace moeca

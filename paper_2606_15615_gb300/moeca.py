@@ -1,0 +1,303 @@
+"""Python binding of libmoeca.so (include/moeca.h): ctypes marshalling only.
+
+The functions keep the C names (moeca_create, moeca_step, ...) and raise
+MoecaError on a non-OK status.  Every step of the layer runs in the CUDA
+library; there is no Python or CPU fallback: importing this module fails
+loudly when the library has not been built.  ``Stack`` is a convenience
+wrapper that holds torch tensors (device memory) and passes their pointers.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import math
+import os
+import re
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libmoeca.so")
+HEADER = os.path.join(os.path.dirname(PKG), "include", "moeca.h")
+
+MOECA_OK = 0
+STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "OOM", -5: "STATE",
+                -6: "TIMEOUT", -7: "DEVICE_STATUS"}
+MOECA_F32, MOECA_BF16 = 0, 1
+MOECA_FFN_AUTO, MOECA_FFN_SIMT = 0, 1
+KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine"]
+
+
+class moeca_config(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("hidden", C.c_int32), ("ffn", C.c_int32),
+                ("n_experts", C.c_int32), ("top_k", C.c_int32), ("n_shared", C.c_int32),
+                ("max_tokens", C.c_int32), ("dtype", C.c_int32),
+                ("lambda1", C.c_float), ("lambda2", C.c_float), ("tau0", C.c_float),
+                ("alpha", C.c_float), ("beta", C.c_float),
+                ("refresh_period", C.c_int32), ("renorm_topk", C.c_int32), ("entropy_norm", C.c_int32),
+                ("shared_policy", C.c_int32), ("reused_meta_policy", C.c_int32),
+                ("gelu_tanh", C.c_int32), ("ffn_impl", C.c_int32)]
+
+
+class moeca_layer_weights(C.Structure):
+    _fields_ = [("w_gate", C.c_void_p), ("b_gate", C.c_void_p), ("w1", C.c_void_p),
+                ("w2", C.c_void_p), ("ws1", C.c_void_p), ("ws2", C.c_void_p)]
+
+
+class moeca_step_args(C.Structure):
+    _fields_ = [("n_tokens", C.c_int32), ("step_index", C.c_int32), ("force_refresh", C.c_int32),
+                ("tau0_override", C.c_float)]
+
+
+class moeca_stats(C.Structure):
+    _fields_ = [(n, C.c_int64) for n in (
+        "layer_steps", "refresh_layer_steps", "branches", "cache_step_branches", "matched",
+        "recomputed", "reused", "tokens_fully_reused", "shared_recomputed",
+        "near_margin_route", "near_margin_score")] + [("device_status", C.c_int32),
+                                                      ("device_detail", C.c_int32)]
+
+    def as_dict(self) -> dict:
+        return {n: getattr(self, n) for n, _ in self._fields_}
+
+
+class moeca_layer_state(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema")]
+
+
+class moeca_layer_trace(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("route_e", "route_w", "tau", "recompute", "slot", "matched",
+                                            "token_any", "counts", "offsets", "list", "layer_in")]
+
+
+class moeca_kernel_times(C.Structure):
+    _fields_ = [("total_ms", C.c_double * 6), ("launches", C.c_int64 * 6)]
+
+
+class MoecaError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with paper_2606_15615_gb300.build.build()")
+    lib = C.CDLL(LIB_PATH)
+    H = C.c_void_p
+    sig = {
+        "moeca_config_default": (None, [C.POINTER(moeca_config)]),
+        "moeca_create": (C.c_int, [C.POINTER(moeca_config), C.POINTER(moeca_layer_weights), C.c_int32,
+                                   C.POINTER(H)]),
+        "moeca_step": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args), C.c_void_p]),
+        "moeca_get_stats": (C.c_int, [H, C.c_int32, C.POINTER(moeca_stats)]),
+        "moeca_reset_stats": (C.c_int, [H]),
+        "moeca_get_layer_state": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_state),
+                                            C.POINTER(C.c_int32), C.c_void_p]),
+        "moeca_set_layer_state": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_state), C.c_int32,
+                                            C.c_void_p]),
+        "moeca_get_layer_trace": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_trace), C.c_void_p]),
+        "moeca_reset": (C.c_int, [H]),
+        "moeca_set_kernel_timing": (C.c_int, [H, C.c_int32]),
+        "moeca_get_kernel_times": (C.c_int, [H, C.POINTER(moeca_kernel_times), C.c_int32]),
+        "moeca_destroy": (C.c_int, [H]),
+        "moeca_status_string": (C.c_char_p, [C.c_int]),
+        "moeca_last_error": (C.c_char_p, [H]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+LIB = _load()
+
+
+def header_functions() -> list:
+    """Names of the functions include/moeca.h declares."""
+    with open(HEADER) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(moeca_[a-z_]+)\s*\(", text)))
+
+
+def _check(status: int, handle=None):
+    if status != MOECA_OK:
+        msg = LIB.moeca_last_error(handle)
+        raise MoecaError(status, msg.decode() if msg else "")
+
+
+def moeca_config_default(**kw) -> moeca_config:
+    cfg = moeca_config()
+    LIB.moeca_config_default(C.byref(cfg))
+    for k, v in kw.items():
+        if not hasattr(cfg, k):
+            raise AttributeError(k)
+        setattr(cfg, k, v)
+    return cfg
+
+
+def moeca_create(cfg: moeca_config, layers: list, device: int = 0):
+    arr = (moeca_layer_weights * len(layers))(*layers)
+    h = C.c_void_p()
+    _check(LIB.moeca_create(C.byref(cfg), arr, device, C.byref(h)))
+    return h
+
+
+def moeca_step(h, x_in_ptr: int, x_out_ptr: int, n_tokens: int, step_index: int,
+               force_refresh: bool = False, tau0_override: float = math.nan, stream: int = 0):
+    args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override)
+    _check(LIB.moeca_step(h, x_in_ptr, x_out_ptr, C.byref(args), stream or None), h)
+
+
+def moeca_get_stats(h, layer: int = -1) -> dict:
+    st = moeca_stats()
+    _check(LIB.moeca_get_stats(h, layer, C.byref(st)), h)
+    return st.as_dict()
+
+
+def moeca_reset_stats(h):
+    _check(LIB.moeca_reset_stats(h), h)
+
+
+def moeca_get_layer_state(h, layer: int, dst: moeca_layer_state, stream: int = 0) -> int:
+    n = C.c_int32()
+    _check(LIB.moeca_get_layer_state(h, layer, C.byref(dst), C.byref(n), stream or None), h)
+    return n.value
+
+
+def moeca_set_layer_state(h, layer: int, src: moeca_layer_state, n_tokens: int, stream: int = 0):
+    _check(LIB.moeca_set_layer_state(h, layer, C.byref(src), n_tokens, stream or None), h)
+
+
+def moeca_get_layer_trace(h, layer: int, dst: moeca_layer_trace, stream: int = 0):
+    _check(LIB.moeca_get_layer_trace(h, layer, C.byref(dst), stream or None), h)
+
+
+def moeca_reset(h):
+    _check(LIB.moeca_reset(h), h)
+
+
+def moeca_set_kernel_timing(h, enable: bool):
+    _check(LIB.moeca_set_kernel_timing(h, int(enable)), h)
+
+
+def moeca_get_kernel_times(h, reset: bool = False) -> dict:
+    kt = moeca_kernel_times()
+    _check(LIB.moeca_get_kernel_times(h, C.byref(kt), int(reset)), h)
+    return {n: (kt.total_ms[i], kt.launches[i]) for i, n in enumerate(KERNEL_KINDS)}
+
+
+def moeca_destroy(h):
+    if h is not None and h.value:
+        _check(LIB.moeca_destroy(h))
+
+
+def moeca_status_string(status: int) -> str:
+    return LIB.moeca_status_string(status).decode()
+
+
+# ---------------------------------------------------------------------------
+# torch convenience wrapper (device memory + streams only)
+# ---------------------------------------------------------------------------
+
+class Stack:
+    """A MoECa layer stack on one GPU, fed with torch CUDA tensors.
+
+    ``layer_weights`` is a list of dicts of numpy float32 arrays (bf16-exact
+    for bf16) as made by ``workloads.make_layer_weights``; they are copied to
+    the device once and kept alive here.
+    """
+
+    def __init__(self, cfg: moeca_config, layer_weights: list, device: int = 0):
+        import numpy as np
+        import torch
+        self.torch = torch
+        self.cfg = cfg
+        self.device = torch.device("cuda", device)
+        self.dtype = torch.bfloat16 if cfg.dtype == MOECA_BF16 else torch.float32
+        self._keep = []
+        cl = []
+        for w in layer_weights:
+            def dev(a, dt=self.dtype):
+                if a is None:
+                    return None
+                if isinstance(a, torch.Tensor):
+                    t = a.to(self.device).to(dt).contiguous()
+                else:
+                    t = torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(self.device).to(dt).contiguous()
+                self._keep.append(t)
+                return t
+            lw = moeca_layer_weights()
+            lw.w_gate = dev(w["w_gate"]).data_ptr()
+            b = dev(w.get("b_gate"), torch.float32)
+            lw.b_gate = b.data_ptr() if b is not None else None
+            lw.w1 = dev(w["w1"]).data_ptr()
+            lw.w2 = dev(w["w2"]).data_ptr()
+            if cfg.n_shared:
+                lw.ws1 = dev(w["ws1"][0]).data_ptr()
+                lw.ws2 = dev(w["ws2"][0]).data_ptr()
+            cl.append(lw)
+        self.handle = moeca_create(cfg, cl, device)
+
+    def close(self):
+        if getattr(self, "handle", None) is not None:
+            moeca_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def stream_ptr(self) -> int:
+        return self.torch.cuda.current_stream(self.device).cuda_stream
+
+    def step(self, x, step_index: int, force_refresh: bool = False, tau0=math.nan, out=None):
+        torch = self.torch
+        T = x.shape[0]
+        if out is None:
+            out = torch.empty_like(x)
+        moeca_step(self.handle, x.data_ptr(), out.data_ptr(), T, step_index, force_refresh, tau0,
+                   self.stream_ptr())
+        return out
+
+    def _empty(self, shape, dtype):
+        return self.torch.empty(shape, dtype=dtype, device=self.device)
+
+    def get_state(self, layer: int) -> dict:
+        torch = self.torch
+        c = self.cfg
+        T = c.max_tokens
+        t = dict(cache_e=self._empty((T, c.top_k), torch.int32), cache_w=self._empty((T, c.top_k), torch.float32),
+                 cache_norm=self._empty((T, c.top_k), torch.float32),
+                 cache_h=self._empty((T, c.top_k, c.hidden), self.dtype),
+                 shared_h=self._empty((T, c.hidden), self.dtype) if c.n_shared else None,
+                 ema=self._empty((T, c.n_experts), torch.float32))
+        st = moeca_layer_state(**{k: (v.data_ptr() if v is not None else None) for k, v in t.items()})
+        n = moeca_get_layer_state(self.handle, layer, st, self.stream_ptr())
+        return {k: (v[:n] if v is not None else None) for k, v in t.items()} | {"n_tokens": n}
+
+    def set_state(self, layer: int, state: dict):
+        n = int(state["cache_e"].shape[0])
+        keep = {k: v.contiguous() for k, v in state.items() if k != "n_tokens" and v is not None}
+        st = moeca_layer_state(**{k: keep[k].data_ptr() if k in keep else None
+                                  for k in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema")})
+        moeca_set_layer_state(self.handle, layer, st, n, self.stream_ptr())
+        self.torch.cuda.current_stream(self.device).synchronize()
+
+    def get_trace(self, layer: int, n_tokens: int) -> dict:
+        torch = self.torch
+        c = self.cfg
+        T, k, G = n_tokens, c.top_k, c.n_experts + c.n_shared
+        t = dict(route_e=self._empty((T, k), torch.int32), route_w=self._empty((T, k), torch.float32),
+                 tau=self._empty((c.n_experts,), torch.float32), recompute=self._empty((T, k), torch.uint8),
+                 slot=self._empty((T, k), torch.int8), matched=self._empty((T, k), torch.uint8),
+                 token_any=self._empty((T,), torch.uint8), counts=self._empty((G,), torch.int32),
+                 offsets=self._empty((G + 1,), torch.int32),
+                 list=self._empty((T * (k + c.n_shared),), torch.int32),
+                 layer_in=self._empty((T, c.hidden), self.dtype))
+        tr = moeca_layer_trace(**{kk: v.data_ptr() for kk, v in t.items()})
+        moeca_get_layer_trace(self.handle, layer, tr, self.stream_ptr())
+        return t
+
+    def stats(self, layer: int = -1) -> dict:
+        return moeca_get_stats(self.handle, layer)

@@ -238,3 +238,34 @@ def tiny_layer(seed: int, T: int, D: int, E: int, k: int, F: int, n_shared: int 
     }
     x0 = st(rng.standard_normal((T, D), dtype=np.float32))
     return w, x0, rng
+
+
+def make_layer_weights_device(wl: Workload, layer: int, device) -> dict:
+    """The layer's weights drawn on the GPU with torch's seeded generator.
+
+    Same distribution and layout as ``make_layer_weights`` (N(0, 0.02^2),
+    rounded to the workload dtype) but drawn by torch's CUDA generator, which
+    makes the multi-GB stacks in seconds.  The values differ from the numpy
+    draw; a CPU consumer (the timed oracle baseline) copies them back.
+    """
+    import torch
+    dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    E, D, F, S = wl.n_experts, wl.hidden, wl.ffn, wl.n_shared
+    seed = (_WEIGHT_SEED + wl.index) * 1_000_003 + layer * 1009
+
+    def draw(tid, shape):
+        g = torch.Generator(device=device)
+        g.manual_seed(seed + tid)
+        t = torch.empty(shape, dtype=torch.float32, device=device)
+        t.normal_(0.0, 0.02, generator=g)
+        return t.to(dt).contiguous()
+
+    out = {"w_gate": draw(_T_GATE, (E, D)), "w1": draw(_T_W1, (E, F, D)), "w2": draw(_T_W2, (E, D, F))}
+    b = _skew_bias(wl)
+    out["b_gate"] = None if b is None else torch.from_numpy(b).to(device)
+    if S:
+        out["ws1"] = draw(_T_WS1, (S, F, D))
+        out["ws2"] = draw(_T_WS2, (S, D, F))
+    else:
+        out["ws1"] = out["ws2"] = None
+    return out

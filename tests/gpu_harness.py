@@ -1,0 +1,212 @@
+"""Helpers for the GPU parity tests: run the CUDA stack and check every layer of
+every step against the oracle, stage by stage (teacher forcing).
+
+For each layer the oracle gets what the GPU had at the start of that stage:
+  router    the layer input            -> top-k ids (exact unless near a tie),
+                                          weights, EMA statistic, tau_e
+  select    the GPU routing, tau and     -> recompute mask (exact unless
+            the pre-step cache              |s - tau| < 1e-5 |tau|), slots,
+                                            matched flags (exact)
+  compact   the GPU mask                  -> per-group row lists (exact)
+  FFN and   the GPU decisions and the     -> layer output, fresh cache rows
+  combine   pre-step cache                   (tolerance), kept rows (exact)
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+from oracle import moeca_oracle as O
+
+NEAR = 1e-5
+
+
+def np_of(t):
+    import torch
+    if t is None:
+        return None
+    if t.dtype == torch.bfloat16:
+        t = t.float()
+    return t.cpu().numpy()
+
+
+def rel_l2(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+@dataclass
+class Report:
+    steps: int = 0
+    layers_checked: int = 0
+    near_route: int = 0
+    near_score: int = 0
+    branches: int = 0
+    recomputed: int = 0
+    reused: int = 0
+    unmatched: int = 0
+    max_rel_l2: float = 0.0
+    max_abs: float = 0.0
+    notes: list = field(default_factory=list)
+
+
+def params_of(cfg) -> O.Params:
+    return O.Params(
+        top_k=cfg.top_k, lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau0=cfg.tau0, alpha=cfg.alpha,
+        beta=cfg.beta, refresh_period=cfg.refresh_period, renorm_topk=bool(cfg.renorm_topk),
+        entropy_norm="log_t" if cfg.entropy_norm == 0 else "minmax",
+        shared_policy="sync" if cfg.shared_policy == 0 else "always",
+        reused_meta_policy="keep" if cfg.reused_meta_policy == 0 else "overwrite",
+        gelu="tanh" if cfg.gelu_tanh else "erf")
+
+
+def oracle_weights(w: dict) -> dict:
+    return {k: (None if v is None else np.asarray(v, np.float64)) for k, v in w.items()}
+
+
+def state_to_oracle(st: dict | None, T, D, E, k, S) -> O.LayerState:
+    if st is None or st["n_tokens"] == 0:
+        return O.LayerState.empty(T, D, E, k, S)
+    return O.LayerState(
+        cache_e=np_of(st["cache_e"]).astype(np.int32), cache_w=np_of(st["cache_w"]).astype(np.float64),
+        cache_norm=np_of(st["cache_norm"]).astype(np.float64), cache_h=np_of(st["cache_h"]).astype(np.float64),
+        shared_h=None if st["shared_h"] is None else np_of(st["shared_h"]).astype(np.float64),
+        C=np_of(st["ema"]).astype(np.float64).T.copy(), valid=True)
+
+
+def expected_lists(e, rec, slot, token_any, E, k, n_shared, refresh, shared_always):
+    """Rows of every expert group in ascending token order (the compaction's contract)."""
+    T = e.shape[0]
+    groups = [[] for _ in range(E + n_shared)]
+    for i in range(T):
+        for p in range(k):
+            if rec[i, p]:
+                groups[int(e[i, p])].append(i * k + int(slot[i, p]))
+        if n_shared and (refresh or shared_always or token_any[i]):
+            groups[E].append(i)
+    counts = np.array([len(g) for g in groups], np.int32)
+    offsets = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    flat = np.array([r for g in groups for r in g], np.int32)
+    return counts, offsets, flat
+
+
+def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dict, out_gpu: np.ndarray,
+                refresh: bool, bf16: bool, out_tol=None):
+    """Teacher-forced comparison of one layer step.  Raises AssertionError."""
+    T = tr["route_e"].shape[0]
+    D, E, k, S = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.n_shared
+    prm = params_of(cfg)
+    wo = oracle_weights(w)
+    u = np_of(tr["layer_in"]).astype(np.float64)
+    e_g = np_of(tr["route_e"]).astype(np.int64)
+    w_g = np_of(tr["route_w"]).astype(np.float64)
+    # ---- router (Eq. 7)
+    e_o, w_o, near = O.route(u, wo["w_gate"], wo.get("b_gate"), k, prm.renorm_topk)
+    ok = near >= NEAR
+    rep.near_route += int((~ok).sum())
+    bad = np.nonzero(ok & (e_o != e_g).any(axis=1))[0]
+    assert len(bad) == 0, f"top-k ids differ on {len(bad)} tokens, e.g. {bad[:5]}: gpu {e_g[bad[:3]]} oracle {e_o[bad[:3]]}"
+    wt = 2e-6
+    assert np.allclose(w_g[ok], w_o[ok], rtol=0, atol=wt), f"gate weights: max err {np.abs(w_g[ok]-w_o[ok]).max()}"
+    # ---- EMA (Eq. 10) from the GPU's pre-step statistic and routing
+    C_pre = np.zeros((E, T)) if (pre is None or pre["n_tokens"] == 0) else np_of(pre["ema"]).astype(np.float64).T
+    C_o = O.ema_update(C_pre, e_g, prm.beta)
+    C_g = np_of(post["ema"]).astype(np.float64).T
+    assert np.allclose(C_g, C_o, rtol=2e-6, atol=1e-7), f"EMA: max err {np.abs(C_g - C_o).max()}"
+    # ---- tau (Eq. 11-12) from the GPU's statistic
+    tau_o = O.expert_threshold(O.normalized_entropy(C_g, prm.entropy_norm), prm.tau0, prm.alpha)
+    tau_g = np_of(tr["tau"]).astype(np.float64)
+    fin = np.isfinite(tau_o)
+    assert np.allclose(tau_g[fin], tau_o[fin], rtol=1e-5, atol=1e-6), f"tau: {tau_g} vs {tau_o}"
+    assert np.array_equal(np.isinf(tau_g), np.isinf(tau_o))
+    # ---- select (Sec. 4.2, Eq. 9) from the GPU routing, tau and pre-step cache
+    st_pre = state_to_oracle(pre, T, D, E, k, S)
+    sel = O.select_branches(e_g, w_g, st_pre.cache_e, st_pre.cache_w, st_pre.cache_norm, tau_g,
+                            prm.lambda1, prm.lambda2, refresh)
+    rec_g = np_of(tr["recompute"]).astype(bool)
+    slot_g = np_of(tr["slot"]).astype(np.int64)
+    mat_g = np_of(tr["matched"]).astype(bool)
+    assert np.array_equal(slot_g, sel["slot"]), "slots differ"
+    assert np.array_equal(mat_g, sel["matched"]), "matched flags differ"
+    far = sel["margin"] >= NEAR
+    rep.near_score += int((~far).sum())
+    diff = far & (rec_g != sel["recompute"])
+    assert not diff.any(), f"recompute mask differs on {int(diff.sum())} branches"
+    any_g = np_of(tr["token_any"]).astype(bool)
+    assert np.array_equal(any_g, rec_g.any(axis=1))
+    # ---- compaction
+    cnt, off, flat = expected_lists(e_g, rec_g, slot_g, any_g, E, k, S, refresh, cfg.shared_policy == 1)
+    assert np.array_equal(np_of(tr["counts"]), cnt), "group counts"
+    assert np.array_equal(np_of(tr["offsets"]), off), "group offsets"
+    assert np.array_equal(np_of(tr["list"])[: off[-1]], flat), "row lists"
+    # ---- FFN + combine (Eq. 5, Eq. 8) from the GPU decisions and pre-step cache
+    out_o, new_o, _ = O.recompute_and_combine(st_pre, u, e_g, w_g, rec_g, slot_g, wo, prm, refresh)
+    rl = rel_l2(out_gpu, out_o)
+    ma = float(np.abs(out_gpu - out_o).max())
+    rep.max_rel_l2 = max(rep.max_rel_l2, rl)
+    rep.max_abs = max(rep.max_abs, ma)
+    if out_tol is None:
+        out_tol = (1e-2, 5e-2) if bf16 else (1e-5, None)
+    assert rl <= out_tol[0], f"layer output rel L2 {rl:.3e}"
+    if out_tol[1] is not None:
+        assert ma <= out_tol[1], f"layer output max abs {ma:.3e}"
+    ch_g = np_of(post["cache_h"]).astype(np.float64)
+    fresh = np.zeros((T, k), bool)
+    for i, p in np.argwhere(rec_g):
+        fresh[i, slot_g[i, p]] = True
+    if fresh.any():
+        rf = rel_l2(ch_g[fresh], new_o.cache_h[fresh])
+        assert rf <= (1e-2 if bf16 else 1e-5), f"fresh cache rows rel L2 {rf:.3e}"
+    if (~fresh).any() and pre is not None and pre["n_tokens"]:
+        assert np.array_equal(ch_g[~fresh], st_pre.cache_h[~fresh]), "reused cache rows changed"
+    assert np.array_equal(np_of(post["cache_e"]), new_o.cache_e), "cache expert ids"
+    assert np.array_equal(np_of(post["cache_w"]).astype(np.float64), new_o.cache_w.astype(np.float32).astype(np.float64)), "cache weights"
+    nrm = np.sqrt((ch_g ** 2).sum(axis=2))
+    assert np.allclose(np_of(post["cache_norm"]), nrm, rtol=2e-5, atol=1e-6), "cached norms"
+    if S:
+        sh_g = np_of(post["shared_h"]).astype(np.float64)
+        rs = rel_l2(sh_g, new_o.shared_h)
+        assert rs <= (1e-2 if bf16 else 1e-5), f"shared rows rel L2 {rs:.3e}"
+    rep.layers_checked += 1
+    rep.branches += T * k
+    rep.recomputed += int(rec_g.sum())
+    rep.reused += int((~rec_g).sum())
+    rep.unmatched += int((~mat_g).sum()) if not refresh else 0
+
+
+def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True, bf16=True, out_tol=None,
+                   forces=None):
+    """Step the GPU stack over ``xs`` and check every layer of every step."""
+    import torch
+    rep = Report()
+    dt = torch.bfloat16 if bf16 else torch.float32
+    L = cfg.n_layers
+    prev_T = None
+    for t, x in enumerate(xs):
+        T = x.shape[0]
+        force = bool(forces and forces[t])
+        N = cfg.refresh_period
+        refresh = force or prev_T != T or t == 0 or (N > 0 and t % N == 0)
+        if refresh_flags is not None:
+            refresh_flags.append(refresh)
+        pre = [stack.get_state(l) for l in range(L)] if check else None
+        if check and prev_T != T:
+            pre = [None] * L
+        xd = torch.from_numpy(np.ascontiguousarray(x, np.float32)).cuda().to(dt)
+        out = stack.step(xd, t, force_refresh=force)
+        torch.cuda.synchronize()
+        if check:
+            for l in range(L):
+                tr = stack.get_trace(l, T)
+                post = stack.get_state(l)
+                if l + 1 < L:
+                    out_l = np_of(stack.get_trace(l + 1, T)["layer_in"]).astype(np.float64)
+                else:
+                    out_l = np_of(out).astype(np.float64)
+                check_layer(rep, cfg, layer_weights[l], pre[l], post, tr, out_l, refresh, bf16, out_tol)
+        rep.steps += 1
+        prev_T = T
+    return rep, out

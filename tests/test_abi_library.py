@@ -1,0 +1,51 @@
+"""The C-ABI library builds, loads without a GPU and exports what the header declares."""
+import ctypes
+
+import pytest
+
+from paper_2606_15615_gb300 import build
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    from paper_2606_15615_gb300 import moeca
+    return moeca
+
+
+def test_every_declared_function_is_exported(lib):
+    names = lib.header_functions()
+    assert len(names) >= 14
+    so = ctypes.CDLL(lib.LIB_PATH)
+    missing = [n for n in names if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_defaults(lib):
+    assert lib.moeca_status_string(0) == "ok"
+    assert lib.moeca_status_string(-1) == "invalid argument"
+    assert lib.moeca_status_string(-6) == "device wait timed out"
+    cfg = lib.moeca_config_default()
+    assert (cfg.lambda1, cfg.lambda2) == (1.0, 0.5)
+    assert abs(cfg.tau0 - 0.8) < 1e-7 and abs(cfg.alpha - 0.6) < 1e-7 and abs(cfg.beta - 0.65) < 1e-7
+    assert cfg.renorm_topk == 1 and cfg.gelu_tanh == 1 and cfg.dtype == lib.MOECA_BF16
+
+
+def test_host_validation_needs_no_gpu(lib):
+    L = lib.LIB
+    h = ctypes.c_void_p()
+    assert L.moeca_create(None, None, 0, ctypes.byref(h)) == -1
+    assert b"NULL" in L.moeca_last_error(None)
+    cfg = lib.moeca_config_default(n_layers=1, hidden=64, ffn=64, n_experts=4, top_k=5, max_tokens=8)
+    w = (lib.moeca_layer_weights * 1)()
+    assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # top_k > E
+    cfg.top_k = 2
+    cfg.alpha = 1.0
+    assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # alpha outside [0, 1)
+    cfg.alpha = 0.6
+    assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # NULL weights
+    cfg.hidden = 60
+    w[0].w_gate = w[0].w1 = w[0].w2 = 4096
+    assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -2  # hidden not a multiple of 8
+    assert L.moeca_step(None, None, None, None, None) == -1
+    assert L.moeca_destroy(None) == 0
