@@ -194,7 +194,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
                           int32_t device, moeca_handle** out);
 
 /* Run the stack for one denoising step on `stream`.  x_in [T, D] and
- * x_out [T, D] are device buffers of the config dtype that must not overlap.
+ * x_out [T, D] are device buffers of the config dtype that must not overlap
+ * (both may be NULL when T = 0, which does nothing).
  * The step is a full-computation step when forced, on the first step after
  * create / reset, when T differs from the previous step, or when
  * refresh_period > 0 divides step_index (Sec. 4.1); otherwise a cache step.

@@ -336,13 +336,14 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
 moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const moeca_step_args* args,
                         void* stream) {
   if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
-  if (!args || !x_in || !x_out) return fail(h, MOECA_ERR_INVALID_ARG, "args, x_in or x_out is NULL");
+  if (!args) return fail(h, MOECA_ERR_INVALID_ARG, "args is NULL");
   const moeca_config& c = h->cfg;
   const int T = args->n_tokens;
   if (T < 0 || T > c.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of [0, max_tokens]");
   moeca_status st = check_device_status(h);
   if (st != MOECA_OK) return st;
   if (T == 0) return MOECA_OK;
+  if (!x_in || !x_out) return fail(h, MOECA_ERR_INVALID_ARG, "x_in or x_out is NULL");
   const size_t xbytes = static_cast<size_t>(T) * c.hidden * h->es;
   if (overlaps(x_in, x_out, xbytes)) return fail(h, MOECA_ERR_INVALID_ARG, "x_in and x_out overlap");
   if (reinterpret_cast<uintptr_t>(x_in) % 16 || reinterpret_cast<uintptr_t>(x_out) % 16)
