@@ -376,6 +376,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--ref-tau0", type=float, default=0.8)
+    ap.add_argument("--tau0", type=float, default=None,
+                    help="use this tau0 for the headline point instead of calibrating it (profiling runs)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -400,7 +402,10 @@ def main():
     head = None
     pk, pk_src = peaks()
     for tgt in targets:
-        tau0, achieved = runner.calibrate(tgt, W_, K)
+        if args.tau0 is not None and abs(tgt - args.reuse) < 1e-9:
+            tau0 = args.tau0
+        else:
+            tau0, achieved = runner.calibrate(tgt, W_, K)
         is_head = abs(tgt - args.reuse) < 1e-9
         sampler = None
         if is_head and rank == 0:

@@ -14,7 +14,9 @@ namespace {
 
 constexpr int kWarps = 8;
 
-template <typename TI>
+// CG 16-byte chunks per lane are in flight at once (all k cache rows, the
+// shared row and x loaded before any arithmetic).
+template <typename TI, int KMAX, int CG>
 __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -25,11 +27,11 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   TI* out = static_cast<TI*>(a.out) + static_cast<size_t>(i) * D;
   const TI* ch = static_cast<const TI*>(a.cache_h) + static_cast<size_t>(i) * k * D;
   const TI* sh = a.shared_h ? static_cast<const TI*>(a.shared_h) + static_cast<size_t>(i) * D : nullptr;
-  float w[kMaxTopK];
-  int q[kMaxTopK];
+  float w[KMAX];
+  int q[KMAX];
   bool bad = false;
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) {
+  for (int p = 0; p < KMAX; ++p) {
     w[p] = 0.f;
     q[p] = 0;
     if (p < k) {
@@ -42,52 +44,71 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
     if (lane == 0) report_status(a.status, kStatusBadIndex, 3000000 + i);
     return;
   }
-  float ss[kMaxTopK];
+  float ss[KMAX];
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) ss[p] = 0.f;
-  for (int c = lane; c < nvec; c += 32) {
-    float y[V];
+  for (int p = 0; p < KMAX; ++p) ss[p] = 0.f;
+  for (int c0 = 0; c0 < nvec; c0 += 32 * CG) {
+    float h[CG][KMAX][V], xs[CG][V], hs[CG][V];
 #pragma unroll
-    for (int j = 0; j < V; ++j) y[j] = 0.f;
+    for (int g = 0; g < CG; ++g) {
+      const int c = c0 + g * 32 + lane;
+      if (c < nvec) {
 #pragma unroll
-    for (int p = 0; p < kMaxTopK; ++p) {
-      if (p < k) {
-        float h[V];
-        load_vec(ch + static_cast<size_t>(q[p]) * D + c * V, h);
-#pragma unroll
-        for (int j = 0; j < V; ++j) {
-          y[j] = fmaf(w[p], h[j], y[j]);
-          ss[p] = fmaf(h[j], h[j], ss[p]);
-        }
+        for (int p = 0; p < KMAX; ++p)
+          if (p < k) load_vec(ch + static_cast<size_t>(q[p]) * D + c * V, h[g][p]);
+        load_vec(x + c * V, xs[g]);
+        if (sh) load_vec(sh + c * V, hs[g]);
       }
     }
-    if (sh) {
-      float h[V];
-      load_vec(sh + c * V, h);
 #pragma unroll
-      for (int j = 0; j < V; ++j) y[j] += h[j];
+    for (int g = 0; g < CG; ++g) {
+      const int c = c0 + g * 32 + lane;
+      if (c < nvec) {
+        float y[V];
+#pragma unroll
+        for (int j = 0; j < V; ++j) y[j] = 0.f;
+#pragma unroll
+        for (int p = 0; p < KMAX; ++p) {
+          if (p < k) {
+#pragma unroll
+            for (int j = 0; j < V; ++j) {
+              y[j] = fmaf(w[p], h[g][p][j], y[j]);
+              ss[p] = fmaf(h[g][p][j], h[g][p][j], ss[p]);
+            }
+          }
+        }
+        if (sh) {
+#pragma unroll
+          for (int j = 0; j < V; ++j) y[j] += hs[g][j];
+        }
+#pragma unroll
+        for (int j = 0; j < V; ++j) xs[g][j] += y[j];
+        store_vec(out + c * V, xs[g]);
+      }
     }
-    float xv[V];
-    load_vec(x + c * V, xv);
-#pragma unroll
-    for (int j = 0; j < V; ++j) xv[j] += y[j];
-    store_vec(out + c * V, xv);
   }
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) {
+  for (int p = 0; p < KMAX; ++p) {
     if (p < k) {
-      const float s = warp_sum(ss[p]);
-      if (lane == 0) a.cache_norm[static_cast<size_t>(i) * k + q[p]] = sqrtf(s);
+      const float s2 = warp_sum(ss[p]);
+      if (lane == 0) a.cache_norm[static_cast<size_t>(i) * k + q[p]] = sqrtf(s2);
     }
   }
+}
+
+template <typename TI>
+void launch_t(const CombineArgs& a, cudaStream_t s) {
+  const int grid = (a.T + kWarps - 1) / kWarps;
+  if (a.k <= 2) combine_kernel<TI, 2, 4><<<grid, kWarps * 32, 0, s>>>(a);
+  else if (a.k <= 4) combine_kernel<TI, 4, 2><<<grid, kWarps * 32, 0, s>>>(a);
+  else combine_kernel<TI, 8, 1><<<grid, kWarps * 32, 0, s>>>(a);
 }
 
 }  // namespace
 
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s) {
-  const int grid = (a.T + kWarps - 1) / kWarps;
-  if (bf16) combine_kernel<__nv_bfloat16><<<grid, kWarps * 32, 0, s>>>(a);
-  else combine_kernel<float><<<grid, kWarps * 32, 0, s>>>(a);
+  if (bf16) launch_t<__nv_bfloat16>(a, s);
+  else launch_t<float>(a, s);
   return cudaGetLastError();
 }
 

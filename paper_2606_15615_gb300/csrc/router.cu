@@ -167,17 +167,37 @@ __global__ void __launch_bounds__(kWarps * 32) router_kernel(RouterArgs a) {
   __syncthreads();
   if (ticket != gridDim.x - 1) return;
   __threadfence();
+  // Thread t sums blocks j, j + J, j + 2J, ... of expert e = t % E (J = 256 / E
+  // lanes per expert, loads independent); the J sums are then added in j order.
   __shared__ double sm_H[EMAX];
   __shared__ int sm_live[EMAX];
   __shared__ double sm_lo, sm_hi;
-  if (t < E) {
+  __shared__ double sm_red[kWarps * 32][2];
+  {
+    const int J = (kWarps * 32) / E;
+    const int e = t % E, j = t / E;
     double S = 0.0, U = 0.0;
-    for (unsigned b = 0; b < gridDim.x; ++b) {
-      S += static_cast<double>(__ldcg(a.partials + (static_cast<size_t>(b) * E + t) * 2 + 0));
-      U += static_cast<double>(__ldcg(a.partials + (static_cast<size_t>(b) * E + t) * 2 + 1));
+    if (j < J) {
+      const float2* part = reinterpret_cast<const float2*>(a.partials);
+#pragma unroll 4
+      for (unsigned b = j; b < gridDim.x; b += J) {
+        const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
+        S += static_cast<double>(v.x);
+        U += static_cast<double>(v.y);
+      }
     }
-    sm_live[t] = S > 0.0;
-    sm_H[t] = S > 0.0 ? log(S) - U / S : 0.0;
+    sm_red[t][0] = S;
+    sm_red[t][1] = U;
+    __syncthreads();
+    if (t < E) {
+      double Ss = 0.0, Us = 0.0;
+      for (int jj = 0; jj < J; ++jj) {
+        Ss += sm_red[jj * E + t][0];
+        Us += sm_red[jj * E + t][1];
+      }
+      sm_live[t] = Ss > 0.0;
+      sm_H[t] = Ss > 0.0 ? log(Ss) - Us / Ss : 0.0;
+    }
   }
   __syncthreads();
   if (t == 0) {

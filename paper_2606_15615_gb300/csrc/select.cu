@@ -205,18 +205,28 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
   __syncthreads();
   if (ticket != gridDim.x - 1) return;
   __threadfence();
+  // Chunks of 16 blocks: every thread loads counts in parallel, then one
+  // thread per group scans the chunk in block order.
   __shared__ int sm_tot[kMaxGroups];
-  for (int g = t; g < G; g += kThreads) {
-    int run = 0;
-    for (unsigned b = 0; b < gridDim.x; ++b) {
-      const int c = __ldcg(a.block_counts + static_cast<size_t>(b) * G + g);
-      a.block_offsets[static_cast<size_t>(b) * G + g] = run;
-      run += c;
+  __shared__ int sm_chunk[16][kMaxGroups];
+  for (int g = t; g < G; g += kThreads) sm_tot[g] = 0;
+  for (unsigned b0 = 0; b0 < gridDim.x; b0 += 16) {
+    const int nb = min(16u, gridDim.x - b0);
+    __syncthreads();
+    for (int idx = t; idx < nb * G; idx += kThreads)
+      sm_chunk[idx / G][idx % G] = __ldcg(a.block_counts + static_cast<size_t>(b0 + idx / G) * G + idx % G);
+    __syncthreads();
+    for (int g = t; g < G; g += kThreads) {
+      int run = sm_tot[g];
+      for (int j = 0; j < nb; ++j) {
+        a.block_offsets[static_cast<size_t>(b0 + j) * G + g] = run;
+        run += sm_chunk[j][g];
+      }
+      sm_tot[g] = run;
     }
-    sm_tot[g] = run;
-    a.counts[g] = run;
   }
   __syncthreads();
+  for (int g = t; g < G; g += kThreads) a.counts[g] = sm_tot[g];
   if (t == 0) {
     int off = 0;
     for (int g = 0; g < G; ++g) {
@@ -303,11 +313,28 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
   const int nv = a.D * static_cast<int>(sizeof(TI)) / 16;
   const uint4* x = static_cast<const uint4*>(a.x);
   uint4* xg = static_cast<uint4*>(a.xg);
+  // Four rows per warp at a time, every load issued before the stores.
   const int n = sm_nrows;
-  for (int r = warp; r < n; r += kWarps) {
-    const size_t dst = static_cast<size_t>(sm_rows[r][0]) * nv;
-    const size_t src = static_cast<size_t>(sm_rows[r][1]) * nv;
-    for (int c = lane; c < nv; c += 32) xg[dst + c] = x[src + c];
+  for (int r0 = warp * 4; r0 < n; r0 += kWarps * 4) {
+    for (int c0 = 0; c0 < nv; c0 += 32 * 4) {
+      uint4 v[4][4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int c = c0 + q * 32 + lane;
+          if (r0 + j < n && c < nv) v[j][q] = x[static_cast<size_t>(sm_rows[r0 + j][1]) * nv + c];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int c = c0 + q * 32 + lane;
+          if (r0 + j < n && c < nv) xg[static_cast<size_t>(sm_rows[r0 + j][0]) * nv + c] = v[j][q];
+        }
+      }
+    }
   }
 }
 
