@@ -105,11 +105,16 @@ def router_logits(u: np.ndarray, w_gate: np.ndarray, b_gate=None) -> np.ndarray:
 def route(u, w_gate, b_gate, k: int, renorm: bool):
     """Top-k routing set B_i^t = {(e_p, w_p)}, p = 1..k (Eq. 7).
 
-    Returns (e [T,k] int32, w [T,k] float64, near [T] float64) where ``near``
-    is the smallest gap between adjacent ranks 1..k+1 of the float32 logits,
-    relative to the token's largest |logit| (how close the choice is to a tie).
+    Returns (e [T,k] int32, w [T,k] float64, near [T] float64, cond [T]) where
+    ``near`` is the smallest gap between adjacent ranks 1..k+1 of the float32
+    logits relative to ``cond``, the token's largest sum_d |u_d W_ed| (+|b_e|):
+    the magnitude a float32 dot product accumulates, which sets its rounding.
     """
     z = router_logits(u, w_gate, b_gate)
+    cond = np.abs(np.asarray(u, np.float64)) @ np.abs(np.asarray(w_gate, np.float64)).T
+    if b_gate is not None:
+        cond = cond + np.abs(np.asarray(b_gate, np.float64))[None, :]
+    cond = np.maximum(cond.max(axis=1), _TINY)
     T, E = z.shape
     if not (1 <= k <= E):
         raise ValueError("top_k must be in [1, E]")
@@ -125,12 +130,11 @@ def route(u, w_gate, b_gate, k: int, renorm: bool):
         w = w / w.sum(axis=1, keepdims=True)
     ranks = min(k + 1, E)
     zs = np.take_along_axis(z32.astype(np.float64), order[:, :ranks], axis=1)
-    scale = np.maximum(np.abs(z32).max(axis=1).astype(np.float64), _TINY)
     if ranks > 1:
-        near = (zs[:, :-1] - zs[:, 1:]).min(axis=1) / scale
+        near = (zs[:, :-1] - zs[:, 1:]).min(axis=1) / cond
     else:
         near = np.full(T, np.inf)
-    return e_sel, w, near
+    return e_sel, w, near, cond
 
 
 # ---------------------------------------------------------------------------
@@ -341,7 +345,7 @@ def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, ref
     u = np.asarray(u, np.float64)
     T, D = u.shape
     k = prm.top_k
-    e_cur, w_cur, near = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
+    e_cur, w_cur, near, _ = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
     C = ema_update(state.C, e_cur, prm.beta)
     Hbar = normalized_entropy(C, prm.entropy_norm)
     tau = expert_threshold(Hbar, prm.tau0, prm.alpha)

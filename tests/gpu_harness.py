@@ -77,6 +77,22 @@ def state_to_oracle(st: dict | None, T, D, E, k, S) -> O.LayerState:
         C=np_of(st["ema"]).astype(np.float64).T.copy(), valid=True)
 
 
+def gate_weight_tol(w_o, cond):
+    """Tolerance of float32 gate weights against the float64 oracle.
+
+    A float32 dot product over D terms misses the exact logit by about
+    2^-24 * sum_d |u_d W_ed| (= cond); a softmax weight moves by at most
+    2 w (1 - w) times a logit error.  8x that, plus 2e-6 of float32 softmax.
+    """
+    return 2e-6 + 8 * 2.0 ** -24 * cond[:, None] * 2 * w_o * (1 - w_o)
+
+
+def check_gate_weights(w_g, w_o, cond):
+    tol = gate_weight_tol(w_o, cond)
+    err = np.abs(w_g - w_o)
+    assert (err <= tol).all(), f"gate weights: worst err {err.max():.3e}, tol there {tol.flat[err.argmax()]:.3e}"
+
+
 def expected_lists(e, rec, slot, token_any, E, k, n_shared, refresh, shared_always):
     """Rows of every expert group in ascending token order (the compaction's contract)."""
     T = e.shape[0]
@@ -104,13 +120,12 @@ def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
     e_g = np_of(tr["route_e"]).astype(np.int64)
     w_g = np_of(tr["route_w"]).astype(np.float64)
     # ---- router (Eq. 7)
-    e_o, w_o, near = O.route(u, wo["w_gate"], wo.get("b_gate"), k, prm.renorm_topk)
+    e_o, w_o, near, cond = O.route(u, wo["w_gate"], wo.get("b_gate"), k, prm.renorm_topk)
     ok = near >= NEAR
     rep.near_route += int((~ok).sum())
     bad = np.nonzero(ok & (e_o != e_g).any(axis=1))[0]
     assert len(bad) == 0, f"top-k ids differ on {len(bad)} tokens, e.g. {bad[:5]}: gpu {e_g[bad[:3]]} oracle {e_o[bad[:3]]}"
-    wt = 2e-6
-    assert np.allclose(w_g[ok], w_o[ok], rtol=0, atol=wt), f"gate weights: max err {np.abs(w_g[ok]-w_o[ok]).max()}"
+    check_gate_weights(w_g[ok], w_o[ok], cond[ok])
     # ---- EMA (Eq. 10) from the GPU's pre-step statistic and routing
     C_pre = np.zeros((E, T)) if (pre is None or pre["n_tokens"] == 0) else np_of(pre["ema"]).astype(np.float64).T
     C_o = O.ema_update(C_pre, e_g, prm.beta)

@@ -54,7 +54,7 @@ def textbook_moe(u, w, k):
 
 def test_topk_weights_renormalised_sum_to_one():
     w, x, _ = tiny_layer(1, T=64, D=16, E=8, k=3, F=8, bias=True)
-    e, wt, _ = O.route(x, w["w_gate"], w["b_gate"], 3, renorm=True)
+    e, wt, _, _ = O.route(x, w["w_gate"], w["b_gate"], 3, renorm=True)
     np.testing.assert_allclose(wt.sum(axis=1), 1.0, rtol=0, atol=1e-12)
     assert (wt[:, :-1] >= wt[:, 1:] - 1e-15).all(), "branches are ordered by descending weight"
     for row in e:
@@ -64,7 +64,7 @@ def test_topk_weights_renormalised_sum_to_one():
 def test_topk_without_renorm_keeps_softmax_ratios():
     # Softmax fixes w_p / w_p' = exp(z_p - z_p') and sum over all E of p = 1.
     w, x, _ = tiny_layer(2, T=32, D=12, E=6, k=2, F=4)
-    e, wt, _ = O.route(x, w["w_gate"], None, 2, renorm=False)
+    e, wt, _, _ = O.route(x, w["w_gate"], None, 2, renorm=False)
     z = x.astype(np.float64) @ w["w_gate"].astype(np.float64).T
     for t in range(32):
         np.testing.assert_allclose(wt[t, 0] / wt[t, 1], math.exp(z[t, e[t, 0]] - z[t, e[t, 1]]), rtol=1e-12)
@@ -74,7 +74,7 @@ def test_topk_without_renorm_keeps_softmax_ratios():
 
 def test_topk_ties_go_to_lower_expert_id():
     wg = np.array([[1.0, 0.0], [1.0, 0.0], [0.5, 0.0], [1.0, 0.0]])
-    e, wt, near = O.route(np.array([[2.0, 1.0]]), wg, None, 2, renorm=True)
+    e, wt, near, _ = O.route(np.array([[2.0, 1.0]]), wg, None, 2, renorm=True)
     assert e.tolist() == [[0, 1]]
     np.testing.assert_allclose(wt, [[0.5, 0.5]])
     assert near[0] == 0.0
