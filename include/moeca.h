@@ -239,6 +239,57 @@ moeca_status moeca_get_kernel_times(moeca_handle* h, moeca_kernel_times* out, in
 /* Free everything the handle owns.  NULL is accepted. */
 moeca_status moeca_destroy(moeca_handle* h);
 
+/* ---- Allocation-free router call ---------------------------------------
+ * The paper has no counterpart to this call.  It exists for callers that
+ * cannot allocate device memory, so cannot create a handle (moeca_create
+ * allocates the caches and the workspace): code running inside a host
+ * framework that owns every device allocation through its own pool, or a
+ * deployment whose device memory budget is fixed when it starts.
+ *
+ * moeca_route_noalloc runs the router of one layer on caller-owned device
+ * buffers: gate logits, softmax, top-k (Eq. 7), the EMA statistic update
+ * (Eq. 10) and the per-expert thresholds (Eq. 11-12), the same computation
+ * moeca_step runs first in every layer.  It allocates nothing (no cudaMalloc,
+ * no cudaFree, no allocating library routine).  Its only scratch memory, the
+ * per-block entropy partial sums and a completion counter, is one fixed
+ * array compiled into the library: 256 KB + 256 B, held by every GPU that
+ * loads the library until the process exits.
+ *
+ * Limit: ceil(n_tokens / 16) * n_experts <= 32768 (up to 8192 tokens with 64
+ * experts, 32768 tokens with 16).  A larger call returns MOECA_ERR_UNSUPPORTED
+ * and launches nothing.  Other errors: MOECA_ERR_INVALID_ARG (NULL or
+ * misaligned pointer, a size out of range), MOECA_ERR_CUDA (the scratch
+ * address lookup or the launch failed).
+ *
+ * The first call on each device looks up that device's address of the scratch
+ * array (cudaGetSymbolAddress, with that device current), so make the first
+ * call on a device before any stream capture.  Every call shares the one
+ * array, which keeps the last call's contents; each call clears what must
+ * start at zero itself.  Calls that overlap on the GPU (on different streams
+ * or from different host threads) race on the scratch: serialise them.
+ * Runs on the current device, asynchronously on `stream`. */
+typedef struct {
+  int32_t dtype;         /* moeca_dtype of x and w_gate                       */
+  int32_t n_tokens;      /* T >= 1                                             */
+  int32_t hidden;        /* D: multiple of 8 (bf16) or 4 (fp32)                */
+  int32_t n_experts;     /* E, 1..64                                           */
+  int32_t top_k;         /* k, 1..min(8, E)                                    */
+  int32_t renorm_topk;   /* as in moeca_config                                 */
+  int32_t entropy_norm;  /* as in moeca_config                                 */
+  float beta;            /* Eq. 10 EMA decay, [0, 1)                           */
+  float tau0;            /* Eq. 12 base threshold                              */
+  float alpha;           /* Eq. 12 adaptation strength, [0, 1)                 */
+  const void* x;         /* [T, D] device, 16-byte aligned                     */
+  const void* w_gate;    /* [E, D] device, 16-byte aligned                     */
+  const float* b_gate;   /* [E] device, or NULL                                */
+  float* ema;            /* [T, E] device, C_{e,i} at [i*E + e]: read, then updated in place */
+  int32_t* route_e;      /* [T, k] device output: expert ids, descending logit */
+  float* route_w;        /* [T, k] device output: gate weights                */
+  float* tau;            /* [E] device output: thresholds tau_e               */
+} moeca_route_args;
+
+moeca_status moeca_route_noalloc(const moeca_route_args* args, void* stream);
+
 const char* moeca_status_string(moeca_status s);
 /* Message of the last error on this handle ("" if none); NULL handle: the
  * last moeca_create() failure of this thread. */

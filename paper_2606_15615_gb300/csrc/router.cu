@@ -9,8 +9,11 @@
 // which the last block to finish derives the spatial entropy
 //   H_e = ln S_e - U_e / S_e  (= -sum_i P ln P with P = C / S, Eq. 11),
 // its normalisation and the expert threshold tau_e (Eq. 12).
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.h"
+#include "moeca.h"
 
 namespace moeca {
 namespace {
@@ -245,3 +248,98 @@ cudaError_t launch_router(const RouterArgs& a, bool bf16, cudaStream_t s) {
 }
 
 }  // namespace moeca
+
+// ---------------------------------------------------------------------------
+// Allocation-free router call (moeca_route_noalloc).
+//
+// For callers that may not allocate device memory.  The router kernel above
+// needs scratch for its per-block entropy partial sums, its last-block ticket
+// and a near-tie counter; here that scratch is one array compiled into the
+// library instead of a workspace from moeca_create.  Host code must not pass
+// g_route_scratch itself to a kernel (on the host that name is only a stand-in
+// for the device array): its device address, per device, comes from
+// cudaGetSymbolAddress on the first call made with that device current.
+// ---------------------------------------------------------------------------
+namespace moeca {
+namespace {
+
+constexpr size_t kScratchHeader = 256;      // ticket at 0, counters at 64
+constexpr size_t kScratchPartials = 32768;  // float2 (sum C, sum C ln C) per (block, expert)
+constexpr size_t kScratchBytes = kScratchHeader + kScratchPartials * sizeof(float2);
+constexpr int kScratchDevices = 64;
+
+static __device__ __align__(256) unsigned char g_route_scratch[kScratchBytes];
+
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kScratchDevices] = {};
+
+}  // namespace
+
+}  // namespace moeca
+
+extern "C" moeca_status moeca_route_noalloc(const moeca_route_args* r, void* stream) {
+  using namespace moeca;
+  if (!r || !r->x || !r->w_gate || !r->ema || !r->route_e || !r->route_w || !r->tau) return MOECA_ERR_INVALID_ARG;
+  const bool bf16 = r->dtype == MOECA_BF16;
+  if (r->dtype != MOECA_BF16 && r->dtype != MOECA_F32) return MOECA_ERR_INVALID_ARG;
+  if (r->n_tokens < 1 || r->hidden < 1 || r->hidden % (bf16 ? 8 : 4) || r->n_experts < 1 ||
+      r->n_experts > kMaxExperts || r->top_k < 1 || r->top_k > kMaxTopK || r->top_k > r->n_experts)
+    return MOECA_ERR_INVALID_ARG;
+  if (!(r->beta >= 0.f && r->beta < 1.f) || !(r->alpha >= 0.f && r->alpha < 1.f) || r->tau0 != r->tau0)
+    return MOECA_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(r->x) % 16 || reinterpret_cast<uintptr_t>(r->w_gate) % 16)
+    return MOECA_ERR_INVALID_ARG;
+  const size_t blocks = (static_cast<size_t>(r->n_tokens) + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
+  if (blocks * static_cast<size_t>(r->n_experts) > kScratchPartials) return MOECA_ERR_UNSUPPORTED;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return MOECA_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kScratchDevices) return MOECA_ERR_UNSUPPORTED;
+  void* base = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (!g_scratch_addr[dev]) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_route_scratch) != cudaSuccess || !p) {
+        cudaGetLastError();
+        return MOECA_ERR_CUDA;
+      }
+      g_scratch_addr[dev] = p;
+    }
+    base = g_scratch_addr[dev];
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // The ticket and the counters must start at zero; the partials are written
+  // by every block before the last block reads them.
+  if (cudaMemsetAsync(base, 0, kScratchHeader, s) != cudaSuccess) {
+    cudaGetLastError();
+    return MOECA_ERR_CUDA;
+  }
+  RouterArgs a{};
+  a.x = r->x;
+  a.w_gate = r->w_gate;
+  a.b_gate = r->b_gate;
+  a.T = r->n_tokens;
+  a.D = r->hidden;
+  a.E = r->n_experts;
+  a.k = r->top_k;
+  a.renorm = r->renorm_topk;
+  a.beta = r->beta;
+  a.tau0 = r->tau0;
+  a.alpha = r->alpha;
+  a.entropy_norm = r->entropy_norm;
+  a.route_e = r->route_e;
+  a.route_w = r->route_w;
+  a.ema = r->ema;
+  a.partials = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + kScratchHeader);
+  a.done = static_cast<unsigned*>(base);
+  a.tau = r->tau;
+  a.stats = reinterpret_cast<unsigned long long*>(static_cast<unsigned char*>(base) + 64);
+  if (launch_router(a, bf16, s) != cudaSuccess) {
+    cudaGetLastError();
+    return MOECA_ERR_CUDA;
+  }
+  return MOECA_OK;
+}

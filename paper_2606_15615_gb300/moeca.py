@@ -70,6 +70,14 @@ class moeca_kernel_times(C.Structure):
     _fields_ = [("total_ms", C.c_double * 6), ("launches", C.c_int64 * 6)]
 
 
+class moeca_route_args(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("n_tokens", C.c_int32), ("hidden", C.c_int32),
+                ("n_experts", C.c_int32), ("top_k", C.c_int32), ("renorm_topk", C.c_int32),
+                ("entropy_norm", C.c_int32), ("beta", C.c_float), ("tau0", C.c_float), ("alpha", C.c_float),
+                ("x", C.c_void_p), ("w_gate", C.c_void_p), ("b_gate", C.c_void_p), ("ema", C.c_void_p),
+                ("route_e", C.c_void_p), ("route_w", C.c_void_p), ("tau", C.c_void_p)]
+
+
 class MoecaError(RuntimeError):
     def __init__(self, status: int, msg: str):
         super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
@@ -99,6 +107,7 @@ def _load():
         "moeca_destroy": (C.c_int, [H]),
         "moeca_status_string": (C.c_char_p, [C.c_int]),
         "moeca_last_error": (C.c_char_p, [H]),
+        "moeca_route_noalloc": (C.c_int, [C.POINTER(moeca_route_args), C.c_void_p]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -188,6 +197,13 @@ def moeca_get_kernel_times(h, reset: bool = False) -> dict:
 def moeca_destroy(h):
     if h is not None and h.value:
         _check(LIB.moeca_destroy(h))
+
+
+def moeca_route_noalloc(args: moeca_route_args, stream: int = 0):
+    """The allocation-free router of one layer (see include/moeca.h)."""
+    st = LIB.moeca_route_noalloc(C.byref(args), stream or None)
+    if st != MOECA_OK:
+        raise MoecaError(st, "moeca_route_noalloc")
 
 
 def moeca_status_string(status: int) -> str:
