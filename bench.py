@@ -180,7 +180,7 @@ def recorded_traffic(kind: str, workload: str, reuse_target: float):
 # ---------------------------------------------------------------------------
 
 class Runner:
-    def __init__(self, wl, device_index: int, n_steps: int):
+    def __init__(self, wl, device_index: int, n_steps: int, tile_n: int = 0, split_k: int = 0):
         import numpy as np
         import torch
         from paper_2606_15615_gb300 import build
@@ -195,7 +195,8 @@ class Runner:
         cfg = M.moeca_config_default(
             n_layers=wl.n_layers, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts, top_k=wl.top_k,
             n_shared=wl.n_shared, max_tokens=wl.n_tokens,
-            dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period)
+            dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period,
+            ffn_tile_n=tile_n, ffn_split_k=split_k)
         self.cfg = cfg
         self.stack = M.Stack(cfg, self.weights, device=device_index)
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -376,6 +377,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--reps", type=int, default=5)
     ap.add_argument("--ref-tau0", type=float, default=0.8)
+    ap.add_argument("--ffn-tile-n", type=int, default=0, help="force the tensor-core FFN tile width (0: auto)")
+    ap.add_argument("--ffn-split-k", type=int, default=0, help="force the tensor-core FFN K splits (0: auto)")
     ap.add_argument("--tau0", type=float, default=None,
                     help="use this tau0 for the headline point instead of calibrating it (profiling runs)")
     args = ap.parse_args()
@@ -392,7 +395,7 @@ def main():
 
     import torch
     dist = init_group(world, "nccl")
-    runner = Runner(wl, local, args.warmup + args.steps)
+    runner = Runner(wl, local, args.warmup + args.steps, args.ffn_tile_n, args.ffn_split_k)
     dev = runner.dev
     W_, K = args.warmup, args.steps
     targets = [args.reuse] if args.no_sweep else sorted(set(wl.reuse_targets) | {args.reuse})

@@ -80,6 +80,9 @@ typedef struct {
   int32_t reused_meta_policy; /* 0: a reused slot keeps w^{t0} (default); 1: it takes w^t */
   int32_t gelu_tanh;          /* 1: tanh-form GELU (default); 0: erf form */
   int32_t ffn_impl;           /* moeca_ffn_impl */
+  int32_t ffn_tile_n;         /* tensor-core FFN tile width: 0 = chosen per launch from the group
+                                 sizes (default), else 64 / 128 / 192 / 256 where it divides N */
+  int32_t ffn_split_k;        /* tensor-core FFN K splits: 0 = chosen per launch (default), else 1..4 */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters

@@ -19,6 +19,7 @@ constexpr int kWarps = 8;
 template <typename TI, int KMAX, int CG>
 __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
+  pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * kWarps + warp;
   if (i >= a.T) return;
@@ -47,17 +48,21 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   float ss[KMAX];
 #pragma unroll
   for (int p = 0; p < KMAX; ++p) ss[p] = 0.f;
+  // Raw 16-byte vectors stay packed in registers until used.
+  const uint4* ch4 = reinterpret_cast<const uint4*>(ch);
+  const uint4* x4 = reinterpret_cast<const uint4*>(x);
+  const uint4* sh4 = reinterpret_cast<const uint4*>(sh);
   for (int c0 = 0; c0 < nvec; c0 += 32 * CG) {
-    float h[CG][KMAX][V], xs[CG][V], hs[CG][V];
+    uint4 h[CG][KMAX], xr[CG], hr[CG];
 #pragma unroll
     for (int g = 0; g < CG; ++g) {
       const int c = c0 + g * 32 + lane;
       if (c < nvec) {
 #pragma unroll
         for (int p = 0; p < KMAX; ++p)
-          if (p < k) load_vec(ch + static_cast<size_t>(q[p]) * D + c * V, h[g][p]);
-        load_vec(x + c * V, xs[g]);
-        if (sh) load_vec(sh + c * V, hs[g]);
+          if (p < k) h[g][p] = ch4[static_cast<size_t>(q[p]) * nvec + c];
+        xr[g] = x4[c];
+        if (sh) hr[g] = sh4[c];
       }
     }
 #pragma unroll
@@ -70,20 +75,26 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
 #pragma unroll
         for (int p = 0; p < KMAX; ++p) {
           if (p < k) {
+            float hv[V];
+            unpack_vec(h[g][p], hv, static_cast<TI*>(nullptr));
 #pragma unroll
             for (int j = 0; j < V; ++j) {
-              y[j] = fmaf(w[p], h[g][p][j], y[j]);
-              ss[p] = fmaf(h[g][p][j], h[g][p][j], ss[p]);
+              y[j] = fmaf(w[p], hv[j], y[j]);
+              ss[p] = fmaf(hv[j], hv[j], ss[p]);
             }
           }
         }
         if (sh) {
+          float hv[V];
+          unpack_vec(hr[g], hv, static_cast<TI*>(nullptr));
 #pragma unroll
-          for (int j = 0; j < V; ++j) y[j] += hs[g][j];
+          for (int j = 0; j < V; ++j) y[j] += hv[j];
         }
+        float xs[V];
+        unpack_vec(xr[g], xs, static_cast<TI*>(nullptr));
 #pragma unroll
-        for (int j = 0; j < V; ++j) xs[g][j] += y[j];
-        store_vec(out + c * V, xs[g]);
+        for (int j = 0; j < V; ++j) xs[j] += y[j];
+        store_vec(out + c * V, xs);
       }
     }
   }
@@ -99,9 +110,9 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
 template <typename TI>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
-  if (a.k <= 2) combine_kernel<TI, 2, 4><<<grid, kWarps * 32, 0, s>>>(a);
-  else if (a.k <= 4) combine_kernel<TI, 4, 2><<<grid, kWarps * 32, 0, s>>>(a);
-  else combine_kernel<TI, 8, 1><<<grid, kWarps * 32, 0, s>>>(a);
+  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, 4>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else launch_pdl(combine_kernel<TI, 8, 1>, dim3(grid), dim3(kWarps * 32), 0, s, a);
 }
 
 }  // namespace

@@ -18,6 +18,7 @@ constexpr int BM = 64, BN = 64, BK = 16;
 
 template <typename TI, int PHASE>
 __global__ void __launch_bounds__(256) ffn_simt_kernel(FfnArgs a) {
+  pdl_entry();
   const int N = PHASE == 1 ? a.F : a.D;
   const int K = PHASE == 1 ? a.D : a.F;
   int mt = blockIdx.y, g = -1, m0 = 0;
@@ -111,9 +112,8 @@ template <typename TI>
 cudaError_t launch_t(const FfnArgs& a, int phase, cudaStream_t s) {
   const int N = phase == 1 ? a.F : a.D;
   const dim3 grid((N + BN - 1) / BN, (a.max_rows + BM - 1) / BM + a.G);
-  if (phase == 1) ffn_simt_kernel<TI, 1><<<grid, 256, 0, s>>>(a);
-  else ffn_simt_kernel<TI, 2><<<grid, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  if (phase == 1) return launch_pdl(ffn_simt_kernel<TI, 1>, grid, dim3(256), 0, s, a);
+  return launch_pdl(ffn_simt_kernel<TI, 2>, grid, dim3(256), 0, s, a);
 }
 
 }  // namespace

@@ -8,7 +8,7 @@
 //
 // Persistent kernel, one CTA per SM, 6 warps:
 //   warp 0  TMA producer: 128 x 64 A tile and BN x 64 weight tile per stage,
-//           128-byte swizzle, into a kStages-deep shared-memory ring;
+//           128-byte swizzle, into a 192 KB shared-memory ring (4-8 stages);
 //   warp 1  allocates 512 TMEM columns and issues tcgen05.mma (M = 128,
 //           N = BN, K = 16) from one thread; tcgen05.commit frees each stage
 //           and signals a finished accumulator;
@@ -35,15 +35,16 @@ namespace {
 constexpr int kBM = 128;          // rows per tile (MMA M)
 constexpr int kBK = 64;           // K per stage: 64 bf16 = one 128-byte swizzle row
 constexpr int kMaxBN = 256;
-constexpr int kStages = 4;
+constexpr int kMaxStages = 8;
+constexpr int kRingBytes = 4 * (16384 + 256 * 128);  // 192 KB of stages, any tile width
 constexpr int kThreads = 192;
 constexpr int kTmemCols = 512;
 constexpr int kABytes = kBM * kBK * 2;        // 16 KB
 constexpr int kBBytesMax = kMaxBN * kBK * 2;  // 32 KB
-constexpr int kStageBytes = kABytes + kBBytesMax;
-constexpr int kSmemBytes = kStages * kStageBytes + 1024;
+constexpr int kSmemBytes = kRingBytes + 1024;
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr unsigned long long kWaitNs = 1000000000ull;
+constexpr int kMaxSplit = 4;
 
 struct TcArgs {
   int G, E, N, K, BN, k, T, phase, gelu_tanh;
@@ -53,39 +54,58 @@ struct TcArgs {
   void* hmid;      // phase 1 output [rows, F]
   void* cache_h;   // phase 2 routed destination [T*k, D]
   void* shared_h;  // phase 2 shared destination [T, D]
+  float* partial;  // split-K partial tiles, [max_units][128][BN] fp32
+  int* tile_sem;   // split-K arrival counters, [max_units], left at 0
+  int max_units;   // capacity of partial / tile_sem
+  int gather;      // phase 1: A rows gathered from the layer input by token (tile::gather4)
+  int bn[3];       // candidate tile widths (0 = none), matching the maps' B boxes
+  int force_bn;    // 0: choose; else use this width
+  int force_split; // 0: choose; else use this many K splits
+  float split_cost;  // cost of one split unit's partial round trip, in BN-256 k-blocks
   int* status;
 };
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
+// Weight and activation tensor maps of one phase: A (activation rows) and,
+// for each candidate width, B (routed experts) and Bs (shared expert).
+struct alignas(64) TcMaps {
+  CUtensorMap a;
+  CUtensorMap b[3];
+  CUtensorMap bs[3];
+};
 
-__device__ __forceinline__ unsigned long long globaltimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
+// Tile width and K split for this launch.  Every CTA evaluates the same cost
+// model on the same device-resident counts.  A unit is one (tile, K range).
+// Cost = waves of units over the grid x per-unit time, where per-unit time is
+// k-blocks x stage time (a stage streams 128 + BN rows of 128 bytes; its MMAs
+// take about 0.7 of a 256-wide stage's load time), plus one for pipeline fill
+// and epilogue, plus, for split units, the fp32 partial round trip.
+struct Plan {
+  int bi, S;
+};
 
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
+__device__ Plan choose_plan(const TcArgs& a, int m_tiles, int KB, int grid) {
+  Plan best{-1, 1};
+  float best_cost = 3.0e38f;
+  for (int bi = 0; bi < 3; ++bi) {
+    const int BN = a.bn[bi];
+    if (BN == 0 || (a.force_bn && BN != a.force_bn)) continue;
+    const int tiles = m_tiles * (a.N / BN);
+    const float stage = fmaxf((128.f + BN) / 384.f, 0.7f * BN / 256.f);
+    for (int S = 1; S <= 4 && S <= KB; ++S) {
+      if (a.force_split && S != a.force_split) continue;
+      if (S > 1 && tiles * S > a.max_units) break;
+      const int units = tiles * S;
+      const int waves = (units + grid - 1) / grid;
+      const float per = ((KB + S - 1) / S) * stage + 1.0f + (S > 1 ? a.split_cost * BN / 256.f : 0.f);
+      const float cost = waves * per;
+      if (cost < best_cost - 1e-3f) {
+        best_cost = cost;
+        best = Plan{bi, S};
+      }
+    }
+  }
+  if (best.bi < 0) best = Plan{0, 1};  // forced values matched nothing: widest tile, no split
+  return best;
 }
 
 // Bounded wait for phase `parity` of a barrier.  False on timeout or abort.
@@ -106,6 +126,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Four rows (one 128-byte box column each) gathered by row index; the map's
+// box is 64 x 1.  They land as 4 consecutive 128-byte rows at dst.
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, int col, int r0, int r1, int r2,
+                                            int r3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile::gather4.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(col), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar)
       : "memory");
 }
 
@@ -158,6 +189,24 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// 32 fp32 values of one row -> (GELU) -> bf16 -> 64 contiguous bytes.
+__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const uint32_t* v, bool gelu, int tanh_form) {
+  uint32_t packed[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    float x0 = __uint_as_float(v[2 * j]), x1 = __uint_as_float(v[2 * j + 1]);
+    if (gelu) {
+      x0 = gelu_f(x0, tanh_form);
+      x1 = gelu_f(x1, tanh_form);
+    }
+    __nv_bfloat162 h2 = __floats2bfloat162_rn(x0, x1);
+    packed[j] = *reinterpret_cast<uint32_t*>(&h2);
+  }
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) d4[j] = make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
+}
+
 struct TileCoord {
   int g, m_tile, n_tile;
 };
@@ -172,12 +221,11 @@ __device__ __forceinline__ TileCoord decode_tile(int tile, const int* tiles_befo
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    ffn_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                  const __grid_constant__ CUtensorMap tmBs, TcArgs a) {
+    ffn_tc_kernel(const __grid_constant__ TcMaps maps, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full_bar[kStages];
-  __shared__ __align__(8) uint64_t empty_bar[kStages];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
   __shared__ __align__(8) uint64_t tfull_bar[2];
   __shared__ __align__(8) uint64_t tempty_bar[2];
   __shared__ __align__(8) uint64_t drain_bar;
@@ -186,24 +234,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ int cnt_sh[kMaxGroups];
   __shared__ int off_sh[kMaxGroups];
   __shared__ volatile int abort_flag;
+  __shared__ int split_sh, bi_sh;
+  __shared__ int rows_sh[kBM];  // producer: token of each row of the current tile (gather)
+  __shared__ volatile int ep_abort;
+  __shared__ volatile int ep_last;
 
+  pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int G = a.G, BN = a.BN;
-  const int n_tiles = a.N / BN;
+  const int G = a.G;
   const int KB = a.K / kBK;
 
   if (threadIdx.x == 0) {
-    int acc = 0;
+    int m_tiles = 0;
     for (int g = 0; g < G; ++g) {
       const int c = a.counts[g];
       cnt_sh[g] = c;
       off_sh[g] = a.offsets[g];
+      m_tiles += (c + kBM - 1) / kBM;
+    }
+    const Plan pl = choose_plan(a, m_tiles, KB, gridDim.x);
+    bi_sh = pl.bi;
+    split_sh = pl.S;
+    const int nt = a.N / a.bn[pl.bi];
+    int acc = 0;
+    for (int g = 0; g < G; ++g) {
       tiles_before[g] = acc;
-      acc += ((c + kBM - 1) / kBM) * n_tiles;
+      acc += ((cnt_sh[g] + kBM - 1) / kBM) * nt;
     }
     tiles_before[G] = acc;
     abort_flag = 0;
-    for (int s = 0; s < kStages; ++s) {
+    ep_abort = 0;
+    for (int s = 0; s < kMaxStages; ++s) {
       mbar_init(smem_u32(&full_bar[s]), 1);
       mbar_init(smem_u32(&empty_bar[s]), 1);
     }
@@ -224,47 +285,85 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
-  const int total = tiles_before[G];
+  const int BN = a.bn[bi_sh];
+  const int n_tiles = a.N / BN;
+  // Ring depth for this width: as many stages as fit the 192 KB ring.
+  const int stage_bytes = kABytes + BN * kBK * 2;
+  const int nst = min(kMaxStages, kRingBytes / stage_bytes);
+  const CUtensorMap* tmA = &maps.a;
+  const CUtensorMap* tmB = &maps.b[bi_sh];
+  const CUtensorMap* tmBs = &maps.bs[bi_sh];
+  const int tiles = tiles_before[G];
+  const int S = split_sh;
+  const int total = tiles * S;  // units: unit u is tile u % tiles, K split u / tiles
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer ----------------
+  if (warp == 0) {
+    // ---------------- TMA producer (lane 0 issues; the warp fetches row indices) ----------------
     int stage = 0;
     uint32_t phase = 0;
     int issued = 0;
     const uint32_t bbytes = static_cast<uint32_t>(BN) * kBK * 2;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      const int tile = u % tiles, sp = u / tiles;
       const TileCoord tc = decode_tile(tile, tiles_before, cnt_sh, G, n_tiles);
-      const CUtensorMap* tb = tc.g < a.E ? &tmB : &tmBs;
+      const CUtensorMap* tb = tc.g < a.E ? tmB : tmBs;
       const int brow = (tc.g < a.E ? tc.g * a.N : 0) + tc.n_tile * BN;
       const int arow = off_sh[tc.g] + tc.m_tile * kBM;
-      for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, &abort_flag)) {
-          ok = false;
-          break;
+      const int kb0 = sp * KB / S, kb1 = (sp + 1) * KB / S;
+      if (a.gather) {
+        // Token of each of the tile's 128 rows; rows past the group's end
+        // repeat its first row (their results are never stored).
+        const int valid = cnt_sh[tc.g] - tc.m_tile * kBM;
+#pragma unroll
+        for (int j = 0; j < kBM / 32; ++j) {
+          const int r = lane * (kBM / 32) + j;
+          const int ent = a.list[arow + (r < valid ? r : 0)];
+          int tok = tc.g < a.E ? ent / a.k : ent;
+          tok = tok < 0 ? 0 : (tok >= a.T ? a.T - 1 : tok);
+          rows_sh[r] = tok;
         }
-        const uint32_t fb = smem_u32(&full_bar[stage]);
-        mbar_expect_tx(fb, kABytes + bbytes);
-        uint8_t* sa = smem + stage * kStageBytes;
-        tma_load_2d(smem_u32(sa), &tmA, kb * kBK, arow, fb);
-        tma_load_2d(smem_u32(sa + kABytes), tb, kb * kBK, brow, fb);
-        ++issued;
-        if (++stage == kStages) {
-          stage = 0;
-          phase ^= 1u;
+        __syncwarp();
+      }
+      if (lane == 0) {
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, &abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&full_bar[stage]);
+          mbar_expect_tx(fb, kABytes + bbytes);
+          uint8_t* sa = smem + stage * stage_bytes;
+          if (a.gather) {
+#pragma unroll 4
+            for (int j = 0; j < kBM / 4; ++j)
+              tma_gather4(smem_u32(sa + j * 512), tmA, kb * kBK, rows_sh[4 * j], rows_sh[4 * j + 1],
+                          rows_sh[4 * j + 2], rows_sh[4 * j + 3], fb);
+          } else {
+            tma_load_2d(smem_u32(sa), tmA, kb * kBK, arow, fb);
+          }
+          tma_load_2d(smem_u32(sa + kABytes), tb, kb * kBK, brow, fb);
+          ++issued;
+          if (++stage == nst) {
+            stage = 0;
+            phase ^= 1u;
+          }
         }
       }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();
+      if (!ok) break;
     }
-    if (!ok) {
+    if (!ok && lane == 0) {
       if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 100 + a.phase);
       abort_flag = 1;
       // Let the copies already issued land before the CTA can exit.
-      const int pending = issued < kStages ? issued : kStages;
+      const int pending = issued < nst ? issued : nst;
       int s = stage;
       uint32_t ph = phase;
       for (int j = 0; j < pending; ++j) {
         if (--s < 0) {
-          s = kStages - 1;
+          s = nst - 1;
           ph ^= 1u;
         }
         unsigned long long t0 = globaltimer();
@@ -280,27 +379,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t acc_phase = 0;
     const uint32_t idesc = instr_desc(kBM, BN);
     bool ok = true;
-    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+    for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+      const int sp = u / tiles;
+      const int kb0 = sp * KB / S, kb1 = (sp + 1) * KB / S;
       if (!mbar_wait(smem_u32(&tempty_bar[acc]), acc_phase ^ 1u, &abort_flag)) {
         ok = false;
         break;
       }
       tc_fence_after();
       const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * BN);
-      for (int kb = 0; kb < KB; ++kb) {
+      for (int kb = kb0; kb < kb1; ++kb) {
         if (!mbar_wait(smem_u32(&full_bar[stage]), phase, &abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + stage * kStageBytes);
+        const uint32_t sa = smem_u32(smem + stage * stage_bytes);
         const uint32_t sb = sa + kABytes;
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk) {
-          mma_bf16(d_tmem, smem_desc(sa + kk * 32), smem_desc(sb + kk * 32), idesc, (kb | kk) != 0);
+          mma_bf16(d_tmem, smem_desc(sa + kk * 32), smem_desc(sb + kk * 32), idesc, (kb != kb0) || kk != 0);
         }
         mma_commit(smem_u32(&empty_bar[stage]));
-        if (++stage == kStages) {
+        if (++stage == nst) {
           stage = 0;
           phase ^= 1u;
         }
@@ -323,16 +424,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 2) {
     // ---------------- Epilogue ----------------
+    // The 4 epilogue warps (128 threads) agree on every abort and every
+    // split-K decision through named barrier 1, so none can wait alone.
     const int quad = warp & 3;  // TMEM lanes [32 quad, 32 quad + 32)
     const int r = quad * 32 + lane;
+    const bool leader = warp == 2 && lane == 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      const int tile = u % tiles, sp = u / tiles;
       const TileCoord tc = decode_tile(tile, tiles_before, cnt_sh, G, n_tiles);
-      // Warp-uniform outcome: tcgen05.ld below needs the whole warp converged.
       const bool got = __all_sync(0xffffffffu, mbar_wait(smem_u32(&tfull_bar[acc]), acc_phase, &abort_flag));
-      if (!got) {
-        if (lane == 0 && !abort_flag) report_status(a.status, kStatusWaitTimeout, 300 + a.phase);
+      if (!got && lane == 0) ep_abort = 1;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (ep_abort) {
+        if (leader && !abort_flag) report_status(a.status, kStatusWaitTimeout, 300 + a.phase);
         abort_flag = 1;
         break;
       }
@@ -356,29 +462,74 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(acc * BN);
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tbase + c * 32, v);
-        if (dst) {
-          uint32_t packed[16];
+      if (S == 1) {
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tbase + c * 32, v);
+          if (dst) store_row32(dst + c * 32, v, a.phase == 1, a.gelu_tanh);
+        }
+        tc_fence_before();
+        mbar_arrive(smem_u32(&tempty_bar[acc]));
+      } else {
+        // Split K: park this split's fp32 rows, free TMEM, then the last
+        // split to arrive for the tile sums the splits in split order.
+        float* mine = a.partial + (static_cast<size_t>(tile) * S + sp) * kBM * BN + static_cast<size_t>(r) * BN;
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tbase + c * 32, v);
+          float4* d4 = reinterpret_cast<float4*>(mine + c * 32);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            float x0 = __uint_as_float(v[2 * j]), x1 = __uint_as_float(v[2 * j + 1]);
-            if (a.phase == 1) {
-              x0 = gelu_f(x0, a.gelu_tanh);
-              x1 = gelu_f(x1, a.gelu_tanh);
+          for (int j = 0; j < 8; ++j)
+            d4[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+        }
+        tc_fence_before();
+        mbar_arrive(smem_u32(&tempty_bar[acc]));
+        __threadfence();
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (leader) ep_last = atomicAdd(a.tile_sem + tile, 1) == S - 1;
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (ep_last) {
+          __threadfence();
+          const float* base = a.partial + static_cast<size_t>(tile) * S * kBM * BN + static_cast<size_t>(r) * BN;
+          for (int c = 0; c < BN / 32; ++c) {
+            uint32_t v[32];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              // All splits' 16 values in flight at once, then added in split order.
+              float4 f[kMaxSplit][4];
+#pragma unroll
+              for (int q = 0; q < kMaxSplit; ++q) {
+                if (q < S) {
+                  const float4* s4 = reinterpret_cast<const float4*>(
+                      base + static_cast<size_t>(q) * kBM * BN + c * 32 + h * 16);
+#pragma unroll
+                  for (int j = 0; j < 4; ++j) f[q][j] = __ldcg(s4 + j);
+                }
+              }
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                float4 acc4 = f[0][j];
+#pragma unroll
+                for (int q = 1; q < kMaxSplit; ++q) {
+                  if (q < S) {
+                    acc4.x += f[q][j].x;
+                    acc4.y += f[q][j].y;
+                    acc4.z += f[q][j].z;
+                    acc4.w += f[q][j].w;
+                  }
+                }
+                v[h * 16 + 4 * j] = __float_as_uint(acc4.x);
+                v[h * 16 + 4 * j + 1] = __float_as_uint(acc4.y);
+                v[h * 16 + 4 * j + 2] = __float_as_uint(acc4.z);
+                v[h * 16 + 4 * j + 3] = __float_as_uint(acc4.w);
+              }
             }
-            __nv_bfloat162 h2 = __floats2bfloat162_rn(x0, x1);
-            packed[j] = *reinterpret_cast<uint32_t*>(&h2);
+            if (dst) store_row32(dst + c * 32, v, a.phase == 1, a.gelu_tanh);
           }
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            d4[j] = make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
+          if (leader) a.tile_sem[tile] = 0;
         }
       }
-      tc_fence_before();
-      mbar_arrive(smem_u32(&tempty_bar[acc]));
       if (++acc == 2) {
         acc = 0;
         acc_phase ^= 1u;
@@ -423,39 +574,71 @@ bool encode_2d(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, u
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int pick_bn(int n) {
-  const int cands[] = {256, 192, 128, 64};
-  for (int c : cands)
-    if (n % c == 0) return c;
-  return 0;
+}  // namespace
+
+struct TcPlan {
+  TcMaps p1, p2;         // phase 1 (N = F, K = D) and phase 2 (N = D, K = F)
+  TcMaps p1g;            // phase 1 with A gathered from the layer input (box 64 x 1)
+  const void* g_src = nullptr;  // layer input the gather map was encoded for
+  int g_rows = 0;
+  int bn1[3], bn2[3];
+  int n_sms;
+  int force_bn, force_split;
+  float split_cost;
+};
+
+size_t tc_split_units(int n_sms) { return static_cast<size_t>(4) * n_sms; }
+size_t tc_partial_bytes(int n_sms) { return tc_split_units(n_sms) * kBM * kMaxBN * sizeof(float); }
+
+namespace {
+
+// Candidate widths for N: the widest of {256, 192} dividing N, then 128, 64.
+void candidates(int n, int* bn) {
+  bn[0] = n % 256 == 0 ? 256 : (n % 192 == 0 ? 192 : 0);
+  bn[1] = n % 128 == 0 ? 128 : 0;
+  bn[2] = n % 64 == 0 ? 64 : 0;
+  if (!bn[0]) {  // keep slot 0 filled with the widest available width
+    bn[0] = bn[1] ? bn[1] : bn[2];
+    if (bn[0] == bn[1]) bn[1] = 0;
+    else bn[2] = 0;
+  }
+}
+
+bool encode_phase(TcMaps* m, const int* bn, const void* a_base, uint64_t rows, uint64_t K, const void* w,
+                  uint64_t w_rows, const void* ws, uint64_t ws_rows) {
+  if (!encode_2d(&m->a, a_base, rows, K, kBM)) return false;
+  for (int i = 0; i < 3; ++i) {
+    if (!bn[i]) {
+      m->b[i] = m->b[0];
+      m->bs[i] = m->bs[0];
+      continue;
+    }
+    if (!encode_2d(&m->b[i], w, w_rows, K, bn[i])) return false;
+    if (ws) {
+      if (!encode_2d(&m->bs[i], ws, ws_rows, K, bn[i])) return false;
+    } else {
+      m->bs[i] = m->b[i];  // never read: there is no shared group
+    }
+  }
+  return true;
 }
 
 }  // namespace
 
-struct TcPlan {
-  CUtensorMap a1, b1, bs1, a2, b2, bs2;
-  int bn1, bn2;
-  int n_sms;
-};
-
 TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen) {
   TcPlan* p = new TcPlan();
   p->n_sms = n_sms;
-  p->bn1 = pick_bn(a.F);
-  p->bn2 = pick_bn(a.D);
+  p->force_bn = a.tile_n;
+  p->force_split = a.split_k;
+  p->split_cost = 40.0f;  // measured: split units rarely pay for their partial round trip
+  candidates(a.F, p->bn1);
+  candidates(a.D, p->bn2);
   const char* what = nullptr;
-  if (!p->bn1 || !p->bn2 || a.D % kBK || a.F % kBK) what = "hidden and ffn must be multiples of 64";
+  if (!p->bn1[0] || !p->bn2[0] || a.D % kBK || a.F % kBK) what = "hidden and ffn must be multiples of 64";
   else if (!get_encoder()) what = "cuTensorMapEncodeTiled is unavailable";
-  else if (!encode_2d(&p->a1, a.xg, a.max_rows, a.D, kBM) || !encode_2d(&p->a2, a.hmid, a.max_rows, a.F, kBM) ||
-           !encode_2d(&p->b1, a.w1, static_cast<uint64_t>(a.E) * a.F, a.D, p->bn1) ||
-           !encode_2d(&p->b2, a.w2, static_cast<uint64_t>(a.E) * a.D, a.F, p->bn2))
+  else if (!encode_phase(&p->p1, p->bn1, a.xg, a.max_rows, a.D, a.w1, static_cast<uint64_t>(a.E) * a.F, a.ws1, a.F) ||
+           !encode_phase(&p->p2, p->bn2, a.hmid, a.max_rows, a.F, a.w2, static_cast<uint64_t>(a.E) * a.D, a.ws2, a.D))
     what = "tensor map encoding failed";
-  else if (a.ws1 && (!encode_2d(&p->bs1, a.ws1, a.F, a.D, p->bn1) || !encode_2d(&p->bs2, a.ws2, a.D, a.F, p->bn2)))
-    what = "shared-expert tensor map encoding failed";
-  if (!a.ws1) {
-    p->bs1 = p->b1;  // never read: there is no shared group
-    p->bs2 = p->b2;
-  }
   if (!what && cudaFuncSetAttribute(ffn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
                    cudaSuccess) {
     cudaGetLastError();
@@ -477,7 +660,6 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
   t.E = a.E;
   t.N = phase == 1 ? a.F : a.D;
   t.K = phase == 1 ? a.D : a.F;
-  t.BN = phase == 1 ? p->bn1 : p->bn2;
   t.k = a.k;
   t.T = a.T;
   t.phase = phase;
@@ -488,13 +670,29 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
   t.hmid = a.hmid;
   t.cache_h = a.cache_h;
   t.shared_h = a.shared_h;
+  t.partial = a.partial;
+  t.tile_sem = a.tile_sem;
+  t.max_units = a.partial ? static_cast<int>(tc_split_units(p->n_sms)) : 0;
+  const int* bn = phase == 1 ? p->bn1 : p->bn2;
+  for (int i = 0; i < 3; ++i) t.bn[i] = bn[i];
+  t.force_bn = p->force_bn;
+  t.force_split = p->force_split;
+  t.split_cost = p->split_cost;
   t.status = a.status;
-  const long long max_tiles =
-      (static_cast<long long>(a.max_rows + kBM - 1) / kBM + a.G) * static_cast<long long>(t.N / t.BN);
-  const int grid = static_cast<int>(max_tiles < p->n_sms ? max_tiles : p->n_sms);
-  if (phase == 1) ffn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p->a1, p->b1, p->bs1, t);
-  else ffn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p->a2, p->b2, p->bs2, t);
-  return cudaGetLastError();
+  const TcMaps* maps = phase == 1 ? &p->p1 : &p->p2;
+  if (phase == 1 && a.x) {
+    // Phase 1 reads its rows straight from the layer input; re-encode the
+    // gather map when that buffer or its row count changes.
+    if (a.x != p->g_src || a.T != p->g_rows) {
+      p->p1g = p->p1;
+      if (!encode_2d(&p->p1g.a, a.x, a.T, a.D, 1)) return cudaErrorInvalidValue;
+      p->g_src = a.x;
+      p->g_rows = a.T;
+    }
+    maps = &p->p1g;
+    t.gather = 1;
+  }
+  return launch_pdl(ffn_tc_kernel, dim3(p->n_sms), dim3(kThreads), kSmemBytes, s, *maps, t);
 }
 
 }  // namespace moeca

@@ -38,6 +38,7 @@ struct RouterArgs {
   unsigned* done;       // last-block ticket, left at 0
   float* tau;           // [E]
   unsigned long long* stats;
+  int* status;          // device status word (or null)
 };
 cudaError_t launch_router(const RouterArgs& a, bool bf16, cudaStream_t s);
 
@@ -80,7 +81,7 @@ struct CompactArgs {
   const int32_t* offsets;
   int32_t* list;        // [rows]
   const void* x;        // [T, D]
-  void* xg;             // [rows, D] gathered inputs
+  void* xg;             // [rows, D] gathered inputs, or null when the GEMM gathers itself
 };
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s);
 
@@ -91,7 +92,8 @@ struct FfnArgs {
   const int32_t* counts;
   const int32_t* offsets;
   const int32_t* list;
-  const void* xg;        // [rows, D]
+  const void* xg;        // [rows, D]   gathered inputs (SIMT path)
+  const void* x;         // [T, D]      layer input: the tensor-core path gathers rows from it
   void* hmid;            // [rows, F]
   const void* w1;        // [E, F, D]
   const void* w2;        // [E, D, F]
@@ -100,6 +102,10 @@ struct FfnArgs {
   void* cache_h;         // [T*k, D]   destination rows of routed groups
   void* shared_h;        // [T, D]     destination rows of the shared group
   int gelu_tanh;
+  int tile_n;            // tensor-core tile width to force (0: chosen per launch)
+  int split_k;           // tensor-core K splits to force (0: chosen per launch)
+  float* partial;        // split-K workspace of the tensor-core path (or null: no split)
+  int* tile_sem;         // split-K arrival counters, zeroed once
   int* status;
 };
 cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s);
@@ -108,6 +114,8 @@ cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t
 // handle; `TcPlan` owns them.
 struct TcPlan;
 TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen);
+size_t tc_split_units(int n_sms);      // split-K units the workspace holds
+size_t tc_partial_bytes(int n_sms);    // bytes of the split-K partial workspace
 void tc_plan_destroy(TcPlan* p);
 cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s);
 

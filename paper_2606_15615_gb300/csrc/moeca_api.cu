@@ -24,6 +24,13 @@ namespace {
 
 thread_local std::string g_create_error;
 
+// Phase 1 of the tensor-core FFN can gather its A rows from the layer input
+// with TMA tile::gather4 instead of reading rows that compact_kernel copied
+// into a contiguous buffer.  Measured on GB300 the gather issue rate (32
+// gather4 per 64-wide k-block from one thread) costs more than the copy, so
+// the copy path is the default.
+constexpr bool kGemmGathersRows = false;
+
 struct LayerBuf {
   moeca_layer_weights w;
   int32_t* cache_e = nullptr;
@@ -69,6 +76,8 @@ struct moeca_handle {
   int32_t* block_offsets = nullptr;
   void* xg = nullptr;
   void* hmid = nullptr;
+  float* tc_partial = nullptr;
+  int* tc_sem = nullptr;
   std::vector<void*> act;  // input of layer l (l >= 1)
   int* status_host = nullptr;
   int* status_dev = nullptr;
@@ -227,6 +236,9 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (c.refresh_period < 0) return fail(nullptr, MOECA_ERR_INVALID_ARG, "refresh_period < 0");
   if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
+  if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&
+       c.ffn_tile_n != 256) || c.ffn_split_k < 0 || c.ffn_split_k > 4)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_tile_n must be 0/64/128/192/256, ffn_split_k 0..4");
   const int vec = bf16 ? 8 : 4;
   if (c.hidden % vec) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "hidden must be a multiple of 8 (bf16) / 4 (fp32)");
   const bool use_tc = bf16 && c.ffn_impl == MOECA_FFN_AUTO;
@@ -292,6 +304,10 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   A((void**)&h->block_offsets, nblk_sel * G * 4);
   A(&h->xg, static_cast<size_t>(h->max_rows) * D * es);
   A(&h->hmid, static_cast<size_t>(h->max_rows) * F * es);
+  if (use_tc) {
+    A((void**)&h->tc_partial, tc_partial_bytes(h->n_sms));
+    A((void**)&h->tc_sem, tc_split_units(h->n_sms) * sizeof(int));
+  }
   h->act.assign(c.n_layers, nullptr);
   for (int l = 1; l < c.n_layers && ok; ++l) A(&h->act[l], T * D * es);
   if (!ok) {
@@ -315,6 +331,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
       fa.max_rows = h->max_rows;
       fa.xg = h->xg; fa.hmid = h->hmid;
       fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
+      fa.tile_n = c.ffn_tile_n; fa.split_k = c.ffn_split_k;
       char err[256] = {0};
       L.tc = tc_plan_create(fa, h->n_sms, err, sizeof err);
       if (!L.tc) {
@@ -377,6 +394,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ra.entropy_norm = c.entropy_norm;
     ra.route_e = L.route_e; ra.route_w = L.route_w; ra.ema = L.ema;
     ra.partials = h->partials; ra.done = h->done; ra.tau = L.tau; ra.stats = L.stats;
+    ra.status = h->status_dev;
     if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
 
     SelectArgs sa{};
@@ -396,16 +414,17 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ca.refresh = refresh; ca.shared_policy = c.shared_policy;
     ca.route_e = L.route_e; ca.recompute = L.recompute; ca.slot = L.slot; ca.token_any = L.token_any;
     ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
-    ca.x = in; ca.xg = h->xg;
+    ca.x = in; ca.xg = (use_tc && kGemmGathersRows) ? nullptr : h->xg;
     if ((e = timed(h, MOECA_K_COMPACT, s, [&] { return launch_compact(ca, h->bf16, s); })) != cudaSuccess) break;
 
     FfnArgs fa{};
     fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;
     fa.max_rows = T * (c.top_k + c.n_shared);
     fa.counts = L.counts; fa.offsets = L.offsets; fa.list = L.list;
-    fa.xg = h->xg; fa.hmid = h->hmid;
+    fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? in : nullptr;
     fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
     fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
+    fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
     for (int phase = 1; phase <= 2 && e == cudaSuccess; ++phase) {
       const int kind = phase == 1 ? MOECA_K_FFN1 : MOECA_K_FFN2;
       e = timed(h, kind, s, [&] {

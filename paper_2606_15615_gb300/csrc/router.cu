@@ -1,7 +1,7 @@
 // Router of the branch-cached MoE layer.
 //
-// Per token i (one warp): gate logits z = x_i W_g^T (+ b) with fp32
-// accumulation, softmax over the E experts, top-k by descending logit with
+// Per token i (a group of up to 8 lanes): gate logits z = x_i W_g^T (+ b)
+// with fp32 accumulation, softmax over the E experts, top-k by descending logit with
 // ties to the lower expert id, optional renormalisation of the k weights
 // (Eq. 7).  The same pass updates the EMA statistic
 //   C_{e,i} <- beta C_{e,i} + (1 - beta) 1[e in B_i]        (Eq. 10)
@@ -18,150 +18,224 @@
 namespace moeca {
 namespace {
 
-constexpr int kWarps = 8;
-constexpr int kTokensPerWarp = kRouterTokensPerBlock / kWarps;
 
-template <typename TI, int EMAX>
-__global__ void __launch_bounds__(kWarps * 32) router_kernel(RouterArgs a) {
+// Bit-exact group reductions over the G lanes of one token (G divides 32).
+template <int G>
+__device__ __forceinline__ float group_max(float v) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+template <int G>
+__device__ __forceinline__ float group_sum(float v) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// One token per group of G lanes (G = min(E, 8) rounded down to a power of
+// two); lane g of a group owns experts e = g + G j, j < EPL.  One thread
+// stages the block's token rows and the gate matrix into shared memory with
+// bulk async copies completing on one mbarrier (rows padded by 16 bytes, so
+// the tokens of a warp and the G experts of a group hit different banks);
+// shapes too large for shared memory read the same data through L1 / L2.
+// Each lane accumulates its logits over D in fp32; softmax and top-k run as
+// shuffles inside the group.
+template <typename TI, int G, int EPL, int NT>
+__global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, int stage_wg) {
   constexpr int V = Elem<TI>::kVec;
-  constexpr int EPL = (EMAX + 31) / 32;  // EMA experts per lane
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const TI* __restrict__ x = static_cast<const TI*>(a.x);
-  const TI* __restrict__ wg = static_cast<const TI*>(a.w_gate);
-  const int E = a.E, k = a.k, nvec = a.D / V;
-
-  __shared__ float sm_S[kWarps][EMAX];
-  __shared__ float sm_U[kWarps][EMAX];
-  __shared__ int sm_near[kWarps];
-
-  float accS[EPL], accU[EPL];
+  constexpr int TB = NT / G;                  // tokens per block
+  constexpr int EMAXB = G * EPL;              // experts covered by a group
+  constexpr int kThreads = NT;
+  extern __shared__ uint4 sm_dyn[];           // [E][rowv + 1] gate rows, then [TB][rowv + 1] token rows
+  __shared__ float sm_S[TB * EMAXB];
+  __shared__ float sm_U[TB * EMAXB];
+  __shared__ int sm_near;
+  __shared__ __align__(8) uint64_t sm_bar;
+  const int t = threadIdx.x;
+  const int g = t % G, tok = t / G;
+  const int E = a.E, k = a.k;
+  const int rowv = a.D / V, pstride = rowv + 1;
+  const int i = blockIdx.x * TB + tok;
+  const bool valid = i < a.T;
+  const int ntok = min(TB, a.T - static_cast<int>(blockIdx.x) * TB);
+  pdl_entry();
+  const uint4* wsrc = static_cast<const uint4*>(a.w_gate);
+  int wstride = rowv;
+  const uint4* xsrc = static_cast<const uint4*>(a.x) + static_cast<size_t>(i) * rowv;
+  uint4* sm_wg = sm_dyn;
+  uint4* sm_x = sm_dyn + (stage_wg ? E * pstride : 0);
+  if (t == 0) {
+    sm_near = 0;
+    if (stage_wg || stage_x) {
+      mbar_init(smem_u32(&sm_bar), 1);
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+  }
+  __syncthreads();
+  if (stage_wg || stage_x) {
+    const uint32_t bar = smem_u32(&sm_bar);
+    const uint32_t row_bytes = static_cast<uint32_t>(rowv) * 16;
+    if (t == 0) {
+      mbar_expect_tx(bar, row_bytes * ((stage_wg ? E : 0) + (stage_x ? ntok : 0)));
+      if (stage_wg)
+        for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(sm_wg + e * pstride), wsrc + e * rowv, row_bytes, bar);
+      if (stage_x)
+        for (int q = 0; q < ntok; ++q)
+          bulk_g2s(smem_u32(sm_x + q * pstride),
+                   static_cast<const uint4*>(a.x) + static_cast<size_t>(blockIdx.x * TB + q) * rowv, row_bytes, bar);
+    }
+    if (!mbar_wait_for(bar, 0, 1000000000ull) && t == 0) report_status(a.status, kStatusWaitTimeout, 500);
+    if (stage_wg) {
+      wsrc = sm_wg;
+      wstride = pstride;
+    }
+    if (stage_x) xsrc = sm_x + tok * pstride;
+  }
+  float z[EPL];
 #pragma unroll
-  for (int j = 0; j < EPL; ++j) accS[j] = accU[j] = 0.f;
-  int near_count = 0;
-
-  for (int tt = 0; tt < kTokensPerWarp; ++tt) {
-    const int i = blockIdx.x * kRouterTokensPerBlock + warp * kTokensPerWarp + tt;
-    if (i >= a.T) break;  // warp-uniform
-    float z[EMAX];
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e) z[e] = 0.f;
-    const TI* xr = x + static_cast<size_t>(i) * a.D;
-    for (int c = lane; c < nvec; c += 32) {
+  for (int j = 0; j < EPL; ++j) z[j] = 0.f;
+  if (valid) {
+#pragma unroll 2
+    for (int c = 0; c < rowv; ++c) {
       float xv[V];
-      load_vec(xr + c * V, xv);
+      unpack_vec(xsrc[c], xv, static_cast<TI*>(nullptr));
 #pragma unroll
-      for (int e = 0; e < EMAX; ++e) {
+      for (int j = 0; j < EPL; ++j) {
+        const int e = g + G * j;
         if (e < E) {
           float wv[V];
-          load_vec(wg + static_cast<size_t>(e) * a.D + c * V, wv);
+          unpack_vec(wsrc[e * wstride + c], wv, static_cast<TI*>(nullptr));
 #pragma unroll
-          for (int j = 0; j < V; ++j) z[e] = fmaf(xv[j], wv[j], z[e]);
+          for (int q = 0; q < V; ++q) z[j] = fmaf(xv[q], wv[q], z[j]);
         }
       }
     }
+  }
+// Logits of experts this lane does not own (e >= E) are -inf.
+  float zl[EPL];
+  float lmax = -INFINITY, labs = 0.f;
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e) {
-      if (e < E) {
-        z[e] = warp_sum(z[e]);
-        if (a.b_gate) z[e] += a.b_gate[e];
-      }
+  for (int j = 0; j < EPL; ++j) {
+    const int e = g + G * j;
+    if (e < E) {
+      zl[j] = z[j] + (a.b_gate ? a.b_gate[e] : 0.f);
+      lmax = fmaxf(lmax, zl[j]);
+      labs = fmaxf(labs, fabsf(zl[j]));
+    } else {
+      zl[j] = -INFINITY;
     }
-    // Top-(k+1) by repeated argmax (every lane holds every logit).
-    unsigned long long taken = 0ull, topk_mask = 0ull;
-    int sel[kMaxTopK];
-    float selz[kMaxTopK + 1];
-    const int ranks = (k + 1 < E) ? k + 1 : E;
-    float zabs = 0.f;
+  }
+  const float m = group_max<G>(lmax);
+  const float zabs = group_max<G>(labs);
+  float lsum = 0.f;
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) zabs = fmaxf(zabs, fabsf(z[e]));
+  for (int j = 0; j < EPL; ++j)
+    if (g + G * j < E) lsum += expf(zl[j] - m);
+  const float denom = group_sum<G>(lsum);
+  // Top-(k+1): repeated group argmax, ties to the lower expert id.
+  const int ranks = (k + 1 < E) ? k + 1 : E;
+  unsigned taken = 0u;
+  unsigned long long topk_mask = 0ull;
+  int sel_e[kMaxTopK + 1];
+  float sel_z[kMaxTopK + 1];
 #pragma unroll
-    for (int p = 0; p < kMaxTopK + 1; ++p) {
-      if (p < ranks) {
-        int be = -1;
-        float best = 0.f;
+  for (int r = 0; r < kMaxTopK + 1; ++r) {
+    sel_e[r] = 0;
+    sel_z[r] = 0.f;
+    if (r < ranks) {
+      float bv = -INFINITY;
+      int be = 0x7fffffff;
 #pragma unroll
-        for (int e = 0; e < EMAX; ++e) {
-          if (e < E && !((taken >> e) & 1ull) && (be < 0 || z[e] > best)) {
-            best = z[e];
-            be = e;
-          }
-        }
-        taken |= 1ull << be;
-        selz[p] = best;
-        if (p < k) {
-          sel[p] = be;
-          topk_mask |= 1ull << be;
+      for (int j = 0; j < EPL; ++j) {
+        const int e = g + G * j;
+        if (e < E && !((taken >> j) & 1u) && (zl[j] > bv || (zl[j] == bv && e < be))) {
+          bv = zl[j];
+          be = e;
         }
       }
-    }
-    // Softmax over all E from the top logit, then the k weights.
-    const float m = selz[0];
-    float denom = 0.f;
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) denom += expf(z[e] - m);
-    float w[kMaxTopK];
-    float wsum = 0.f;
+      for (int o = G / 2; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oe = __shfl_xor_sync(0xffffffffu, be, o);
+        if (ov > bv || (ov == bv && oe < be)) {
+          bv = ov;
+          be = oe;
+        }
+      }
+      if (be < E && be % G == g) taken |= 1u << (be / G);
+      sel_e[r] = be;
+      sel_z[r] = bv;
+      if (r < k && be < E) topk_mask |= 1ull << be;
+    }
+  }
+  if (valid) {
+    float wsum = 0.f, w[kMaxTopK];
 #pragma unroll
     for (int p = 0; p < kMaxTopK; ++p) {
+      w[p] = 0.f;
       if (p < k) {
-        w[p] = expf(selz[p] - m) / denom;
+        w[p] = expf(sel_z[p] - m) / denom;
         wsum += w[p];
       }
     }
     bool near = false;
 #pragma unroll
     for (int p = 0; p < kMaxTopK; ++p)
-      if (p + 1 < ranks && (selz[p] - selz[p + 1]) < 1e-5f * zabs) near = true;
-    if (lane == 0 && near) ++near_count;
+      if (p + 1 < ranks && (sel_z[p] - sel_z[p + 1]) < 1e-5f * zabs) near = true;
+    if (g == 0 && near) atomicAdd(&sm_near, 1);
 #pragma unroll
     for (int p = 0; p < kMaxTopK; ++p) {
-      if (p < k && lane == p) {
-        a.route_e[static_cast<size_t>(i) * k + p] = sel[p];
+      if (p < k && p % G == g) {
+        a.route_e[static_cast<size_t>(i) * k + p] = sel_e[p];
         a.route_w[static_cast<size_t>(i) * k + p] = a.renorm ? w[p] / wsum : w[p];
       }
     }
-    // EMA statistic and entropy partial sums.
-#pragma unroll
-    for (int j = 0; j < EPL; ++j) {
-      const int e = lane + 32 * j;
-      if (e < E) {
-        float* cp = a.ema + static_cast<size_t>(i) * E + e;
-        const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
-        const float c = a.beta * (*cp) + (1.f - a.beta) * ind;
-        *cp = c;
-        accS[j] += c;
-        if (c > 0.f) accU[j] += c * logf(c);
-      }
-    }
   }
+  // EMA statistic (Eq. 10) and this token's entropy terms.
 #pragma unroll
   for (int j = 0; j < EPL; ++j) {
-    const int e = lane + 32 * j;
-    if (e < EMAX) {
-      sm_S[warp][e] = accS[j];
-      sm_U[warp][e] = accU[j];
+    const int e = g + G * j;
+    if (e < EMAXB) {
+      float c = 0.f, u = 0.f;
+      if (valid && e < E) {
+        float* cp = a.ema + static_cast<size_t>(i) * E + e;
+        const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
+        c = a.beta * (*cp) + (1.f - a.beta) * ind;
+        *cp = c;
+        if (c > 0.f) u = c * logf(c);
+      }
+      sm_S[tok * EMAXB + e] = c;
+      sm_U[tok * EMAXB + e] = u;
     }
   }
-  if (lane == 0) sm_near[warp] = near_count;
   __syncthreads();
-  const int t = threadIdx.x;
-  if (t < E) {
+  // Block partials per expert, summed over the block's tokens in token order
+  // split into J interleaved runs that are added in run order.
+  __shared__ float sm_rs[kThreads][2];
+  {
+    const int J = kThreads / E;
+    const int e = t % E, jr = t / E;
     float S = 0.f, U = 0.f;
-#pragma unroll
-    for (int w8 = 0; w8 < kWarps; ++w8) {
-      S += sm_S[w8][t];
-      U += sm_U[w8][t];
+    if (jr < J)
+      for (int q = jr; q < TB; q += J) {
+        S += sm_S[q * EMAXB + e];
+        U += sm_U[q * EMAXB + e];
+      }
+    sm_rs[t][0] = S;
+    sm_rs[t][1] = U;
+    __syncthreads();
+    if (t < E) {
+      float Ss = 0.f, Us = 0.f;
+      for (int q = 0; q < J; ++q) {
+        Ss += sm_rs[q * E + t][0];
+        Us += sm_rs[q * E + t][1];
+      }
+      a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 0] = Ss;
+      a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 1] = Us;
     }
-    a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 0] = S;
-    a.partials[(static_cast<size_t>(blockIdx.x) * E + t) * 2 + 1] = U;
   }
-  if (t == 0) {
-    int n = 0;
-    for (int w8 = 0; w8 < kWarps; ++w8) n += sm_near[w8];
-    if (n) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(n));
-  }
+  if (t == 0 && sm_near) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(sm_near));
   // The last block to arrive reduces all partials in block order.
   __threadfence();
   __syncthreads();
@@ -170,41 +244,42 @@ __global__ void __launch_bounds__(kWarps * 32) router_kernel(RouterArgs a) {
   __syncthreads();
   if (ticket != gridDim.x - 1) return;
   __threadfence();
-  // Thread t sums blocks j, j + J, j + 2J, ... of expert e = t % E (J = 256 / E
-  // lanes per expert, loads independent); the J sums are then added in j order.
-  __shared__ double sm_H[EMAX];
-  __shared__ int sm_live[EMAX];
-  __shared__ double sm_lo, sm_hi;
-  __shared__ double sm_red[kWarps * 32][2];
+  // Thread t sums blocks j, j + J, j + 2J, ... of expert e = t % E (J runs per
+  // expert, loads independent); the J sums are then added in j order.  fp32
+  // throughout: FP64 is slow on this part and the sums need no more.
+  __shared__ float sm_H[kMaxExperts];
+  __shared__ int sm_live[kMaxExperts];
+  __shared__ float sm_lo, sm_hi;
+  __shared__ float sm_red[kThreads][2];
   {
-    const int J = (kWarps * 32) / E;
+    const int J = kThreads / E;
     const int e = t % E, j = t / E;
-    double S = 0.0, U = 0.0;
+    float S = 0.f, U = 0.f;
     if (j < J) {
       const float2* part = reinterpret_cast<const float2*>(a.partials);
 #pragma unroll 4
       for (unsigned b = j; b < gridDim.x; b += J) {
         const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
-        S += static_cast<double>(v.x);
-        U += static_cast<double>(v.y);
+        S += v.x;
+        U += v.y;
       }
     }
     sm_red[t][0] = S;
     sm_red[t][1] = U;
     __syncthreads();
     if (t < E) {
-      double Ss = 0.0, Us = 0.0;
+      float Ss = 0.f, Us = 0.f;
       for (int jj = 0; jj < J; ++jj) {
         Ss += sm_red[jj * E + t][0];
         Us += sm_red[jj * E + t][1];
       }
-      sm_live[t] = Ss > 0.0;
-      sm_H[t] = Ss > 0.0 ? log(Ss) - Us / Ss : 0.0;
+      sm_live[t] = Ss > 0.f;
+      sm_H[t] = Ss > 0.f ? logf(Ss) - Us / Ss : 0.f;
     }
   }
   __syncthreads();
   if (t == 0) {
-    double lo = 0.0, hi = 0.0;
+    float lo = 0.f, hi = 0.f;
     bool any = false;
     for (int e = 0; e < E; ++e) {
       if (!sm_live[e]) continue;
@@ -218,27 +293,57 @@ __global__ void __launch_bounds__(kWarps * 32) router_kernel(RouterArgs a) {
   }
   __syncthreads();
   if (t < E) {
-    double hb = 0.5;
+    float hb = 0.5f;
     if (sm_live[t]) {
       if (a.entropy_norm == 0) {
-        if (a.T > 1) hb = fmin(1.0, fmax(0.0, sm_H[t] / log(static_cast<double>(a.T))));
+        if (a.T > 1) hb = fminf(1.f, fmaxf(0.f, sm_H[t] / logf(static_cast<float>(a.T))));
       } else if (sm_hi > sm_lo) {
         hb = (sm_H[t] - sm_lo) / (sm_hi - sm_lo);
       }
     }
-    a.tau[t] = a.tau0 * (1.0f + a.alpha * (2.0f * static_cast<float>(hb) - 1.0f));
+    a.tau[t] = a.tau0 * (1.0f + a.alpha * (2.0f * hb - 1.0f));
   }
+}
+
+// The padded gate matrix, and the block's token rows when they also fit, go
+// to shared memory; otherwise lanes read them through L1 / L2.  The staging
+// cap is what the 227 KB per-block limit leaves beside the kernel's static
+// shared memory.
+constexpr size_t kSmemPerBlock = 227 * 1024;
+
+template <typename TI, int G, int EPL, int NT>
+cudaError_t launch_g(const RouterArgs& a, cudaStream_t s) {
+  constexpr int TB = NT / G;
+  static size_t cap = 0;  // per instantiation, set on first use
+  if (cap == 0) {
+    cudaFuncAttributes attr;
+    cudaError_t e = cudaFuncGetAttributes(&attr, router_kernel<TI, G, EPL, NT>);
+    if (e != cudaSuccess) return e;
+    const size_t c = kSmemPerBlock - attr.sharedSizeBytes - 1024;
+    e = cudaFuncSetAttribute(router_kernel<TI, G, EPL, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(c));
+    if (e != cudaSuccess) return e;
+    cap = c;
+  }
+  const int grid = (a.T + TB - 1) / TB;
+  const size_t row = static_cast<size_t>(a.D / Elem<TI>::kVec + 1) * 16;
+  const size_t wg_bytes = a.E * row, x_bytes = TB * row;
+  const int stage_wg = wg_bytes <= cap;
+  const int stage_x = stage_wg && wg_bytes + x_bytes <= cap;
+  const size_t smem = (stage_wg ? wg_bytes : 0) + (stage_x ? x_bytes : 0);
+  return launch_pdl(router_kernel<TI, G, EPL, NT>, dim3(grid), dim3(NT), smem, s, a, stage_x, stage_wg);
 }
 
 template <typename TI>
 cudaError_t launch_t(const RouterArgs& a, cudaStream_t s) {
-  const int grid = (a.T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
-  const dim3 block(kWarps * 32);
-  if (a.E <= 8) router_kernel<TI, 8><<<grid, block, 0, s>>>(a);
-  else if (a.E <= 16) router_kernel<TI, 16><<<grid, block, 0, s>>>(a);
-  else if (a.E <= 32) router_kernel<TI, 32><<<grid, block, 0, s>>>(a);
-  else router_kernel<TI, 64><<<grid, block, 0, s>>>(a);
-  return cudaGetLastError();
+  const int E = a.E;
+  if (E == 1) return launch_g<TI, 1, 1, 128>(a, s);
+  if (E <= 3) return launch_g<TI, 2, 2, 128>(a, s);
+  if (E <= 7) return launch_g<TI, 4, 2, 128>(a, s);
+  if (E <= 8) return launch_g<TI, 8, 1, 128>(a, s);
+  if (E <= 16) return launch_g<TI, 8, 2, 128>(a, s);
+  if (E <= 32) return launch_g<TI, 8, 4, 256>(a, s);
+  return launch_g<TI, 8, 8, 256>(a, s);
 }
 
 }  // namespace

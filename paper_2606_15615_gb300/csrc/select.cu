@@ -27,6 +27,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kMaxGroups = kMaxExperts + 1;
 
 __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
+  pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int i = blockIdx.x * kThreads + t;
   const bool valid = i < a.T;
@@ -240,6 +241,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
 
 template <typename TI>
 __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
+  pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int i = blockIdx.x * kThreads + t;
   const bool valid = i < a.T;
@@ -310,6 +312,7 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
   }
   __syncthreads();
   // Gather the inputs of this block's rows, one warp per row, 16-byte vectors.
+  if (a.xg == nullptr) return;  // the tensor-core GEMM gathers its rows itself
   const int nv = a.D * static_cast<int>(sizeof(TI)) / 16;
   const uint4* x = static_cast<const uint4*>(a.x);
   uint4* xg = static_cast<uint4*>(a.xg);
@@ -342,15 +345,13 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t s) {
   const int grid = (a.T + kThreads - 1) / kThreads;
-  select_kernel<<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(select_kernel, dim3(grid), dim3(kThreads), 0, s, a);
 }
 
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s) {
   const int grid = (a.T + kThreads - 1) / kThreads;
-  if (bf16) compact_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(a);
-  else compact_kernel<float><<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  if (bf16) return launch_pdl(compact_kernel<__nv_bfloat16>, dim3(grid), dim3(kThreads), 0, s, a);
+  return launch_pdl(compact_kernel<float>, dim3(grid), dim3(kThreads), 0, s, a);
 }
 
 }  // namespace moeca
