@@ -34,7 +34,7 @@ if ROOT not in sys.path:
 METRIC = "branch-cached MoE layer tokens/s and effective TFLOP/s vs reuse ratio; % roofline"
 DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine"]
+KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep"]
 
 
 # ---------------------------------------------------------------------------
@@ -155,7 +155,7 @@ def peaks():
 
 def kernel_source_sha(kind: str) -> str:
     fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
-             "compact": "select.cu", "combine": "combine.cu"}[kind]
+             "compact": "select.cu", "combine": "combine.cu", "prep": "prep.cu"}[kind]
     with open(os.path.join(ROOT, "paper_2606_15615_gb300", "csrc", fname), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
@@ -286,6 +286,11 @@ def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float):
         return active_groups * F * D * es + rows_per_launch * (F + D) * es, 2.0 * rows_per_launch * D * F
     if kind == "combine":
         return T * D * es * (2 + k + S) + T * k * 9, 0.0
+    if kind == "prep":
+        return (algorithmic("router", wl, rows_per_launch, active_groups)[0]
+                + algorithmic("select", wl, rows_per_launch, active_groups)[0]
+                + algorithmic("compact", wl, rows_per_launch, active_groups)[0],
+                algorithmic("router", wl, rows_per_launch, active_groups)[1])
     raise KeyError(kind)
 
 

@@ -180,7 +180,8 @@ enum {
   MOECA_K_FFN1 = 3,    /* grouped GEMM X W1^T + GELU                        */
   MOECA_K_FFN2 = 4,    /* grouped GEMM Hmid W2^T -> cache rows              */
   MOECA_K_COMBINE = 5, /* Eq. 8 combine + residual + cached norms           */
-  MOECA_K_COUNT = 6
+  MOECA_K_PREP = 6,    /* router + select + compact fused in one launch (bf16) */
+  MOECA_K_COUNT = 7
 };
 
 typedef struct {

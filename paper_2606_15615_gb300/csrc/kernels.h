@@ -119,6 +119,38 @@ size_t tc_partial_bytes(int n_sms);    // bytes of the split-K partial workspace
 void tc_plan_destroy(TcPlan* p);
 cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s);
 
+// Fused router + select + compact (one cooperative launch, bf16 only).
+struct PrepArgs {
+  const void* x;          // [T, D] layer input
+  const void* w_gate;     // [E, D]
+  const float* b_gate;    // [E] or null
+  int T, D, E, k, G;      // G = E + n_shared groups
+  int renorm, entropy_norm;
+  float beta, tau0, alpha;
+  int32_t* route_e;       // [T, k]
+  float* route_w;         // [T, k]
+  float* ema;             // [T, E]
+  float* partials;        // [blocks, E, 2]
+  float* tau;             // [E] (written by block 0)
+  SelectArgs sel;         // decision inputs and outputs (its tau is replaced in-kernel)
+  int32_t* block_counts;  // [blocks, G]
+  int32_t* counts;        // [G]
+  int32_t* offsets;       // [G + 1]
+  int32_t* list;          // [rows]
+  void* xg;               // [rows, D]
+  unsigned* gbar;         // grid barrier: arrivals, generation (zeroed once)
+  unsigned long long* stats;
+  int* status;
+};
+struct PrepShape {
+  int tokens_per_block;   // 0: the fused kernel cannot run this shape
+  int epad;               // experts padded to a multiple of 8
+  size_t smem;            // dynamic shared memory per block
+};
+constexpr size_t kPrepSmemMax = 200 * 1024;
+PrepShape prep_plan(int D, int E, int max_tokens, int n_sms);
+cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
+
 // Eq. 8 combine + residual + cached branch norms.
 struct CombineArgs {
   int T, D, k, n_shared;

@@ -78,6 +78,9 @@ struct moeca_handle {
   void* hmid = nullptr;
   float* tc_partial = nullptr;
   int* tc_sem = nullptr;
+  PrepShape prep{0, 0, 0};      // fused router + select + compact, when it fits
+  int32_t* prep_counts = nullptr;
+  unsigned* prep_bar = nullptr;
   std::vector<void*> act;  // input of layer l (l >= 1)
   int* status_host = nullptr;
   int* status_dev = nullptr;
@@ -307,6 +310,12 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (use_tc) {
     A((void**)&h->tc_partial, tc_partial_bytes(h->n_sms));
     A((void**)&h->tc_sem, tc_split_units(h->n_sms) * sizeof(int));
+    h->prep = prep_plan(c.hidden, c.n_experts, c.max_tokens, h->n_sms);
+    if (h->prep.tokens_per_block) {
+      const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
+      A((void**)&h->prep_counts, nb * G * 4);
+      A((void**)&h->prep_bar, 2 * sizeof(unsigned));
+    }
   }
   h->act.assign(c.n_layers, nullptr);
   for (int l = 1; l < c.n_layers && ok; ++l) A(&h->act[l], T * D * es);
@@ -387,6 +396,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     const void* in = l == 0 ? x_in : h->act[l];
     void* out = l + 1 == c.n_layers ? x_out : h->act[l + 1];
 
+    const bool fused = h->prep.tokens_per_block != 0;
     RouterArgs ra{};
     ra.x = in; ra.w_gate = L.w.w_gate; ra.b_gate = L.w.b_gate;
     ra.T = T; ra.D = c.hidden; ra.E = c.n_experts; ra.k = c.top_k;
@@ -395,7 +405,6 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ra.route_e = L.route_e; ra.route_w = L.route_w; ra.ema = L.ema;
     ra.partials = h->partials; ra.done = h->done; ra.tau = L.tau; ra.stats = L.stats;
     ra.status = h->status_dev;
-    if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
 
     SelectArgs sa{};
     sa.T = T; sa.k = c.top_k; sa.E = c.n_experts; sa.G = h->G; sa.refresh = refresh;
@@ -407,7 +416,6 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     sa.block_counts = h->block_counts; sa.block_offsets = h->block_offsets;
     sa.counts = L.counts; sa.offsets = L.offsets; sa.done = h->done + 1;
     sa.stats = L.stats; sa.status = h->status_dev;
-    if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
 
     CompactArgs ca{};
     ca.T = T; ca.k = c.top_k; ca.E = c.n_experts; ca.G = h->G; ca.D = c.hidden; ca.n_shared = c.n_shared;
@@ -415,7 +423,22 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ca.route_e = L.route_e; ca.recompute = L.recompute; ca.slot = L.slot; ca.token_any = L.token_any;
     ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
     ca.x = in; ca.xg = (use_tc && kGemmGathersRows) ? nullptr : h->xg;
-    if ((e = timed(h, MOECA_K_COMPACT, s, [&] { return launch_compact(ca, h->bf16, s); })) != cudaSuccess) break;
+    if (fused) {
+      PrepArgs pa{};
+      pa.x = in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
+      pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
+      pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
+      pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
+      pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.partials = h->partials; pa.tau = L.tau;
+      pa.sel = sa;
+      pa.block_counts = h->prep_counts; pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
+      pa.xg = h->xg; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
+      if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
+    } else {
+      if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_COMPACT, s, [&] { return launch_compact(ca, h->bf16, s); })) != cudaSuccess) break;
+    }
 
     FfnArgs fa{};
     fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;

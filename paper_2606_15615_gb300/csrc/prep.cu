@@ -1,0 +1,607 @@
+// Fused per-layer preparation of the branch-cached MoE layer, one cooperative
+// launch with two grid barriers:
+//
+//   A  router (Eq. 7): gate logits on the tensor cores (mma.sync m16n8k16,
+//      bf16 in, fp32 accumulate) from the block's token rows and the gate
+//      matrix staged in shared memory by bulk async copies; fp32 softmax and
+//      top-k with ties to the lower expert id; the EMA statistic (Eq. 10) and
+//      the block's entropy partial sums.
+//   -- grid barrier --
+//   B  every block reduces all blocks' partials in block order to the same
+//      thresholds tau_e (Eq. 11-12), then decides its tokens' branches
+//      (Sec. 4.2, Eq. 9) and counts recomputed rows per expert group.
+//   -- grid barrier --
+//   C  every block scans the per-block counts into group offsets and its own
+//      prefix, writes its rows into the per-group lists (ascending token
+//      order) and gathers their inputs for the grouped FFN.
+//
+// The results are those of router_kernel + select_kernel + compact_kernel,
+// which remain the path for fp32, for shapes whose staging does not fit in
+// shared memory, and for grids that cannot be co-resident.  The grid barrier
+// spins with a one-second bound; on timeout it records MOECA's timeout status
+// and later phases are skipped.
+#include "common.cuh"
+#include "kernels.h"
+#include "select_token.cuh"
+
+namespace moeca {
+namespace {
+
+constexpr int kThreads = 128;
+constexpr int kMaxGroups = kMaxExperts + 1;
+constexpr unsigned long long kBarrierNs = 1000000000ull;
+
+template <int G>
+__device__ __forceinline__ float grp_max(float v) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+template <int G>
+__device__ __forceinline__ float grp_sum(float v) {
+#pragma unroll
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Grid-wide barrier over co-resident blocks (cooperative launch).  bar[0]
+// counts arrivals, bar[1] is the generation.  Returns false after a timeout.
+__device__ bool grid_sync(unsigned* bar, unsigned nblocks, int* status) {
+  __shared__ int ok_sh;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile unsigned* genp = bar + 1;
+    const unsigned gen = *genp;
+    __threadfence();
+    bool ok = true;
+    if (atomicAdd(bar, 1u) == nblocks - 1) {
+      atomicExch(bar, 0u);
+      __threadfence();
+      atomicAdd(bar + 1, 1u);
+    } else {
+      const unsigned long long t0 = globaltimer();
+      while (*genp == gen) {
+        if (globaltimer() - t0 > kBarrierNs) {
+          ok = false;
+          report_status(status, kStatusWaitTimeout, 600);
+          break;
+        }
+      }
+    }
+    __threadfence();
+    ok_sh = ok;
+  }
+  __syncthreads();
+  return ok_sh != 0;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+__device__ __forceinline__ void mma_16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                          uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// TB tokens per block (16 or 32); EPAD experts padded to a multiple of 8.
+template <int TB, int EPAD>
+__global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
+  constexpr int G = kThreads / TB;       // lanes per token in the routing epilogue (4 or 8)
+  constexpr int EPL = EPAD / G;          // experts per lane (>= 1)
+  constexpr int NTILE = EPAD / 8;        // mma n-tiles
+  constexpr int TOKG = TB / 16;          // 16-token mma groups
+  constexpr int WPG = 4 / TOKG;          // warps per token group
+  constexpr int NPW = (NTILE + WPG - 1) / WPG;  // n-tiles per warp
+  static_assert(EPL >= 1 && EPL * G == EPAD, "experts per lane");
+  extern __shared__ __align__(128) uint8_t dyn[];
+  __shared__ float sm_S[TB * EPAD];
+  __shared__ float sm_U[TB * EPAD];
+  __shared__ float sm_rs[kThreads][2];
+  __shared__ float sm_tau[kMaxExperts];
+  __shared__ float sm_H[kMaxExperts];
+  __shared__ int sm_live[kMaxExperts];
+  __shared__ float sm_lo, sm_hi;
+  __shared__ int sm_near;
+  __shared__ unsigned sm_bal[kMaxGroups];
+  __shared__ int sm_pre[kMaxGroups];
+  __shared__ int sm_tot[kMaxGroups];
+  __shared__ int sm_off[kMaxGroups + 1];
+  __shared__ int sm_rows[TB * (kMaxTopK + 1)][2];
+  __shared__ int sm_nrows;
+  __shared__ __align__(8) uint64_t sm_bar;
+
+  pdl_entry();
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int E = a.E, k = a.k, D = a.D, T = a.T;
+  const int ldw = D + 8;  // padded row, in bf16
+  __nv_bfloat16* s_w = reinterpret_cast<__nv_bfloat16*>(dyn);
+  __nv_bfloat16* s_x = s_w + EPAD * ldw;
+  float* s_logit = reinterpret_cast<float*>(s_x + TB * ldw);  // [TB][EPAD + 1]
+  const int tok0 = blockIdx.x * TB;
+  const int ntok = min(TB, T - tok0);
+
+  // ---- A0: stage gate rows and token rows ----
+  if (t == 0) {
+    sm_near = 0;
+    sm_nrows = 0;
+    mbar_init(smem_u32(&sm_bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const uint32_t bar = smem_u32(&sm_bar);
+  const uint32_t row_bytes = static_cast<uint32_t>(D) * 2;
+  if (t == 0) {
+    mbar_expect_tx(bar, row_bytes * (E + ntok));
+    const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
+    const __nv_bfloat16* x = static_cast<const __nv_bfloat16*>(a.x);
+    for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
+    for (int q = 0; q < ntok; ++q)
+      bulk_g2s(smem_u32(s_x + q * ldw), x + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
+  }
+  // Zero the padding rows the tensor cores read (experts past E, tokens past T).
+  for (int idx = t; idx < (EPAD - E) * (D / 8); idx += kThreads) {
+    const int r = E + idx / (D / 8), c = idx % (D / 8);
+    reinterpret_cast<uint4*>(s_w + r * ldw)[c] = make_uint4(0, 0, 0, 0);
+  }
+  for (int idx = t; idx < (TB - ntok) * (D / 8); idx += kThreads) {
+    const int r = ntok + idx / (D / 8), c = idx % (D / 8);
+    reinterpret_cast<uint4*>(s_x + r * ldw)[c] = make_uint4(0, 0, 0, 0);
+  }
+  if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);
+  __syncthreads();
+
+  // ---- A1: logits on the tensor cores ----
+  {
+    const int tg = warp / WPG;               // token group of this warp
+    const int nt0 = (warp % WPG) * NPW;      // first n-tile of this warp
+    float acc[NPW][4];
+#pragma unroll
+    for (int j = 0; j < NPW; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    if (tg < TOKG && nt0 < NTILE) {
+      const uint32_t a_addr = smem_u32(s_x + (tg * 16 + (lane & 15)) * ldw + (lane >> 4) * 8);
+      const int bl = lane & 15;
+      for (int k0 = 0; k0 < D; k0 += 16) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
+#pragma unroll
+        for (int j = 0; j < NPW; ++j) {
+          const int nt = nt0 + j;
+          if (nt < NTILE) {
+            uint32_t b0, b1;
+            ldsm_x2(smem_u32(s_w + (nt * 8 + (bl & 7)) * ldw + k0 + (bl >> 3) * 8), b0, b1);
+            mma_16816(acc[j], a0, a1, a2, a3, b0, b1);
+          }
+        }
+      }
+      const int g = lane >> 2, c2 = (lane & 3) * 2;
+#pragma unroll
+      for (int j = 0; j < NPW; ++j) {
+        const int nt = nt0 + j;
+        if (nt < NTILE) {
+          const int r0 = tg * 16 + g, e0 = nt * 8 + c2;
+          s_logit[r0 * (EPAD + 1) + e0] = acc[j][0];
+          s_logit[r0 * (EPAD + 1) + e0 + 1] = acc[j][1];
+          s_logit[(r0 + 8) * (EPAD + 1) + e0] = acc[j][2];
+          s_logit[(r0 + 8) * (EPAD + 1) + e0 + 1] = acc[j][3];
+        }
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- A2: softmax, top-k, EMA, entropy terms (G lanes per token) ----
+  {
+    const int tok = t / G, g = t % G;
+    const int i = tok0 + tok;
+    const bool valid = tok < ntok;
+    float zl[EPL];
+    float lmax = -INFINITY, labs = 0.f;
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+      const int e = g + G * j;
+      if (e < E) {
+        zl[j] = s_logit[tok * (EPAD + 1) + e] + (a.b_gate ? a.b_gate[e] : 0.f);
+        lmax = fmaxf(lmax, zl[j]);
+        labs = fmaxf(labs, fabsf(zl[j]));
+      } else {
+        zl[j] = -INFINITY;
+      }
+    }
+    const float m = grp_max<G>(lmax);
+    const float zabs = grp_max<G>(labs);
+    float lsum = 0.f;
+#pragma unroll
+    for (int j = 0; j < EPL; ++j)
+      if (g + G * j < E) lsum += expf(zl[j] - m);
+    const float denom = grp_sum<G>(lsum);
+    const int ranks = (k + 1 < E) ? k + 1 : E;
+    unsigned taken = 0u;
+    unsigned long long topk_mask = 0ull;
+    int sel_e[kMaxTopK + 1];
+    float sel_z[kMaxTopK + 1];
+#pragma unroll
+    for (int r = 0; r < kMaxTopK + 1; ++r) {
+      sel_e[r] = 0;
+      sel_z[r] = 0.f;
+      if (r < ranks) {
+        float bv = -INFINITY;
+        int be = 0x7fffffff;
+#pragma unroll
+        for (int j = 0; j < EPL; ++j) {
+          const int e = g + G * j;
+          if (e < E && !((taken >> j) & 1u) && (zl[j] > bv || (zl[j] == bv && e < be))) {
+            bv = zl[j];
+            be = e;
+          }
+        }
+#pragma unroll
+        for (int o = G / 2; o > 0; o >>= 1) {
+          const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+          const int oe = __shfl_xor_sync(0xffffffffu, be, o);
+          if (ov > bv || (ov == bv && oe < be)) {
+            bv = ov;
+            be = oe;
+          }
+        }
+        if (be < E && be % G == g) taken |= 1u << (be / G);
+        sel_e[r] = be;
+        sel_z[r] = bv;
+        if (r < k && be < E) topk_mask |= 1ull << be;
+      }
+    }
+    if (valid) {
+      float wsum = 0.f, w[kMaxTopK];
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        w[p] = 0.f;
+        if (p < k) {
+          w[p] = expf(sel_z[p] - m) / denom;
+          wsum += w[p];
+        }
+      }
+      bool near = false;
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p)
+        if (p + 1 < ranks && (sel_z[p] - sel_z[p + 1]) < 1e-5f * zabs) near = true;
+      if (g == 0 && near) atomicAdd(&sm_near, 1);
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        if (p < k && p % G == g) {
+          a.route_e[static_cast<size_t>(i) * k + p] = sel_e[p];
+          a.route_w[static_cast<size_t>(i) * k + p] = a.renorm ? w[p] / wsum : w[p];
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+      const int e = g + G * j;
+      float c = 0.f, u = 0.f;
+      if (valid && e < E) {
+        float* cp = a.ema + static_cast<size_t>(i) * E + e;
+        const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
+        c = a.beta * (*cp) + (1.f - a.beta) * ind;
+        *cp = c;
+        if (c > 0.f) u = c * logf(c);
+      }
+      sm_S[tok * EPAD + e] = c;
+      sm_U[tok * EPAD + e] = u;
+    }
+  }
+  __syncthreads();
+  {
+    // Block partials per expert: J interleaved runs over the block's tokens,
+    // added in run order.
+    const int J = kThreads / E;
+    const int e = t % E, jr = t / E;
+    float S = 0.f, U = 0.f;
+    if (jr < J)
+      for (int q = jr; q < TB; q += J) {
+        S += sm_S[q * EPAD + e];
+        U += sm_U[q * EPAD + e];
+      }
+    sm_rs[t][0] = S;
+    sm_rs[t][1] = U;
+    __syncthreads();
+    if (t < E) {
+      float Ss = 0.f, Us = 0.f;
+      for (int q = 0; q < J; ++q) {
+        Ss += sm_rs[q * E + t][0];
+        Us += sm_rs[q * E + t][1];
+      }
+      reinterpret_cast<float2*>(a.partials)[static_cast<size_t>(blockIdx.x) * E + t] = make_float2(Ss, Us);
+    }
+    if (t == 0 && sm_near) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(sm_near));
+  }
+  __threadfence();
+  if (!grid_sync(a.gbar, gridDim.x, a.status)) return;
+
+  // ---- B: thresholds from every block's partials (same order in every block) ----
+  {
+    const int J = kThreads / E;
+    const int e = t % E, j = t / E;
+    float S = 0.f, U = 0.f;
+    if (j < J) {
+      const float2* part = reinterpret_cast<const float2*>(a.partials);
+#pragma unroll 4
+      for (unsigned b = j; b < gridDim.x; b += J) {
+        const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
+        S += v.x;
+        U += v.y;
+      }
+    }
+    sm_rs[t][0] = S;
+    sm_rs[t][1] = U;
+    __syncthreads();
+    if (t < E) {
+      float Ss = 0.f, Us = 0.f;
+      for (int jj = 0; jj < J; ++jj) {
+        Ss += sm_rs[jj * E + t][0];
+        Us += sm_rs[jj * E + t][1];
+      }
+      sm_live[t] = Ss > 0.f;
+      sm_H[t] = Ss > 0.f ? logf(Ss) - Us / Ss : 0.f;
+    }
+    __syncthreads();
+    if (t == 0) {
+      float lo = 0.f, hi = 0.f;
+      bool any = false;
+      for (int ee = 0; ee < E; ++ee) {
+        if (!sm_live[ee]) continue;
+        if (!any || sm_H[ee] < lo) lo = sm_H[ee];
+        if (!any || sm_H[ee] > hi) hi = sm_H[ee];
+        any = true;
+      }
+      sm_lo = lo;
+      sm_hi = hi;
+    }
+    __syncthreads();
+    if (t < E) {
+      float hb = 0.5f;
+      if (sm_live[t]) {
+        if (a.entropy_norm == 0) {
+          if (T > 1) hb = fminf(1.f, fmaxf(0.f, sm_H[t] / logf(static_cast<float>(T))));
+        } else if (sm_hi > sm_lo) {
+          hb = (sm_H[t] - sm_lo) / (sm_hi - sm_lo);
+        }
+      }
+      const float tau = a.tau0 * (1.0f + a.alpha * (2.0f * hb - 1.0f));
+      sm_tau[t] = tau;
+      if (blockIdx.x == 0) a.tau[t] = tau;
+    }
+    __syncthreads();
+  }
+
+  // ---- B: branch decisions of the block's tokens (warp 0, one token per lane) ----
+  const int GG = a.G;
+  TokenDecision d;
+  if (warp == 0) {
+    SelectArgs sa = a.sel;
+    sa.tau = sm_tau;
+    const bool valid = lane < ntok;
+    decide_token(sa, tok0 + lane, valid, d);
+    int n_full = (valid && !d.bad && !d.any) ? 1 : 0;
+    for (int g = 0; g < GG; ++g) {
+      bool has = false;
+      if (g < E) {
+#pragma unroll
+        for (int p = 0; p < kMaxTopK; ++p) has |= (d.rec[p] && d.e[p] == g);
+      } else {
+        has = d.shared_row;
+      }
+      const unsigned b = __ballot_sync(0xffffffffu, has);
+      if (lane == 0) {
+        sm_bal[g] = b;
+        a.block_counts[static_cast<size_t>(blockIdx.x) * GG + g] = __popc(b);
+      }
+    }
+    const int c_matched = warp_sum_i(d.n_matched), c_rec = warp_sum_i(d.n_rec), c_near = warp_sum_i(d.n_near);
+    const int c_full = warp_sum_i(n_full), c_shared = warp_sum_i(d.shared_row ? 1 : 0);
+    if (lane == 0) {
+      unsigned long long* st = a.stats;
+      atomicAdd(st + kStRecomputed, static_cast<unsigned long long>(c_rec));
+      atomicAdd(st + kStReused, static_cast<unsigned long long>(ntok * k - c_rec));
+      if (c_shared) atomicAdd(st + kStSharedRecomputed, static_cast<unsigned long long>(c_shared));
+      if (!sa.refresh) {
+        atomicAdd(st + kStMatched, static_cast<unsigned long long>(c_matched));
+        atomicAdd(st + kStTokensFullyReused, static_cast<unsigned long long>(c_full));
+        if (c_near) atomicAdd(st + kStNearScore, static_cast<unsigned long long>(c_near));
+      }
+      if (blockIdx.x == 0) {
+        const unsigned long long br = static_cast<unsigned long long>(T) * k;
+        atomicAdd(st + kStLayerSteps, 1ull);
+        atomicAdd(st + kStBranches, br);
+        if (sa.refresh) atomicAdd(st + kStRefreshSteps, 1ull);
+        else atomicAdd(st + kStCacheBranches, br);
+      }
+    }
+  }
+  __threadfence();
+  if (!grid_sync(a.gbar, gridDim.x, a.status)) return;
+
+  // ---- C: group offsets, this block's prefix, row lists and row gather ----
+  {
+    const int nb = gridDim.x;
+    int* s_cnt = reinterpret_cast<int*>(dyn);  // [nb][GG], reusing the staging area
+    for (int idx = t; idx < nb * GG; idx += kThreads) s_cnt[idx] = __ldcg(a.block_counts + idx);
+    __syncthreads();
+    for (int g = t; g < GG; g += kThreads) {
+      int pre = 0, tot = 0;
+      for (int b = 0; b < nb; ++b) {
+        const int c = s_cnt[b * GG + g];
+        if (b < static_cast<int>(blockIdx.x)) pre += c;
+        tot += c;
+      }
+      sm_pre[g] = pre;
+      sm_tot[g] = tot;
+    }
+    __syncthreads();
+    if (t == 0) {
+      int off = 0;
+      for (int g = 0; g < GG; ++g) {
+        sm_off[g] = off;
+        off += sm_tot[g];
+      }
+      sm_off[GG] = off;
+    }
+    __syncthreads();
+    if (blockIdx.x == 0) {
+      for (int g = t; g < GG; g += kThreads) a.counts[g] = sm_tot[g];
+      for (int g = t; g <= GG; g += kThreads) a.offsets[g] = sm_off[g];
+    }
+    if (warp == 0) {
+      const int i = tok0 + lane;
+      const unsigned lt = (1u << lane) - 1u;
+#pragma unroll
+      for (int p = 0; p < kMaxTopK; ++p) {
+        if (d.rec[p]) {
+          const int g = d.e[p];
+          const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
+          const int sl = a.sel.slot[static_cast<size_t>(i) * k + p];
+          a.list[pos] = i * k + sl;
+          const int r = atomicAdd(&sm_nrows, 1);
+          sm_rows[r][0] = pos;
+          sm_rows[r][1] = i;
+        }
+      }
+      if (d.shared_row) {
+        const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
+        a.list[pos] = i;
+        const int r = atomicAdd(&sm_nrows, 1);
+        sm_rows[r][0] = pos;
+        sm_rows[r][1] = i;
+      }
+    }
+    __syncthreads();
+    // Gather the rows' inputs, four rows per warp in flight.
+    const int nv = D / 8;
+    const uint4* x = static_cast<const uint4*>(a.x);
+    uint4* xg = static_cast<uint4*>(a.xg);
+    const int n = sm_nrows;
+    for (int r0 = warp * 4; r0 < n; r0 += 16) {
+      for (int c0 = 0; c0 < nv; c0 += 32 * 4) {
+        uint4 v[4][4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int c = c0 + q * 32 + lane;
+            if (r0 + j < n && c < nv) v[j][q] = x[static_cast<size_t>(sm_rows[r0 + j][1]) * nv + c];
+          }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int c = c0 + q * 32 + lane;
+            if (r0 + j < n && c < nv) xg[static_cast<size_t>(sm_rows[r0 + j][0]) * nv + c] = v[j][q];
+          }
+      }
+    }
+  }
+}
+
+template <int TB, int EPAD>
+size_t prep_smem(int D, int n_blocks, int G) {
+  const size_t ldw = static_cast<size_t>(D) + 8;
+  const size_t stage = (EPAD + TB) * ldw * 2 + static_cast<size_t>(TB) * (EPAD + 1) * 4;
+  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;
+  return stage > counts ? stage : counts;
+}
+
+template <int TB, int EPAD>
+cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(prep_kernel<TB, EPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kPrepSmemMax);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(n_blocks);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD>, a);
+}
+
+template <int TB, int EPAD>
+int prep_occupancy(size_t smem) {
+  static bool configured = false;
+  if (!configured) {
+    if (cudaFuncSetAttribute(prep_kernel<TB, EPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPrepSmemMax) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    configured = true;
+  }
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD>, kThreads, smem) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+// Dispatch on (TB, EPAD) at run time.
+template <typename F>
+auto with_shape(int TB, int epad, F&& f) {
+#define MOECA_PREP_CASE(tb, ep) \
+  if (TB == tb && epad == ep) return f.template operator()<tb, ep>();
+  MOECA_PREP_CASE(32, 8) MOECA_PREP_CASE(32, 16) MOECA_PREP_CASE(32, 24) MOECA_PREP_CASE(32, 32)
+  MOECA_PREP_CASE(16, 8) MOECA_PREP_CASE(16, 16) MOECA_PREP_CASE(16, 24) MOECA_PREP_CASE(16, 32)
+  MOECA_PREP_CASE(16, 40) MOECA_PREP_CASE(16, 48) MOECA_PREP_CASE(16, 56) MOECA_PREP_CASE(16, 64)
+#undef MOECA_PREP_CASE
+  return f.template operator()<0, 0>();
+}
+
+}  // namespace
+
+PrepShape prep_plan(int D, int E, int max_tokens, int n_sms) {
+  PrepShape p{0, 0, 0};
+  if (D % 16 || E < 1 || E > kMaxExperts) return p;
+  const int epad = (E + 7) / 8 * 8;
+  for (int TB : {32, 16}) {
+    if (TB == 32 && epad > 32) continue;  // 32-token blocks keep EPAD * 32 / 4 lanes' registers bounded
+    const int nb = (max_tokens + TB - 1) / TB;
+    const size_t smem = with_shape(TB, epad, [&]<int tb, int ep>() -> size_t {
+      if constexpr (tb == 0) return 0;
+      else return prep_smem<tb, ep>(D, nb, E + 1);
+    });
+    if (smem == 0 || smem > kPrepSmemMax) continue;
+    const int occ = with_shape(TB, epad, [&]<int tb, int ep>() -> int {
+      if constexpr (tb == 0) return 0;
+      else return prep_occupancy<tb, ep>(smem);
+    });
+    if (occ <= 0 || static_cast<long long>(occ) * n_sms < nb) continue;
+    p.tokens_per_block = TB;
+    p.epad = epad;
+    p.smem = smem;
+    return p;
+  }
+  return p;
+}
+
+cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
+  const int nb = (a.T + p.tokens_per_block - 1) / p.tokens_per_block;
+  return with_shape(p.tokens_per_block, p.epad, [&]<int tb, int ep>() -> cudaError_t {
+    if constexpr (tb == 0) return cudaErrorInvalidValue;
+    else return prep_launch<tb, ep>(a, nb, p.smem, s);
+  });
+}
+
+}  // namespace moeca
