@@ -138,17 +138,19 @@ struct PrepArgs {
   int32_t* offsets;       // [G + 1]
   int32_t* list;          // [rows]
   void* xg;               // [rows, D]
-  unsigned* gbar;         // grid barrier: arrivals, generation (zeroed once)
+  unsigned* gbar;         // grid barrier arrival counter (zeroed once, only grows)
+  unsigned bar_base;      // arrivals on gbar from earlier launches (mod 2^32)
   unsigned long long* stats;
   int* status;
 };
 struct PrepShape {
   int tokens_per_block;   // 0: the fused kernel cannot run this shape
   int epad;               // experts padded to a multiple of 8
+  int kmax;               // compile-time bound on top-k (2, 4 or 8)
   size_t smem;            // dynamic shared memory per block
 };
 constexpr size_t kPrepSmemMax = 200 * 1024;
-PrepShape prep_plan(int D, int E, int max_tokens, int n_sms);
+PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms);
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 
 // Eq. 8 combine + residual + cached branch norms.

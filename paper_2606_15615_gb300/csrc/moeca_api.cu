@@ -78,7 +78,8 @@ struct moeca_handle {
   void* hmid = nullptr;
   float* tc_partial = nullptr;
   int* tc_sem = nullptr;
-  PrepShape prep{0, 0, 0};      // fused router + select + compact, when it fits
+  PrepShape prep{0, 0, 0, 0};   // fused router + select + compact, when it fits
+  unsigned prep_arrivals = 0;   // grid-barrier arrivals of all fused launches so far (mod 2^32)
   int32_t* prep_counts = nullptr;
   unsigned* prep_bar = nullptr;
   std::vector<void*> act;  // input of layer l (l >= 1)
@@ -310,7 +311,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (use_tc) {
     A((void**)&h->tc_partial, tc_partial_bytes(h->n_sms));
     A((void**)&h->tc_sem, tc_split_units(h->n_sms) * sizeof(int));
-    h->prep = prep_plan(c.hidden, c.n_experts, c.max_tokens, h->n_sms);
+    h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
       A((void**)&h->prep_counts, nb * G * 4);
@@ -433,7 +434,9 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       pa.sel = sa;
       pa.block_counts = h->prep_counts; pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
       pa.xg = h->xg; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
+      pa.bar_base = h->prep_arrivals;
       if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
+      h->prep_arrivals += 2u * static_cast<unsigned>((T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block);
     } else {
       if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
@@ -593,6 +596,11 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
 moeca_status moeca_reset(moeca_handle* h) {
   if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
   cudaSetDevice(h->device);
+  if (h->prep_bar) {
+    cudaError_t e = cudaMemset(h->prep_bar, 0, 2 * sizeof(unsigned));
+    if (e != cudaSuccess) return cuda_fail(h, e, "reset barrier");
+    h->prep_arrivals = 0;
+  }
   for (auto& L : h->layers) {
     L.valid = false;
     cudaError_t e = cudaMemset(L.ema, 0, static_cast<size_t>(h->cfg.max_tokens) * h->cfg.n_experts * 4);

@@ -44,31 +44,28 @@ __device__ __forceinline__ float grp_sum(float v) {
   return v;
 }
 
-// Grid-wide barrier over co-resident blocks (cooperative launch).  bar[0]
-// counts arrivals, bar[1] is the generation.  Returns false after a timeout.
-__device__ bool grid_sync(unsigned* bar, unsigned nblocks, int* status) {
+// Grid-wide barrier over co-resident blocks (cooperative launch).  *cnt only
+// grows: barrier b (0 or 1) of a launch is passed once it reaches
+// base + (b + 1) * nblocks arrivals, base being the arrivals of all earlier
+// launches (kept by the host).  Arrive is a release add, the wait an
+// acquire poll bounded by one second.  Returns false after a timeout.
+__device__ bool grid_sync(unsigned* cnt, unsigned target, int* status) {
   __shared__ int ok_sh;
   __syncthreads();
   if (threadIdx.x == 0) {
-    volatile unsigned* genp = bar + 1;
-    const unsigned gen = *genp;
-    __threadfence();
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
     bool ok = true;
-    if (atomicAdd(bar, 1u) == nblocks - 1) {
-      atomicExch(bar, 0u);
-      __threadfence();
-      atomicAdd(bar + 1, 1u);
-    } else {
-      const unsigned long long t0 = globaltimer();
-      while (*genp == gen) {
-        if (globaltimer() - t0 > kBarrierNs) {
-          ok = false;
-          report_status(status, kStatusWaitTimeout, 600);
-          break;
-        }
+    const unsigned long long t0 = globaltimer();
+    for (;;) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
+      if (static_cast<int>(v - target) >= 0) break;
+      if (globaltimer() - t0 > kBarrierNs) {
+        ok = false;
+        report_status(status, kStatusWaitTimeout, 600);
+        break;
       }
     }
-    __threadfence();
     ok_sh = ok;
   }
   __syncthreads();
@@ -93,7 +90,7 @@ __device__ __forceinline__ void mma_16816(float* c, uint32_t a0, uint32_t a1, ui
 }
 
 // TB tokens per block (16 or 32); EPAD experts padded to a multiple of 8.
-template <int TB, int EPAD>
+template <int TB, int EPAD, int KMAX>
 __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   constexpr int G = kThreads / TB;       // lanes per token in the routing epilogue (4 or 8)
   constexpr int EPL = EPAD / G;          // experts per lane (>= 1)
@@ -115,9 +112,16 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __shared__ int sm_pre[kMaxGroups];
   __shared__ int sm_tot[kMaxGroups];
   __shared__ int sm_off[kMaxGroups + 1];
-  __shared__ int sm_rows[TB * (kMaxTopK + 1)][2];
+  __shared__ int sm_rows[TB * (KMAX + 1)][2];
   __shared__ int sm_nrows;
   __shared__ __align__(8) uint64_t sm_bar;
+  // Per-token inputs of the decision, fetched at the start and kept here.
+  __shared__ int32_t sm_re[TB * KMAX];
+  __shared__ float sm_rw[TB * KMAX];
+  __shared__ int32_t sm_ce[TB * KMAX];
+  __shared__ float sm_cw[TB * KMAX];
+  __shared__ float sm_cn[TB * KMAX];
+  __shared__ float sm_ema[TB * EPAD];
 
   pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
@@ -146,6 +150,18 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
     for (int q = 0; q < ntok; ++q)
       bulk_g2s(smem_u32(s_x + q * ldw), x + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
+  }
+  // Prefetch what later phases read: cached metadata and EMA rows.
+  {
+    const size_t cb = static_cast<size_t>(tok0) * k;
+    if (!a.sel.refresh)
+      for (int idx = t; idx < ntok * k; idx += kThreads) {
+        sm_ce[idx] = a.sel.cache_e[cb + idx];
+        sm_cw[idx] = a.sel.cache_w[cb + idx];
+        sm_cn[idx] = a.sel.cache_norm[cb + idx];
+      }
+    const size_t eb = static_cast<size_t>(tok0) * E;
+    for (int idx = t; idx < ntok * E; idx += kThreads) sm_ema[(idx / E) * EPAD + idx % E] = a.ema[eb + idx];
   }
   // Zero the padding rows the tensor cores read (experts past E, tokens past T).
   for (int idx = t; idx < (EPAD - E) * (D / 8); idx += kThreads) {
@@ -226,10 +242,10 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     const int ranks = (k + 1 < E) ? k + 1 : E;
     unsigned taken = 0u;
     unsigned long long topk_mask = 0ull;
-    int sel_e[kMaxTopK + 1];
-    float sel_z[kMaxTopK + 1];
+    int sel_e[KMAX + 1];
+    float sel_z[KMAX + 1];
 #pragma unroll
-    for (int r = 0; r < kMaxTopK + 1; ++r) {
+    for (int r = 0; r < KMAX + 1; ++r) {
       sel_e[r] = 0;
       sel_z[r] = 0.f;
       if (r < ranks) {
@@ -259,9 +275,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       }
     }
     if (valid) {
-      float wsum = 0.f, w[kMaxTopK];
+      float wsum = 0.f, w[KMAX];
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         w[p] = 0.f;
         if (p < k) {
           w[p] = expf(sel_z[p] - m) / denom;
@@ -270,14 +286,17 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       }
       bool near = false;
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p)
+      for (int p = 0; p < KMAX; ++p)
         if (p + 1 < ranks && (sel_z[p] - sel_z[p + 1]) < 1e-5f * zabs) near = true;
       if (g == 0 && near) atomicAdd(&sm_near, 1);
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         if (p < k && p % G == g) {
+          const float wp = a.renorm ? w[p] / wsum : w[p];
           a.route_e[static_cast<size_t>(i) * k + p] = sel_e[p];
-          a.route_w[static_cast<size_t>(i) * k + p] = a.renorm ? w[p] / wsum : w[p];
+          a.route_w[static_cast<size_t>(i) * k + p] = wp;
+          sm_re[tok * k + p] = sel_e[p];
+          sm_rw[tok * k + p] = wp;
         }
       }
     }
@@ -286,10 +305,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       const int e = g + G * j;
       float c = 0.f, u = 0.f;
       if (valid && e < E) {
-        float* cp = a.ema + static_cast<size_t>(i) * E + e;
         const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
-        c = a.beta * (*cp) + (1.f - a.beta) * ind;
-        *cp = c;
+        c = a.beta * sm_ema[tok * EPAD + e] + (1.f - a.beta) * ind;
+        a.ema[static_cast<size_t>(i) * E + e] = c;
         if (c > 0.f) u = c * logf(c);
       }
       sm_S[tok * EPAD + e] = c;
@@ -322,7 +340,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     if (t == 0 && sm_near) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(sm_near));
   }
   __threadfence();
-  if (!grid_sync(a.gbar, gridDim.x, a.status)) return;
+  if (!grid_sync(a.gbar, a.bar_base + gridDim.x, a.status)) return;
 
   // ---- B: thresholds from every block's partials (same order in every block) ----
   {
@@ -331,7 +349,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     float S = 0.f, U = 0.f;
     if (j < J) {
       const float2* part = reinterpret_cast<const float2*>(a.partials);
-#pragma unroll 4
+#pragma unroll 8
       for (unsigned b = j; b < gridDim.x; b += J) {
         const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
         S += v.x;
@@ -382,18 +400,19 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
 
   // ---- B: branch decisions of the block's tokens (warp 0, one token per lane) ----
   const int GG = a.G;
-  TokenDecision d;
+  TokenDecisionT<KMAX> d;
   if (warp == 0) {
     SelectArgs sa = a.sel;
     sa.tau = sm_tau;
     const bool valid = lane < ntok;
-    decide_token(sa, tok0 + lane, valid, d);
+    const int q = valid ? lane * k : 0;
+    decide_token(sa, tok0 + lane, valid, sm_re + q, sm_rw + q, sm_ce + q, sm_cw + q, sm_cn + q, d);
     int n_full = (valid && !d.bad && !d.any) ? 1 : 0;
     for (int g = 0; g < GG; ++g) {
       bool has = false;
       if (g < E) {
 #pragma unroll
-        for (int p = 0; p < kMaxTopK; ++p) has |= (d.rec[p] && d.e[p] == g);
+        for (int p = 0; p < KMAX; ++p) has |= (d.rec[p] && d.e[p] == g);
       } else {
         has = d.shared_row;
       }
@@ -425,13 +444,29 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     }
   }
   __threadfence();
-  if (!grid_sync(a.gbar, gridDim.x, a.status)) return;
+  if (!grid_sync(a.gbar, a.bar_base + 2 * gridDim.x, a.status)) return;
 
   // ---- C: group offsets, this block's prefix, row lists and row gather ----
   {
     const int nb = gridDim.x;
     int* s_cnt = reinterpret_cast<int*>(dyn);  // [nb][GG], reusing the staging area
-    for (int idx = t; idx < nb * GG; idx += kThreads) s_cnt[idx] = __ldcg(a.block_counts + idx);
+    {
+      // All loads in flight before any store.
+      constexpr int kU = 8;
+      for (int base = 0; base < nb * GG; base += kThreads * kU) {
+        int v[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int idx = base + u * kThreads + t;
+          v[u] = idx < nb * GG ? __ldcg(a.block_counts + idx) : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int idx = base + u * kThreads + t;
+          if (idx < nb * GG) s_cnt[idx] = v[u];
+        }
+      }
+    }
     __syncthreads();
     for (int g = t; g < GG; g += kThreads) {
       int pre = 0, tot = 0;
@@ -461,7 +496,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       const int i = tok0 + lane;
       const unsigned lt = (1u << lane) - 1u;
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         if (d.rec[p]) {
           const int g = d.e[p];
           const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
@@ -516,11 +551,11 @@ size_t prep_smem(int D, int n_blocks, int G) {
   return stage > counts ? stage : counts;
 }
 
-template <int TB, int EPAD>
+template <int TB, int EPAD, int KMAX>
 cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(prep_kernel<TB, EPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(prep_kernel<TB, EPAD, KMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kPrepSmemMax);
     if (e != cudaSuccess) return e;
     configured = true;
@@ -535,14 +570,14 @@ cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD>, a);
+  return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD, KMAX>, a);
 }
 
-template <int TB, int EPAD>
+template <int TB, int EPAD, int KMAX>
 int prep_occupancy(size_t smem) {
   static bool configured = false;
   if (!configured) {
-    if (cudaFuncSetAttribute(prep_kernel<TB, EPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPrepSmemMax) !=
+    if (cudaFuncSetAttribute(prep_kernel<TB, EPAD, KMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPrepSmemMax) !=
         cudaSuccess) {
       cudaGetLastError();
       return 0;
@@ -550,46 +585,52 @@ int prep_occupancy(size_t smem) {
     configured = true;
   }
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD>, kThreads, smem) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD, KMAX>, kThreads, smem) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   return n;
 }
 
-// Dispatch on (TB, EPAD) at run time.
+// Dispatch on (TB, EPAD, KMAX) at run time.
 template <typename F>
-auto with_shape(int TB, int epad, F&& f) {
-#define MOECA_PREP_CASE(tb, ep) \
-  if (TB == tb && epad == ep) return f.template operator()<tb, ep>();
-  MOECA_PREP_CASE(32, 8) MOECA_PREP_CASE(32, 16) MOECA_PREP_CASE(32, 24) MOECA_PREP_CASE(32, 32)
-  MOECA_PREP_CASE(16, 8) MOECA_PREP_CASE(16, 16) MOECA_PREP_CASE(16, 24) MOECA_PREP_CASE(16, 32)
-  MOECA_PREP_CASE(16, 40) MOECA_PREP_CASE(16, 48) MOECA_PREP_CASE(16, 56) MOECA_PREP_CASE(16, 64)
+auto with_shape(int TB, int epad, int kmax, F&& f) {
+#define MOECA_PREP_CASE(tb, ep, km) \
+  if (TB == tb && epad == ep && kmax == km) return f.template operator()<tb, ep, km>();
+#define MOECA_PREP_K(tb, ep) MOECA_PREP_CASE(tb, ep, 2) MOECA_PREP_CASE(tb, ep, 4) MOECA_PREP_CASE(tb, ep, 8)
+  MOECA_PREP_K(32, 8) MOECA_PREP_K(32, 16) MOECA_PREP_K(32, 24) MOECA_PREP_K(32, 32)
+  MOECA_PREP_K(16, 8) MOECA_PREP_K(16, 16) MOECA_PREP_K(16, 24) MOECA_PREP_K(16, 32)
+  MOECA_PREP_K(16, 40) MOECA_PREP_K(16, 48) MOECA_PREP_K(16, 56) MOECA_PREP_K(16, 64)
+#undef MOECA_PREP_K
 #undef MOECA_PREP_CASE
-  return f.template operator()<0, 0>();
+  return f.template operator()<0, 0, 0>();
 }
+
+int kmax_of(int k) { return k <= 2 ? 2 : (k <= 4 ? 4 : 8); }
 
 }  // namespace
 
-PrepShape prep_plan(int D, int E, int max_tokens, int n_sms) {
-  PrepShape p{0, 0, 0};
-  if (D % 16 || E < 1 || E > kMaxExperts) return p;
+PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms) {
+  PrepShape p{0, 0, 0, 0};
+  if (D % 16 || E < 1 || E > kMaxExperts || k < 1 || k > kMaxTopK) return p;
   const int epad = (E + 7) / 8 * 8;
+  const int km = kmax_of(k);
   for (int TB : {32, 16}) {
-    if (TB == 32 && epad > 32) continue;  // 32-token blocks keep EPAD * 32 / 4 lanes' registers bounded
+    if (TB == 32 && epad > 32) continue;  // keeps 32-token blocks' per-lane expert arrays short
     const int nb = (max_tokens + TB - 1) / TB;
-    const size_t smem = with_shape(TB, epad, [&]<int tb, int ep>() -> size_t {
+    const size_t smem = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> size_t {
       if constexpr (tb == 0) return 0;
       else return prep_smem<tb, ep>(D, nb, E + 1);
     });
     if (smem == 0 || smem > kPrepSmemMax) continue;
-    const int occ = with_shape(TB, epad, [&]<int tb, int ep>() -> int {
+    const int occ = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> int {
       if constexpr (tb == 0) return 0;
-      else return prep_occupancy<tb, ep>(smem);
+      else return prep_occupancy<tb, ep, kk>(smem);
     });
     if (occ <= 0 || static_cast<long long>(occ) * n_sms < nb) continue;
     p.tokens_per_block = TB;
     p.epad = epad;
+    p.kmax = km;
     p.smem = smem;
     return p;
   }
@@ -598,9 +639,9 @@ PrepShape prep_plan(int D, int E, int max_tokens, int n_sms) {
 
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
   const int nb = (a.T + p.tokens_per_block - 1) / p.tokens_per_block;
-  return with_shape(p.tokens_per_block, p.epad, [&]<int tb, int ep>() -> cudaError_t {
+  return with_shape(p.tokens_per_block, p.epad, p.kmax, [&]<int tb, int ep, int kk>() -> cudaError_t {
     if constexpr (tb == 0) return cudaErrorInvalidValue;
-    else return prep_launch<tb, ep>(a, nb, p.smem, s);
+    else return prep_launch<tb, ep, kk>(a, nb, p.smem, s);
   });
 }
 

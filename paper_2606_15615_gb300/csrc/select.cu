@@ -34,7 +34,8 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
   const bool valid = i < a.T;
   const int k = a.k, E = a.E, G = a.G;
   TokenDecision d;
-  decide_token(a, i, valid, d);
+  const size_t b0 = static_cast<size_t>(valid ? i : 0) * a.k;
+  decide_token<kMaxTopK>(a, i, valid, a.route_e + b0, a.route_w + b0, a.cache_e + b0, a.cache_w + b0, a.cache_norm + b0, d);
   const int* e = d.e;
   const bool* rec = d.rec;
   const bool any = d.any, bad = d.bad, shared_row = d.shared_row;

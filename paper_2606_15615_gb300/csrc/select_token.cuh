@@ -16,14 +16,23 @@
 
 namespace moeca {
 
-struct TokenDecision {
-  int e[kMaxTopK];
-  bool rec[kMaxTopK];
+template <int KMAX>
+struct TokenDecisionT {
+  int e[KMAX];
+  bool rec[KMAX];
   bool any, bad, shared_row;
   int n_matched, n_rec, n_near;
 };
+using TokenDecision = TokenDecisionT<kMaxTopK>;
 
-__device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool valid, TokenDecision& d) {
+// The token's inputs come through re/rw (routing, k entries) and ce/cw/cn
+// (cached ids, weights, norms, k entries each), which may point to global or
+// shared memory; outputs go to a's global arrays at row i.
+// KMAX >= k bounds every loop at compile time.
+template <int KMAX>
+__device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool valid, const int32_t* re,
+                                             const float* rw, const int32_t* ce_in, const float* cw_in,
+                                             const float* cn_in, TokenDecisionT<KMAX>& d) {
   const int k = a.k, E = a.E;
   int* e = d.e;
   bool* rec = d.rec;
@@ -31,20 +40,20 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
   int n_matched = 0, n_rec = 0, n_near = 0;
   bool bad = false;
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) {
+  for (int p = 0; p < KMAX; ++p) {
     e[p] = -1;
     rec[p] = false;
   }
   if (valid) {
     const size_t base = static_cast<size_t>(i) * k;
-    float w[kMaxTopK];
-    int sl[kMaxTopK];
-    bool mat[kMaxTopK];
+    float w[KMAX];
+    int sl[KMAX];
+    bool mat[KMAX];
 #pragma unroll
-    for (int p = 0; p < kMaxTopK; ++p) {
+    for (int p = 0; p < KMAX; ++p) {
       if (p < k) {
-        e[p] = a.route_e[base + p];
-        w[p] = a.route_w[base + p];
+        e[p] = re[p];
+        w[p] = rw[p];
         if (e[p] < 0 || e[p] >= E) bad = true;
       }
       mat[p] = false;
@@ -53,31 +62,31 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
     if (bad) {
       report_status(a.status, kStatusBadIndex, 1000000 + i);
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) e[p] = -1;
+      for (int p = 0; p < KMAX; ++p) e[p] = -1;
     } else if (a.refresh) {
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) rec[p] = p < k;
+      for (int p = 0; p < KMAX; ++p) rec[p] = p < k;
     } else {
-      int ce[kMaxTopK];
-      float cw[kMaxTopK], cn[kMaxTopK];
+      int ce[KMAX];
+      float cw[KMAX], cn[KMAX];
       float nsum = 0.f;
 #pragma unroll
-      for (int q = 0; q < kMaxTopK; ++q) {
+      for (int q = 0; q < KMAX; ++q) {
         if (q < k) {
-          ce[q] = a.cache_e[base + q];
-          cw[q] = a.cache_w[base + q];
-          cn[q] = a.cache_norm[base + q];
+          ce[q] = ce_in[q];
+          cw[q] = cw_in[q];
+          cn[q] = cn_in[q];
           nsum += cn[q];
         }
       }
       unsigned used = 0u;
-      int qof[kMaxTopK];
+      int qof[KMAX];
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         qof[p] = -1;
         if (p < k) {
 #pragma unroll
-          for (int q = kMaxTopK - 1; q >= 0; --q)
+          for (int q = KMAX - 1; q >= 0; --q)
             if (q < k && ce[q] == e[p]) qof[p] = q;  // lowest matching slot
           if (qof[p] >= 0) {
             const int q = qof[p];
@@ -86,7 +95,7 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
             ++n_matched;
             float cwq = 0.f, cnq = 0.f;
 #pragma unroll
-            for (int qq = 0; qq < kMaxTopK; ++qq)
+            for (int qq = 0; qq < KMAX; ++qq)
               if (qq == q) { cwq = cw[qq]; cnq = cn[qq]; }
             const float delta = fabsf(w[p] - cwq);
             const float o = nsum > 0.f ? cnq / nsum : 0.f;
@@ -100,7 +109,7 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
         }
       }
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         if (p < k) {
           if (qof[p] >= 0) {
             sl[p] = qof[p];
@@ -115,7 +124,7 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
     }
     if (!bad) {
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) {
+      for (int p = 0; p < KMAX; ++p) {
         if (p < k) {
           any |= rec[p];
           n_rec += rec[p];
