@@ -34,7 +34,7 @@ if ROOT not in sys.path:
 METRIC = "branch-cached MoE layer tokens/s and effective TFLOP/s vs reuse ratio; % roofline"
 DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep"]
+KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn"]
 
 
 # ---------------------------------------------------------------------------
@@ -154,7 +154,7 @@ def peaks():
 
 
 def kernel_source_sha(kind: str) -> str:
-    fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
+    fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "ffn": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
              "compact": "select.cu", "combine": "combine.cu", "prep": "prep.cu"}[kind]
     with open(os.path.join(ROOT, "paper_2606_15615_gb300", "csrc", fname), "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
@@ -284,6 +284,10 @@ def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float):
         return active_groups * F * D * es + rows_per_launch * (D + F) * es, 2.0 * rows_per_launch * D * F
     if kind == "ffn2":
         return active_groups * F * D * es + rows_per_launch * (F + D) * es, 2.0 * rows_per_launch * D * F
+    if kind == "ffn":
+        b1, f1 = algorithmic("ffn1", wl, rows_per_launch, active_groups)
+        b2, f2 = algorithmic("ffn2", wl, rows_per_launch, active_groups)
+        return b1 + b2, f1 + f2
     if kind == "combine":
         return T * D * es * (2 + k + S) + T * k * 9, 0.0
     if kind == "prep":

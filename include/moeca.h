@@ -181,7 +181,8 @@ enum {
   MOECA_K_FFN2 = 4,    /* grouped GEMM Hmid W2^T -> cache rows              */
   MOECA_K_COMBINE = 5, /* Eq. 8 combine + residual + cached norms           */
   MOECA_K_PREP = 6,    /* router + select + compact fused in one launch (bf16) */
-  MOECA_K_COUNT = 7
+  MOECA_K_FFN = 7,     /* both grouped GEMMs in one persistent launch (bf16) */
+  MOECA_K_COUNT = 8
 };
 
 typedef struct {

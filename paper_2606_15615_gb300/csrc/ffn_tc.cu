@@ -6,13 +6,14 @@
 // where rows r of expert group g are [offsets[g], offsets[g] + counts[g]) and
 // dst is the branch cache (token*k + slot) or the shared-expert rows.
 //
-// Persistent kernel, one CTA per SM, 6 warps:
+// Persistent kernel, one CTA per SM, 10 warps:
 //   warp 0  TMA producer: 128 x 64 A tile and BN x 64 weight tile per stage,
 //           128-byte swizzle, into a 192 KB shared-memory ring (4-8 stages);
 //   warp 1  allocates 512 TMEM columns and issues tcgen05.mma (M = 128,
 //           N = BN, K = 16) from one thread; tcgen05.commit frees each stage
 //           and signals a finished accumulator;
-//   warps 2-5  epilogue: tcgen05.ld of their TMEM lane quadrant, GELU / bf16
+//   warps 2-9  epilogue, two warps per TMEM lane quadrant (each takes half of
+//           the columns): tcgen05.ld, GELU / bf16
 //           rounding, row stores (phase 2 scatters through the row list).
 // Two TMEM accumulators (2 x BN columns) let the epilogue of one tile overlap
 // the MMAs of the next.  Tiles run group by group, n-tile major and m-tile
@@ -23,7 +24,9 @@
 // that runs out records MOECA's timeout status, raises a CTA-wide abort flag,
 // drains the copies and MMAs this CTA issued, frees TMEM and returns.
 #include <cuda.h>
+#include <algorithm>
 #include <cstdio>
+#include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -33,21 +36,41 @@ namespace moeca {
 namespace {
 
 constexpr int kBM = 128;          // rows per tile (MMA M)
-constexpr int kBK = 64;           // K per stage: 64 bf16 = one 128-byte swizzle row
+constexpr int kBK = 64;           // K per sub-block: 64 bf16 = one 128-byte swizzle row
 constexpr int kMaxBN = 256;
 constexpr int kMaxStages = 8;
 constexpr int kRingBytes = 4 * (16384 + 256 * 128);  // 192 KB of stages, any tile width
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;  // warps 2-9
 constexpr int kTmemCols = 512;
-constexpr int kABytes = kBM * kBK * 2;        // 16 KB
-constexpr int kBBytesMax = kMaxBN * kBK * 2;  // 32 KB
-constexpr int kSmemBytes = kRingBytes + 1024;
+constexpr int kABytes = kBM * kBK * 2;        // 16 KB: one A sub-block
+constexpr int kStageOut = 32 * 64;  // per epilogue warp: 32 rows x 32 bf16 columns
+constexpr int kSmemBytes = kRingBytes + 8 * kStageOut + 1024;
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr unsigned long long kWaitNs = 1000000000ull;
 constexpr int kMaxSplit = 4;
+constexpr int kPlanTab = 512;     // plan entries by m-tile count kept in shared memory
+
+// Stage geometry of one phase at one candidate tile width, fixed per handle.
+// A stage holds `sub` K sub-blocks of 64: sub x (A 128 x 64 | B BN x 64),
+// A sub-blocks first.  Wider stages mean fewer ring round trips per byte.
+struct TcShape {
+  int BN;           // tile width (0 = candidate absent)
+  int nt;           // N / BN
+  int KB;           // stages along K: K / (64 sub)
+  int sub;          // K sub-blocks per stage (1 or 2)
+  int stage_bytes;  // sub x (16 KB + BN x 128)
+  int nst;          // stages in the ring
+  uint64_t nt_magic;  // floor(2^32 / nt) + 1: (n x magic) >> 32 is n / nt for n < 2^32 / nt
+};
 
 struct TcArgs {
-  int G, E, N, K, BN, k, T, phase, gelu_tanh;
+  int G, E, k, T, gelu_tanh;
+  int first, last;   // GEMM phases of this launch: 1..1, 2..2, or 1..2 (both, fused)
+  int N[2];          // per phase: output width
+  TcShape shp[2][3]; // per phase and candidate width
+  const int* plan_tab;  // packed plans by m-tile count, [3][tab_n]: fused, phase 1 alone, phase 2 alone
+  int tab_n;
   const int32_t* counts;
   const int32_t* offsets;
   const int32_t* list;
@@ -56,14 +79,14 @@ struct TcArgs {
   void* shared_h;  // phase 2 shared destination [T, D]
   float* partial;  // split-K partial tiles, [max_units][128][BN] fp32
   int* tile_sem;   // split-K arrival counters, [max_units], left at 0
-  int max_units;   // capacity of partial / tile_sem
+  int* dep;        // fused launch: per m-tile {phase-1 tiles stored, phase-2 units started}, left at 0
+  int max_mtiles;  // capacity of dep (pairs)
   int gather;      // phase 1: A rows gathered from the layer input by token (tile::gather4)
-  int bn[3];       // candidate tile widths (0 = none), matching the maps' B boxes
-  int force_bn;    // 0: choose; else use this width
-  int force_split; // 0: choose; else use this many K splits
-  float split_cost;  // cost of one split unit's partial round trip, in BN-256 k-blocks
   int* status;
 };
+
+// Plan word: tile-width index of phase 1 (bits 0-3) and phase 2 (4-7), K splits (8-11).
+__host__ __device__ constexpr int plan_word(int bi0, int bi1, int S) { return bi0 | (bi1 << 4) | (S << 8); }
 
 // Weight and activation tensor maps of one phase: A (activation rows) and,
 // for each candidate width, B (routed experts) and Bs (shared expert).
@@ -72,41 +95,9 @@ struct alignas(64) TcMaps {
   CUtensorMap b[3];
   CUtensorMap bs[3];
 };
-
-// Tile width and K split for this launch.  Every CTA evaluates the same cost
-// model on the same device-resident counts.  A unit is one (tile, K range).
-// Cost = waves of units over the grid x per-unit time, where per-unit time is
-// k-blocks x stage time (a stage streams 128 + BN rows of 128 bytes; its MMAs
-// take about 0.7 of a 256-wide stage's load time), plus one for pipeline fill
-// and epilogue, plus, for split units, the fp32 partial round trip.
-struct Plan {
-  int bi, S;
+struct TcMapPair {
+  TcMaps p[2];
 };
-
-__device__ Plan choose_plan(const TcArgs& a, int m_tiles, int KB, int grid) {
-  Plan best{-1, 1};
-  float best_cost = 3.0e38f;
-  for (int bi = 0; bi < 3; ++bi) {
-    const int BN = a.bn[bi];
-    if (BN == 0 || (a.force_bn && BN != a.force_bn)) continue;
-    const int tiles = m_tiles * (a.N / BN);
-    const float stage = fmaxf((128.f + BN) / 384.f, 0.7f * BN / 256.f);
-    for (int S = 1; S <= 4 && S <= KB; ++S) {
-      if (a.force_split && S != a.force_split) continue;
-      if (S > 1 && tiles * S > a.max_units) break;
-      const int units = tiles * S;
-      const int waves = (units + grid - 1) / grid;
-      const float per = ((KB + S - 1) / S) * stage + 1.0f + (S > 1 ? a.split_cost * BN / 256.f : 0.f);
-      const float cost = waves * per;
-      if (cost < best_cost - 1e-3f) {
-        best_cost = cost;
-        best = Plan{bi, S};
-      }
-    }
-  }
-  if (best.bi < 0) best = Plan{0, 1};  // forced values matched nothing: widest tile, no split
-  return best;
-}
 
 // Bounded wait for phase `parity` of a barrier.  False on timeout or abort.
 __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
@@ -189,88 +180,182 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// 32 fp32 values of one row -> (GELU) -> bf16 -> 64 contiguous bytes.
-__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const uint32_t* v, bool gelu, int tanh_form) {
+// Tanh-form GELU with the hardware tanh approximation (MUFU; relative error
+// about 2^-11).  The result is rounded to bf16 (relative step 2^-8) right
+// after, so the approximation stays below the output rounding.
+__device__ __forceinline__ float gelu_tanh_hw(float z) {
+  const float u = 0.7978845608028654f * fmaf(0.044715f * z, z * z, z);
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(u));
+  const float hz = 0.5f * z;
+  return fmaf(hz, t, hz);
+}
+
+// One warp's 32 x 32 output chunk: lane i holds row i's 32 fp32 values.
+// They go through GELU (phase 1) and bf16 rounding, then through a 2 KB
+// shared-memory stage so that each global store writes 64 contiguous bytes
+// of 8 rows (instead of 16 bytes of 32 rows).  `dst` is this lane's row at
+// the chunk's first column, or null for a row that is not stored.  The stage
+// is XOR-swizzled by row pairs so both of its accesses are conflict-free.
+__device__ __forceinline__ void store_chunk(uint8_t* stage, __nv_bfloat16* dst, const uint32_t* v, bool gelu,
+                                            int tanh_form, int lane) {
   uint32_t packed[16];
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     float x0 = __uint_as_float(v[2 * j]), x1 = __uint_as_float(v[2 * j + 1]);
     if (gelu) {
-      x0 = gelu_f(x0, tanh_form);
-      x1 = gelu_f(x1, tanh_form);
+      x0 = tanh_form ? gelu_tanh_hw(x0) : gelu_f(x0, 0);
+      x1 = tanh_form ? gelu_tanh_hw(x1) : gelu_f(x1, 0);
     }
     __nv_bfloat162 h2 = __floats2bfloat162_rn(x0, x1);
     packed[j] = *reinterpret_cast<uint32_t*>(&h2);
   }
-  uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-  for (int j = 0; j < 4; ++j) d4[j] = make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
+  for (int j = 0; j < 4; ++j)
+    *reinterpret_cast<uint4*>(stage + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) =
+        make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
+  __syncwarp();
+  const unsigned long long mine = reinterpret_cast<unsigned long long>(dst);
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int row = it * 8 + (lane >> 2), j = lane & 3;
+    const uint4 val = *reinterpret_cast<const uint4*>(stage + row * 64 + ((j ^ ((row >> 1) & 3)) << 4));
+    __nv_bfloat16* d = reinterpret_cast<__nv_bfloat16*>(__shfl_sync(0xffffffffu, mine, row));
+    if (d) *reinterpret_cast<uint4*>(d + j * 8) = val;
+  }
+  __syncwarp();
 }
 
-struct TileCoord {
-  int g, m_tile, n_tile;
+// Shape of one phase for this launch, identical in every CTA.
+struct PhaseShape {
+  int BN, nt, KB, sub, stage_bytes, nst, S, units;
+  uint64_t nt_magic;
 };
 
-__device__ __forceinline__ TileCoord decode_tile(int tile, const int* tiles_before, const int* cnt, int G,
-                                                 int n_tiles) {
-  int g = 0;
-  while (g + 1 < G && tile >= tiles_before[g + 1]) ++g;
-  const int local = tile - tiles_before[g];
-  const int mt = (cnt[g] + kBM - 1) / kBM;
-  return TileCoord{g, local % mt, local / mt};
+__device__ __forceinline__ PhaseShape phase_shape(const TcArgs& a, int p, int bi, int S, int m_tiles) {
+  const TcShape& t = a.shp[p][bi];
+  PhaseShape r;
+  r.BN = t.BN;
+  r.nt = t.nt;
+  r.KB = t.KB;
+  r.sub = t.sub;
+  r.stage_bytes = t.stage_bytes;
+  r.nst = t.nst;
+  r.S = S;
+  r.units = m_tiles * t.nt * S;
+  r.nt_magic = t.nt_magic;
+  return r;
+}
+
+// One unit of work: phase p, tile (group g, m-tile m, n-tile n), K split sp.
+// mi is the m-tile's index over all groups (the dependency slot).
+struct Unit {
+  int p, tile, sp, g, m, n, mi;
+};
+
+// Units of phase 0 come first, then those of phase 1.  Within a phase, tiles
+// run m-tile major (groups in order) and n-tile minor: CTAs working at the
+// same time share the A rows of an m-tile, and an expert's m-tiles, which
+// read the same weight tiles, run close together.  Splits of a tile are a
+// whole tile list apart.
+__device__ __forceinline__ Unit decode_unit(int u, const PhaseShape& s0, const PhaseShape& s1, int U0,
+                                            const int* mt_before, int G) {
+  Unit r;
+  r.p = u < U0 ? 0 : 1;
+  const int v = u - (r.p ? U0 : 0);
+  const int nt = r.p ? s1.nt : s0.nt;
+  const int S = r.p ? s1.S : s0.S;
+  if (S == 1) {
+    r.tile = v;
+    r.sp = 0;
+  } else {
+    const int tiles = mt_before[G] * nt;
+    r.tile = v % tiles;
+    r.sp = v / tiles;
+  }
+  r.mi = static_cast<int>((static_cast<uint64_t>(r.tile) * (r.p ? s1.nt_magic : s0.nt_magic)) >> 32);
+  r.n = r.tile - r.mi * nt;
+  // Last group whose first m-tile is at or before mi (empty groups precede
+  // the non-empty group that shares their start).
+  int lo = 0, hi = G - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (mt_before[mid] <= r.mi) lo = mid;
+    else hi = mid - 1;
+  }
+  r.g = lo;
+  r.m = r.mi - mt_before[lo];
+  return r;
+}
+
+// First ring slot of the second phase of a fused launch: the one that starts
+// at or after the end of the newest first-phase stage, so the first
+// second-phase copies overwrite the oldest first-phase stages.
+__device__ __forceinline__ int second_phase_first_slot(int issued0, const PhaseShape& s0, const PhaseShape& s1) {
+  if (issued0 == 0) return 0;
+  const int end = ((issued0 - 1) % s0.nst + 1) * s0.stage_bytes;
+  return ((end + s1.stage_bytes - 1) / s1.stage_bytes) % s1.nst;
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Bounded wait until *p >= target (another CTA's release).  False on timeout or abort.
+__device__ __noinline__ bool wait_count(const int* p, int target, volatile int* abort_flag) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 1;; ++it) {
+    if (ld_acquire(p) >= target) return true;
+    if ((it & 15u) == 0) {
+      if (*abort_flag) return false;
+      const unsigned long long now = globaltimer();
+      if (t0 == 0) t0 = now;
+      else if (now - t0 > kWaitNs) return false;
+    }
+  }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    ffn_tc_kernel(const __grid_constant__ TcMaps maps, TcArgs a) {
+    ffn_tc_kernel(const __grid_constant__ TcMapPair maps, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t full_bar[2][kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[2][kMaxStages];
   __shared__ __align__(8) uint64_t tfull_bar[2];
   __shared__ __align__(8) uint64_t tempty_bar[2];
   __shared__ __align__(8) uint64_t drain_bar;
   __shared__ uint32_t tmem_base_sh;
-  __shared__ int tiles_before[kMaxGroups + 1];
+  __shared__ int mt_before[kMaxGroups + 1];  // m-tiles ahead of each group; [G] = all
   __shared__ int cnt_sh[kMaxGroups];
   __shared__ int off_sh[kMaxGroups];
   __shared__ volatile int abort_flag;
-  __shared__ int split_sh, bi_sh;
+  __shared__ int bi_sh[2], split_sh;
+  __shared__ int plan_sh[kPlanTab];
   __shared__ int rows_sh[kBM];  // producer: token of each row of the current tile (gather)
   __shared__ volatile int ep_abort;
   __shared__ volatile int ep_last;
 
-  pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G;
-  const int KB = a.K / kBK;
+  const int p_lo = a.first - 1, p_hi = a.last - 1;
+  const bool fused = p_lo != p_hi;
 
+  // Everything that does not read the previous kernel's output happens
+  // before the programmatic-dependency wait: barriers, TMEM, map prefetch.
   if (threadIdx.x == 0) {
-    int m_tiles = 0;
-    for (int g = 0; g < G; ++g) {
-      const int c = a.counts[g];
-      cnt_sh[g] = c;
-      off_sh[g] = a.offsets[g];
-      m_tiles += (c + kBM - 1) / kBM;
-    }
-    const Plan pl = choose_plan(a, m_tiles, KB, gridDim.x);
-    bi_sh = pl.bi;
-    split_sh = pl.S;
-    const int nt = a.N / a.bn[pl.bi];
-    int acc = 0;
-    for (int g = 0; g < G; ++g) {
-      tiles_before[g] = acc;
-      acc += ((cnt_sh[g] + kBM - 1) / kBM) * nt;
-    }
-    tiles_before[G] = acc;
     abort_flag = 0;
     ep_abort = 0;
-    for (int s = 0; s < kMaxStages; ++s) {
-      mbar_init(smem_u32(&full_bar[s]), 1);
-      mbar_init(smem_u32(&empty_bar[s]), 1);
+    for (int p = 0; p < 2; ++p) {
+      for (int s = 0; s < kMaxStages; ++s) {
+        mbar_init(smem_u32(&full_bar[p][s]), 1);
+        mbar_init(smem_u32(&empty_bar[p][s]), 1);
+      }
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&tfull_bar[s]), 1);
-      mbar_init(smem_u32(&tempty_bar[s]), 128);
+      mbar_init(smem_u32(&tempty_bar[s]), kEpiThreads);
     }
     mbar_init(smem_u32(&drain_bar), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -282,72 +367,170 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     tc_fence_before();
   }
+  if (warp == 2 && lane < 14) {
+    const TcMaps& m = maps.p[lane / 7];
+    const int j = lane % 7;
+    const CUtensorMap* t = j == 0 ? &m.a : (j < 4 ? &m.b[j - 1] : &m.bs[j - 4]);
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(t)) : "memory");
+  }
+  if (warp == 2) {
+    // Bring the launch parameters into the constant cache while the previous
+    // kernel finishes (the roles read them right after the wait).
+    const TcShape& w = a.shp[lane / 3 & 1][lane % 3];
+    asm volatile("" ::"r"(w.BN), "r"(w.nt), "r"(w.KB), "r"(w.sub), "r"(w.stage_bytes), "r"(w.nst), "l"(w.nt_magic));
+    asm volatile("" ::"r"(a.N[lane & 1]), "l"(a.counts), "l"(a.list), "l"(a.hmid), "l"(a.dep), "l"(a.status),
+                 "l"(a.cache_h), "r"(a.max_mtiles), "r"(a.gather), "l"(a.partial));
+  }
+  const int tab_n = min(a.tab_n, kPlanTab);
+  if (warp == 0) {
+    // This launch's plan table (it does not depend on the previous kernel).
+    const int* tab = a.plan_tab + (fused ? 0 : a.first) * a.tab_n;
+    for (int i = lane; i < tab_n; i += 32) plan_sh[i] = tab[i];
+    __syncwarp();
+  }
+  pdl_entry();
+  if (warp == 0) {
+    // Group sizes, loaded by all lanes at once, and the m-tiles ahead of each group.
+    int m_tiles = 0;
+    for (int g0 = 0; g0 < G; g0 += 32) {
+      const int g = g0 + lane;
+      const int c = g < G ? a.counts[g] : 0;
+      const int o = g < G ? a.offsets[g] : 0;
+      const int mt = (c + kBM - 1) / kBM;
+      int incl = mt;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += v;
+      }
+      if (g < G) {
+        cnt_sh[g] = c;
+        off_sh[g] = o;
+        mt_before[g] = m_tiles + incl - mt;
+      }
+      m_tiles += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) {
+      // Beyond the table, the largest tabulated count's widths, without splits.
+      const int w = plan_sh[min(m_tiles, tab_n - 1)];
+      mt_before[G] = m_tiles;
+      bi_sh[0] = w & 15;
+      bi_sh[1] = (w >> 4) & 15;
+      split_sh = fused || m_tiles >= tab_n ? 1 : (w >> 8) & 15;
+      if (fused && m_tiles > a.max_mtiles) {
+        report_status(a.status, kStatusBadIndex, 5000000 + m_tiles);
+        abort_flag = 1;
+      }
+    }
+  }
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
-  const int BN = a.bn[bi_sh];
-  const int n_tiles = a.N / BN;
-  // Ring depth for this width: as many stages as fit the 192 KB ring.
-  const int stage_bytes = kABytes + BN * kBK * 2;
-  const int nst = min(kMaxStages, kRingBytes / stage_bytes);
-  const CUtensorMap* tmA = &maps.a;
-  const CUtensorMap* tmB = &maps.b[bi_sh];
-  const CUtensorMap* tmBs = &maps.bs[bi_sh];
-  const int tiles = tiles_before[G];
-  const int S = split_sh;
-  const int total = tiles * S;  // units: unit u is tile u % tiles, K split u / tiles
+  const int m_tiles = mt_before[G];
+  const PhaseShape s0 = phase_shape(a, 0, bi_sh[0], split_sh, m_tiles);
+  const PhaseShape s1 = phase_shape(a, 1, bi_sh[1], split_sh, m_tiles);
+  const int U0 = p_lo == 0 ? s0.units : 0;
+  const int total = abort_flag ? 0 : U0 + (p_hi == 1 ? s1.units : 0);
 
   if (warp == 0) {
     // ---------------- TMA producer (lane 0 issues; the warp fetches row indices) ----------------
-    int stage = 0;
-    uint32_t phase = 0;
-    int issued = 0;
-    const uint32_t bbytes = static_cast<uint32_t>(BN) * kBK * 2;
+    // Each phase has its own ring partition (slot size = its stage size) and
+    // barriers; per-slot parity bits let the second phase start mid-ring.
+    // A CTA's units run phase 0 first, so the state of the current phase
+    // lives in (sl, par, used) and phase 0's is kept in (par0, used0).
+    int cp = -1, sl = 0;
+    uint32_t par = 0u, used = 0u;    // bit s: uses of slot s so far mod 2; slot s used at all
+    uint32_t par0 = 0u, used0 = 0u;  // phase 0's, once phase 1 has begun
+    int issued0 = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
-      const int tile = u % tiles, sp = u / tiles;
-      const TileCoord tc = decode_tile(tile, tiles_before, cnt_sh, G, n_tiles);
-      const CUtensorMap* tb = tc.g < a.E ? tmB : tmBs;
-      const int brow = (tc.g < a.E ? tc.g * a.N : 0) + tc.n_tile * BN;
-      const int arow = off_sh[tc.g] + tc.m_tile * kBM;
-      const int kb0 = sp * KB / S, kb1 = (sp + 1) * KB / S;
-      if (a.gather) {
+      const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
+      const PhaseShape sh = t.p ? s1 : s0;
+      if (t.p != cp) {
+        if (cp == 0) {
+          par0 = par;
+          used0 = used;
+          sl = second_phase_first_slot(issued0, s0, s1);
+        } else {
+          sl = 0;
+        }
+        par = 0u;
+        used = 0u;
+        cp = t.p;
+      }
+      const TcMaps& mp = maps.p[t.p];
+      const int bsel = bi_sh[t.p];
+      const CUtensorMap* tb = t.g < a.E ? &mp.b[bsel] : &mp.bs[bsel];
+      const CUtensorMap* ta = &mp.a;
+      const int brow = (t.g < a.E ? t.g * a.N[t.p] : 0) + t.n * sh.BN;
+      const int arow = off_sh[t.g] + t.m * kBM;
+      const int kb0 = sh.S == 1 ? 0 : t.sp * sh.KB / sh.S, kb1 = sh.S == 1 ? sh.KB : (t.sp + 1) * sh.KB / sh.S;
+      const bool gather = a.gather && t.p == 0;
+      if (gather) {
         // Token of each of the tile's 128 rows; rows past the group's end
         // repeat its first row (their results are never stored).
-        const int valid = cnt_sh[tc.g] - tc.m_tile * kBM;
+        const int valid = cnt_sh[t.g] - t.m * kBM;
 #pragma unroll
         for (int j = 0; j < kBM / 32; ++j) {
           const int r = lane * (kBM / 32) + j;
           const int ent = a.list[arow + (r < valid ? r : 0)];
-          int tok = tc.g < a.E ? ent / a.k : ent;
+          int tok = t.g < a.E ? ent / a.k : ent;
           tok = tok < 0 ? 0 : (tok >= a.T ? a.T - 1 : tok);
           rows_sh[r] = tok;
         }
         __syncwarp();
       }
       if (lane == 0) {
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(smem_u32(&empty_bar[stage]), phase ^ 1u, &abort_flag)) {
+        if (fused && t.p == 1) {
+          // The m-tile's hidden rows come from every phase-1 tile of it, stored
+          // by other CTAs' epilogues with generic stores and read here by TMA.
+          int* d = a.dep + 2 * t.mi;
+          if (!wait_count(d, s0.nt, &abort_flag)) {
+            ok = false;
+          } else {
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            // The last phase-2 unit to start on this m-tile re-arms its counters.
+            if (atomicAdd(d + 1, 1) == s1.nt - 1) {
+              d[0] = 0;
+              d[1] = 0;
+            }
+          }
+        }
+        for (int kb = kb0; kb < kb1 && ok; ++kb) {
+          if (fused && t.p == 1 && !((used >> sl) & 1u)) {
+            // First use of this second-phase slot: wait until the first-phase
+            // stages it overlaps have been consumed by their MMAs.
+            const int lo = sl * s1.stage_bytes / s0.stage_bytes;
+            const int hi = min(((sl + 1) * s1.stage_bytes - 1) / s0.stage_bytes, s0.nst - 1);
+            for (int q = lo; q <= hi && ok; ++q)
+              if ((used0 >> q) & 1u)
+                ok = mbar_wait(smem_u32(&empty_bar[0][q]), ((par0 >> q) & 1u) ^ 1u, &abort_flag);
+            if (!ok) break;
+          }
+          if (!mbar_wait(smem_u32(&empty_bar[t.p][sl]), ((par >> sl) & 1u) ^ 1u, &abort_flag)) {
             ok = false;
             break;
           }
-          const uint32_t fb = smem_u32(&full_bar[stage]);
-          mbar_expect_tx(fb, kABytes + bbytes);
-          uint8_t* sa = smem + stage * stage_bytes;
-          if (a.gather) {
+          const uint32_t fb = smem_u32(&full_bar[t.p][sl]);
+          mbar_expect_tx(fb, sh.stage_bytes);
+          uint8_t* sa = smem + sl * sh.stage_bytes;
+          uint8_t* sb = sa + sh.sub * kABytes;
+          for (int j = 0; j < sh.sub; ++j) {
+            const int x = (kb * sh.sub + j) * kBK;
+            if (gather) {
 #pragma unroll 4
-            for (int j = 0; j < kBM / 4; ++j)
-              tma_gather4(smem_u32(sa + j * 512), tmA, kb * kBK, rows_sh[4 * j], rows_sh[4 * j + 1],
-                          rows_sh[4 * j + 2], rows_sh[4 * j + 3], fb);
-          } else {
-            tma_load_2d(smem_u32(sa), tmA, kb * kBK, arow, fb);
+              for (int q = 0; q < kBM / 4; ++q)
+                tma_gather4(smem_u32(sa + j * kABytes + q * 512), ta, x, rows_sh[4 * q], rows_sh[4 * q + 1],
+                            rows_sh[4 * q + 2], rows_sh[4 * q + 3], fb);
+            } else {
+              tma_load_2d(smem_u32(sa + j * kABytes), ta, x, arow, fb);
+            }
+            tma_load_2d(smem_u32(sb + j * sh.BN * kBK * 2), tb, x, brow, fb);
           }
-          tma_load_2d(smem_u32(sa + kABytes), tb, kb * kBK, brow, fb);
-          ++issued;
-          if (++stage == nst) {
-            stage = 0;
-            phase ^= 1u;
-          }
+          par ^= 1u << sl;
+          used |= 1u << sl;
+          if (t.p == 0) ++issued0;
+          sl = sl + 1 == sh.nst ? 0 : sl + 1;
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -355,56 +538,67 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
     }
     if (!ok && lane == 0) {
-      if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 100 + a.phase);
+      if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 100 + a.first);
       abort_flag = 1;
-      // Let the copies already issued land before the CTA can exit.
-      const int pending = issued < nst ? issued : nst;
-      int s = stage;
-      uint32_t ph = phase;
-      for (int j = 0; j < pending; ++j) {
-        if (--s < 0) {
-          s = nst - 1;
-          ph ^= 1u;
-        }
-        unsigned long long t0 = globaltimer();
-        while (!mbar_try(smem_u32(&full_bar[s]), ph) && globaltimer() - t0 < kWaitNs) {
-        }
+      // Let the copies already issued land before the CTA can exit: wait for
+      // the last use of every slot that was used.
+      if (cp == 0) {
+        par0 = par;
+        used0 = used;
       }
+      const uint32_t par1 = cp == 1 ? par : 0u, used1 = cp == 1 ? used : 0u;
+      for (int p = 0; p < 2; ++p)
+        for (int q = 0; q < kMaxStages; ++q)
+          if ((((p ? used1 : used0)) >> q) & 1u) {
+            const uint32_t ph = (((p ? par1 : par0) >> q) & 1u) ^ 1u;
+            unsigned long long t0 = globaltimer();
+            while (!mbar_try(smem_u32(&full_bar[p][q]), ph) && globaltimer() - t0 < kWaitNs) {
+            }
+          }
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
-    int stage = 0;
-    uint32_t phase = 0;
+    int cp = -1, sl = 0;
+    uint32_t par = 0u;
+    int consumed0 = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    const uint32_t idesc = instr_desc(kBM, BN);
     bool ok = true;
     for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
-      const int sp = u / tiles;
-      const int kb0 = sp * KB / S, kb1 = (sp + 1) * KB / S;
+      const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
+      const PhaseShape sh = t.p ? s1 : s0;
+      const int kb0 = sh.S == 1 ? 0 : t.sp * sh.KB / sh.S, kb1 = sh.S == 1 ? sh.KB : (t.sp + 1) * sh.KB / sh.S;
+      const uint32_t idesc = instr_desc(kBM, sh.BN);
+      if (t.p != cp) {
+        sl = cp == 0 ? second_phase_first_slot(consumed0, s0, s1) : 0;
+        par = 0u;
+        cp = t.p;
+      }
       if (!mbar_wait(smem_u32(&tempty_bar[acc]), acc_phase ^ 1u, &abort_flag)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * BN);
+      const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * kMaxBN);
       for (int kb = kb0; kb < kb1; ++kb) {
-        if (!mbar_wait(smem_u32(&full_bar[stage]), phase, &abort_flag)) {
+        if (!mbar_wait(smem_u32(&full_bar[t.p][sl]), (par >> sl) & 1u, &abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + stage * stage_bytes);
-        const uint32_t sb = sa + kABytes;
+        const uint32_t sa = smem_u32(smem + sl * sh.stage_bytes);
+        const uint32_t sb = sa + sh.sub * kABytes;
+        for (int j = 0; j < sh.sub; ++j) {
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          mma_bf16(d_tmem, smem_desc(sa + kk * 32), smem_desc(sb + kk * 32), idesc, (kb != kb0) || kk != 0);
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            mma_bf16(d_tmem, smem_desc(sa + j * kABytes + kk * 32), smem_desc(sb + j * sh.BN * kBK * 2 + kk * 32),
+                     idesc, (kb != kb0) || j != 0 || kk != 0);
+          }
         }
-        mma_commit(smem_u32(&empty_bar[stage]));
-        if (++stage == nst) {
-          stage = 0;
-          phase ^= 1u;
-        }
+        mma_commit(smem_u32(&empty_bar[t.p][sl]));
+        par ^= 1u << sl;
+        if (t.p == 0) ++consumed0;
+        sl = sl + 1 == sh.nst ? 0 : sl + 1;
       }
       if (!ok) break;
       mma_commit(smem_u32(&tfull_bar[acc]));
@@ -414,7 +608,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (!ok) {
-      if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 200 + a.phase);
+      if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 200 + a.first);
       abort_flag = 1;
     }
     // Every MMA this thread issued has completed once the drain barrier fires.
@@ -424,57 +618,71 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 2) {
     // ---------------- Epilogue ----------------
-    // The 4 epilogue warps (128 threads) agree on every abort and every
+    // The 8 epilogue warps (256 threads) agree on every abort and every
     // split-K decision through named barrier 1, so none can wait alone.
-    const int quad = warp & 3;  // TMEM lanes [32 quad, 32 quad + 32)
+    const int quad = warp & 3;         // TMEM lanes [32 quad, 32 quad + 32)
+    const int half = (warp - 2) >> 2;  // which half of the tile's columns
+    uint8_t* stage = smem + kRingBytes + (warp - 2) * kStageOut;  // this warp's store stage
     const int r = quad * 32 + lane;
     const bool leader = warp == 2 && lane == 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
-      const int tile = u % tiles, sp = u / tiles;
-      const TileCoord tc = decode_tile(tile, tiles_before, cnt_sh, G, n_tiles);
+      const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
+      const PhaseShape sh = t.p ? s1 : s0;
+      const int BN = sh.BN, S = sh.S, N = a.N[t.p];
       const bool got = __all_sync(0xffffffffu, mbar_wait(smem_u32(&tfull_bar[acc]), acc_phase, &abort_flag));
       if (!got && lane == 0) ep_abort = 1;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
+      asm volatile("bar.sync 1, 256;" ::: "memory");
       if (ep_abort) {
-        if (leader && !abort_flag) report_status(a.status, kStatusWaitTimeout, 300 + a.phase);
+        if (leader && !abort_flag) report_status(a.status, kStatusWaitTimeout, 300 + a.first);
         abort_flag = 1;
         break;
       }
       tc_fence_after();
-      const int mrow = tc.m_tile * kBM + r;
-      const bool live = mrow < cnt_sh[tc.g];
-      const size_t grow = static_cast<size_t>(off_sh[tc.g]) + mrow;
-      const int n0 = tc.n_tile * BN;
+      const int mrow = t.m * kBM + r;
+      const bool live = mrow < cnt_sh[t.g];
+      const size_t grow = static_cast<size_t>(off_sh[t.g]) + mrow;
+      const int n0 = t.n * BN;
       __nv_bfloat16* dst = nullptr;
       if (live) {
-        if (a.phase == 1) {
-          dst = static_cast<__nv_bfloat16*>(a.hmid) + grow * a.N + n0;
+        if (t.p == 0) {
+          dst = static_cast<__nv_bfloat16*>(a.hmid) + grow * N + n0;
         } else {
           const int dr = a.list[grow];
-          const int lim = tc.g < a.E ? a.T * a.k : a.T;
+          const int lim = t.g < a.E ? a.T * a.k : a.T;
           if (dr >= 0 && dr < lim) {
-            dst = static_cast<__nv_bfloat16*>(tc.g < a.E ? a.cache_h : a.shared_h) + static_cast<size_t>(dr) * a.N + n0;
+            dst = static_cast<__nv_bfloat16*>(t.g < a.E ? a.cache_h : a.shared_h) + static_cast<size_t>(dr) * N + n0;
           } else {
             report_status(a.status, kStatusBadIndex, 4000000 + static_cast<int>(grow));
           }
         }
       }
-      const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(acc * kMaxBN);
+      const int nch = BN / 64;  // 32-column chunks per half
+      const int c_lo = half * nch, c_hi = c_lo + nch;
       if (S == 1) {
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = c_lo; c < c_hi; ++c) {
           uint32_t v[32];
           tmem_ld32(tbase + c * 32, v);
-          if (dst) store_row32(dst + c * 32, v, a.phase == 1, a.gelu_tanh);
+          store_chunk(stage, dst ? dst + c * 32 : nullptr, v, t.p == 0, a.gelu_tanh, lane);
         }
         tc_fence_before();
         mbar_arrive(smem_u32(&tempty_bar[acc]));
+        if (fused && t.p == 0) {
+          // Publish this tile's hidden rows to the phase-2 units of its m-tile,
+          // which read them through the async (TMA) proxy: every writer orders
+          // its stores before later async-proxy accesses, the barrier collects
+          // the writers, and one release add makes them visible with the count.
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+          asm volatile("bar.sync 1, 256;" ::: "memory");
+          if (leader) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.dep + 2 * t.mi) : "memory");
+        }
       } else {
         // Split K: park this split's fp32 rows, free TMEM, then the last
         // split to arrive for the tile sums the splits in split order.
-        float* mine = a.partial + (static_cast<size_t>(tile) * S + sp) * kBM * BN + static_cast<size_t>(r) * BN;
-        for (int c = 0; c < BN / 32; ++c) {
+        float* mine = a.partial + (static_cast<size_t>(t.tile) * S + t.sp) * kBM * BN + static_cast<size_t>(r) * BN;
+        for (int c = c_lo; c < c_hi; ++c) {
           uint32_t v[32];
           tmem_ld32(tbase + c * 32, v);
           float4* d4 = reinterpret_cast<float4*>(mine + c * 32);
@@ -486,13 +694,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         mbar_arrive(smem_u32(&tempty_bar[acc]));
         __threadfence();
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (leader) ep_last = atomicAdd(a.tile_sem + tile, 1) == S - 1;
-        asm volatile("bar.sync 1, 128;" ::: "memory");
+        asm volatile("bar.sync 1, 256;" ::: "memory");
+        if (leader) ep_last = atomicAdd(a.tile_sem + t.tile, 1) == S - 1;
+        asm volatile("bar.sync 1, 256;" ::: "memory");
         if (ep_last) {
           __threadfence();
-          const float* base = a.partial + static_cast<size_t>(tile) * S * kBM * BN + static_cast<size_t>(r) * BN;
-          for (int c = 0; c < BN / 32; ++c) {
+          const float* base = a.partial + static_cast<size_t>(t.tile) * S * kBM * BN + static_cast<size_t>(r) * BN;
+          for (int c = c_lo; c < c_hi; ++c) {
             uint32_t v[32];
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
@@ -525,9 +733,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 v[h * 16 + 4 * j + 3] = __float_as_uint(acc4.w);
               }
             }
-            if (dst) store_row32(dst + c * 32, v, a.phase == 1, a.gelu_tanh);
+            store_chunk(stage, dst ? dst + c * 32 : nullptr, v, t.p == 0, a.gelu_tanh, lane);
           }
-          if (leader) a.tile_sem[tile] = 0;
+          if (leader) a.tile_sem[t.tile] = 0;
         }
       }
       if (++acc == 2) {
@@ -582,13 +790,16 @@ struct TcPlan {
   const void* g_src = nullptr;  // layer input the gather map was encoded for
   int g_rows = 0;
   int bn1[3], bn2[3];
+  TcShape shp[2][3];
+  int* d_tab = nullptr;  // device plan table [3][tab_n]
+  int tab_n = 0;
   int n_sms;
-  int force_bn, force_split;
-  float split_cost;
+  int force_split;
 };
 
 size_t tc_split_units(int n_sms) { return static_cast<size_t>(4) * n_sms; }
 size_t tc_partial_bytes(int n_sms) { return tc_split_units(n_sms) * kBM * kMaxBN * sizeof(float); }
+size_t tc_dep_pairs(int max_rows, int G) { return static_cast<size_t>((max_rows + kBM - 1) / kBM + G); }
 
 namespace {
 
@@ -602,6 +813,80 @@ void candidates(int n, int* bn) {
     if (bn[0] == bn[1]) bn[1] = 0;
     else bn[2] = 0;
   }
+}
+
+// Stage geometry: two K sub-blocks per stage when the tile is at most 128
+// wide (and K allows), so every stage moves 48-64 KB.
+TcShape make_shape(int N, int K, int BN) {
+  TcShape t{};
+  if (!BN) return t;
+  t.BN = BN;
+  t.nt = N / BN;
+  t.sub = (BN <= 128 && K % (2 * kBK) == 0) ? 2 : 1;
+  t.KB = K / (kBK * t.sub);
+  t.stage_bytes = t.sub * (kABytes + BN * kBK * 2);
+  t.nst = std::min(kMaxStages, kRingBytes / t.stage_bytes);
+  t.nt_magic = (1ull << 32) / static_cast<uint64_t>(t.nt) + 1;
+  return t;
+}
+
+// Cost model, in microseconds of one SM: a stage costs the larger of a
+// fixed ring round trip (~0.31 us) and its bytes at ~150 GB/s; a unit adds
+// 1.5 us of pipeline fill and epilogue; a split unit adds its fp32 partial
+// round trip (split_cost x a 256-wide stage x BN / 256).
+float stage_us(const TcShape& t) { return std::max(0.31f, t.stage_bytes / 150000.0f); }
+float unit_us(const TcShape& t, int S, float split_cost) {
+  return ((t.KB + S - 1) / S) * stage_us(t) + 1.5f + (S > 1 ? split_cost * 0.33f * t.BN / 256.0f : 0.0f);
+}
+
+// Busiest CTA's time when U0 units of time t0 precede U1 units of time t1,
+// dealt round-robin over the grid.
+float makespan(int U0, float t0, int U1, float t1, int grid) {
+  const int U = U0 + U1, r0 = U0 % grid, rt = U % grid;
+  float worst = 0.0f;
+  for (int b : {0, std::min(r0, rt), std::max(r0, rt)}) {
+    if (b >= grid) continue;
+    const int n0 = U0 / grid + (b < r0), nt = U / grid + (b < rt);
+    worst = std::max(worst, n0 * t0 + (nt - n0) * t1);
+  }
+  return worst;
+}
+
+// Plan for `mt` m-tiles: fused (section 0) or one phase alone (section 1 + p).
+int best_plan(const TcPlan* p, int section, int mt, int force_bn, int force_split, float split_cost) {
+  const int grid = p->n_sms;
+  const int max_units = static_cast<int>(tc_split_units(grid));
+  float best = 3.0e38f;
+  int word = plan_word(0, 0, 1);
+  if (section == 0) {
+    for (int i0 = 0; i0 < 3; ++i0)
+      for (int i1 = 0; i1 < 3; ++i1) {
+        const TcShape &a0 = p->shp[0][i0], &a1 = p->shp[1][i1];
+        if (!a0.BN || !a1.BN || (force_bn && (a0.BN != force_bn || a1.BN != force_bn))) continue;
+        const float c = makespan(mt * a0.nt, unit_us(a0, 1, 0.0f), mt * a1.nt, unit_us(a1, 1, 0.0f), grid);
+        if (c < best - 1e-3f) {
+          best = c;
+          word = plan_word(i0, i1, 1);
+        }
+      }
+    return word;
+  }
+  const int ph = section - 1;
+  for (int bi = 0; bi < 3; ++bi) {
+    const TcShape& t = p->shp[ph][bi];
+    if (!t.BN || (force_bn && t.BN != force_bn)) continue;
+    for (int S = 1; S <= kMaxSplit && S <= t.KB; ++S) {
+      if (force_split && S != force_split) continue;
+      const int tiles = mt * t.nt;
+      if (S > 1 && tiles * S > max_units) break;
+      const float c = static_cast<float>((tiles * S + grid - 1) / grid) * unit_us(t, S, split_cost);
+      if (c < best - 1e-3f) {
+        best = c;
+        word = ph == 0 ? plan_word(bi, 0, S) : plan_word(0, bi, S);
+      }
+    }
+  }
+  return word;
 }
 
 bool encode_phase(TcMaps* m, const int* bn, const void* a_base, uint64_t rows, uint64_t K, const void* w,
@@ -628,9 +913,7 @@ bool encode_phase(TcMaps* m, const int* bn, const void* a_base, uint64_t rows, u
 TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen) {
   TcPlan* p = new TcPlan();
   p->n_sms = n_sms;
-  p->force_bn = a.tile_n;
   p->force_split = a.split_k;
-  p->split_cost = 40.0f;  // measured: split units rarely pay for their partial round trip
   candidates(a.F, p->bn1);
   candidates(a.D, p->bn2);
   const char* what = nullptr;
@@ -639,6 +922,26 @@ TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen) {
   else if (!encode_phase(&p->p1, p->bn1, a.xg, a.max_rows, a.D, a.w1, static_cast<uint64_t>(a.E) * a.F, a.ws1, a.F) ||
            !encode_phase(&p->p2, p->bn2, a.hmid, a.max_rows, a.F, a.w2, static_cast<uint64_t>(a.E) * a.D, a.ws2, a.D))
     what = "tensor map encoding failed";
+  if (!what) {
+    for (int i = 0; i < 3; ++i) {
+      p->shp[0][i] = make_shape(a.F, a.D, p->bn1[i]);
+      p->shp[1][i] = make_shape(a.D, a.F, p->bn2[i]);
+    }
+    // One plan per possible m-tile count, for the fused launch and for each
+    // phase alone.  Split units cost a partial round trip that rarely pays
+    // (measured), hence the large split cost; forced values bypass it.
+    const float split_cost = 40.0f;
+    p->tab_n = std::min(static_cast<int>(tc_dep_pairs(a.max_rows, a.G)) + 1, kPlanTab);
+    std::vector<int> tab(3 * static_cast<size_t>(p->tab_n));
+    for (int sec = 0; sec < 3; ++sec)
+      for (int mt = 0; mt < p->tab_n; ++mt)
+        tab[sec * p->tab_n + mt] = best_plan(p, sec, mt, a.tile_n, a.split_k, split_cost);
+    if (cudaMalloc(&p->d_tab, tab.size() * sizeof(int)) != cudaSuccess ||
+        cudaMemcpy(p->d_tab, tab.data(), tab.size() * sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess) {
+      cudaGetLastError();
+      what = "cannot allocate the GEMM plan table";
+    }
+  }
   if (!what && cudaFuncSetAttribute(ffn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
                    cudaSuccess) {
     cudaGetLastError();
@@ -646,24 +949,40 @@ TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen) {
   }
   if (what) {
     if (err && errlen > 0) snprintf(err, errlen, "%s", what);
-    delete p;
+    tc_plan_destroy(p);
     return nullptr;
   }
   return p;
 }
 
-void tc_plan_destroy(TcPlan* p) { delete p; }
+void tc_plan_destroy(TcPlan* p) {
+  if (!p) return;
+  if (p->d_tab) cudaFree(p->d_tab);
+  delete p;
+}
 
 cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s) {
   TcArgs t{};
   t.G = a.G;
   t.E = a.E;
-  t.N = phase == 1 ? a.F : a.D;
-  t.K = phase == 1 ? a.D : a.F;
   t.k = a.k;
   t.T = a.T;
-  t.phase = phase;
   t.gelu_tanh = a.gelu_tanh;
+  // phase 0: both phases in one launch, unless K splits are forced (they
+  // need single-phase launches) or there is no dependency workspace.
+  const bool fuse = phase == 0 && a.dep && p->force_split <= 1;
+  if (phase == 0 && !fuse) {
+    cudaError_t e = launch_ffn_tc(p, a, 1, s);
+    return e != cudaSuccess ? e : launch_ffn_tc(p, a, 2, s);
+  }
+  t.first = fuse ? 1 : phase;
+  t.last = fuse ? 2 : phase;
+  t.N[0] = a.F;
+  t.N[1] = a.D;
+  for (int q = 0; q < 2; ++q)
+    for (int i = 0; i < 3; ++i) t.shp[q][i] = p->shp[q][i];
+  t.plan_tab = p->d_tab;
+  t.tab_n = p->tab_n;
   t.counts = a.counts;
   t.offsets = a.offsets;
   t.list = a.list;
@@ -672,15 +991,13 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
   t.shared_h = a.shared_h;
   t.partial = a.partial;
   t.tile_sem = a.tile_sem;
-  t.max_units = a.partial ? static_cast<int>(tc_split_units(p->n_sms)) : 0;
-  const int* bn = phase == 1 ? p->bn1 : p->bn2;
-  for (int i = 0; i < 3; ++i) t.bn[i] = bn[i];
-  t.force_bn = p->force_bn;
-  t.force_split = p->force_split;
-  t.split_cost = p->split_cost;
+  t.dep = a.dep;
+  t.max_mtiles = a.max_mtiles;
   t.status = a.status;
-  const TcMaps* maps = phase == 1 ? &p->p1 : &p->p2;
-  if (phase == 1 && a.x) {
+  TcMapPair maps;
+  maps.p[0] = p->p1;
+  maps.p[1] = p->p2;
+  if (a.x && t.first == 1) {
     // Phase 1 reads its rows straight from the layer input; re-encode the
     // gather map when that buffer or its row count changes.
     if (a.x != p->g_src || a.T != p->g_rows) {
@@ -689,10 +1006,10 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
       p->g_src = a.x;
       p->g_rows = a.T;
     }
-    maps = &p->p1g;
+    maps.p[0] = p->p1g;
     t.gather = 1;
   }
-  return launch_pdl(ffn_tc_kernel, dim3(p->n_sms), dim3(kThreads), kSmemBytes, s, *maps, t);
+  return launch_pdl(ffn_tc_kernel, dim3(p->n_sms), dim3(kThreads), kSmemBytes, s, maps, t);
 }
 
 }  // namespace moeca

@@ -106,6 +106,8 @@ struct FfnArgs {
   int split_k;           // tensor-core K splits to force (0: chosen per launch)
   float* partial;        // split-K workspace of the tensor-core path (or null: no split)
   int* tile_sem;         // split-K arrival counters, zeroed once
+  int* dep;              // tensor-core fused launch: per m-tile counter pairs, zeroed once (or null)
+  int max_mtiles;        // capacity of dep, tc_dep_pairs(max_rows, G)
   int* status;
 };
 cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s);
@@ -116,7 +118,10 @@ struct TcPlan;
 TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen);
 size_t tc_split_units(int n_sms);      // split-K units the workspace holds
 size_t tc_partial_bytes(int n_sms);    // bytes of the split-K partial workspace
+size_t tc_dep_pairs(int max_rows, int G);  // m-tile counter pairs a fused launch can need
 void tc_plan_destroy(TcPlan* p);
+// phase 1 or 2: that GEMM alone; phase 0: both, fused into one persistent
+// launch when a.dep is set and no K split is forced (else two launches).
 cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s);
 
 // Fused router + select + compact (one cooperative launch, bf16 only).

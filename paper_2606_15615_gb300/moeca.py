@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "
                 -6: "TIMEOUT", -7: "DEVICE_STATUS"}
 MOECA_F32, MOECA_BF16 = 0, 1
 MOECA_FFN_AUTO, MOECA_FFN_SIMT = 0, 1
-KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep"]
+KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn"]
 
 
 class moeca_config(C.Structure):
@@ -68,7 +68,7 @@ class moeca_layer_trace(C.Structure):
 
 
 class moeca_kernel_times(C.Structure):
-    _fields_ = [("total_ms", C.c_double * 7), ("launches", C.c_int64 * 7)]
+    _fields_ = [("total_ms", C.c_double * 8), ("launches", C.c_int64 * 8)]
 
 
 class moeca_route_args(C.Structure):
