@@ -50,6 +50,7 @@ constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr unsigned long long kWaitNs = 1000000000ull;
 constexpr int kMaxSplit = 4;
 constexpr int kPlanTab = 512;     // plan entries by m-tile count kept in shared memory
+constexpr int kUQ = 4;            // unit queue from the producer to the MMA and epilogue roles
 
 // Stage geometry of one phase at one candidate tile width, fixed per handle.
 // A stage holds `sub` K sub-blocks of 64: sub x (A 128 x 64 | B BN x 64),
@@ -79,8 +80,9 @@ struct TcArgs {
   void* shared_h;  // phase 2 shared destination [T, D]
   float* partial;  // split-K partial tiles, [max_units][128][BN] fp32
   int* tile_sem;   // split-K arrival counters, [max_units], left at 0
-  int* dep;        // fused launch: per m-tile {phase-1 tiles stored, phase-2 units started}, left at 0
-  int max_mtiles;  // capacity of dep (pairs)
+  int* dep;        // fused launch: per (m-tile, phase-2 split) {phase-1 tiles stored, phase-2 units started}, left at 0
+  int dep_pairs;   // capacity of dep (pairs); pair (mi, q) is at mi x 4 + q
+  int* work;       // {next unit ticket, CTAs done}, left at 0: units past the first go to whoever asks
   int gather;      // phase 1: A rows gathered from the layer input by token (tile::gather4)
   int* status;
 };
@@ -257,7 +259,7 @@ struct Unit {
 // run m-tile major (groups in order) and n-tile minor: CTAs working at the
 // same time share the A rows of an m-tile, and an expert's m-tiles, which
 // read the same weight tiles, run close together.  Splits of a tile are a
-// whole tile list apart.
+// adjacent (consecutive CTAs), so the last of them to finish reduces soon.
 __device__ __forceinline__ Unit decode_unit(int u, const PhaseShape& s0, const PhaseShape& s1, int U0,
                                             const int* mt_before, int G) {
   Unit r;
@@ -269,9 +271,8 @@ __device__ __forceinline__ Unit decode_unit(int u, const PhaseShape& s0, const P
     r.tile = v;
     r.sp = 0;
   } else {
-    const int tiles = mt_before[G] * nt;
-    r.tile = v % tiles;
-    r.sp = v / tiles;
+    r.tile = v / S;
+    r.sp = v - r.tile * S;
   }
   r.mi = static_cast<int>((static_cast<uint64_t>(r.tile) * (r.p ? s1.nt_magic : s0.nt_magic)) >> 32);
   r.n = r.tile - r.mi * nt;
@@ -336,6 +337,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ int rows_sh[kBM];  // producer: token of each row of the current tile (gather)
   __shared__ volatile int ep_abort;
   __shared__ volatile int ep_last;
+  __shared__ volatile int uq[kUQ];
+  __shared__ __align__(8) uint64_t uq_full[kUQ];
+  __shared__ __align__(8) uint64_t uq_empty[kUQ];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G;
@@ -358,6 +362,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&tempty_bar[s]), kEpiThreads);
     }
     mbar_init(smem_u32(&drain_bar), 1);
+    for (int q = 0; q < kUQ; ++q) {
+      mbar_init(smem_u32(&uq_full[q]), 1);
+      mbar_init(smem_u32(&uq_empty[q]), 2);  // the MMA thread and the epilogue leader
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -379,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const TcShape& w = a.shp[lane / 3 & 1][lane % 3];
     asm volatile("" ::"r"(w.BN), "r"(w.nt), "r"(w.KB), "r"(w.sub), "r"(w.stage_bytes), "r"(w.nst), "l"(w.nt_magic));
     asm volatile("" ::"r"(a.N[lane & 1]), "l"(a.counts), "l"(a.list), "l"(a.hmid), "l"(a.dep), "l"(a.status),
-                 "l"(a.cache_h), "r"(a.max_mtiles), "r"(a.gather), "l"(a.partial));
+                 "l"(a.cache_h), "r"(a.dep_pairs), "r"(a.gather), "l"(a.partial));
   }
   const int tab_n = min(a.tab_n, kPlanTab);
   if (warp == 0) {
@@ -416,8 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mt_before[G] = m_tiles;
       bi_sh[0] = w & 15;
       bi_sh[1] = (w >> 4) & 15;
-      split_sh = fused || m_tiles >= tab_n ? 1 : (w >> 8) & 15;
-      if (fused && m_tiles > a.max_mtiles) {
+      split_sh = m_tiles >= tab_n ? 1 : (w >> 8) & 15;
+      if (fused && m_tiles * kMaxSplit > a.dep_pairs) {
         report_status(a.status, kStatusBadIndex, 5000000 + m_tiles);
         abort_flag = 1;
       }
@@ -427,8 +435,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
   const int m_tiles = mt_before[G];
-  const PhaseShape s0 = phase_shape(a, 0, bi_sh[0], split_sh, m_tiles);
+  // K splits apply to the launched phase alone, or to phase 2 of a fused launch.
+  const PhaseShape s0 = phase_shape(a, 0, bi_sh[0], fused ? 1 : split_sh, m_tiles);
   const PhaseShape s1 = phase_shape(a, 1, bi_sh[1], split_sh, m_tiles);
+  // Fused: phase-2 split q reads the hidden columns of phase-1 n-tiles
+  // [q gq, (q + 1) gq); its dependency slot is (m-tile, q).
+  const int gq = s0.nt / s1.S;
   const int U0 = p_lo == 0 ? s0.units : 0;
   const int total = abort_flag ? 0 : U0 + (p_hi == 1 ? s1.units : 0);
 
@@ -443,7 +455,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t par0 = 0u, used0 = 0u;  // phase 0's, once phase 1 has begun
     int issued0 = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+    // Units: blockIdx.x first, then tickets from the shared counter, in
+    // increasing order (so phase 0 before phase 1 here too).  Each is passed
+    // to the MMA and epilogue roles through the unit queue; -1 ends it.
+    int qs = 0;
+    uint32_t qpar = 0u;
+    int u = static_cast<int>(blockIdx.x) < total ? static_cast<int>(blockIdx.x) : -1;
+    for (;;) {
+      if (lane == 0) {
+        ok = mbar_wait(smem_u32(&uq_empty[qs]), qpar ^ 1u, &abort_flag);
+        if (ok) {
+          uq[qs] = u;
+          mbar_arrive(smem_u32(&uq_full[qs]));
+        }
+      }
+      if (++qs == kUQ) {
+        qs = 0;
+        qpar ^= 1u;
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok || u < 0) break;
       const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
       const PhaseShape sh = t.p ? s1 : s0;
       if (t.p != cp) {
@@ -484,8 +515,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (fused && t.p == 1) {
           // The m-tile's hidden rows come from every phase-1 tile of it, stored
           // by other CTAs' epilogues with generic stores and read here by TMA.
-          int* d = a.dep + 2 * t.mi;
-          if (!wait_count(d, s0.nt, &abort_flag)) {
+          int* d = a.dep + 2 * (t.mi * kMaxSplit + t.sp);
+          if (!wait_count(d, gq, &abort_flag)) {
             ok = false;
           } else {
             asm volatile("fence.proxy.async.global;" ::: "memory");
@@ -536,6 +567,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       __syncwarp();
       if (!ok) break;
+      int next = 0;
+      if (lane == 0) next = static_cast<int>(gridDim.x) + atomicAdd(a.work, 1);
+      next = __shfl_sync(0xffffffffu, next, 0);
+      u = next < total ? next : -1;
     }
     if (!ok && lane == 0) {
       if (!abort_flag) report_status(a.status, kStatusWaitTimeout, 100 + a.first);
@@ -564,7 +599,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+    int qs = 0;
+    uint32_t qpar = 0u;
+    for (;;) {
+      if (!mbar_wait(smem_u32(&uq_full[qs]), qpar, &abort_flag)) {
+        ok = false;
+        break;
+      }
+      const int u = uq[qs];
+      mbar_arrive(smem_u32(&uq_empty[qs]));
+      if (++qs == kUQ) {
+        qs = 0;
+        qpar ^= 1u;
+      }
+      if (u < 0) break;
       const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
       const PhaseShape sh = t.p ? s1 : s0;
       const int kb0 = sh.S == 1 ? 0 : t.sp * sh.KB / sh.S, kb1 = sh.S == 1 ? sh.KB : (t.sp + 1) * sh.KB / sh.S;
@@ -627,7 +675,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool leader = warp == 2 && lane == 0;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+    int qs = 0;
+    uint32_t qpar = 0u;
+    for (;;) {
+      const bool gotq = __all_sync(0xffffffffu, mbar_wait(smem_u32(&uq_full[qs]), qpar, &abort_flag));
+      const int u = uq[qs];
+      if (!gotq && lane == 0) ep_abort = 1;
+      asm volatile("bar.sync 1, 256;" ::: "memory");  // every epilogue thread has read the queue slot
+      if (ep_abort) {
+        if (leader && !abort_flag) report_status(a.status, kStatusWaitTimeout, 300 + a.first);
+        abort_flag = 1;
+        break;
+      }
+      if (leader) mbar_arrive(smem_u32(&uq_empty[qs]));
+      if (++qs == kUQ) {
+        qs = 0;
+        qpar ^= 1u;
+      }
+      if (u < 0) break;
       const Unit t = decode_unit(u, s0, s1, U0, mt_before, G);
       const PhaseShape sh = t.p ? s1 : s0;
       const int BN = sh.BN, S = sh.S, N = a.N[t.p];
@@ -676,20 +741,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the writers, and one release add makes them visible with the count.
           asm volatile("fence.proxy.async.global;" ::: "memory");
           asm volatile("bar.sync 1, 256;" ::: "memory");
-          if (leader) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.dep + 2 * t.mi) : "memory");
+          if (leader)
+            asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.dep + 2 * (t.mi * kMaxSplit + t.n / gq))
+                         : "memory");
         }
       } else {
-        // Split K: park this split's fp32 rows, free TMEM, then the last
-        // split to arrive for the tile sums the splits in split order.
-        float* mine = a.partial + (static_cast<size_t>(t.tile) * S + t.sp) * kBM * BN + static_cast<size_t>(r) * BN;
+        // Split K: park this split's fp32 tile, free TMEM, then the last split
+        // to arrive for the tile sums the splits in split order.  A parked
+        // tile is laid out [32-column chunk][4-column group][row][4], so each
+        // warp access covers 512 contiguous bytes.
+        float4* mine = reinterpret_cast<float4*>(a.partial + (static_cast<size_t>(t.tile) * S + t.sp) * kBM * BN);
         for (int c = c_lo; c < c_hi; ++c) {
           uint32_t v[32];
           tmem_ld32(tbase + c * 32, v);
-          float4* d4 = reinterpret_cast<float4*>(mine + c * 32);
 #pragma unroll
           for (int j = 0; j < 8; ++j)
-            d4[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+            mine[(c * 8 + j) * kBM + r] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                                      __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
         }
         tc_fence_before();
         mbar_arrive(smem_u32(&tempty_bar[acc]));
@@ -699,7 +767,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("bar.sync 1, 256;" ::: "memory");
         if (ep_last) {
           __threadfence();
-          const float* base = a.partial + static_cast<size_t>(t.tile) * S * kBM * BN + static_cast<size_t>(r) * BN;
+          const float4* base = reinterpret_cast<const float4*>(a.partial + static_cast<size_t>(t.tile) * S * kBM * BN);
+          const size_t split_stride = static_cast<size_t>(kBM) * BN / 4;  // float4s per parked tile
           for (int c = c_lo; c < c_hi; ++c) {
             uint32_t v[32];
 #pragma unroll
@@ -709,10 +778,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int q = 0; q < kMaxSplit; ++q) {
                 if (q < S) {
-                  const float4* s4 = reinterpret_cast<const float4*>(
-                      base + static_cast<size_t>(q) * kBM * BN + c * 32 + h * 16);
 #pragma unroll
-                  for (int j = 0; j < 4; ++j) f[q][j] = __ldcg(s4 + j);
+                  for (int j = 0; j < 4; ++j) f[q][j] = __ldcg(base + q * split_stride + (c * 8 + h * 4 + j) * kBM + r);
                 }
               }
 #pragma unroll
@@ -749,6 +816,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
+  if (threadIdx.x == 0) {
+    // The last CTA out re-arms the unit counter (every CTA has taken its
+    // final ticket by now); the next launch reads it after this one ends.
+    __threadfence();
+    if (atomicAdd(a.work + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.work[0] = 0;
+      a.work[1] = 0;
+    }
   }
 }
 
@@ -799,7 +875,9 @@ struct TcPlan {
 
 size_t tc_split_units(int n_sms) { return static_cast<size_t>(4) * n_sms; }
 size_t tc_partial_bytes(int n_sms) { return tc_split_units(n_sms) * kBM * kMaxBN * sizeof(float); }
-size_t tc_dep_pairs(int max_rows, int G) { return static_cast<size_t>((max_rows + kBM - 1) / kBM + G); }
+// m-tiles a launch can have: every group's rows rounded up to 128.
+static int max_mtiles_of(int max_rows, int G) { return (max_rows + kBM - 1) / kBM + G; }
+size_t tc_dep_pairs(int max_rows, int G) { return static_cast<size_t>(max_mtiles_of(max_rows, G)) * kMaxSplit; }
 
 namespace {
 
@@ -830,63 +908,42 @@ TcShape make_shape(int N, int K, int BN) {
   return t;
 }
 
-// Cost model, in microseconds of one SM: a stage costs the larger of a
-// fixed ring round trip (~0.31 us) and its bytes at ~150 GB/s; a unit adds
-// 1.5 us of pipeline fill and epilogue; a split unit adds its fp32 partial
-// round trip (split_cost x a 256-wide stage x BN / 256).
-float stage_us(const TcShape& t) { return std::max(0.31f, t.stage_bytes / 150000.0f); }
-float unit_us(const TcShape& t, int S, float split_cost) {
-  return ((t.KB + S - 1) / S) * stage_us(t) + 1.5f + (S > 1 ? split_cost * 0.33f * t.BN / 256.0f : 0.0f);
-}
-
-// Busiest CTA's time when U0 units of time t0 precede U1 units of time t1,
-// dealt round-robin over the grid.
-float makespan(int U0, float t0, int U1, float t1, int grid) {
-  const int U = U0 + U1, r0 = U0 % grid, rt = U % grid;
-  float worst = 0.0f;
-  for (int b : {0, std::min(r0, rt), std::max(r0, rt)}) {
-    if (b >= grid) continue;
-    const int n0 = U0 / grid + (b < r0), nt = U / grid + (b < rt);
-    worst = std::max(worst, n0 * t0 + (nt - n0) * t1);
+// Tile-width choice: the widest candidate that still yields at least half
+// a wave of tiles (wider tiles re-read the 128 activation rows fewer times
+// per weight byte; too few tiles leave SMs idle), else the narrowest.
+// Measured on the 12-layer D768 stack at ~60% reuse (16 m-tiles, one
+// fused launch): phase-2 width 128 took 51 us, 64 took 59 us, and 256
+// (48 tiles) 56 us with two K splits.  K splits are used only when forced:
+// their parked partials and reductions cost 4-9 us of epilogue per unit.
+int pick_width(const TcShape* shp, int mt, int grid, int force_bn) {
+  int last = -1;
+  for (int i = 0; i < 3; ++i) {
+    if (!shp[i].BN || (force_bn && shp[i].BN != force_bn)) continue;
+    if (2 * mt * shp[i].nt >= grid) return i;
+    last = i;
   }
-  return worst;
+  return last < 0 ? 0 : last;  // forced width absent: the widest
 }
 
 // Plan for `mt` m-tiles: fused (section 0) or one phase alone (section 1 + p).
-int best_plan(const TcPlan* p, int section, int mt, int force_bn, int force_split, float split_cost) {
+// A fused launch splits phase 2 along K only when the split boundaries fall
+// on phase-1 tile and stage boundaries.
+int best_plan(const TcPlan* p, int section, int mt, int force_bn, int force_split) {
   const int grid = p->n_sms;
   const int max_units = static_cast<int>(tc_split_units(grid));
-  float best = 3.0e38f;
-  int word = plan_word(0, 0, 1);
   if (section == 0) {
-    for (int i0 = 0; i0 < 3; ++i0)
-      for (int i1 = 0; i1 < 3; ++i1) {
-        const TcShape &a0 = p->shp[0][i0], &a1 = p->shp[1][i1];
-        if (!a0.BN || !a1.BN || (force_bn && (a0.BN != force_bn || a1.BN != force_bn))) continue;
-        const float c = makespan(mt * a0.nt, unit_us(a0, 1, 0.0f), mt * a1.nt, unit_us(a1, 1, 0.0f), grid);
-        if (c < best - 1e-3f) {
-          best = c;
-          word = plan_word(i0, i1, 1);
-        }
-      }
-    return word;
+    const int i0 = pick_width(p->shp[0], mt, grid, force_bn), i1 = pick_width(p->shp[1], mt, grid, force_bn);
+    const TcShape &a0 = p->shp[0][i0], &a1 = p->shp[1][i1];
+    int S = force_split > 1 ? force_split : 1;
+    if (S > 1 && (a0.nt % S || a1.KB % S || mt * a1.nt * S > max_units)) S = 1;
+    return plan_word(i0, i1, S);
   }
   const int ph = section - 1;
-  for (int bi = 0; bi < 3; ++bi) {
-    const TcShape& t = p->shp[ph][bi];
-    if (!t.BN || (force_bn && t.BN != force_bn)) continue;
-    for (int S = 1; S <= kMaxSplit && S <= t.KB; ++S) {
-      if (force_split && S != force_split) continue;
-      const int tiles = mt * t.nt;
-      if (S > 1 && tiles * S > max_units) break;
-      const float c = static_cast<float>((tiles * S + grid - 1) / grid) * unit_us(t, S, split_cost);
-      if (c < best - 1e-3f) {
-        best = c;
-        word = ph == 0 ? plan_word(bi, 0, S) : plan_word(0, bi, S);
-      }
-    }
-  }
-  return word;
+  const int bi = pick_width(p->shp[ph], mt, grid, force_bn);
+  const TcShape& t = p->shp[ph][bi];
+  int S = force_split > 1 ? force_split : 1;
+  if (S > 1 && (S > t.KB || mt * t.nt * S > max_units)) S = 1;
+  return ph == 0 ? plan_word(bi, 0, S) : plan_word(0, bi, S);
 }
 
 bool encode_phase(TcMaps* m, const int* bn, const void* a_base, uint64_t rows, uint64_t K, const void* w,
@@ -928,14 +985,12 @@ TcPlan* tc_plan_create(const FfnArgs& a, int n_sms, char* err, int errlen) {
       p->shp[1][i] = make_shape(a.D, a.F, p->bn2[i]);
     }
     // One plan per possible m-tile count, for the fused launch and for each
-    // phase alone.  Split units cost a partial round trip that rarely pays
-    // (measured), hence the large split cost; forced values bypass it.
-    const float split_cost = 40.0f;
-    p->tab_n = std::min(static_cast<int>(tc_dep_pairs(a.max_rows, a.G)) + 1, kPlanTab);
+    // phase alone.
+    p->tab_n = std::min(max_mtiles_of(a.max_rows, a.G) + 1, kPlanTab);
     std::vector<int> tab(3 * static_cast<size_t>(p->tab_n));
     for (int sec = 0; sec < 3; ++sec)
       for (int mt = 0; mt < p->tab_n; ++mt)
-        tab[sec * p->tab_n + mt] = best_plan(p, sec, mt, a.tile_n, a.split_k, split_cost);
+        tab[sec * p->tab_n + mt] = best_plan(p, sec, mt, a.tile_n, a.split_k);
     if (cudaMalloc(&p->d_tab, tab.size() * sizeof(int)) != cudaSuccess ||
         cudaMemcpy(p->d_tab, tab.data(), tab.size() * sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess) {
       cudaGetLastError();
@@ -968,9 +1023,8 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
   t.k = a.k;
   t.T = a.T;
   t.gelu_tanh = a.gelu_tanh;
-  // phase 0: both phases in one launch, unless K splits are forced (they
-  // need single-phase launches) or there is no dependency workspace.
-  const bool fuse = phase == 0 && a.dep && p->force_split <= 1;
+  // phase 0: both phases in one launch (two, without a dependency workspace).
+  const bool fuse = phase == 0 && a.dep;
   if (phase == 0 && !fuse) {
     cudaError_t e = launch_ffn_tc(p, a, 1, s);
     return e != cudaSuccess ? e : launch_ffn_tc(p, a, 2, s);
@@ -992,7 +1046,8 @@ cudaError_t launch_ffn_tc(TcPlan* p, const FfnArgs& a, int phase, cudaStream_t s
   t.partial = a.partial;
   t.tile_sem = a.tile_sem;
   t.dep = a.dep;
-  t.max_mtiles = a.max_mtiles;
+  t.dep_pairs = a.max_mtiles;
+  t.work = a.work;
   t.status = a.status;
   TcMapPair maps;
   maps.p[0] = p->p1;

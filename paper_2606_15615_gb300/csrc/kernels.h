@@ -108,6 +108,7 @@ struct FfnArgs {
   int* tile_sem;         // split-K arrival counters, zeroed once
   int* dep;              // tensor-core fused launch: per m-tile counter pairs, zeroed once (or null)
   int max_mtiles;        // capacity of dep, tc_dep_pairs(max_rows, G)
+  int* work;             // tensor-core path: unit ticket counter pair, zeroed once
   int* status;
 };
 cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s);

@@ -79,6 +79,7 @@ struct moeca_handle {
   float* tc_partial = nullptr;
   int* tc_sem = nullptr;
   int* tc_dep = nullptr;        // fused GEMM launch: m-tile dependency counters, left at 0
+  int* tc_work = nullptr;       // GEMM unit tickets {next, CTAs done}, left at 0
   int tc_dep_pairs_n = 0;
   PrepShape prep{0, 0, 0, 0};   // fused router + select + compact, when it fits
   unsigned prep_arrivals = 0;   // grid-barrier arrivals of all fused launches so far (mod 2^32)
@@ -315,6 +316,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     A((void**)&h->tc_sem, tc_split_units(h->n_sms) * sizeof(int));
     h->tc_dep_pairs_n = static_cast<int>(tc_dep_pairs(h->max_rows, h->G));
     A((void**)&h->tc_dep, static_cast<size_t>(h->tc_dep_pairs_n) * 2 * sizeof(int));
+    A((void**)&h->tc_work, 2 * sizeof(int));
     h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
@@ -455,8 +457,8 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
     fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
     fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
-    fa.dep = h->tc_dep; fa.max_mtiles = h->tc_dep_pairs_n;
-    if (use_tc && c.ffn_split_k <= 1) {
+    fa.dep = h->tc_dep; fa.max_mtiles = h->tc_dep_pairs_n; fa.work = h->tc_work;
+    if (use_tc) {
       // Both GEMMs in one persistent launch: phase-2 tiles start as soon as
       // the phase-1 tiles of their rows are stored.
       e = timed(h, MOECA_K_FFN, s, [&] { return launch_ffn_tc(L.tc, fa, 0, s); });
@@ -616,6 +618,7 @@ moeca_status moeca_reset(moeca_handle* h) {
   if (h->tc_dep) {
     cudaError_t e = cudaMemset(h->tc_dep, 0, static_cast<size_t>(h->tc_dep_pairs_n) * 2 * sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(h->tc_sem, 0, tc_split_units(h->n_sms) * sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(h->tc_work, 0, 2 * sizeof(int));
     if (e != cudaSuccess) return cuda_fail(h, e, "reset GEMM counters");
   }
   for (auto& L : h->layers) {
