@@ -123,7 +123,6 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __shared__ float sm_cn[TB * KMAX];
   __shared__ float sm_ema[TB * EPAD];
 
-  pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int E = a.E, k = a.k, D = a.D, T = a.T;
   const int ldw = D + 8;  // padded row, in bf16
@@ -134,6 +133,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   const int ntok = min(TB, T - tok0);
 
   // ---- A0: stage gate rows and token rows ----
+  // Before the programmatic-dependency wait: everything that the previous
+  // kernel (the layer below's combine) does not write.  The gate matrix is a
+  // weight; the cached metadata and the EMA rows were last written by this
+  // layer's own kernels one step earlier, which completed before the
+  // previous kernel could start.
   if (t == 0) {
     sm_near = 0;
     sm_nrows = 0;
@@ -146,10 +150,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   if (t == 0) {
     mbar_expect_tx(bar, row_bytes * (E + ntok));
     const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
-    const __nv_bfloat16* x = static_cast<const __nv_bfloat16*>(a.x);
     for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
-    for (int q = 0; q < ntok; ++q)
-      bulk_g2s(smem_u32(s_x + q * ldw), x + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
   }
   // Prefetch what later phases read: cached metadata and EMA rows.
   {
@@ -171,6 +172,12 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   for (int idx = t; idx < (TB - ntok) * (D / 8); idx += kThreads) {
     const int r = ntok + idx / (D / 8), c = idx % (D / 8);
     reinterpret_cast<uint4*>(s_x + r * ldw)[c] = make_uint4(0, 0, 0, 0);
+  }
+  pdl_entry();
+  if (t == 0) {
+    const __nv_bfloat16* x = static_cast<const __nv_bfloat16*>(a.x);
+    for (int q = 0; q < ntok; ++q)
+      bulk_g2s(smem_u32(s_x + q * ldw), x + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
   }
   if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);
   __syncthreads();
@@ -369,7 +376,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       sm_H[t] = Ss > 0.f ? logf(Ss) - Us / Ss : 0.f;
     }
     __syncthreads();
-    if (t == 0) {
+    if (t == 0 && a.entropy_norm != 0) {  // min-max normalisation only
       float lo = 0.f, hi = 0.f;
       bool any = false;
       for (int ee = 0; ee < E; ++ee) {
@@ -449,7 +456,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   // ---- C: group offsets, this block's prefix, row lists and row gather ----
   {
     const int nb = gridDim.x;
-    int* s_cnt = reinterpret_cast<int*>(dyn);  // [nb][GG], reusing the staging area
+    int* s_cnt = reinterpret_cast<int*>(s_logit);  // [nb][GG], after the staged rows (the logits are done)
     {
       // All loads in flight before any store.
       constexpr int kU = 8;
@@ -468,24 +475,59 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       }
     }
     __syncthreads();
-    for (int g = t; g < GG; g += kThreads) {
+    // Per group: rows of the blocks before this one and of all blocks.  Each
+    // group's sum is split over kThreads / GG threads (block ranges), whose
+    // parts are then added in range order.
+    {
+      const int R = GG <= kThreads ? kThreads / GG : 1;
+      const int g = t % GG, j = t / GG;
       int pre = 0, tot = 0;
-      for (int b = 0; b < nb; ++b) {
-        const int c = s_cnt[b * GG + g];
-        if (b < static_cast<int>(blockIdx.x)) pre += c;
-        tot += c;
+      if (j < R && t < R * GG) {
+        const int b0 = j * nb / R, b1 = (j + 1) * nb / R;
+        for (int b = b0; b < b1; ++b) {
+          const int c = s_cnt[b * GG + g];
+          if (b < static_cast<int>(blockIdx.x)) pre += c;
+          tot += c;
+        }
       }
-      sm_pre[g] = pre;
-      sm_tot[g] = tot;
+      sm_rs[t][0] = __int_as_float(pre);
+      sm_rs[t][1] = __int_as_float(tot);
+      __syncthreads();
+      for (int gg = t; gg < GG; gg += kThreads) {
+        int p2 = 0, t2 = 0;
+        if (R * GG <= kThreads) {
+          for (int jj = 0; jj < R; ++jj) {
+            p2 += __float_as_int(sm_rs[jj * GG + gg][0]);
+            t2 += __float_as_int(sm_rs[jj * GG + gg][1]);
+          }
+        } else {  // more groups than threads: plain loop over blocks
+          for (int b = 0; b < nb; ++b) {
+            const int c = s_cnt[b * GG + gg];
+            if (b < static_cast<int>(blockIdx.x)) p2 += c;
+            t2 += c;
+          }
+        }
+        sm_pre[gg] = p2;
+        sm_tot[gg] = t2;
+      }
     }
     __syncthreads();
-    if (t == 0) {
-      int off = 0;
-      for (int g = 0; g < GG; ++g) {
-        sm_off[g] = off;
-        off += sm_tot[g];
+    if (warp == 0) {
+      // Exclusive scan of the group totals into offsets, 32 groups at a time.
+      int carry = 0;
+      for (int g0 = 0; g0 < GG; g0 += 32) {
+        const int g = g0 + lane;
+        const int v = g < GG ? sm_tot[g] : 0;
+        int incl = v;
+#pragma unroll
+        for (int dd = 1; dd < 32; dd <<= 1) {
+          const int u = __shfl_up_sync(0xffffffffu, incl, dd);
+          if (lane >= dd) incl += u;
+        }
+        if (g < GG) sm_off[g] = carry + incl - v;
+        carry += __shfl_sync(0xffffffffu, incl, 31);
       }
-      sm_off[GG] = off;
+      if (lane == 0) sm_off[GG] = carry;
     }
     __syncthreads();
     if (blockIdx.x == 0) {
@@ -500,8 +542,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         if (d.rec[p]) {
           const int g = d.e[p];
           const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
-          const int sl = a.sel.slot[static_cast<size_t>(i) * k + p];
-          a.list[pos] = i * k + sl;
+          a.list[pos] = i * k + d.sl[p];
           const int r = atomicAdd(&sm_nrows, 1);
           sm_rows[r][0] = pos;
           sm_rows[r][1] = i;
@@ -516,29 +557,14 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       }
     }
     __syncthreads();
-    // Gather the rows' inputs, four rows per warp in flight.
+    // Gather the rows' inputs from the token rows staged in phase A.
     const int nv = D / 8;
-    const uint4* x = static_cast<const uint4*>(a.x);
     uint4* xg = static_cast<uint4*>(a.xg);
     const int n = sm_nrows;
-    for (int r0 = warp * 4; r0 < n; r0 += 16) {
-      for (int c0 = 0; c0 < nv; c0 += 32 * 4) {
-        uint4 v[4][4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int c = c0 + q * 32 + lane;
-            if (r0 + j < n && c < nv) v[j][q] = x[static_cast<size_t>(sm_rows[r0 + j][1]) * nv + c];
-          }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int c = c0 + q * 32 + lane;
-            if (r0 + j < n && c < nv) xg[static_cast<size_t>(sm_rows[r0 + j][0]) * nv + c] = v[j][q];
-          }
-      }
+    for (int r = warp; r < n; r += kThreads / 32) {
+      const uint4* src = reinterpret_cast<const uint4*>(s_x + (sm_rows[r][1] - tok0) * ldw);
+      uint4* dst = xg + static_cast<size_t>(sm_rows[r][0]) * nv;
+      for (int c = lane; c < nv; c += 32) dst[c] = src[c];
     }
   }
 }
@@ -546,9 +572,10 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
 template <int TB, int EPAD>
 size_t prep_smem(int D, int n_blocks, int G) {
   const size_t ldw = static_cast<size_t>(D) + 8;
-  const size_t stage = (EPAD + TB) * ldw * 2 + static_cast<size_t>(TB) * (EPAD + 1) * 4;
-  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;
-  return stage > counts ? stage : counts;
+  const size_t rows = (EPAD + TB) * ldw * 2;                        // gate rows, token rows
+  const size_t logits = static_cast<size_t>(TB) * (EPAD + 1) * 4;    // phase A
+  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;       // phase C, same place
+  return rows + (logits > counts ? logits : counts);
 }
 
 template <int TB, int EPAD, int KMAX>

@@ -19,6 +19,7 @@ namespace moeca {
 template <int KMAX>
 struct TokenDecisionT {
   int e[KMAX];
+  int sl[KMAX];  // cache slot of each branch (valid tokens)
   bool rec[KMAX];
   bool any, bad, shared_row;
   int n_matched, n_rec, n_near;
@@ -43,6 +44,7 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
   for (int p = 0; p < KMAX; ++p) {
     e[p] = -1;
     rec[p] = false;
+    d.sl[p] = p;
   }
   if (valid) {
     const size_t base = static_cast<size_t>(i) * k;
@@ -130,6 +132,7 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
           n_rec += rec[p];
           a.recompute[base + p] = rec[p];
           a.slot[base + p] = static_cast<int8_t>(sl[p]);
+          d.sl[p] = sl[p];
           a.matched[base + p] = mat[p];
           if (rec[p]) {
             a.cache_e[base + sl[p]] = e[p];
