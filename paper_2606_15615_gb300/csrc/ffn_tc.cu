@@ -512,56 +512,88 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
       }
       if (lane == 0) {
+        // Issue one stage: its weight half (B) and/or activation half (A).
+        // A stage issued without A gets its A half later into the same slot
+        // (the barrier already expects the whole stage).
+        auto issue = [&](int kb, bool with_a, bool with_b, int slot) {
+          uint8_t* sa = smem + slot * sh.stage_bytes;
+          uint8_t* sb = sa + sh.sub * kABytes;
+          const uint32_t fb = smem_u32(&full_bar[t.p][slot]);
+          for (int j = 0; j < sh.sub; ++j) {
+            const int x = (kb * sh.sub + j) * kBK;
+            if (with_a) {
+              if (gather) {
+#pragma unroll 4
+                for (int q = 0; q < kBM / 4; ++q)
+                  tma_gather4(smem_u32(sa + j * kABytes + q * 512), ta, x, rows_sh[4 * q], rows_sh[4 * q + 1],
+                              rows_sh[4 * q + 2], rows_sh[4 * q + 3], fb);
+              } else {
+                tma_load_2d(smem_u32(sa + j * kABytes), ta, x, arow, fb);
+              }
+            }
+            if (with_b) tma_load_2d(smem_u32(sb + j * sh.BN * kBK * 2), tb, x, brow, fb);
+          }
+        };
+        // Claim the next slot for a new stage: wait until it is free (and, on a
+        // second-phase slot's first use, until the first-phase stages it
+        // overlaps are consumed), arm its barrier for the whole stage.
+        auto claim = [&]() -> bool {
+          if (fused && t.p == 1 && !((used >> sl) & 1u)) {
+            const int lo = sl * s1.stage_bytes / s0.stage_bytes;
+            const int hi = min(((sl + 1) * s1.stage_bytes - 1) / s0.stage_bytes, s0.nst - 1);
+            for (int q = lo; q <= hi; ++q)
+              if (((used0 >> q) & 1u) &&
+                  !mbar_wait(smem_u32(&empty_bar[0][q]), ((par0 >> q) & 1u) ^ 1u, &abort_flag))
+                return false;
+          }
+          if (!mbar_wait(smem_u32(&empty_bar[t.p][sl]), ((par >> sl) & 1u) ^ 1u, &abort_flag)) return false;
+          mbar_expect_tx(smem_u32(&full_bar[t.p][sl]), sh.stage_bytes);
+          return true;
+        };
+        auto advance = [&]() {
+          par ^= 1u << sl;
+          used |= 1u << sl;
+          if (t.p == 0) ++issued0;
+          sl = sl + 1 == sh.nst ? 0 : sl + 1;
+        };
+        int pre = 0;
         if (fused && t.p == 1) {
           // The m-tile's hidden rows come from every phase-1 tile of it, stored
           // by other CTAs' epilogues with generic stores and read here by TMA.
+          // While they are not all there, the weight halves of the first
+          // stages (which do not depend on them) are already on their way.
           int* d = a.dep + 2 * (t.mi * kMaxSplit + t.sp);
-          if (!wait_count(d, gq, &abort_flag)) {
-            ok = false;
-          } else {
+          const int sl_pre = sl;
+          if (ld_acquire(d) < gq) {
+            const int P = min(sh.nst, kb1 - kb0);
+            for (; pre < P && ok; ++pre) {
+              ok = claim();
+              if (ok) {
+                issue(kb0 + pre, false, true, sl);
+                advance();
+              }
+            }
+          }
+          if (ok && !wait_count(d, gq, &abort_flag)) ok = false;
+          if (ok) {
             asm volatile("fence.proxy.async.global;" ::: "memory");
             // The last phase-2 unit to start on this m-tile re-arms its counters.
             if (atomicAdd(d + 1, 1) == s1.nt - 1) {
               d[0] = 0;
               d[1] = 0;
             }
+            for (int j = 0; j < pre; ++j) {
+              const int slot = (sl_pre + j) % sh.nst;
+              issue(kb0 + j, true, false, slot);
+            }
           }
         }
-        for (int kb = kb0; kb < kb1 && ok; ++kb) {
-          if (fused && t.p == 1 && !((used >> sl) & 1u)) {
-            // First use of this second-phase slot: wait until the first-phase
-            // stages it overlaps have been consumed by their MMAs.
-            const int lo = sl * s1.stage_bytes / s0.stage_bytes;
-            const int hi = min(((sl + 1) * s1.stage_bytes - 1) / s0.stage_bytes, s0.nst - 1);
-            for (int q = lo; q <= hi && ok; ++q)
-              if ((used0 >> q) & 1u)
-                ok = mbar_wait(smem_u32(&empty_bar[0][q]), ((par0 >> q) & 1u) ^ 1u, &abort_flag);
-            if (!ok) break;
+        for (int kb = kb0 + pre; kb < kb1 && ok; ++kb) {
+          ok = claim();
+          if (ok) {
+            issue(kb, true, true, sl);
+            advance();
           }
-          if (!mbar_wait(smem_u32(&empty_bar[t.p][sl]), ((par >> sl) & 1u) ^ 1u, &abort_flag)) {
-            ok = false;
-            break;
-          }
-          const uint32_t fb = smem_u32(&full_bar[t.p][sl]);
-          mbar_expect_tx(fb, sh.stage_bytes);
-          uint8_t* sa = smem + sl * sh.stage_bytes;
-          uint8_t* sb = sa + sh.sub * kABytes;
-          for (int j = 0; j < sh.sub; ++j) {
-            const int x = (kb * sh.sub + j) * kBK;
-            if (gather) {
-#pragma unroll 4
-              for (int q = 0; q < kBM / 4; ++q)
-                tma_gather4(smem_u32(sa + j * kABytes + q * 512), ta, x, rows_sh[4 * q], rows_sh[4 * q + 1],
-                            rows_sh[4 * q + 2], rows_sh[4 * q + 3], fb);
-            } else {
-              tma_load_2d(smem_u32(sa + j * kABytes), ta, x, arow, fb);
-            }
-            tma_load_2d(smem_u32(sb + j * sh.BN * kBK * 2), tb, x, brow, fb);
-          }
-          par ^= 1u << sl;
-          used |= 1u << sl;
-          if (t.p == 0) ++issued0;
-          sl = sl + 1 == sh.nst ? 0 : sl + 1;
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
