@@ -63,6 +63,8 @@ class Params:
     shared_policy: str = "sync"        # or "always"
     reused_meta_policy: str = "keep"   # or "overwrite"
     gelu: str = "tanh"                 # or "erf"
+    score_terms: int = 7               # Eq. 9 terms kept: 1 = w, 2 = lambda1 Delta, 4 = lambda2 o (Table 5)
+    granularity: str = "branch"        # or "token": a token's k branches share one decision
 
 
 # ---------------------------------------------------------------------------
@@ -205,13 +207,21 @@ def historical_contribution(cache_norm: np.ndarray) -> np.ndarray:
 
 
 def select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, lambda1, lambda2,
-                    refresh: bool):
+                    refresh: bool, score_terms: int = 7, granularity: str = "branch"):
     """Partition B_i^t into the recompute set R_i^t and the reuse set.
+
+    Eq. 9 scores a matched branch with s = w + lambda1 Delta + lambda2 o;
+    `score_terms` keeps a subset of the three terms (the signal ablation of
+    Table 5: bit 1 = w, 2 = lambda1 Delta, 4 = lambda2 o).  With granularity
+    "token", a token's k branches share one decision, as in token-level
+    caching (Sec. 3): all of them are recomputed when the branch rule would
+    recompute any of them, else all are reused.
 
     Returns a dict of [T, k] arrays:
       recompute (bool), slot (int32: cache slot that holds branch p after the
       step), matched (bool), score (float64, NaN if unmatched) and margin
-      (|s - tau| / |tau|, inf where no threshold decides).
+      (|s - tau| / |tau|, inf where no threshold decides; in token mode the
+      smallest margin of the token, which decides all its branches).
     """
     e_cur = np.asarray(e_cur)
     T, k = e_cur.shape
@@ -236,12 +246,18 @@ def select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, lambda1, la
             matched[i, p] = True
             w = float(w_cur[i, p])
             delta = abs(w - float(cache_w[i, q]))
-            s = w + lambda1 * delta + lambda2 * float(o[i, q])
+            s = ((w if score_terms & 1 else 0.0)
+                 + (lambda1 * delta if score_terms & 2 else 0.0)
+                 + (lambda2 * float(o[i, q]) if score_terms & 4 else 0.0))
             score[i, p] = s
             t = float(tau[e])
             recompute[i, p] = bool(np.float32(s) > np.float32(t))
             if math.isfinite(t):
                 margin[i, p] = abs(s - t) / max(abs(t), _TINY)
+        if granularity == "token":
+            if recompute[i].any():
+                recompute[i, :] = True
+            margin[i, :] = margin[i].min()
         # Matched branches keep their slot; unmatched ones take the freed slots.
         free = [q for q in range(k) if q not in q_of]
         unmatched = [p for p in range(k) if q_of[p] < 0]
@@ -350,7 +366,7 @@ def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, ref
     Hbar = normalized_entropy(C, prm.entropy_norm)
     tau = expert_threshold(Hbar, prm.tau0, prm.alpha)
     sel = select_branches(e_cur, w_cur, state.cache_e, state.cache_w, state.cache_norm, tau,
-                          prm.lambda1, prm.lambda2, refresh)
+                          prm.lambda1, prm.lambda2, refresh, prm.score_terms, prm.granularity)
     out, new, token_any = recompute_and_combine(state, u, e_cur, w_cur, sel["recompute"], sel["slot"],
                                                 weights, prm, refresh)
     new.C = C

@@ -108,8 +108,17 @@ def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool):
                 taken.append(q_hit)
                 delta = abs(w_cur[i][p] - state["cache_w"][i][q_hit])
                 o = norms[q_hit] / tot if tot > 0.0 else 0.0
-                s = w_cur[i][p] + prm["lambda1"] * delta + prm["lambda2"] * o
+                terms = prm.get("score_terms", 7)
+                s = 0.0
+                if terms & 1:
+                    s += w_cur[i][p]
+                if terms & 2:
+                    s += prm["lambda1"] * delta
+                if terms & 4:
+                    s += prm["lambda2"] * o
                 rec[i][p] = _f32(s) > _f32(tau[e_cur[i][p]])
+            if prm.get("granularity", "branch") == "token" and True in rec[i]:
+                rec[i] = [True] * k
             free = [q for q in range(k) if q not in taken]
             for p in range(k):
                 if taken[p] is not None:

@@ -23,6 +23,15 @@ CASES = [
     (7, 5, 4, 4, 4, 3, 0, False, {"gelu": "erf"}),
     (8, 8, 6, 4, 2, 5, 0, False, {"renorm_topk": False, "tau0": 0.5}),
     (9, 1, 4, 3, 2, 3, 0, False, {}),
+    # Table 5's score-signal subsets and token-level granularity (Sec. 3)
+    (10, 8, 6, 4, 2, 5, 0, False, {"score_terms": 1, "tau0": 0.55}),
+    (11, 8, 6, 4, 2, 5, 0, False, {"score_terms": 2, "tau0": 0.08}),
+    (18, 8, 6, 4, 2, 5, 0, False, {"score_terms": 4, "tau0": 0.25}),
+    (13, 8, 6, 4, 2, 5, 0, False, {"score_terms": 3, "tau0": 0.6}),
+    (14, 8, 6, 4, 2, 5, 0, False, {"score_terms": 5, "tau0": 0.75}),
+    (15, 8, 6, 4, 2, 5, 0, False, {"score_terms": 6, "tau0": 0.3}),
+    (16, 8, 6, 4, 2, 5, 1, False, {"granularity": "token", "tau0": 1.1}),
+    (17, 8, 5, 4, 3, 4, 0, True, {"granularity": "token", "score_terms": 3, "tau0": 0.9}),
 ]
 
 
@@ -30,7 +39,8 @@ def _bf_params(prm: O.Params) -> dict:
     return dict(top_k=prm.top_k, lambda1=prm.lambda1, lambda2=prm.lambda2, tau0=prm.tau0,
                 alpha=prm.alpha, beta=prm.beta, renorm_topk=prm.renorm_topk,
                 entropy_norm=prm.entropy_norm, shared_policy=prm.shared_policy,
-                reused_meta_policy=prm.reused_meta_policy, gelu=prm.gelu)
+                reused_meta_policy=prm.reused_meta_policy, gelu=prm.gelu, score_terms=prm.score_terms,
+                granularity=prm.granularity)
 
 
 @pytest.mark.parametrize("case", CASES, ids=[f"case{c[0]}" for c in CASES])

@@ -264,3 +264,75 @@ def test_refresh_schedule():
     assert flags == [True, False, False, True, False, False, True]
     assert st.step(x[:5], 7)[1][0]["refresh"], "a new token count forces a full step"
     assert st.step(x[:5], 8, force=True)[1][0]["refresh"]
+
+
+def _random_selection_inputs(seed, T=64, k=3, E=6):
+    rng = np.random.default_rng(seed)
+    e_cur = np.stack([rng.permutation(E)[:k] for _ in range(T)])
+    w_cur = rng.dirichlet(np.ones(k), size=T)
+    # Caches that share some experts with the current routing.
+    cache_e = np.stack([rng.permutation(E)[:k] for _ in range(T)])
+    cache_e[: T // 2] = e_cur[: T // 2][:, rng.permutation(k)]
+    cache_w = rng.dirichlet(np.ones(k), size=T)
+    cache_norm = rng.uniform(0.1, 2.0, size=(T, k))
+    tau = rng.uniform(0.3, 0.9, size=E)
+    return e_cur, w_cur, cache_e, cache_w, cache_norm, tau
+
+
+@pytest.mark.parametrize("terms", [1, 2, 4, 3, 5, 6, 7])
+def test_score_subsets_follow_table5_terms(terms):
+    """Each subset scores a matched branch with exactly its terms (Eq. 9, Table 5)."""
+    e_cur, w_cur, cache_e, cache_w, cache_norm, tau = _random_selection_inputs(3)
+    l1, l2 = 0.7, 0.4
+    sel = O.select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, l1, l2, False, score_terms=terms)
+    T, k = e_cur.shape
+    checked = 0
+    for i in range(T):
+        for p in range(k):
+            hits = np.nonzero(cache_e[i] == e_cur[i, p])[0]
+            if hits.size == 0:
+                assert sel["recompute"][i, p] and not sel["matched"][i, p]
+                continue
+            q = hits[0]
+            w = w_cur[i, p]
+            parts = {1: w, 2: l1 * abs(w - cache_w[i, q]), 4: l2 * cache_norm[i, q] / cache_norm[i].sum()}
+            s = sum(v for bit, v in parts.items() if terms & bit)
+            assert sel["score"][i, p] == pytest.approx(s, rel=1e-12, abs=1e-15)
+            assert sel["recompute"][i, p] == (np.float32(s) > np.float32(tau[e_cur[i, p]]))
+            checked += 1
+    assert checked > 20
+
+
+def test_all_terms_equals_default_score():
+    args = _random_selection_inputs(4)
+    a = O.select_branches(*args, 1.0, 0.5, False)
+    b = O.select_branches(*args, 1.0, 0.5, False, score_terms=7, granularity="branch")
+    for key in ("recompute", "slot", "matched"):
+        assert np.array_equal(a[key], b[key])
+
+
+def test_token_granularity_is_the_or_of_branch_decisions():
+    """Token-level reuse (Sec. 3): a token's branches share one decision, which
+    recomputes all of them when any branch would be recomputed."""
+    e_cur, w_cur, cache_e, cache_w, cache_norm, _ = _random_selection_inputs(5)
+    args = (e_cur, w_cur, cache_e, cache_w, cache_norm, np.full(6, 1.0))
+    br = O.select_branches(*args, 1.0, 0.5, False)
+    tk = O.select_branches(*args, 1.0, 0.5, False, granularity="token")
+    anyr = br["recompute"].any(axis=1)
+    assert np.array_equal(tk["recompute"], np.repeat(anyr[:, None], br["recompute"].shape[1], axis=1))
+    assert np.array_equal(tk["slot"], br["slot"]) and np.array_equal(tk["matched"], br["matched"])
+    # Both kinds of token occur, so the rule is exercised.
+    assert anyr.any() and (~anyr).any()
+    # Every branch of a token carries the token's smallest margin.
+    assert np.array_equal(tk["margin"], np.repeat(br["margin"].min(axis=1)[:, None], 3, axis=1))
+
+
+def test_token_granularity_never_reuses_more_than_branch_granularity():
+    e_cur, w_cur, cache_e, cache_w, cache_norm, _ = _random_selection_inputs(6)
+    for tau0 in (0.2, 0.5, 0.8, 1.2):
+        tau = np.full(6, tau0)
+        br = O.select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, 1.0, 0.5, False)
+        tk = O.select_branches(e_cur, w_cur, cache_e, cache_w, cache_norm, tau, 1.0, 0.5, False,
+                               granularity="token")
+        assert tk["recompute"].sum() >= br["recompute"].sum()
+        assert np.all(tk["recompute"] | ~br["recompute"])
