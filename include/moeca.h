@@ -83,6 +83,11 @@ typedef struct {
   int32_t ffn_tile_n;         /* tensor-core FFN tile width: 0 = chosen per launch from the group
                                  sizes (default), else 64 / 128 / 192 / 256 where it divides N */
   int32_t ffn_split_k;        /* tensor-core FFN K splits: 0 = chosen per launch (default), else 1..4 */
+  int32_t score_terms;        /* Eq. 9 terms in the branch score, a bit mask (Table 5's signal
+                                 ablation): 1 = w, 2 = lambda1 Delta, 4 = lambda2 o; 7 (default) = all */
+  int32_t granularity;        /* 0: branch-level decisions (MoECa, default); 1: token-level, a
+                                 token's k branches share one decision: all are recomputed when
+                                 the branch rule would recompute any of them (Sec. 3) */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters

@@ -49,6 +49,8 @@ struct SelectArgs {
   int refresh;
   float lambda1, lambda2;
   int reused_meta_policy, shared_policy, n_shared;
+  int score_terms;      // Eq. 9 terms kept: 1 = w, 2 = lambda1 Delta, 4 = lambda2 o
+  int token_level;      // 1: a token's branches share one decision
   const int32_t* route_e;
   const float* route_w;
   const float* tau;

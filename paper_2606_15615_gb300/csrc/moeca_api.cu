@@ -198,6 +198,8 @@ void moeca_config_default(moeca_config* c) {
   c->entropy_norm = 0;
   c->shared_policy = 0;
   c->reused_meta_policy = 0;
+  c->score_terms = 7;
+  c->granularity = 0;
   c->gelu_tanh = 1;
   c->ffn_impl = MOECA_FFN_AUTO;
 }
@@ -240,6 +242,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "alpha and beta must be in [0, 1)");
   if (std::isnan(c.tau0) || !std::isfinite(c.lambda1) || !std::isfinite(c.lambda2))
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "tau0, lambda1, lambda2");
+  if (c.score_terms < 1 || c.score_terms > 7 || (c.granularity != 0 && c.granularity != 1))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "score_terms must be 1..7 and granularity 0 or 1");
   if (c.refresh_period < 0) return fail(nullptr, MOECA_ERR_INVALID_ARG, "refresh_period < 0");
   if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
@@ -416,6 +420,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     SelectArgs sa{};
     sa.T = T; sa.k = c.top_k; sa.E = c.n_experts; sa.G = h->G; sa.refresh = refresh;
     sa.lambda1 = c.lambda1; sa.lambda2 = c.lambda2;
+    sa.score_terms = c.score_terms; sa.token_level = c.granularity;
     sa.reused_meta_policy = c.reused_meta_policy; sa.shared_policy = c.shared_policy; sa.n_shared = c.n_shared;
     sa.route_e = L.route_e; sa.route_w = L.route_w; sa.tau = L.tau;
     sa.cache_e = L.cache_e; sa.cache_w = L.cache_w; sa.cache_norm = L.cache_norm;

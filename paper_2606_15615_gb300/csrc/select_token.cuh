@@ -101,7 +101,8 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
               if (qq == q) { cwq = cw[qq]; cnq = cn[qq]; }
             const float delta = fabsf(w[p] - cwq);
             const float o = nsum > 0.f ? cnq / nsum : 0.f;
-            const float s = w[p] + a.lambda1 * delta + a.lambda2 * o;
+            const float s = ((a.score_terms & 1) ? w[p] : 0.f) + ((a.score_terms & 2) ? a.lambda1 * delta : 0.f) +
+                            ((a.score_terms & 4) ? a.lambda2 * o : 0.f);
             const float tau = a.tau[e[p]];
             rec[p] = s > tau;
             if (isfinite(tau) && fabsf(s - tau) < 1e-5f * fabsf(tau)) ++n_near;
@@ -109,6 +110,14 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
             rec[p] = true;
           }
         }
+      }
+      if (a.token_level) {
+        // Token-level granularity: one decision for all of the token's branches.
+        bool anyr = false;
+#pragma unroll
+        for (int p = 0; p < KMAX; ++p) anyr |= (p < k) && rec[p];
+#pragma unroll
+        for (int p = 0; p < KMAX; ++p) rec[p] = (p < k) && anyr;
       }
 #pragma unroll
       for (int p = 0; p < KMAX; ++p) {

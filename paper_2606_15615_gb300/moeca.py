@@ -34,7 +34,7 @@ class moeca_config(C.Structure):
                 ("refresh_period", C.c_int32), ("renorm_topk", C.c_int32), ("entropy_norm", C.c_int32),
                 ("shared_policy", C.c_int32), ("reused_meta_policy", C.c_int32),
                 ("gelu_tanh", C.c_int32), ("ffn_impl", C.c_int32), ("ffn_tile_n", C.c_int32),
-                ("ffn_split_k", C.c_int32)]
+                ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):

@@ -60,7 +60,8 @@ def params_of(cfg) -> O.Params:
         entropy_norm="log_t" if cfg.entropy_norm == 0 else "minmax",
         shared_policy="sync" if cfg.shared_policy == 0 else "always",
         reused_meta_policy="keep" if cfg.reused_meta_policy == 0 else "overwrite",
-        gelu="tanh" if cfg.gelu_tanh else "erf")
+        gelu="tanh" if cfg.gelu_tanh else "erf", score_terms=cfg.score_terms,
+        granularity="branch" if cfg.granularity == 0 else "token")
 
 
 def oracle_weights(w: dict) -> dict:
@@ -140,7 +141,7 @@ def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
     # ---- select (Sec. 4.2, Eq. 9) from the GPU routing, tau and pre-step cache
     st_pre = state_to_oracle(pre, T, D, E, k, S)
     sel = O.select_branches(e_g, w_g, st_pre.cache_e, st_pre.cache_w, st_pre.cache_norm, tau_g,
-                            prm.lambda1, prm.lambda2, refresh)
+                            prm.lambda1, prm.lambda2, refresh, prm.score_terms, prm.granularity)
     rec_g = np_of(tr["recompute"]).astype(bool)
     slot_g = np_of(tr["slot"]).astype(np.int64)
     mat_g = np_of(tr["matched"]).astype(bool)

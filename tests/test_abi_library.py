@@ -29,6 +29,7 @@ def test_status_strings_and_defaults(lib):
     assert (cfg.lambda1, cfg.lambda2) == (1.0, 0.5)
     assert abs(cfg.tau0 - 0.8) < 1e-7 and abs(cfg.alpha - 0.6) < 1e-7 and abs(cfg.beta - 0.65) < 1e-7
     assert cfg.renorm_topk == 1 and cfg.gelu_tanh == 1 and cfg.dtype == lib.MOECA_BF16
+    assert cfg.score_terms == 7 and cfg.granularity == 0
 
 
 def test_host_validation_needs_no_gpu(lib):
@@ -43,6 +44,10 @@ def test_host_validation_needs_no_gpu(lib):
     cfg.alpha = 1.0
     assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # alpha outside [0, 1)
     cfg.alpha = 0.6
+    for bad in (dict(score_terms=0), dict(score_terms=8), dict(granularity=2)):
+        c2 = lib.moeca_config_default(n_layers=1, hidden=64, ffn=64, n_experts=4, top_k=2, max_tokens=8, **bad)
+        assert L.moeca_create(ctypes.byref(c2), w, 0, ctypes.byref(h)) == -1
+        assert b"score_terms" in L.moeca_last_error(None)
     assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # NULL weights
     cfg.hidden = 60
     w[0].w_gate = w[0].w1 = w[0].w2 = 4096

@@ -104,7 +104,11 @@ def test_bf16_fine_grained_64_experts_top8(M):
 
 @pytest.mark.parametrize("switch", [
     dict(entropy_norm=1), dict(reused_meta_policy=1), dict(shared_policy=1, n_shared=1),
-    dict(gelu_tanh=0), dict(renorm_topk=0, tau0=0.45)])
+    dict(gelu_tanh=0), dict(renorm_topk=0, tau0=0.45),
+    # Table 5's score-signal subsets and token-level granularity (Sec. 3)
+    dict(score_terms=1, tau0=0.55), dict(score_terms=2, tau0=0.05), dict(score_terms=4, tau0=0.25),
+    dict(score_terms=3, tau0=0.6), dict(score_terms=6, tau0=0.3), dict(granularity=1, tau0=0.9),
+    dict(granularity=1, score_terms=5, tau0=0.8)])
 def test_reading_switches(M, switch):
     sw = dict(switch)
     S = sw.pop("n_shared", 0)
