@@ -19,10 +19,12 @@ constexpr int kWarps = 8;
 template <typename TI, int KMAX, int CG>
 __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
-  pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * kWarps + warp;
-  if (i >= a.T) return;
+  if (i >= a.T) {
+    pdl_entry();
+    return;
+  }
   const int k = a.k, D = a.D, nvec = D / V;
   const TI* x = static_cast<const TI*>(a.x) + static_cast<size_t>(i) * D;
   TI* out = static_cast<TI*>(a.out) + static_cast<size_t>(i) * D;
@@ -41,6 +43,18 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
       if (q[p] < 0 || q[p] >= k) bad = true;
     }
   }
+  // The gate weights, slots and layer input come from earlier kernels than
+  // the one before (prep, the layer below's combine); only the cache rows
+  // (and shared rows) are the previous kernel's output.  Load the first
+  // input chunks, then wait.
+  const uint4* x4 = reinterpret_cast<const uint4*>(x);
+  uint4 x_first[CG];
+#pragma unroll
+  for (int g = 0; g < CG; ++g) {
+    const int c = g * 32 + lane;
+    if (c < nvec) x_first[g] = x4[c];
+  }
+  pdl_entry();
   if (bad) {
     if (lane == 0) report_status(a.status, kStatusBadIndex, 3000000 + i);
     return;
@@ -50,7 +64,6 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   for (int p = 0; p < KMAX; ++p) ss[p] = 0.f;
   // Raw 16-byte vectors stay packed in registers until used.
   const uint4* ch4 = reinterpret_cast<const uint4*>(ch);
-  const uint4* x4 = reinterpret_cast<const uint4*>(x);
   const uint4* sh4 = reinterpret_cast<const uint4*>(sh);
   for (int c0 = 0; c0 < nvec; c0 += 32 * CG) {
     uint4 h[CG][KMAX], xr[CG], hr[CG];
@@ -61,7 +74,7 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
 #pragma unroll
         for (int p = 0; p < KMAX; ++p)
           if (p < k) h[g][p] = ch4[static_cast<size_t>(q[p]) * nvec + c];
-        xr[g] = x4[c];
+        xr[g] = c0 == 0 ? x_first[g] : x4[c];
         if (sh) hr[g] = sh4[c];
       }
     }
