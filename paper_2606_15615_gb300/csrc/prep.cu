@@ -592,9 +592,17 @@ cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
+  // A programmatic dependent launch, like every kernel of the step: the
+  // blocks start while the previous kernel drains and wait in
+  // griddepcontrol.wait.  (A cooperative launch would not start early.)  The
+  // grid barriers need every block resident: the plan keeps the grid within
+  // one block per SM's occupancy, the kernels before it never wait on it,
+  // and the kernel after it is launched only once every block has passed
+  // the wait, so all blocks are resident by the first barrier; the barrier
+  // waits are bounded regardless.
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD, KMAX>, a);
