@@ -25,6 +25,11 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
     pdl_entry();
     return;
   }
+  if (a.rearm && blockIdx.x == 0 && threadIdx.x == 0) {
+    // The grouped GEMM before this kernel has ended: re-arm its ticket.
+    pdl_entry();
+    *a.rearm = 0;
+  }
   const int k = a.k, D = a.D, nvec = D / V;
   const TI* x = static_cast<const TI*>(a.x) + static_cast<size_t>(i) * D;
   TI* out = static_cast<TI*>(a.out) + static_cast<size_t>(i) * D;

@@ -82,7 +82,8 @@ struct TcArgs {
   int* tile_sem;   // split-K arrival counters, [max_units], left at 0
   int* dep;        // fused launch: per (m-tile, phase-2 split) {phase-1 tiles stored, phase-2 units started}, left at 0
   int dep_pairs;   // capacity of dep (pairs); pair (mi, q) is at mi x 4 + q
-  int* work;       // {next unit ticket, CTAs done}, left at 0: units past the first go to whoever asks
+  int* work;       // next unit ticket (units past each CTA's first go to whoever asks); the kernel
+                   // after this one re-arms it to 0 (launch_ffn_tc's contract)
   int gather;      // phase 1: A rows gathered from the layer input by token (tile::gather4)
   int* status;
 };
@@ -848,15 +849,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
-  }
-  if (threadIdx.x == 0) {
-    // The last CTA out re-arms the unit counter (every CTA has taken its
-    // final ticket by now); the next launch reads it after this one ends.
-    __threadfence();
-    if (atomicAdd(a.work + 1, 1) == static_cast<int>(gridDim.x) - 1) {
-      a.work[0] = 0;
-      a.work[1] = 0;
-    }
   }
 }
 

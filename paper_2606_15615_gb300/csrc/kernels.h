@@ -110,7 +110,8 @@ struct FfnArgs {
   int* tile_sem;         // split-K arrival counters, zeroed once
   int* dep;              // tensor-core fused launch: per m-tile counter pairs, zeroed once (or null)
   int max_mtiles;        // capacity of dep, tc_dep_pairs(max_rows, G)
-  int* work;             // tensor-core path: unit ticket counter pair, zeroed once
+  int* work;             // tensor-core path: unit ticket counter; 0 before every launch (the combine
+                         // kernel that follows re-arms it)
   int* status;
 };
 cudaError_t launch_ffn_simt(const FfnArgs& a, bool bf16, int phase, cudaStream_t s);
@@ -171,6 +172,8 @@ struct CombineArgs {
   const float* route_w;   // [T, k]
   const int8_t* slot;     // [T, k]
   float* cache_norm;      // [T, k]
+  int* rearm;             // a counter the previous kernel leaves for re-arming (the GEMM's unit
+                          // ticket), set to 0 after the dependency wait, or null
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);

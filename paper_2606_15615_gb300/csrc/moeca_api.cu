@@ -481,6 +481,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
     cb.x = in; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
     cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
+    cb.rearm = use_tc ? h->tc_work : nullptr;
     if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
     L.valid = true;
   }
