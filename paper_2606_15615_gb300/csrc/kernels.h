@@ -84,7 +84,9 @@ struct CompactArgs {
   int32_t* list;        // [rows]
   const void* x;        // [T, D]
   void* xg;             // [rows, D] gathered inputs, or null when the GEMM gathers itself
+  int* status;
 };
+// compact_kernel (row lists), then, unless xg is null, gather_kernel (rows).
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s);
 
 // Grouped expert FFN over the compacted rows (Eq. 5 / Eq. 6 on R only).

@@ -434,7 +434,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ca.refresh = refresh; ca.shared_policy = c.shared_policy;
     ca.route_e = L.route_e; ca.recompute = L.recompute; ca.slot = L.slot; ca.token_any = L.token_any;
     ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
-    ca.x = in; ca.xg = (use_tc && kGemmGathersRows) ? nullptr : h->xg;
+    ca.x = in; ca.xg = (use_tc && kGemmGathersRows) ? nullptr : h->xg; ca.status = h->status_dev;
     if (fused) {
       PrepArgs pa{};
       pa.x = in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;

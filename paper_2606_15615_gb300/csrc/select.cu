@@ -13,9 +13,10 @@
 // The last block scans the per-block counts into per-group row offsets.
 //
 // compact_kernel, same token blocks: ranks each recomputed row inside its
-// group in ascending token order (ballot + popc prefix), writes the row list
-// (token * k + slot for routed experts, token for the shared expert) and
-// gathers the rows' layer inputs into a contiguous buffer for the GEMMs.
+// group in ascending token order (ballot + popc prefix) and writes the row
+// list (token * k + slot for routed experts, token for the shared expert).
+// gather_kernel then copies every listed row's layer input into a
+// contiguous buffer for the GEMMs, one warp per row over the whole list.
 #include "common.cuh"
 #include "kernels.h"
 #include "select_token.cuh"
@@ -166,9 +167,6 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
 
   __shared__ unsigned sm_bal[kWarps][kMaxGroups];
   __shared__ int sm_pre[kWarps][kMaxGroups];
-  __shared__ int sm_rows[kThreads * (kMaxTopK + 1)][2];
-  __shared__ int sm_nrows;
-  if (t == 0) sm_nrows = 0;
   for (int g = 0; g < G; ++g) {
     bool has = false;
     if (g < E) {
@@ -197,46 +195,44 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
       const int g = e[p];
       const int pos = sm_pre[warp][g] + __popc(sm_bal[warp][g] & lt);
       a.list[pos] = i * k + sl[p];
-      const int r = atomicAdd(&sm_nrows, 1);
-      sm_rows[r][0] = pos;
-      sm_rows[r][1] = i;
     }
   }
   if (shared_row) {
     const int pos = sm_pre[warp][E] + __popc(sm_bal[warp][E] & lt);
     a.list[pos] = i;
-    const int r = atomicAdd(&sm_nrows, 1);
-    sm_rows[r][0] = pos;
-    sm_rows[r][1] = i;
   }
-  __syncthreads();
-  // Gather the inputs of this block's rows, one warp per row, 16-byte vectors.
-  if (a.xg == nullptr) return;  // the tensor-core GEMM gathers its rows itself
+}
+
+// Gather of every listed row's layer input into the group-contiguous buffer
+// the GEMMs read: one warp per row over the whole list (rows of group g are
+// [offsets[g], offsets[g + 1])), 16-byte vectors.  A list entry is
+// token * k + slot for a routed group and the token for the shared group.
+template <typename TI>
+__global__ void __launch_bounds__(256) gather_kernel(CompactArgs a) {
+  pdl_entry();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = a.G, E = a.E;
+  const int rows = a.offsets[G];
   const int nv = a.D * static_cast<int>(sizeof(TI)) / 16;
   const uint4* x = static_cast<const uint4*>(a.x);
   uint4* xg = static_cast<uint4*>(a.xg);
-  // Four rows per warp at a time, every load issued before the stores.
-  const int n = sm_nrows;
-  for (int r0 = warp * 4; r0 < n; r0 += kWarps * 4) {
-    for (int c0 = 0; c0 < nv; c0 += 32 * 4) {
-      uint4 v[4][4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int c = c0 + q * 32 + lane;
-          if (r0 + j < n && c < nv) v[j][q] = x[static_cast<size_t>(sm_rows[r0 + j][1]) * nv + c];
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int c = c0 + q * 32 + lane;
-          if (r0 + j < n && c < nv) xg[static_cast<size_t>(sm_rows[r0 + j][0]) * nv + c] = v[j][q];
-        }
-      }
+  for (int r = blockIdx.x * 8 + warp; r < rows; r += gridDim.x * 8) {
+    // Group of row r: the last g with offsets[g] <= r (G <= 65: a short search).
+    int lo = 0, hi = G - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.offsets[mid] <= r) lo = mid;
+      else hi = mid - 1;
     }
+    const int ent = a.list[r];
+    const int tok = lo < E ? ent / a.k : ent;
+    if (tok < 0 || tok >= a.T) {
+      if (lane == 0) report_status(a.status, kStatusBadIndex, 5100000 + r);
+      continue;
+    }
+    const uint4* src = x + static_cast<size_t>(tok) * nv;
+    uint4* dst = xg + static_cast<size_t>(r) * nv;
+    for (int c = lane; c < nv; c += 32) dst[c] = src[c];
   }
 }
 
@@ -249,8 +245,14 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t s) {
 
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s) {
   const int grid = (a.T + kThreads - 1) / kThreads;
-  if (bf16) return launch_pdl(compact_kernel<__nv_bfloat16>, dim3(grid), dim3(kThreads), 0, s, a);
-  return launch_pdl(compact_kernel<float>, dim3(grid), dim3(kThreads), 0, s, a);
+  cudaError_t e = bf16 ? launch_pdl(compact_kernel<__nv_bfloat16>, dim3(grid), dim3(kThreads), 0, s, a)
+                       : launch_pdl(compact_kernel<float>, dim3(grid), dim3(kThreads), 0, s, a);
+  if (e != cudaSuccess || a.xg == nullptr) return e;
+  // The row gather runs over the whole list, one warp per row.
+  const int rows = a.T * (a.k + a.n_shared);
+  const int ggrid = (rows + 7) / 8;
+  return bf16 ? launch_pdl(gather_kernel<__nv_bfloat16>, dim3(ggrid), dim3(256), 0, s, a)
+              : launch_pdl(gather_kernel<float>, dim3(ggrid), dim3(256), 0, s, a);
 }
 
 }  // namespace moeca
