@@ -10,6 +10,7 @@
 //   H_e = ln S_e - U_e / S_e  (= -sum_i P ln P with P = C / S, Eq. 11),
 // its normalisation and the expert threshold tau_e (Eq. 12).
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -41,13 +42,19 @@ __device__ __forceinline__ float group_sum(float v) {
 // shapes too large for shared memory read the same data through L1 / L2.
 // Each lane accumulates its logits over D in fp32; softmax and top-k run as
 // shuffles inside the group.
+//
+// bf16 with both staged: the logits come from the tensor cores instead
+// (mma.sync m16n8k16, bf16 in, fp32 accumulate over D in order): 16-token
+// groups by 8-expert tiles, the gate rows zero-padded to a multiple of 8,
+// into a shared logit table the lanes then read.
 template <typename TI, int G, int EPL, int NT>
 __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, int stage_wg) {
   constexpr int V = Elem<TI>::kVec;
   constexpr int TB = NT / G;                  // tokens per block
   constexpr int EMAXB = G * EPL;              // experts covered by a group
   constexpr int kThreads = NT;
-  extern __shared__ uint4 sm_dyn[];           // [E][rowv + 1] gate rows, then [TB][rowv + 1] token rows
+  constexpr bool kTensor = std::is_same_v<TI, __nv_bfloat16> && TB % 16 == 0 && TB / 16 <= NT / 32;
+  extern __shared__ uint4 sm_dyn[];           // [EPAD][rowv + 1] gate rows, [TB][rowv + 1] token rows, logits
   __shared__ float sm_S[TB * EMAXB];
   __shared__ float sm_U[TB * EMAXB];
   __shared__ int sm_near;
@@ -63,8 +70,11 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   const uint4* wsrc = static_cast<const uint4*>(a.w_gate);
   int wstride = rowv;
   const uint4* xsrc = static_cast<const uint4*>(a.x) + static_cast<size_t>(i) * rowv;
+  const int epad = (E + 7) / 8 * 8;
   uint4* sm_wg = sm_dyn;
-  uint4* sm_x = sm_dyn + (stage_wg ? E * pstride : 0);
+  uint4* sm_x = sm_dyn + (stage_wg ? epad * pstride : 0);
+  const bool tensor = kTensor && stage_x && stage_wg;
+  float* sm_logit = reinterpret_cast<float*>(sm_x + TB * pstride);  // [TB][epad + 1], tensor path
   if (t == 0) {
     sm_near = 0;
     if (stage_wg || stage_x) {
@@ -85,7 +95,15 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
           bulk_g2s(smem_u32(sm_x + q * pstride),
                    static_cast<const uint4*>(a.x) + static_cast<size_t>(blockIdx.x * TB + q) * rowv, row_bytes, bar);
     }
+    if (tensor) {
+      // Zero the padding rows the tensor cores read: gate rows past E, token rows past ntok.
+      for (int idx = t; idx < (epad - E) * rowv; idx += kThreads)
+        sm_wg[(E + idx / rowv) * pstride + idx % rowv] = make_uint4(0, 0, 0, 0);
+      for (int idx = t; idx < (TB - ntok) * rowv; idx += kThreads)
+        sm_x[(ntok + idx / rowv) * pstride + idx % rowv] = make_uint4(0, 0, 0, 0);
+    }
     if (!mbar_wait_for(bar, 0, 1000000000ull) && t == 0) report_status(a.status, kStatusWaitTimeout, 500);
+    if (tensor) __syncthreads();
     if (stage_wg) {
       wsrc = sm_wg;
       wstride = pstride;
@@ -95,7 +113,40 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   float z[EPL];
 #pragma unroll
   for (int j = 0; j < EPL; ++j) z[j] = 0.f;
-  if (valid) {
+  if constexpr (kTensor) {
+    if (tensor) {
+      constexpr int NW = NT / 32, TOKG = TB / 16, WPG = NW / TOKG;
+      const int warp = t >> 5, lane = t & 31;
+      const int ntile = epad / 8, ldw = pstride * 8;  // row stride in bf16
+      const int tg = warp / WPG;
+      const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(sm_x);
+      const __nv_bfloat16* wb = reinterpret_cast<const __nv_bfloat16*>(sm_wg);
+      const uint32_t a_addr = smem_u32(xb + (tg * 16 + (lane & 15)) * ldw + (lane >> 4) * 8);
+      const int bl = lane & 15;
+      for (int nt = warp % WPG; nt < ntile; nt += WPG) {
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint32_t b_addr = smem_u32(wb + (nt * 8 + (bl & 7)) * ldw + (bl >> 3) * 8);
+        for (int k0 = 0; k0 < a.D; k0 += 16) {
+          uint32_t a0, a1, a2, a3, b0, b1;
+          ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
+          ldsm_x2(b_addr + k0 * 2, b0, b1);
+          mma_16816(acc, a0, a1, a2, a3, b0, b1);
+        }
+        const int r0 = tg * 16 + (lane >> 2), e0 = nt * 8 + (lane & 3) * 2;
+        sm_logit[r0 * (epad + 1) + e0] = acc[0];
+        sm_logit[r0 * (epad + 1) + e0 + 1] = acc[1];
+        sm_logit[(r0 + 8) * (epad + 1) + e0] = acc[2];
+        sm_logit[(r0 + 8) * (epad + 1) + e0 + 1] = acc[3];
+      }
+      __syncthreads();
+#pragma unroll
+      for (int j = 0; j < EPL; ++j) {
+        const int e = g + G * j;
+        if (e < E) z[j] = sm_logit[tok * (epad + 1) + e];
+      }
+    }
+  }
+  if (valid && !tensor) {
 #pragma unroll 2
     for (int c = 0; c < rowv; ++c) {
       float xv[V];
@@ -256,12 +307,20 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
     const int e = t % E, j = t / E;
     float S = 0.f, U = 0.f;
     if (j < J) {
+      // 16 loads in flight per thread, then added in block order.
       const float2* part = reinterpret_cast<const float2*>(a.partials);
-#pragma unroll 4
-      for (unsigned b = j; b < gridDim.x; b += J) {
-        const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
-        S += v.x;
-        U += v.y;
+      for (unsigned b0 = j; b0 < gridDim.x; b0 += 16u * J) {
+        float2 v[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const unsigned b = b0 + u * J;
+          v[u] = b < gridDim.x ? __ldcg(part + static_cast<size_t>(b) * E + e) : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          S += v[u].x;
+          U += v[u].y;
+        }
       }
     }
     sm_red[t][0] = S;
@@ -327,10 +386,11 @@ cudaError_t launch_g(const RouterArgs& a, cudaStream_t s) {
   }
   const int grid = (a.T + TB - 1) / TB;
   const size_t row = static_cast<size_t>(a.D / Elem<TI>::kVec + 1) * 16;
-  const size_t wg_bytes = a.E * row, x_bytes = TB * row;
+  const size_t epad = (a.E + 7) / 8 * 8;
+  const size_t wg_bytes = epad * row, x_bytes = TB * row, logit_bytes = TB * (epad + 1) * 4;
   const int stage_wg = wg_bytes <= cap;
-  const int stage_x = stage_wg && wg_bytes + x_bytes <= cap;
-  const size_t smem = (stage_wg ? wg_bytes : 0) + (stage_x ? x_bytes : 0);
+  const int stage_x = stage_wg && wg_bytes + x_bytes + logit_bytes <= cap;
+  const size_t smem = (stage_wg ? wg_bytes : 0) + (stage_x ? x_bytes + logit_bytes : 0);
   return launch_pdl(router_kernel<TI, G, EPL, NT>, dim3(grid), dim3(NT), smem, s, a, stage_x, stage_wg);
 }
 
@@ -342,8 +402,10 @@ cudaError_t launch_t(const RouterArgs& a, cudaStream_t s) {
   if (E <= 7) return launch_g<TI, 4, 2, 128>(a, s);
   if (E <= 8) return launch_g<TI, 8, 1, 128>(a, s);
   if (E <= 16) return launch_g<TI, 8, 2, 128>(a, s);
-  if (E <= 32) return launch_g<TI, 8, 4, 256>(a, s);
-  return launch_g<TI, 8, 8, 256>(a, s);
+  // 16 tokens per block for wide gates, so the token rows and the logit
+  // table fit beside the staged gate matrix (the tensor-core path).
+  if (E <= 32) return launch_g<TI, 8, 4, 128>(a, s);
+  return launch_g<TI, 8, 8, 128>(a, s);
 }
 
 }  // namespace
