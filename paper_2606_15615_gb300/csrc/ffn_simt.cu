@@ -108,12 +108,17 @@ __global__ void __launch_bounds__(256) ffn_simt_kernel(FfnArgs a) {
   }
 }
 
+// Plain launches: the grid covers the worst case, and its blocks launched
+// early under a programmatic dependency would sit resident beside the
+// previous kernel's blocks and slow them (measured: 455 vs 209 us per step
+// of the fp32 workload).
 template <typename TI>
 cudaError_t launch_t(const FfnArgs& a, int phase, cudaStream_t s) {
   const int N = phase == 1 ? a.F : a.D;
   const dim3 grid((N + BN - 1) / BN, (a.max_rows + BM - 1) / BM + a.G);
-  if (phase == 1) return launch_pdl(ffn_simt_kernel<TI, 1>, grid, dim3(256), 0, s, a);
-  return launch_pdl(ffn_simt_kernel<TI, 2>, grid, dim3(256), 0, s, a);
+  if (phase == 1) ffn_simt_kernel<TI, 1><<<grid, 256, 0, s>>>(a);
+  else ffn_simt_kernel<TI, 2><<<grid, 256, 0, s>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace
