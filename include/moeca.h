@@ -237,8 +237,24 @@ moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_l
 moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_layer_trace* dst,
                                    void* stream);
 
-/* Drop every cache and zero the EMA statistics; the next step is a full step. */
+/* Drop every cache and zero the EMA statistics; the next step is a full step.
+ * Synchronises the device, then clears a recorded device status (a timeout or
+ * a bad index reported by an earlier kernel) and re-arms every internal
+ * counter a cut-short launch may have left mid-count: the way back after
+ * MOECA_ERR_TIMEOUT or MOECA_ERR_DEVICE_STATUS. */
 moeca_status moeca_reset(moeca_handle* h);
+
+/* Host-side fault injection for tests of failure detection (no counterpart
+ * in the paper).  MOECA_FAULT_BARRIER_STALL: the next step's fused
+ * preparation kernels wait at their grid barriers for an arrival count that
+ * never comes; every block gives up after about one second of %globaltimer,
+ * records MOECA_ERR_TIMEOUT in the device status and skips its later phases,
+ * so the step's outputs are garbage and the next call that checks the device
+ * status returns MOECA_ERR_TIMEOUT until moeca_reset.  Nothing faults or
+ * hangs.  Returns MOECA_ERR_UNSUPPORTED when the handle does not run the
+ * fused preparation kernel (fp32, or shapes it does not fit). */
+typedef enum { MOECA_FAULT_BARRIER_STALL = 1 } moeca_fault;
+moeca_status moeca_inject_fault(moeca_handle* h, int32_t kind);
 
 /* Record CUDA events around every kernel launch (enable = 1) and accumulate
  * their durations; moeca_get_kernel_times() synchronises and reads them, and

@@ -14,6 +14,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "moeca.h"
@@ -83,6 +85,7 @@ struct moeca_handle {
   int tc_dep_pairs_n = 0;
   PrepShape prep{0, 0, 0, 0};   // fused router + select + compact, when it fits
   unsigned prep_arrivals = 0;   // grid-barrier arrivals of all fused launches so far (mod 2^32)
+  bool inject_stall = false;    // moeca_inject_fault: next step's barrier targets unreachable
   int32_t* prep_counts = nullptr;
   unsigned* prep_bar = nullptr;
   std::vector<void*> act;  // input of layer l (l >= 1)
@@ -151,8 +154,20 @@ cudaEvent_t take_event(moeca_handle* h) {
 }
 
 // Launch `fn` with optional CUDA events around it.
+// Scoped NVTX range for profilers (layer and kernel launches of a step).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 template <typename Fn>
 cudaError_t timed(moeca_handle* h, int kind, cudaStream_t s, Fn&& fn) {
+  // An NVTX range per launch (a no-op unless a profiler is attached).
+  static const char* const kNames[MOECA_K_COUNT] = {"router", "select", "compact", "ffn1", "ffn2",
+                                                   "combine", "prep", "ffn"};
+  NvtxRange range(kNames[kind]);
   if (!h->timing) return fn();
   PendingTiming pt{kind, take_event(h), take_event(h)};
   cudaEventRecord(pt.start, s);
@@ -402,8 +417,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   const float tau0 = std::isnan(args->tau0_override) ? c.tau0 : args->tau0_override;
   const bool use_tc = h->bf16 && c.ffn_impl == MOECA_FFN_AUTO;
   cudaError_t e = cudaSuccess;
+  NvtxRange step_range("moeca_step");
   for (int l = 0; l < c.n_layers; ++l) {
     LayerBuf& L = h->layers[l];
+    NvtxRange layer_range("layer");
     const void* in = l == 0 ? x_in : h->act[l];
     void* out = l + 1 == c.n_layers ? x_out : h->act[l + 1];
 
@@ -446,6 +463,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       pa.block_counts = h->prep_counts; pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
       pa.xg = h->xg; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
       pa.bar_base = h->prep_arrivals;
+      if (h->inject_stall) pa.bar_base += 0x40000000u;  // targets no launch will reach
       if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
       h->prep_arrivals += 2u * static_cast<unsigned>((T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block);
     } else {
@@ -487,10 +505,12 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   }
   if (e != cudaSuccess) {
     for (auto& L : h->layers) L.valid = false;
+    h->inject_stall = false;
     return cuda_fail(h, e, "kernel launch");
   }
   h->state_T = T;
   h->last_x_in = x_in;
+  h->inject_stall = false;
   return MOECA_OK;
 }
 
@@ -615,6 +635,14 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
 moeca_status moeca_reset(moeca_handle* h) {
   if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
   cudaSetDevice(h->device);
+  {
+    // Let every kernel of earlier steps finish before the counters and the
+    // device status are cleared.
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(h, e, "synchronise before reset");
+    h->status_host[0] = 0;
+    h->status_host[1] = 0;
+  }
   if (h->prep_bar) {
     cudaError_t e = cudaMemset(h->prep_bar, 0, 2 * sizeof(unsigned));
     if (e != cudaSuccess) return cuda_fail(h, e, "reset barrier");
@@ -633,6 +661,14 @@ moeca_status moeca_reset(moeca_handle* h) {
     if (e != cudaSuccess) return cuda_fail(h, e, "reset EMA");
   }
   h->state_T = 0;
+  return MOECA_OK;
+}
+
+moeca_status moeca_inject_fault(moeca_handle* h, int32_t kind) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  if (kind != MOECA_FAULT_BARRIER_STALL) return fail(h, MOECA_ERR_INVALID_ARG, "unknown fault kind");
+  if (h->prep.tokens_per_block == 0) return fail(h, MOECA_ERR_UNSUPPORTED, "no fused preparation kernel on this handle");
+  h->inject_stall = true;
   return MOECA_OK;
 }
 

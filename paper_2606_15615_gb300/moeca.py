@@ -18,6 +18,8 @@ LIB_PATH = os.path.join(PKG, "libmoeca.so")
 HEADER = os.path.join(os.path.dirname(PKG), "include", "moeca.h")
 
 MOECA_OK = 0
+MOECA_ERR_INVALID_ARG, MOECA_ERR_UNSUPPORTED, MOECA_ERR_CUDA, MOECA_ERR_OOM = -1, -2, -3, -4
+MOECA_ERR_STATE, MOECA_ERR_TIMEOUT, MOECA_ERR_DEVICE_STATUS = -5, -6, -7
 STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "OOM", -5: "STATE",
                 -6: "TIMEOUT", -7: "DEVICE_STATUS"}
 MOECA_F32, MOECA_BF16 = 0, 1
@@ -103,6 +105,7 @@ def _load():
                                             C.c_void_p]),
         "moeca_get_layer_trace": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_trace), C.c_void_p]),
         "moeca_reset": (C.c_int, [H]),
+        "moeca_inject_fault": (C.c_int, [H, C.c_int32]),
         "moeca_set_kernel_timing": (C.c_int, [H, C.c_int32]),
         "moeca_get_kernel_times": (C.c_int, [H, C.POINTER(moeca_kernel_times), C.c_int32]),
         "moeca_destroy": (C.c_int, [H]),
@@ -183,6 +186,14 @@ def moeca_get_layer_trace(h, layer: int, dst: moeca_layer_trace, stream: int = 0
 
 def moeca_reset(h):
     _check(LIB.moeca_reset(h), h)
+
+
+MOECA_FAULT_BARRIER_STALL = 1
+
+
+def moeca_inject_fault(h, kind: int):
+    """Test hook: arm a host-side fault for the next step (see include/moeca.h)."""
+    _check(LIB.moeca_inject_fault(h, kind), h)
 
 
 def moeca_set_kernel_timing(h, enable: bool):
