@@ -73,14 +73,19 @@ __device__ __forceinline__ void decide_token(const SelectArgs& a, int i, bool va
       float cw[KMAX], cn[KMAX];
       float nsum = 0.f;
 #pragma unroll
+      bool corrupt = false;
       for (int q = 0; q < KMAX; ++q) {
         if (q < k) {
           ce[q] = ce_in[q];
           cw[q] = cw_in[q];
           cn[q] = cn_in[q];
           nsum += cn[q];
+          corrupt |= ce[q] < -1 || ce[q] >= E;  // -1: no cached branch
         }
       }
+      // A cached expert id out of range (state written by the host) never
+      // matches, so its branches are recomputed; the status word reports it.
+      if (corrupt) report_status(a.status, kStatusBadIndex, 1100000 + i);
       unsigned used = 0u;
       int qof[KMAX];
 #pragma unroll

@@ -7,6 +7,8 @@
   results identical to a fresh handle's.
 * A device allocation that cannot succeed is reported as MOECA_ERR_OOM and
   leaves nothing behind: a normal handle can be created right after.
+* A cached expert id out of range, written by the host, is reported as a
+  device status and cleared by moeca_reset.
 """
 import ctypes
 
@@ -92,4 +94,28 @@ def test_unsatisfiable_allocation_is_reported_and_leaves_nothing(M):
     cfg2, w, xs = _stack(M)
     st = M.Stack(cfg2, [w])
     _run(st, xs[:1])
+    st.close()
+
+
+def test_corrupted_cache_metadata_is_reported(M):
+    """A cached expert id out of range, written by the host through
+    moeca_set_layer_state, is reported as MOECA_ERR_DEVICE_STATUS; the branch
+    is treated as unmatched, and moeca_reset clears the status."""
+    import torch
+    cfg, w, xs = _stack(M, seed=5)
+    st = M.Stack(cfg, [w])
+    st.step(xs[0], 0)
+    state = st.get_state(0)
+    torch.cuda.synchronize()
+    bad = {k_: (v.clone() if isinstance(v, torch.Tensor) else v) for k_, v in state.items()}
+    bad["cache_e"][5, 0] = 999
+    st.set_state(0, bad)
+    st.step(xs[1], 1)
+    torch.cuda.synchronize()
+    with pytest.raises(M.MoecaError) as err:
+        st.stats()
+    assert err.value.status == M.MOECA_ERR_DEVICE_STATUS
+    M.moeca_reset(st.handle)
+    _run(st, xs)
+    st.stats()
     st.close()
