@@ -18,6 +18,10 @@ Each function names the passage of the paper it follows:
   Eq. 10          EMA spatial activation statistic C_{e,i}
   Eq. 11          spatial response entropy H_e and its normalisation
   Eq. 12          expert-aware threshold tau_e = tau0 (1 + alpha (2 Hbar_e - 1))
+  Sec. 4.1        attention output a_i cached with the branches; a token's
+                  attention is recomputed on the step its recompute set is
+                  non-empty (synchronized MoE / attention update)
+  Table 4         "without sync. update": attention reused on every cache step
 
 Readings where the paper is silent (each is a switch in ``Params``):
   * gate weights: softmax over all E experts, top-k, then renormalised over
@@ -36,6 +40,20 @@ Readings where the paper is silent (each is a switch in ``Params``):
   * shared experts are recomputed on full-computation steps and for tokens
     with a non-empty recompute set ("sync"), or always ("always");
   * GELU is the tanh form ("tanh") or the erf form ("erf"); experts have no bias.
+  * a DiT block (n_heads > 0) is x -> u = x + Attn(x) -> u + MoE(u), without
+    normalisation or modulation; attention is multi-head self-attention over
+    the seq_len consecutive token rows of each sample, with all of the
+    sample's keys and values taken from the current block input;
+  * on a cache step the recompute decision comes before the attention
+    update, so the router sees u' = x + a^{t0} (cached attention output);
+    a token with a non-empty recompute set then recomputes its attention,
+    and its recomputed branches and its residual use u = x + a^t; a token
+    without one keeps u' (``attn_policy`` "sync"); "stale" reuses a^{t0} on
+    every cache step (Table 4's ablation); "full" recomputes attention for
+    every token on every step and routes on the fresh input;
+  * ``act_store`` "bf16" rounds the block's stored activations (a, u) to
+    bfloat16, the storage type of the bf16 kernels, so that decisions taken
+    on u' use the same input on both sides; "f64" keeps them exact.
 """
 from __future__ import annotations
 
@@ -65,6 +83,10 @@ class Params:
     gelu: str = "tanh"                 # or "erf"
     score_terms: int = 7               # Eq. 9 terms kept: 1 = w, 2 = lambda1 Delta, 4 = lambda2 o (Table 5)
     granularity: str = "branch"        # or "token": a token's k branches share one decision
+    n_heads: int = 0                   # > 0: each layer is a DiT block with an attention sub-layer
+    seq_len: int = 0                   # token rows per sample (attention scope); 0: all T rows
+    attn_policy: str = "sync"          # or "stale" (Table 4 ablation) or "full"
+    act_store: str = "f64"             # or "bf16": storage rounding of the block's a and u
 
 
 # ---------------------------------------------------------------------------
@@ -90,6 +112,68 @@ def expert_ffn(u_rows: np.ndarray, w1: np.ndarray, w2: np.ndarray, form: str) ->
     u = np.asarray(u_rows, dtype=np.float64)
     hmid = gelu(u @ np.asarray(w1, np.float64).T, form)
     return hmid @ np.asarray(w2, np.float64).T
+
+
+# ---------------------------------------------------------------------------
+# Attention path of a DiT block (Sec. 4.1)
+# ---------------------------------------------------------------------------
+
+def round_bf16(a) -> np.ndarray:
+    """Nearest bfloat16 value of each element (ties to even), as float64.
+
+    bfloat16 keeps the top 16 bits of a float32: the value is rounded to
+    float32 first (exact for a sum of two bfloat16 values), then its low
+    16 bits are rounded away.  Infinities and NaNs pass through.
+    """
+    f = np.ascontiguousarray(np.asarray(a, np.float64).astype(np.float32))
+    bits = f.view(np.uint32).astype(np.uint64)
+    keep = (bits >> 16) & 1
+    r = ((bits + 0x7FFF + keep) & 0xFFFF0000).astype(np.uint32)
+    out = r.view(np.float32).astype(np.float64)
+    special = ~np.isfinite(f)
+    out[special] = f[special]
+    return out
+
+
+def attention(x, w_qkv, b_qkv, w_o, b_o, n_heads: int, seq_len: int, rows=None) -> np.ndarray:
+    """Multi-head self-attention output a_i of a DiT block (the a_i of Sec. 4.1).
+
+    x is [T, D]; token rows come in samples of ``seq_len`` consecutive rows
+    (0: one sample of T rows) and attend to every row of their own sample.
+    w_qkv is [3D, D]: rows [0, D) give queries, [D, 2D) keys, [2D, 3D)
+    values, head h owning rows [h dh, (h + 1) dh) of each (dh = D / n_heads);
+    b_qkv [3D] and b_o [D] may be None.  Per head,
+        A_h = softmax(Q_h K_h^T / sqrt(dh)) V_h   (softmax over the keys),
+    the heads are concatenated and a = A w_o^T + b_o.  Returns a for the
+    token rows ``rows`` (ascending ids; None: all), [len(rows), D].
+    """
+    x = np.asarray(x, np.float64)
+    T, D = x.shape
+    H = int(n_heads)
+    dh = D // H
+    S = int(seq_len) or T
+    qkv = x @ np.asarray(w_qkv, np.float64).T
+    if b_qkv is not None:
+        qkv = qkv + np.asarray(b_qkv, np.float64)[None, :]
+    q, k, v = qkv[:, :D], qkv[:, D:2 * D], qkv[:, 2 * D:]
+    rows = np.arange(T) if rows is None else np.asarray(rows, np.int64)
+    A = np.zeros((len(rows), D))
+    for b in range(T // S):
+        mine = np.nonzero(rows // S == b)[0]
+        if len(mine) == 0:
+            continue
+        qi = rows[mine]
+        keys = slice(b * S, (b + 1) * S)
+        for h in range(H):
+            hs = slice(h * dh, (h + 1) * dh)
+            s = q[qi, hs] @ k[keys, hs].T / math.sqrt(dh)          # [n, S]
+            p = np.exp(s - s.max(axis=1, keepdims=True))
+            p /= p.sum(axis=1, keepdims=True)
+            A[mine, hs] = p @ v[keys, hs]
+    a = A @ np.asarray(w_o, np.float64).T
+    if b_o is not None:
+        a = a + np.asarray(b_o, np.float64)[None, :]
+    return a
 
 
 # ---------------------------------------------------------------------------
@@ -284,18 +368,20 @@ class LayerState:
     shared_h: np.ndarray | None  # [T, D] float64, shared-expert output
     C: np.ndarray              # [E, T] float64 C_{e,i}
     valid: bool = False
+    attn_a: np.ndarray | None = None  # [T, D] float64 a_i^{t0} of a DiT block (Sec. 4.1)
 
     @staticmethod
-    def empty(T: int, D: int, E: int, k: int, n_shared: int) -> "LayerState":
+    def empty(T: int, D: int, E: int, k: int, n_shared: int, attention: bool = False) -> "LayerState":
         return LayerState(
             cache_e=np.full((T, k), -1, np.int32), cache_w=np.zeros((T, k)),
             cache_norm=np.zeros((T, k)), cache_h=np.zeros((T, k, D)),
-            shared_h=np.zeros((T, D)) if n_shared else None, C=np.zeros((E, T)), valid=False)
+            shared_h=np.zeros((T, D)) if n_shared else None, C=np.zeros((E, T)), valid=False,
+            attn_a=np.zeros((T, D)) if attention else None)
 
     def copy(self) -> "LayerState":
         return LayerState(self.cache_e.copy(), self.cache_w.copy(), self.cache_norm.copy(),
                           self.cache_h.copy(), None if self.shared_h is None else self.shared_h.copy(),
-                          self.C.copy(), self.valid)
+                          self.C.copy(), self.valid, None if self.attn_a is None else self.attn_a.copy())
 
 
 def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, slot, weights: dict,
@@ -358,8 +444,20 @@ def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, ref
     under the synchronized rule (Sec. 4.1) -> combine with current gate weights
     (Eq. 8) plus the residual (Eq. 5 / 6) -> refresh the cached norms.
     """
+    info = decide(state, u, weights, prm, refresh)
+    out, new, token_any = recompute_and_combine(state, u, info["e"], info["w"], info["recompute"],
+                                                info["slot"], weights, prm, refresh)
+    new.C = info["C"]
+    info["token_any"] = token_any
+    return out, new, info
+
+
+def decide(state: LayerState, u: np.ndarray, weights: dict, prm: Params, refresh: bool) -> dict:
+    """The decision half of a layer step, taken on the router input u:
+    route (Eq. 7) -> EMA (Eq. 10) -> entropy and tau (Eq. 11-12) -> match,
+    score, decide and assign slots (Sec. 4.2, Eq. 9).  Returns the routing,
+    the new statistic C, tau and the select_branches fields."""
     u = np.asarray(u, np.float64)
-    T, D = u.shape
     k = prm.top_k
     e_cur, w_cur, near, _ = route(u, weights["w_gate"], weights.get("b_gate"), k, prm.renorm_topk)
     C = ema_update(state.C, e_cur, prm.beta)
@@ -367,11 +465,61 @@ def layer_step(state: LayerState, u: np.ndarray, weights: dict, prm: Params, ref
     tau = expert_threshold(Hbar, prm.tau0, prm.alpha)
     sel = select_branches(e_cur, w_cur, state.cache_e, state.cache_w, state.cache_norm, tau,
                           prm.lambda1, prm.lambda2, refresh, prm.score_terms, prm.granularity)
-    out, new, token_any = recompute_and_combine(state, u, e_cur, w_cur, sel["recompute"], sel["slot"],
-                                                weights, prm, refresh)
-    new.C = C
-    info = dict(e=e_cur, w=w_cur, near_route=near, C=C, Hbar=Hbar, tau=tau,
-                token_any=token_any, refresh=refresh, **sel)
+    return dict(e=e_cur, w=w_cur, near_route=near, C=C, Hbar=Hbar, tau=tau,
+                token_any=sel["recompute"].any(axis=1), refresh=refresh, **sel)
+
+
+def block_step(state: LayerState, x: np.ndarray, weights: dict, prm: Params, refresh: bool):
+    """One DiT-MoE block at one denoising step: the attention sub-layer, then
+    the MoE sub-layer, with the attention output a_i cached beside the
+    branches (Sec. 4.1).  Returns (out [T, D], new state, info).
+
+    Full-computation step, or attn_policy "full": a = Attn(x) for every
+    token, u = x + a, and the MoE layer step runs on u.
+    Cache step, "sync" (Sec. 4.1): the decision is taken on u' = x + a^{t0};
+    tokens with a non-empty recompute set recompute a_i from the current x
+    (all keys of their sample), store it, and take u_i = x_i + a_i; the
+    others keep u'_i.  The recomputed branches take u as their input, Eq. 8
+    combines with the gate weights routed on u', and the residual adds u.
+    Cache step, "stale" (Table 4, without sync update): u = x + a^{t0} for
+    every token and a is left as it is.
+    ``info`` adds u (MoE input), route_in (router input) and attn_rows.
+    """
+    x = np.asarray(x, np.float64)
+    T, D = x.shape
+    store = round_bf16 if prm.act_store == "bf16" else (lambda v: np.asarray(v, np.float64))
+
+    def attn(rows=None):
+        return attention(x, weights["w_qkv"], weights.get("b_qkv"), weights["w_o"], weights.get("b_o"),
+                         prm.n_heads, prm.seq_len, rows)
+
+    if refresh or prm.attn_policy == "full":
+        a = store(attn())
+        u = store(x + a)
+        out, new, info = layer_step(state, u, weights, prm, refresh)
+        new.attn_a = a
+        info.update(u=u, route_in=u, attn_rows=np.arange(T))
+        return out, new, info
+    u_pre = store(x + state.attn_a)
+    if prm.attn_policy == "stale":
+        out, new, info = layer_step(state, u_pre, weights, prm, refresh)
+        new.attn_a = state.attn_a.copy()
+        info.update(u=u_pre, route_in=u_pre, attn_rows=np.zeros(0, np.int64))
+        return out, new, info
+    if prm.attn_policy != "sync":
+        raise ValueError(prm.attn_policy)
+    info = decide(state, u_pre, weights, prm, refresh)
+    rows = np.nonzero(info["token_any"])[0]
+    a = state.attn_a.copy()
+    u = u_pre.copy()
+    if len(rows):
+        a[rows] = store(attn(rows))
+        u[rows] = store(x[rows] + a[rows])
+    out, new, token_any = recompute_and_combine(state, u, info["e"], info["w"], info["recompute"],
+                                                info["slot"], weights, prm, refresh)
+    new.C = info["C"]
+    new.attn_a = a
+    info.update(u=u, route_in=u_pre, attn_rows=rows)
     return out, new, info
 
 
@@ -384,7 +532,8 @@ def stats_of(info: dict) -> dict:
 
 
 class Stack:
-    """A stack of L MoE layers run over denoising steps (Sec. 4.1 schedule).
+    """A stack of L MoE layers (DiT-MoE blocks when n_heads > 0) run over
+    denoising steps (Sec. 4.1 schedule).
 
     A step is a full-computation step when it is forced, when the caches are
     not valid or the token count changed, or when ``refresh_period`` N > 0
@@ -409,11 +558,12 @@ class Stack:
         T = x.shape[0]
         refresh = self.is_refresh(step_index, T, force)
         if self.states is None or T != self.T:
-            self.states = [LayerState.empty(T, self.D, self.E, self.prm.top_k, self.S)
+            self.states = [LayerState.empty(T, self.D, self.E, self.prm.top_k, self.S, self.prm.n_heads > 0)
                            for _ in self.layers]
             self.T = T
         infos = []
+        step_fn = block_step if self.prm.n_heads > 0 else layer_step
         for l, w in enumerate(self.layers):
-            x, self.states[l], info = layer_step(self.states[l], x, w, self.prm, refresh)
+            x, self.states[l], info = step_fn(self.states[l], x, w, self.prm, refresh)
             infos.append(info)
         return x, infos

@@ -24,7 +24,7 @@ _WEIGHT_SEED = 1000
 _TRAJ_SEED = 2000
 
 # Tensor ids inside a layer's weight seed tuple.
-_T_GATE, _T_W1, _T_W2, _T_WS1, _T_WS2, _T_BIAS = range(6)
+_T_GATE, _T_W1, _T_W2, _T_WS1, _T_WS2, _T_BIAS, _T_QKV, _T_BQKV, _T_WO, _T_BO = range(10)
 
 
 @dataclass(frozen=True)
@@ -47,6 +47,7 @@ class Workload:
     drift: str = "decay"      # "per_token" (sigma_i ~ U) or "decay" (sigma_t linear)
     router_skew: tuple = ()   # target top-k load shares, e.g. (4, 2, 1, 1)
     reuse_targets: tuple = (0.5,)
+    n_heads: int = 0          # > 0: DiT-MoE blocks (self-attention over each sample's seq tokens, then MoE)
 
     @property
     def n_tokens(self) -> int:
@@ -86,10 +87,25 @@ WORKLOADS = {
 
 WORKLOAD_ORDER = list(WORKLOADS)
 
+# Attention heads of the DiT models each bf16 stack stands in for: DiT-B (768,
+# 12 x 64), DiT-XL (1152, 16 x 72), HiDream-I1 (2560, 20 x 128).
+_HEADS = {384: 6, 768: 12, 1152: 16, 2560: 20}
+
+
+def dit_variant(wl: Workload) -> Workload:
+    """The same stack with every layer a DiT-MoE block (attention sub-layer first)."""
+    name = wl.name.replace("moe_d%d_" % wl.hidden, "dit_d%d_h%d_" % (wl.hidden, _HEADS[wl.hidden]), 1)
+    return replace(wl, name=name, n_heads=_HEADS[wl.hidden])
+
+
+DIT_WORKLOADS = {d.name: d for d in (dit_variant(w) for w in WORKLOADS.values() if w.dtype == "bf16")}
+
 
 def workload(name_or_index) -> Workload:
     if isinstance(name_or_index, int):
         return WORKLOADS[WORKLOAD_ORDER[name_or_index - 1]]
+    if name_or_index in DIT_WORKLOADS:
+        return DIT_WORKLOADS[name_or_index]
     return WORKLOADS[name_or_index]
 
 
@@ -188,6 +204,33 @@ def make_layer_weights(wl: Workload, layer: int) -> dict:
     return out
 
 
+def make_attn_weights(wl: Workload, layer: int) -> dict:
+    """Attention weights of one DiT block, all N(0, 0.02^2), matrices in the
+    workload dtype and biases float32:
+      w_qkv [3D, D] (query, key, value projections stacked, heads contiguous
+      within each), b_qkv [3D], w_o [D, D], b_o [D]."""
+    seed = _WEIGHT_SEED + wl.index
+    D = wl.hidden
+    return {
+        "w_qkv": _store(wl, 0.02 * _rng(seed, layer, _T_QKV).standard_normal((3 * D, D), dtype=np.float32)),
+        "b_qkv": (0.02 * _rng(seed, layer, _T_BQKV).standard_normal(3 * D)).astype(np.float32),
+        "w_o": _store(wl, 0.02 * _rng(seed, layer, _T_WO).standard_normal((D, D), dtype=np.float32)),
+        "b_o": (0.02 * _rng(seed, layer, _T_BO).standard_normal(D)).astype(np.float32),
+    }
+
+
+def tiny_attn(seed: int, D: int, dtype: str = "f32", bias: bool = True, wscale: float = 0.2) -> dict:
+    """Small random attention weights for pins and parity cases."""
+    rng = _rng(7500 + seed)
+    st = round_to_bf16 if dtype == "bf16" else (lambda a: np.asarray(a, np.float32))
+    return {
+        "w_qkv": st(wscale * rng.standard_normal((3 * D, D), dtype=np.float32)),
+        "b_qkv": (0.1 * rng.standard_normal(3 * D)).astype(np.float32) if bias else None,
+        "w_o": st(wscale * rng.standard_normal((D, D), dtype=np.float32)),
+        "b_o": (0.1 * rng.standard_normal(D)).astype(np.float32) if bias else None,
+    }
+
+
 # ---------------------------------------------------------------------------
 # Trajectories of the first layer's input
 # ---------------------------------------------------------------------------
@@ -261,6 +304,11 @@ def make_layer_weights_device(wl: Workload, layer: int, device) -> dict:
         return t.to(dt).contiguous()
 
     out = {"w_gate": draw(_T_GATE, (E, D)), "w1": draw(_T_W1, (E, F, D)), "w2": draw(_T_W2, (E, D, F))}
+    if wl.n_heads:
+        out["w_qkv"] = draw(_T_QKV, (3 * D, D))
+        out["b_qkv"] = draw(_T_BQKV, (3 * D,)).float()
+        out["w_o"] = draw(_T_WO, (D, D))
+        out["b_o"] = draw(_T_BO, (D,)).float()
     b = _skew_bias(wl)
     out["b_gate"] = None if b is None else torch.from_numpy(b).to(device)
     if S:
