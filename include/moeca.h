@@ -10,6 +10,13 @@
  *   -> combine fresh and cached branch outputs with the current gate weights
  *   and add the residual (Eq. 8) -> refresh the cached branch norms.
  * Full-computation and cache steps alternate as in Sec. 4.1.
+ * With n_heads > 0 every layer is a DiT-MoE block: a multi-head
+ * self-attention sub-layer, whose output a_i is cached beside the branches,
+ * runs before the MoE sub-layer.  On a cache step a token recomputes its
+ * attention exactly when its recompute set is non-empty (Sec. 4.1, the
+ * synchronized MoE / attention update); the decision is taken on
+ * u'_i = x_i + a_i^{t0}, and a token that recomputes continues with
+ * u_i = x_i + a_i^t.
  *
  * Conventions
  *  - All tensors are row-major.  "device" pointers are CUDA global memory of
@@ -88,6 +95,16 @@ typedef struct {
   int32_t granularity;        /* 0: branch-level decisions (MoECa, default); 1: token-level, a
                                  token's k branches share one decision: all are recomputed when
                                  the branch rule would recompute any of them (Sec. 3) */
+  int32_t n_heads;            /* 0 (default): each layer is the MoE sub-layer alone; H > 0: each
+                                 layer is a DiT-MoE block whose attention sub-layer has H heads of
+                                 D / H (64, 72, 80, 96 or 128) channels; bf16 only */
+  int32_t seq_len;            /* token rows per sample: attention runs within each run of seq_len
+                                 consecutive rows (0: all T rows are one sample); T must be a
+                                 multiple of it */
+  int32_t attn_policy;        /* attention output on cache steps: 0 = recomputed for the tokens
+                                 with a non-empty recompute set (Sec. 4.1 sync rule, default);
+                                 1 = reused for every token ("without sync update", Table 4);
+                                 2 = recomputed for every token, routing on the fresh input */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters
@@ -100,6 +117,10 @@ void moeca_config_default(moeca_config* cfg);
  *   w_gate [E, D], b_gate [E] fp32 or NULL,
  *   w1 [E, F, D], w2 [E, D, F]  (FFN_e(u) = w2_e GELU(w1_e u), no bias),
  *   ws1 [F, D], ws2 [D, F] for the shared expert (NULL when n_shared == 0).
+ * Attention sub-layer (n_heads > 0; NULL otherwise), a = Attn(x):
+ *   w_qkv [3D, D]: rows [0, D) queries, [D, 2D) keys, [2D, 3D) values, head h
+ *   at rows h*dh .. h*dh + dh - 1 of each; b_qkv [3D] fp32 or NULL;
+ *   w_o [D, D] output projection; b_o [D] fp32 or NULL.
  * Base pointers must be 16-byte aligned. */
 typedef struct {
   const void* w_gate;
@@ -108,6 +129,10 @@ typedef struct {
   const void* w2;
   const void* ws1;
   const void* ws2;
+  const void* w_qkv;
+  const float* b_qkv;
+  const void* w_o;
+  const float* b_o;
 } moeca_layer_weights;
 
 /* Per-step arguments. */
@@ -133,6 +158,7 @@ typedef struct {
   int64_t near_margin_score;    /* matched branches with |s - tau| < 1e-5 |tau|         */
   int32_t device_status;        /* 0, or the first kernel status code seen              */
   int32_t device_detail;        /* kernel-specific detail of that status                */
+  int64_t attn_recomputed;      /* token rows whose attention output was computed (n_heads > 0) */
 } moeca_stats;
 
 /* Caller-owned DEVICE buffers for one layer's cached state, T rows each.
@@ -143,7 +169,8 @@ typedef struct {
  *   cache_norm [T, k] fp32 ||h^{t0}|| over D                (Eq. 9, o)
  *   cache_h [T, k, D] dtype cached branch outputs h^{t0}    (Eq. 7)
  *   shared_h [T, D] dtype  cached shared-expert output      (Eq. 6)
- *   ema [T, E] fp32        C_{e,i} stored at [i * E + e]     (Eq. 10) */
+ *   ema [T, E] fp32        C_{e,i} stored at [i * E + e]     (Eq. 10)
+ *   attn_a [T, D] dtype    cached attention output a^{t0}   (Sec. 4.1; n_heads > 0) */
 typedef struct {
   int32_t* cache_e;
   float* cache_w;
@@ -151,6 +178,7 @@ typedef struct {
   void* cache_h;
   void* shared_h;
   float* ema;
+  void* attn_a;
 } moeca_layer_state;
 
 /* Caller-owned DEVICE buffers for what one layer computed on the last step.
@@ -162,7 +190,10 @@ typedef struct {
  *   token_any [T] uint8                          recompute set non-empty (Sec. 4.1)
  *   counts [G] int32, offsets [G + 1] int32      rows per expert group
  *   list [offsets[G]] int32                      rows: token * k + slot (routed), token (shared)
- *   layer_in [T, D] dtype                        the layer's input activations */
+ *   layer_in [T, D] dtype                        the MoE sub-layer's input: the layer input, or
+ *                                                for a DiT-MoE block u = x + a after the
+ *                                                attention update (the FFN rows and the residual)
+ *   block_in [T, D] dtype                        the DiT-MoE block's input x (n_heads > 0) */
 typedef struct {
   int32_t* route_e;
   float* route_w;
@@ -175,6 +206,7 @@ typedef struct {
   int32_t* offsets;
   int32_t* list;
   void* layer_in;
+  void* block_in;
 } moeca_layer_trace;
 
 /* Kernel kinds timed by moeca_set_kernel_timing(). */
@@ -187,7 +219,11 @@ enum {
   MOECA_K_COMBINE = 5, /* Eq. 8 combine + residual + cached norms           */
   MOECA_K_PREP = 6,    /* router + select + compact fused in one launch (bf16) */
   MOECA_K_FFN = 7,     /* both grouped GEMMs in one persistent launch (bf16) */
-  MOECA_K_COUNT = 8
+  MOECA_K_QKV = 8,     /* attention: query / key / value projection GEMM     */
+  MOECA_K_ATTN = 9,    /* attention: softmax(q k^T / sqrt(dh)) v of the recomputed rows */
+  MOECA_K_OPROJ = 10,  /* attention: output projection GEMM + x + a          */
+  MOECA_K_ATTN_AUX = 11, /* attention: u = x + a^{t0}, recomputed-token list, FFN row gather */
+  MOECA_K_COUNT = 12
 };
 
 typedef struct {

@@ -13,7 +13,7 @@ namespace moeca {
 enum StatIndex {
   kStLayerSteps = 0, kStRefreshSteps, kStBranches, kStCacheBranches, kStMatched,
   kStRecomputed, kStReused, kStTokensFullyReused, kStSharedRecomputed,
-  kStNearRoute, kStNearScore, kStCount
+  kStNearRoute, kStNearScore, kStAttnRows, kStCount
 };
 
 constexpr int kMaxExperts = 64;
@@ -88,6 +88,8 @@ struct CompactArgs {
 };
 // compact_kernel (row lists), then, unless xg is null, gather_kernel (rows).
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s);
+// gather_kernel alone: the listed rows of a.x into a.xg (lists already built).
+cudaError_t launch_gather(const CompactArgs& a, bool bf16, cudaStream_t s);
 
 // Grouped expert FFN over the compacted rows (Eq. 5 / Eq. 6 on R only).
 struct FfnArgs {
@@ -148,7 +150,7 @@ struct PrepArgs {
   int32_t* counts;        // [G]
   int32_t* offsets;       // [G + 1]
   int32_t* list;          // [rows]
-  void* xg;               // [rows, D]
+  void* xg;               // [rows, D], or null: the rows are gathered later (launch_gather)
   unsigned* gbar;         // grid barrier arrival counter (zeroed once, only grows)
   unsigned bar_base;      // arrivals on gbar from earlier launches (mod 2^32)
   unsigned long long* stats;
@@ -179,5 +181,50 @@ struct CombineArgs {
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);
+
+// ---- Attention path of a DiT-MoE block (Sec. 4.1), bf16 only ----
+
+// Tensor-core projection GEMM: C = A B^T + bias (proj_tc.cu).
+enum ProjMode { kProjStore = 0, kProjResidual = 1 };
+struct ProjArgs {
+  const void* A;          // [a_rows, K] bf16, row-major
+  int a_rows;             // rows A holds (>= M)
+  const void* B;          // [N, K] bf16 weights
+  const float* bias;      // [N] or null
+  int M, N, K;            // N a multiple of 64, K of 64
+  const int* m_dev;       // device row count (<= M), or null
+  int mode;               // ProjMode
+  void* out;              // kProjStore: [M, ldo] bf16
+  int ldo;
+  const int32_t* rows;    // kProjResidual: token of row m, or null (m)
+  int n_tok;              // kProjResidual: rows of x / a_out / u_out
+  const void* x;          // kProjResidual: [n_tok, N]
+  void* a_out;            // kProjResidual: [n_tok, N]  a_i
+  void* u_out;            // kProjResidual: [n_tok, N]  x_i + a_i
+  unsigned long long* row_stat;  // or null: the launch adds its row count here
+  int* status;
+};
+int proj_tile_n(int N);   // tile width the launch uses for N (0: N not a multiple of 64)
+cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s);
+
+// u = x + a, row by row (the MoE input of a token that keeps its cached attention).
+cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, int D, int* status,
+                                 cudaStream_t s);
+
+// Ascending list of tokens whose recompute set is non-empty, and its length.
+cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int32_t* rows, int* n_rows, cudaStream_t s);
+
+// Multi-head self-attention rows: o[r] = concat_h softmax(q_t k_S^T / sqrt(dh)) v_S for the
+// r-th listed token t, keys and values of t's sample (S consecutive token rows).
+struct AttnArgs {
+  const void* qkv;        // [T, 3D] bf16: q | k | v, head h at columns h dh .. of each
+  int T, D, H, S;         // S tokens per sample, T a multiple of S
+  const int32_t* rows;    // ascending token list, or null: every token (row r = token r)
+  const int* n_rows;      // device length of rows (when rows is set)
+  void* o;                // [rows, D] bf16
+  int* status;
+};
+bool attn_supported(int D, int H);
+cudaError_t launch_attn_core(const AttnArgs& a, cudaStream_t s);
 
 }  // namespace moeca

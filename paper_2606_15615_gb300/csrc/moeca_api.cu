@@ -5,6 +5,14 @@
 //   router (Eq. 7, Eq. 10-12) -> select (Sec. 4.2, Eq. 9) -> compact ->
 //   grouped FFN phase 1 and 2 over the recompute rows (Eq. 5 / Eq. 6) ->
 //   combine (Eq. 8) writing the next layer's input.
+// A DiT-MoE block (n_heads > 0) adds its attention sub-layer (Sec. 4.1):
+//   full step:  q/k/v projection -> attention of every row -> output
+//               projection writing a and u = x + a -> the MoE sub-layer on u;
+//   cache step: u = x + a^{t0} -> router / decisions on u -> (sync rule)
+//               list of tokens with a non-empty recompute set -> q/k/v
+//               projection -> attention of the listed rows -> output
+//               projection updating their a and u -> FFN row gather from u
+//               -> FFN -> combine with the residual u.
 // It decides full-computation vs cache steps (Sec. 4.1), owns every state and
 // workspace buffer, and reports errors as status codes.
 #include <cmath>
@@ -52,6 +60,8 @@ struct LayerBuf {
   int32_t* offsets = nullptr;
   int32_t* list = nullptr;
   unsigned long long* stats = nullptr;
+  void* attn_a = nullptr;    // [T, D] cached attention output a^{t0} (DiT-MoE block)
+  void* attn_u = nullptr;    // [T, D] MoE sub-layer input u of the last step
   TcPlan* tc = nullptr;
   bool valid = false;
 };
@@ -88,6 +98,10 @@ struct moeca_handle {
   bool inject_stall = false;    // moeca_inject_fault: next step's barrier targets unreachable
   int32_t* prep_counts = nullptr;
   unsigned* prep_bar = nullptr;
+  void* qkv = nullptr;          // attention workspace: [T, 3D] q | k | v
+  void* attn_o = nullptr;       // [T, D] attention rows before the output projection
+  int32_t* attn_rows = nullptr; // [T] tokens that recompute their attention
+  int* attn_n = nullptr;        // their count
   std::vector<void*> act;  // input of layer l (l >= 1)
   int* status_host = nullptr;
   int* status_dev = nullptr;
@@ -165,8 +179,8 @@ struct NvtxRange {
 template <typename Fn>
 cudaError_t timed(moeca_handle* h, int kind, cudaStream_t s, Fn&& fn) {
   // An NVTX range per launch (a no-op unless a profiler is attached).
-  static const char* const kNames[MOECA_K_COUNT] = {"router", "select", "compact", "ffn1", "ffn2",
-                                                   "combine", "prep", "ffn"};
+  static const char* const kNames[MOECA_K_COUNT] = {"router", "select", "compact", "ffn1", "ffn2", "combine",
+                                                   "prep", "ffn", "qkv", "attn", "oproj", "attn_aux"};
   NvtxRange range(kNames[kind]);
   if (!h->timing) return fn();
   PendingTiming pt{kind, take_event(h), take_event(h)};
@@ -217,6 +231,9 @@ void moeca_config_default(moeca_config* c) {
   c->granularity = 0;
   c->gelu_tanh = 1;
   c->ffn_impl = MOECA_FFN_AUTO;
+  c->n_heads = 0;
+  c->seq_len = 0;
+  c->attn_policy = 0;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -265,6 +282,13 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&
        c.ffn_tile_n != 256) || c.ffn_split_k < 0 || c.ffn_split_k > 4)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_tile_n must be 0/64/128/192/256, ffn_split_k 0..4");
+  if (c.n_heads < 0 || c.seq_len < 0 || c.attn_policy < 0 || c.attn_policy > 2)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_heads and seq_len must be >= 0, attn_policy 0..2");
+  const bool attn = c.n_heads > 0;
+  if (attn && !bf16) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "the attention sub-layer is built for bf16 only");
+  if (attn && (!attn_supported(c.hidden, c.n_heads) || c.hidden % 64))
+    return fail(nullptr, MOECA_ERR_UNSUPPORTED,
+                "attention needs hidden a multiple of 64 and hidden / n_heads in {64, 72, 80, 96, 128}");
   const int vec = bf16 ? 8 : 4;
   if (c.hidden % vec) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "hidden must be a multiple of 8 (bf16) / 4 (fp32)");
   const bool use_tc = bf16 && c.ffn_impl == MOECA_FFN_AUTO;
@@ -278,7 +302,9 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     const moeca_layer_weights& w = layers[l];
     if (!w.w_gate || !w.w1 || !w.w2) return fail(nullptr, MOECA_ERR_INVALID_ARG, "layer weight pointer is NULL");
     if (c.n_shared && (!w.ws1 || !w.ws2)) return fail(nullptr, MOECA_ERR_INVALID_ARG, "shared expert weights are NULL");
-    const void* ps[] = {w.w_gate, w.w1, w.w2, w.ws1, w.ws2};
+    if (attn && (!w.w_qkv || !w.w_o)) return fail(nullptr, MOECA_ERR_INVALID_ARG, "attention weights are NULL");
+    const void* ps[] = {w.w_gate, w.w1, w.w2, w.ws1, w.ws2, attn ? w.w_qkv : nullptr, attn ? w.b_qkv : nullptr,
+                        attn ? w.w_o : nullptr, attn ? w.b_o : nullptr};
     for (const void* p : ps)
       if (reinterpret_cast<uintptr_t>(p) % 16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "weights must be 16-byte aligned");
   }
@@ -321,6 +347,16 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     A((void**)&L.offsets, (G + 1) * 4);
     A((void**)&L.list, static_cast<size_t>(h->max_rows) * 4);
     A((void**)&L.stats, kStCount * 8);
+    if (attn) {
+      A(&L.attn_a, T * D * es);
+      A(&L.attn_u, T * D * es);
+    }
+  }
+  if (attn) {
+    A(&h->qkv, T * 3 * D * es);
+    A(&h->attn_o, T * D * es);
+    A((void**)&h->attn_rows, T * 4);
+    A((void**)&h->attn_n, 16);
   }
   const size_t nblk_router = (T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
   const size_t nblk_sel = (T + kSelectTokensPerBlock - 1) / kSelectTokensPerBlock;
@@ -416,6 +452,9 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   }
   const float tau0 = std::isnan(args->tau0_override) ? c.tau0 : args->tau0_override;
   const bool use_tc = h->bf16 && c.ffn_impl == MOECA_FFN_AUTO;
+  const bool attn = c.n_heads > 0;
+  const int seq = c.seq_len ? c.seq_len : T;
+  if (attn && T % seq) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens must be a multiple of seq_len");
   cudaError_t e = cudaSuccess;
   NvtxRange step_range("moeca_step");
   for (int l = 0; l < c.n_layers; ++l) {
@@ -423,10 +462,46 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     NvtxRange layer_range("layer");
     const void* in = l == 0 ? x_in : h->act[l];
     void* out = l + 1 == c.n_layers ? x_out : h->act[l + 1];
+    const bool attn_full = attn && (refresh || c.attn_policy == 2);
+    const bool attn_sync = attn && !attn_full && c.attn_policy == 0;
+    // The MoE sub-layer's input: the layer input, or u of a DiT-MoE block.
+    const void* moe_in = attn ? L.attn_u : in;
+    ProjArgs qa{};
+    qa.A = in; qa.a_rows = T; qa.B = L.w.w_qkv; qa.bias = L.w.b_qkv;
+    qa.M = T; qa.N = 3 * c.hidden; qa.K = c.hidden; qa.mode = kProjStore;
+    qa.out = h->qkv; qa.ldo = 3 * c.hidden; qa.status = h->status_dev;
+    AttnArgs aa{};
+    aa.qkv = h->qkv; aa.T = T; aa.D = c.hidden; aa.H = c.n_heads; aa.S = seq;
+    aa.o = h->attn_o; aa.status = h->status_dev;
+    ProjArgs oa{};
+    oa.A = h->attn_o; oa.a_rows = T; oa.B = L.w.w_o; oa.bias = L.w.b_o;
+    oa.M = T; oa.N = c.hidden; oa.K = c.hidden; oa.mode = kProjResidual;
+    oa.n_tok = T; oa.x = in; oa.a_out = L.attn_a; oa.u_out = L.attn_u;
+    oa.row_stat = L.stats + kStAttnRows; oa.status = h->status_dev;
+    if (attn_sync) {
+      aa.rows = h->attn_rows; aa.n_rows = h->attn_n;
+      oa.rows = h->attn_rows; oa.m_dev = h->attn_n;
+    }
+    if (attn_full) {
+      // Every token's attention output, before the router sees u = x + a.
+      if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
+    } else if (attn) {
+      // u' = x + a^{t0}: the router input, and the MoE input of every token
+      // that keeps its cached attention.
+      if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
+             return launch_attn_residual(in, L.attn_a, L.attn_u, T, c.hidden, h->status_dev, s);
+           })) != cudaSuccess)
+        break;
+    }
+    // Under the sync rule the rows' inputs change after the decision: the
+    // FFN rows are gathered once the attention update is done.
+    void* xg_now = (use_tc && kGemmGathersRows) || attn_sync ? nullptr : h->xg;
 
     const bool fused = h->prep.tokens_per_block != 0;
     RouterArgs ra{};
-    ra.x = in; ra.w_gate = L.w.w_gate; ra.b_gate = L.w.b_gate;
+    ra.x = moe_in; ra.w_gate = L.w.w_gate; ra.b_gate = L.w.b_gate;
     ra.T = T; ra.D = c.hidden; ra.E = c.n_experts; ra.k = c.top_k;
     ra.renorm = c.renorm_topk; ra.beta = c.beta; ra.tau0 = tau0; ra.alpha = c.alpha;
     ra.entropy_norm = c.entropy_norm;
@@ -451,17 +526,17 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ca.refresh = refresh; ca.shared_policy = c.shared_policy;
     ca.route_e = L.route_e; ca.recompute = L.recompute; ca.slot = L.slot; ca.token_any = L.token_any;
     ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
-    ca.x = in; ca.xg = (use_tc && kGemmGathersRows) ? nullptr : h->xg; ca.status = h->status_dev;
+    ca.x = moe_in; ca.xg = xg_now; ca.status = h->status_dev;
     if (fused) {
       PrepArgs pa{};
-      pa.x = in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
+      pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
       pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
       pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
       pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
       pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.partials = h->partials; pa.tau = L.tau;
       pa.sel = sa;
       pa.block_counts = h->prep_counts; pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
-      pa.xg = h->xg; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
+      pa.xg = xg_now; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
       pa.bar_base = h->prep_arrivals;
       if (h->inject_stall) pa.bar_base += 0x40000000u;  // targets no launch will reach
       if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
@@ -471,12 +546,30 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_COMPACT, s, [&] { return launch_compact(ca, h->bf16, s); })) != cudaSuccess) break;
     }
+    if (attn_sync) {
+      // Sec. 4.1: the tokens with a non-empty recompute set recompute their
+      // attention output over all keys of their sample; their a and u rows
+      // are replaced, then the FFN rows are gathered from u.
+      if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
+             return launch_attn_rows(L.token_any, T, h->attn_rows, h->attn_n, s);
+           })) != cudaSuccess)
+        break;
+      if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
+      if (!(use_tc && kGemmGathersRows)) {
+        CompactArgs ga = ca;
+        ga.xg = h->xg;
+        if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] { return launch_gather(ga, h->bf16, s); })) != cudaSuccess)
+          break;
+      }
+    }
 
     FfnArgs fa{};
     fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;
     fa.max_rows = T * (c.top_k + c.n_shared);
     fa.counts = L.counts; fa.offsets = L.offsets; fa.list = L.list;
-    fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? in : nullptr;
+    fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? moe_in : nullptr;
     fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
     fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
     fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
@@ -497,7 +590,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
 
     CombineArgs cb{};
     cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
-    cb.x = in; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+    cb.x = moe_in; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
     cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
     cb.rearm = use_tc ? h->tc_work : nullptr;
     if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
@@ -538,6 +631,7 @@ moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out) {
     out->shared_recomputed += v[kStSharedRecomputed];
     out->near_margin_route += v[kStNearRoute];
     out->near_margin_score += v[kStNearScore];
+    out->attn_recomputed += v[kStAttnRows];
   }
   volatile int* st = h->status_host;
   out->device_status = st[0];
@@ -568,7 +662,8 @@ moeca_status moeca_get_layer_state(moeca_handle* h, int32_t layer, const moeca_l
   struct { void* d; const void* s; size_t n; } cp[] = {
       {dst->cache_e, L.cache_e, T * k * 4},      {dst->cache_w, L.cache_w, T * k * 4},
       {dst->cache_norm, L.cache_norm, T * k * 4}, {dst->cache_h, L.cache_h, T * k * D * h->es},
-      {dst->shared_h, L.shared_h, T * D * h->es}, {dst->ema, L.ema, T * E * 4}};
+      {dst->shared_h, L.shared_h, T * D * h->es}, {dst->ema, L.ema, T * E * 4},
+      {dst->attn_a, L.attn_a, T * D * h->es}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
@@ -583,7 +678,7 @@ moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_l
   if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
   if (n_tokens < 1 || n_tokens > h->cfg.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of range");
   if (!src->cache_e || !src->cache_w || !src->cache_norm || !src->cache_h || !src->ema ||
-      (h->cfg.n_shared && !src->shared_h))
+      (h->cfg.n_shared && !src->shared_h) || (h->cfg.n_heads && !src->attn_a))
     return fail(h, MOECA_ERR_INVALID_ARG, "every state buffer is required");
   LayerBuf& L = h->layers[layer];
   const size_t T = n_tokens, k = h->cfg.top_k, D = h->cfg.hidden, E = h->cfg.n_experts;
@@ -592,7 +687,8 @@ moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_l
   struct { void* d; const void* s; size_t n; } cp[] = {
       {L.cache_e, src->cache_e, T * k * 4},      {L.cache_w, src->cache_w, T * k * 4},
       {L.cache_norm, src->cache_norm, T * k * 4}, {L.cache_h, src->cache_h, T * k * D * h->es},
-      {L.shared_h, src->shared_h, T * D * h->es}, {L.ema, src->ema, T * E * 4}};
+      {L.shared_h, src->shared_h, T * D * h->es}, {L.ema, src->ema, T * E * 4},
+      {L.attn_a, src->attn_a, T * D * h->es}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
@@ -616,6 +712,7 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
   cudaSetDevice(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const void* in = layer == 0 ? h->last_x_in : h->act[layer];
+  const void* moe_in = h->cfg.n_heads ? L.attn_u : in;
   struct { void* d; const void* s; size_t n; } cp[] = {
       {dst->route_e, L.route_e, T * k * 4}, {dst->route_w, L.route_w, T * k * 4},
       {dst->tau, L.tau, E * 4},             {dst->recompute, L.recompute, T * k},
@@ -623,7 +720,8 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
       {dst->token_any, L.token_any, T},     {dst->counts, L.counts, G * 4},
       {dst->offsets, L.offsets, (G + 1) * 4},
       {dst->list, L.list, T * (k + h->cfg.n_shared) * 4},
-      {dst->layer_in, in, T * D * h->es}};
+      {dst->layer_in, moe_in, T * D * h->es},
+      {dst->block_in, h->cfg.n_heads ? in : nullptr, T * D * h->es}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);

@@ -540,10 +540,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       }
     }
     __syncthreads();
-    // Gather the rows' inputs from the token rows staged in phase A.
+    // Gather the rows' inputs from the token rows staged in phase A (unless
+    // the caller gathers them later: xg null).
     const int nv = D / 8;
     uint4* xg = static_cast<uint4*>(a.xg);
-    const int n = sm_nrows;
+    const int n = xg ? sm_nrows : 0;
     for (int r = warp; r < n; r += kThreads / 32) {
       const uint4* src = reinterpret_cast<const uint4*>(s_x + (sm_rows[r][1] - tok0) * ldw);
       uint4* dst = xg + static_cast<size_t>(sm_rows[r][0]) * nv;

@@ -255,4 +255,11 @@ cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s) {
               : launch_pdl(gather_kernel<float>, dim3(ggrid), dim3(256), 0, s, a);
 }
 
+cudaError_t launch_gather(const CompactArgs& a, bool bf16, cudaStream_t s) {
+  const int rows = a.T * (a.k + a.n_shared);
+  const int ggrid = (rows + 7) / 8;
+  return bf16 ? launch_pdl(gather_kernel<__nv_bfloat16>, dim3(ggrid), dim3(256), 0, s, a)
+              : launch_pdl(gather_kernel<float>, dim3(ggrid), dim3(256), 0, s, a);
+}
+
 }  // namespace moeca

@@ -24,7 +24,9 @@ STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "
                 -6: "TIMEOUT", -7: "DEVICE_STATUS"}
 MOECA_F32, MOECA_BF16 = 0, 1
 MOECA_FFN_AUTO, MOECA_FFN_SIMT = 0, 1
-KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn"]
+KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn",
+                "qkv", "attn", "oproj", "attn_aux"]
+ATTN_SYNC, ATTN_STALE, ATTN_FULL = 0, 1, 2
 
 
 class moeca_config(C.Structure):
@@ -36,12 +38,14 @@ class moeca_config(C.Structure):
                 ("refresh_period", C.c_int32), ("renorm_topk", C.c_int32), ("entropy_norm", C.c_int32),
                 ("shared_policy", C.c_int32), ("reused_meta_policy", C.c_int32),
                 ("gelu_tanh", C.c_int32), ("ffn_impl", C.c_int32), ("ffn_tile_n", C.c_int32),
-                ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32)]
+                ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32),
+                ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):
     _fields_ = [("w_gate", C.c_void_p), ("b_gate", C.c_void_p), ("w1", C.c_void_p),
-                ("w2", C.c_void_p), ("ws1", C.c_void_p), ("ws2", C.c_void_p)]
+                ("w2", C.c_void_p), ("ws1", C.c_void_p), ("ws2", C.c_void_p),
+                ("w_qkv", C.c_void_p), ("b_qkv", C.c_void_p), ("w_o", C.c_void_p), ("b_o", C.c_void_p)]
 
 
 class moeca_step_args(C.Structure):
@@ -54,23 +58,26 @@ class moeca_stats(C.Structure):
         "layer_steps", "refresh_layer_steps", "branches", "cache_step_branches", "matched",
         "recomputed", "reused", "tokens_fully_reused", "shared_recomputed",
         "near_margin_route", "near_margin_score")] + [("device_status", C.c_int32),
-                                                      ("device_detail", C.c_int32)]
+                                                      ("device_detail", C.c_int32),
+                                                      ("attn_recomputed", C.c_int64)]
 
     def as_dict(self) -> dict:
         return {n: getattr(self, n) for n, _ in self._fields_}
 
 
 class moeca_layer_state(C.Structure):
-    _fields_ = [(n, C.c_void_p) for n in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema")]
+    _fields_ = [(n, C.c_void_p) for n in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema",
+                                            "attn_a")]
 
 
 class moeca_layer_trace(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("route_e", "route_w", "tau", "recompute", "slot", "matched",
-                                            "token_any", "counts", "offsets", "list", "layer_in")]
+                                            "token_any", "counts", "offsets", "list", "layer_in",
+                                            "block_in")]
 
 
 class moeca_kernel_times(C.Structure):
-    _fields_ = [("total_ms", C.c_double * 8), ("launches", C.c_int64 * 8)]
+    _fields_ = [("total_ms", C.c_double * 12), ("launches", C.c_int64 * 12)]
 
 
 class moeca_route_args(C.Structure):
@@ -262,6 +269,12 @@ class Stack:
             if cfg.n_shared:
                 lw.ws1 = dev(w["ws1"][0]).data_ptr()
                 lw.ws2 = dev(w["ws2"][0]).data_ptr()
+            if cfg.n_heads:
+                lw.w_qkv = dev(w["w_qkv"]).data_ptr()
+                lw.w_o = dev(w["w_o"]).data_ptr()
+                for name in ("b_qkv", "b_o"):
+                    bt = dev(w.get(name), torch.float32)
+                    setattr(lw, name, bt.data_ptr() if bt is not None else None)
             cl.append(lw)
         self.handle = moeca_create(cfg, cl, device)
 
@@ -299,7 +312,8 @@ class Stack:
                  cache_norm=self._empty((T, c.top_k), torch.float32),
                  cache_h=self._empty((T, c.top_k, c.hidden), self.dtype),
                  shared_h=self._empty((T, c.hidden), self.dtype) if c.n_shared else None,
-                 ema=self._empty((T, c.n_experts), torch.float32))
+                 ema=self._empty((T, c.n_experts), torch.float32),
+                 attn_a=self._empty((T, c.hidden), self.dtype) if c.n_heads else None)
         st = moeca_layer_state(**{k: (v.data_ptr() if v is not None else None) for k, v in t.items()})
         n = moeca_get_layer_state(self.handle, layer, st, self.stream_ptr())
         return {k: (v[:n] if v is not None else None) for k, v in t.items()} | {"n_tokens": n}
@@ -308,7 +322,8 @@ class Stack:
         n = int(state["cache_e"].shape[0])
         keep = {k: v.contiguous() for k, v in state.items() if k != "n_tokens" and v is not None}
         st = moeca_layer_state(**{k: keep[k].data_ptr() if k in keep else None
-                                  for k in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema")})
+                                  for k in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema",
+                                            "attn_a")})
         moeca_set_layer_state(self.handle, layer, st, n, self.stream_ptr())
         self.torch.cuda.current_stream(self.device).synchronize()
 
@@ -322,7 +337,9 @@ class Stack:
                  token_any=self._empty((T,), torch.uint8), counts=self._empty((G,), torch.int32),
                  offsets=self._empty((G + 1,), torch.int32),
                  list=self._empty((T * (k + c.n_shared),), torch.int32),
-                 layer_in=self._empty((T, c.hidden), self.dtype))
+                 layer_in=self._empty((T, c.hidden), self.dtype),
+                 block_in=self._empty((T, c.hidden), self.dtype) if c.n_heads else None)
+        t = {kk: v for kk, v in t.items() if v is not None}
         tr = moeca_layer_trace(**{kk: v.data_ptr() for kk, v in t.items()})
         moeca_get_layer_trace(self.handle, layer, tr, self.stream_ptr())
         return t

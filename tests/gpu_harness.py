@@ -10,6 +10,12 @@ For each layer the oracle gets what the GPU had at the start of that stage:
   compact   the GPU mask                  -> per-group row lists (exact)
   FFN and   the GPU decisions and the     -> layer output, fresh cache rows
   combine   pre-step cache                   (tolerance), kept rows (exact)
+A DiT-MoE block (n_heads > 0) first checks its attention sub-layer:
+  attention the GPU block input x         -> recomputed a rows (tolerance), kept
+                                             a rows (exact), u = bf16(x + a) (exact)
+and the router check then takes the input the rule routes on: u on full
+steps (and under the "stale" and "full" policies), bf16(x + a^{t0}) on a
+sync cache step.
 """
 from __future__ import annotations
 
@@ -48,6 +54,8 @@ class Report:
     recomputed: int = 0
     reused: int = 0
     unmatched: int = 0
+    attn_rows: int = 0
+    max_attn_rel_l2: float = 0.0
     max_rel_l2: float = 0.0
     max_abs: float = 0.0
     notes: list = field(default_factory=list)
@@ -61,7 +69,9 @@ def params_of(cfg) -> O.Params:
         shared_policy="sync" if cfg.shared_policy == 0 else "always",
         reused_meta_policy="keep" if cfg.reused_meta_policy == 0 else "overwrite",
         gelu="tanh" if cfg.gelu_tanh else "erf", score_terms=cfg.score_terms,
-        granularity="branch" if cfg.granularity == 0 else "token")
+        granularity="branch" if cfg.granularity == 0 else "token",
+        n_heads=cfg.n_heads, seq_len=cfg.seq_len, attn_policy=("sync", "stale", "full")[cfg.attn_policy],
+        act_store="bf16" if cfg.dtype == 1 else "f64")
 
 
 def oracle_weights(w: dict) -> dict:
@@ -110,18 +120,62 @@ def expected_lists(e, rec, slot, token_any, E, k, n_shared, refresh, shared_alwa
     return counts, offsets, flat
 
 
+def check_attention(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dict, refresh: bool,
+                    tol: float = 1e-2) -> np.ndarray:
+    """Teacher-forced check of a DiT-MoE block's attention sub-layer (Sec. 4.1).
+
+    bf16 storage of q, k, v, the softmax weights in the p v product and the
+    attention rows bounds the relative L2 error of a fresh a row near 2^-8;
+    ``tol`` allows a few times that.  Returns the router input the oracle
+    must use for this layer."""
+    wo = oracle_weights(w)
+    x = np_of(tr["block_in"]).astype(np.float64)
+    u = np_of(tr["layer_in"]).astype(np.float64)
+    a_post = np_of(post["attn_a"]).astype(np.float64)
+    T = x.shape[0]
+    full = refresh or cfg.attn_policy == 2
+    has_pre = pre is not None and pre["n_tokens"]
+    a_pre = np_of(pre["attn_a"]).astype(np.float64) if has_pre else None
+    if full:
+        rows = np.arange(T)
+    elif cfg.attn_policy == 1:
+        rows = np.zeros(0, np.int64)
+    else:
+        rows = np.nonzero(np_of(tr["token_any"]))[0]
+    if len(rows):
+        a_o = O.attention(x, wo["w_qkv"], wo.get("b_qkv"), wo["w_o"], wo.get("b_o"), cfg.n_heads, cfg.seq_len, rows)
+        rl = rel_l2(a_post[rows], a_o)
+        rep.max_attn_rel_l2 = max(rep.max_attn_rel_l2, rl)
+        assert rl <= tol, f"attention rows rel L2 {rl:.3e}"
+        per_row = np.linalg.norm(a_post[rows] - a_o, axis=1) / np.maximum(np.linalg.norm(a_o, axis=1), 1e-30)
+        assert per_row.max() <= 4 * tol, f"worst attention row rel L2 {per_row.max():.3e}"
+    kept = np.setdiff1d(np.arange(T), rows)
+    if len(kept):
+        assert a_pre is not None, "a cache step without a cached attention output"
+        assert np.array_equal(a_post[kept], a_pre[kept]), "kept attention rows changed"
+    assert np.array_equal(u, O.round_bf16(x + a_post)), "MoE input u differs from bf16(x + a)"
+    rep.attn_rows += len(rows)
+    if full or cfg.attn_policy == 1:
+        return u
+    return O.round_bf16(x + a_pre)
+
+
 def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dict, out_gpu: np.ndarray,
-                refresh: bool, bf16: bool, out_tol=None):
-    """Teacher-forced comparison of one layer step.  Raises AssertionError."""
+                refresh: bool, bf16: bool, out_tol=None, route_in=None):
+    """Teacher-forced comparison of one layer step.  Raises AssertionError.
+
+    ``route_in`` is the router input when it differs from the FFN input
+    (a DiT-MoE block on a sync cache step)."""
     T = tr["route_e"].shape[0]
     D, E, k, S = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.n_shared
     prm = params_of(cfg)
     wo = oracle_weights(w)
     u = np_of(tr["layer_in"]).astype(np.float64)
+    u_route = u if route_in is None else np.asarray(route_in, np.float64)
     e_g = np_of(tr["route_e"]).astype(np.int64)
     w_g = np_of(tr["route_w"]).astype(np.float64)
     # ---- router (Eq. 7)
-    e_o, w_o, near, cond = O.route(u, wo["w_gate"], wo.get("b_gate"), k, prm.renorm_topk)
+    e_o, w_o, near, cond = O.route(u_route, wo["w_gate"], wo.get("b_gate"), k, prm.renorm_topk)
     ok = near >= NEAR
     rep.near_route += int((~ok).sum())
     bad = np.nonzero(ok & (e_o != e_g).any(axis=1))[0]
@@ -215,14 +269,17 @@ def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True
         out = stack.step(xd, t, force_refresh=force)
         torch.cuda.synchronize()
         if check:
+            block = cfg.n_heads > 0
             for l in range(L):
                 tr = stack.get_trace(l, T)
                 post = stack.get_state(l)
                 if l + 1 < L:
-                    out_l = np_of(stack.get_trace(l + 1, T)["layer_in"]).astype(np.float64)
+                    out_l = np_of(stack.get_trace(l + 1, T)["block_in" if block else "layer_in"]).astype(np.float64)
                 else:
                     out_l = np_of(out).astype(np.float64)
-                check_layer(rep, cfg, layer_weights[l], pre[l], post, tr, out_l, refresh, bf16, out_tol)
+                route_in = check_attention(rep, cfg, layer_weights[l], pre[l], post, tr, refresh) if block else None
+                check_layer(rep, cfg, layer_weights[l], pre[l], post, tr, out_l, refresh, bf16, out_tol,
+                            route_in=route_in)
         rep.steps += 1
         prev_T = T
     return rep, out

@@ -30,6 +30,7 @@ def test_status_strings_and_defaults(lib):
     assert abs(cfg.tau0 - 0.8) < 1e-7 and abs(cfg.alpha - 0.6) < 1e-7 and abs(cfg.beta - 0.65) < 1e-7
     assert cfg.renorm_topk == 1 and cfg.gelu_tanh == 1 and cfg.dtype == lib.MOECA_BF16
     assert cfg.score_terms == 7 and cfg.granularity == 0
+    assert (cfg.n_heads, cfg.seq_len, cfg.attn_policy) == (0, 0, lib.ATTN_SYNC)
 
 
 def test_host_validation_needs_no_gpu(lib):
@@ -54,3 +55,25 @@ def test_host_validation_needs_no_gpu(lib):
     assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -2  # hidden not a multiple of 8
     assert L.moeca_step(None, None, None, None, None) == -1
     assert L.moeca_destroy(None) == 0
+
+
+def test_attention_config_validation_needs_no_gpu(lib):
+    """DiT-MoE block settings are checked before any device call."""
+    L = lib.LIB
+    h = ctypes.c_void_p()
+    w = (lib.moeca_layer_weights * 1)()
+    w[0].w_gate = w[0].w1 = w[0].w2 = 4096
+
+    def create(**kw):
+        base = dict(n_layers=1, hidden=768, ffn=256, n_experts=4, top_k=2, max_tokens=8)
+        base.update(kw)
+        c = lib.moeca_config_default(**base)
+        return L.moeca_create(ctypes.byref(c), w, 0, ctypes.byref(h))
+
+    for bad in (dict(n_heads=-1), dict(seq_len=-2), dict(attn_policy=3), dict(n_heads=12, attn_policy=-1)):
+        assert create(**bad) == lib.MOECA_ERR_INVALID_ARG, bad
+    assert create(n_heads=12, dtype=lib.MOECA_F32) == lib.MOECA_ERR_UNSUPPORTED   # bf16 only
+    assert create(n_heads=7) == lib.MOECA_ERR_UNSUPPORTED                      # 768 / 7 not a head size
+    assert create(n_heads=24) == lib.MOECA_ERR_UNSUPPORTED                     # 32 channels per head
+    assert create(n_heads=12) == lib.MOECA_ERR_INVALID_ARG                     # no attention weights
+    assert b"attention weights" in L.moeca_last_error(None)

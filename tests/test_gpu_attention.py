@@ -1,0 +1,146 @@
+"""GPU vs oracle parity of the DiT-MoE block's attention path (Sec. 4.1),
+through the C ABI (marked gpu).
+
+Every layer of every step is teacher-forced (see gpu_harness): the oracle's
+attention of the GPU's block input must match the recomputed a rows, the
+kept rows must be untouched, u must equal bf16(x + a), and the MoE
+sub-layer is then checked with the router input the sync rule prescribes.
+Cases cover every built head size (64, 72, 80, 96, 128), samples that are
+ragged against the 64-row query blocks and the 128-row GEMM tiles, one
+sample per step (seq_len 0), the three attention policies, a shared expert,
+the full-size 12-head block of the D 768 stack, and degenerate steps.
+"""
+import math
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from gpu_harness import np_of, run_trajectory  # noqa: E402
+from paper_2606_15615_gb300 import workloads as W  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def M():
+    if not torch.cuda.is_available():
+        pytest.fail("a CUDA GPU is required for gpu-marked tests")
+    from paper_2606_15615_gb300 import build
+    build.build()
+    from paper_2606_15615_gb300 import moeca
+    return moeca
+
+
+def drift(x0, rng, n, sigma):
+    xs = [x0]
+    for _ in range(1, n):
+        xs.append((xs[-1] + sigma * rng.standard_normal(x0.shape)).astype(np.float32))
+    return [W.round_to_bf16(x) for x in xs]
+
+
+def make_block_stack(M, T, D, H, E, k, F, L=1, S=0, n_shared=0, seed=0, wscale=0.05, **cfg_kw):
+    ws = []
+    for l in range(L):
+        w, _, _ = W.tiny_layer(300 + 10 * seed + l, T, D, E, k, F, n_shared=n_shared, dtype="bf16",
+                               bias=n_shared > 0, wscale=wscale)
+        w.update(W.tiny_attn(300 + 10 * seed + l, D, dtype="bf16", wscale=wscale))
+        ws.append(w)
+    cfg = M.moeca_config_default(n_layers=L, hidden=D, ffn=F, n_experts=E, top_k=k, n_shared=n_shared,
+                                 max_tokens=cfg_kw.pop("max_tokens", T), dtype=M.MOECA_BF16,
+                                 n_heads=H, seq_len=S, **cfg_kw)
+    return M.Stack(cfg, ws), cfg, ws
+
+
+@pytest.mark.parametrize("D,H,S,T", [(256, 4, 200, 400), (576, 8, 100, 300), (320, 4, 72, 216),
+                                     (384, 4, 130, 260), (384, 3, 96, 384)])
+def test_sync_blocks_every_head_size(M, D, H, S, T):
+    """Heads of 64, 72, 80, 96 and 128 channels; samples ragged against the
+    64-row query blocks and the 128-row tiles; two layers; a full step every 3."""
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=D + H, tau0=0.72, refresh_period=3)
+    rng = np.random.default_rng(D + H)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 5, 0.08)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    cache_rows = rep.attn_rows - 2 * 2 * T          # full steps 0 and 3, two layers
+    assert rep.reused > 0 and rep.recomputed > 0
+    assert 0 < cache_rows < 2 * 3 * T, rep          # some, not all, tokens recompute attention
+    stats = st.stats()
+    assert stats["attn_recomputed"] == rep.attn_rows
+    st.close()
+
+
+@pytest.mark.parametrize("policy", [1, 2])
+def test_stale_and_full_policies(M, policy):
+    """Table 4's "without sync update" (attention reused on every cache step)
+    and the always-recompute policy that routes on the fresh input."""
+    T, D, H, S = 256, 256, 4, 128
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=7, tau0=0.72, attn_policy=policy)
+    rng = np.random.default_rng(70 + policy)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.08)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    assert rep.attn_rows == (2 * T if policy == 1 else 2 * 4 * T)
+    assert rep.reused > 0
+    st.close()
+
+
+def test_one_sample_shared_expert(M):
+    """seq_len 0 (every token attends to all T rows) with a shared expert
+    under the synchronized rule."""
+    T, D, H = 300, 256, 2
+    st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 192, L=1, S=0, n_shared=1, seed=8, tau0=0.7)
+    rng = np.random.default_rng(80)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    assert rep.reused > 0 and rep.attn_rows > T
+    st.close()
+
+
+def test_block_full_size_d768_12_heads(M):
+    """The 12-head block of the D 768 stack at full size (T 2048 = 8 samples
+    of 256, E 16, top-2, F 3072), two of its layers, three steps."""
+    wl = W.workload("dit_d768_h12_e16_k2_f3072_t2048_l12_bf16")
+    ws = []
+    for l in range(2):
+        w = W.make_layer_weights(wl, l)
+        w.update(W.make_attn_weights(wl, l))
+        ws.append(w)
+    cfg = M.moeca_config_default(n_layers=2, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts,
+                                 top_k=wl.top_k, max_tokens=wl.n_tokens, dtype=M.MOECA_BF16,
+                                 n_heads=wl.n_heads, seq_len=wl.seq, tau0=0.665)
+    st = M.Stack(cfg, ws)
+    xs = list(W.trajectory(wl, n_steps=3))
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    assert rep.reused > 0 and 2 * 2 * wl.n_tokens > rep.attn_rows - 2 * wl.n_tokens > 0
+    st.close()
+
+
+def test_repeated_input_all_reused_is_bitwise_previous_output(M):
+    """tau0 = +inf with the same input: no branch and no attention row is
+    recomputed and the output repeats the previous step exactly."""
+    T, D, H, S = 200, 256, 4, 100
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=9, tau0=math.inf)
+    rng = np.random.default_rng(90)
+    x = torch.from_numpy(W.round_to_bf16(rng.standard_normal((T, D)).astype(np.float32))).cuda().to(torch.bfloat16)
+    o0 = st.step(x, 0).clone()
+    o1 = st.step(x, 1).clone()
+    torch.cuda.synchronize()
+    assert torch.equal(o0, o1)
+    s = st.stats()
+    assert s["attn_recomputed"] == 2 * T and s["reused"] == 2 * T * 2
+    st.close()
+
+
+def test_token_count_change_and_empty_step(M):
+    """A new T forces a full step (every token's attention); T = 0 is a no-op."""
+    D, H, S = 256, 4, 64
+    st, cfg, ws = make_block_stack(M, 256, D, H, 8, 2, 256, L=1, S=S, seed=10, tau0=0.72)
+    rng = np.random.default_rng(100)
+    a = drift(rng.standard_normal((256, D)).astype(np.float32), rng, 2, 0.05)
+    b = drift(rng.standard_normal((128, D)).astype(np.float32), rng, 2, 0.05)
+    flags = []
+    rep, _ = run_trajectory(st, cfg, ws, a + b, refresh_flags=flags)
+    assert flags == [True, False, True, False]
+    st.step(torch.empty((0, D), dtype=torch.bfloat16, device="cuda"), 9)
+    with pytest.raises(M.MoecaError):
+        st.step(torch.zeros((100, D), dtype=torch.bfloat16, device="cuda"), 10)   # not a multiple of 64
+    st.close()
