@@ -22,6 +22,7 @@ import hashlib
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -34,7 +35,7 @@ if ROOT not in sys.path:
 METRIC = "branch-cached MoE layer tokens/s and effective TFLOP/s vs reuse ratio; % roofline"
 DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn"]
+KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn", "qkv", "attn", "oproj", "attn_aux"]
 
 
 # ---------------------------------------------------------------------------
@@ -154,10 +155,20 @@ def peaks():
 
 
 def kernel_source_sha(kind: str) -> str:
+    """First 16 hex digits of sha256 over the kernel's .cu file and the local
+    headers it includes (so a recorded ncu figure expires with the code)."""
     fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "ffn": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
-             "compact": "select.cu", "combine": "combine.cu", "prep": "prep.cu"}[kind]
-    with open(os.path.join(ROOT, "paper_2606_15615_gb300", "csrc", fname), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+             "compact": "select.cu", "combine": "combine.cu", "prep": "prep.cu", "qkv": "proj_tc.cu",
+             "oproj": "proj_tc.cu", "attn": "attention.cu", "attn_aux": "attention.cu"}[kind]
+    csrc = os.path.join(ROOT, "paper_2606_15615_gb300", "csrc")
+    h = hashlib.sha256()
+    with open(os.path.join(csrc, fname), "rb") as f:
+        src = f.read()
+    h.update(src)
+    for inc in sorted(set(re.findall(rb'#include "([^"]+\.cuh)"', src))):
+        with open(os.path.join(csrc, inc.decode()), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def recorded_traffic(kind: str, workload: str, reuse_target: float):
@@ -196,7 +207,7 @@ class Runner:
             n_layers=wl.n_layers, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts, top_k=wl.top_k,
             n_shared=wl.n_shared, max_tokens=wl.n_tokens,
             dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period,
-            ffn_tile_n=tile_n, ffn_split_k=split_k)
+            ffn_tile_n=tile_n, ffn_split_k=split_k, n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
         self.cfg = cfg
         self.stack = M.Stack(cfg, self.weights, device=device_index)
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -270,10 +281,21 @@ class Runner:
         return best
 
 
-def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float):
-    """Algorithmic (bytes, flops) of one launch of a kernel kind for this workload."""
+def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float, attn_rows: float = 0.0):
+    """Algorithmic (bytes, flops) of one launch of a kernel kind for this workload.
+
+    ``attn_rows`` is the mean number of token rows one attention launch
+    computes (every token on a full step, the recomputing tokens otherwise)."""
     T, D, E, k, F, S = wl.n_tokens, wl.hidden, wl.n_experts, wl.top_k, wl.ffn, wl.n_shared
     es = 2 if wl.dtype == "bf16" else 4
+    if kind == "qkv":      # x [T, D] and W_qkv [3D, D] in, q | k | v [T, 3D] out
+        return T * D * es + 3 * D * D * es + 3 * D * 4 + 3 * T * D * es, 2.0 * T * D * 3 * D
+    if kind == "attn":     # q rows, every key and value row once, o rows
+        return 2 * attn_rows * D * es + 2 * T * D * es, 4.0 * attn_rows * wl.seq * D
+    if kind == "oproj":    # o rows and W_o in; x rows in; a and u rows out
+        return 4 * attn_rows * D * es + D * D * es + D * 4, 2.0 * attn_rows * D * D
+    if kind == "attn_aux":  # u = x + a^{t0} (x, a in, u out), the token list, the FFN row gather
+        return 3 * T * D * es + T + rows_per_launch * 2 * D * es, 0.0
     if kind == "router":
         return T * D * es + E * D * es + T * E * 8 + T * k * 8, 2.0 * T * D * E
     if kind == "select":
@@ -306,7 +328,8 @@ def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
     w = {k: (None if v is None else v.float().cpu().numpy().astype(np.float64)) for k, v in runner.weights[0].items()}
     if w["ws1"] is None:
         w["ws1"] = w["ws2"] = None
-    prm = O.Params(top_k=wl.top_k, tau0=tau0 if math.isfinite(tau0) else tau0, refresh_period=wl.refresh_period)
+    prm = O.Params(top_k=wl.top_k, tau0=tau0 if math.isfinite(tau0) else tau0, refresh_period=wl.refresh_period,
+                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
     st = O.Stack([w], prm, wl.hidden, wl.n_experts, wl.n_shared)
     xs = runner.x_host.float().numpy()
     st.step(xs[0], 0)
@@ -344,8 +367,12 @@ def reference_arm(args, wl):
     from paper_2606_15615_gb300 import workloads as W
     rng_layers = min(wl.n_layers, 2)
     ws = [W.make_layer_weights(wl, l) for l in range(rng_layers)]
+    if wl.n_heads:
+        for l in range(rng_layers):
+            ws[l].update(W.make_attn_weights(wl, l))
     xs = list(W.trajectory(wl, args.warmup + args.steps + 1))
-    prm = O.Params(top_k=wl.top_k, tau0=args.ref_tau0, refresh_period=wl.refresh_period)
+    prm = O.Params(top_k=wl.top_k, tau0=args.ref_tau0, refresh_period=wl.refresh_period,
+                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
     stacks = [O.Stack([ws[l]], prm, wl.hidden, wl.n_experts, wl.n_shared) for l in range(rng_layers)]
     for t in range(args.warmup):
         stacks[t % rng_layers].step(xs[t], t)
@@ -438,6 +465,11 @@ def main():
         tps = tokens_all / (ms / 1e3)
         executed = (st["recomputed"] + st["shared_recomputed"]) * 4.0 * wl.hidden * wl.ffn  # per rank, K steps
         dense = wl.dense_flops_per_layer() * wl.n_layers * K
+        if wl.n_heads:
+            D, T = wl.hidden, wl.n_tokens
+            executed += (2.0 * T * D * 3 * D * wl.n_layers * K
+                         + st["attn_recomputed"] * (4.0 * wl.seq * D + 2.0 * D * D))
+            dense += (2.0 * T * D * 3 * D + T * (4.0 * wl.seq * D + 2.0 * D * D)) * wl.n_layers * K
         row = {"reuse_target": tgt, "reuse_achieved": round(runner.reuse_of(st), 4),
                "tau0": None if not math.isfinite(tau0) else round(tau0, 5), "tokens_per_s": tps,
                "ms_per_step": ms / K, "effective_tflops": dense * world / (ms / 1e3) / 1e12,
@@ -454,10 +486,11 @@ def main():
     e2e_reps = [runner._run(head["tau0_raw"], W_, K, e2e=True)[0] for _ in range(max(1, args.reps))]
     e2e_ms, _ = aggregate(statistics.median(e2e_reps), 0, dist, dev)
     rows_per_launch = (st_k["recomputed"] + st_k["shared_recomputed"]) / (K * wl.n_layers)
+    attn_rows = st_k["attn_recomputed"] / max(kt["attn"][1], 1)
     kernels = {}
     for kind in KINDS:
         tot, n = kt[kind]
-        nb, nf = algorithmic(kind, wl, rows_per_launch, wl.n_experts + wl.n_shared)
+        nb, nf = algorithmic(kind, wl, rows_per_launch, wl.n_experts + wl.n_shared, attn_rows)
         avg = tot / max(n, 1)
         kernels[kind] = {"launches": n, "avg_us": avg * 1e3, "share": tot / max(sum(v[0] for v in kt.values()), 1e-12),
                          "alg_bytes": nb, "alg_flops": nf,
@@ -490,6 +523,9 @@ def main():
         "config": {"workload": wl.name, "tokens": wl.n_tokens, "hidden": wl.hidden, "experts": wl.n_experts,
                    "shared_experts": wl.n_shared, "top_k": wl.top_k, "ffn": wl.ffn, "layers": wl.n_layers,
                    "refresh_period": wl.refresh_period, "reuse_target": args.reuse,
+                   **({"attn_heads": wl.n_heads, "seq_len": wl.seq,
+                       "attn_rows_recomputed_per_step": head["stats"]["attn_recomputed"] / K}
+                      if wl.n_heads else {}),
                    "reuse_achieved": head["reuse_achieved"], "tau0": head["tau0"],
                    "effective_tflops": head["effective_tflops"], "executed_tflops": head["executed_tflops"],
                    "timed": f"median of {args.reps} reps of {K} steps after {W_} warm-up steps (step 0 full)",

@@ -53,17 +53,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// First index in rows[0, n) whose token is >= key (rows ascending).
-__device__ __forceinline__ int lower_bound(const int32_t* rows, int n, int key) {
-  int lo = 0, hi = n;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (rows[mid] < key) lo = mid + 1;
-    else hi = mid;
-  }
-  return lo;
-}
-
 __global__ void __launch_bounds__(256) attn_residual_kernel(const uint4* x, const uint4* a, uint4* u, size_t nvec) {
   pdl_entry();
   for (size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
@@ -82,7 +71,10 @@ __global__ void __launch_bounds__(256) attn_residual_kernel(const uint4* x, cons
 }
 
 // One block of 1024 threads: thread j scans tokens [j per, (j + 1) per).
-__global__ void __launch_bounds__(1024) attn_rows_kernel(const uint8_t* any, int T, int32_t* rows, int* n_rows) {
+// Also writes where each sample's tokens start in the list (sample_lo[b] for
+// sample b of S tokens, sample_lo[T / S] = the list's length).
+__global__ void __launch_bounds__(1024) attn_rows_kernel(const uint8_t* any, int T, int S, int32_t* rows,
+                                                         int* n_rows, int32_t* sample_lo) {
   pdl_entry();
   __shared__ int warp_tot[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -109,18 +101,32 @@ __global__ void __launch_bounds__(1024) attn_rows_kernel(const uint8_t* any, int
   }
   __syncthreads();
   int pos = incl - c + (warp ? warp_tot[warp - 1] : 0);
-  for (int i = beg; i < end; ++i)
+  for (int i = beg; i < end; ++i) {
+    if (i % S == 0) sample_lo[i / S] = pos;
     if (any[i]) rows[pos++] = i;
-  if (tid == 1023) *n_rows = warp_tot[31];
+  }
+  if (tid == 1023) {
+    *n_rows = warp_tot[31];
+    sample_lo[T / S] = warp_tot[31];
+  }
 }
 
-// Shared memory of attn_core_kernel<DH>: Q [64][DK + 8], K [2][64][DK + 8],
-// V [2][64][DH + 8] (bf16; 16 bytes of padding per row keep ldmatrix free
+// Key / value blocks in flight: a ring of NBUF blocks of 64 keys, NBUF - 1
+// loading while one is used (a 256-key sample arrives in one round trip for
+// heads up to 80 channels); two CTAs still fit on an SM.
+template <int DH>
+__host__ __device__ constexpr int core_nbuf() {
+  return DH <= 80 ? 4 : (DH <= 96 ? 3 : 2);
+}
+
+// Shared memory of attn_core_kernel<DH>: Q [64][DK + 8], K [NBUF][64][DK + 8],
+// V [NBUF][64][DH + 8] (bf16; 16 bytes of padding per row keep ldmatrix free
 // of bank conflicts).  DK = DH rounded up to 16 (the q k^T contraction).
 template <int DH>
 constexpr size_t core_smem() {
   constexpr int DK = (DH + 15) / 16 * 16;
-  return (static_cast<size_t>(kQRows) * (DK + 8) + 2 * kKeys * (DK + 8) + 2 * kKeys * (DH + 8)) * 2;
+  constexpr int NB = core_nbuf<DH>();
+  return (static_cast<size_t>(kQRows) * (DK + 8) + NB * kKeys * (DK + 8) + NB * kKeys * (DH + 8)) * 2;
 }
 
 template <int DH>
@@ -129,10 +135,11 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
   constexpr int LDQ = DK + 8, LDV = DH + 8;
   constexpr int NT = DH / 8;   // 8-column tiles of the output
   constexpr int CH = DH / 8;   // 16-byte chunks of one head row
+  constexpr int NB = core_nbuf<DH>();
   extern __shared__ __align__(16) uint8_t smem[];
   __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(smem);
   __nv_bfloat16* sK = sQ + kQRows * LDQ;
-  __nv_bfloat16* sV = sK + 2 * kKeys * LDQ;
+  __nv_bfloat16* sV = sK + NB * kKeys * LDQ;
   __shared__ int s_tok[kQRows];
 
   pdl_entry();
@@ -142,9 +149,8 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
   const int key0 = b * S;
   int lo = key0, hi = key0 + S;
   if (a.rows) {
-    const int n = *reinterpret_cast<const volatile int*>(a.n_rows);
-    lo = lower_bound(a.rows, n, key0);
-    hi = lower_bound(a.rows, n, key0 + S);
+    lo = a.sample_lo[b];
+    hi = a.sample_lo[b + 1];
   }
   const int r0 = lo + blockIdx.x * kQRows;
   if (r0 >= hi) return;
@@ -162,7 +168,7 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
   }
   if (DK > DH) {
     // Columns DH..DK of the q and k rows take part in q k^T: keep them 0.
-    for (int i = tid; i < kQRows + 2 * kKeys; i += kCoreThreads) {
+    for (int i = tid; i < kQRows + NB * kKeys; i += kCoreThreads) {
       __nv_bfloat16* row = i < kQRows ? sQ + i * LDQ : sK + (i - kQRows) * LDQ;
 #pragma unroll
       for (int c = DH; c < DK; ++c) row[c] = __float2bfloat16_rn(0.f);
@@ -186,10 +192,14 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
       cp_async16(smem_u32(sV + (buf * kKeys + r) * LDV + c * 8), src + D, v);
     }
   };
-  load_kv(0, 0);
-  cp_async_commit();
-
   const int nkb = (S + kKeys - 1) / kKeys;
+  // Groups: block 0 (with q), then one per block; empty groups keep the count.
+#pragma unroll
+  for (int j = 0; j < NB - 1; ++j) {
+    if (j < nkb) load_kv(j, j);
+    cp_async_commit();
+  }
+
   const int g = lane >> 2, q4 = lane & 3;
   const int mat = lane >> 3, mr = lane & 7;
   float o[NT][4];
@@ -199,13 +209,9 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
   uint32_t qf[DK / 16][4];
 
   for (int kb = 0; kb < nkb; ++kb) {
-    if (kb + 1 < nkb) {
-      load_kv(kb + 1, (kb + 1) & 1);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
+    if (kb + NB - 1 < nkb) load_kv(kb + NB - 1, (kb + NB - 1) % NB);
+    cp_async_commit();
+    cp_async_wait<NB - 1>();  // block kb (and q) have landed
     __syncthreads();
     if (kb == 0) {
 #pragma unroll
@@ -213,8 +219,8 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
         ldsm_x4(smem_u32(sQ + (warp * 16 + (mat & 1) * 8 + mr) * LDQ + kc * 16 + (mat >> 1) * 8), qf[kc][0],
                 qf[kc][1], qf[kc][2], qf[kc][3]);
     }
-    const __nv_bfloat16* kbuf = sK + (kb & 1) * kKeys * LDQ;
-    const __nv_bfloat16* vbuf = sV + (kb & 1) * kKeys * LDV;
+    const __nv_bfloat16* kbuf = sK + (kb % NB) * kKeys * LDQ;
+    const __nv_bfloat16* vbuf = sV + (kb % NB) * kKeys * LDV;
     // ---- scores of this warp's 16 rows against 64 keys
     float s[8][4];
 #pragma unroll
@@ -351,8 +357,9 @@ cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, i
                     static_cast<const uint4*>(a), static_cast<uint4*>(u), nvec);
 }
 
-cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int32_t* rows, int* n_rows, cudaStream_t s) {
-  return launch_pdl(attn_rows_kernel, dim3(1), dim3(1024), 0, s, token_any, T, rows, n_rows);
+cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int S, int32_t* rows, int* n_rows,
+                             int32_t* sample_lo, cudaStream_t s) {
+  return launch_pdl(attn_rows_kernel, dim3(1), dim3(1024), 0, s, token_any, T, S, rows, n_rows, sample_lo);
 }
 
 }  // namespace moeca

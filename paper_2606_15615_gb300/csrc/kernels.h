@@ -151,6 +151,13 @@ struct PrepArgs {
   int32_t* offsets;       // [G + 1]
   int32_t* list;          // [rows]
   void* xg;               // [rows, D], or null: the rows are gathered later (launch_gather)
+  const void* attn_a;     // DiT-MoE block cache step: [T, D] cached attention rows a^{t0}, or null;
+                          // then the rows staged from x become u = x + a^{t0}, written to u_out
+  void* u_out;            // [T, D]
+  int gather_final_only;  // 1: gather only the rows of tokens without recomputed branches
+  int32_t* row_of;        // or null: [T, k + n_shared] list position of each branch's row
+                          // (p < k routed, p = k shared), -1 when not recomputed
+  int n_shared;
   unsigned* gbar;         // grid barrier arrival counter (zeroed once, only grows)
   unsigned bar_base;      // arrivals on gbar from earlier launches (mod 2^32)
   unsigned long long* stats;
@@ -163,7 +170,7 @@ struct PrepShape {
   size_t smem;            // dynamic shared memory per block
 };
 constexpr size_t kPrepSmemMax = 200 * 1024;
-PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms);
+PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn);
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 
 // Eq. 8 combine + residual + cached branch norms.
@@ -192,6 +199,7 @@ struct ProjArgs {
   const void* B;          // [N, K] bf16 weights
   const float* bias;      // [N] or null
   int M, N, K;            // N a multiple of 64, K of 64
+  int tile_n;             // output tile width (0: the widest of 256 / 128 / 64 dividing N)
   const int* m_dev;       // device row count (<= M), or null
   int mode;               // ProjMode
   void* out;              // kProjStore: [M, ldo] bf16
@@ -202,17 +210,24 @@ struct ProjArgs {
   void* a_out;            // kProjResidual: [n_tok, N]  a_i
   void* u_out;            // kProjResidual: [n_tok, N]  x_i + a_i
   unsigned long long* row_stat;  // or null: the launch adds its row count here
+  const int32_t* row_of;  // kProjResidual, or null: [n_tok, row_w] FFN row positions of the token
+  int row_w;              //   (-1: none); u is also written to those rows of xg
+  void* xg;               // [rows, N] FFN input rows
   int* status;
 };
-int proj_tile_n(int N);   // tile width the launch uses for N (0: N not a multiple of 64)
+// Tile width a launch uses for N: `want` (64 / 128 / 256) if it divides N,
+// else (want = 0) the widest that does; 0 when none fits.
+int proj_tile_n(int N, int want);
 cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s);
 
 // u = x + a, row by row (the MoE input of a token that keeps its cached attention).
 cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, int D, int* status,
                                  cudaStream_t s);
 
-// Ascending list of tokens whose recompute set is non-empty, and its length.
-cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int32_t* rows, int* n_rows, cudaStream_t s);
+// Ascending list of tokens whose recompute set is non-empty, its length, and
+// where each sample's tokens start in it (sample_lo [T / S + 1]).
+cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int S, int32_t* rows, int* n_rows,
+                             int32_t* sample_lo, cudaStream_t s);
 
 // Multi-head self-attention rows: o[r] = concat_h softmax(q_t k_S^T / sqrt(dh)) v_S for the
 // r-th listed token t, keys and values of t's sample (S consecutive token rows).
@@ -220,7 +235,7 @@ struct AttnArgs {
   const void* qkv;        // [T, 3D] bf16: q | k | v, head h at columns h dh .. of each
   int T, D, H, S;         // S tokens per sample, T a multiple of S
   const int32_t* rows;    // ascending token list, or null: every token (row r = token r)
-  const int* n_rows;      // device length of rows (when rows is set)
+  const int32_t* sample_lo;  // with rows: sample b's tokens are rows[sample_lo[b] .. sample_lo[b + 1])
   void* o;                // [rows, D] bf16
   int* status;
 };

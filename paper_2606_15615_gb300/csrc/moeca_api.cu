@@ -102,6 +102,8 @@ struct moeca_handle {
   void* attn_o = nullptr;       // [T, D] attention rows before the output projection
   int32_t* attn_rows = nullptr; // [T] tokens that recompute their attention
   int* attn_n = nullptr;        // their count
+  int32_t* attn_samp = nullptr; // [T + 1] where each sample's tokens start in attn_rows
+  int32_t* attn_rowof = nullptr; // [T, k + n_shared] FFN row of each branch (fused sync path)
   std::vector<void*> act;  // input of layer l (l >= 1)
   int* status_host = nullptr;
   int* status_dev = nullptr;
@@ -357,6 +359,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     A(&h->attn_o, T * D * es);
     A((void**)&h->attn_rows, T * 4);
     A((void**)&h->attn_n, 16);
+    A((void**)&h->attn_samp, (T + 1) * 4);
+    A((void**)&h->attn_rowof, T * (k + c.n_shared) * 4);
   }
   const size_t nblk_router = (T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
   const size_t nblk_sel = (T + kSelectTokensPerBlock - 1) / kSelectTokensPerBlock;
@@ -372,7 +376,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     h->tc_dep_pairs_n = static_cast<int>(tc_dep_pairs(h->max_rows, h->G));
     A((void**)&h->tc_dep, static_cast<size_t>(h->tc_dep_pairs_n) * 2 * sizeof(int));
     A((void**)&h->tc_work, 2 * sizeof(int));
-    h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms);
+    h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms, attn);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
       A((void**)&h->prep_counts, nb * G * 4);
@@ -476,10 +480,14 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ProjArgs oa{};
     oa.A = h->attn_o; oa.a_rows = T; oa.B = L.w.w_o; oa.bias = L.w.b_o;
     oa.M = T; oa.N = c.hidden; oa.K = c.hidden; oa.mode = kProjResidual;
+    // Narrow tiles: the recomputed rows are few and the residual epilogue
+    // (x in; a, u and the FFN rows out) is latency-bound, so more CTAs with
+    // two 32-column chunks each beat fewer wide ones.
+    oa.tile_n = 64;
     oa.n_tok = T; oa.x = in; oa.a_out = L.attn_a; oa.u_out = L.attn_u;
     oa.row_stat = L.stats + kStAttnRows; oa.status = h->status_dev;
     if (attn_sync) {
-      aa.rows = h->attn_rows; aa.n_rows = h->attn_n;
+      aa.rows = h->attn_rows; aa.sample_lo = h->attn_samp;
       oa.rows = h->attn_rows; oa.m_dev = h->attn_n;
     }
     if (attn_full) {
@@ -487,9 +495,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
-    } else if (attn) {
+    } else if (attn && h->prep.tokens_per_block == 0) {
       // u' = x + a^{t0}: the router input, and the MoE input of every token
-      // that keeps its cached attention.
+      // that keeps its cached attention (the fused preparation kernel forms
+      // it itself while staging the rows).
       if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
              return launch_attn_residual(in, L.attn_a, L.attn_u, T, c.hidden, h->status_dev, s);
            })) != cudaSuccess)
@@ -497,7 +506,8 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     }
     // Under the sync rule the rows' inputs change after the decision: the
     // FFN rows are gathered once the attention update is done.
-    void* xg_now = (use_tc && kGemmGathersRows) || attn_sync ? nullptr : h->xg;
+    const bool xg_gather = !(use_tc && kGemmGathersRows);  // the FFN reads gathered rows
+    void* xg_now = !xg_gather || attn_sync ? nullptr : h->xg;
 
     const bool fused = h->prep.tokens_per_block != 0;
     RouterArgs ra{};
@@ -530,6 +540,22 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     if (fused) {
       PrepArgs pa{};
       pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
+      pa.n_shared = c.n_shared;
+      if (attn && !attn_full) {
+        pa.x = in;
+        pa.attn_a = L.attn_a;
+        pa.u_out = L.attn_u;
+      }
+      if (attn_sync && xg_gather) {
+        // The rows of tokens that keep their attention are final now; the
+        // output projection writes the others (row_of says where).
+        pa.xg = h->xg;
+        pa.gather_final_only = 1;
+        pa.row_of = h->attn_rowof;
+        oa.row_of = h->attn_rowof;
+        oa.row_w = c.top_k + c.n_shared;
+        oa.xg = h->xg;
+      }
       pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
       pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
       pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
@@ -551,13 +577,13 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       // attention output over all keys of their sample; their a and u rows
       // are replaced, then the FFN rows are gathered from u.
       if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
-             return launch_attn_rows(L.token_any, T, h->attn_rows, h->attn_n, s);
+             return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp, s);
            })) != cudaSuccess)
         break;
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
-      if (!(use_tc && kGemmGathersRows)) {
+      if (xg_gather && !fused) {
         CompactArgs ga = ca;
         ga.xg = h->xg;
         if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] { return launch_gather(ga, h->bf16, s); })) != cudaSuccess)

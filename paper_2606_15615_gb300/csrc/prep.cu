@@ -73,6 +73,14 @@ __device__ bool grid_sync(unsigned* cnt, unsigned target, int* status) {
 }
 
 // TB tokens per block (16 or 32); EPAD experts padded to a multiple of 8.
+// Bytes of the region holding the logits (phase A) and, later, the per-block
+// group counts (phase C), rounded up to 16.
+__host__ __device__ constexpr size_t prep_region_bytes(int TB, int EPAD, int n_blocks, int G) {
+  const size_t logits = static_cast<size_t>(TB) * (EPAD + 1) * 4;
+  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;
+  return ((logits > counts ? logits : counts) + 15) / 16 * 16;
+}
+
 template <int TB, int EPAD, int KMAX>
 __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   constexpr int G = kThreads / TB;       // lanes per token in the routing epilogue (4 or 8)
@@ -114,6 +122,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   float* s_logit = reinterpret_cast<float*>(s_x + TB * ldw);  // [TB][EPAD + 1]
   const int tok0 = blockIdx.x * TB;
   const int ntok = min(TB, T - tok0);
+  // DiT-MoE block on a cache step: the cached attention rows, after the
+  // logits / counts region (sized as prep_smem sizes it for this grid).
+  const bool add_a = a.attn_a != nullptr;
+  __nv_bfloat16* s_a = reinterpret_cast<__nv_bfloat16*>(
+      reinterpret_cast<uint8_t*>(s_logit) + prep_region_bytes(TB, EPAD, gridDim.x, E + 1));
 
   // ---- A0: stage gate rows and token rows ----
   // Before the programmatic-dependency wait: everything that the previous
@@ -131,9 +144,15 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   const uint32_t bar = smem_u32(&sm_bar);
   const uint32_t row_bytes = static_cast<uint32_t>(D) * 2;
   if (t == 0) {
-    mbar_expect_tx(bar, row_bytes * (E + ntok));
+    mbar_expect_tx(bar, row_bytes * (E + ntok + (add_a ? ntok : 0)));
     const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
     for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
+    if (add_a) {
+      // a^{t0} of this layer was written on an earlier step.
+      const __nv_bfloat16* ar = static_cast<const __nv_bfloat16*>(a.attn_a);
+      for (int q = 0; q < ntok; ++q)
+        bulk_g2s(smem_u32(s_a + q * ldw), ar + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
+    }
   }
   // Prefetch what later phases read: cached metadata and EMA rows.
   {
@@ -164,6 +183,28 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
   if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);
   __syncthreads();
+  if (add_a) {
+    // u = x + a^{t0} (rounded to bf16): the router input, the rows the FFN
+    // gathers, and the residual; written out for the kernels after this one.
+    __nv_bfloat16* u_out = static_cast<__nv_bfloat16*>(a.u_out);
+    const int nv = D / 8;
+    for (int idx = t; idx < ntok * nv; idx += kThreads) {
+      const int q = idx / nv, c = idx % nv;
+      uint4* xs = reinterpret_cast<uint4*>(s_x + q * ldw) + c;
+      float xv[8], av[8];
+      unpack_vec(*xs, xv, static_cast<__nv_bfloat16*>(nullptr));
+      unpack_vec(*(reinterpret_cast<const uint4*>(s_a + q * ldw) + c), av, static_cast<__nv_bfloat16*>(nullptr));
+#pragma unroll
+      for (int j = 0; j < 8; ++j) xv[j] += av[j];
+      uint4 uv;
+      __nv_bfloat162* uh = reinterpret_cast<__nv_bfloat162*>(&uv);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) uh[j] = __floats2bfloat162_rn(xv[2 * j], xv[2 * j + 1]);
+      *xs = uv;
+      reinterpret_cast<uint4*>(u_out + static_cast<size_t>(tok0 + q) * D)[c] = uv;
+    }
+    __syncthreads();
+  }
 
   // ---- A1: logits on the tensor cores ----
   {
@@ -520,23 +561,36 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     if (warp == 0) {
       const int i = tok0 + lane;
       const unsigned lt = (1u << lane) - 1u;
+      // Under the sync rule the rows of a token with recomputed branches are
+      // written by the attention output projection (row_of says where).
+      const bool gather_here = !(a.gather_final_only && d.any);
+      const int W = k + a.n_shared;
+      int32_t* row_of = (a.row_of && i < T) ? a.row_of + static_cast<size_t>(i) * W : nullptr;
 #pragma unroll
       for (int p = 0; p < KMAX; ++p) {
+        if (p < k && row_of) row_of[p] = -1;
         if (d.rec[p]) {
           const int g = d.e[p];
           const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
           a.list[pos] = i * k + d.sl[p];
+          if (row_of) row_of[p] = pos;
+          if (gather_here) {
+            const int r = atomicAdd(&sm_nrows, 1);
+            sm_rows[r][0] = pos;
+            sm_rows[r][1] = i;
+          }
+        }
+      }
+      if (row_of && a.n_shared) row_of[k] = -1;
+      if (d.shared_row) {
+        const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
+        a.list[pos] = i;
+        if (row_of) row_of[k] = pos;
+        if (gather_here) {
           const int r = atomicAdd(&sm_nrows, 1);
           sm_rows[r][0] = pos;
           sm_rows[r][1] = i;
         }
-      }
-      if (d.shared_row) {
-        const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
-        a.list[pos] = i;
-        const int r = atomicAdd(&sm_nrows, 1);
-        sm_rows[r][0] = pos;
-        sm_rows[r][1] = i;
       }
     }
     __syncthreads();
@@ -554,12 +608,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
 }
 
 template <int TB, int EPAD>
-size_t prep_smem(int D, int n_blocks, int G) {
+size_t prep_smem(int D, int n_blocks, int G, bool attn) {
   const size_t ldw = static_cast<size_t>(D) + 8;
   const size_t rows = (EPAD + TB) * ldw * 2;                        // gate rows, token rows
-  const size_t logits = static_cast<size_t>(TB) * (EPAD + 1) * 4;    // phase A
-  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;       // phase C, same place
-  return rows + (logits > counts ? logits : counts);
+  const size_t a_rows = attn ? TB * ldw * 2 : 0;                    // cached attention rows
+  return rows + prep_region_bytes(TB, EPAD, n_blocks, G) + a_rows;
 }
 
 template <int TB, int EPAD, int KMAX>
@@ -629,7 +682,7 @@ int kmax_of(int k) { return k <= 2 ? 2 : (k <= 4 ? 4 : 8); }
 
 }  // namespace
 
-PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms) {
+PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn) {
   PrepShape p{0, 0, 0, 0};
   if (D % 16 || E < 1 || E > kMaxExperts || k < 1 || k > kMaxTopK) return p;
   const int epad = (E + 7) / 8 * 8;
@@ -639,7 +692,7 @@ PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms) {
     const int nb = (max_tokens + TB - 1) / TB;
     const size_t smem = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> size_t {
       if constexpr (tb == 0) return 0;
-      else return prep_smem<tb, ep>(D, nb, E + 1);
+      else return prep_smem<tb, ep>(D, nb, E + 1, attn);
     });
     if (smem == 0 || smem > kPrepSmemMax) continue;
     const int occ = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> int {

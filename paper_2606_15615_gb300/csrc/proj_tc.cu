@@ -9,7 +9,8 @@
 //   kProjStore     out[m, n] = bf16(C[m, n])              (q, k, v rows)
 //   kProjResidual  row m belongs to token t = rows[m] (or m):
 //                  a = bf16(C[m, :]), a_out[t, :] = a, u_out[t, :] = bf16(x[t, :] + a)
-//                  (the attention output a_i and the MoE input u_i = x_i + a_i)
+//                  (the attention output a_i and the MoE input u_i = x_i + a_i);
+//                  u_i also goes to the token's FFN input rows when row_of is set
 // M is a host bound; when m_dev is set the launch reads the actual row count
 // there (rows recomputed this step) and tiles past it return at once.
 //
@@ -20,9 +21,11 @@
 //             N = BN, K = 16) from one thread; tcgen05.commit frees a stage
 //             and finally signals the finished accumulator;
 //   warps 2-5 epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31 (its rows),
-//             32 columns at a time, adds the bias, rounds to bf16 and stores
-//             through a 2 KB shared-memory stage so that each store writes
-//             64 contiguous bytes of 8 rows.
+//             32 columns at a time, and adds the bias (staged in shared memory
+//             while the MMAs run).  Store mode rounds to bf16 and writes
+//             through a 2 KB shared-memory stage, so each store covers 64
+//             contiguous bytes of 8 rows; residual mode loads the token's x
+//             one chunk ahead and writes a and u, 64 bytes per lane.
 // Every wait is bounded (about one second); a wait that runs out records the
 // timeout status, raises a CTA abort flag, waits (bounded) for the copies and
 // MMAs already issued, frees TMEM and returns.
@@ -57,16 +60,20 @@ struct ProjParams {
   __nv_bfloat16* u_out;      // kProjResidual: [n_tok, N]
   int nst;                   // ring stages
   unsigned long long* row_stat;
+  const int32_t* row_of;     // kProjResidual: [n_tok, row_w] FFN rows of the token (-1: none), or null
+  int row_w;
+  __nv_bfloat16* xg;         // [rows, N] FFN input rows that also take u
   int* status;
 };
 
-// One warp's 32 x 32 chunk: lane i holds row i's 32 values (bias added).
-// They are rounded to bf16 and staged, then written 16 bytes per lane with
-// four lanes per row.  Store mode: `dst` is this lane's row at the chunk's
-// first column (null: not stored).  Residual mode: `dst` is the a row, `xr`
-// and `ur` the x and u rows of the same token.
-__device__ __forceinline__ void epi_chunk(uint8_t* stage, const float* v, __nv_bfloat16* dst,
-                                          const __nv_bfloat16* xr, __nv_bfloat16* ur, int lane) {
+constexpr int kMaxRowOf = kMaxTopK + 1;
+
+// Store mode, one warp's 32 x 32 chunk: lane i holds row i's 32 values
+// (bias added).  They are rounded to bf16 and staged, then written 16 bytes
+// per lane with four lanes per row, so each store covers 64 contiguous bytes
+// of 8 rows.  `dst` is this lane's row at the chunk's first column (null:
+// not stored).
+__device__ __forceinline__ void store_chunk_staged(uint8_t* stage, const float* v, __nv_bfloat16* dst, int lane) {
   uint32_t packed[16];
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
@@ -79,26 +86,45 @@ __device__ __forceinline__ void epi_chunk(uint8_t* stage, const float* v, __nv_b
         make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
   __syncwarp();
   const unsigned long long d_mine = reinterpret_cast<unsigned long long>(dst);
-  const unsigned long long x_mine = reinterpret_cast<unsigned long long>(xr);
-  const unsigned long long u_mine = reinterpret_cast<unsigned long long>(ur);
 #pragma unroll
   for (int it = 0; it < 4; ++it) {
     const int row = it * 8 + (lane >> 2), j = lane & 3;
     const uint4 val = *reinterpret_cast<const uint4*>(stage + row * 64 + ((j ^ ((row >> 1) & 3)) << 4));
     __nv_bfloat16* d = reinterpret_cast<__nv_bfloat16*>(__shfl_sync(0xffffffffu, d_mine, row));
-    const __nv_bfloat16* xp = reinterpret_cast<const __nv_bfloat16*>(__shfl_sync(0xffffffffu, x_mine, row));
-    __nv_bfloat16* up = reinterpret_cast<__nv_bfloat16*>(__shfl_sync(0xffffffffu, u_mine, row));
     if (d) *reinterpret_cast<uint4*>(d + j * 8) = val;
-    if (up) {
-      float a[8], xv[8];
-      unpack_vec(val, a, static_cast<__nv_bfloat16*>(nullptr));
-      load_vec(xp + j * 8, xv);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) a[q] += xv[q];
-      store_vec(up + j * 8, a);
-    }
   }
   __syncwarp();
+}
+
+// Residual mode, one lane's row: a = bf16(v), u = bf16(x + a), each 64
+// contiguous bytes (two full 32-byte sectors) written by the lane itself;
+// u also goes to the token's FFN input rows (g_dst[q], or null).
+__device__ __forceinline__ void store_residual(const float* v, const uint4* xv, __nv_bfloat16* a_dst,
+                                               __nv_bfloat16* u_dst, __nv_bfloat16* const* g_dst, int n_g) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    uint4 av, uv;
+    __nv_bfloat162* ah = reinterpret_cast<__nv_bfloat162*>(&av);
+    __nv_bfloat162* uh = reinterpret_cast<__nv_bfloat162*>(&uv);
+    const __nv_bfloat162* xh = reinterpret_cast<const __nv_bfloat162*>(&xv[j]);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      ah[q] = __floats2bfloat162_rn(v[8 * j + 2 * q], v[8 * j + 2 * q + 1]);
+      const float2 af = __bfloat1622float2(ah[q]);
+      const float2 xf = __bfloat1622float2(xh[q]);
+      uh[q] = __floats2bfloat162_rn(xf.x + af.x, xf.y + af.y);
+    }
+    reinterpret_cast<uint4*>(a_dst)[j] = av;
+    reinterpret_cast<uint4*>(u_dst)[j] = uv;
+#pragma unroll
+    for (int q = 0; q < kMaxRowOf; ++q)
+      if (q < n_g && g_dst[q]) reinterpret_cast<uint4*>(g_dst[q])[j] = uv;
+  }
+}
+
+__device__ __forceinline__ void load_x_chunk(const __nv_bfloat16* xr, uint4* xv) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) xv[j] = __ldg(reinterpret_cast<const uint4*>(xr) + j);
 }
 
 template <int BN>
@@ -113,6 +139,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
   __shared__ __align__(8) uint64_t drain_bar;
   __shared__ uint32_t tmem_sh;
   __shared__ volatile int abort_flag;
+  __shared__ float s_bias[BN];
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* epi = smem + p.nst * kStage;
@@ -202,43 +229,66 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const int r = quad * 32 + lane;
     const int m = m0 + r;
     uint8_t* stage = epi + (warp - 2) * kPEpiStage;
-    if (mbar_wait(smem_u32(&acc_bar), 0, &abort_flag)) {
-      tc_fence_after();
-      __nv_bfloat16* dst = nullptr;
-      const __nv_bfloat16* xr = nullptr;
-      __nv_bfloat16* ur = nullptr;
-      if (m < M) {
-        if (p.mode == kProjStore) {
-          dst = p.out + static_cast<size_t>(m) * p.ldo + n0;
-        } else {
-          const int t = p.rows ? p.rows[m] : m;
-          if (t >= 0 && t < p.n_tok) {
-            const size_t off = static_cast<size_t>(t) * p.N + n0;
-            dst = p.a_out + off;
-            xr = p.x + off;
-            ur = p.u_out + off;
-          } else {
-            report_status(p.status, kStatusBadIndex, 6000000 + m);
+    // While the MMAs run: the tile's bias into shared memory, this lane's
+    // row pointers, and the residual rows' first chunk of x.
+    for (int j = threadIdx.x - 64; j < BN; j += 128) s_bias[j] = p.bias ? __ldg(p.bias + n0 + j) : 0.f;
+    __nv_bfloat16* dst = nullptr;
+    const __nv_bfloat16* xr = nullptr;
+    __nv_bfloat16* ur = nullptr;
+    __nv_bfloat16* gr[kMaxRowOf];
+#pragma unroll
+    for (int q = 0; q < kMaxRowOf; ++q) gr[q] = nullptr;
+    const int n_g = p.row_of ? p.row_w : 0;
+    if (m < M) {
+      if (p.mode == kProjStore) {
+        dst = p.out + static_cast<size_t>(m) * p.ldo + n0;
+      } else {
+        const int t = p.rows ? p.rows[m] : m;
+        if (t >= 0 && t < p.n_tok) {
+          const size_t off = static_cast<size_t>(t) * p.N + n0;
+          dst = p.a_out + off;
+          xr = p.x + off;
+          ur = p.u_out + off;
+#pragma unroll
+          for (int q = 0; q < kMaxRowOf; ++q) {
+            if (q < n_g) {
+              const int pos = p.row_of[static_cast<size_t>(t) * p.row_w + q];
+              if (pos >= 0) gr[q] = p.xg + static_cast<size_t>(pos) * p.N + n0;
+            }
           }
+        } else {
+          report_status(p.status, kStatusBadIndex, 6000000 + m);
         }
       }
+    }
+    uint4 xb[2][4];  // x of chunks c and c + 1 in flight
+    if (xr) {
+      load_x_chunk(xr, xb[0]);
+      if (BN > 32) load_x_chunk(xr + 32, xb[1]);
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps: bias staged
+    if (mbar_wait(smem_u32(&acc_bar), 0, &abort_flag)) {
+      tc_fence_after();
       const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+#pragma unroll
       for (int c = 0; c < BN / 32; ++c) {
+        uint4 xc[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) xc[j] = xb[c & 1][j];
+        if (xr && c + 2 < BN / 32) load_x_chunk(xr + (c + 2) * 32, xb[c & 1]);  // two chunks ahead
         uint32_t raw[32];
         tmem_ld32(tbase + c * 32, raw);
         float v[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]);
-        if (p.bias) {
-          const float4* b4 = reinterpret_cast<const float4*>(p.bias + n0 + c * 32);
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
+        if (p.mode == kProjStore) {
+          store_chunk_staged(stage, v, dst ? dst + c * 32 : nullptr, lane);
+        } else if (dst) {
+          __nv_bfloat16* gc[kMaxRowOf];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const float4 b = __ldg(b4 + j);
-            v[4 * j] += b.x; v[4 * j + 1] += b.y; v[4 * j + 2] += b.z; v[4 * j + 3] += b.w;
-          }
+          for (int q = 0; q < kMaxRowOf; ++q) gc[q] = gr[q] ? gr[q] + c * 32 : nullptr;
+          store_residual(v, xc, dst + c * 32, ur + c * 32, gc, n_g);
         }
-        epi_chunk(stage, v, dst ? dst + c * 32 : nullptr, xr ? xr + c * 32 : nullptr, ur ? ur + c * 32 : nullptr,
-                  lane);
       }
     } else if (lane == 0) {
       if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 602);
@@ -272,7 +322,8 @@ constexpr int stage_bytes() {
 
 }  // namespace
 
-int proj_tile_n(int N) {
+int proj_tile_n(int N, int want) {
+  if (want) return (want == 64 || want == 128 || want == 256) && N % want == 0 ? want : 0;
   if (N % 256 == 0) return 256;
   if (N % 128 == 0) return 128;
   if (N % 64 == 0) return 64;
@@ -280,7 +331,7 @@ int proj_tile_n(int N) {
 }
 
 cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
-  const int BN = proj_tile_n(a.N);
+  const int BN = proj_tile_n(a.N, a.tile_n);
   if (BN == 0 || a.K % 64 || a.M <= 0) return cudaErrorInvalidValue;
   CUtensorMap amap, bmap;
   if (!encode_2d(&amap, a.A, static_cast<uint64_t>(a.a_rows), static_cast<uint64_t>(a.K), kPM) ||
@@ -294,6 +345,9 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
   p.a_out = static_cast<__nv_bfloat16*>(a.a_out);
   p.u_out = static_cast<__nv_bfloat16*>(a.u_out);
   p.row_stat = a.row_stat;
+  p.row_of = a.row_of;
+  p.row_w = a.row_w;
+  p.xg = static_cast<__nv_bfloat16*>(a.xg);
   p.status = a.status;
   const int kb = a.K / 64;
   const int stage = kPABytes + BN * 128;

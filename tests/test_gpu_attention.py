@@ -144,3 +144,17 @@ def test_token_count_change_and_empty_step(M):
     with pytest.raises(M.MoecaError):
         st.step(torch.zeros((100, D), dtype=torch.bfloat16, device="cuda"), 10)   # not a multiple of 64
     st.close()
+
+
+@pytest.mark.parametrize("policy", [0, 1])
+def test_separate_kernel_path(M, policy):
+    """The SIMT FFN takes the separate router / select / compact kernels, so
+    u = x + a^{t0} and the FFN row gather run as their own launches."""
+    T, D, H, S = 256, 256, 4, 128
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=11, tau0=0.72, attn_policy=policy,
+                                   ffn_impl=M.MOECA_FFN_SIMT)
+    rng = np.random.default_rng(110 + policy)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.08)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    assert rep.reused > 0 and rep.attn_rows >= 2 * T + (1 if policy == 0 else 0)
+    st.close()
