@@ -100,11 +100,15 @@ typedef struct {
                                  D / H (64, 72, 80, 96 or 128) channels; bf16 only */
   int32_t seq_len;            /* token rows per sample: attention runs within each run of seq_len
                                  consecutive rows (0: all T rows are one sample); T must be a
-                                 multiple of it */
+                                 multiple of it and it a multiple of 8 */
   int32_t attn_policy;        /* attention output on cache steps: 0 = recomputed for the tokens
                                  with a non-empty recompute set (Sec. 4.1 sync rule, default);
                                  1 = reused for every token ("without sync update", Table 4);
                                  2 = recomputed for every token, routing on the fresh input */
+  int32_t attn_impl;          /* attention core: 0 = chosen per sample length (default: tcgen05 /
+                                 TMEM kernel from 512 tokens per sample, warp-level mma.sync kernel
+                                 below, where a CTA sees too few key blocks to fill its pipeline);
+                                 1 = mma.sync kernel; 2 = tcgen05 kernel */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters

@@ -40,14 +40,6 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr));
-}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -74,7 +66,7 @@ __global__ void __launch_bounds__(256) attn_residual_kernel(const uint4* x, cons
 // Also writes where each sample's tokens start in the list (sample_lo[b] for
 // sample b of S tokens, sample_lo[T / S] = the list's length).
 __global__ void __launch_bounds__(1024) attn_rows_kernel(const uint8_t* any, int T, int S, int32_t* rows,
-                                                         int* n_rows, int32_t* sample_lo) {
+                                                         int* n_rows, int32_t* sample_lo, int32_t* inv) {
   pdl_entry();
   __shared__ int warp_tot[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -103,7 +95,12 @@ __global__ void __launch_bounds__(1024) attn_rows_kernel(const uint8_t* any, int
   int pos = incl - c + (warp ? warp_tot[warp - 1] : 0);
   for (int i = beg; i < end; ++i) {
     if (i % S == 0) sample_lo[i / S] = pos;
-    if (any[i]) rows[pos++] = i;
+    if (any[i]) {
+      inv[i] = pos;
+      rows[pos++] = i;
+    } else {
+      inv[i] = -1;
+    }
   }
   if (tid == 1023) {
     *n_rows = warp_tot[31];
@@ -120,19 +117,20 @@ __host__ __device__ constexpr int core_nbuf() {
 }
 
 // Shared memory of attn_core_kernel<DH>: Q [64][DK + 8], K [NBUF][64][DK + 8],
-// V [NBUF][64][DH + 8] (bf16; 16 bytes of padding per row keep ldmatrix free
-// of bank conflicts).  DK = DH rounded up to 16 (the q k^T contraction).
+// V^T [NBUF][DH][64 + 8] (bf16; 16 bytes of padding per row keep ldmatrix
+// free of bank conflicts).  DK = DH rounded up to 16 (the q k^T contraction).
+constexpr int kLdVt = kKeys + 8;
 template <int DH>
 constexpr size_t core_smem() {
   constexpr int DK = (DH + 15) / 16 * 16;
   constexpr int NB = core_nbuf<DH>();
-  return (static_cast<size_t>(kQRows) * (DK + 8) + NB * kKeys * (DK + 8) + NB * kKeys * (DH + 8)) * 2;
+  return (static_cast<size_t>(kQRows) * (DK + 8) + NB * kKeys * (DK + 8) + NB * DH * kLdVt) * 2;
 }
 
 template <int DH>
 __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, float scale_log2) {
   constexpr int DK = (DH + 15) / 16 * 16;
-  constexpr int LDQ = DK + 8, LDV = DH + 8;
+  constexpr int LDQ = DK + 8;
   constexpr int NT = DH / 8;   // 8-column tiles of the output
   constexpr int CH = DH / 8;   // 16-byte chunks of one head row
   constexpr int NB = core_nbuf<DH>();
@@ -145,7 +143,7 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
   pdl_entry();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int b = blockIdx.y, h = blockIdx.z;
-  const int S = a.S, D = a.D, ld = 3 * D;
+  const int S = a.S, D = a.D, T = a.T;
   const int key0 = b * S;
   int lo = key0, hi = key0 + S;
   if (a.rows) {
@@ -175,21 +173,30 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
     }
   }
   __syncthreads();
-  const __nv_bfloat16* qkv = static_cast<const __nv_bfloat16*>(a.qkv);
+  const __nv_bfloat16* qg = static_cast<const __nv_bfloat16*>(a.q);
+  const __nv_bfloat16* kg = static_cast<const __nv_bfloat16*>(a.k);
+  const __nv_bfloat16* vtg = static_cast<const __nv_bfloat16*>(a.vt);
   for (int i = tid; i < kQRows * CH; i += kCoreThreads) {
     const int r = i / CH, c = i % CH;
-    const int t = s_tok[r];
-    const __nv_bfloat16* src = qkv + static_cast<size_t>(t < 0 ? key0 : t) * ld + h * DH + c * 8;
-    cp_async16(smem_u32(sQ + r * LDQ + c * 8), src, t >= 0);
+    const bool v = s_tok[r] >= 0;
+    const __nv_bfloat16* src = qg + static_cast<size_t>(v ? r0 + r : 0) * D + h * DH + c * 8;
+    cp_async16(smem_u32(sQ + r * LDQ + c * 8), src, v);
   }
   auto load_kv = [&](int kb, int buf) {
     for (int i = tid; i < kKeys * CH; i += kCoreThreads) {
       const int r = i / CH, c = i % CH;
       const int key = kb * kKeys + r;
       const bool v = key < S;
-      const __nv_bfloat16* src = qkv + static_cast<size_t>(key0 + (v ? key : 0)) * ld + D + h * DH + c * 8;
+      const __nv_bfloat16* src = kg + static_cast<size_t>(key0 + (v ? key : 0)) * D + h * DH + c * 8;
       cp_async16(smem_u32(sK + (buf * kKeys + r) * LDQ + c * 8), src, v);
-      cp_async16(smem_u32(sV + (buf * kKeys + r) * LDV + c * 8), src + D, v);
+    }
+    // v^T rows (channels) of this head, 8 keys per copy (S is a multiple of 8).
+    for (int i = tid; i < DH * (kKeys / 8); i += kCoreThreads) {
+      const int d = i / (kKeys / 8), c = i % (kKeys / 8);
+      const int key = kb * kKeys + c * 8;
+      const bool v = key < S;
+      const __nv_bfloat16* src = vtg + static_cast<size_t>(h * DH + d) * T + key0 + (v ? key : 0);
+      cp_async16(smem_u32(sV + (buf * DH + d) * kLdVt + c * 8), src, v);
     }
   };
   const int nkb = (S + kKeys - 1) / kKeys;
@@ -220,7 +227,7 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
                 qf[kc][1], qf[kc][2], qf[kc][3]);
     }
     const __nv_bfloat16* kbuf = sK + (kb % NB) * kKeys * LDQ;
-    const __nv_bfloat16* vbuf = sV + (kb % NB) * kKeys * LDV;
+    const __nv_bfloat16* vbuf = sV + (kb % NB) * DH * kLdVt;
     // ---- scores of this warp's 16 rows against 64 keys
     float s[8][4];
 #pragma unroll
@@ -242,7 +249,8 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int key = kb * kKeys + t * 8 + 2 * q4 + (j & 1);
-        const float v = key < S ? s[t][j] * scale_log2 : -INFINITY;
+        // One rounded product, used for the maximum and the exponent alike.
+        const float v = key < S ? __fmul_rn(s[t][j], scale_log2) : -INFINITY;
         s[t][j] = v;
         mx[j >> 1] = fmaxf(mx[j >> 1], v);
       }
@@ -280,17 +288,18 @@ __global__ void __launch_bounds__(kCoreThreads) attn_core_kernel(AttnArgs a, flo
       const uint32_t a1 = pack_bf16(s[2 * kc][2], s[2 * kc][3]);
       const uint32_t a2 = pack_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1]);
       const uint32_t a3 = pack_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3]);
-      const __nv_bfloat16* vrow = vbuf + (kc * 16 + (mat & 1) * 8 + mr) * LDV;
+      // v^T rows are channels, keys contiguous: the B operand without transposing.
+      const int kcol = kc * 16 + (mat & 1) * 8;
 #pragma unroll
       for (int np = 0; np < NT / 2; ++np) {
         uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(smem_u32(vrow + np * 16 + (mat >> 1) * 8), b0, b1, b2, b3);
+        ldsm_x4(smem_u32(vbuf + (np * 16 + (mat >> 1) * 8 + mr) * kLdVt + kcol), b0, b1, b2, b3);
         mma_16816(o[2 * np], a0, a1, a2, a3, b0, b1);
         mma_16816(o[2 * np + 1], a0, a1, a2, a3, b2, b3);
       }
       if (NT & 1) {
         uint32_t b0, b1;
-        ldsm_x2_t(smem_u32(vrow + (NT - 1) * 8), b0, b1);
+        ldsm_x2(smem_u32(vbuf + ((NT - 1) * 8 + mr) * kLdVt + kcol), b0, b1);
         mma_16816(o[NT - 1], a0, a1, a2, a3, b0, b1);
       }
     }
@@ -328,13 +337,13 @@ cudaError_t run_core(const AttnArgs& a, cudaStream_t s) {
 }  // namespace
 
 bool attn_supported(int D, int H) {
-  if (H < 1 || D % H) return false;
+  if (H < 1 || D % H || D % 64) return false;
   const int dh = D / H;
   return dh == 64 || dh == 72 || dh == 80 || dh == 96 || dh == 128;
 }
 
 cudaError_t launch_attn_core(const AttnArgs& a, cudaStream_t s) {
-  if (!attn_supported(a.D, a.H) || a.S < 1 || a.T % a.S) return cudaErrorInvalidValue;
+  if (!attn_supported(a.D, a.H) || a.S < 1 || a.S % 8 || a.T % a.S) return cudaErrorInvalidValue;
   switch (a.D / a.H) {
     case 64: return run_core<64>(a, s);
     case 72: return run_core<72>(a, s);
@@ -358,8 +367,8 @@ cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, i
 }
 
 cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int S, int32_t* rows, int* n_rows,
-                             int32_t* sample_lo, cudaStream_t s) {
-  return launch_pdl(attn_rows_kernel, dim3(1), dim3(1024), 0, s, token_any, T, S, rows, n_rows, sample_lo);
+                             int32_t* sample_lo, int32_t* inv, cudaStream_t s) {
+  return launch_pdl(attn_rows_kernel, dim3(1), dim3(1024), 0, s, token_any, T, S, rows, n_rows, sample_lo, inv);
 }
 
 }  // namespace moeca

@@ -1,0 +1,416 @@
+// Tensor-core attention core of the DiT-MoE block (Sec. 4.1) for sm_103a:
+// for the listed query rows of one sample and one head,
+//   o = softmax(q k^T / sqrt(dh)) v      over all keys of the sample,
+// bf16 operands, fp32 scores and accumulation, one pass over the keys with a
+// running maximum and sum (online softmax).
+//
+// One CTA per (128 query rows, sample, head), 6 warps:
+//   warp 0    TMA producer: the q tile once, then per block of 128 keys the
+//             k block (K-major, 128-byte swizzle) and the v^T block
+//             (channels x keys, K-major for p v) into a ring of stages;
+//   warp 1    allocates 512 TMEM columns and issues tcgen05.mma from one
+//             thread: S_j = q k_j^T into one of two S buffers (columns 0-127,
+//             128-255), then O += P_{j-1} v_{j-1} (columns 256 ..), so the
+//             scores of block j are computed while block j-1's softmax runs;
+//   warps 2-5 softmax, one query row per thread (TMEM lane quadrant warp % 4):
+//             reads S_j from TMEM (tcgen05.ld), keeps the row maximum m and
+//             sum l in base 2, rescales the O row in TMEM only when m rises
+//             (tcgen05.ld / st), writes P_j = 2^(s - m) in bf16 into shared
+//             memory in the 128-byte-swizzle K-major layout the MMA reads as
+//             its A operand, and at the end writes o = O / l.
+// q k^T contracts over dh rounded up to 16 (heads of 72 channels: 80, the
+// q tile's columns 72-79 zeroed in shared memory); p v produces dh rounded
+// up to 16 columns, of which the first dh are stored.
+// Every wait is bounded (about one second); a wait that runs out records the
+// timeout status, raises the CTA's abort flag, drains what was issued, frees
+// TMEM and returns.
+#include <cuda.h>
+
+#include <cmath>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_common.cuh"
+
+namespace moeca {
+
+namespace {
+
+constexpr int kTQ = 128;        // query rows per CTA (MMA M)
+constexpr int kTK = 128;        // keys per block (N of q k^T, K of p v)
+constexpr int kTThreads = 192;
+constexpr int kSubBytes = 128 * 128;  // one 128-row x 64-column bf16 sub-block (16 KB)
+
+template <int DH>
+struct TcAttnShape {
+  static constexpr int DKP = (DH + 15) / 16 * 16;   // q k^T contraction and p v width
+  static constexpr int QSUB = (DKP + 63) / 64;      // 64-column sub-blocks of q and k rows
+  static constexpr int KSTEPS = DKP / 16;           // MMAs of q k^T per block
+  static constexpr int QBYTES = QSUB * kSubBytes;   // q tile
+  static constexpr int KBYTES = QSUB * kSubBytes;   // k block: 128 keys
+  static constexpr int VSUB = DKP * 128;            // v^T sub-block: DKP channels x 64 keys
+  static constexpr int VBYTES = 2 * VSUB;           // v^T block: 128 keys
+  static constexpr int STAGE = KBYTES + VBYTES;
+  static constexpr int PBYTES = 2 * kSubBytes;      // P: 128 rows x 128 keys
+  static constexpr int NST = (200 * 1024 - QBYTES - PBYTES) / STAGE >= 3 ? 3 : 2;
+  static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + PBYTES + NST * STAGE + 1024;
+};
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+        "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};"
+      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ float ex2f_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Bounded wait on a barrier phase that no one may abort (draining).
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
+  const unsigned long long t0 = globaltimer();
+  while (!mbar_try(bar, parity) && globaltimer() - t0 < kTcWaitNs) {
+  }
+}
+
+struct TcAttnParams {
+  int T, D, S;
+  const int32_t* rows;       // list of query tokens, or null (all tokens)
+  const int32_t* sample_lo;  // with rows: sample b's rows are [sample_lo[b], sample_lo[b + 1])
+  __nv_bfloat16* o;          // [rows, D]
+  float scale_log2;          // log2(e) / sqrt(dh)
+  int* status;
+};
+
+
+// All lanes of a warp take the same branch after a wait (tcgen05.ld / st
+// are warp-collective): the warp proceeds only if every lane's wait ended.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag));
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kTThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                   const __grid_constant__ CUtensorMap vmap, const TcAttnParams p) {
+  using Sh = TcAttnShape<DH>;
+  constexpr int NST = Sh::NST;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t q_full, q_ready, p_full, o_done, drain_bar;
+  __shared__ __align__(8) uint64_t s_full[2], s_free[2], kv_full[NST], kv_empty[NST];
+  __shared__ uint32_t tmem_sh;
+  __shared__ volatile int abort_flag;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sP = smem + Sh::QBYTES;
+  uint8_t* sKV = sP + Sh::PBYTES;  // stage s: k block at + s STAGE, v^T block after it
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.y, h = blockIdx.z;
+  const int S = p.S, key0 = b * S;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(smem_u32(&q_full), 1);
+    mbar_init(smem_u32(&q_ready), 128);
+    mbar_init(smem_u32(&p_full), 128);
+    mbar_init(smem_u32(&o_done), 1);
+    mbar_init(smem_u32(&drain_bar), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&s_full[i]), 1);
+      mbar_init(smem_u32(&s_free[i]), 128);
+    }
+    for (int i = 0; i < NST; ++i) {
+      mbar_init(smem_u32(&kv_full[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&kmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
+  }
+  pdl_entry();
+  int lo = key0, hi = key0 + S;
+  if (p.rows) {
+    lo = p.sample_lo[b];
+    hi = p.sample_lo[b + 1];
+  }
+  const int r0 = lo + blockIdx.x * kTQ;
+  if (r0 >= hi) return;  // uniform over the CTA, before TMEM is taken
+  const int nq = min(kTQ, hi - r0);
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_sh)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_sh;
+  const int nkb = (S + kTK - 1) / kTK;
+  int issued = 0;  // producer: k / v blocks issued
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_expect_tx(smem_u32(&q_full), Sh::QBYTES);
+      for (int sub = 0; sub < Sh::QSUB; ++sub)
+        tma_load_2d(smem_u32(sQ + sub * kSubBytes), &qmap, h * DH + sub * 64, r0, smem_u32(&q_full));
+      for (int j = 0; j < nkb; ++j) {
+        const int s = j % NST;
+        if (j >= NST && !mbar_wait(smem_u32(&kv_empty[s]), ((j / NST) - 1) & 1, &abort_flag)) {
+          if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 700);
+          abort_flag = 1;
+          break;
+        }
+        uint8_t* st = sKV + s * Sh::STAGE;
+        const uint32_t bar = smem_u32(&kv_full[s]);
+        mbar_expect_tx(bar, Sh::STAGE);
+        for (int sub = 0; sub < Sh::QSUB; ++sub)
+          tma_load_2d(smem_u32(st + sub * kSubBytes), &kmap, h * DH + sub * 64, key0 + j * kTK, bar);
+        for (int sub = 0; sub < 2; ++sub)
+          tma_load_2d(smem_u32(st + Sh::KBYTES + sub * Sh::VSUB), &vmap, key0 + j * kTK + sub * 64, h * DH, bar);
+        ++issued;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id_s = instr_desc(kTQ, kTK), id_o = instr_desc(kTQ, Sh::DKP);
+      const uint32_t t_o = tmem + 256;
+      bool ok = mbar_wait(smem_u32(&q_ready), 0, &abort_flag);
+      // O += P_j v_j, then free block j's stage.
+      auto pv = [&](int j) -> bool {
+        if (!mbar_wait(smem_u32(&p_full), j & 1, &abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t pa = smem_u32(sP);
+        const uint32_t vb = smem_u32(sKV + (j % NST) * Sh::STAGE + Sh::KBYTES);
+#pragma unroll
+        for (int kk = 0; kk < kTK / 16; ++kk) {
+          const int sub = kk >> 2, off = (kk & 3) * 32;
+          mma_bf16(t_o, smem_desc(pa + sub * kSubBytes + off), smem_desc(vb + sub * Sh::VSUB + off), id_o,
+                   (j > 0) || (kk > 0));
+        }
+        mma_commit(smem_u32(&o_done));
+        mma_commit(smem_u32(&kv_empty[j % NST]));
+        return true;
+      };
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int s = j % NST, bb = j & 1;
+        if (!mbar_wait(smem_u32(&kv_full[s]), (j / NST) & 1, &abort_flag) ||
+            (j >= 2 && !mbar_wait(smem_u32(&s_free[bb]), ((j >> 1) - 1) & 1, &abort_flag))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t qa = smem_u32(sQ), kb = smem_u32(sKV + s * Sh::STAGE);
+#pragma unroll
+        for (int kk = 0; kk < Sh::KSTEPS; ++kk) {
+          const int sub = kk >> 2, off = (kk & 3) * 32;
+          mma_bf16(tmem + bb * kTK, smem_desc(qa + sub * kSubBytes + off), smem_desc(kb + sub * kSubBytes + off),
+                   id_s, kk > 0);
+        }
+        mma_commit(smem_u32(&s_full[bb]));
+        if (j >= 1 && !pv(j - 1)) ok = false;
+      }
+      if (ok && !pv(nkb - 1)) ok = false;
+      if (!ok) {
+        if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 701);
+        abort_flag = 1;
+      }
+      // Every MMA issued so far has completed once the drain barrier fires.
+      mma_commit(smem_u32(&drain_bar));
+      drain_wait(smem_u32(&drain_bar), 0);
+    }
+  } else {
+    // ---- softmax: one query row per thread
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const uint32_t t_o = tmem + lane_off + 256;
+    const float sc = p.scale_log2;
+    bool ok = warp_wait(smem_u32(&q_full), 0, &abort_flag);
+    if (ok && Sh::DKP > DH) {
+      // The q tile's columns DH .. DKP-1 hold the next head's values: zero
+      // them so they add nothing to q k^T (k's columns there are finite).
+#pragma unroll
+      for (int cidx = DH / 8; cidx < Sh::DKP / 8; ++cidx) {
+        const int sub = cidx >> 3, ch = cidx & 7;
+        *reinterpret_cast<uint4*>(sQ + sub * kSubBytes + r * 128 + ((ch ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    mbar_arrive(smem_u32(&q_ready));
+    float m = -INFINITY, l = 0.f;  // running maximum (scaled, base 2) and sum of this row
+    for (int j = 0; ok && j < nkb; ++j) {
+      const int bb = j & 1;
+      if (!warp_wait(smem_u32(&s_full[bb]), (j >> 1) & 1, &abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t t_s = tmem + lane_off + bb * kTK;
+      const int nvalid = S - j * kTK;  // keys of this block inside the sample (>= 1)
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kTK / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(t_s + c * 32, v);
+#pragma unroll
+        for (int q = 0; q < 32; ++q)
+          if (c * 32 + q < nvalid) mx = fmaxf(mx, __fmul_rn(__uint_as_float(v[q]), sc));
+      }
+      // Both passes use the same rounded product s sc (no fused multiply-add),
+      // so the row's largest term is exactly 2^0: with scores of 1e11 an
+      // unrounded product would differ from m by thousands.
+      const float m_new = fmaxf(m, mx);
+      if (j >= 1) {
+        // O and P are free once block j-1's p v has completed.
+        if (!warp_wait(smem_u32(&o_done), (j - 1) & 1, &abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, m_new > m)) {
+          const float alpha = ex2f_approx(m - m_new);  // 1 for rows whose maximum held
+#pragma unroll
+          for (int c = 0; c < Sh::DKP / 16; ++c) {
+            uint32_t v[16];
+            tmem_ld16(t_o + c * 16, v);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * alpha);
+            tmem_st16(t_o + c * 16, v);
+          }
+          l *= alpha;
+        }
+      }
+      m = m_new;
+      // P_j = 2^(s sc - m) in bf16, written as the 128-byte-swizzle K-major A tile.
+#pragma unroll
+      for (int c = 0; c < kTK / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(t_s + c * 32, v);
+        uint32_t pk[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          const int kk = c * 32 + 2 * q;
+          const float p0 = kk < nvalid ? ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q]), sc) - m) : 0.f;
+          const float p1 = kk + 1 < nvalid ? ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q + 1]), sc) - m) : 0.f;
+          l += p0 + p1;
+          pk[q] = pack2(p0, p1);
+        }
+        const int sub = c >> 1;
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const int ch = (c & 1) * 4 + q4;
+          *reinterpret_cast<uint4*>(sP + sub * kSubBytes + r * 128 + ((ch ^ (r & 7)) << 4)) =
+              make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&s_free[bb]));
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(smem_u32(&p_full));
+    }
+    if (ok && !warp_wait(smem_u32(&o_done), (nkb - 1) & 1, &abort_flag)) ok = false;
+    if (ok) {
+      tc_fence_after();
+      const float inv_l = 1.f / l;
+      __nv_bfloat16* dst = p.o + static_cast<size_t>(r0 + r) * p.D + h * DH;
+#pragma unroll
+      for (int c = 0; c < Sh::DKP / 16; ++c) {
+        uint32_t v[16];
+        tmem_ld16(t_o + c * 16, v);  // every lane: the load is warp-collective
+        if (r < nq) {
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int col = c * 16 + half * 8;
+            if (col < DH) {
+              uint4 w;
+              w.x = pack2(__uint_as_float(v[half * 8 + 0]) * inv_l, __uint_as_float(v[half * 8 + 1]) * inv_l);
+              w.y = pack2(__uint_as_float(v[half * 8 + 2]) * inv_l, __uint_as_float(v[half * 8 + 3]) * inv_l);
+              w.z = pack2(__uint_as_float(v[half * 8 + 4]) * inv_l, __uint_as_float(v[half * 8 + 5]) * inv_l);
+              w.w = pack2(__uint_as_float(v[half * 8 + 6]) * inv_l, __uint_as_float(v[half * 8 + 7]) * inv_l);
+              *reinterpret_cast<uint4*>(dst + col) = w;
+            }
+          }
+        }
+      }
+    } else if (lane == 0) {
+      if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 702);
+      abort_flag = 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0 && lane == 0 && abort_flag) {
+    // Copies issued but never consumed still land in shared memory.
+    drain_wait(smem_u32(&q_full), 0);
+    for (int s = 0; s < NST && s < issued; ++s) {
+      const int last = issued - 1 - ((issued - 1 - s) % NST);  // newest block issued on stage s
+      drain_wait(smem_u32(&kv_full[s]), (last / NST) & 1);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+  }
+}
+
+
+template <int DH>
+cudaError_t run_attn_tc(const AttnArgs& a, cudaStream_t s) {
+  using Sh = TcAttnShape<DH>;
+  CUtensorMap qm, km, vm;
+  if (!encode_2d(&qm, a.q, static_cast<uint64_t>(a.T), static_cast<uint64_t>(a.D), kTQ) ||
+      !encode_2d(&km, a.k, static_cast<uint64_t>(a.T), static_cast<uint64_t>(a.D), kTK) ||
+      !encode_2d(&vm, a.vt, static_cast<uint64_t>(a.D), static_cast<uint64_t>(a.T), Sh::DKP))
+    return cudaErrorInvalidValue;
+  TcAttnParams p{};
+  p.T = a.T; p.D = a.D; p.S = a.S; p.rows = a.rows; p.sample_lo = a.sample_lo;
+  p.o = static_cast<__nv_bfloat16*>(a.o);
+  p.scale_log2 = 1.4426950408889634f / std::sqrt(static_cast<float>(DH));
+  p.status = a.status;
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(Sh::SMEM));
+  if (e != cudaSuccess) return e;
+  const dim3 grid((a.S + kTQ - 1) / kTQ, a.T / a.S, a.H);
+  return launch_pdl(attn_tc_kernel<DH>, grid, dim3(kTThreads), Sh::SMEM, s, qm, km, vm, p);
+}
+
+}  // namespace
+
+cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s) {
+  if (!attn_supported(a.D, a.H) || a.S < 1 || a.S % 8 || a.T % a.S) return cudaErrorInvalidValue;
+  switch (a.D / a.H) {
+    case 64: return run_attn_tc<64>(a, s);
+    case 72: return run_attn_tc<72>(a, s);
+    case 80: return run_attn_tc<80>(a, s);
+    case 96: return run_attn_tc<96>(a, s);
+    default: return run_attn_tc<128>(a, s);
+  }
+}
+
+}  // namespace moeca

@@ -192,7 +192,7 @@ cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);
 // ---- Attention path of a DiT-MoE block (Sec. 4.1), bf16 only ----
 
 // Tensor-core projection GEMM: C = A B^T + bias (proj_tc.cu).
-enum ProjMode { kProjStore = 0, kProjResidual = 1 };
+enum ProjMode { kProjStore = 0, kProjResidual = 1, kProjQKV = 2 };
 struct ProjArgs {
   const void* A;          // [a_rows, K] bf16, row-major
   int a_rows;             // rows A holds (>= M)
@@ -213,6 +213,10 @@ struct ProjArgs {
   const int32_t* row_of;  // kProjResidual, or null: [n_tok, row_w] FFN row positions of the token
   int row_w;              //   (-1: none); u is also written to those rows of xg
   void* xg;               // [rows, N] FFN input rows
+  const int32_t* inv;     // kProjQKV (N = 3D): list place of token m, -1 if not listed, or null (m)
+  void* q_out;            // kProjQKV: [list rows, D] q of the listed tokens, in list order
+  void* k_out;            // kProjQKV: [n_tok, D] k
+  void* vt_out;           // kProjQKV: [D, n_tok] v transposed
   int* status;
 };
 // Tile width a launch uses for N: `want` (64 / 128 / 256) if it divides N,
@@ -224,22 +228,26 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s);
 cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, int D, int* status,
                                  cudaStream_t s);
 
-// Ascending list of tokens whose recompute set is non-empty, its length, and
-// where each sample's tokens start in it (sample_lo [T / S + 1]).
+// Ascending list of tokens whose recompute set is non-empty, its length,
+// where each sample's tokens start in it (sample_lo [T / S + 1]), and each
+// token's place in it (inv [T], -1 if absent).
 cudaError_t launch_attn_rows(const uint8_t* token_any, int T, int S, int32_t* rows, int* n_rows,
-                             int32_t* sample_lo, cudaStream_t s);
+                             int32_t* sample_lo, int32_t* inv, cudaStream_t s);
 
 // Multi-head self-attention rows: o[r] = concat_h softmax(q_t k_S^T / sqrt(dh)) v_S for the
 // r-th listed token t, keys and values of t's sample (S consecutive token rows).
 struct AttnArgs {
-  const void* qkv;        // [T, 3D] bf16: q | k | v, head h at columns h dh .. of each
-  int T, D, H, S;         // S tokens per sample, T a multiple of S
+  const void* q;          // [rows, D] bf16: q of the listed tokens in list order (head h at columns h dh ..)
+  const void* k;          // [T, D] bf16
+  const void* vt;         // [D, T] bf16: v transposed
+  int T, D, H, S;         // S tokens per sample (a multiple of 8), T a multiple of S
   const int32_t* rows;    // ascending token list, or null: every token (row r = token r)
   const int32_t* sample_lo;  // with rows: sample b's tokens are rows[sample_lo[b] .. sample_lo[b + 1])
   void* o;                // [rows, D] bf16
   int* status;
 };
 bool attn_supported(int D, int H);
-cudaError_t launch_attn_core(const AttnArgs& a, cudaStream_t s);
+cudaError_t launch_attn_core(const AttnArgs& a, cudaStream_t s);   // mma.sync (warp-level) core
+cudaError_t launch_attn_tc(const AttnArgs& a, cudaStream_t s);     // tcgen05 / TMEM core (attn_tc.cu)
 
 }  // namespace moeca

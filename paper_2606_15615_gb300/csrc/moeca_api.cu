@@ -98,7 +98,8 @@ struct moeca_handle {
   bool inject_stall = false;    // moeca_inject_fault: next step's barrier targets unreachable
   int32_t* prep_counts = nullptr;
   unsigned* prep_bar = nullptr;
-  void* qkv = nullptr;          // attention workspace: [T, 3D] q | k | v
+  void* qkv = nullptr;          // attention workspace: q [T, D] (list order), k [T, D], v^T [D, T]
+  int32_t* attn_inv = nullptr;  // [T] each token's place in attn_rows (-1: absent)
   void* attn_o = nullptr;       // [T, D] attention rows before the output projection
   int32_t* attn_rows = nullptr; // [T] tokens that recompute their attention
   int* attn_n = nullptr;        // their count
@@ -236,6 +237,7 @@ void moeca_config_default(moeca_config* c) {
   c->n_heads = 0;
   c->seq_len = 0;
   c->attn_policy = 0;
+  c->attn_impl = 0;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -284,8 +286,9 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&
        c.ffn_tile_n != 256) || c.ffn_split_k < 0 || c.ffn_split_k > 4)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_tile_n must be 0/64/128/192/256, ffn_split_k 0..4");
-  if (c.n_heads < 0 || c.seq_len < 0 || c.attn_policy < 0 || c.attn_policy > 2)
-    return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_heads and seq_len must be >= 0, attn_policy 0..2");
+  if (c.n_heads < 0 || c.seq_len < 0 || c.attn_policy < 0 || c.attn_policy > 2 || c.attn_impl < 0 ||
+      c.attn_impl > 2)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "n_heads and seq_len must be >= 0, attn_policy 0..2, attn_impl 0..2");
   const bool attn = c.n_heads > 0;
   if (attn && !bf16) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "the attention sub-layer is built for bf16 only");
   if (attn && (!attn_supported(c.hidden, c.n_heads) || c.hidden % 64))
@@ -360,6 +363,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     A((void**)&h->attn_rows, T * 4);
     A((void**)&h->attn_n, 16);
     A((void**)&h->attn_samp, (T + 1) * 4);
+    A((void**)&h->attn_inv, T * 4);
     A((void**)&h->attn_rowof, T * (k + c.n_shared) * 4);
   }
   const size_t nblk_router = (T + kRouterTokensPerBlock - 1) / kRouterTokensPerBlock;
@@ -458,7 +462,11 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   const bool use_tc = h->bf16 && c.ffn_impl == MOECA_FFN_AUTO;
   const bool attn = c.n_heads > 0;
   const int seq = c.seq_len ? c.seq_len : T;
-  if (attn && T % seq) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens must be a multiple of seq_len");
+  if (attn && (T % seq || seq % 8))
+    return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens must be a multiple of seq_len, and seq_len of 8");
+  // The tcgen05 attention core pays off once a CTA streams at least four
+  // 128-key blocks; shorter samples go to the warp-level core.
+  const bool use_attn_tc = c.attn_impl == 2 || (c.attn_impl == 0 && seq >= 512);
   cudaError_t e = cudaSuccess;
   NvtxRange step_range("moeca_step");
   for (int l = 0; l < c.n_layers; ++l) {
@@ -470,12 +478,16 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     const bool attn_sync = attn && !attn_full && c.attn_policy == 0;
     // The MoE sub-layer's input: the layer input, or u of a DiT-MoE block.
     const void* moe_in = attn ? L.attn_u : in;
+    const size_t TD = static_cast<size_t>(T) * c.hidden;
+    void* q_buf = h->qkv;
+    void* k_buf = static_cast<char*>(h->qkv) + TD * h->es;
+    void* vt_buf = static_cast<char*>(h->qkv) + 2 * TD * h->es;
     ProjArgs qa{};
     qa.A = in; qa.a_rows = T; qa.B = L.w.w_qkv; qa.bias = L.w.b_qkv;
-    qa.M = T; qa.N = 3 * c.hidden; qa.K = c.hidden; qa.mode = kProjStore;
-    qa.out = h->qkv; qa.ldo = 3 * c.hidden; qa.status = h->status_dev;
+    qa.M = T; qa.N = 3 * c.hidden; qa.K = c.hidden; qa.mode = kProjQKV;
+    qa.q_out = q_buf; qa.k_out = k_buf; qa.vt_out = vt_buf; qa.n_tok = T; qa.status = h->status_dev;
     AttnArgs aa{};
-    aa.qkv = h->qkv; aa.T = T; aa.D = c.hidden; aa.H = c.n_heads; aa.S = seq;
+    aa.q = q_buf; aa.k = k_buf; aa.vt = vt_buf; aa.T = T; aa.D = c.hidden; aa.H = c.n_heads; aa.S = seq;
     aa.o = h->attn_o; aa.status = h->status_dev;
     ProjArgs oa{};
     oa.A = h->attn_o; oa.a_rows = T; oa.B = L.w.w_o; oa.bias = L.w.b_o;
@@ -488,12 +500,15 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     oa.row_stat = L.stats + kStAttnRows; oa.status = h->status_dev;
     if (attn_sync) {
       aa.rows = h->attn_rows; aa.sample_lo = h->attn_samp;
+      qa.inv = h->attn_inv;
       oa.rows = h->attn_rows; oa.m_dev = h->attn_n;
     }
     if (attn_full) {
       // Every token's attention output, before the router sees u = x + a.
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
-      if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_ATTN, s, [&] {
+             return use_attn_tc ? launch_attn_tc(aa, s) : launch_attn_core(aa, s);
+           })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
     } else if (attn && h->prep.tokens_per_block == 0) {
       // u' = x + a^{t0}: the router input, and the MoE input of every token
@@ -577,11 +592,13 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       // attention output over all keys of their sample; their a and u rows
       // are replaced, then the FFN rows are gathered from u.
       if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
-             return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp, s);
+             return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp, h->attn_inv, s);
            })) != cudaSuccess)
         break;
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
-      if ((e = timed(h, MOECA_K_ATTN, s, [&] { return launch_attn_core(aa, s); })) != cudaSuccess) break;
+      if ((e = timed(h, MOECA_K_ATTN, s, [&] {
+             return use_attn_tc ? launch_attn_tc(aa, s) : launch_attn_core(aa, s);
+           })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
       if (xg_gather && !fused) {
         CompactArgs ga = ca;

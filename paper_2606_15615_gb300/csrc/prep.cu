@@ -565,7 +565,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       // written by the attention output projection (row_of says where).
       const bool gather_here = !(a.gather_final_only && d.any);
       const int W = k + a.n_shared;
-      int32_t* row_of = (a.row_of && i < T) ? a.row_of + static_cast<size_t>(i) * W : nullptr;
+      // Only this block's tokens: with 16-token blocks lanes 16-31 hold the
+      // next block's tokens, whose entries that block writes.
+      int32_t* row_of = (a.row_of && lane < ntok) ? a.row_of + static_cast<size_t>(i) * W : nullptr;
 #pragma unroll
       for (int p = 0; p < KMAX; ++p) {
         if (p < k && row_of) row_of[p] = -1;

@@ -6,7 +6,12 @@
 // with A [rows, K] row-major (the block input for the query / key / value
 // projection, the attention rows for the output projection) and B [N, K] a
 // weight matrix.  Two epilogues:
-//   kProjStore     out[m, n] = bf16(C[m, n])              (q, k, v rows)
+//   kProjStore     out[m, n] = bf16(C[m, n])
+//   kProjQKV       N = 3D split into the attention's operand layouts: the q
+//                  columns of token m go to row inv[m] of q_out (the token's
+//                  place in the recomputing-token list; none if -1), the k
+//                  columns to row m of k_out, and the v columns, transposed,
+//                  to column m of vt_out [D, n_tok]
 //   kProjResidual  row m belongs to token t = rows[m] (or m):
 //                  a = bf16(C[m, :]), a_out[t, :] = a, u_out[t, :] = bf16(x[t, :] + a)
 //                  (the attention output a_i and the MoE input u_i = x_i + a_i);
@@ -63,6 +68,10 @@ struct ProjParams {
   const int32_t* row_of;     // kProjResidual: [n_tok, row_w] FFN rows of the token (-1: none), or null
   int row_w;
   __nv_bfloat16* xg;         // [rows, N] FFN input rows that also take u
+  const int32_t* inv;        // kProjQKV: list place of token m (-1: none), or null (m)
+  __nv_bfloat16* q_out;      // kProjQKV: [list rows, D]
+  __nv_bfloat16* k_out;      // kProjQKV: [n_tok, D]
+  __nv_bfloat16* vt_out;     // kProjQKV: [D, n_tok]
   int* status;
 };
 
@@ -92,6 +101,27 @@ __device__ __forceinline__ void store_chunk_staged(uint8_t* stage, const float* 
     const uint4 val = *reinterpret_cast<const uint4*>(stage + row * 64 + ((j ^ ((row >> 1) & 3)) << 4));
     __nv_bfloat16* d = reinterpret_cast<__nv_bfloat16*>(__shfl_sync(0xffffffffu, d_mine, row));
     if (d) *reinterpret_cast<uint4*>(d + j * 8) = val;
+  }
+  __syncwarp();
+}
+
+// q/k/v mode, v columns: the warp's 32 x 32 chunk transposed through the
+// stage, so each lane writes 16 bytes (8 consecutive tokens) of one v^T row.
+// `vt` is v^T's row of the chunk's first column, `tok0` the warp's first
+// token (a multiple of 32), `M` the token count (a multiple of 8).
+__device__ __forceinline__ void store_chunk_transposed(uint8_t* stage, const float* v, __nv_bfloat16* vt, int tok0,
+                                                       int M, size_t ld, int lane) {
+  __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(stage);  // [32 columns][32 tokens]
+#pragma unroll
+  for (int j = 0; j < 32; ++j) st[j * 32 + lane] = __float2bfloat16_rn(v[j]);
+  __syncwarp();
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int j = it * 8 + (lane >> 2), seg = lane & 3;
+    const int tok = tok0 + seg * 8;
+    if (tok < M)
+      *reinterpret_cast<uint4*>(vt + static_cast<size_t>(j) * ld + tok) =
+          *reinterpret_cast<const uint4*>(st + j * 32 + seg * 8);
   }
   __syncwarp();
 }
@@ -239,9 +269,15 @@ __global__ void __launch_bounds__(kPThreads, 1)
 #pragma unroll
     for (int q = 0; q < kMaxRowOf; ++q) gr[q] = nullptr;
     const int n_g = p.row_of ? p.row_w : 0;
+    __nv_bfloat16* krow = nullptr;  // kProjQKV: this lane's k row (dst holds its q row)
     if (m < M) {
       if (p.mode == kProjStore) {
         dst = p.out + static_cast<size_t>(m) * p.ldo + n0;
+      } else if (p.mode == kProjQKV) {
+        const int qi = p.inv ? p.inv[m] : m;
+        const int Dm = p.N / 3;
+        if (qi >= 0) dst = p.q_out + static_cast<size_t>(qi) * Dm;
+        krow = p.k_out + static_cast<size_t>(m) * Dm;
       } else {
         const int t = p.rows ? p.rows[m] : m;
         if (t >= 0 && t < p.n_tok) {
@@ -283,6 +319,19 @@ __global__ void __launch_bounds__(kPThreads, 1)
         for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
         if (p.mode == kProjStore) {
           store_chunk_staged(stage, v, dst ? dst + c * 32 : nullptr, lane);
+        } else if (p.mode == kProjQKV) {
+          // The chunk lies in one of q, k, v (D is a multiple of 64): warp-uniform.
+          const int Dm = p.N / 3;
+          const int col = n0 + c * 32;
+          const int region = col / Dm, cc = col - region * Dm;
+          if (region == 0) {
+            store_chunk_staged(stage, v, dst ? dst + cc : nullptr, lane);
+          } else if (region == 1) {
+            store_chunk_staged(stage, v, krow ? krow + cc : nullptr, lane);
+          } else {
+            store_chunk_transposed(stage, v, p.vt_out + static_cast<size_t>(cc) * p.n_tok, m0 + quad * 32, M,
+                                   static_cast<size_t>(p.n_tok), lane);
+          }
         } else if (dst) {
           __nv_bfloat16* gc[kMaxRowOf];
 #pragma unroll
@@ -348,6 +397,10 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
   p.row_of = a.row_of;
   p.row_w = a.row_w;
   p.xg = static_cast<__nv_bfloat16*>(a.xg);
+  p.inv = a.inv;
+  p.q_out = static_cast<__nv_bfloat16*>(a.q_out);
+  p.k_out = static_cast<__nv_bfloat16*>(a.k_out);
+  p.vt_out = static_cast<__nv_bfloat16*>(a.vt_out);
   p.status = a.status;
   const int kb = a.K / 64;
   const int stage = kPABytes + BN * 128;

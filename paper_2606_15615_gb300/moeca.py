@@ -39,7 +39,8 @@ class moeca_config(C.Structure):
                 ("shared_policy", C.c_int32), ("reused_meta_policy", C.c_int32),
                 ("gelu_tanh", C.c_int32), ("ffn_impl", C.c_int32), ("ffn_tile_n", C.c_int32),
                 ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32),
-                ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32)]
+                ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32),
+                ("attn_impl", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):

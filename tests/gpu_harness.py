@@ -223,13 +223,21 @@ def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
     assert rl <= out_tol[0], f"layer output rel L2 {rl:.3e}"
     if out_tol[1] is not None:
         assert ma <= out_tol[1], f"layer output max abs {ma:.3e}"
+    # A few wrong rows can hide under a global bound: every token row too.
+    row_err = np.linalg.norm(out_gpu - out_o, axis=1) / np.maximum(np.linalg.norm(out_o, axis=1), 1e-30)
+    worst = int(row_err.argmax())
+    assert row_err[worst] <= 4 * out_tol[0], f"layer output row {worst} rel L2 {row_err[worst]:.3e}"
     ch_g = np_of(post["cache_h"]).astype(np.float64)
     fresh = np.zeros((T, k), bool)
     for i, p in np.argwhere(rec_g):
         fresh[i, slot_g[i, p]] = True
     if fresh.any():
+        tol_h = 1e-2 if bf16 else 1e-5
         rf = rel_l2(ch_g[fresh], new_o.cache_h[fresh])
-        assert rf <= (1e-2 if bf16 else 1e-5), f"fresh cache rows rel L2 {rf:.3e}"
+        assert rf <= tol_h, f"fresh cache rows rel L2 {rf:.3e}"
+        per = (np.linalg.norm(ch_g[fresh] - new_o.cache_h[fresh], axis=1)
+               / np.maximum(np.linalg.norm(new_o.cache_h[fresh], axis=1), 1e-30))
+        assert per.max() <= 4 * tol_h, f"worst fresh cache row rel L2 {per.max():.3e}"
     if (~fresh).any() and pre is not None and pre["n_tokens"]:
         assert np.array_equal(ch_g[~fresh], st_pre.cache_h[~fresh]), "reused cache rows changed"
     assert np.array_equal(np_of(post["cache_e"]), new_o.cache_e), "cache expert ids"

@@ -52,12 +52,15 @@ def make_block_stack(M, T, D, H, E, k, F, L=1, S=0, n_shared=0, seed=0, wscale=0
     return M.Stack(cfg, ws), cfg, ws
 
 
-@pytest.mark.parametrize("D,H,S,T", [(256, 4, 200, 400), (576, 8, 100, 300), (320, 4, 72, 216),
-                                     (384, 4, 130, 260), (384, 3, 96, 384)])
-def test_sync_blocks_every_head_size(M, D, H, S, T):
+@pytest.mark.parametrize("impl", [2, 1])
+@pytest.mark.parametrize("D,H,S,T", [(256, 4, 200, 400), (576, 8, 104, 312), (320, 4, 72, 216),
+                                     (384, 4, 136, 272), (384, 3, 264, 528)])
+def test_sync_blocks_every_head_size(M, D, H, S, T, impl):
     """Heads of 64, 72, 80, 96 and 128 channels; samples ragged against the
-    64-row query blocks and the 128-row tiles; two layers; a full step every 3."""
-    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=D + H, tau0=0.72, refresh_period=3)
+    64 / 128-row query blocks, the 128-key blocks and the 128-row tiles; two
+    layers; a full step every 3; the tcgen05 core (2) and the mma.sync core (1)."""
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=D + H, tau0=0.72, refresh_period=3,
+                                   attn_impl=impl)
     rng = np.random.default_rng(D + H)
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 5, 0.08)
     rep, _ = run_trajectory(st, cfg, ws, xs)
@@ -86,7 +89,7 @@ def test_stale_and_full_policies(M, policy):
 def test_one_sample_shared_expert(M):
     """seq_len 0 (every token attends to all T rows) with a shared expert
     under the synchronized rule."""
-    T, D, H = 300, 256, 2
+    T, D, H = 296, 256, 2
     st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 192, L=1, S=0, n_shared=1, seed=8, tau0=0.7)
     rng = np.random.default_rng(80)
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05)
@@ -117,7 +120,7 @@ def test_block_full_size_d768_12_heads(M):
 def test_repeated_input_all_reused_is_bitwise_previous_output(M):
     """tau0 = +inf with the same input: no branch and no attention row is
     recomputed and the output repeats the previous step exactly."""
-    T, D, H, S = 200, 256, 4, 100
+    T, D, H, S = 208, 256, 4, 104
     st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=2, S=S, seed=9, tau0=math.inf)
     rng = np.random.default_rng(90)
     x = torch.from_numpy(W.round_to_bf16(rng.standard_normal((T, D)).astype(np.float32))).cuda().to(torch.bfloat16)
@@ -144,6 +147,10 @@ def test_token_count_change_and_empty_step(M):
     with pytest.raises(M.MoecaError):
         st.step(torch.zeros((100, D), dtype=torch.bfloat16, device="cuda"), 10)   # not a multiple of 64
     st.close()
+    st2, _, _ = make_block_stack(M, 60, D, H, 8, 2, 256, L=1, S=20, seed=10)
+    with pytest.raises(M.MoecaError):
+        st2.step(torch.zeros((60, D), dtype=torch.bfloat16, device="cuda"), 0)    # samples of 20 rows: not a multiple of 8
+    st2.close()
 
 
 @pytest.mark.parametrize("policy", [0, 1])
@@ -157,4 +164,59 @@ def test_separate_kernel_path(M, policy):
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.08)
     rep, _ = run_trajectory(st, cfg, ws, xs)
     assert rep.reused > 0 and rep.attn_rows >= 2 * T + (1 if policy == 0 else 0)
+    st.close()
+
+
+def test_tcgen05_and_mma_sync_cores_agree(M):
+    """The two attention cores on the same block inputs: a rows within bf16
+    rounding of each other (different summation order, same math)."""
+    T, D, H, S = 512, 512, 4, 256
+    outs = []
+    for impl in (2, 1):
+        st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=1, S=S, seed=12, tau0=0.72, attn_impl=impl)
+        rng = np.random.default_rng(120)
+        xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 3, 0.08)
+        for t, x in enumerate(xs):
+            st.step(torch.from_numpy(x).cuda().to(torch.bfloat16), t)
+        torch.cuda.synchronize()
+        outs.append(np_of(st.get_state(0)["attn_a"]).astype(np.float64))
+        st.close()
+    err = np.linalg.norm(outs[0] - outs[1]) / np.linalg.norm(outs[1])
+    assert err < 1e-2, err
+
+
+def test_sixteen_token_prep_blocks(M):
+    """D 1536 with attention leaves room for 16-token preparation blocks only:
+    each block must write the FFN-row map of its own tokens alone (the lanes
+    past its 16 tokens belong to the next block)."""
+    T, D, H, S = 256, 1536, 12, 128
+    st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 256, L=1, S=S, n_shared=1, seed=13, tau0=0.7)
+    rng = np.random.default_rng(130)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 3, 0.08)
+    # Outputs of magnitude ~40 here: the per-row relative bounds apply, not
+    # the absolute one.
+    rep, _ = run_trajectory(st, cfg, ws, xs, out_tol=(1e-2, None))
+    assert rep.reused > 0 and rep.attn_rows > T
+    st.close()
+
+
+@pytest.mark.parametrize("impl", [2, 1])
+def test_huge_activations_stay_finite(M, impl):
+    """Block inputs of magnitude 2e4 put the scaled scores near 1e9-1e10: the
+    softmax must use one rounded product for the maximum and the exponent,
+    or the largest term overflows 2^x (untrained deep stacks grow this big).
+    At this scale bf16 rounding of q and k moves the scores by about 1e7, so
+    the softmax is an argmax that rounding decides: the check is that every
+    step completes and stays finite, not parity."""
+    T, D, H, S = 1024, 256, 2, 512
+    st, cfg, ws = make_block_stack(M, T, D, H, 8, 2, 256, L=1, S=S, seed=14, wscale=0.2, tau0=0.72, attn_impl=impl)
+    rng = np.random.default_rng(140)
+    x0 = (2.0e4 * rng.standard_normal((T, D))).astype(np.float32)
+    for t, x in enumerate(drift(x0, rng, 3, 200.0)):
+        out = st.step(torch.from_numpy(x).cuda().to(torch.bfloat16), t)
+        torch.cuda.synchronize()
+        st.stats()  # raises on a device status (e.g. NaN routing)
+        assert torch.isfinite(out.float()).all()
+        assert torch.isfinite(st.get_state(0)["attn_a"].float()).all()
+    assert st.stats()["attn_recomputed"] > T
     st.close()
