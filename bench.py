@@ -417,11 +417,15 @@ def main():
     ap.add_argument("--ffn-split-k", type=int, default=0, help="force the tensor-core FFN K splits (0: auto)")
     ap.add_argument("--tau0", type=float, default=None,
                     help="use this tau0 for the headline point instead of calibrating it (profiling runs)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only the first N layers of the workload (small ncu captures; not a bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from paper_2606_15615_gb300 import workloads as W
     wl = W.workload(args.workload)
+    if args.layers:
+        wl = wl.scaled(n_layers=min(args.layers, wl.n_layers))
     world, rank, local = dist_env()
 
     if args.impl == "reference":

@@ -13,11 +13,15 @@
 //             128-255), then O += P_{j-1} v_{j-1} (columns 256 ..), so the
 //             scores of block j are computed while block j-1's softmax runs;
 //   warps 2-5 softmax, one query row per thread (TMEM lane quadrant warp % 4):
-//             reads S_j from TMEM (tcgen05.ld), keeps the row maximum m and
-//             sum l in base 2, rescales the O row in TMEM only when m rises
+//             reads S_j from TMEM (tcgen05.ld), keeps the row maximum m in
+//             base 2, rescales the O row in TMEM only when m rises
 //             (tcgen05.ld / st), writes P_j = 2^(s - m) in bf16 into shared
 //             memory in the 128-byte-swizzle K-major layout the MMA reads as
 //             its A operand, and at the end writes o = O / l.
+// The row sum l comes from the tensor core: each v^T tile carries one more
+// channel row of ones (and 15 rows of zeros to keep N a multiple of 16), so
+// O's column DKP accumulates sum_k P[k], from the same rounded P as O and
+// rescaled with it.
 // q k^T contracts over dh rounded up to 16 (heads of 72 channels: 80, the
 // q tile's columns 72-79 zeroed in shared memory); p v produces dh rounded
 // up to 16 columns, of which the first dh are stored.
@@ -48,9 +52,11 @@ struct TcAttnShape {
   static constexpr int KSTEPS = DKP / 16;           // MMAs of q k^T per block
   static constexpr int QBYTES = QSUB * kSubBytes;   // q tile
   static constexpr int KBYTES = QSUB * kSubBytes;   // k block: 128 keys
-  static constexpr int VSUB = DKP * 128;            // v^T sub-block: DKP channels x 64 keys
+  static constexpr int NV = DKP + 16;               // p v width: the channels, then the ones row
+  static constexpr int VSUB = NV * 128;             // v^T sub-block: NV rows x 64 keys
   static constexpr int VBYTES = 2 * VSUB;           // v^T block: 128 keys
   static constexpr int STAGE = KBYTES + VBYTES;
+  static constexpr int STAGE_TX = KBYTES + 2 * DKP * 128;  // bytes TMA writes per stage
   static constexpr int PBYTES = 2 * kSubBytes;      // P: 128 rows x 128 keys
   static constexpr int NST = (200 * 1024 - QBYTES - PBYTES) / STAGE >= 3 ? 3 : 2;
   static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + PBYTES + NST * STAGE + 1024;
@@ -187,7 +193,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
         }
         uint8_t* st = sKV + s * Sh::STAGE;
         const uint32_t bar = smem_u32(&kv_full[s]);
-        mbar_expect_tx(bar, Sh::STAGE);
+        mbar_expect_tx(bar, Sh::STAGE_TX);
         for (int sub = 0; sub < Sh::QSUB; ++sub)
           tma_load_2d(smem_u32(st + sub * kSubBytes), &kmap, h * DH + sub * 64, key0 + j * kTK, bar);
         for (int sub = 0; sub < 2; ++sub)
@@ -197,7 +203,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t id_s = instr_desc(kTQ, kTK), id_o = instr_desc(kTQ, Sh::DKP);
+      const uint32_t id_s = instr_desc(kTQ, kTK), id_o = instr_desc(kTQ, Sh::NV);
       const uint32_t t_o = tmem + 256;
       bool ok = mbar_wait(smem_u32(&q_ready), 0, &abort_flag);
       // O += P_j v_j, then free block j's stage.
@@ -250,6 +256,17 @@ __global__ void __launch_bounds__(kTThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const uint32_t t_o = tmem + lane_off + 256;
     const float sc = p.scale_log2;
+    // The ones row (channel DKP) and 15 zero rows after each v^T sub-block's
+    // channels; TMA never writes them.  Rows DKP.. start an 8-row swizzle
+    // group, and a row of equal chunks is the same under any chunk swizzle.
+    for (int idx = threadIdx.x - 64; idx < NST * 2 * 16 * 8; idx += 128) {
+      const int row = idx >> 3, ch = idx & 7;            // row over (stage, sub-block, 16 rows)
+      const int sv = row >> 4, rr = row & 15;
+      uint8_t* base = sKV + (sv >> 1) * Sh::STAGE + Sh::KBYTES + (sv & 1) * Sh::VSUB + (Sh::DKP + rr) * 128;
+      const uint32_t one2 = 0x3F803F80u;                 // two bf16 1.0
+      *reinterpret_cast<uint4*>(base + ch * 16) = rr == 0 ? make_uint4(one2, one2, one2, one2) : make_uint4(0, 0, 0, 0);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     bool ok = warp_wait(smem_u32(&q_full), 0, &abort_flag);
     if (ok && Sh::DKP > DH) {
       // The q tile's columns DH .. DKP-1 hold the next head's values: zero
@@ -262,7 +279,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     mbar_arrive(smem_u32(&q_ready));
-    float m = -INFINITY, l = 0.f;  // running maximum (scaled, base 2) and sum of this row
+    float m = -INFINITY;  // running maximum of this row (scaled, base 2)
     for (int j = 0; ok && j < nkb; ++j) {
       const int bb = j & 1;
       if (!warp_wait(smem_u32(&s_full[bb]), (j >> 1) & 1, &abort_flag)) {
@@ -272,19 +289,26 @@ __global__ void __launch_bounds__(kTThreads, 1)
       tc_fence_after();
       const uint32_t t_s = tmem + lane_off + bb * kTK;
       const int nvalid = S - j * kTK;  // keys of this block inside the sample (>= 1)
+      const bool full = nvalid >= kTK;  // warp-uniform: only a sample's last block is partial
       float mx = -INFINITY;
 #pragma unroll
       for (int c = 0; c < kTK / 32; ++c) {
         uint32_t v[32];
         tmem_ld32(t_s + c * 32, v);
+        if (full) {
 #pragma unroll
-        for (int q = 0; q < 32; ++q)
-          if (c * 32 + q < nvalid) mx = fmaxf(mx, __fmul_rn(__uint_as_float(v[q]), sc));
+          for (int q = 0; q < 32; ++q) mx = fmaxf(mx, __uint_as_float(v[q]));
+        } else {
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            if (c * 32 + q < nvalid) mx = fmaxf(mx, __uint_as_float(v[q]));
+        }
       }
-      // Both passes use the same rounded product s sc (no fused multiply-add),
-      // so the row's largest term is exactly 2^0: with scores of 1e11 an
-      // unrounded product would differ from m by thousands.
-      const float m_new = fmaxf(m, mx);
+      // The maximum is taken on raw scores and scaled once: rounding is
+      // monotonic, so fl(max s * sc) is the maximum of the fl(s * sc) that
+      // pass 2 forms (no fused multiply-add), and the row's largest term is
+      // exactly 2^0 however large the scores are.
+      const float m_new = fmaxf(m, __fmul_rn(mx, sc));
       if (j >= 1) {
         // O and P are free once block j-1's p v has completed.
         if (!warp_wait(smem_u32(&o_done), (j - 1) & 1, &abort_flag)) {
@@ -295,14 +319,13 @@ __global__ void __launch_bounds__(kTThreads, 1)
         if (__any_sync(0xffffffffu, m_new > m)) {
           const float alpha = ex2f_approx(m - m_new);  // 1 for rows whose maximum held
 #pragma unroll
-          for (int c = 0; c < Sh::DKP / 16; ++c) {
+          for (int c = 0; c < Sh::NV / 16; ++c) {  // the channels and the row sum
             uint32_t v[16];
             tmem_ld16(t_o + c * 16, v);
 #pragma unroll
             for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * alpha);
             tmem_st16(t_o + c * 16, v);
           }
-          l *= alpha;
         }
       }
       m = m_new;
@@ -315,9 +338,12 @@ __global__ void __launch_bounds__(kTThreads, 1)
 #pragma unroll
         for (int q = 0; q < 16; ++q) {
           const int kk = c * 32 + 2 * q;
-          const float p0 = kk < nvalid ? ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q]), sc) - m) : 0.f;
-          const float p1 = kk + 1 < nvalid ? ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q + 1]), sc) - m) : 0.f;
-          l += p0 + p1;
+          float p0 = ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q]), sc) - m);
+          float p1 = ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q + 1]), sc) - m);
+          if (!full) {
+            p0 = kk < nvalid ? p0 : 0.f;
+            p1 = kk + 1 < nvalid ? p1 : 0.f;
+          }
           pk[q] = pack2(p0, p1);
         }
         const int sub = c >> 1;
@@ -336,7 +362,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
     if (ok && !warp_wait(smem_u32(&o_done), (nkb - 1) & 1, &abort_flag)) ok = false;
     if (ok) {
       tc_fence_after();
-      const float inv_l = 1.f / l;
+      uint32_t lv[16];
+      tmem_ld16(t_o + Sh::DKP, lv);  // column DKP: the row sum l
+      const float inv_l = 1.f / __uint_as_float(lv[0]);
       __nv_bfloat16* dst = p.o + static_cast<size_t>(r0 + r) * p.D + h * DH;
 #pragma unroll
       for (int c = 0; c < Sh::DKP / 16; ++c) {

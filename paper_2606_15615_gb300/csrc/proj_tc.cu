@@ -37,6 +37,7 @@
 #include <cuda.h>
 
 #include <cstdio>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -157,7 +158,7 @@ __device__ __forceinline__ void load_x_chunk(const __nv_bfloat16* xr, uint4* xv)
   for (int j = 0; j < 4; ++j) xv[j] = __ldg(reinterpret_cast<const uint4*>(xr) + j);
 }
 
-template <int BN>
+template <int BN, int MODE>
 __global__ void __launch_bounds__(kPThreads, 1)
     proj_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                    const ProjParams p) {
@@ -271,9 +272,9 @@ __global__ void __launch_bounds__(kPThreads, 1)
     const int n_g = p.row_of ? p.row_w : 0;
     __nv_bfloat16* krow = nullptr;  // kProjQKV: this lane's k row (dst holds its q row)
     if (m < M) {
-      if (p.mode == kProjStore) {
+      if constexpr (MODE == kProjStore) {
         dst = p.out + static_cast<size_t>(m) * p.ldo + n0;
-      } else if (p.mode == kProjQKV) {
+      } else if constexpr (MODE == kProjQKV) {
         const int qi = p.inv ? p.inv[m] : m;
         const int Dm = p.N / 3;
         if (qi >= 0) dst = p.q_out + static_cast<size_t>(qi) * Dm;
@@ -297,46 +298,62 @@ __global__ void __launch_bounds__(kPThreads, 1)
         }
       }
     }
-    uint4 xb[2][4];  // x of chunks c and c + 1 in flight
-    if (xr) {
-      load_x_chunk(xr, xb[0]);
-      if (BN > 32) load_x_chunk(xr + 32, xb[1]);
+    uint4 xb[2][4];  // residual mode: x of chunks c and c + 1 in flight
+    if constexpr (MODE == kProjResidual) {
+      if (xr) {
+        load_x_chunk(xr, xb[0]);
+        if (BN > 32) load_x_chunk(xr + 32, xb[1]);
+      }
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps: bias staged
     if (mbar_wait(smem_u32(&acc_bar), 0, &abort_flag)) {
       tc_fence_after();
       const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+      if constexpr (MODE == kProjResidual) {
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
-        uint4 xc[4];
+        for (int c = 0; c < BN / 32; ++c) {
+          uint4 xc[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) xc[j] = xb[c & 1][j];
-        if (xr && c + 2 < BN / 32) load_x_chunk(xr + (c + 2) * 32, xb[c & 1]);  // two chunks ahead
-        uint32_t raw[32];
-        tmem_ld32(tbase + c * 32, raw);
-        float v[32];
+          for (int j = 0; j < 4; ++j) xc[j] = xb[c & 1][j];
+          if (xr && c + 2 < BN / 32) load_x_chunk(xr + (c + 2) * 32, xb[c & 1]);  // two chunks ahead
+          uint32_t raw[32];
+          tmem_ld32(tbase + c * 32, raw);
+          float v[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
-        if (p.mode == kProjStore) {
-          store_chunk_staged(stage, v, dst ? dst + c * 32 : nullptr, lane);
-        } else if (p.mode == kProjQKV) {
-          // The chunk lies in one of q, k, v (D is a multiple of 64): warp-uniform.
-          const int Dm = p.N / 3;
-          const int col = n0 + c * 32;
-          const int region = col / Dm, cc = col - region * Dm;
-          if (region == 0) {
-            store_chunk_staged(stage, v, dst ? dst + cc : nullptr, lane);
-          } else if (region == 1) {
-            store_chunk_staged(stage, v, krow ? krow + cc : nullptr, lane);
-          } else {
-            store_chunk_transposed(stage, v, p.vt_out + static_cast<size_t>(cc) * p.n_tok, m0 + quad * 32, M,
-                                   static_cast<size_t>(p.n_tok), lane);
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
+          if (dst) {
+            __nv_bfloat16* gc[kMaxRowOf];
+#pragma unroll
+            for (int q = 0; q < kMaxRowOf; ++q) gc[q] = gr[q] ? gr[q] + c * 32 : nullptr;
+            store_residual(v, xc, dst + c * 32, ur + c * 32, gc, n_g);
           }
-        } else if (dst) {
-          __nv_bfloat16* gc[kMaxRowOf];
+        }
+      } else {
+        // Store-type epilogues stay rolled: the chunk body is large and an
+        // unrolled copy per chunk spills out of the instruction cache.
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t raw[32];
+          tmem_ld32(tbase + c * 32, raw);
+          float v[32];
 #pragma unroll
-          for (int q = 0; q < kMaxRowOf; ++q) gc[q] = gr[q] ? gr[q] + c * 32 : nullptr;
-          store_residual(v, xc, dst + c * 32, ur + c * 32, gc, n_g);
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
+          if constexpr (MODE == kProjStore) {
+            store_chunk_staged(stage, v, dst ? dst + c * 32 : nullptr, lane);
+          } else {
+            // The chunk lies in one of q, k, v (D is a multiple of 64): warp-uniform.
+            const int Dm = p.N / 3;
+            const int col = n0 + c * 32;
+            const int region = col / Dm, cc = col - region * Dm;
+            if (region == 0) {
+              store_chunk_staged(stage, v, dst ? dst + cc : nullptr, lane);
+            } else if (region == 1) {
+              store_chunk_staged(stage, v, krow ? krow + cc : nullptr, lane);
+            } else {
+              store_chunk_transposed(stage, v, p.vt_out + static_cast<size_t>(cc) * p.n_tok, m0 + quad * 32, M,
+                                     static_cast<size_t>(p.n_tok), lane);
+            }
+          }
         }
       }
     } else if (lane == 0) {
@@ -416,10 +433,18 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     return launch_pdl(kern, grid, dim3(kPThreads), smem, s, amap, bmap, p);
   };
+  auto by_mode = [&](auto bn) -> cudaError_t {
+    constexpr int kBN = decltype(bn)::value;
+    switch (a.mode) {
+      case kProjQKV: return run(proj_tc_kernel<kBN, kProjQKV>);
+      case kProjResidual: return run(proj_tc_kernel<kBN, kProjResidual>);
+      default: return run(proj_tc_kernel<kBN, kProjStore>);
+    }
+  };
   switch (BN) {
-    case 256: return run(proj_tc_kernel<256>);
-    case 128: return run(proj_tc_kernel<128>);
-    default: return run(proj_tc_kernel<64>);
+    case 256: return by_mode(std::integral_constant<int, 256>{});
+    case 128: return by_mode(std::integral_constant<int, 128>{});
+    default: return by_mode(std::integral_constant<int, 64>{});
   }
 }
 
