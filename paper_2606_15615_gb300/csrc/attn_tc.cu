@@ -12,7 +12,10 @@
 //             thread: S_j = q k_j^T into one of two S buffers (columns 0-127,
 //             128-255), then O += P_{j-1} v_{j-1} (columns 256 ..), so the
 //             scores of block j are computed while block j-1's softmax runs;
-//   warps 2-5 softmax, one query row per thread (TMEM lane quadrant warp % 4):
+//   warps 2-9 softmax, two warps per TMEM lane quadrant (warp % 4), each
+//             thread one query row and one half (64 keys) of each block; the
+//             two halves of a row exchange their maxima through shared
+//             memory and a bounded barrier.  Per thread:
 //             reads S_j from TMEM (tcgen05.ld), keeps the row maximum m in
 //             base 2, rescales the O row in TMEM only when m rises
 //             (tcgen05.ld / st), writes P_j = 2^(s - m) in bf16 into shared
@@ -42,7 +45,8 @@ namespace {
 
 constexpr int kTQ = 128;        // query rows per CTA (MMA M)
 constexpr int kTK = 128;        // keys per block (N of q k^T, K of p v)
-constexpr int kTThreads = 192;
+constexpr int kTThreads = 320;  // warps 0-1 copy and issue, warps 2-9 softmax
+constexpr int kSoftThreads = 256;
 constexpr int kSubBytes = 128 * 128;  // one 128-row x 64-column bf16 sub-block (16 KB)
 
 template <int DH>
@@ -57,9 +61,8 @@ struct TcAttnShape {
   static constexpr int VBYTES = 2 * VSUB;           // v^T block: 128 keys
   static constexpr int STAGE = KBYTES + VBYTES;
   static constexpr int STAGE_TX = KBYTES + 2 * DKP * 128;  // bytes TMA writes per stage
-  static constexpr int PBYTES = 2 * kSubBytes;      // P: 128 rows x 128 keys
-  static constexpr int NST = (200 * 1024 - QBYTES - PBYTES) / STAGE >= 3 ? 3 : 2;
-  static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + PBYTES + NST * STAGE + 1024;
+  static constexpr int NST = (200 * 1024 - QBYTES) / STAGE >= 3 ? 3 : 2;
+  static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + NST * STAGE + 1024;
 };
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* v) {
@@ -80,6 +83,28 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
         "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
       : "memory");
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};"
+      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+        "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]),
+        "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// D (TMEM) += A (TMEM, M rows on the lanes, K packed two bf16 per column) x B (shared memory).
+__device__ __forceinline__ void mma_bf16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}"
+      ::"r"(d_tmem), "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
 }
 
 __device__ __forceinline__ float ex2f_approx(float x) {
@@ -123,15 +148,16 @@ __global__ void __launch_bounds__(kTThreads, 1)
   using Sh = TcAttnShape<DH>;
   constexpr int NST = Sh::NST;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t q_full, q_ready, p_full, o_done, drain_bar;
-  __shared__ __align__(8) uint64_t s_full[2], s_free[2], kv_full[NST], kv_empty[NST];
+  __shared__ __align__(8) uint64_t q_full, q_ready, p_full, drain_bar;
+  __shared__ __align__(8) uint64_t o_done[2];  // p v of block j completes a phase of o_done[j & 1]
+  __shared__ __align__(8) uint64_t s_full[2], kv_full[NST], kv_empty[NST], max_bar[2];
+  __shared__ float s_max[2][2][kTQ];  // [block parity][key half][row]: partial row maxima
   __shared__ uint32_t tmem_sh;
   __shared__ volatile int abort_flag;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
-  uint8_t* sP = smem + Sh::QBYTES;
-  uint8_t* sKV = sP + Sh::PBYTES;  // stage s: k block at + s STAGE, v^T block after it
+  uint8_t* sKV = smem + Sh::QBYTES;  // stage s: k block at + s STAGE, v^T block after it
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.y, h = blockIdx.z;
   const int S = p.S, key0 = b * S;
@@ -139,13 +165,14 @@ __global__ void __launch_bounds__(kTThreads, 1)
   if (threadIdx.x == 0) {
     abort_flag = 0;
     mbar_init(smem_u32(&q_full), 1);
-    mbar_init(smem_u32(&q_ready), 128);
-    mbar_init(smem_u32(&p_full), 128);
-    mbar_init(smem_u32(&o_done), 1);
+    mbar_init(smem_u32(&q_ready), kSoftThreads);
+    mbar_init(smem_u32(&p_full), kSoftThreads);
+    mbar_init(smem_u32(&o_done[0]), 1);
+    mbar_init(smem_u32(&o_done[1]), 1);
     mbar_init(smem_u32(&drain_bar), 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_free[i]), 128);
+      mbar_init(smem_u32(&max_bar[i]), kSoftThreads);
     }
     for (int i = 0; i < NST; ++i) {
       mbar_init(smem_u32(&kv_full[i]), 1);
@@ -210,22 +237,23 @@ __global__ void __launch_bounds__(kTThreads, 1)
       auto pv = [&](int j) -> bool {
         if (!mbar_wait(smem_u32(&p_full), j & 1, &abort_flag)) return false;
         tc_fence_after();
-        const uint32_t pa = smem_u32(sP);
+        // P_j sits in S_j's TMEM columns, two bf16 per column: 8 columns per 16 keys.
+        const uint32_t pa = tmem + (j & 1) * kTK;
         const uint32_t vb = smem_u32(sKV + (j % NST) * Sh::STAGE + Sh::KBYTES);
 #pragma unroll
         for (int kk = 0; kk < kTK / 16; ++kk) {
           const int sub = kk >> 2, off = (kk & 3) * 32;
-          mma_bf16(t_o, smem_desc(pa + sub * kSubBytes + off), smem_desc(vb + sub * Sh::VSUB + off), id_o,
-                   (j > 0) || (kk > 0));
+          mma_bf16_ta(t_o, pa + kk * 8, smem_desc(vb + sub * Sh::VSUB + off), id_o, (j > 0) || (kk > 0));
         }
-        mma_commit(smem_u32(&o_done));
+        mma_commit(smem_u32(&o_done[j & 1]));
         mma_commit(smem_u32(&kv_empty[j % NST]));
         return true;
       };
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j % NST, bb = j & 1;
-        if (!mbar_wait(smem_u32(&kv_full[s]), (j / NST) & 1, &abort_flag) ||
-            (j >= 2 && !mbar_wait(smem_u32(&s_free[bb]), ((j >> 1) - 1) & 1, &abort_flag))) {
+        // S_j overwrites S_{j-2} / P_{j-2}: p v of block j-2 was issued
+        // before this, and MMAs of one thread run in issue order.
+        if (!mbar_wait(smem_u32(&kv_full[s]), (j / NST) & 1, &abort_flag)) {
           ok = false;
           break;
         }
@@ -250,25 +278,30 @@ __global__ void __launch_bounds__(kTThreads, 1)
       drain_wait(smem_u32(&drain_bar), 0);
     }
   } else {
-    // ---- softmax: one query row per thread
+    // ---- softmax: one query row and one key half per thread
     const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;  // keys [half 64, half 64 + 64) of each block
     const int r = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const uint32_t t_o = tmem + lane_off + 256;
+    constexpr int NCH = Sh::NV / 16;      // O chunks of 16 columns (the row sum's included)
+    constexpr int C0 = (NCH + 1) / 2;     // half 0 rescales / stores chunks [0, C0), half 1 the rest
+    const int cb = half ? C0 : 0, ce = half ? NCH : C0;
     const float sc = p.scale_log2;
     // The ones row (channel DKP) and 15 zero rows after each v^T sub-block's
     // channels; TMA never writes them.  Rows DKP.. start an 8-row swizzle
     // group, and a row of equal chunks is the same under any chunk swizzle.
-    for (int idx = threadIdx.x - 64; idx < NST * 2 * 16 * 8; idx += 128) {
-      const int row = idx >> 3, ch = idx & 7;            // row over (stage, sub-block, 16 rows)
+    for (int idx = threadIdx.x - 64; idx < NST * 2 * 16 * 8; idx += kSoftThreads) {
+      const int row = idx >> 3, ch = idx & 7;  // row over (stage, sub-block, 16 rows)
       const int sv = row >> 4, rr = row & 15;
       uint8_t* base = sKV + (sv >> 1) * Sh::STAGE + Sh::KBYTES + (sv & 1) * Sh::VSUB + (Sh::DKP + rr) * 128;
-      const uint32_t one2 = 0x3F803F80u;                 // two bf16 1.0
-      *reinterpret_cast<uint4*>(base + ch * 16) = rr == 0 ? make_uint4(one2, one2, one2, one2) : make_uint4(0, 0, 0, 0);
+      const uint32_t one2 = 0x3F803F80u;       // two bf16 1.0
+      *reinterpret_cast<uint4*>(base + ch * 16) =
+          rr == 0 ? make_uint4(one2, one2, one2, one2) : make_uint4(0, 0, 0, 0);
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     bool ok = warp_wait(smem_u32(&q_full), 0, &abort_flag);
-    if (ok && Sh::DKP > DH) {
+    if (ok && Sh::DKP > DH && half == 0) {
       // The q tile's columns DH .. DKP-1 hold the next head's values: zero
       // them so they add nothing to q k^T (k's columns there are finite).
 #pragma unroll
@@ -279,7 +312,22 @@ __global__ void __launch_bounds__(kTThreads, 1)
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     mbar_arrive(smem_u32(&q_ready));
-    float m = -INFINITY;  // running maximum of this row (scaled, base 2)
+    float m = -INFINITY;  // this row's reference maximum (scaled, base 2)
+    // Completions of each o_done barrier are observed in order.  At block j
+    // the latest p v that can have completed is block j-1's, so neither
+    // barrier is ever more than one completion past its next wait (no
+    // parity aliasing).
+    int obs[2] = {0, 1};  // next unobserved p v block of each parity
+    auto wait_pv = [&](int i) -> bool {  // p v of block i complete
+      if (i < 0) return true;
+      const int b2 = i & 1;
+      while (obs[b2] <= i) {
+        if (!warp_wait(smem_u32(&o_done[b2]), (obs[b2] >> 1) & 1, &abort_flag)) return false;
+        obs[b2] += 2;
+      }
+      tc_fence_after();
+      return true;
+    };
     for (int j = 0; ok && j < nkb; ++j) {
       const int bb = j & 1;
       if (!warp_wait(smem_u32(&s_full[bb]), (j >> 1) & 1, &abort_flag)) {
@@ -287,99 +335,99 @@ __global__ void __launch_bounds__(kTThreads, 1)
         break;
       }
       tc_fence_after();
-      const uint32_t t_s = tmem + lane_off + bb * kTK;
-      const int nvalid = S - j * kTK;  // keys of this block inside the sample (>= 1)
-      const bool full = nvalid >= kTK;  // warp-uniform: only a sample's last block is partial
+      const uint32_t t_s = tmem + lane_off + bb * kTK + half * 64;
+      const int nvalid = S - j * kTK - half * 64;  // keys of this half inside the sample (may be <= 0)
+      const bool full = nvalid >= 64;              // warp-uniform
+      uint32_t sv[64];                             // this half's scores, kept for pass 2
+      tmem_ld32(t_s, sv);
+      tmem_ld32(t_s + 32, sv + 32);
       float mx = -INFINITY;
+      if (full) {
 #pragma unroll
-      for (int c = 0; c < kTK / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(t_s + c * 32, v);
-        if (full) {
+        for (int q = 0; q < 64; ++q) mx = fmaxf(mx, __uint_as_float(sv[q]));
+      } else {
 #pragma unroll
-          for (int q = 0; q < 32; ++q) mx = fmaxf(mx, __uint_as_float(v[q]));
-        } else {
-#pragma unroll
-          for (int q = 0; q < 32; ++q)
-            if (c * 32 + q < nvalid) mx = fmaxf(mx, __uint_as_float(v[q]));
-        }
+        for (int q = 0; q < 64; ++q)
+          if (q < nvalid) mx = fmaxf(mx, __uint_as_float(sv[q]));
       }
+      // Exchange with the other half of the row; past this point both halves
+      // have read S_j, so P_j may overwrite it.
+      s_max[bb][half][r] = mx;
+      tc_fence_before();
+      mbar_arrive(smem_u32(&max_bar[bb]));
+      if (!warp_wait(smem_u32(&max_bar[bb]), (j >> 1) & 1, &abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      mx = fmaxf(mx, s_max[bb][half ^ 1][r]);
       // The maximum is taken on raw scores and scaled once: rounding is
       // monotonic, so fl(max s * sc) is the maximum of the fl(s * sc) that
-      // pass 2 forms (no fused multiply-add), and the row's largest term is
-      // exactly 2^0 however large the scores are.
-      const float m_new = fmaxf(m, __fmul_rn(mx, sc));
-      if (j >= 1) {
-        // O and P are free once block j-1's p v has completed.
-        if (!warp_wait(smem_u32(&o_done), (j - 1) & 1, &abort_flag)) {
+      // pass 2 forms (no fused multiply-add).
+      const float cand = fmaxf(m, __fmul_rn(mx, sc));
+      // Lazy rescaling: the reference maximum moves (and O is rescaled) only
+      // when some row of the warp rises by more than 2^8; otherwise P keeps
+      // the old reference and stays below 2^8.  The rows of a warp are the
+      // same in both halves, so both take the same decision.
+      if (j == 0) {
+        m = cand;
+      } else if (__any_sync(0xffffffffu, cand > m + 8.f)) {
+        if (!wait_pv(j - 2) || !wait_pv(j - 1)) {  // O is quiet: p v of every earlier block done
           ok = false;
           break;
         }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, m_new > m)) {
-          const float alpha = ex2f_approx(m - m_new);  // 1 for rows whose maximum held
+        const float alpha = ex2f_approx(m - cand);
+        for (int c = cb; c < ce; ++c) {
+          uint32_t v[16];
+          tmem_ld16(t_o + c * 16, v);
 #pragma unroll
-          for (int c = 0; c < Sh::NV / 16; ++c) {  // the channels and the row sum
-            uint32_t v[16];
-            tmem_ld16(t_o + c * 16, v);
-#pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * alpha);
-            tmem_st16(t_o + c * 16, v);
-          }
+          for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * alpha);
+          tmem_st16(t_o + c * 16, v);
         }
+        m = cand;
       }
-      m = m_new;
-      // P_j = 2^(s sc - m) in bf16, written as the 128-byte-swizzle K-major A tile.
-#pragma unroll
-      for (int c = 0; c < kTK / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(t_s + c * 32, v);
-        uint32_t pk[16];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const int kk = c * 32 + 2 * q;
-          float p0 = ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q]), sc) - m);
-          float p1 = ex2f_approx(__fmul_rn(__uint_as_float(v[2 * q + 1]), sc) - m);
-          if (!full) {
-            p0 = kk < nvalid ? p0 : 0.f;
-            p1 = kk + 1 < nvalid ? p1 : 0.f;
-          }
-          pk[q] = pack2(p0, p1);
-        }
-        const int sub = c >> 1;
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const int ch = (c & 1) * 4 + q4;
-          *reinterpret_cast<uint4*>(sP + sub * kSubBytes + r * 128 + ((ch ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
-        }
+      // Keep the o_done observations in step: block j-2's p v finished long ago.
+      if (!wait_pv(j - 2)) {
+        ok = false;
+        break;
       }
+      // P_j = 2^(s sc - m) in bf16, packed two per column into S_j's own
+      // columns: this half's 64 keys are columns [half 32, half 32 + 32).
+      uint32_t pk[32];
+#pragma unroll
+      for (int q = 0; q < 32; ++q) {
+        float p0 = ex2f_approx(__fmul_rn(__uint_as_float(sv[2 * q]), sc) - m);
+        float p1 = ex2f_approx(__fmul_rn(__uint_as_float(sv[2 * q + 1]), sc) - m);
+        if (!full) {
+          p0 = 2 * q < nvalid ? p0 : 0.f;
+          p1 = 2 * q + 1 < nvalid ? p1 : 0.f;
+        }
+        pk[q] = pack2(p0, p1);
+      }
+      tmem_st32(tmem + lane_off + bb * kTK + half * 32, pk);
       tc_fence_before();
-      mbar_arrive(smem_u32(&s_free[bb]));
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_arrive(smem_u32(&p_full));
     }
-    if (ok && !warp_wait(smem_u32(&o_done), (nkb - 1) & 1, &abort_flag)) ok = false;
+    if (ok && (!wait_pv(nkb - 2) || !wait_pv(nkb - 1))) ok = false;
     if (ok) {
-      tc_fence_after();
       uint32_t lv[16];
       tmem_ld16(t_o + Sh::DKP, lv);  // column DKP: the row sum l
       const float inv_l = 1.f / __uint_as_float(lv[0]);
       __nv_bfloat16* dst = p.o + static_cast<size_t>(r0 + r) * p.D + h * DH;
-#pragma unroll
-      for (int c = 0; c < Sh::DKP / 16; ++c) {
+      for (int c = cb; c < ce; ++c) {
+        if (c * 16 >= DH) break;        // warp-uniform: the row-sum chunk is not stored
         uint32_t v[16];
-        tmem_ld16(t_o + c * 16, v);  // every lane: the load is warp-collective
+        tmem_ld16(t_o + c * 16, v);     // every lane: the load is warp-collective
         if (r < nq) {
 #pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            const int col = c * 16 + half * 8;
+          for (int hh = 0; hh < 2; ++hh) {
+            const int col = c * 16 + hh * 8;
             if (col < DH) {
               uint4 w;
-              w.x = pack2(__uint_as_float(v[half * 8 + 0]) * inv_l, __uint_as_float(v[half * 8 + 1]) * inv_l);
-              w.y = pack2(__uint_as_float(v[half * 8 + 2]) * inv_l, __uint_as_float(v[half * 8 + 3]) * inv_l);
-              w.z = pack2(__uint_as_float(v[half * 8 + 4]) * inv_l, __uint_as_float(v[half * 8 + 5]) * inv_l);
-              w.w = pack2(__uint_as_float(v[half * 8 + 6]) * inv_l, __uint_as_float(v[half * 8 + 7]) * inv_l);
+              w.x = pack2(__uint_as_float(v[hh * 8 + 0]) * inv_l, __uint_as_float(v[hh * 8 + 1]) * inv_l);
+              w.y = pack2(__uint_as_float(v[hh * 8 + 2]) * inv_l, __uint_as_float(v[hh * 8 + 3]) * inv_l);
+              w.z = pack2(__uint_as_float(v[hh * 8 + 4]) * inv_l, __uint_as_float(v[hh * 8 + 5]) * inv_l);
+              w.w = pack2(__uint_as_float(v[hh * 8 + 6]) * inv_l, __uint_as_float(v[hh * 8 + 7]) * inv_l);
               *reinterpret_cast<uint4*>(dst + col) = w;
             }
           }
