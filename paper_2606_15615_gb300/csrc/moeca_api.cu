@@ -492,10 +492,12 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ProjArgs oa{};
     oa.A = h->attn_o; oa.a_rows = T; oa.B = L.w.w_o; oa.bias = L.w.b_o;
     oa.M = T; oa.N = c.hidden; oa.K = c.hidden; oa.mode = kProjResidual;
-    // Narrow tiles: the recomputed rows are few and the residual epilogue
-    // (x in; a, u and the FFN rows out) is latency-bound, so more CTAs with
-    // two 32-column chunks each beat fewer wide ones.
-    oa.tile_n = 64;
+    // Narrow tiles at moderate width: the recomputed rows are few and the
+    // residual epilogue (x in; a, u and the FFN rows out) is latency-bound,
+    // so more CTAs with two 32-column chunks each beat fewer wide ones.  At
+    // D above 2048 the K loop dominates and narrow tiles would re-read the
+    // operands four times over: the widest tile.
+    oa.tile_n = c.hidden > 2048 ? 0 : 64;
     oa.n_tok = T; oa.x = in; oa.a_out = L.attn_a; oa.u_out = L.attn_u;
     oa.row_stat = L.stats + kStAttnRows; oa.status = h->status_dev;
     if (attn_sync) {

@@ -220,3 +220,17 @@ def test_huge_activations_stay_finite(M, impl):
         assert torch.isfinite(st.get_state(0)["attn_a"].float()).all()
     assert st.stats()["attn_recomputed"] > T
     st.close()
+
+
+def test_wide_block_separate_path(M):
+    """D 2560 with 20 heads of 128: the preparation kernel does not fit next to
+    the cached attention rows, so the separate router / select / compact
+    kernels run with the tensor-core FFN; the output projection takes 256-wide
+    tiles (residual epilogue over eight chunks)."""
+    T, D, H, S = 256, 2560, 20, 256
+    st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 512, L=1, S=S, n_shared=1, seed=15, wscale=0.02, tau0=0.7)
+    rng = np.random.default_rng(150)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 3, 0.08)
+    rep, _ = run_trajectory(st, cfg, ws, xs, out_tol=(1e-2, None))
+    assert rep.reused > 0 and rep.attn_rows > T
+    st.close()
