@@ -5,9 +5,11 @@
 // running maximum and sum (online softmax).
 //
 // One CTA per (128 query rows, sample, head), 6 warps:
-//   warp 0    TMA producer: the q tile once, then per block of 128 keys the
-//             k block (K-major, 128-byte swizzle) and the v^T block
-//             (channels x keys, K-major for p v) into a ring of stages;
+//   warp 0    TMA producers: lane 0 loads the q tile once, then per block of
+//             128 keys the k block (K-major, 128-byte swizzle) into a ring of
+//             two or three, freed as soon as q k^T has read it; lane 1 loads
+//             the v^T block (channels x keys, K-major for p v) into a ring of
+//             three, freed by p v;
 //   warp 1    allocates 512 TMEM columns and issues tcgen05.mma from one
 //             thread: S_j = q k_j^T into one of two S buffers (columns 0-127,
 //             128-255), then O += P_{j-1} v_{j-1} (columns 256 ..), so the
@@ -59,10 +61,14 @@ struct TcAttnShape {
   static constexpr int NV = DKP + 16;               // p v width: the channels, then the ones row
   static constexpr int VSUB = NV * 128;             // v^T sub-block: NV rows x 64 keys
   static constexpr int VBYTES = 2 * VSUB;           // v^T block: 128 keys
-  static constexpr int STAGE = KBYTES + VBYTES;
-  static constexpr int STAGE_TX = KBYTES + 2 * DKP * 128;  // bytes TMA writes per stage
-  static constexpr int NST = (200 * 1024 - QBYTES) / STAGE >= 3 ? 3 : 2;
-  static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + NST * STAGE + 1024;
+  static constexpr int V_TX = 2 * DKP * 128;        // bytes TMA writes per v^T block
+  // Separate rings: a k block is free once q k^T has used it, a v^T block
+  // once p v has.  A strided v^T box takes about 2.7 us to land, so v^T runs
+  // three blocks ahead; k three if that still fits, else two (a k block is
+  // needed one softmax earlier but freed one p v earlier).
+  static constexpr int NV_ST = 3;
+  static constexpr int NK = QBYTES + 3 * KBYTES + NV_ST * VBYTES <= 212 * 1024 ? 3 : 2;
+  static constexpr size_t SMEM = static_cast<size_t>(QBYTES) + NK * KBYTES + NV_ST * VBYTES + 1024;
 };
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* v) {
@@ -146,18 +152,21 @@ __global__ void __launch_bounds__(kTThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                    const __grid_constant__ CUtensorMap vmap, const TcAttnParams p) {
   using Sh = TcAttnShape<DH>;
-  constexpr int NST = Sh::NST;
+  constexpr int NK = Sh::NK, NVS = Sh::NV_ST;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t q_full, q_ready, p_full, drain_bar;
   __shared__ __align__(8) uint64_t o_done[2];  // p v of block j completes a phase of o_done[j & 1]
-  __shared__ __align__(8) uint64_t s_full[2], kv_full[NST], kv_empty[NST], max_bar[2];
+  __shared__ __align__(8) uint64_t s_full[2], max_bar[2];
+  __shared__ __align__(8) uint64_t k_full[NK], k_empty[NK], v_full[NVS], v_empty[NVS];
+  __shared__ int s_issued[2];  // k and v^T blocks each producer lane issued (for the drain)
   __shared__ float s_max[2][2][kTQ];  // [block parity][key half][row]: partial row maxima
   __shared__ uint32_t tmem_sh;
   __shared__ volatile int abort_flag;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
-  uint8_t* sKV = smem + Sh::QBYTES;  // stage s: k block at + s STAGE, v^T block after it
+  uint8_t* sK = smem + Sh::QBYTES;          // k ring: NK blocks of KBYTES
+  uint8_t* sV = sK + NK * Sh::KBYTES;        // v^T ring: NVS blocks of VBYTES
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.y, h = blockIdx.z;
   const int S = p.S, key0 = b * S;
@@ -174,10 +183,15 @@ __global__ void __launch_bounds__(kTThreads, 1)
       mbar_init(smem_u32(&s_full[i]), 1);
       mbar_init(smem_u32(&max_bar[i]), kSoftThreads);
     }
-    for (int i = 0; i < NST; ++i) {
-      mbar_init(smem_u32(&kv_full[i]), 1);
-      mbar_init(smem_u32(&kv_empty[i]), 1);
+    for (int i = 0; i < NK; ++i) {
+      mbar_init(smem_u32(&k_full[i]), 1);
+      mbar_init(smem_u32(&k_empty[i]), 1);
     }
+    for (int i = 0; i < NVS; ++i) {
+      mbar_init(smem_u32(&v_full[i]), 1);
+      mbar_init(smem_u32(&v_empty[i]), 1);
+    }
+    s_issued[0] = s_issued[1] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
@@ -204,29 +218,44 @@ __global__ void __launch_bounds__(kTThreads, 1)
   tc_fence_after();
   const uint32_t tmem = tmem_sh;
   const int nkb = (S + kTK - 1) / kTK;
-  int issued = 0;  // producer: k / v blocks issued
-
   if (warp == 0) {
+    // Lane 0 fills the k ring (and loads q first), lane 1 the v^T ring; the
+    // two lanes run independent loops.
     if (lane == 0) {
       mbar_expect_tx(smem_u32(&q_full), Sh::QBYTES);
       for (int sub = 0; sub < Sh::QSUB; ++sub)
         tma_load_2d(smem_u32(sQ + sub * kSubBytes), &qmap, h * DH + sub * 64, r0, smem_u32(&q_full));
+      int n = 0;
       for (int j = 0; j < nkb; ++j) {
-        const int s = j % NST;
-        if (j >= NST && !mbar_wait(smem_u32(&kv_empty[s]), ((j / NST) - 1) & 1, &abort_flag)) {
+        const int s = j % NK;
+        if (j >= NK && !mbar_wait(smem_u32(&k_empty[s]), ((j / NK) - 1) & 1, &abort_flag)) {
           if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 700);
           abort_flag = 1;
           break;
         }
-        uint8_t* st = sKV + s * Sh::STAGE;
-        const uint32_t bar = smem_u32(&kv_full[s]);
-        mbar_expect_tx(bar, Sh::STAGE_TX);
+        const uint32_t bar = smem_u32(&k_full[s]);
+        mbar_expect_tx(bar, Sh::KBYTES);
         for (int sub = 0; sub < Sh::QSUB; ++sub)
-          tma_load_2d(smem_u32(st + sub * kSubBytes), &kmap, h * DH + sub * 64, key0 + j * kTK, bar);
-        for (int sub = 0; sub < 2; ++sub)
-          tma_load_2d(smem_u32(st + Sh::KBYTES + sub * Sh::VSUB), &vmap, key0 + j * kTK + sub * 64, h * DH, bar);
-        ++issued;
+          tma_load_2d(smem_u32(sK + s * Sh::KBYTES + sub * kSubBytes), &kmap, h * DH + sub * 64, key0 + j * kTK, bar);
+        ++n;
       }
+      s_issued[0] = n;
+    } else if (lane == 1) {
+      int n = 0;
+      for (int j = 0; j < nkb; ++j) {
+        const int s = j % NVS;
+        if (j >= NVS && !mbar_wait(smem_u32(&v_empty[s]), ((j / NVS) - 1) & 1, &abort_flag)) {
+          if (!abort_flag) report_status(p.status, kStatusWaitTimeout, 703);
+          abort_flag = 1;
+          break;
+        }
+        const uint32_t bar = smem_u32(&v_full[s]);
+        mbar_expect_tx(bar, Sh::V_TX);
+        for (int sub = 0; sub < 2; ++sub)
+          tma_load_2d(smem_u32(sV + s * Sh::VBYTES + sub * Sh::VSUB), &vmap, key0 + j * kTK + sub * 64, h * DH, bar);
+        ++n;
+      }
+      s_issued[1] = n;
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -235,30 +264,32 @@ __global__ void __launch_bounds__(kTThreads, 1)
       bool ok = mbar_wait(smem_u32(&q_ready), 0, &abort_flag);
       // O += P_j v_j, then free block j's stage.
       auto pv = [&](int j) -> bool {
-        if (!mbar_wait(smem_u32(&p_full), j & 1, &abort_flag)) return false;
+        if (!mbar_wait(smem_u32(&p_full), j & 1, &abort_flag) ||
+            !mbar_wait(smem_u32(&v_full[j % NVS]), (j / NVS) & 1, &abort_flag))
+          return false;
         tc_fence_after();
         // P_j sits in S_j's TMEM columns, two bf16 per column: 8 columns per 16 keys.
         const uint32_t pa = tmem + (j & 1) * kTK;
-        const uint32_t vb = smem_u32(sKV + (j % NST) * Sh::STAGE + Sh::KBYTES);
+        const uint32_t vb = smem_u32(sV + (j % NVS) * Sh::VBYTES);
 #pragma unroll
         for (int kk = 0; kk < kTK / 16; ++kk) {
           const int sub = kk >> 2, off = (kk & 3) * 32;
           mma_bf16_ta(t_o, pa + kk * 8, smem_desc(vb + sub * Sh::VSUB + off), id_o, (j > 0) || (kk > 0));
         }
         mma_commit(smem_u32(&o_done[j & 1]));
-        mma_commit(smem_u32(&kv_empty[j % NST]));
+        mma_commit(smem_u32(&v_empty[j % NVS]));
         return true;
       };
       for (int j = 0; ok && j < nkb; ++j) {
-        const int s = j % NST, bb = j & 1;
+        const int s = j % NK, bb = j & 1;
         // S_j overwrites S_{j-2} / P_{j-2}: p v of block j-2 was issued
         // before this, and MMAs of one thread run in issue order.
-        if (!mbar_wait(smem_u32(&kv_full[s]), (j / NST) & 1, &abort_flag)) {
+        if (!mbar_wait(smem_u32(&k_full[s]), (j / NK) & 1, &abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t qa = smem_u32(sQ), kb = smem_u32(sKV + s * Sh::STAGE);
+        const uint32_t qa = smem_u32(sQ), kb = smem_u32(sK + s * Sh::KBYTES);
 #pragma unroll
         for (int kk = 0; kk < Sh::KSTEPS; ++kk) {
           const int sub = kk >> 2, off = (kk & 3) * 32;
@@ -266,6 +297,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
                    id_s, kk > 0);
         }
         mma_commit(smem_u32(&s_full[bb]));
+        mma_commit(smem_u32(&k_empty[s]));  // q k^T has read k block j
         if (j >= 1 && !pv(j - 1)) ok = false;
       }
       if (ok && !pv(nkb - 1)) ok = false;
@@ -291,10 +323,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
     // The ones row (channel DKP) and 15 zero rows after each v^T sub-block's
     // channels; TMA never writes them.  Rows DKP.. start an 8-row swizzle
     // group, and a row of equal chunks is the same under any chunk swizzle.
-    for (int idx = threadIdx.x - 64; idx < NST * 2 * 16 * 8; idx += kSoftThreads) {
+    for (int idx = threadIdx.x - 64; idx < NVS * 2 * 16 * 8; idx += kSoftThreads) {
       const int row = idx >> 3, ch = idx & 7;  // row over (stage, sub-block, 16 rows)
       const int sv = row >> 4, rr = row & 15;
-      uint8_t* base = sKV + (sv >> 1) * Sh::STAGE + Sh::KBYTES + (sv & 1) * Sh::VSUB + (Sh::DKP + rr) * 128;
+      uint8_t* base = sV + (sv >> 1) * Sh::VBYTES + (sv & 1) * Sh::VSUB + (Sh::DKP + rr) * 128;
       const uint32_t one2 = 0x3F803F80u;       // two bf16 1.0
       *reinterpret_cast<uint4*>(base + ch * 16) =
           rr == 0 ? make_uint4(one2, one2, one2, one2) : make_uint4(0, 0, 0, 0);
@@ -443,9 +475,14 @@ __global__ void __launch_bounds__(kTThreads, 1)
   if (warp == 0 && lane == 0 && abort_flag) {
     // Copies issued but never consumed still land in shared memory.
     drain_wait(smem_u32(&q_full), 0);
-    for (int s = 0; s < NST && s < issued; ++s) {
-      const int last = issued - 1 - ((issued - 1 - s) % NST);  // newest block issued on stage s
-      drain_wait(smem_u32(&kv_full[s]), (last / NST) & 1);
+    const int nk_iss = s_issued[0], nv_iss = s_issued[1];
+    for (int s = 0; s < NK && s < nk_iss; ++s) {
+      const int last = nk_iss - 1 - ((nk_iss - 1 - s) % NK);  // newest block issued on stage s
+      drain_wait(smem_u32(&k_full[s]), (last / NK) & 1);
+    }
+    for (int s = 0; s < NVS && s < nv_iss; ++s) {
+      const int last = nv_iss - 1 - ((nv_iss - 1 - s) % NVS);
+      drain_wait(smem_u32(&v_full[s]), (last / NVS) & 1);
     }
   }
   __syncthreads();
