@@ -158,6 +158,13 @@ struct PrepArgs {
   int32_t* row_of;        // or null: [T, k + n_shared] list position of each branch's row
                           // (p < k routed, p = k shared), -1 when not recomputed
   int n_shared;
+  int attn_list;          // 1: also list the tokens with a non-empty recompute set (group G)
+  int32_t* attn_rows;     //   [T] ascending tokens,
+  int* attn_n;            //   their count,
+  int32_t* attn_inv;      //   [T] each token's place (-1 if absent),
+  int32_t* sample_lo;     //   [T / seq + 1] where each sample's tokens start
+  int seq;                //   tokens per sample
+  int region_groups;      // groups the counts region was sized for: prep_region_groups(E, attn)
   unsigned* gbar;         // grid barrier arrival counter (zeroed once, only grows)
   unsigned bar_base;      // arrivals on gbar from earlier launches (mod 2^32)
   unsigned long long* stats;
@@ -171,6 +178,9 @@ struct PrepShape {
 };
 constexpr size_t kPrepSmemMax = 200 * 1024;
 PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn);
+// Groups of the fused kernel's count scan: E routed + a shared one (sized for
+// always), + the recomputing-token list of a DiT-MoE block.
+inline int prep_region_groups(int E, bool attn) { return E + 1 + (attn ? 1 : 0); }
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 
 // Eq. 8 combine + residual + cached branch norms.

@@ -383,7 +383,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms, attn);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
-      A((void**)&h->prep_counts, nb * G * 4);
+      A((void**)&h->prep_counts, nb * (G + 1) * 4);
       A((void**)&h->prep_bar, 2 * sizeof(unsigned));
     }
   }
@@ -558,10 +558,17 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       PrepArgs pa{};
       pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
       pa.n_shared = c.n_shared;
+      pa.region_groups = prep_region_groups(c.n_experts, attn);
       if (attn && !attn_full) {
         pa.x = in;
         pa.attn_a = L.attn_a;
         pa.u_out = L.attn_u;
+      }
+      if (attn_sync) {
+        // The recomputing-token list comes out of the same compaction.
+        pa.attn_list = 1;
+        pa.attn_rows = h->attn_rows; pa.attn_n = h->attn_n; pa.attn_inv = h->attn_inv;
+        pa.sample_lo = h->attn_samp; pa.seq = seq;
       }
       if (attn_sync && xg_gather) {
         // The rows of tokens that keep their attention are final now; the
@@ -593,9 +600,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       // Sec. 4.1: the tokens with a non-empty recompute set recompute their
       // attention output over all keys of their sample; their a and u rows
       // are replaced, then the FFN rows are gathered from u.
-      if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
-             return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp, h->attn_inv, s);
-           })) != cudaSuccess)
+      if (!fused && (e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
+                       return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp,
+                                               h->attn_inv, s);
+                     })) != cudaSuccess)
         break;
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_ATTN, s, [&] {

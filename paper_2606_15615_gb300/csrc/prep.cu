@@ -99,10 +99,12 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __shared__ int sm_live[kMaxExperts];
   __shared__ float sm_lo, sm_hi;
   __shared__ int sm_near;
-  __shared__ unsigned sm_bal[kMaxGroups];
-  __shared__ int sm_pre[kMaxGroups];
-  __shared__ int sm_tot[kMaxGroups];
-  __shared__ int sm_off[kMaxGroups + 1];
+  // Groups: E routed, the shared expert, and (DiT-MoE block) the list of
+  // tokens that recompute their attention.
+  __shared__ unsigned sm_bal[kMaxGroups + 1];
+  __shared__ int sm_pre[kMaxGroups + 1];
+  __shared__ int sm_tot[kMaxGroups + 1];
+  __shared__ int sm_off[kMaxGroups + 2];
   __shared__ int sm_rows[TB * (KMAX + 1)][2];
   __shared__ int sm_nrows;
   __shared__ __align__(8) uint64_t sm_bar;
@@ -126,7 +128,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   // logits / counts region (sized as prep_smem sizes it for this grid).
   const bool add_a = a.attn_a != nullptr;
   __nv_bfloat16* s_a = reinterpret_cast<__nv_bfloat16*>(
-      reinterpret_cast<uint8_t*>(s_logit) + prep_region_bytes(TB, EPAD, gridDim.x, E + 1));
+      reinterpret_cast<uint8_t*>(s_logit) + prep_region_bytes(TB, EPAD, gridDim.x, a.region_groups));
 
   // ---- A0: stage gate rows and token rows ----
   // Before the programmatic-dependency wait: everything that the previous
@@ -430,7 +432,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
 
   // ---- B: branch decisions of the block's tokens (warp 0, one token per lane) ----
-  const int GG = a.G;
+  const int GG = a.G + (a.attn_list ? 1 : 0);  // the attention list is group G, after the FFN groups
   TokenDecisionT<KMAX> d;
   if (warp == 0) {
     SelectArgs sa = a.sel;
@@ -444,8 +446,10 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       if (g < E) {
 #pragma unroll
         for (int p = 0; p < KMAX; ++p) has |= (d.rec[p] && d.e[p] == g);
-      } else {
+      } else if (g < a.G) {
         has = d.shared_row;
+      } else {
+        has = valid && d.any;  // recomputes its attention (Sec. 4.1)
       }
       const unsigned b = __ballot_sync(0xffffffffu, has);
       if (lane == 0) {
@@ -555,8 +559,12 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     }
     __syncthreads();
     if (blockIdx.x == 0) {
-      for (int g = t; g < GG; g += kThreads) a.counts[g] = sm_tot[g];
-      for (int g = t; g <= GG; g += kThreads) a.offsets[g] = sm_off[g];
+      for (int g = t; g < a.G; g += kThreads) a.counts[g] = sm_tot[g];
+      for (int g = t; g <= a.G; g += kThreads) a.offsets[g] = sm_off[g];
+      if (a.attn_list && t == 0) {
+        *a.attn_n = sm_tot[a.G];
+        a.sample_lo[T / a.seq] = sm_tot[a.G];
+      }
     }
     if (warp == 0) {
       const int i = tok0 + lane;
@@ -584,6 +592,14 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         }
       }
       if (row_of && a.n_shared) row_of[k] = -1;
+      if (a.attn_list && lane < ntok) {
+        // Place in the recomputing-token list (its own array, from 0), and
+        // where each sample starting in this block begins in it.
+        const int pos = sm_pre[a.G] + __popc(sm_bal[a.G] & lt);
+        if (d.any) a.attn_rows[pos] = i;
+        a.attn_inv[i] = d.any ? pos : -1;
+        if (i % a.seq == 0) a.sample_lo[i / a.seq] = pos;
+      }
       if (d.shared_row) {
         const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
         a.list[pos] = i;
@@ -610,7 +626,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
 }
 
 template <int TB, int EPAD>
-size_t prep_smem(int D, int n_blocks, int G, bool attn) {
+size_t prep_smem(int D, int n_blocks, int G, bool attn) {  // G: groups of the counts region
   const size_t ldw = static_cast<size_t>(D) + 8;
   const size_t rows = (EPAD + TB) * ldw * 2;                        // gate rows, token rows
   const size_t a_rows = attn ? TB * ldw * 2 : 0;                    // cached attention rows
@@ -694,7 +710,7 @@ PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn) {
     const int nb = (max_tokens + TB - 1) / TB;
     const size_t smem = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> size_t {
       if constexpr (tb == 0) return 0;
-      else return prep_smem<tb, ep>(D, nb, E + 1, attn);
+      else return prep_smem<tb, ep>(D, nb, prep_region_groups(E, attn), attn);
     });
     if (smem == 0 || smem > kPrepSmemMax) continue;
     const int occ = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> int {
