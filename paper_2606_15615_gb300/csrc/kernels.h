@@ -175,9 +175,15 @@ struct PrepShape {
   int epad;               // experts padded to a multiple of 8
   int kmax;               // compile-time bound on top-k (2, 4 or 8)
   size_t smem;            // dynamic shared memory per block
+  bool attn;              // the DiT-MoE block build of the kernel
 };
 constexpr size_t kPrepSmemMax = 200 * 1024;
 PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn);
+// The two builds of prep.cu (plain, and prep_attn.cu for DiT-MoE blocks).
+PrepShape prep_plan_plain(int D, int E, int k, int max_tokens, int n_sms);
+PrepShape prep_plan_attn(int D, int E, int k, int max_tokens, int n_sms);
+cudaError_t launch_prep_plain(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
+cudaError_t launch_prep_attn(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 // Groups of the fused kernel's count scan: E routed + a shared one (sized for
 // always), + the recomputing-token list of a DiT-MoE block.
 inline int prep_region_groups(int E, bool attn) { return E + 1 + (attn ? 1 : 0); }

@@ -93,7 +93,7 @@ struct moeca_handle {
   int* tc_dep = nullptr;        // fused GEMM launch: m-tile dependency counters, left at 0
   int* tc_work = nullptr;       // GEMM unit tickets {next, CTAs done}, left at 0
   int tc_dep_pairs_n = 0;
-  PrepShape prep{0, 0, 0, 0};   // fused router + select + compact, when it fits
+  PrepShape prep{0, 0, 0, 0, false};  // fused router + select + compact, when it fits
   unsigned prep_arrivals = 0;   // grid-barrier arrivals of all fused launches so far (mod 2^32)
   bool inject_stall = false;    // moeca_inject_fault: next step's barrier targets unreachable
   int32_t* prep_counts = nullptr;

@@ -24,8 +24,18 @@
 #include "kernels.h"
 #include "select_token.cuh"
 
+// This file is compiled twice: plain (the MoE layer alone) and, from
+// prep_attn.cu with MOECA_PREP_ATTN 1, for DiT-MoE blocks.  The block's work
+// (u = x + a^{t0}, the FFN-row map, the recomputing-token list) exists only
+// in the second build, so the MoE path's code -- phases run once per launch
+// and on the critical path -- carries none of it.
+#ifndef MOECA_PREP_ATTN
+#define MOECA_PREP_ATTN 0
+#endif
+
 namespace moeca {
 namespace {
+constexpr bool kAttn = MOECA_PREP_ATTN != 0;
 
 constexpr int kThreads = 128;
 constexpr int kMaxGroups = kMaxExperts + 1;
@@ -81,6 +91,57 @@ __host__ __device__ constexpr size_t prep_region_bytes(int TB, int EPAD, int n_b
   return ((logits > counts ? logits : counts) + 15) / 16 * 16;
 }
 
+// DiT-MoE block work kept out of line, so the MoE-only path's code (phases
+// run once per launch, on the critical path) is what it is without it.
+// Bulk copies of the block's cached attention rows a^{t0} (thread 0).
+static __device__ __noinline__ void issue_attn_rows(const PrepArgs& a, __nv_bfloat16* s_a, int ldw, int tok0,
+                                                    int ntok, uint32_t row_bytes, uint32_t bar) {
+  const __nv_bfloat16* ar = static_cast<const __nv_bfloat16*>(a.attn_a);
+  for (int q = 0; q < ntok; ++q)
+    bulk_g2s(smem_u32(s_a + q * ldw), ar + static_cast<size_t>(tok0 + q) * a.D, row_bytes, bar);
+}
+
+// u = x + a^{t0} (rounded to bf16) in place of the staged x rows, and to u_out.
+static __device__ __noinline__ void form_u(const PrepArgs& a, __nv_bfloat16* s_x, const __nv_bfloat16* s_a, int ldw,
+                                           int tok0, int ntok, int t) {
+  __nv_bfloat16* u_out = static_cast<__nv_bfloat16*>(a.u_out);
+  const int nv = a.D / 8;
+  for (int idx = t; idx < ntok * nv; idx += kThreads) {
+    const int q = idx / nv, c = idx % nv;
+    uint4* xs = reinterpret_cast<uint4*>(s_x + q * ldw) + c;
+    float xv[8], av[8];
+    unpack_vec(*xs, xv, static_cast<__nv_bfloat16*>(nullptr));
+    unpack_vec(*(reinterpret_cast<const uint4*>(s_a + q * ldw) + c), av, static_cast<__nv_bfloat16*>(nullptr));
+#pragma unroll
+    for (int j = 0; j < 8; ++j) xv[j] += av[j];
+    uint4 uv;
+    __nv_bfloat162* uh = reinterpret_cast<__nv_bfloat162*>(&uv);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) uh[j] = __floats2bfloat162_rn(xv[2 * j], xv[2 * j + 1]);
+    *xs = uv;
+    reinterpret_cast<uint4*>(u_out + static_cast<size_t>(tok0 + q) * a.D)[c] = uv;
+  }
+}
+
+// One lane's token (warp 0 of phase C): its FFN-row map entries (the list
+// positions of its recomputed branches, -1 elsewhere) and its place in the
+// recomputing-token list.  `pos[p]` are the positions the list loop wrote.
+static __device__ __noinline__ void attn_bookkeeping(const PrepArgs& a, int i, int lane, int ntok, bool any,
+                                                     const int* pos, int shared_pos, int list_pos) {
+  if (lane >= ntok) return;  // 16-token blocks: lanes 16-31 hold the next block's tokens
+  if (a.row_of) {
+    const int W = a.sel.k + a.n_shared;
+    int32_t* row_of = a.row_of + static_cast<size_t>(i) * W;
+    for (int p = 0; p < a.sel.k; ++p) row_of[p] = pos[p];
+    if (a.n_shared) row_of[a.sel.k] = shared_pos;
+  }
+  if (a.attn_list) {
+    if (any) a.attn_rows[list_pos] = i;
+    a.attn_inv[i] = any ? list_pos : -1;
+    if (i % a.seq == 0) a.sample_lo[i / a.seq] = list_pos;
+  }
+}
+
 template <int TB, int EPAD, int KMAX>
 __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   constexpr int G = kThreads / TB;       // lanes per token in the routing epilogue (4 or 8)
@@ -106,6 +167,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __shared__ int sm_tot[kMaxGroups + 1];
   __shared__ int sm_off[kMaxGroups + 2];
   __shared__ int sm_rows[TB * (KMAX + 1)][2];
+  __shared__ bool sm_any[kAttn ? TB : 1];
   __shared__ int sm_nrows;
   __shared__ __align__(8) uint64_t sm_bar;
   // Per-token inputs of the decision, fetched at the start and kept here.
@@ -126,7 +188,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   const int ntok = min(TB, T - tok0);
   // DiT-MoE block on a cache step: the cached attention rows, after the
   // logits / counts region (sized as prep_smem sizes it for this grid).
-  const bool add_a = a.attn_a != nullptr;
+  const bool add_a = kAttn && a.attn_a != nullptr;
   __nv_bfloat16* s_a = reinterpret_cast<__nv_bfloat16*>(
       reinterpret_cast<uint8_t*>(s_logit) + prep_region_bytes(TB, EPAD, gridDim.x, a.region_groups));
 
@@ -149,11 +211,8 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     mbar_expect_tx(bar, row_bytes * (E + ntok + (add_a ? ntok : 0)));
     const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
     for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
-    if (add_a) {
-      // a^{t0} of this layer was written on an earlier step.
-      const __nv_bfloat16* ar = static_cast<const __nv_bfloat16*>(a.attn_a);
-      for (int q = 0; q < ntok; ++q)
-        bulk_g2s(smem_u32(s_a + q * ldw), ar + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
+    if constexpr (kAttn) {
+      if (add_a) issue_attn_rows(a, s_a, ldw, tok0, ntok, row_bytes, bar);  // written on an earlier step
     }
   }
   // Prefetch what later phases read: cached metadata and EMA rows.
@@ -185,27 +244,13 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
   if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);
   __syncthreads();
-  if (add_a) {
-    // u = x + a^{t0} (rounded to bf16): the router input, the rows the FFN
-    // gathers, and the residual; written out for the kernels after this one.
-    __nv_bfloat16* u_out = static_cast<__nv_bfloat16*>(a.u_out);
-    const int nv = D / 8;
-    for (int idx = t; idx < ntok * nv; idx += kThreads) {
-      const int q = idx / nv, c = idx % nv;
-      uint4* xs = reinterpret_cast<uint4*>(s_x + q * ldw) + c;
-      float xv[8], av[8];
-      unpack_vec(*xs, xv, static_cast<__nv_bfloat16*>(nullptr));
-      unpack_vec(*(reinterpret_cast<const uint4*>(s_a + q * ldw) + c), av, static_cast<__nv_bfloat16*>(nullptr));
-#pragma unroll
-      for (int j = 0; j < 8; ++j) xv[j] += av[j];
-      uint4 uv;
-      __nv_bfloat162* uh = reinterpret_cast<__nv_bfloat162*>(&uv);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) uh[j] = __floats2bfloat162_rn(xv[2 * j], xv[2 * j + 1]);
-      *xs = uv;
-      reinterpret_cast<uint4*>(u_out + static_cast<size_t>(tok0 + q) * D)[c] = uv;
+  if constexpr (kAttn) {
+    if (add_a) {
+      // u = x + a^{t0}: the router input, the rows the FFN gathers, and the
+      // residual; written out for the kernels after this one.
+      form_u(a, s_x, s_a, ldw, tok0, ntok, t);
+      __syncthreads();
     }
-    __syncthreads();
   }
 
   // ---- A1: logits on the tensor cores ----
@@ -432,7 +477,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
 
   // ---- B: branch decisions of the block's tokens (warp 0, one token per lane) ----
-  const int GG = a.G + (a.attn_list ? 1 : 0);  // the attention list is group G, after the FFN groups
+  const int GG = a.G + ((kAttn && a.attn_list) ? 1 : 0);  // the attention list is group G, after the FFN groups
   TokenDecisionT<KMAX> d;
   if (warp == 0) {
     SelectArgs sa = a.sel;
@@ -561,7 +606,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     if (blockIdx.x == 0) {
       for (int g = t; g < a.G; g += kThreads) a.counts[g] = sm_tot[g];
       for (int g = t; g <= a.G; g += kThreads) a.offsets[g] = sm_off[g];
-      if (a.attn_list && t == 0) {
+      if (kAttn && a.attn_list && t == 0) {
         *a.attn_n = sm_tot[a.G];
         a.sample_lo[T / a.seq] = sm_tot[a.G];
       }
@@ -569,45 +614,35 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     if (warp == 0) {
       const int i = tok0 + lane;
       const unsigned lt = (1u << lane) - 1u;
-      // Under the sync rule the rows of a token with recomputed branches are
-      // written by the attention output projection (row_of says where).
-      const bool gather_here = !(a.gather_final_only && d.any);
-      const int W = k + a.n_shared;
-      // Only this block's tokens: with 16-token blocks lanes 16-31 hold the
-      // next block's tokens, whose entries that block writes.
-      int32_t* row_of = (a.row_of && lane < ntok) ? a.row_of + static_cast<size_t>(i) * W : nullptr;
+      const bool track = kAttn && a.row_of != nullptr;  // DiT-MoE block, sync rule: record the FFN rows
+      int pos_of[KMAX];
+      int shared_pos = -1;
 #pragma unroll
       for (int p = 0; p < KMAX; ++p) {
-        if (p < k && row_of) row_of[p] = -1;
+        if (track) pos_of[p] = -1;
         if (d.rec[p]) {
           const int g = d.e[p];
           const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
           a.list[pos] = i * k + d.sl[p];
-          if (row_of) row_of[p] = pos;
-          if (gather_here) {
-            const int r = atomicAdd(&sm_nrows, 1);
-            sm_rows[r][0] = pos;
-            sm_rows[r][1] = i;
-          }
+          if (track) pos_of[p] = pos;
+          const int r = atomicAdd(&sm_nrows, 1);
+          sm_rows[r][0] = pos;
+          sm_rows[r][1] = i;
         }
-      }
-      if (row_of && a.n_shared) row_of[k] = -1;
-      if (a.attn_list && lane < ntok) {
-        // Place in the recomputing-token list (its own array, from 0), and
-        // where each sample starting in this block begins in it.
-        const int pos = sm_pre[a.G] + __popc(sm_bal[a.G] & lt);
-        if (d.any) a.attn_rows[pos] = i;
-        a.attn_inv[i] = d.any ? pos : -1;
-        if (i % a.seq == 0) a.sample_lo[i / a.seq] = pos;
       }
       if (d.shared_row) {
         const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
         a.list[pos] = i;
-        if (row_of) row_of[k] = pos;
-        if (gather_here) {
-          const int r = atomicAdd(&sm_nrows, 1);
-          sm_rows[r][0] = pos;
-          sm_rows[r][1] = i;
+        shared_pos = pos;
+        const int r = atomicAdd(&sm_nrows, 1);
+        sm_rows[r][0] = pos;
+        sm_rows[r][1] = i;
+      }
+      if constexpr (kAttn) {
+        if (lane < TB) sm_any[lane] = d.any;
+        if (a.row_of || a.attn_list) {
+          const int list_pos = a.attn_list ? sm_pre[a.G] + __popc(sm_bal[a.G] & lt) : 0;
+          attn_bookkeeping(a, i, lane, ntok, d.any, pos_of, shared_pos, list_pos);
         }
       }
     }
@@ -618,6 +653,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     uint4* xg = static_cast<uint4*>(a.xg);
     const int n = xg ? sm_nrows : 0;
     for (int r = warp; r < n; r += kThreads / 32) {
+      // Under the sync rule the rows of a token with recomputed branches are
+      // written by the attention output projection (the FFN-row map).
+      if constexpr (kAttn) {
+        if (a.gather_final_only && sm_any[sm_rows[r][1] - tok0]) continue;
+      }
       const uint4* src = reinterpret_cast<const uint4*>(s_x + (sm_rows[r][1] - tok0) * ldw);
       uint4* dst = xg + static_cast<size_t>(sm_rows[r][0]) * nv;
       for (int c = lane; c < nv; c += 32) dst[c] = src[c];
@@ -700,7 +740,13 @@ int kmax_of(int k) { return k <= 2 ? 2 : (k <= 4 ? 4 : 8); }
 
 }  // namespace
 
-PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn) {
+#if MOECA_PREP_ATTN
+PrepShape prep_plan_attn(int D, int E, int k, int max_tokens, int n_sms) {
+  const bool attn = true;
+#else
+PrepShape prep_plan_plain(int D, int E, int k, int max_tokens, int n_sms) {
+  const bool attn = false;
+#endif
   PrepShape p{0, 0, 0, 0};
   if (D % 16 || E < 1 || E > kMaxExperts || k < 1 || k > kMaxTopK) return p;
   const int epad = (E + 7) / 8 * 8;
@@ -722,17 +768,32 @@ PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn) {
     p.epad = epad;
     p.kmax = km;
     p.smem = smem;
+    p.attn = attn;
     return p;
   }
   return p;
 }
 
-cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
+#if MOECA_PREP_ATTN
+cudaError_t launch_prep_attn(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
+#else
+cudaError_t launch_prep_plain(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
+#endif
   const int nb = (a.T + p.tokens_per_block - 1) / p.tokens_per_block;
   return with_shape(p.tokens_per_block, p.epad, p.kmax, [&]<int tb, int ep, int kk>() -> cudaError_t {
     if constexpr (tb == 0) return cudaErrorInvalidValue;
     else return prep_launch<tb, ep, kk>(a, nb, p.smem, s);
   });
 }
+
+#if !MOECA_PREP_ATTN
+PrepShape prep_plan(int D, int E, int k, int max_tokens, int n_sms, bool attn) {
+  return attn ? prep_plan_attn(D, E, k, max_tokens, n_sms) : prep_plan_plain(D, E, k, max_tokens, n_sms);
+}
+
+cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
+  return p.attn ? launch_prep_attn(a, p, s) : launch_prep_plain(a, p, s);
+}
+#endif
 
 }  // namespace moeca
