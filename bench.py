@@ -217,9 +217,14 @@ class Runner:
         self.x_dev = self.x_host.to(self.dev)
         T, D = wl.n_tokens, wl.hidden
         self.out = torch.empty((T, D), dtype=dt, device=self.dev)
-        self.in_buf = torch.empty((T, D), dtype=dt, device=self.dev)
-        self.out_host = torch.empty((T, D), dtype=dt).pin_memory()
         self.stream = torch.cuda.current_stream(self.dev)
+        # End to end: two input and two output buffers, so the upload of step
+        # t + 1 and the read-back of step t run on a copy stream while the
+        # neighbouring steps compute (every step still moves its own bytes).
+        self.in_bufs = [torch.empty((T, D), dtype=dt, device=self.dev) for _ in range(2)]
+        self.out_bufs = [torch.empty((T, D), dtype=dt, device=self.dev) for _ in range(2)]
+        self.out_host = [torch.empty((T, D), dtype=dt).pin_memory() for _ in range(2)]
+        self.copy_stream = torch.cuda.Stream(device=self.dev)
 
     def _run(self, tau0, W_, K, kernel_timing=False, e2e=False):
         torch, M = self.torch, self.M
@@ -238,12 +243,10 @@ class Runner:
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(self.stream)
-        for t in range(W_, W_ + K):
-            if e2e:
-                self.in_buf.copy_(self.x_host[t], non_blocking=True)
-                M.moeca_step(h, self.in_buf.data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
-                self.out_host.copy_(self.out, non_blocking=True)
-            else:
+        if e2e:
+            self._e2e_steps(tau0, W_, K)
+        else:
+            for t in range(W_, W_ + K):
                 M.moeca_step(h, self.x_dev[t].data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
         e1.record(self.stream)
         torch.cuda.synchronize(self.dev)
@@ -254,6 +257,42 @@ class Runner:
             kt = M.moeca_get_kernel_times(h, reset=True)
         st = M.moeca_get_stats(h)
         return ms, st, kt
+
+    def _e2e_steps(self, tau0, W_, K):
+        """Steps W_ .. W_ + K - 1 from pinned host inputs to pinned host outputs.
+
+        Step t reads in_bufs[t % 2] and writes out_bufs[t % 2].  The copy
+        stream uploads step t + 1's input once step t - 1 (its buffer's last
+        reader) is done, then reads step t's output back once step t is done;
+        the compute stream starts step t after its upload and, for t >= 2,
+        after step t - 2's read-back (its output buffer's last reader).
+        """
+        torch, M = self.torch, self.M
+        h, T, sp, cs = self.stack.handle, self.wl.n_tokens, self.stream.cuda_stream, self.copy_stream
+        ev = lambda: torch.cuda.Event()  # noqa: E731
+        up, done, back = [ev(), ev()], [ev(), ev()], [ev(), ev()]
+        cs.wait_stream(self.stream)
+        with torch.cuda.stream(cs):
+            self.in_bufs[W_ % 2].copy_(self.x_host[W_], non_blocking=True)
+            up[W_ % 2].record(cs)
+        for t in range(W_, W_ + K):
+            b = t % 2
+            self.stream.wait_event(up[b])
+            if t - 2 >= W_:
+                self.stream.wait_event(back[b])
+            M.moeca_step(h, self.in_bufs[b].data_ptr(), self.out_bufs[b].data_ptr(), T, t, False, tau0, sp)
+            done[b].record(self.stream)
+            with torch.cuda.stream(cs):
+                if t + 1 < W_ + K:
+                    nb = (t + 1) % 2
+                    if t - 1 >= W_:
+                        cs.wait_event(done[nb])
+                    self.in_bufs[nb].copy_(self.x_host[t + 1], non_blocking=True)
+                    up[nb].record(cs)
+                cs.wait_event(done[b])
+                self.out_host[b].copy_(self.out_bufs[b], non_blocking=True)
+                back[b].record(cs)
+        self.stream.wait_stream(cs)  # the last read-back is inside the timed region
 
     def reuse_of(self, st) -> float:
         return st["reused"] / max(st["branches"], 1)
@@ -539,7 +578,9 @@ def main():
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": {"value": wl.n_tokens * K * world / (e2e_ms / 1e3), "unit": "tokens/s",
-                "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes},
+                "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes,
+                "pipelining": "each step's upload and read-back run on a copy stream, overlapping the "
+                              "neighbouring steps' compute (double-buffered input and output)"},
         "gpu_launches": sum(kt[k_][1] for k_ in KINDS),
         "clocks": head["clocks"],
         "sweep": sweep,
