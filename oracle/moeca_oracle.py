@@ -22,6 +22,9 @@ Each function names the passage of the paper it follows:
                   attention is recomputed on the step its recompute set is
                   non-empty (synchronized MoE / attention update)
   Table 4         "without sync. update": attention reused on every cache step
+  Sec. 3, Eq. 2   DiT block: attention then MLP (MoE) sub-layer, each in the
+                  residual form x + AdaLN o f(x)
+  Sec. 3, Eq. 1   reverse transition of the sampler
 
 Readings where the paper is silent (each is a switch in ``Params``):
   * gate weights: softmax over all E experts, top-k, then renormalised over
@@ -54,6 +57,15 @@ Readings where the paper is silent (each is a switch in ``Params``):
   * ``act_store`` "bf16" rounds the block's stored activations (a, u) to
     bfloat16, the storage type of the bf16 kernels, so that decisions taken
     on u' use the same input on both sides; "f64" keeps them exact.
+  * an AdaLN block (``adaln``; Sec. 3 names AdaLN, the form is DiT's): per
+    sample, SiLU(c) W_ada^T + b_ada gives shift, scale and gate for each
+    sub-layer; a sub-layer reads LN(v) (1 + scale) + shift (LN over D, no
+    affine, eps 1e-6) and is added as v + gate f; the caches hold ungated
+    outputs and each step applies its own modulation; under the sync rule
+    the router sees m' = modulate(LN(x + gate_a a^{t0})).
+  * sampler (Eq. 1): linear betas 1e-4 .. 0.02 over 1000 training steps, a
+    run of n steps visits n evenly spaced training steps (rounded half up),
+    variance beta_t, no noise on the last step.
 """
 from __future__ import annotations
 
@@ -87,6 +99,8 @@ class Params:
     seq_len: int = 0                   # token rows per sample (attention scope); 0: all T rows
     attn_policy: str = "sync"          # or "stale" (Table 4 ablation) or "full"
     act_store: str = "f64"             # or "bf16": storage rounding of the block's a and u
+    adaln: bool = False                # DiT block with AdaLN modulation of both sub-layers (Sec. 3)
+    ln_eps: float = 1e-6               # layer-normalisation epsilon of the AdaLN block
 
 
 # ---------------------------------------------------------------------------
@@ -385,7 +399,7 @@ class LayerState:
 
 
 def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, slot, weights: dict,
-                          prm: Params, refresh: bool):
+                          prm: Params, refresh: bool, resid=None, gate=None):
     """Apply a recompute decision and form the layer output (Sec. 4.1, Eq. 5-8).
 
     Recomputes FFN_e(u_i) for the branches in R (rows of one expert together),
@@ -393,6 +407,9 @@ def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, s
     under the synchronized rule, combines every branch p from slot(p) with the
     current weight w^t (Eq. 8), adds the residual and refreshes the cached
     norms.  Returns (out [T, D], new state, token_any [T]).
+
+    ``resid`` and ``gate`` ([T, D], or None) give the AdaLN block's output
+    resid + gate * y (Sec. 3 residual form) instead of u + y.
     """
     u = np.asarray(u, np.float64)
     T, D = u.shape
@@ -430,7 +447,9 @@ def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, s
         y += np.asarray(w_cur, np.float64)[:, p:p + 1] * new.cache_h[np.arange(T), slot[:, p]]
     if new.shared_h is not None:
         y += new.shared_h
-    out = u + y
+    if gate is not None:
+        y = np.asarray(gate, np.float64) * y
+    out = (u if resid is None else np.asarray(resid, np.float64)) + y
     new.cache_norm = np.sqrt(np.sum(new.cache_h ** 2, axis=2))
     new.valid = True
     return out, new, token_any
@@ -523,6 +542,157 @@ def block_step(state: LayerState, x: np.ndarray, weights: dict, prm: Params, ref
     return out, new, info
 
 
+# ---------------------------------------------------------------------------
+# DiT-MoE block with AdaLN modulation (Sec. 3, Eq. 2) and the sampler (Eq. 1)
+# ---------------------------------------------------------------------------
+
+def silu(z: np.ndarray) -> np.ndarray:
+    """SiLU(z) = z / (1 + exp(-z)), the activation before the AdaLN projection."""
+    z = np.asarray(z, np.float64)
+    return z / (1.0 + np.exp(-z))
+
+
+def layer_norm(v: np.ndarray, eps: float) -> np.ndarray:
+    """Normalisation of each row over its D features, without affine
+    parameters: (v - mean) / sqrt(var + eps), var the biased row variance."""
+    v = np.asarray(v, np.float64)
+    mu = v.mean(axis=-1, keepdims=True)
+    var = ((v - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (v - mu) / np.sqrt(var + eps)
+
+
+def adaln_modulation(c: np.ndarray, w_ada: np.ndarray, b_ada=None) -> np.ndarray:
+    """The six AdaLN vectors of one block for every sample (Sec. 3).
+
+    c is [B, D], one conditioning vector per sample (timestep and class
+    embedding); w_ada is [6D, D] and b_ada [6D] or None.  Returns
+    mod [B, 6, D] = reshape(SiLU(c) w_ada^T + b_ada): along axis 1 the
+    attention sub-layer's shift, scale and gate, then the MoE sub-layer's.
+    """
+    c = np.asarray(c, np.float64)
+    B, D = c.shape
+    mod = silu(c) @ np.asarray(w_ada, np.float64).T
+    if b_ada is not None:
+        mod = mod + np.asarray(b_ada, np.float64)[None, :]
+    return mod.reshape(B, 6, D)
+
+
+def modulate(v: np.ndarray, shift: np.ndarray, scale: np.ndarray) -> np.ndarray:
+    """AdaLN's affine map of a normalised row: v (1 + scale) + shift."""
+    return np.asarray(v, np.float64) * (1.0 + np.asarray(scale, np.float64)) + np.asarray(shift, np.float64)
+
+
+def token_rows(vec: np.ndarray, T: int, seq_len: int) -> np.ndarray:
+    """Expand per-sample rows [B, D] to token rows [T, D] (samples of seq_len rows)."""
+    S = int(seq_len) or T
+    vec = np.asarray(vec, np.float64)
+    if vec.shape[0] * S != T:
+        raise ValueError("n_tokens must be n_samples * seq_len")
+    return np.repeat(vec, S, axis=0)
+
+
+def adaln_block_step(state: LayerState, x: np.ndarray, mod: np.ndarray, weights: dict, prm: Params,
+                     refresh: bool):
+    """One DiT-MoE block with AdaLN modulation at one denoising step (Sec. 3
+    residual form, cached under Sec. 4.1).  mod is the block's [B, 6, D]
+    output of ``adaln_modulation``.  Returns (out [T, D], new state, info).
+
+        h = modulate(LN(x), shift_a, scale_a)          attention input
+        a = Attn(h)                                     (cached: a^{t0})
+        u = x + gate_a a
+        m = modulate(LN(u), shift_m, scale_m)          MoE input
+        out = u + gate_m y,  y of Eq. 8 on m
+
+    The caches hold the ungated a and branch outputs; every step applies
+    its own modulation.  Full-computation step, or attn_policy "full": a
+    for every token, routed on m.  Cache step, "sync": the decision is taken
+    on m' = modulate(LN(u'), ...) with u' = x + gate_a a^{t0}; tokens with a
+    non-empty recompute set recompute a_i (all keys of their sample, from
+    the current h), u_i and m_i, and their branches read m_i; the others
+    keep u'_i and m'_i.  "stale": u' and m' for every token, a kept.
+    ``info`` adds h, u (residual), m (FFN input), route_in and attn_rows.
+    """
+    x = np.asarray(x, np.float64)
+    T, D = x.shape
+    S = prm.seq_len or T
+    mod = np.asarray(mod, np.float64)
+    sh_a, sc_a, g_a, sh_m, sc_m, g_m = (token_rows(mod[:, j], T, S) for j in range(6))
+    store = round_bf16 if prm.act_store == "bf16" else (lambda v: np.asarray(v, np.float64))
+    eps = prm.ln_eps
+    h = store(modulate(layer_norm(x, eps), sh_a, sc_a))
+
+    def attn(rows=None):
+        return attention(h, weights["w_qkv"], weights.get("b_qkv"), weights["w_o"], weights.get("b_o"),
+                         prm.n_heads, prm.seq_len, rows)
+
+    def moe_input(u, rows):
+        return store(modulate(layer_norm(u, eps), sh_m[rows], sc_m[rows]))
+
+    every = np.arange(T)
+    if refresh or prm.attn_policy == "full":
+        a = store(attn())
+        u = store(x + g_a * a)
+        m = moe_input(u, every)
+        route_in, rows = m, every
+    else:
+        u = store(x + g_a * state.attn_a)
+        m = moe_input(u, every)
+        route_in = m
+        a = state.attn_a.copy()
+        rows = np.zeros(0, np.int64)
+    info = decide(state, route_in, weights, prm, refresh)
+    if not (refresh or prm.attn_policy == "full"):
+        if prm.attn_policy == "sync":
+            rows = np.nonzero(info["token_any"])[0]
+            if len(rows):
+                m = m.copy()
+                u = u.copy()
+                a[rows] = store(attn(rows))
+                u[rows] = store(x[rows] + g_a[rows] * a[rows])
+                m[rows] = moe_input(u[rows], rows)
+        elif prm.attn_policy != "stale":
+            raise ValueError(prm.attn_policy)
+    out, new, token_any = recompute_and_combine(state, m, info["e"], info["w"], info["recompute"],
+                                                info["slot"], weights, prm, refresh, resid=u, gate=g_m)
+    new.C = info["C"]
+    new.attn_a = a
+    info.update(h=h, u=u, m=m, route_in=route_in, attn_rows=rows, token_any=token_any)
+    return out, new, info
+
+
+def ddpm_schedule(n_steps: int, n_train: int = 1000, beta_start: float = 1e-4, beta_end: float = 0.02):
+    """Per-step coefficients of Eq. 1 for a sampling run of ``n_steps`` steps.
+
+    The training schedule is beta_s linear from beta_start to beta_end over
+    n_train steps, abar_s = prod_{r <= s} (1 - beta_r).  A run of n steps
+    visits the training steps t_j = floor(j (n_train - 1) / (n_steps - 1) + 1/2),
+    j = 0 .. n - 1, and takes abar'_j = abar_{t_j},
+    alpha'_j = abar'_j / abar'_{j-1} (abar'_{-1} = 1), beta'_j = 1 - alpha'_j.
+    Returns (t, alpha, alpha_bar, beta), each [n_steps], in j order (a run
+    goes from j = n - 1 down to 0).
+    """
+    if n_steps < 2 or n_steps > n_train:
+        raise ValueError("2 <= n_steps <= n_train")
+    betas = np.linspace(beta_start, beta_end, n_train, dtype=np.float64)
+    abar = np.cumprod(1.0 - betas)
+    t = np.floor(np.arange(n_steps) * (n_train - 1) / (n_steps - 1) + 0.5).astype(np.int64)
+    ab = abar[t]
+    prev = np.concatenate([[1.0], ab[:-1]])
+    alpha = ab / prev
+    return t, alpha, ab, 1.0 - alpha
+
+
+def ddpm_step(x_t, eps, z, alpha_t: float, alpha_bar_t: float, sigma_t: float) -> np.ndarray:
+    """One reverse transition of Eq. 1: the mean
+    (x_t - (1 - alpha_t) / sqrt(1 - abar_t) eps) / sqrt(alpha_t), plus sigma_t z.
+    Eq. 1's variance is beta_t I, so sigma_t = sqrt(beta_t); the last step
+    of a run (j = 0) takes sigma = 0 and returns the mean.  z is the
+    standard normal draw, an input."""
+    x_t = np.asarray(x_t, np.float64)
+    mean = (x_t - (1.0 - alpha_t) / math.sqrt(1.0 - alpha_bar_t) * np.asarray(eps, np.float64)) / math.sqrt(alpha_t)
+    return mean + sigma_t * np.asarray(z, np.float64)
+
+
 def stats_of(info: dict) -> dict:
     """Branch counts of one layer step (Fig. 8's reuse-over-match ratio inputs)."""
     rec, matched = info["recompute"], info["matched"]
@@ -553,7 +723,9 @@ class Stack:
                     or not all(s.valid for s in self.states)
                     or (N > 0 and step_index % N == 0))
 
-    def step(self, x: np.ndarray, step_index: int, force: bool = False):
+    def step(self, x: np.ndarray, step_index: int, force: bool = False, cond=None):
+        """One denoising step of the stack; ``cond`` [B, D] is the per-sample
+        conditioning of AdaLN blocks (``prm.adaln``)."""
         x = np.asarray(x, np.float64)
         T = x.shape[0]
         refresh = self.is_refresh(step_index, T, force)
@@ -564,6 +736,11 @@ class Stack:
         infos = []
         step_fn = block_step if self.prm.n_heads > 0 else layer_step
         for l, w in enumerate(self.layers):
-            x, self.states[l], info = step_fn(self.states[l], x, w, self.prm, refresh)
+            if self.prm.adaln:
+                mod = adaln_modulation(cond, w["w_ada"], w.get("b_ada"))
+                x, self.states[l], info = adaln_block_step(self.states[l], x, mod, w, self.prm, refresh)
+                info["mod"] = mod
+            else:
+                x, self.states[l], info = step_fn(self.states[l], x, w, self.prm, refresh)
             infos.append(info)
         return x, infos

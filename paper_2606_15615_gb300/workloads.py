@@ -231,6 +231,34 @@ def tiny_attn(seed: int, D: int, dtype: str = "f32", bias: bool = True, wscale: 
     }
 
 
+def tiny_adaln(seed: int, D: int, dtype: str = "f32", wscale: float = 0.2, bias: bool = True) -> dict:
+    """Small random AdaLN projection of one block: w_ada [6D, D] in the given
+    dtype, b_ada [6D] float32 (or None)."""
+    rng = _rng(7700 + seed)
+    st = round_to_bf16 if dtype == "bf16" else (lambda a: np.asarray(a, np.float32))
+    return {
+        "w_ada": st(wscale * rng.standard_normal((6 * D, D), dtype=np.float32)),
+        "b_ada": (0.1 * rng.standard_normal(6 * D)).astype(np.float32) if bias else None,
+    }
+
+
+def conditioning(seed: int, n_samples: int, D: int, n_steps: int) -> np.ndarray:
+    """Per-step, per-sample conditioning vectors c [n_steps, n_samples, D]
+    (float32) standing in for timestep + class embeddings: a fixed class part
+    ~ N(0, 1) per sample plus a timestep part that varies smoothly with the
+    step, sinusoids of the step index at D / 2 geometric frequencies."""
+    rng = _rng(7900 + seed)
+    cls = rng.standard_normal((n_samples, D)).astype(np.float64)
+    half = D // 2
+    freq = np.exp(-math.log(1000.0) * np.arange(half) / max(half, 1))
+    out = np.empty((n_steps, n_samples, D), np.float32)
+    for t in range(n_steps):
+        ang = (n_steps - t) * 4.0 * freq
+        emb = np.concatenate([np.cos(ang), np.sin(ang), np.zeros(D - 2 * half)])
+        out[t] = (cls + emb[None, :]).astype(np.float32)
+    return out
+
+
 # ---------------------------------------------------------------------------
 # Trajectories of the first layer's input
 # ---------------------------------------------------------------------------
