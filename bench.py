@@ -35,7 +35,8 @@ if ROOT not in sys.path:
 METRIC = "branch-cached MoE layer tokens/s and effective TFLOP/s vs reuse ratio; % roofline"
 DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn", "qkv", "attn", "oproj", "attn_aux"]
+KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn", "qkv", "attn", "oproj", "attn_aux",
+         "adaln"]
 
 
 # ---------------------------------------------------------------------------
@@ -159,7 +160,7 @@ def kernel_source_sha(kind: str) -> str:
     headers it includes (so a recorded ncu figure expires with the code)."""
     fname = {"ffn1": "ffn_tc.cu", "ffn2": "ffn_tc.cu", "ffn": "ffn_tc.cu", "router": "router.cu", "select": "select.cu",
              "compact": "select.cu", "combine": "combine.cu", "prep": "prep.cu", "qkv": "proj_tc.cu",
-             "oproj": "proj_tc.cu", "attn": "attention.cu", "attn_aux": "attention.cu"}[kind]
+             "oproj": "proj_tc.cu", "attn": "attention.cu", "attn_aux": "attention.cu", "adaln": "adaln.cu"}[kind]
     csrc = os.path.join(ROOT, "paper_2606_15615_gb300", "csrc")
     h = hashlib.sha256()
     with open(os.path.join(csrc, fname), "rb") as f:
@@ -207,7 +208,8 @@ class Runner:
             n_layers=wl.n_layers, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts, top_k=wl.top_k,
             n_shared=wl.n_shared, max_tokens=wl.n_tokens,
             dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period,
-            ffn_tile_n=tile_n, ffn_split_k=split_k, n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
+            ffn_tile_n=tile_n, ffn_split_k=split_k, n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0,
+            adaln=int(wl.adaln))
         self.cfg = cfg
         self.stack = M.Stack(cfg, self.weights, device=device_index)
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -225,6 +227,35 @@ class Runner:
         self.out_bufs = [torch.empty((T, D), dtype=dt, device=self.dev) for _ in range(2)]
         self.out_host = [torch.empty((T, D), dtype=dt).pin_memory() for _ in range(2)]
         self.copy_stream = torch.cuda.Stream(device=self.dev)
+        # AdaLN workloads: a conditioning vector per sample and step, and the
+        # Eq. 1 update of each step's output (x_t kept in float32; the noise
+        # draw z is one fixed buffer, an input of the update).
+        self.cond_host = self.cond_dev = None
+        if wl.adaln:
+            c = torch.from_numpy(W.workload_conditioning(wl, n_steps))
+            self.cond_host = c.pin_memory()
+            self.cond_dev = c.to(self.dev)
+            self.cond_bufs = [torch.empty_like(self.cond_dev[0]) for _ in range(2)]
+            g = torch.Generator(device=self.dev)
+            g.manual_seed(3000 + wl.index)
+            self.x_state = torch.empty((T, D), dtype=torch.float32, device=self.dev).normal_(generator=g)
+            self.z = torch.empty((T, D), dtype=torch.float32, device=self.dev).normal_(generator=g)
+            _, self.alpha, self.abar, self.beta = M.moeca_ddpm_schedule(max(wl.n_steps, n_steps, 2))
+
+    def _sampler_update(self, t, eps):
+        """Eq. 1: x_{t-1} from x_t and this step's output; run step t visits schedule step n - 1 - t."""
+        j = len(self.alpha) - 1 - (t % len(self.alpha))
+        sigma = math.sqrt(self.beta[j]) if j > 0 else 0.0
+        self.M.ddpm_step(self.x_state, eps, self.alpha[j], self.abar[j], sigma, z=self.z if sigma else None,
+                         x_prev=self.x_state, stream=self.stream.cuda_stream)
+
+    def _step(self, h, x_ptr, out, t, tau0, sp, cond=None):
+        cp = None
+        if self.wl.adaln:
+            cp = (self.cond_dev[t] if cond is None else cond).data_ptr()
+        self.M.moeca_step(h, x_ptr, out.data_ptr(), self.wl.n_tokens, t, False, tau0, sp, cp)
+        if self.wl.adaln:
+            self._sampler_update(t, out)
 
     def _run(self, tau0, W_, K, kernel_timing=False, e2e=False):
         torch, M = self.torch, self.M
@@ -234,7 +265,7 @@ class Runner:
         sp = self.stream.cuda_stream
         T = self.wl.n_tokens
         for t in range(W_):
-            M.moeca_step(h, self.x_dev[t].data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
+            self._step(h, self.x_dev[t].data_ptr(), self.out, t, tau0, sp)
         torch.cuda.synchronize(self.dev)
         M.moeca_reset_stats(h)
         if kernel_timing:
@@ -247,7 +278,7 @@ class Runner:
             self._e2e_steps(tau0, W_, K)
         else:
             for t in range(W_, W_ + K):
-                M.moeca_step(h, self.x_dev[t].data_ptr(), self.out.data_ptr(), T, t, False, tau0, sp)
+                self._step(h, self.x_dev[t].data_ptr(), self.out, t, tau0, sp)
         e1.record(self.stream)
         torch.cuda.synchronize(self.dev)
         ms = e0.elapsed_time(e1)
@@ -272,15 +303,19 @@ class Runner:
         ev = lambda: torch.cuda.Event()  # noqa: E731
         up, done, back = [ev(), ev()], [ev(), ev()], [ev(), ev()]
         cs.wait_stream(self.stream)
+        ada = self.wl.adaln
         with torch.cuda.stream(cs):
             self.in_bufs[W_ % 2].copy_(self.x_host[W_], non_blocking=True)
+            if ada:
+                self.cond_bufs[W_ % 2].copy_(self.cond_host[W_], non_blocking=True)
             up[W_ % 2].record(cs)
         for t in range(W_, W_ + K):
             b = t % 2
             self.stream.wait_event(up[b])
             if t - 2 >= W_:
                 self.stream.wait_event(back[b])
-            M.moeca_step(h, self.in_bufs[b].data_ptr(), self.out_bufs[b].data_ptr(), T, t, False, tau0, sp)
+            self._step(h, self.in_bufs[b].data_ptr(), self.out_bufs[b], t, tau0, sp,
+                       cond=self.cond_bufs[b] if ada else None)
             done[b].record(self.stream)
             with torch.cuda.stream(cs):
                 if t + 1 < W_ + K:
@@ -288,6 +323,8 @@ class Runner:
                     if t - 1 >= W_:
                         cs.wait_event(done[nb])
                     self.in_bufs[nb].copy_(self.x_host[t + 1], non_blocking=True)
+                    if ada:
+                        self.cond_bufs[nb].copy_(self.cond_host[t + 1], non_blocking=True)
                     up[nb].record(cs)
                 cs.wait_event(done[b])
                 self.out_host[b].copy_(self.out_bufs[b], non_blocking=True)
@@ -335,6 +372,15 @@ def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float, att
         return 4 * attn_rows * D * es + D * D * es + D * 4, 2.0 * attn_rows * D * D
     if kind == "attn_aux":  # u = x + a^{t0} (x, a in, u out), the token list, the FFN row gather
         return 3 * T * D * es + T + rows_per_launch * 2 * D * es, 0.0
+    if kind == "adaln":
+        # Mean over a cache step's 1 + 2L launches: the modulation GEMV (every
+        # layer's W_ada once), then per layer the row pass (x, a^{t0} in; u',
+        # m', h out) and the recomputing rows' m = LN-modulate(u).
+        L, B = wl.n_layers, wl.batch
+        mod = L * 6 * D * D * es + L * 6 * D * 4 + B * D * 4 + L * B * 6 * D * 4
+        pre = 5 * T * D * es + B * 6 * D * 4
+        mrows = attn_rows * (2 * D * es + 4)
+        return (mod + L * (pre + mrows)) / (1 + 2 * L), 2.0 * L * B * 6 * D * D / (1 + 2 * L)
     if kind == "router":
         return T * D * es + E * D * es + T * E * 8 + T * k * 8, 2.0 * T * D * E
     if kind == "select":
@@ -368,18 +414,20 @@ def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
     if w["ws1"] is None:
         w["ws1"] = w["ws2"] = None
     prm = O.Params(top_k=wl.top_k, tau0=tau0 if math.isfinite(tau0) else tau0, refresh_period=wl.refresh_period,
-                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
+                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0, adaln=wl.adaln,
+                   act_store="bf16" if wl.adaln else "f64")
     st = O.Stack([w], prm, wl.hidden, wl.n_experts, wl.n_shared)
     xs = runner.x_host.float().numpy()
-    st.step(xs[0], 0)
+    conds = runner.cond_host.numpy().astype(np.float64) if wl.adaln else [None] * xs.shape[0]
+    st.step(xs[0], 0, cond=conds[0])
     times = []
     t_all = time.perf_counter()
     for t in range(1, xs.shape[0]):
         if wl.refresh_period and t % wl.refresh_period == 0:
-            st.step(xs[t], t)
+            st.step(xs[t], t, cond=conds[t])
             continue
         t0 = time.perf_counter()
-        st.step(xs[t], t)
+        st.step(xs[t], t, cond=conds[t])
         times.append(time.perf_counter() - t0)
         if time.perf_counter() - t_all > budget_s:
             break
@@ -409,18 +457,22 @@ def reference_arm(args, wl):
     if wl.n_heads:
         for l in range(rng_layers):
             ws[l].update(W.make_attn_weights(wl, l))
+            if wl.adaln:
+                ws[l].update(W.make_adaln_weights(wl, l))
     xs = list(W.trajectory(wl, args.warmup + args.steps + 1))
+    conds = W.workload_conditioning(wl, len(xs)) if wl.adaln else [None] * len(xs)
     prm = O.Params(top_k=wl.top_k, tau0=args.ref_tau0, refresh_period=wl.refresh_period,
-                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0)
+                   n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0, adaln=wl.adaln,
+                   act_store="bf16" if wl.adaln else "f64")
     stacks = [O.Stack([ws[l]], prm, wl.hidden, wl.n_experts, wl.n_shared) for l in range(rng_layers)]
     for t in range(args.warmup):
-        stacks[t % rng_layers].step(xs[t], t)
+        stacks[t % rng_layers].step(xs[t], t, cond=conds[t])
     times = []
     for j in range(args.steps):
         t = args.warmup + j
         s = stacks[t % rng_layers]
         t0 = time.perf_counter()
-        s.step(xs[t], t)
+        s.step(xs[t], t, cond=conds[t])
         times.append(time.perf_counter() - t0)
     per_layer = statistics.mean(times)
     value = wl.n_tokens / (per_layer * wl.n_layers)
@@ -559,6 +611,7 @@ def main():
         cpu = cpu_oracle_baseline(wl, runner, head["tau0_raw"])
     es = 2 if wl.dtype == "bf16" else 4
     io_bytes = wl.n_tokens * wl.hidden * es
+    cond_bytes = wl.batch * wl.hidden * 4 if wl.adaln else 0
     line = {
         "metric": METRIC, "value": head["tokens_per_s"], "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": W_, "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak",
@@ -569,6 +622,12 @@ def main():
                    **({"attn_heads": wl.n_heads, "seq_len": wl.seq,
                        "attn_rows_recomputed_per_step": head["stats"]["attn_recomputed"] / K}
                       if wl.n_heads else {}),
+                   **({"adaln": True,
+                       "step": "AdaLN modulation of every block from the step's conditioning, the L blocks, "
+                               "then the Eq. 1 update of the step's output (x_t in float32); the blocks' "
+                               "inputs follow the synthetic drift trajectory, not the update, so the reuse "
+                               "ratio is controlled as for the other workloads"}
+                      if wl.adaln else {}),
                    "reuse_achieved": head["reuse_achieved"], "tau0": head["tau0"],
                    "effective_tflops": head["effective_tflops"], "executed_tflops": head["executed_tflops"],
                    "timed": f"median of {args.reps} reps of {K} steps after {W_} warm-up steps (step 0 full)",
@@ -578,10 +637,10 @@ def main():
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": {"value": wl.n_tokens * K * world / (e2e_ms / 1e3), "unit": "tokens/s",
-                "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes,
+                "h2d_bytes_per_step": io_bytes + cond_bytes, "d2h_bytes_per_step": io_bytes,
                 "pipelining": "each step's upload and read-back run on a copy stream, overlapping the "
                               "neighbouring steps' compute (double-buffered input and output)"},
-        "gpu_launches": sum(kt[k_][1] for k_ in KINDS),
+        "gpu_launches": sum(kt[k_][1] for k_ in KINDS) + (K if wl.adaln else 0),
         "clocks": head["clocks"],
         "sweep": sweep,
         "kernels": kernels,

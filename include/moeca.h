@@ -109,6 +109,21 @@ typedef struct {
                                  TMEM kernel from 512 tokens per sample, warp-level mma.sync kernel
                                  below, where a CTA sees too few key blocks to fill its pipeline);
                                  1 = mma.sync kernel; 2 = tcgen05 kernel */
+  int32_t adaln;              /* 1: each DiT-MoE block (n_heads > 0) enters both sub-layers through
+                                 AdaLN, the residual form x + AdaLN o f(x) of Sec. 3 in DiT's shape:
+                                 per sample b, SiLU(c_b) w_ada^T + b_ada gives six D-vectors
+                                 (shift_a, scale_a, gate_a, shift_m, scale_m, gate_m);
+                                 h = LN(x)(1 + scale_a) + shift_a, a = Attn(h),
+                                 u = x + gate_a a, m = LN(u)(1 + scale_m) + shift_m,
+                                 out = u + gate_m MoE(m); LN over D without affine parameters.
+                                 The caches hold the ungated a and branch outputs, every step
+                                 applies its own modulation, and under the sync rule the router
+                                 sees m' from u' = x + gate_a a^{t0}.  moeca_step_args.cond then
+                                 carries c.  0 (default): no normalisation or modulation */
+  float ln_eps;               /* AdaLN layer-normalisation epsilon (default 1e-6) */
+  int32_t keep_route_in;      /* 1: keep each AdaLN block's router input (m' on sync cache steps)
+                                 for moeca_get_layer_trace, one more [T, D] write per layer;
+                                 0 (default) */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters
@@ -125,6 +140,9 @@ void moeca_config_default(moeca_config* cfg);
  *   w_qkv [3D, D]: rows [0, D) queries, [D, 2D) keys, [2D, 3D) values, head h
  *   at rows h*dh .. h*dh + dh - 1 of each; b_qkv [3D] fp32 or NULL;
  *   w_o [D, D] output projection; b_o [D] fp32 or NULL.
+ * AdaLN projection (adaln = 1; NULL otherwise): w_ada [6D, D] bf16, the six
+ *   D-row blocks in the order shift_a, scale_a, gate_a, shift_m, scale_m,
+ *   gate_m; b_ada [6D] fp32 or NULL.
  * Base pointers must be 16-byte aligned. */
 typedef struct {
   const void* w_gate;
@@ -137,6 +155,8 @@ typedef struct {
   const float* b_qkv;
   const void* w_o;
   const float* b_o;
+  const void* w_ada;
+  const float* b_ada;
 } moeca_layer_weights;
 
 /* Per-step arguments. */
@@ -145,6 +165,9 @@ typedef struct {
   int32_t step_index;    /* denoising step counter used by the refresh schedule             */
   int32_t force_refresh; /* 1: make this a full-computation step (Sec. 4.1)                 */
   float tau0_override;   /* NaN: use config tau0; otherwise the Eq. 12 base threshold now   */
+  const float* cond;     /* adaln = 1: [n_tokens / seq_len, D] fp32 device, each sample's
+                            conditioning c (timestep + class embedding), read during the step;
+                            NULL otherwise */
 } moeca_step_args;
 
 /* Branch counters, cumulative since create / moeca_reset_stats (Fig. 8 inputs). */
@@ -197,7 +220,14 @@ typedef struct {
  *   layer_in [T, D] dtype                        the MoE sub-layer's input: the layer input, or
  *                                                for a DiT-MoE block u = x + a after the
  *                                                attention update (the FFN rows and the residual)
- *   block_in [T, D] dtype                        the DiT-MoE block's input x (n_heads > 0) */
+ *   block_in [T, D] dtype                        the DiT-MoE block's input x (n_heads > 0)
+ *   route_in [T, D] dtype                        an AdaLN block's router input: m on full
+ *                                                steps, m' on sync cache steps (keep_route_in
+ *                                                = 1; skipped otherwise)
+ *   resid [T, D] dtype                           the residual stream u the MoE output is added
+ *                                                to (n_heads > 0); for an AdaLN block layer_in
+ *                                                is m, the FFN rows' input
+ *   mod [T / seq_len, 6D] fp32                   an AdaLN block's modulation this step */
 typedef struct {
   int32_t* route_e;
   float* route_w;
@@ -211,6 +241,9 @@ typedef struct {
   int32_t* list;
   void* layer_in;
   void* block_in;
+  void* route_in;
+  void* resid;
+  float* mod;
 } moeca_layer_trace;
 
 /* Kernel kinds timed by moeca_set_kernel_timing(). */
@@ -227,7 +260,8 @@ enum {
   MOECA_K_ATTN = 9,    /* attention: softmax(q k^T / sqrt(dh)) v of the recomputed rows */
   MOECA_K_OPROJ = 10,  /* attention: output projection GEMM + x + a          */
   MOECA_K_ATTN_AUX = 11, /* attention: u = x + a^{t0}, recomputed-token list, FFN row gather */
-  MOECA_K_COUNT = 12
+  MOECA_K_ADALN = 12,  /* AdaLN: modulation vectors, layer norm + modulation of the rows */
+  MOECA_K_COUNT = 13
 };
 
 typedef struct {
@@ -355,6 +389,41 @@ typedef struct {
 } moeca_route_args;
 
 moeca_status moeca_route_noalloc(const moeca_route_args* args, void* stream);
+
+/* ---- Sampler (Eq. 1) ------------------------------------------------------
+ * The reverse transition of Eq. 1 with the denoiser's output eps:
+ *   x_{t-1} = (x_t - (1 - alpha_t) / sqrt(1 - abar_t) eps) / sqrt(alpha_t) + sigma_t z.
+ *
+ * moeca_ddpm_schedule fills host arrays [n_steps] for a sampling run of
+ * n_steps steps over a linear training schedule of n_train betas from
+ * beta_start to beta_end (abar_s = prod_{r <= s} (1 - beta_r)): run step j
+ * visits training step t_j = floor(j (n_train - 1) / (n_steps - 1) + 1/2) and
+ * takes abar'_j = abar_{t_j}, alpha'_j = abar'_j / abar'_{j-1} (abar'_{-1} = 1),
+ * beta'_j = 1 - alpha'_j.  A run goes from j = n_steps - 1 down to 0; Eq. 1's
+ * variance gives sigma_j = sqrt(beta'_j), and the last step (j = 0) adds no
+ * noise.  Any output pointer may be NULL.  INVALID_ARG unless
+ * 2 <= n_steps <= n_train and 0 < beta_start <= beta_end < 1. */
+moeca_status moeca_ddpm_schedule(int32_t n_steps, int32_t n_train, double beta_start, double beta_end,
+                                 int32_t* t, double* alpha, double* alpha_bar, double* beta);
+
+/* moeca_ddpm_step runs the update on device buffers, asynchronously on
+ * `stream` (the current device).  x_prev may alias x_t; x_next (optional)
+ * receives x_prev in eps_dtype, the next denoiser input.  n must be a
+ * multiple of 8 and every pointer 16-byte aligned (INVALID_ARG otherwise);
+ * z may be NULL only when sigma == 0.  The noise z is the caller's draw. */
+typedef struct {
+  int64_t n;             /* elements                                   */
+  int32_t eps_dtype;     /* moeca_dtype of eps and x_next              */
+  double alpha;          /* alpha'_j                                   */
+  double alpha_bar;      /* abar'_j (< 1)                              */
+  double sigma;          /* sigma_j >= 0                               */
+  const float* x_t;      /* [n] fp32                                   */
+  const void* eps;       /* [n] eps_dtype                              */
+  const float* z;        /* [n] fp32 standard normal draw, or NULL     */
+  float* x_prev;         /* [n] fp32                                   */
+  void* x_next;          /* [n] eps_dtype, or NULL                     */
+} moeca_ddpm_args;
+moeca_status moeca_ddpm_step(const moeca_ddpm_args* args, void* stream);
 
 const char* moeca_status_string(moeca_status s);
 /* Message of the last error on this handle ("" if none); NULL handle: the

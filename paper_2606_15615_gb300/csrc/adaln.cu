@@ -1,0 +1,277 @@
+// AdaLN modulation of a DiT-MoE block (Sec. 3: each sub-layer f enters the
+// residual stream as x + AdaLN o f(x)) and the reverse-diffusion update of the
+// sampler (Eq. 1).
+//
+// ada_mod_kernel      the six modulation vectors of every block for every
+//                     sample, SiLU(c) W_ada^T + b_ada, all layers in one launch
+//                     at the start of a step (HBM-bound: it streams W_ada once)
+// adaln_rows_kernel   per token row: layer normalisation over D and the
+//                     modulation, the gated attention residual u = x + g a,
+//                     and the MoE input m; one warp per row, the row in
+//                     registers
+// ddpm_kernel         x_{t-1} = (x_t - c1 eps) / sqrt(alpha_t) + sigma_t z
+#include "common.cuh"
+#include "kernels.h"
+
+namespace moeca {
+namespace {
+
+constexpr int kModWarps = 8;
+constexpr int kModB = 8;  // samples accumulated per pass over a weight row
+
+__global__ void __launch_bounds__(kModWarps * 32) ada_mod_kernel(AdaModArgs a) {
+  extern __shared__ __align__(16) float s_c[];  // [B, D] SiLU(c)
+  const int D = a.D, B = a.B;
+  // The previous step's last kernels still read `out` (the gates), and the
+  // caller may have written cond with a kernel: wait first.
+  pdl_entry();
+  for (int i = threadIdx.x; i < B * D; i += blockDim.x) {
+    const float z = a.cond[i];
+    s_c[i] = z / (1.f + expf(-z));
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int per_layer = 6 * D;
+  const long long n_rows = static_cast<long long>(a.L) * per_layer;
+  const int nvec = D / 8;
+  for (long long r = static_cast<long long>(blockIdx.x) * kModWarps + warp; r < n_rows;
+       r += static_cast<long long>(gridDim.x) * kModWarps) {
+    const int l = static_cast<int>(r / per_layer);
+    const int j = static_cast<int>(r - static_cast<long long>(l) * per_layer);
+    const uint4* wrow = reinterpret_cast<const uint4*>(a.w[l]) + static_cast<size_t>(j) * nvec;
+    const float* bl = a.b[l];
+    const float bias = bl ? bl[j] : 0.f;
+    float* out = a.out + static_cast<size_t>(l) * B * per_layer + j;
+    for (int b0 = 0; b0 < B; b0 += kModB) {
+      float acc[kModB];
+#pragma unroll
+      for (int q = 0; q < kModB; ++q) acc[q] = 0.f;
+#pragma unroll 4
+      for (int c = lane; c < nvec; c += 32) {
+        float wf[8];
+        unpack_vec(__ldg(wrow + c), wf, static_cast<__nv_bfloat16*>(nullptr));
+#pragma unroll
+        for (int q = 0; q < kModB; ++q) {
+          if (b0 + q < B) {
+            const float4* cp = reinterpret_cast<const float4*>(s_c + static_cast<size_t>(b0 + q) * D + 8 * c);
+            const float4 c0 = cp[0], c1 = cp[1];
+            float s = acc[q];
+            s = fmaf(wf[0], c0.x, s); s = fmaf(wf[1], c0.y, s); s = fmaf(wf[2], c0.z, s); s = fmaf(wf[3], c0.w, s);
+            s = fmaf(wf[4], c1.x, s); s = fmaf(wf[5], c1.y, s); s = fmaf(wf[6], c1.z, s); s = fmaf(wf[7], c1.w, s);
+            acc[q] = s;
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kModB; ++q) {
+        const float v = warp_sum(acc[q]);
+        if (lane == 0 && b0 + q < B) out[static_cast<size_t>(b0 + q) * per_layer] = v + bias;
+      }
+    }
+  }
+}
+
+constexpr int kLnWarps = 8;
+constexpr int kLnChunks = kAdaLnMaxD / 256;  // 16-byte chunks per lane
+
+__device__ __forceinline__ void load8f(const float* p, float* v) {
+  const float4 a = __ldg(reinterpret_cast<const float4*>(p));
+  const float4 b = __ldg(reinterpret_cast<const float4*>(p) + 1);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+__device__ __forceinline__ uint4 pack8(const float* f) {
+  uint4 v;
+  __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) h[q] = __floats2bfloat162_rn(f[2 * q], f[2 * q + 1]);
+  return v;
+}
+
+// Mean and 1 / sqrt(var + eps) of the row held as bf16 chunks (chunk c = lane + 32 q),
+// two passes over the registers.
+__device__ __forceinline__ void row_stats(const uint4* v, int nvec, int lane, int D, float eps, float& mean,
+                                          float& rstd) {
+  float s = 0.f;
+#pragma unroll
+  for (int q = 0; q < kLnChunks; ++q) {
+    if (lane + 32 * q < nvec) {
+      float f[8];
+      unpack_vec(v[q], f, static_cast<__nv_bfloat16*>(nullptr));
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s += f[j];
+    }
+  }
+  mean = warp_sum(s) / static_cast<float>(D);
+  float ss = 0.f;
+#pragma unroll
+  for (int q = 0; q < kLnChunks; ++q) {
+    if (lane + 32 * q < nvec) {
+      float f[8];
+      unpack_vec(v[q], f, static_cast<__nv_bfloat16*>(nullptr));
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float d = f[j] - mean;
+        ss = fmaf(d, d, ss);
+      }
+    }
+  }
+  rstd = rsqrtf(warp_sum(ss) / static_cast<float>(D) + eps);
+}
+
+// dst = bf16((v - mean) rstd (1 + scale) + shift), chunk by chunk.
+__device__ __forceinline__ void store_modulated(const uint4* v, int nvec, int lane, float mean, float rstd,
+                                                const float* shift, const float* scale, __nv_bfloat16* dst,
+                                                __nv_bfloat16* dst2) {
+#pragma unroll
+  for (int q = 0; q < kLnChunks; ++q) {
+    const int c = lane + 32 * q;
+    if (c < nvec) {
+      float f[8], sh[8], sc[8];
+      unpack_vec(v[q], f, static_cast<__nv_bfloat16*>(nullptr));
+      load8f(shift + 8 * c, sh);
+      load8f(scale + 8 * c, sc);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) f[j] = fmaf((f[j] - mean) * rstd, 1.f + sc[j], sh[j]);
+      const uint4 o = pack8(f);
+      reinterpret_cast<uint4*>(dst)[c] = o;
+      if (dst2) reinterpret_cast<uint4*>(dst2)[c] = o;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kLnWarps * 32) adaln_rows_kernel(AdaLnArgs a) {
+  pdl_entry();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * kLnWarps + warp;
+  const int n = a.rows ? *a.n_rows : a.T;
+  if (i >= n || i >= a.T) return;
+  const int t = a.rows ? a.rows[i] : i;
+  if (t < 0 || t >= a.T) {
+    if (lane == 0) report_status(a.status, kStatusBadIndex, 7000000 + i);
+    return;
+  }
+  const int D = a.D, nvec = D / 8;
+  const size_t off = static_cast<size_t>(t) * D;
+  const float* md = a.mod + static_cast<size_t>(t / a.seq) * 6 * D;
+  const uint4* x4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) + off);
+  __nv_bfloat16* u = static_cast<__nv_bfloat16*>(a.u) + off;
+  uint4 v[kLnChunks];
+  if (a.h_out || a.a) {
+#pragma unroll
+    for (int q = 0; q < kLnChunks; ++q)
+      if (lane + 32 * q < nvec) v[q] = x4[lane + 32 * q];
+  }
+  float mean, rstd;
+  if (a.h_out) {
+    row_stats(v, nvec, lane, D, a.eps, mean, rstd);
+    store_modulated(v, nvec, lane, mean, rstd, md, md + D, static_cast<__nv_bfloat16*>(a.h_out) + off, nullptr);
+  }
+  if (a.a) {
+    // u = bf16(x + gate_a a): one rounding of the fused product-sum.
+    const uint4* a4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.a) + off);
+    uint4 av[kLnChunks];
+#pragma unroll
+    for (int q = 0; q < kLnChunks; ++q)
+      if (lane + 32 * q < nvec) av[q] = a4[lane + 32 * q];
+#pragma unroll
+    for (int q = 0; q < kLnChunks; ++q) {
+      const int c = lane + 32 * q;
+      if (c < nvec) {
+        float xf[8], af[8], g[8];
+        unpack_vec(v[q], xf, static_cast<__nv_bfloat16*>(nullptr));
+        unpack_vec(av[q], af, static_cast<__nv_bfloat16*>(nullptr));
+        load8f(md + 2 * D + 8 * c, g);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) xf[j] = fmaf(g[j], af[j], xf[j]);
+        v[q] = pack8(xf);
+        reinterpret_cast<uint4*>(u)[c] = v[q];
+      }
+    }
+  } else if (a.m_out) {
+#pragma unroll
+    for (int q = 0; q < kLnChunks; ++q)
+      if (lane + 32 * q < nvec) v[q] = reinterpret_cast<const uint4*>(u)[lane + 32 * q];
+  }
+  if (a.m_out) {
+    row_stats(v, nvec, lane, D, a.eps, mean, rstd);
+    store_modulated(v, nvec, lane, mean, rstd, md + 3 * D, md + 4 * D,
+                    static_cast<__nv_bfloat16*>(a.m_out) + off,
+                    a.m_copy ? static_cast<__nv_bfloat16*>(a.m_copy) + off : nullptr);
+  }
+}
+
+constexpr int kDdpmThreads = 256;
+
+template <bool BF>
+__global__ void __launch_bounds__(kDdpmThreads) ddpm_kernel(DdpmArgs a) {
+  pdl_entry();
+  const long long nv = a.n / 8;
+  for (long long c = static_cast<long long>(blockIdx.x) * kDdpmThreads + threadIdx.x; c < nv;
+       c += static_cast<long long>(gridDim.x) * kDdpmThreads) {
+    float x[8], e[8], z[8];
+    load8f(a.x_t + 8 * c, x);
+    if constexpr (BF) {
+      unpack_vec(__ldg(reinterpret_cast<const uint4*>(a.eps) + c), e, static_cast<__nv_bfloat16*>(nullptr));
+    } else {
+      load8f(static_cast<const float*>(a.eps) + 8 * c, e);
+    }
+    if (a.z) {
+      load8f(a.z + 8 * c, z);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) z[j] = 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) x[j] = fmaf(a.sigma, z[j], fmaf(-a.c1, e[j], x[j]) * a.inv_sqrt_alpha);
+    float4* xp = reinterpret_cast<float4*>(a.x_prev + 8 * c);
+    xp[0] = make_float4(x[0], x[1], x[2], x[3]);
+    xp[1] = make_float4(x[4], x[5], x[6], x[7]);
+    if (a.x_next) {
+      if constexpr (BF) {
+        reinterpret_cast<uint4*>(a.x_next)[c] = pack8(x);
+      } else {
+        float4* xn = reinterpret_cast<float4*>(a.x_next) + 2 * c;
+        xn[0] = make_float4(x[0], x[1], x[2], x[3]);
+        xn[1] = make_float4(x[4], x[5], x[6], x[7]);
+      }
+    }
+  }
+}
+
+}  // namespace
+
+size_t ada_mod_smem(int B, int D) { return static_cast<size_t>(B) * D * sizeof(float); }
+
+cudaError_t launch_ada_mod(const AdaModArgs& a, int n_sms, cudaStream_t s) {
+  const size_t smem = ada_mod_smem(a.B, a.D);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(ada_mod_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  // Up to four blocks per SM, fewer when the staged conditioning is large.
+  int per_sm = static_cast<int>((200 * 1024) / (smem + 1024));
+  per_sm = per_sm < 1 ? 1 : (per_sm > 4 ? 4 : per_sm);
+  const long long rows = static_cast<long long>(a.L) * 6 * a.D;
+  long long grid = static_cast<long long>(n_sms) * per_sm;
+  const long long need = (rows + kModWarps - 1) / kModWarps;
+  if (grid > need) grid = need;
+  return launch_pdl(ada_mod_kernel, dim3(static_cast<unsigned>(grid)), dim3(kModWarps * 32), smem, s, a);
+}
+
+cudaError_t launch_adaln_rows(const AdaLnArgs& a, cudaStream_t s) {
+  if (a.T <= 0) return cudaSuccess;
+  const int grid = (a.T + kLnWarps - 1) / kLnWarps;
+  return launch_pdl(adaln_rows_kernel, dim3(grid), dim3(kLnWarps * 32), 0, s, a);
+}
+
+cudaError_t launch_ddpm(const DdpmArgs& a, cudaStream_t s) {
+  if (a.n <= 0) return cudaSuccess;
+  long long blocks = (a.n / 8 + kDdpmThreads - 1) / kDdpmThreads;
+  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (a.bf16) return launch_pdl(ddpm_kernel<true>, dim3(static_cast<unsigned>(blocks)), dim3(kDdpmThreads), 0, s, a);
+  return launch_pdl(ddpm_kernel<false>, dim3(static_cast<unsigned>(blocks)), dim3(kDdpmThreads), 0, s, a);
+}
+
+}  // namespace moeca

@@ -4,6 +4,7 @@
 // One warp per token, 16-byte vectors over D:
 //   y_i = sum_{p=1..k} w_{i,p}^t cache_h[i, slot(p)]  (+ shared_h[i])
 //   out_i = x_i + y_i            (fp32 accumulation in p order, rounded once)
+//   out_i = x_i + g_i * y_i      in an AdaLN block (g the sample's MoE gate, Sec. 3)
 //   cache_norm[i, q] = ||cache_h[i, q]||_2 for every slot q (slot is a
 //   permutation of 0..k-1, so the k rows read are all of the token's slots).
 #include "common.cuh"
@@ -16,7 +17,7 @@ constexpr int kWarps = 8;
 
 // CG 16-byte chunks per lane are in flight at once (all k cache rows, the
 // shared row and x loaded before any arithmetic).
-template <typename TI, int KMAX, int CG>
+template <typename TI, int KMAX, int CG, bool GATED>
 __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -35,6 +36,7 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   TI* out = static_cast<TI*>(a.out) + static_cast<size_t>(i) * D;
   const TI* ch = static_cast<const TI*>(a.cache_h) + static_cast<size_t>(i) * k * D;
   const TI* sh = a.shared_h ? static_cast<const TI*>(a.shared_h) + static_cast<size_t>(i) * D : nullptr;
+  const float* gr = GATED ? a.gate + static_cast<size_t>(i / a.seq) * a.gate_ld : nullptr;
   float w[KMAX];
   int q[KMAX];
   bool bad = false;
@@ -110,8 +112,16 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
         }
         float xs[V];
         unpack_vec(xr[g], xs, static_cast<TI*>(nullptr));
+        if constexpr (GATED) {
+          float gv[V];
 #pragma unroll
-        for (int j = 0; j < V; ++j) xs[j] += y[j];
+          for (int j = 0; j < V; j += 4) load_vec(gr + c * V + j, gv + j);
+#pragma unroll
+          for (int j = 0; j < V; ++j) xs[j] = fmaf(gv[j], y[j], xs[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < V; ++j) xs[j] += y[j];
+        }
         store_vec(out + c * V, xs);
       }
     }
@@ -125,19 +135,21 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   }
 }
 
-template <typename TI>
+template <typename TI, bool GATED>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
-  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, 4>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else launch_pdl(combine_kernel<TI, 8, 1>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, 4, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else launch_pdl(combine_kernel<TI, 8, 1, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
 }
 
 }  // namespace
 
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s) {
-  if (bf16) launch_t<__nv_bfloat16>(a, s);
-  else launch_t<float>(a, s);
+  if (a.gate && !bf16) return cudaErrorInvalidValue;  // AdaLN blocks are bf16 only
+  if (bf16 && a.gate) launch_t<__nv_bfloat16, true>(a, s);
+  else if (bf16) launch_t<__nv_bfloat16, false>(a, s);
+  else launch_t<float, false>(a, s);
   return cudaGetLastError();
 }
 

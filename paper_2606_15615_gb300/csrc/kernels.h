@@ -201,6 +201,8 @@ struct CombineArgs {
   float* cache_norm;      // [T, k]
   int* rearm;             // a counter the previous kernel leaves for re-arming (the GEMM's unit
                           // ticket), set to 0 after the dependency wait, or null
+  const float* gate;      // AdaLN block (bf16): out = x + gate * y, gate row of token i at
+  int gate_ld, seq;       //   gate + (i / seq) * gate_ld; null: out = x + y
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);
@@ -208,7 +210,7 @@ cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);
 // ---- Attention path of a DiT-MoE block (Sec. 4.1), bf16 only ----
 
 // Tensor-core projection GEMM: C = A B^T + bias (proj_tc.cu).
-enum ProjMode { kProjStore = 0, kProjResidual = 1, kProjQKV = 2 };
+enum ProjMode { kProjStore = 0, kProjResidual = 1, kProjQKV = 2, kProjResidualGated = 3 };
 struct ProjArgs {
   const void* A;          // [a_rows, K] bf16, row-major
   int a_rows;             // rows A holds (>= M)
@@ -233,12 +235,67 @@ struct ProjArgs {
   void* q_out;            // kProjQKV: [list rows, D] q of the listed tokens, in list order
   void* k_out;            // kProjQKV: [n_tok, D] k
   void* vt_out;           // kProjQKV: [D, n_tok] v transposed
+  const float* gate;      // kProjResidualGated: u = x + gate * a, the gate row of token t at
+  int gate_ld, seq;       //   gate + (t / seq) * gate_ld (AdaLN block)
   int* status;
 };
 // Tile width a launch uses for N: `want` (64 / 128 / 256) if it divides N,
 // else (want = 0) the widest that does; 0 when none fits.
 int proj_tile_n(int N, int want);
 cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s);
+
+// ---- AdaLN modulation of a DiT-MoE block (Sec. 3) and the sampler step (Eq. 1) ----
+
+// mod[l][b][j] = sum_d SiLU(cond[b][d]) w[l][j][d] + b[l][j] for every layer l,
+// sample b < B and row j < 6D, in one launch (adaln.cu).
+struct AdaModArgs {
+  int L, B, D;
+  const float* cond;                    // [B, D] fp32
+  const void* const* w;                 // device array [L] of [6D, D] bf16 matrices
+  const float* const* b;                // device array [L] of [6D] fp32 vectors (entries may be null)
+  float* out;                           // [L, B, 6D]
+};
+// Bytes of shared memory the launch needs (B * D fp32), and whether it fits.
+size_t ada_mod_smem(int B, int D);
+cudaError_t launch_ada_mod(const AdaModArgs& a, int n_sms, cudaStream_t s);
+
+// Row-wise layer normalisation and modulation of one AdaLN block, one warp per
+// row t (rows[i], or i < T):
+//   h = bf16(LN(x) (1 + scale_a) + shift_a)              when h_out is set
+//   u = bf16(x + gate_a a), written to u                 when a is set (else u is read)
+//   m = bf16(LN(u) (1 + scale_m) + shift_m)              when m_out is set (and m_copy)
+// with the six D-vectors of the row's sample at mod + (t / seq) * 6D in the
+// order shift_a, scale_a, gate_a, shift_m, scale_m, gate_m.  bf16 only.
+struct AdaLnArgs {
+  int T, D, seq;
+  float eps;
+  const float* mod;       // [T / seq, 6D]
+  const void* x;          // [T, D]
+  const void* a;          // [T, D] or null
+  void* h_out;            // [T, D] or null
+  void* u;                // [T, D]
+  void* m_out;            // [T, D] or null
+  void* m_copy;           // [T, D] or null
+  const int32_t* rows;    // or null (every row)
+  const int* n_rows;      // device count of rows (with rows)
+  int* status;
+};
+constexpr int kAdaLnMaxD = 2560;
+cudaError_t launch_adaln_rows(const AdaLnArgs& a, cudaStream_t s);
+
+// x_prev = (x_t - c1 eps) inv_sqrt_alpha + sigma z (Eq. 1), n elements, and
+// optionally x_next = x_prev in the denoiser's dtype.
+struct DdpmArgs {
+  long long n;
+  int bf16;               // eps and x_next are bf16 (else fp32)
+  float c1, inv_sqrt_alpha, sigma;
+  const float* x_t;
+  const void* eps;
+  const float* z;         // or null (sigma == 0)
+  float* x_prev;
+  void* x_next;           // or null
+};
+cudaError_t launch_ddpm(const DdpmArgs& a, cudaStream_t s);
 
 // u = x + a, row by row (the MoE input of a token that keeps its cached attention).
 cudaError_t launch_attn_residual(const void* x, const void* a, void* u, int T, int D, int* status,

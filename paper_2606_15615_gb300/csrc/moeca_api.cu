@@ -13,8 +13,18 @@
 //               projection -> attention of the listed rows -> output
 //               projection updating their a and u -> FFN row gather from u
 //               -> FFN -> combine with the residual u.
+// An AdaLN block (adaln = 1, Sec. 3) first computes every layer's modulation
+// vectors from the step's conditioning (one launch), then per layer:
+//   full step:  h = LN-modulate(x) -> q/k/v from h -> attention -> output
+//               projection writing a and u = x + g_a a -> m = LN-modulate(u)
+//               -> the MoE sub-layer on m -> out = u + g_m y;
+//   cache step: u' = x + g_a a^{t0}, m' = LN-modulate(u') (and h) in one pass
+//               -> decisions on m' -> (sync rule) the listed tokens' attention
+//               from h, their a, u and m -> FFN row gather from m -> FFN ->
+//               combine out = u + g_m y.
 // It decides full-computation vs cache steps (Sec. 4.1), owns every state and
 // workspace buffer, and reports errors as status codes.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -61,7 +71,9 @@ struct LayerBuf {
   int32_t* list = nullptr;
   unsigned long long* stats = nullptr;
   void* attn_a = nullptr;    // [T, D] cached attention output a^{t0} (DiT-MoE block)
-  void* attn_u = nullptr;    // [T, D] MoE sub-layer input u of the last step
+  void* attn_u = nullptr;    // [T, D] MoE sub-layer input u of the last step (AdaLN: the residual u)
+  void* attn_m = nullptr;    // [T, D] AdaLN block: the MoE input m of the last step
+  void* route_m = nullptr;   // [T, D] AdaLN block: its router input (keep_route_in)
   TcPlan* tc = nullptr;
   bool valid = false;
 };
@@ -105,6 +117,11 @@ struct moeca_handle {
   int* attn_n = nullptr;        // their count
   int32_t* attn_samp = nullptr; // [T + 1] where each sample's tokens start in attn_rows
   int32_t* attn_rowof = nullptr; // [T, k + n_shared] FFN row of each branch (fused sync path)
+  float* mod = nullptr;         // AdaLN: [L, B, 6D] modulation vectors of the current step
+  int mod_b = 0;                // samples the last step's modulation holds
+  void* ada_h = nullptr;        // AdaLN: [T, D] attention input h = LN-modulate(x)
+  void** ada_w = nullptr;       // AdaLN: device array [L] of w_ada pointers
+  float** ada_b = nullptr;      // AdaLN: device array [L] of b_ada pointers
   std::vector<void*> act;  // input of layer l (l >= 1)
   int* status_host = nullptr;
   int* status_dev = nullptr;
@@ -183,7 +200,8 @@ template <typename Fn>
 cudaError_t timed(moeca_handle* h, int kind, cudaStream_t s, Fn&& fn) {
   // An NVTX range per launch (a no-op unless a profiler is attached).
   static const char* const kNames[MOECA_K_COUNT] = {"router", "select", "compact", "ffn1", "ffn2", "combine",
-                                                   "prep", "ffn", "qkv", "attn", "oproj", "attn_aux"};
+                                                   "prep", "ffn", "qkv", "attn", "oproj", "attn_aux",
+                                                   "adaln"};
   NvtxRange range(kNames[kind]);
   if (!h->timing) return fn();
   PendingTiming pt{kind, take_event(h), take_event(h)};
@@ -238,6 +256,9 @@ void moeca_config_default(moeca_config* c) {
   c->seq_len = 0;
   c->attn_policy = 0;
   c->attn_impl = 0;
+  c->adaln = 0;
+  c->ln_eps = 1e-6f;
+  c->keep_route_in = 0;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -294,6 +315,14 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (attn && (!attn_supported(c.hidden, c.n_heads) || c.hidden % 64))
     return fail(nullptr, MOECA_ERR_UNSUPPORTED,
                 "attention needs hidden a multiple of 64 and hidden / n_heads in {64, 72, 80, 96, 128}");
+  const bool ada = c.adaln != 0;
+  if (c.adaln != 0 && c.adaln != 1) return fail(nullptr, MOECA_ERR_INVALID_ARG, "adaln must be 0 or 1");
+  if (ada && !attn) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "AdaLN modulates a DiT-MoE block: n_heads > 0");
+  if (ada && c.hidden > kAdaLnMaxD) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "AdaLN blocks support hidden <= 2560");
+  if (ada && !(c.ln_eps > 0.f && std::isfinite(c.ln_eps))) return fail(nullptr, MOECA_ERR_INVALID_ARG, "ln_eps must be > 0");
+  const int mod_b_max = ada ? std::max(1, c.seq_len ? c.max_tokens / c.seq_len : 1) : 0;
+  if (ada && ada_mod_smem(mod_b_max, c.hidden) > 200 * 1024)
+    return fail(nullptr, MOECA_ERR_UNSUPPORTED, "AdaLN: samples x hidden x 4 bytes must fit 200 KB of shared memory");
   const int vec = bf16 ? 8 : 4;
   if (c.hidden % vec) return fail(nullptr, MOECA_ERR_UNSUPPORTED, "hidden must be a multiple of 8 (bf16) / 4 (fp32)");
   const bool use_tc = bf16 && c.ffn_impl == MOECA_FFN_AUTO;
@@ -308,8 +337,10 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     if (!w.w_gate || !w.w1 || !w.w2) return fail(nullptr, MOECA_ERR_INVALID_ARG, "layer weight pointer is NULL");
     if (c.n_shared && (!w.ws1 || !w.ws2)) return fail(nullptr, MOECA_ERR_INVALID_ARG, "shared expert weights are NULL");
     if (attn && (!w.w_qkv || !w.w_o)) return fail(nullptr, MOECA_ERR_INVALID_ARG, "attention weights are NULL");
+    if (ada && !w.w_ada) return fail(nullptr, MOECA_ERR_INVALID_ARG, "AdaLN weights are NULL");
     const void* ps[] = {w.w_gate, w.w1, w.w2, w.ws1, w.ws2, attn ? w.w_qkv : nullptr, attn ? w.b_qkv : nullptr,
-                        attn ? w.w_o : nullptr, attn ? w.b_o : nullptr};
+                        attn ? w.w_o : nullptr, attn ? w.b_o : nullptr, ada ? w.w_ada : nullptr,
+                        ada ? w.b_ada : nullptr};
     for (const void* p : ps)
       if (reinterpret_cast<uintptr_t>(p) % 16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "weights must be 16-byte aligned");
   }
@@ -356,6 +387,26 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
       A(&L.attn_a, T * D * es);
       A(&L.attn_u, T * D * es);
     }
+    if (ada) {
+      A(&L.attn_m, T * D * es);
+      if (c.keep_route_in) A(&L.route_m, T * D * es);
+    }
+  }
+  if (ada) {
+    A(&h->ada_h, T * D * es);
+    A((void**)&h->mod, static_cast<size_t>(c.n_layers) * mod_b_max * 6 * D * 4);
+    A((void**)&h->ada_w, c.n_layers * sizeof(void*));
+    A((void**)&h->ada_b, c.n_layers * sizeof(float*));
+    if (ok) {
+      std::vector<const void*> wp(c.n_layers);
+      std::vector<const float*> bp(c.n_layers);
+      for (int l = 0; l < c.n_layers; ++l) {
+        wp[l] = layers[l].w_ada;
+        bp[l] = layers[l].b_ada;
+      }
+      ok = cudaMemcpy(h->ada_w, wp.data(), c.n_layers * sizeof(void*), cudaMemcpyHostToDevice) == cudaSuccess &&
+           cudaMemcpy(h->ada_b, bp.data(), c.n_layers * sizeof(float*), cudaMemcpyHostToDevice) == cudaSuccess;
+    }
   }
   if (attn) {
     A(&h->qkv, T * 3 * D * es);
@@ -380,7 +431,9 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     h->tc_dep_pairs_n = static_cast<int>(tc_dep_pairs(h->max_rows, h->G));
     A((void**)&h->tc_dep, static_cast<size_t>(h->tc_dep_pairs_n) * 2 * sizeof(int));
     A((void**)&h->tc_work, 2 * sizeof(int));
-    h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms, attn);
+    // An AdaLN block forms its router input in its own kernel: the plain
+    // preparation kernel, with the attention list built separately.
+    h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms, attn && !ada);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
       A((void**)&h->prep_counts, nb * (G + 1) * 4);
@@ -467,8 +520,23 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   // The tcgen05 attention core pays off once a CTA streams at least four
   // 128-key blocks; shorter samples go to the warp-level core.
   const bool use_attn_tc = c.attn_impl == 2 || (c.attn_impl == 0 && seq >= 512);
+  const bool ada = c.adaln != 0;
+  const int n_samp = T / seq;
+  const size_t mod_ld = static_cast<size_t>(6) * c.hidden;
+  if (ada && !args->cond) return fail(h, MOECA_ERR_INVALID_ARG, "an AdaLN stack needs cond");
   cudaError_t e = cudaSuccess;
   NvtxRange step_range("moeca_step");
+  if (ada) {
+    // Every layer's six modulation vectors per sample, from this step's c.
+    AdaModArgs ma{};
+    ma.L = c.n_layers; ma.B = n_samp; ma.D = c.hidden; ma.cond = args->cond;
+    ma.w = h->ada_w; ma.b = h->ada_b; ma.out = h->mod;
+    if ((e = timed(h, MOECA_K_ADALN, s, [&] { return launch_ada_mod(ma, h->n_sms, s); })) != cudaSuccess) {
+      for (auto& L : h->layers) L.valid = false;
+      return cuda_fail(h, e, "kernel launch");
+    }
+    h->mod_b = n_samp;
+  }
   for (int l = 0; l < c.n_layers; ++l) {
     LayerBuf& L = h->layers[l];
     NvtxRange layer_range("layer");
@@ -476,14 +544,20 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     void* out = l + 1 == c.n_layers ? x_out : h->act[l + 1];
     const bool attn_full = attn && (refresh || c.attn_policy == 2);
     const bool attn_sync = attn && !attn_full && c.attn_policy == 0;
-    // The MoE sub-layer's input: the layer input, or u of a DiT-MoE block.
-    const void* moe_in = attn ? L.attn_u : in;
+    // The MoE sub-layer's input: the layer input, u of a DiT-MoE block, or
+    // m = LN-modulate(u) of an AdaLN block; its residual: the input or u.
+    const void* moe_in = ada ? L.attn_m : (attn ? L.attn_u : in);
+    const void* resid = attn ? L.attn_u : in;
+    const float* mod_l = ada ? h->mod + static_cast<size_t>(l) * n_samp * mod_ld : nullptr;
+    AdaLnArgs la{};
+    la.T = T; la.D = c.hidden; la.seq = seq; la.eps = c.ln_eps; la.mod = mod_l;
+    la.x = in; la.u = L.attn_u; la.status = h->status_dev;
     const size_t TD = static_cast<size_t>(T) * c.hidden;
     void* q_buf = h->qkv;
     void* k_buf = static_cast<char*>(h->qkv) + TD * h->es;
     void* vt_buf = static_cast<char*>(h->qkv) + 2 * TD * h->es;
     ProjArgs qa{};
-    qa.A = in; qa.a_rows = T; qa.B = L.w.w_qkv; qa.bias = L.w.b_qkv;
+    qa.A = ada ? h->ada_h : in; qa.a_rows = T; qa.B = L.w.w_qkv; qa.bias = L.w.b_qkv;
     qa.M = T; qa.N = 3 * c.hidden; qa.K = c.hidden; qa.mode = kProjQKV;
     qa.q_out = q_buf; qa.k_out = k_buf; qa.vt_out = vt_buf; qa.n_tok = T; qa.status = h->status_dev;
     AttnArgs aa{};
@@ -499,6 +573,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     // operands four times over: the widest tile.
     oa.tile_n = c.hidden > 2048 ? 0 : 64;
     oa.n_tok = T; oa.x = in; oa.a_out = L.attn_a; oa.u_out = L.attn_u;
+    if (ada) {
+      oa.mode = kProjResidualGated;
+      oa.gate = mod_l + 2 * c.hidden; oa.gate_ld = static_cast<int>(mod_ld); oa.seq = seq;
+    }
     oa.row_stat = L.stats + kStAttnRows; oa.status = h->status_dev;
     if (attn_sync) {
       aa.rows = h->attn_rows; aa.sample_lo = h->attn_samp;
@@ -507,11 +585,28 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     }
     if (attn_full) {
       // Every token's attention output, before the router sees u = x + a.
+      if (ada) {
+        AdaLnArgs ha = la;
+        ha.h_out = h->ada_h;
+        if ((e = timed(h, MOECA_K_ADALN, s, [&] { return launch_adaln_rows(ha, s); })) != cudaSuccess) break;
+      }
       if ((e = timed(h, MOECA_K_QKV, s, [&] { return launch_proj_tc(qa, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_ATTN, s, [&] {
              return use_attn_tc ? launch_attn_tc(aa, s) : launch_attn_core(aa, s);
            })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
+      if (ada) {
+        AdaLnArgs mm = la;
+        mm.m_out = L.attn_m; mm.m_copy = L.route_m;
+        if ((e = timed(h, MOECA_K_ADALN, s, [&] { return launch_adaln_rows(mm, s); })) != cudaSuccess) break;
+      }
+    } else if (ada) {
+      // u' = x + g_a a^{t0} and the router input m' for every token, and (sync
+      // rule) the attention input h, in one pass over the rows.
+      AdaLnArgs pa0 = la;
+      pa0.a = L.attn_a; pa0.m_out = L.attn_m; pa0.m_copy = L.route_m;
+      pa0.h_out = attn_sync ? h->ada_h : nullptr;
+      if ((e = timed(h, MOECA_K_ADALN, s, [&] { return launch_adaln_rows(pa0, s); })) != cudaSuccess) break;
     } else if (attn && h->prep.tokens_per_block == 0) {
       // u' = x + a^{t0}: the router input, and the MoE input of every token
       // that keeps its cached attention (the fused preparation kernel forms
@@ -558,19 +653,19 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       PrepArgs pa{};
       pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
       pa.n_shared = c.n_shared;
-      pa.region_groups = prep_region_groups(c.n_experts, attn);
-      if (attn && !attn_full) {
+      pa.region_groups = prep_region_groups(c.n_experts, attn && !ada);
+      if (attn && !ada && !attn_full) {
         pa.x = in;
         pa.attn_a = L.attn_a;
         pa.u_out = L.attn_u;
       }
-      if (attn_sync) {
+      if (attn_sync && !ada) {
         // The recomputing-token list comes out of the same compaction.
         pa.attn_list = 1;
         pa.attn_rows = h->attn_rows; pa.attn_n = h->attn_n; pa.attn_inv = h->attn_inv;
         pa.sample_lo = h->attn_samp; pa.seq = seq;
       }
-      if (attn_sync && xg_gather) {
+      if (attn_sync && !ada && xg_gather) {
         // The rows of tokens that keep their attention are final now; the
         // output projection writes the others (row_of says where).
         pa.xg = h->xg;
@@ -600,7 +695,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       // Sec. 4.1: the tokens with a non-empty recompute set recompute their
       // attention output over all keys of their sample; their a and u rows
       // are replaced, then the FFN rows are gathered from u.
-      if (!fused && (e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
+      if ((!fused || ada) && (e = timed(h, MOECA_K_ATTN_AUX, s, [&] {
                        return launch_attn_rows(L.token_any, T, seq, h->attn_rows, h->attn_n, h->attn_samp,
                                                h->attn_inv, s);
                      })) != cudaSuccess)
@@ -610,7 +705,13 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
              return use_attn_tc ? launch_attn_tc(aa, s) : launch_attn_core(aa, s);
            })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_OPROJ, s, [&] { return launch_proj_tc(oa, s); })) != cudaSuccess) break;
-      if (xg_gather && !fused) {
+      if (ada) {
+        // The listed tokens' MoE input m from their new u.
+        AdaLnArgs mm = la;
+        mm.m_out = L.attn_m; mm.rows = h->attn_rows; mm.n_rows = h->attn_n;
+        if ((e = timed(h, MOECA_K_ADALN, s, [&] { return launch_adaln_rows(mm, s); })) != cudaSuccess) break;
+      }
+      if (xg_gather && (!fused || ada)) {
         CompactArgs ga = ca;
         ga.xg = h->xg;
         if ((e = timed(h, MOECA_K_ATTN_AUX, s, [&] { return launch_gather(ga, h->bf16, s); })) != cudaSuccess)
@@ -643,7 +744,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
 
     CombineArgs cb{};
     cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
-    cb.x = moe_in; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+    cb.x = resid; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+    if (ada) {
+      cb.gate = mod_l + 5 * c.hidden; cb.gate_ld = static_cast<int>(mod_ld); cb.seq = seq;
+    }
     cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
     cb.rearm = use_tc ? h->tc_work : nullptr;
     if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
@@ -765,7 +869,8 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
   cudaSetDevice(h->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const void* in = layer == 0 ? h->last_x_in : h->act[layer];
-  const void* moe_in = h->cfg.n_heads ? L.attn_u : in;
+  const void* moe_in = h->cfg.adaln ? L.attn_m : (h->cfg.n_heads ? L.attn_u : in);
+  const size_t mod_n = static_cast<size_t>(h->mod_b) * 6 * D;
   struct { void* d; const void* s; size_t n; } cp[] = {
       {dst->route_e, L.route_e, T * k * 4}, {dst->route_w, L.route_w, T * k * 4},
       {dst->tau, L.tau, E * 4},             {dst->recompute, L.recompute, T * k},
@@ -774,7 +879,10 @@ moeca_status moeca_get_layer_trace(moeca_handle* h, int32_t layer, const moeca_l
       {dst->offsets, L.offsets, (G + 1) * 4},
       {dst->list, L.list, T * (k + h->cfg.n_shared) * 4},
       {dst->layer_in, moe_in, T * D * h->es},
-      {dst->block_in, h->cfg.n_heads ? in : nullptr, T * D * h->es}};
+      {dst->block_in, h->cfg.n_heads ? in : nullptr, T * D * h->es},
+      {dst->route_in, L.route_m, T * D * h->es},
+      {dst->resid, h->cfg.n_heads ? L.attn_u : in, T * D * h->es},
+      {dst->mod, h->mod ? h->mod + static_cast<size_t>(layer) * mod_n : nullptr, mod_n * 4}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
@@ -851,6 +959,55 @@ moeca_status moeca_get_kernel_times(moeca_handle* h, moeca_kernel_times* out, in
       h->launches[i] = 0;
     }
   }
+  return MOECA_OK;
+}
+
+moeca_status moeca_ddpm_schedule(int32_t n_steps, int32_t n_train, double beta_start, double beta_end,
+                                 int32_t* t, double* alpha, double* alpha_bar, double* beta) {
+  if (n_steps < 2 || n_steps > n_train || !(beta_start > 0.0 && beta_start <= beta_end && beta_end < 1.0))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "2 <= n_steps <= n_train and 0 < beta_start <= beta_end < 1");
+  // Training schedule: linear betas, abar the running product of 1 - beta.
+  std::vector<double> abar(n_train);
+  double prod = 1.0;
+  for (int s = 0; s < n_train; ++s) {
+    const double b = n_train == 1 ? beta_start : beta_start + (beta_end - beta_start) * s / (n_train - 1);
+    prod *= 1.0 - b;
+    abar[s] = prod;
+  }
+  double prev = 1.0;
+  for (int j = 0; j < n_steps; ++j) {
+    const int ts = static_cast<int>(std::floor(static_cast<double>(j) * (n_train - 1) / (n_steps - 1) + 0.5));
+    const double ab = abar[ts];
+    const double al = ab / prev;
+    if (t) t[j] = ts;
+    if (alpha) alpha[j] = al;
+    if (alpha_bar) alpha_bar[j] = ab;
+    if (beta) beta[j] = 1.0 - al;
+    prev = ab;
+  }
+  return MOECA_OK;
+}
+
+moeca_status moeca_ddpm_step(const moeca_ddpm_args* a, void* stream) {
+  if (!a || !a->x_t || !a->eps || !a->x_prev) return fail(nullptr, MOECA_ERR_INVALID_ARG, "NULL argument");
+  if (a->n < 0 || a->n % 8) return fail(nullptr, MOECA_ERR_INVALID_ARG, "n must be a non-negative multiple of 8");
+  if (a->eps_dtype != MOECA_F32 && a->eps_dtype != MOECA_BF16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "eps_dtype");
+  if (!(a->alpha > 0.0 && a->alpha <= 1.0) || !(a->alpha_bar >= 0.0 && a->alpha_bar < 1.0) || !(a->sigma >= 0.0))
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "0 < alpha <= 1, 0 <= alpha_bar < 1, sigma >= 0");
+  if (a->sigma > 0.0 && !a->z) return fail(nullptr, MOECA_ERR_INVALID_ARG, "z is NULL with sigma > 0");
+  const void* ps[] = {a->x_t, a->eps, a->z, a->x_prev, a->x_next};
+  for (const void* p : ps)
+    if (reinterpret_cast<uintptr_t>(p) % 16) return fail(nullptr, MOECA_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  DdpmArgs d{};
+  d.n = a->n;
+  d.bf16 = a->eps_dtype == MOECA_BF16;
+  d.c1 = static_cast<float>((1.0 - a->alpha) / std::sqrt(1.0 - a->alpha_bar));
+  d.inv_sqrt_alpha = static_cast<float>(1.0 / std::sqrt(a->alpha));
+  d.sigma = static_cast<float>(a->sigma);
+  d.x_t = a->x_t; d.eps = a->eps; d.z = a->sigma > 0.0 ? a->z : nullptr;
+  d.x_prev = a->x_prev; d.x_next = a->x_next;
+  cudaError_t e = launch_ddpm(d, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail(nullptr, MOECA_ERR_CUDA, std::string("ddpm step: ") + cudaGetErrorString(e));
   return MOECA_OK;
 }
 

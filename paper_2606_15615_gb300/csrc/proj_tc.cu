@@ -16,6 +16,8 @@
 //                  a = bf16(C[m, :]), a_out[t, :] = a, u_out[t, :] = bf16(x[t, :] + a)
 //                  (the attention output a_i and the MoE input u_i = x_i + a_i);
 //                  u_i also goes to the token's FFN input rows when row_of is set
+//   kProjResidualGated  as kProjResidual with u = bf16(x + g a), g the row's
+//                  AdaLN gate (the sample's gate vector, Sec. 3); no FFN rows
 // M is a host bound; when m_dev is set the launch reads the actual row count
 // there (rows recomputed this step) and tiles past it return at once.
 //
@@ -73,6 +75,8 @@ struct ProjParams {
   __nv_bfloat16* q_out;      // kProjQKV: [list rows, D]
   __nv_bfloat16* k_out;      // kProjQKV: [n_tok, D]
   __nv_bfloat16* vt_out;     // kProjQKV: [D, n_tok]
+  const float* gate;         // kProjResidualGated: gate row of token t at gate + (t / seq) * gate_ld
+  int gate_ld, seq;
   int* status;
 };
 
@@ -153,6 +157,30 @@ __device__ __forceinline__ void store_residual(const float* v, const uint4* xv, 
   }
 }
 
+// Gated residual (AdaLN block): a = bf16(v), u = bf16(x + g a), 32 columns.
+__device__ __forceinline__ void store_residual_gated(const float* v, const uint4* xv, const float* g,
+                                                     __nv_bfloat16* a_dst, __nv_bfloat16* u_dst) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(g + 8 * j));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(g + 8 * j) + 1);
+    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    uint4 av, uv;
+    __nv_bfloat162* ah = reinterpret_cast<__nv_bfloat162*>(&av);
+    __nv_bfloat162* uh = reinterpret_cast<__nv_bfloat162*>(&uv);
+    const __nv_bfloat162* xh = reinterpret_cast<const __nv_bfloat162*>(&xv[j]);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      ah[q] = __floats2bfloat162_rn(v[8 * j + 2 * q], v[8 * j + 2 * q + 1]);
+      const float2 af = __bfloat1622float2(ah[q]);
+      const float2 xf = __bfloat1622float2(xh[q]);
+      uh[q] = __floats2bfloat162_rn(fmaf(gg[2 * q], af.x, xf.x), fmaf(gg[2 * q + 1], af.y, xf.y));
+    }
+    reinterpret_cast<uint4*>(a_dst)[j] = av;
+    reinterpret_cast<uint4*>(u_dst)[j] = uv;
+  }
+}
+
 __device__ __forceinline__ void load_x_chunk(const __nv_bfloat16* xr, uint4* xv) {
 #pragma unroll
   for (int j = 0; j < 4; ++j) xv[j] = __ldg(reinterpret_cast<const uint4*>(xr) + j);
@@ -163,6 +191,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     proj_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                    const ProjParams p) {
   constexpr int kStage = kPABytes + BN * 128;
+  constexpr bool kRes = MODE == kProjResidual || MODE == kProjResidualGated;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[8];
   __shared__ __align__(8) uint64_t empty_bar[8];
@@ -271,6 +300,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     for (int q = 0; q < kMaxRowOf; ++q) gr[q] = nullptr;
     const int n_g = p.row_of ? p.row_w : 0;
     __nv_bfloat16* krow = nullptr;  // kProjQKV: this lane's k row (dst holds its q row)
+    const float* grow = nullptr;    // kProjResidualGated: this lane's gate row
     if (m < M) {
       if constexpr (MODE == kProjStore) {
         dst = p.out + static_cast<size_t>(m) * p.ldo + n0;
@@ -286,6 +316,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
           dst = p.a_out + off;
           xr = p.x + off;
           ur = p.u_out + off;
+          if constexpr (MODE == kProjResidualGated) grow = p.gate + static_cast<size_t>(t / p.seq) * p.gate_ld + n0;
 #pragma unroll
           for (int q = 0; q < kMaxRowOf; ++q) {
             if (q < n_g) {
@@ -299,7 +330,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       }
     }
     uint4 xb[2][4];  // residual mode: x of chunks c and c + 1 in flight
-    if constexpr (MODE == kProjResidual) {
+    if constexpr (kRes) {
       if (xr) {
         load_x_chunk(xr, xb[0]);
         if (BN > 32) load_x_chunk(xr + 32, xb[1]);
@@ -309,7 +340,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     if (mbar_wait(smem_u32(&acc_bar), 0, &abort_flag)) {
       tc_fence_after();
       const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-      if constexpr (MODE == kProjResidual) {
+      if constexpr (kRes) {
 #pragma unroll
         for (int c = 0; c < BN / 32; ++c) {
           uint4 xc[4];
@@ -322,10 +353,14 @@ __global__ void __launch_bounds__(kPThreads, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(raw[j]) + s_bias[c * 32 + j];
           if (dst) {
-            __nv_bfloat16* gc[kMaxRowOf];
+            if constexpr (MODE == kProjResidualGated) {
+              store_residual_gated(v, xc, grow + c * 32, dst + c * 32, ur + c * 32);
+            } else {
+              __nv_bfloat16* gc[kMaxRowOf];
 #pragma unroll
-            for (int q = 0; q < kMaxRowOf; ++q) gc[q] = gr[q] ? gr[q] + c * 32 : nullptr;
-            store_residual(v, xc, dst + c * 32, ur + c * 32, gc, n_g);
+              for (int q = 0; q < kMaxRowOf; ++q) gc[q] = gr[q] ? gr[q] + c * 32 : nullptr;
+              store_residual(v, xc, dst + c * 32, ur + c * 32, gc, n_g);
+            }
           }
         }
       } else {
@@ -399,6 +434,7 @@ int proj_tile_n(int N, int want) {
 cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
   const int BN = proj_tile_n(a.N, a.tile_n);
   if (BN == 0 || a.K % 64 || a.M <= 0) return cudaErrorInvalidValue;
+  if (a.mode == kProjResidualGated && (!a.gate || a.seq <= 0 || a.row_of)) return cudaErrorInvalidValue;
   CUtensorMap amap, bmap;
   if (!encode_2d(&amap, a.A, static_cast<uint64_t>(a.a_rows), static_cast<uint64_t>(a.K), kPM) ||
       !encode_2d(&bmap, a.B, static_cast<uint64_t>(a.N), static_cast<uint64_t>(a.K), static_cast<uint32_t>(BN)))
@@ -418,6 +454,7 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
   p.q_out = static_cast<__nv_bfloat16*>(a.q_out);
   p.k_out = static_cast<__nv_bfloat16*>(a.k_out);
   p.vt_out = static_cast<__nv_bfloat16*>(a.vt_out);
+  p.gate = a.gate; p.gate_ld = a.gate_ld; p.seq = a.seq;
   p.status = a.status;
   const int kb = a.K / 64;
   const int stage = kPABytes + BN * 128;
@@ -438,6 +475,7 @@ cudaError_t launch_proj_tc(const ProjArgs& a, cudaStream_t s) {
     switch (a.mode) {
       case kProjQKV: return run(proj_tc_kernel<kBN, kProjQKV>);
       case kProjResidual: return run(proj_tc_kernel<kBN, kProjResidual>);
+      case kProjResidualGated: return run(proj_tc_kernel<kBN, kProjResidualGated>);
       default: return run(proj_tc_kernel<kBN, kProjStore>);
     }
   };

@@ -25,7 +25,7 @@ STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "
 MOECA_F32, MOECA_BF16 = 0, 1
 MOECA_FFN_AUTO, MOECA_FFN_SIMT = 0, 1
 KERNEL_KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn",
-                "qkv", "attn", "oproj", "attn_aux"]
+                "qkv", "attn", "oproj", "attn_aux", "adaln"]
 ATTN_SYNC, ATTN_STALE, ATTN_FULL = 0, 1, 2
 
 
@@ -40,18 +40,20 @@ class moeca_config(C.Structure):
                 ("gelu_tanh", C.c_int32), ("ffn_impl", C.c_int32), ("ffn_tile_n", C.c_int32),
                 ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32),
                 ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32),
-                ("attn_impl", C.c_int32)]
+                ("attn_impl", C.c_int32), ("adaln", C.c_int32), ("ln_eps", C.c_float),
+                ("keep_route_in", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):
     _fields_ = [("w_gate", C.c_void_p), ("b_gate", C.c_void_p), ("w1", C.c_void_p),
                 ("w2", C.c_void_p), ("ws1", C.c_void_p), ("ws2", C.c_void_p),
-                ("w_qkv", C.c_void_p), ("b_qkv", C.c_void_p), ("w_o", C.c_void_p), ("b_o", C.c_void_p)]
+                ("w_qkv", C.c_void_p), ("b_qkv", C.c_void_p), ("w_o", C.c_void_p), ("b_o", C.c_void_p),
+                ("w_ada", C.c_void_p), ("b_ada", C.c_void_p)]
 
 
 class moeca_step_args(C.Structure):
     _fields_ = [("n_tokens", C.c_int32), ("step_index", C.c_int32), ("force_refresh", C.c_int32),
-                ("tau0_override", C.c_float)]
+                ("tau0_override", C.c_float), ("cond", C.c_void_p)]
 
 
 class moeca_stats(C.Structure):
@@ -74,11 +76,11 @@ class moeca_layer_state(C.Structure):
 class moeca_layer_trace(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("route_e", "route_w", "tau", "recompute", "slot", "matched",
                                             "token_any", "counts", "offsets", "list", "layer_in",
-                                            "block_in")]
+                                            "block_in", "route_in", "resid", "mod")]
 
 
 class moeca_kernel_times(C.Structure):
-    _fields_ = [("total_ms", C.c_double * 12), ("launches", C.c_int64 * 12)]
+    _fields_ = [("total_ms", C.c_double * 13), ("launches", C.c_int64 * 13)]
 
 
 class moeca_route_args(C.Structure):
@@ -87,6 +89,12 @@ class moeca_route_args(C.Structure):
                 ("entropy_norm", C.c_int32), ("beta", C.c_float), ("tau0", C.c_float), ("alpha", C.c_float),
                 ("x", C.c_void_p), ("w_gate", C.c_void_p), ("b_gate", C.c_void_p), ("ema", C.c_void_p),
                 ("route_e", C.c_void_p), ("route_w", C.c_void_p), ("tau", C.c_void_p)]
+
+
+class moeca_ddpm_args(C.Structure):
+    _fields_ = [("n", C.c_int64), ("eps_dtype", C.c_int32), ("alpha", C.c_double), ("alpha_bar", C.c_double),
+                ("sigma", C.c_double), ("x_t", C.c_void_p), ("eps", C.c_void_p), ("z", C.c_void_p),
+                ("x_prev", C.c_void_p), ("x_next", C.c_void_p)]
 
 
 class MoecaError(RuntimeError):
@@ -120,6 +128,9 @@ def _load():
         "moeca_status_string": (C.c_char_p, [C.c_int]),
         "moeca_last_error": (C.c_char_p, [H]),
         "moeca_route_noalloc": (C.c_int, [C.POINTER(moeca_route_args), C.c_void_p]),
+        "moeca_ddpm_schedule": (C.c_int, [C.c_int32, C.c_int32, C.c_double, C.c_double, C.POINTER(C.c_int32),
+                                          C.POINTER(C.c_double), C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+        "moeca_ddpm_step": (C.c_int, [C.POINTER(moeca_ddpm_args), C.c_void_p]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -163,8 +174,9 @@ def moeca_create(cfg: moeca_config, layers: list, device: int = 0):
 
 
 def moeca_step(h, x_in_ptr: int, x_out_ptr: int, n_tokens: int, step_index: int,
-               force_refresh: bool = False, tau0_override: float = math.nan, stream: int = 0):
-    args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override)
+               force_refresh: bool = False, tau0_override: float = math.nan, stream: int = 0,
+               cond_ptr: int | None = None):
+    args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override, cond_ptr)
     _check(LIB.moeca_step(h, x_in_ptr, x_out_ptr, C.byref(args), stream or None), h)
 
 
@@ -226,6 +238,23 @@ def moeca_route_noalloc(args: moeca_route_args, stream: int = 0):
         raise MoecaError(st, "moeca_route_noalloc")
 
 
+def moeca_ddpm_schedule(n_steps: int, n_train: int = 1000, beta_start: float = 1e-4, beta_end: float = 0.02):
+    """Per-step (t, alpha, alpha_bar, beta) lists of a sampling run (Eq. 1; see include/moeca.h)."""
+    t = (C.c_int32 * n_steps)()
+    al, ab, be = (C.c_double * n_steps)(), (C.c_double * n_steps)(), (C.c_double * n_steps)()
+    st = LIB.moeca_ddpm_schedule(n_steps, n_train, beta_start, beta_end, t, al, ab, be)
+    if st != MOECA_OK:
+        _check(st, None)
+    return list(t), list(al), list(ab), list(be)
+
+
+def moeca_ddpm_step(args: moeca_ddpm_args, stream: int = 0):
+    """One reverse transition of Eq. 1 on device buffers (see include/moeca.h)."""
+    st = LIB.moeca_ddpm_step(C.byref(args), stream or None)
+    if st != MOECA_OK:
+        _check(st, None)
+
+
 def moeca_status_string(status: int) -> str:
     return LIB.moeca_status_string(status).decode()
 
@@ -276,6 +305,10 @@ class Stack:
                 for name in ("b_qkv", "b_o"):
                     bt = dev(w.get(name), torch.float32)
                     setattr(lw, name, bt.data_ptr() if bt is not None else None)
+            if cfg.adaln:
+                lw.w_ada = dev(w["w_ada"]).data_ptr()
+                bt = dev(w.get("b_ada"), torch.float32)
+                lw.b_ada = bt.data_ptr() if bt is not None else None
             cl.append(lw)
         self.handle = moeca_create(cfg, cl, device)
 
@@ -293,13 +326,19 @@ class Stack:
     def stream_ptr(self) -> int:
         return self.torch.cuda.current_stream(self.device).cuda_stream
 
-    def step(self, x, step_index: int, force_refresh: bool = False, tau0=math.nan, out=None):
+    def step(self, x, step_index: int, force_refresh: bool = False, tau0=math.nan, out=None, cond=None):
+        """One denoising step; ``cond`` is the [T / seq_len, D] float32 CUDA
+        tensor of per-sample conditioning an AdaLN stack reads."""
         torch = self.torch
         T = x.shape[0]
         if out is None:
             out = torch.empty_like(x)
+        if cond is not None:
+            if cond.dtype != torch.float32 or not cond.is_cuda or not cond.is_contiguous():
+                raise ValueError("cond must be a contiguous float32 CUDA tensor")
+            self._cond = cond  # read by the step's first kernel: keep it alive until then
         moeca_step(self.handle, x.data_ptr(), out.data_ptr(), T, step_index, force_refresh, tau0,
-                   self.stream_ptr())
+                   self.stream_ptr(), cond.data_ptr() if cond is not None else None)
         return out
 
     def _empty(self, shape, dtype):
@@ -339,7 +378,10 @@ class Stack:
                  offsets=self._empty((G + 1,), torch.int32),
                  list=self._empty((T * (k + c.n_shared),), torch.int32),
                  layer_in=self._empty((T, c.hidden), self.dtype),
-                 block_in=self._empty((T, c.hidden), self.dtype) if c.n_heads else None)
+                 block_in=self._empty((T, c.hidden), self.dtype) if c.n_heads else None,
+                 route_in=self._empty((T, c.hidden), self.dtype) if c.adaln and c.keep_route_in else None,
+                 resid=self._empty((T, c.hidden), self.dtype) if c.n_heads else None,
+                 mod=self._empty((T // (c.seq_len or T), 6 * c.hidden), torch.float32) if c.adaln else None)
         t = {kk: v for kk, v in t.items() if v is not None}
         tr = moeca_layer_trace(**{kk: v.data_ptr() for kk, v in t.items()})
         moeca_get_layer_trace(self.handle, layer, tr, self.stream_ptr())
@@ -347,3 +389,19 @@ class Stack:
 
     def stats(self, layer: int = -1) -> dict:
         return moeca_get_stats(self.handle, layer)
+
+
+def ddpm_step(x_t, eps, alpha: float, alpha_bar: float, sigma: float, z=None, x_prev=None, x_next=None,
+              stream: int = 0):
+    """Eq. 1 on torch CUDA tensors: x_prev (fp32) = the reverse step of x_t
+    (fp32) with the denoiser output eps; x_next (eps's dtype) optionally
+    receives x_prev for the next denoiser call.  Returns x_prev."""
+    import torch
+    if x_prev is None:
+        x_prev = torch.empty_like(x_t)
+    args = moeca_ddpm_args(
+        x_t.numel(), MOECA_BF16 if eps.dtype == torch.bfloat16 else MOECA_F32, alpha, alpha_bar, sigma,
+        x_t.data_ptr(), eps.data_ptr(), z.data_ptr() if z is not None else None, x_prev.data_ptr(),
+        x_next.data_ptr() if x_next is not None else None)
+    moeca_ddpm_step(args, stream or torch.cuda.current_stream(x_t.device).cuda_stream)
+    return x_prev

@@ -24,7 +24,7 @@ _WEIGHT_SEED = 1000
 _TRAJ_SEED = 2000
 
 # Tensor ids inside a layer's weight seed tuple.
-_T_GATE, _T_W1, _T_W2, _T_WS1, _T_WS2, _T_BIAS, _T_QKV, _T_BQKV, _T_WO, _T_BO = range(10)
+_T_GATE, _T_W1, _T_W2, _T_WS1, _T_WS2, _T_BIAS, _T_QKV, _T_BQKV, _T_WO, _T_BO, _T_ADA, _T_BADA = range(12)
 
 
 @dataclass(frozen=True)
@@ -48,6 +48,7 @@ class Workload:
     router_skew: tuple = ()   # target top-k load shares, e.g. (4, 2, 1, 1)
     reuse_targets: tuple = (0.5,)
     n_heads: int = 0          # > 0: DiT-MoE blocks (self-attention over each sample's seq tokens, then MoE)
+    adaln: bool = False       # DiT-MoE blocks with AdaLN modulation and a per-sample conditioning input
 
     @property
     def n_tokens(self) -> int:
@@ -101,11 +102,23 @@ def dit_variant(wl: Workload) -> Workload:
 DIT_WORKLOADS = {d.name: d for d in (dit_variant(w) for w in WORKLOADS.values() if w.dtype == "bf16")}
 
 
+def adaln_variant(wl: Workload) -> Workload:
+    """The DiT-MoE variant with AdaLN-modulated blocks (Sec. 3), driven by a
+    per-sample conditioning vector each step."""
+    d = dit_variant(wl)
+    return replace(d, name=d.name.replace("dit_", "ditada_", 1), adaln=True)
+
+
+ADALN_WORKLOADS = {d.name: d for d in (adaln_variant(w) for w in WORKLOADS.values() if w.dtype == "bf16")}
+
+
 def workload(name_or_index) -> Workload:
     if isinstance(name_or_index, int):
         return WORKLOADS[WORKLOAD_ORDER[name_or_index - 1]]
     if name_or_index in DIT_WORKLOADS:
         return DIT_WORKLOADS[name_or_index]
+    if name_or_index in ADALN_WORKLOADS:
+        return ADALN_WORKLOADS[name_or_index]
     return WORKLOADS[name_or_index]
 
 
@@ -217,6 +230,22 @@ def make_attn_weights(wl: Workload, layer: int) -> dict:
         "w_o": _store(wl, 0.02 * _rng(seed, layer, _T_WO).standard_normal((D, D), dtype=np.float32)),
         "b_o": (0.02 * _rng(seed, layer, _T_BO).standard_normal(D)).astype(np.float32),
     }
+
+
+def make_adaln_weights(wl: Workload, layer: int) -> dict:
+    """AdaLN projection of one block, N(0, 0.02^2): w_ada [6D, D] in the
+    workload dtype, b_ada [6D] float32."""
+    seed = _WEIGHT_SEED + wl.index
+    D = wl.hidden
+    return {
+        "w_ada": _store(wl, 0.02 * _rng(seed, layer, _T_ADA).standard_normal((6 * D, D), dtype=np.float32)),
+        "b_ada": (0.02 * _rng(seed, layer, _T_BADA).standard_normal(6 * D)).astype(np.float32),
+    }
+
+
+def workload_conditioning(wl: Workload, n_steps: int | None = None) -> np.ndarray:
+    """Per-step conditioning [n_steps, batch, D] of an AdaLN workload."""
+    return conditioning(_TRAJ_SEED + wl.index, wl.batch, wl.hidden, wl.n_steps if n_steps is None else n_steps)
 
 
 def tiny_attn(seed: int, D: int, dtype: str = "f32", bias: bool = True, wscale: float = 0.2) -> dict:
@@ -337,6 +366,9 @@ def make_layer_weights_device(wl: Workload, layer: int, device) -> dict:
         out["b_qkv"] = draw(_T_BQKV, (3 * D,)).float()
         out["w_o"] = draw(_T_WO, (D, D))
         out["b_o"] = draw(_T_BO, (D,)).float()
+    if wl.adaln:
+        out["w_ada"] = draw(_T_ADA, (6 * D, D))
+        out["b_ada"] = draw(_T_BADA, (6 * D,)).float()
     b = _skew_bias(wl)
     out["b_gate"] = None if b is None else torch.from_numpy(b).to(device)
     if S:

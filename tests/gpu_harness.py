@@ -16,6 +16,15 @@ A DiT-MoE block (n_heads > 0) first checks its attention sub-layer:
 and the router check then takes the input the rule routes on: u on full
 steps (and under the "stale" and "full" policies), bf16(x + a^{t0}) on a
 sync cache step.
+An AdaLN block (adaln = 1) checks instead:
+  modulation the step's conditioning     -> six vectors per sample (tolerance)
+  attention  the GPU x and modulation    -> h = LN-modulate(x), recomputed a rows
+                                            (tolerance), kept a rows (exact)
+  residual   the GPU a                    -> u = bf16(x + g_a a) (within one bf16
+                                            step on a few elements)
+  MoE input  the GPU u                    -> m, and the router input m' (same bound)
+and the MoE check then routes on the GPU's router input, recomputes on m and
+forms u + g_m y.
 """
 from __future__ import annotations
 
@@ -71,7 +80,7 @@ def params_of(cfg) -> O.Params:
         gelu="tanh" if cfg.gelu_tanh else "erf", score_terms=cfg.score_terms,
         granularity="branch" if cfg.granularity == 0 else "token",
         n_heads=cfg.n_heads, seq_len=cfg.seq_len, attn_policy=("sync", "stale", "full")[cfg.attn_policy],
-        act_store="bf16" if cfg.dtype == 1 else "f64")
+        act_store="bf16" if cfg.dtype == 1 else "f64", adaln=bool(cfg.adaln), ln_eps=cfg.ln_eps)
 
 
 def oracle_weights(w: dict) -> dict:
@@ -160,8 +169,83 @@ def check_attention(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr:
     return O.round_bf16(x + a_pre)
 
 
+def close_in_bf16(got, want, what: str, max_frac: float = 2e-3):
+    """``got`` (bf16 values from the GPU) equals bf16(``want``) except on a
+    few elements, and there by at most one bf16 step: the GPU rounds a float32
+    result, the oracle a float64 one, so values within float32 error of a bf16
+    rounding boundary may land on either side."""
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    exact = O.round_bf16(want)
+    diff = got != exact
+    step = np.maximum(np.abs(exact), 1e-30) * 2.0 ** -7
+    assert (np.abs(got - exact)[diff] <= step[diff] + 1e-30).all(), \
+        f"{what}: an element is off by more than one bf16 step"
+    assert diff.mean() <= max_frac, f"{what}: {int(diff.sum())} of {diff.size} elements differ"
+    return int(diff.sum())
+
+
+def check_adaln(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dict, refresh: bool, cond,
+                tol: float = 1e-2):
+    """Teacher-forced check of an AdaLN block's modulation and attention
+    sub-layer (Sec. 3 residual form under the Sec. 4.1 cache).  Returns
+    (router input, residual u, gate_m token rows) for the MoE check; the
+    trace's layer_in is the MoE input m."""
+    wo = oracle_weights(w)
+    D = cfg.hidden
+    x = np_of(tr["block_in"]).astype(np.float64)
+    T = x.shape[0]
+    S = cfg.seq_len or T
+    eps = float(np.float32(cfg.ln_eps))
+    # ---- modulation: float32 dot products of D terms against the float64 oracle
+    c = np.asarray(cond, np.float64)
+    mod_g = np_of(tr["mod"]).astype(np.float64).reshape(T // S, 6, D)
+    mod_o = O.adaln_modulation(c, wo["w_ada"], wo.get("b_ada"))
+    mag = (np.abs(O.silu(c)) @ np.abs(wo["w_ada"]).T).reshape(T // S, 6, D)
+    err = np.abs(mod_g - mod_o)
+    assert (err <= 1e-5 * mag + 1e-6).all(), f"modulation: worst err {err.max():.3e}"
+    rows6 = [O.token_rows(mod_g[:, j], T, S) for j in range(6)]
+    # ---- attention from h = LN-modulate(x)
+    h = O.round_bf16(O.modulate(O.layer_norm(x, eps), rows6[0], rows6[1]))
+    a_post = np_of(post["attn_a"]).astype(np.float64)
+    full = refresh or cfg.attn_policy == 2
+    has_pre = pre is not None and pre["n_tokens"]
+    a_pre = np_of(pre["attn_a"]).astype(np.float64) if has_pre else None
+    if full:
+        rows = np.arange(T)
+    elif cfg.attn_policy == 1:
+        rows = np.zeros(0, np.int64)
+    else:
+        rows = np.nonzero(np_of(tr["token_any"]))[0]
+    if len(rows):
+        a_o = O.attention(h, wo["w_qkv"], wo.get("b_qkv"), wo["w_o"], wo.get("b_o"), cfg.n_heads, cfg.seq_len, rows)
+        rl = rel_l2(a_post[rows], a_o)
+        rep.max_attn_rel_l2 = max(rep.max_attn_rel_l2, rl)
+        assert rl <= tol, f"attention rows rel L2 {rl:.3e}"
+        per_row = np.linalg.norm(a_post[rows] - a_o, axis=1) / np.maximum(np.linalg.norm(a_o, axis=1), 1e-30)
+        assert per_row.max() <= 4 * tol, f"worst attention row rel L2 {per_row.max():.3e}"
+    kept = np.setdiff1d(np.arange(T), rows)
+    if len(kept):
+        assert a_pre is not None, "a cache step without a cached attention output"
+        assert np.array_equal(a_post[kept], a_pre[kept]), "kept attention rows changed"
+    # ---- residual u = x + g_a a and MoE input m = LN-modulate(u), from the GPU's a and u
+    u = np_of(tr["resid"]).astype(np.float64)
+    m = np_of(tr["layer_in"]).astype(np.float64)
+    close_in_bf16(u, x + rows6[2] * a_post, "residual u")
+    close_in_bf16(m, O.modulate(O.layer_norm(u, eps), rows6[3], rows6[4]), "MoE input m")
+    r = np_of(tr["route_in"]).astype(np.float64)
+    if full or cfg.attn_policy == 1:
+        assert np.array_equal(r, m), "router input differs from the MoE input"
+    else:
+        u_pre = O.round_bf16(x + rows6[2] * a_pre)
+        close_in_bf16(r, O.modulate(O.layer_norm(u_pre, eps), rows6[3], rows6[4]), "router input m'")
+        assert np.array_equal(r[kept], m[kept]), "kept tokens' MoE input differs from their router input"
+    rep.attn_rows += len(rows)
+    return r, u, rows6[5]
+
+
 def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dict, out_gpu: np.ndarray,
-                refresh: bool, bf16: bool, out_tol=None, route_in=None):
+                refresh: bool, bf16: bool, out_tol=None, route_in=None, resid=None, gate=None):
     """Teacher-forced comparison of one layer step.  Raises AssertionError.
 
     ``route_in`` is the router input when it differs from the FFN input
@@ -213,7 +297,8 @@ def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
     assert np.array_equal(np_of(tr["offsets"]), off), "group offsets"
     assert np.array_equal(np_of(tr["list"])[: off[-1]], flat), "row lists"
     # ---- FFN + combine (Eq. 5, Eq. 8) from the GPU decisions and pre-step cache
-    out_o, new_o, _ = O.recompute_and_combine(st_pre, u, e_g, w_g, rec_g, slot_g, wo, prm, refresh)
+    out_o, new_o, _ = O.recompute_and_combine(st_pre, u, e_g, w_g, rec_g, slot_g, wo, prm, refresh,
+                                              resid=resid, gate=gate)
     rl = rel_l2(out_gpu, out_o)
     ma = float(np.abs(out_gpu - out_o).max())
     rep.max_rel_l2 = max(rep.max_rel_l2, rl)
@@ -256,14 +341,21 @@ def check_layer(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
 
 
 def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True, bf16=True, out_tol=None,
-                   forces=None):
-    """Step the GPU stack over ``xs`` and check every layer of every step."""
+                   forces=None, conds=None, next_input=None, n_steps=None):
+    """Step the GPU stack over ``xs`` and check every layer of every step
+    (``conds[t]``: the per-sample conditioning of an AdaLN stack).  With
+    ``next_input``, xs[0] starts ``n_steps`` steps and step t > 0 takes
+    next_input(t, previous output)."""
     import torch
     rep = Report()
     dt = torch.bfloat16 if bf16 else torch.float32
     L = cfg.n_layers
     prev_T = None
-    for t, x in enumerate(xs):
+    n = len(xs) if next_input is None else n_steps
+    out = None
+    for t in range(n):
+        # A sampler loop feeds each step's output through ``next_input``.
+        x = xs[t] if next_input is None or t == 0 else next_input(t, out)
         T = x.shape[0]
         force = bool(forces and forces[t])
         N = cfg.refresh_period
@@ -274,7 +366,8 @@ def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True
         if check and prev_T != T:
             pre = [None] * L
         xd = torch.from_numpy(np.ascontiguousarray(x, np.float32)).cuda().to(dt)
-        out = stack.step(xd, t, force_refresh=force)
+        cd = None if conds is None else torch.from_numpy(np.ascontiguousarray(conds[t], np.float32)).cuda()
+        out = stack.step(xd, t, force_refresh=force, cond=cd)
         torch.cuda.synchronize()
         if check:
             block = cfg.n_heads > 0
@@ -285,9 +378,16 @@ def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True
                     out_l = np_of(stack.get_trace(l + 1, T)["block_in" if block else "layer_in"]).astype(np.float64)
                 else:
                     out_l = np_of(out).astype(np.float64)
-                route_in = check_attention(rep, cfg, layer_weights[l], pre[l], post, tr, refresh) if block else None
+                resid = gate = None
+                if cfg.adaln:
+                    route_in, resid, gate = check_adaln(rep, cfg, layer_weights[l], pre[l], post, tr, refresh,
+                                                        conds[t])
+                elif block:
+                    route_in = check_attention(rep, cfg, layer_weights[l], pre[l], post, tr, refresh)
+                else:
+                    route_in = None
                 check_layer(rep, cfg, layer_weights[l], pre[l], post, tr, out_l, refresh, bf16, out_tol,
-                            route_in=route_in)
+                            route_in=route_in, resid=resid, gate=gate)
         rep.steps += 1
         prev_T = T
     return rep, out

@@ -77,3 +77,47 @@ def test_attention_config_validation_needs_no_gpu(lib):
     assert create(n_heads=24) == lib.MOECA_ERR_UNSUPPORTED                     # 32 channels per head
     assert create(n_heads=12) == lib.MOECA_ERR_INVALID_ARG                     # no attention weights
     assert b"attention weights" in L.moeca_last_error(None)
+
+
+def test_adaln_config_validation_needs_no_gpu(lib):
+    """AdaLN settings are checked before any device call."""
+    L = lib.LIB
+    h = ctypes.c_void_p()
+    w = (lib.moeca_layer_weights * 1)()
+    w[0].w_gate = w[0].w1 = w[0].w2 = w[0].w_qkv = w[0].w_o = 4096
+
+    def create(**kw):
+        base = dict(n_layers=1, hidden=768, ffn=256, n_experts=4, top_k=2, max_tokens=512)
+        base.update(kw)
+        c = lib.moeca_config_default(**base)
+        return L.moeca_create(ctypes.byref(c), w, 0, ctypes.byref(h))
+
+    cfg = lib.moeca_config_default()
+    assert cfg.adaln == 0 and cfg.keep_route_in == 0 and abs(cfg.ln_eps - 1e-6) < 1e-12
+    assert create(adaln=2, n_heads=12) == lib.MOECA_ERR_INVALID_ARG
+    assert create(adaln=1) == lib.MOECA_ERR_UNSUPPORTED                     # AdaLN needs a DiT block
+    assert create(adaln=1, n_heads=12, ln_eps=0.0) == lib.MOECA_ERR_INVALID_ARG
+    # 512 one-token samples: 512 x 768 x 4 bytes of staged conditioning do not fit
+    assert create(adaln=1, n_heads=12, seq_len=1) == lib.MOECA_ERR_UNSUPPORTED
+    assert create(adaln=1, n_heads=12, seq_len=256) == lib.MOECA_ERR_INVALID_ARG  # no AdaLN weights
+    assert b"AdaLN weights" in L.moeca_last_error(None)
+
+
+def test_ddpm_schedule_matches_the_oracle(lib):
+    """The library's Eq. 1 schedule (host code) against the oracle's."""
+    import numpy as np
+    from oracle import moeca_oracle as O
+    for n in (2, 7, 50, 250, 1000):
+        t, a, ab, b = lib.moeca_ddpm_schedule(n)
+        to, ao, abo, bo = O.ddpm_schedule(n)
+        assert np.array_equal(t, to)
+        np.testing.assert_allclose(a, ao, rtol=1e-13)
+        np.testing.assert_allclose(ab, abo, rtol=1e-13)
+        np.testing.assert_allclose(b, bo, rtol=1e-9, atol=1e-15)
+    for bad in ((1, 1000), (1001, 1000)):
+        with pytest.raises(lib.MoecaError):
+            lib.moeca_ddpm_schedule(*bad)
+    args = lib.moeca_ddpm_args(n=12, eps_dtype=lib.MOECA_BF16, alpha=0.9, alpha_bar=0.5, sigma=0.1,
+                               x_t=4096, eps=4096, z=4096, x_prev=4096)
+    with pytest.raises(lib.MoecaError):          # n not a multiple of 8: refused before any launch
+        lib.moeca_ddpm_step(args)
