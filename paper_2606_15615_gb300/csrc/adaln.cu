@@ -17,7 +17,8 @@ namespace moeca {
 namespace {
 
 constexpr int kModWarps = 8;
-constexpr int kModB = 8;  // samples accumulated per pass over a weight row
+constexpr int kModB = 8;  // samples accumulated per pass over the weight rows
+constexpr int kModR = 4;  // weight rows per warp pass: each staged SiLU(c) load feeds kModR rows
 
 __global__ void __launch_bounds__(kModWarps * 32) ada_mod_kernel(AdaModArgs a) {
   extern __shared__ __align__(16) float s_c[];  // [B, D] SiLU(c)
@@ -31,41 +32,53 @@ __global__ void __launch_bounds__(kModWarps * 32) ada_mod_kernel(AdaModArgs a) {
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int per_layer = 6 * D;
-  const long long n_rows = static_cast<long long>(a.L) * per_layer;
+  const int per_layer = 6 * D;                   // a multiple of kModR (D is a multiple of 64)
+  const long long n_groups = static_cast<long long>(a.L) * (per_layer / kModR);
   const int nvec = D / 8;
-  for (long long r = static_cast<long long>(blockIdx.x) * kModWarps + warp; r < n_rows;
-       r += static_cast<long long>(gridDim.x) * kModWarps) {
-    const int l = static_cast<int>(r / per_layer);
-    const int j = static_cast<int>(r - static_cast<long long>(l) * per_layer);
-    const uint4* wrow = reinterpret_cast<const uint4*>(a.w[l]) + static_cast<size_t>(j) * nvec;
+  for (long long g = static_cast<long long>(blockIdx.x) * kModWarps + warp; g < n_groups;
+       g += static_cast<long long>(gridDim.x) * kModWarps) {
+    const long long r0 = g * kModR;              // kModR rows of one layer
+    const int l = static_cast<int>(r0 / per_layer);
+    const int j0 = static_cast<int>(r0 - static_cast<long long>(l) * per_layer);
+    const uint4* wrow = reinterpret_cast<const uint4*>(a.w[l]) + static_cast<size_t>(j0) * nvec;
     const float* bl = a.b[l];
-    const float bias = bl ? bl[j] : 0.f;
-    float* out = a.out + static_cast<size_t>(l) * B * per_layer + j;
+    float* out = a.out + static_cast<size_t>(l) * B * per_layer + j0;
     for (int b0 = 0; b0 < B; b0 += kModB) {
-      float acc[kModB];
+      float acc[kModR][kModB];
 #pragma unroll
-      for (int q = 0; q < kModB; ++q) acc[q] = 0.f;
-#pragma unroll 4
+      for (int r = 0; r < kModR; ++r)
+#pragma unroll
+        for (int q = 0; q < kModB; ++q) acc[r][q] = 0.f;
+#pragma unroll 2
       for (int c = lane; c < nvec; c += 32) {
-        float wf[8];
-        unpack_vec(__ldg(wrow + c), wf, static_cast<__nv_bfloat16*>(nullptr));
+        float wf[kModR][8];
+#pragma unroll
+        for (int r = 0; r < kModR; ++r)
+          unpack_vec(__ldg(wrow + static_cast<size_t>(r) * nvec + c), wf[r], static_cast<__nv_bfloat16*>(nullptr));
 #pragma unroll
         for (int q = 0; q < kModB; ++q) {
           if (b0 + q < B) {
             const float4* cp = reinterpret_cast<const float4*>(s_c + static_cast<size_t>(b0 + q) * D + 8 * c);
             const float4 c0 = cp[0], c1 = cp[1];
-            float s = acc[q];
-            s = fmaf(wf[0], c0.x, s); s = fmaf(wf[1], c0.y, s); s = fmaf(wf[2], c0.z, s); s = fmaf(wf[3], c0.w, s);
-            s = fmaf(wf[4], c1.x, s); s = fmaf(wf[5], c1.y, s); s = fmaf(wf[6], c1.z, s); s = fmaf(wf[7], c1.w, s);
-            acc[q] = s;
+            const float cv[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+#pragma unroll
+            for (int r = 0; r < kModR; ++r) {
+              float s = acc[r][q];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) s = fmaf(wf[r][e], cv[e], s);
+              acc[r][q] = s;
+            }
           }
         }
       }
 #pragma unroll
-      for (int q = 0; q < kModB; ++q) {
-        const float v = warp_sum(acc[q]);
-        if (lane == 0 && b0 + q < B) out[static_cast<size_t>(b0 + q) * per_layer] = v + bias;
+      for (int r = 0; r < kModR; ++r) {
+        const float bias = bl ? bl[j0 + r] : 0.f;
+#pragma unroll
+        for (int q = 0; q < kModB; ++q) {
+          const float v = warp_sum(acc[r][q]);
+          if (lane == 0 && b0 + q < B) out[static_cast<size_t>(b0 + q) * per_layer + r] = v + bias;
+        }
       }
     }
   }
@@ -156,24 +169,27 @@ __global__ void __launch_bounds__(kLnWarps * 32) adaln_rows_kernel(AdaLnArgs a) 
   const float* md = a.mod + static_cast<size_t>(t / a.seq) * 6 * D;
   const uint4* x4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) + off);
   __nv_bfloat16* u = static_cast<__nv_bfloat16*>(a.u) + off;
-  uint4 v[kLnChunks];
+  uint4 v[kLnChunks], av[kLnChunks];
+  const uint4* a4 =
+      a.a ? reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.a) + off) : nullptr;
   if (a.h_out || a.a) {
+    // x and the cached attention row in flight together.
 #pragma unroll
     for (int q = 0; q < kLnChunks; ++q)
       if (lane + 32 * q < nvec) v[q] = x4[lane + 32 * q];
+    if (a4) {
+#pragma unroll
+      for (int q = 0; q < kLnChunks; ++q)
+        if (lane + 32 * q < nvec) av[q] = a4[lane + 32 * q];
+    }
   }
   float mean, rstd;
   if (a.h_out) {
     row_stats(v, nvec, lane, D, a.eps, mean, rstd);
     store_modulated(v, nvec, lane, mean, rstd, md, md + D, static_cast<__nv_bfloat16*>(a.h_out) + off, nullptr);
   }
-  if (a.a) {
+  if (a4) {
     // u = bf16(x + gate_a a): one rounding of the fused product-sum.
-    const uint4* a4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.a) + off);
-    uint4 av[kLnChunks];
-#pragma unroll
-    for (int q = 0; q < kLnChunks; ++q)
-      if (lane + 32 * q < nvec) av[q] = a4[lane + 32 * q];
 #pragma unroll
     for (int q = 0; q < kLnChunks; ++q) {
       const int c = lane + 32 * q;
@@ -250,12 +266,13 @@ cudaError_t launch_ada_mod(const AdaModArgs& a, int n_sms, cudaStream_t s) {
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  // Up to four blocks per SM, fewer when the staged conditioning is large.
+  // Two blocks per SM (128 registers a thread), fewer when the staged
+  // conditioning is large; the warps stride over groups of kModR rows.
   int per_sm = static_cast<int>((200 * 1024) / (smem + 1024));
-  per_sm = per_sm < 1 ? 1 : (per_sm > 4 ? 4 : per_sm);
-  const long long rows = static_cast<long long>(a.L) * 6 * a.D;
+  per_sm = per_sm < 1 ? 1 : (per_sm > 2 ? 2 : per_sm);
+  const long long groups = static_cast<long long>(a.L) * 6 * a.D / kModR;
   long long grid = static_cast<long long>(n_sms) * per_sm;
-  const long long need = (rows + kModWarps - 1) / kModWarps;
+  const long long need = (groups + kModWarps - 1) / kModWarps;
   if (grid > need) grid = need;
   return launch_pdl(ada_mod_kernel, dim3(static_cast<unsigned>(grid)), dim3(kModWarps * 32), smem, s, a);
 }

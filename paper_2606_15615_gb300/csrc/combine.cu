@@ -74,6 +74,7 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   const uint4* sh4 = reinterpret_cast<const uint4*>(sh);
   for (int c0 = 0; c0 < nvec; c0 += 32 * CG) {
     uint4 h[CG][KMAX], xr[CG], hr[CG];
+    float4 gq[GATED ? CG : 1][V / 4];  // AdaLN gate values of the chunks, loaded with the rows
 #pragma unroll
     for (int g = 0; g < CG; ++g) {
       const int c = c0 + g * 32 + lane;
@@ -83,6 +84,10 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
           if (p < k) h[g][p] = ch4[static_cast<size_t>(q[p]) * nvec + c];
         xr[g] = c0 == 0 ? x_first[g] : x4[c];
         if (sh) hr[g] = sh4[c];
+        if constexpr (GATED) {
+#pragma unroll
+          for (int j = 0; j < V / 4; ++j) gq[g][j] = __ldg(reinterpret_cast<const float4*>(gr + c * V) + j);
+        }
       }
     }
 #pragma unroll
@@ -113,9 +118,7 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
         float xs[V];
         unpack_vec(xr[g], xs, static_cast<TI*>(nullptr));
         if constexpr (GATED) {
-          float gv[V];
-#pragma unroll
-          for (int j = 0; j < V; j += 4) load_vec(gr + c * V + j, gv + j);
+          const float* gv = reinterpret_cast<const float*>(gq[g]);
 #pragma unroll
           for (int j = 0; j < V; ++j) xs[j] = fmaf(gv[j], y[j], xs[j]);
         } else {
@@ -138,7 +141,8 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
 template <typename TI, bool GATED>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
-  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, 4, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  // The gated form holds the gate values with the rows: half the chunks in flight keeps it near 128 registers.
+  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, GATED ? 2 : 4, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
   else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
   else launch_pdl(combine_kernel<TI, 8, 1, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
 }

@@ -169,18 +169,22 @@ def check_attention(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr:
     return O.round_bf16(x + a_pre)
 
 
-def close_in_bf16(got, want, what: str, max_frac: float = 2e-3):
+def close_in_bf16(got, want, what: str, max_frac: float = 2e-3, floor=0.0):
     """``got`` (bf16 values from the GPU) equals bf16(``want``) except on a
-    few elements, and there by at most one bf16 step: the GPU rounds a float32
-    result, the oracle a float64 one, so values within float32 error of a bf16
-    rounding boundary may land on either side."""
+    few elements, and there by at most one bf16 step plus ``floor``: the GPU
+    rounds a float32 result, the oracle a float64 one, so values within
+    float32 error of a bf16 rounding boundary may land on either side.
+    ``floor`` (per element) is the float32 error of the result's ingredients,
+    which dominates where a sum of larger terms nearly cancels."""
     got = np.asarray(got, np.float64)
     want = np.asarray(want, np.float64)
     exact = O.round_bf16(want)
     diff = got != exact
-    step = np.maximum(np.abs(exact), 1e-30) * 2.0 ** -7
-    assert (np.abs(got - exact)[diff] <= step[diff] + 1e-30).all(), \
-        f"{what}: an element is off by more than one bf16 step"
+    bound = np.maximum(np.abs(exact), 1e-30) * 2.0 ** -7 + np.broadcast_to(floor, exact.shape)
+    off = np.abs(got - exact)
+    bad = diff & (off > bound + 1e-30)
+    assert not bad.any(), (f"{what}: {int(bad.sum())} elements off by more than one bf16 step, worst "
+                           f"{off[bad].max():.3e} at |value| {np.abs(exact[bad][off[bad].argmax()]):.3e}")
     assert diff.mean() <= max_frac, f"{what}: {int(diff.sum())} of {diff.size} elements differ"
     return int(diff.sum())
 
@@ -231,14 +235,20 @@ def check_adaln(rep: Report, cfg, w: dict, pre: dict | None, post: dict, tr: dic
     # ---- residual u = x + g_a a and MoE input m = LN-modulate(u), from the GPU's a and u
     u = np_of(tr["resid"]).astype(np.float64)
     m = np_of(tr["layer_in"]).astype(np.float64)
-    close_in_bf16(u, x + rows6[2] * a_post, "residual u")
-    close_in_bf16(m, O.modulate(O.layer_norm(u, eps), rows6[3], rows6[4]), "MoE input m")
+    close_in_bf16(u, x + rows6[2] * a_post, "residual u", floor=2.0 ** -22 * (np.abs(x) + np.abs(rows6[2] * a_post)))
+
+    def ln_floor(v):
+        # float32 mean / rsqrt over D and the two products: 1e-5 of the terms
+        return 1e-5 * (np.abs(O.layer_norm(v, eps) * (1 + rows6[4])) + np.abs(rows6[3]))
+
+    close_in_bf16(m, O.modulate(O.layer_norm(u, eps), rows6[3], rows6[4]), "MoE input m", floor=ln_floor(u))
     r = np_of(tr["route_in"]).astype(np.float64)
     if full or cfg.attn_policy == 1:
         assert np.array_equal(r, m), "router input differs from the MoE input"
     else:
         u_pre = O.round_bf16(x + rows6[2] * a_pre)
-        close_in_bf16(r, O.modulate(O.layer_norm(u_pre, eps), rows6[3], rows6[4]), "router input m'")
+        close_in_bf16(r, O.modulate(O.layer_norm(u_pre, eps), rows6[3], rows6[4]), "router input m'",
+                      floor=ln_floor(u_pre))
         assert np.array_equal(r[kept], m[kept]), "kept tokens' MoE input differs from their router input"
     rep.attn_rows += len(rows)
     return r, u, rows6[5]
@@ -353,6 +363,10 @@ def run_trajectory(stack, cfg, layer_weights, xs, refresh_flags=None, check=True
     prev_T = None
     n = len(xs) if next_input is None else n_steps
     out = None
+    if cfg.adaln and out_tol is None:
+        # The AdaLN residual stream is larger (one bf16 step above |8| is
+        # 0.0625): relative bounds only, globally and per token row.
+        out_tol = (1e-2, None)
     for t in range(n):
         # A sampler loop feeds each step's output through ``next_input``.
         x = xs[t] if next_input is None or t == 0 else next_input(t, out)
