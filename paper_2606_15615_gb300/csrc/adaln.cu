@@ -87,6 +87,14 @@ __global__ void __launch_bounds__(kModWarps * 32) ada_mod_kernel(AdaModArgs a) {
 constexpr int kLnWarps = 8;
 constexpr int kLnChunks = kAdaLnMaxD / 256;  // 16-byte chunks per lane
 
+// Eight floats from global or shared memory (a generic pointer: the row
+// pass reads the modulation vectors from either).
+__device__ __forceinline__ void load8(const float* p, float* v) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
 __device__ __forceinline__ void load8f(const float* p, float* v) {
   const float4 a = __ldg(reinterpret_cast<const float4*>(p));
   const float4 b = __ldg(reinterpret_cast<const float4*>(p) + 1);
@@ -142,8 +150,8 @@ __device__ __forceinline__ void store_modulated(const uint4* v, int nvec, int la
     if (c < nvec) {
       float f[8], sh[8], sc[8];
       unpack_vec(v[q], f, static_cast<__nv_bfloat16*>(nullptr));
-      load8f(shift + 8 * c, sh);
-      load8f(scale + 8 * c, sc);
+      load8(shift + 8 * c, sh);
+      load8(scale + 8 * c, sc);
 #pragma unroll
       for (int j = 0; j < 8; ++j) f[j] = fmaf((f[j] - mean) * rstd, 1.f + sc[j], sh[j]);
       const uint4 o = pack8(f);
@@ -153,27 +161,33 @@ __device__ __forceinline__ void store_modulated(const uint4* v, int nvec, int la
   }
 }
 
+// With every row (no list), a block's kLnWarps rows are consecutive tokens of
+// one sample (seq is a multiple of 8): the block stages that sample's first
+// five vectors (shift_a .. scale_m, 5D floats) in shared memory, loaded
+// together with the rows.  A listed-row launch reads them from L2 per row.
 __global__ void __launch_bounds__(kLnWarps * 32) adaln_rows_kernel(AdaLnArgs a) {
+  extern __shared__ __align__(16) float s_mod[];  // [5, D] when staged
   pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * kLnWarps + warp;
   const int n = a.rows ? *a.n_rows : a.T;
-  if (i >= n || i >= a.T) return;
-  const int t = a.rows ? a.rows[i] : i;
-  if (t < 0 || t >= a.T) {
-    if (lane == 0) report_status(a.status, kStatusBadIndex, 7000000 + i);
-    return;
-  }
+  const bool staged = a.rows == nullptr;
   const int D = a.D, nvec = D / 8;
-  const size_t off = static_cast<size_t>(t) * D;
-  const float* md = a.mod + static_cast<size_t>(t / a.seq) * 6 * D;
-  const uint4* x4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) + off);
-  __nv_bfloat16* u = static_cast<__nv_bfloat16*>(a.u) + off;
+  int t = -1;
+  if (i < n && i < a.T) {
+    t = a.rows ? a.rows[i] : i;
+    if (t < 0 || t >= a.T) {
+      if (lane == 0) report_status(a.status, kStatusBadIndex, 7000000 + i);
+      t = -1;
+    }
+  }
+  const size_t off = static_cast<size_t>(t < 0 ? 0 : t) * D;
   uint4 v[kLnChunks], av[kLnChunks];
   const uint4* a4 =
       a.a ? reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.a) + off) : nullptr;
-  if (a.h_out || a.a) {
-    // x and the cached attention row in flight together.
+  if (t >= 0 && (a.h_out || a4)) {
+    // x and the cached attention row in flight together (and with the staging below).
+    const uint4* x4 = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) + off);
 #pragma unroll
     for (int q = 0; q < kLnChunks; ++q)
       if (lane + 32 * q < nvec) v[q] = x4[lane + 32 * q];
@@ -183,6 +197,18 @@ __global__ void __launch_bounds__(kLnWarps * 32) adaln_rows_kernel(AdaLnArgs a) 
         if (lane + 32 * q < nvec) av[q] = a4[lane + 32 * q];
     }
   }
+  const int row0 = blockIdx.x * kLnWarps;
+  if (staged) {
+    if (row0 < a.T) {
+      const float4* src = reinterpret_cast<const float4*>(a.mod + static_cast<size_t>(row0 / a.seq) * 6 * D);
+      for (int j = threadIdx.x; j < 5 * D / 4; j += blockDim.x) reinterpret_cast<float4*>(s_mod)[j] = __ldg(src + j);
+    }
+    __syncthreads();
+  }
+  if (t < 0) return;
+  // The sample's vectors: shared when the block staged this row's sample, else global.
+  const float* md = staged && t / a.seq == row0 / a.seq ? s_mod : a.mod + static_cast<size_t>(t / a.seq) * 6 * D;
+  __nv_bfloat16* u = static_cast<__nv_bfloat16*>(a.u) + off;
   float mean, rstd;
   if (a.h_out) {
     row_stats(v, nvec, lane, D, a.eps, mean, rstd);
@@ -197,7 +223,7 @@ __global__ void __launch_bounds__(kLnWarps * 32) adaln_rows_kernel(AdaLnArgs a) 
         float xf[8], af[8], g[8];
         unpack_vec(v[q], xf, static_cast<__nv_bfloat16*>(nullptr));
         unpack_vec(av[q], af, static_cast<__nv_bfloat16*>(nullptr));
-        load8f(md + 2 * D + 8 * c, g);
+        load8(md + 2 * D + 8 * c, g);
 #pragma unroll
         for (int j = 0; j < 8; ++j) xf[j] = fmaf(g[j], af[j], xf[j]);
         v[q] = pack8(xf);
@@ -279,8 +305,15 @@ cudaError_t launch_ada_mod(const AdaModArgs& a, int n_sms, cudaStream_t s) {
 
 cudaError_t launch_adaln_rows(const AdaLnArgs& a, cudaStream_t s) {
   if (a.T <= 0) return cudaSuccess;
+  if (a.seq <= 0 || a.D % 64 || a.D > kAdaLnMaxD) return cudaErrorInvalidValue;
   const int grid = (a.T + kLnWarps - 1) / kLnWarps;
-  return launch_pdl(adaln_rows_kernel, dim3(grid), dim3(kLnWarps * 32), 0, s, a);
+  const size_t smem = a.rows ? 0 : static_cast<size_t>(5) * a.D * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(adaln_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  return launch_pdl(adaln_rows_kernel, dim3(grid), dim3(kLnWarps * 32), smem, s, a);
 }
 
 cudaError_t launch_ddpm(const DdpmArgs& a, cudaStream_t s) {
