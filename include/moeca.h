@@ -427,7 +427,8 @@ moeca_status moeca_ddpm_step(const moeca_ddpm_args* args, void* stream);
 
 const char* moeca_status_string(moeca_status s);
 /* Message of the last error on this handle ("" if none); NULL handle: the
- * last moeca_create() failure of this thread. */
+ * last failure of a call without a handle on this thread (moeca_create,
+ * moeca_ddpm_schedule, moeca_ddpm_step). */
 const char* moeca_last_error(const moeca_handle* h);
 
 #ifdef __cplusplus
