@@ -149,3 +149,17 @@ def test_planted_mistake_is_caught(name):
             np.testing.assert_allclose(m.expert_threshold(Hbar, g["tau0"], g["alpha"]), g["tau"], atol=1e-12)
     with pytest.raises(AssertionError):
         check(mutant)
+
+
+def test_golden_adaln_and_reverse_step():
+    """Hand-worked values of Eq. 1's reverse step and of AdaLN's layer
+    normalisation + modulation and SiLU (tests/golden/adaln_ddpm.json)."""
+    g = _load("adaln_ddpm.json")
+    d = g["ddpm"]
+    got = O.ddpm_step(d["x_t"], d["eps"], d["z"], d["alpha"], d["alpha_bar"], d["sigma"])
+    np.testing.assert_allclose(got, d["x_prev"], rtol=1e-14)
+    m = g["layer_norm_modulate"]
+    got = O.modulate(O.layer_norm(np.array([m["v"]]), m["eps"]), np.array(m["shift"]), np.array(m["scale"]))
+    np.testing.assert_allclose(got[0], m["out"], rtol=1e-14, atol=1e-15)
+    s = g["silu"]
+    np.testing.assert_allclose(O.silu(np.array(s["z"])), s["out"], rtol=1e-15, atol=0)
