@@ -256,3 +256,79 @@ def test_reverse_mean_equals_the_posterior_mean_given_the_true_noise():
 def test_noise_term_scales_with_sigma():
     got = O.ddpm_step(np.zeros(4), np.zeros(4), np.array([1.0, -2.0, 0.5, 0.0]), 0.9, 0.5, math.sqrt(0.1))
     np.testing.assert_allclose(got, math.sqrt(0.1) * np.array([1.0, -2.0, 0.5, 0.0]), rtol=1e-15)
+
+
+# --- planted mistakes: each must fail a pin above ----------------------------------
+
+def _mut_modulate_swapped(v, shift, scale):
+    return np.asarray(v, np.float64) * (1.0 + np.asarray(shift, np.float64)) + np.asarray(scale, np.float64)
+
+
+def _mut_ln_unbiased(v, eps):
+    v = np.asarray(v, np.float64)
+    mu = v.mean(axis=-1, keepdims=True)
+    var = ((v - mu) ** 2).sum(axis=-1, keepdims=True) / (v.shape[-1] - 1)
+    return (v - mu) / np.sqrt(var + eps)
+
+
+def _mut_ddpm_no_sqrt(x_t, eps, z, alpha_t, alpha_bar_t, sigma_t):
+    x_t = np.asarray(x_t, np.float64)
+    return (x_t - (1.0 - alpha_t) / (1.0 - alpha_bar_t) * np.asarray(eps, np.float64)) / math.sqrt(alpha_t) \
+        + sigma_t * np.asarray(z, np.float64)
+
+
+_REAL_RC = O.recompute_and_combine
+
+
+def _mut_gate_ignored(*args, resid=None, gate=None, **kw):
+    return _REAL_RC(*args, resid=resid, gate=None, **kw)
+
+
+_REAL_ATTN = O.attention
+
+
+def _mut_attention_on_raw_input(h, *args, **kw):
+    # An attention sub-layer that reads something other than the normalised,
+    # modulated h: here h rescaled and shifted, as the raw block input would be.
+    return _REAL_ATTN(np.asarray(h) * 3.0 + 1.0, *args, **kw)
+
+
+PLANTED = {
+    "shift_scale_swapped": ("modulate", _mut_modulate_swapped),
+    "unbiased_variance": ("layer_norm", _mut_ln_unbiased),
+    "gate_not_applied": ("recompute_and_combine", _mut_gate_ignored),
+    "attention_input_not_normalised": ("attention", _mut_attention_on_raw_input),
+    "eps_coefficient_without_sqrt": ("ddpm_step", _mut_ddpm_no_sqrt),
+}
+
+
+@pytest.mark.parametrize("name", list(PLANTED))
+def test_planted_mistake_fails_a_pin(name, monkeypatch):
+    attr, fn = PLANTED[name]
+    monkeypatch.setattr(O, attr, fn)
+    pins = [lambda: test_layer_norm_matches_torch_and_its_closed_form(),
+            lambda: test_full_step_matches_independent_torch_block(0),
+            lambda: test_new_gates_reach_reused_branches(),
+            lambda: test_reverse_mean_equals_the_posterior_mean_given_the_true_noise(),
+            lambda: test_golden_values()]
+    failed = 0
+    for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            failed += 1
+    assert failed >= 1, f"planted mistake {name} passed every pin"
+
+
+def test_golden_values():
+    """The hand-worked fixture (tests/golden/adaln_ddpm.json) through this module's view of the oracle."""
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "adaln_ddpm.json")) as f:
+        g = json.load(f)
+    d = g["ddpm"]
+    np.testing.assert_allclose(O.ddpm_step(d["x_t"], d["eps"], d["z"], d["alpha"], d["alpha_bar"], d["sigma"]),
+                               d["x_prev"], rtol=1e-14)
+    m = g["layer_norm_modulate"]
+    got = O.modulate(O.layer_norm(np.array([m["v"]]), m["eps"]), np.array(m["shift"]), np.array(m["scale"]))
+    np.testing.assert_allclose(got[0], m["out"], rtol=1e-14, atol=1e-15)
