@@ -336,6 +336,9 @@ class Stack:
         if cond is not None:
             if cond.dtype != torch.float32 or not cond.is_cuda or not cond.is_contiguous():
                 raise ValueError("cond must be a contiguous float32 CUDA tensor")
+            samples = T // (self.cfg.seq_len or T) if T else 0
+            if cond.numel() != samples * self.cfg.hidden:
+                raise ValueError(f"cond must hold {samples} x {self.cfg.hidden} values (one row per sample)")
             self._cond = cond  # read by the step's first kernel: keep it alive until then
         moeca_step(self.handle, x.data_ptr(), out.data_ptr(), T, step_index, force_refresh, tau0,
                    self.stream_ptr(), cond.data_ptr() if cond is not None else None)
