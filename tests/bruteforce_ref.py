@@ -29,17 +29,18 @@ def _ffn(u, w1, w2, form):
     return [sum(float(w2[d][f]) * mid[f] for f in range(F)) for d in range(D)]
 
 
-def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool):
+def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool, ffn_input=None, resid=None, gate=None):
     """state: dict of python lists {cache_e, cache_w, cache_norm, cache_h, shared_h, C}.
 
     C is indexed C[e][i] as in Eq. 10.  Returns (out, new_state, decisions).
+    x is the router input.  An AdaLN block passes ``ffn_input(rec)``, which
+    returns the FFN rows once the recompute sets are known (the sync rule
+    recomputes attention in between), and the output resid + gate * y.
     """
     T, D = len(x), len(x[0])
     E = len(wts["w_gate"])
     k = prm["top_k"]
     u = [[float(v) for v in row] for row in x]
-    # Dense: every expert on every token.
-    dense = [[_ffn(u[i], wts["w1"][e], wts["w2"][e], prm["gelu"]) for e in range(E)] for i in range(T)]
     # Routing by a full sort of (float32 logit desc, expert id asc).
     e_cur, w_cur = [], []
     for i in range(T):
@@ -125,6 +126,10 @@ def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool):
                     slot[i][p] = taken[p]
                 else:
                     slot[i][p] = free.pop(0)
+    # Dense: every expert on every token's FFN input.
+    if ffn_input is not None:
+        u = ffn_input(rec)
+    dense = [[_ffn(u[i], wts["w1"][e], wts["w2"][e], prm["gelu"]) for e in range(E)] for i in range(T)]
     # Cache update, shared experts, combine (Eq. 8) and norms.
     ce = [list(r) for r in state["cache_e"]]
     cw = [list(r) for r in state["cache_w"]]
@@ -156,7 +161,9 @@ def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool):
         if sh is not None:
             for d in range(D):
                 y[d] += sh[i][d]
-        out.append([u[i][d] + y[d] for d in range(D)])
+        base = u[i] if resid is None else resid[i]
+        g = [1.0] * D if gate is None else gate[i]
+        out.append([base[d] + g[d] * y[d] for d in range(D)])
     cn = [[math.sqrt(sum(v * v for v in ch[i][q])) for q in range(k)] for i in range(T)]
     new = dict(cache_e=ce, cache_w=cw, cache_norm=cn, cache_h=ch, shared_h=sh, C=C)
     dec = dict(e=e_cur, w=w_cur, recompute=rec, slot=slot, tau=tau)
@@ -169,3 +176,94 @@ def empty_state(T, D, E, k, n_shared):
                 cache_h=[[[0.0] * D for _ in range(k)] for _ in range(T)],
                 shared_h=[[0.0] * D for _ in range(T)] if n_shared else None,
                 C=[[0.0] * T for _ in range(E)])
+
+
+# ---------------------------------------------------------------------------
+# AdaLN DiT-MoE block (Sec. 3 residual form, Sec. 4.1 cache)
+# ---------------------------------------------------------------------------
+
+def _silu(z: float) -> float:
+    return z / (1.0 + math.exp(-z))
+
+
+def _layer_norm_mod(v, shift, scale, eps):
+    D = len(v)
+    mean = sum(v) / D
+    var = sum((a - mean) ** 2 for a in v) / D
+    r = 1.0 / math.sqrt(var + eps)
+    return [(v[d] - mean) * r * (1.0 + scale[d]) + shift[d] for d in range(D)]
+
+
+def _attention_row(hq, keys_h, wts, H):
+    """Attention output of one token over the rows keys_h of its sample."""
+    D = len(hq)
+    dh = D // H
+    wq, bq = wts["w_qkv"], wts.get("b_qkv")
+
+    def proj(row, r0):
+        return [sum(float(wq[r0 + j][d]) * row[d] for d in range(D)) + (float(bq[r0 + j]) if bq is not None else 0.0)
+                for j in range(D)]
+
+    q = proj(hq, 0)
+    ks = [proj(r, D) for r in keys_h]
+    vs = [proj(r, 2 * D) for r in keys_h]
+    A = [0.0] * D
+    for hd in range(H):
+        lo = hd * dh
+        sc = [sum(q[lo + j] * kr[lo + j] for j in range(dh)) / math.sqrt(dh) for kr in ks]
+        m = max(sc)
+        ex = [math.exp(v - m) for v in sc]
+        tot = sum(ex)
+        for n, vr in enumerate(vs):
+            for j in range(dh):
+                A[lo + j] += ex[n] / tot * vr[lo + j]
+    wo, bo = wts["w_o"], wts.get("b_o")
+    return [sum(float(wo[j][d]) * A[d] for d in range(D)) + (float(bo[j]) if bo is not None else 0.0)
+            for j in range(D)]
+
+
+def adaln_block_step(state: dict, x, cond, wts: dict, prm: dict, refresh: bool):
+    """One AdaLN block step; state adds attn_a [T][D].  prm adds n_heads,
+    seq_len, attn_policy ("sync" / "stale" / "full") and ln_eps.  Returns
+    (out, new_state, decisions) with decisions adding u, m and attn_rows."""
+    T, D = len(x), len(x[0])
+    S = prm["seq_len"] or T
+    eps = prm["ln_eps"]
+    x = [[float(v) for v in row] for row in x]
+    # Six modulation vectors per sample from SiLU(c).
+    mods = []
+    for b in range(len(cond)):
+        sc = [_silu(float(v)) for v in cond[b]]
+        row = [sum(float(wts["w_ada"][j][d]) * sc[d] for d in range(D))
+               + (float(wts["b_ada"][j]) if wts.get("b_ada") is not None else 0.0) for j in range(6 * D)]
+        mods.append([row[f * D:(f + 1) * D] for f in range(6)])
+    md = [mods[i // S] for i in range(T)]
+    h = [_layer_norm_mod(x[i], md[i][0], md[i][1], eps) for i in range(T)]
+
+    def attn(i):
+        b = i // S
+        return _attention_row(h[i], h[b * S:(b + 1) * S], wts, prm["n_heads"])
+
+    full = refresh or prm["attn_policy"] == "full"
+    a = [attn(i) for i in range(T)] if full else [list(r) for r in state["attn_a"]]
+    u = [[x[i][d] + md[i][2][d] * a[i][d] for d in range(D)] for i in range(T)]
+    m = [_layer_norm_mod(u[i], md[i][3], md[i][4], eps) for i in range(T)]
+    route_in = [list(r) for r in m]
+    rows = list(range(T)) if full else []
+
+    def ffn_input(rec):
+        if full or prm["attn_policy"] != "sync":
+            return m
+        for i in range(T):
+            if any(rec[i]):
+                rows.append(i)
+                a[i] = attn(i)
+                u[i] = [x[i][d] + md[i][2][d] * a[i][d] for d in range(D)]
+                m[i] = _layer_norm_mod(u[i], md[i][3], md[i][4], eps)
+        return m
+
+    out, new, dec = layer_step(state, route_in, wts, prm, refresh, ffn_input=ffn_input, resid=u,
+                               gate=[md[i][5] for i in range(T)])
+    new["attn_a"] = a
+    dec.update(u=u, m=m, attn_rows=rows)
+    return out, new, dec

@@ -80,3 +80,58 @@ def test_oracle_equals_bruteforce(case):
             kinds |= {("unmatched", bool(b)) for b in (~inf["matched"]).ravel()}
     if T > 1 and k < E:
         assert ("reuse", True) in kinds and ("unmatched", True) in kinds, kinds
+
+
+ADALN_CASES = [
+    # (seed, T, S, D, H, E, k, F, n_shared, policy, tau0)
+    (31, 8, 4, 8, 2, 4, 2, 5, 0, "sync", 0.75),
+    (32, 8, 4, 8, 2, 4, 2, 5, 1, "sync", 0.9),
+    (33, 6, 3, 6, 3, 3, 1, 4, 0, "stale", 1.4),  # k = 1: a matched score is 1 + lambda2
+    (34, 8, 8, 8, 2, 4, 2, 5, 0, "full", 0.75),
+]
+
+
+@pytest.mark.parametrize("case", ADALN_CASES, ids=[f"adaln{c[0]}" for c in ADALN_CASES])
+def test_adaln_block_equals_bruteforce(case):
+    """The oracle's AdaLN block (Sec. 3 residual form under the Sec. 4.1 cache)
+    against scalar loops: modulation, layer norm, per-head attention, the
+    sync rule's attention update and the gated combine, over 6 steps with the
+    conditioning changing every step."""
+    from paper_2606_15615_gb300.workloads import conditioning, tiny_adaln, tiny_attn
+    seed, T, S, D, H, E, k, F, n_sh, policy, tau0 = case
+    w, x0, rng = tiny_layer(seed, T, D, E, k, F, n_shared=n_sh, bias=True, wscale=0.6)
+    w.update(tiny_attn(seed, D, wscale=0.5))
+    w.update(tiny_adaln(seed, D, wscale=0.4))
+    prm = O.Params(top_k=k, tau0=tau0, refresh_period=4, n_heads=H, seq_len=S, attn_policy=policy, adaln=True)
+    st = O.Stack([w], prm, D, E, n_sh)
+    bprm = dict(_bf_params(prm), n_heads=H, seq_len=S, attn_policy=policy, ln_eps=prm.ln_eps)
+    bstate = BF.empty_state(T, D, E, k, n_sh)
+    bstate["attn_a"] = [[0.0] * D for _ in range(T)]
+    conds = conditioning(seed, T // S, D, 6)
+    wl = {kk: (None if v is None else v.tolist()) for kk, v in w.items()}
+    kinds = set()
+    x = x0
+    for t in range(6):
+        if t:
+            x = (x + 0.3 * rng.standard_normal(x.shape)).astype(np.float32)
+        refresh = st.is_refresh(t, T)
+        out, infos = st.step(x, t, cond=conds[t])
+        inf = infos[0]
+        bout, bstate, dec = BF.adaln_block_step(bstate, x.tolist(), conds[t].tolist(), wl, bprm, refresh)
+        assert inf["e"].tolist() == dec["e"]
+        assert inf["recompute"].tolist() == dec["recompute"]
+        assert inf["slot"].tolist() == dec["slot"]
+        assert sorted(inf["attn_rows"].tolist()) == sorted(dec["attn_rows"])
+        np.testing.assert_allclose(inf["u"], dec["u"], rtol=1e-11, atol=1e-12)
+        np.testing.assert_allclose(inf["m"], dec["m"], rtol=1e-11, atol=1e-12)
+        np.testing.assert_allclose(out, bout, rtol=1e-10, atol=1e-11)
+        s = st.states[0]
+        np.testing.assert_allclose(s.attn_a, bstate["attn_a"], rtol=1e-11, atol=1e-12)
+        np.testing.assert_allclose(s.cache_h, bstate["cache_h"], rtol=1e-10, atol=1e-12)
+        if not refresh:
+            kinds |= {("reuse", bool(b)) for b in (~inf["recompute"]).ravel()}
+            if policy == "sync":
+                kinds.add(("partial_attention", 0 < len(dec["attn_rows"]) < T))
+    assert ("reuse", True) in kinds and ("reuse", False) in kinds, kinds
+    if policy == "sync":
+        assert ("partial_attention", True) in kinds, kinds
