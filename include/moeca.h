@@ -119,7 +119,10 @@ typedef struct {
                                  The caches hold the ungated a and branch outputs, every step
                                  applies its own modulation, and under the sync rule the router
                                  sees m' from u' = x + gate_a a^{t0}.  moeca_step_args.cond then
-                                 carries c.  0 (default): no normalisation or modulation */
+                                 carries c.  bf16 only; hidden <= 2560; (max_tokens / seq_len) x
+                                 hidden x 4 bytes <= 200 KB (the staged conditioning), else
+                                 MOECA_ERR_UNSUPPORTED at create.  0 (default): no normalisation
+                                 or modulation */
   float ln_eps;               /* AdaLN layer-normalisation epsilon (default 1e-6) */
   int32_t keep_route_in;      /* 1: keep each AdaLN block's router input (m' on sync cache steps)
                                  for moeca_get_layer_trace, one more [T, D] write per layer;
@@ -166,8 +169,10 @@ typedef struct {
   int32_t force_refresh; /* 1: make this a full-computation step (Sec. 4.1)                 */
   float tau0_override;   /* NaN: use config tau0; otherwise the Eq. 12 base threshold now   */
   const float* cond;     /* adaln = 1: [n_tokens / seq_len, D] fp32 device, each sample's
-                            conditioning c (timestep + class embedding), read during the step;
-                            NULL otherwise */
+                            conditioning c (timestep + class embedding); caller-owned, read by
+                            the step's first kernel, so it must stay valid until the stream
+                            reaches it; NULL otherwise (an AdaLN stack refuses NULL with
+                            MOECA_ERR_INVALID_ARG before any launch) */
 } moeca_step_args;
 
 /* Branch counters, cumulative since create / moeca_reset_stats (Fig. 8 inputs). */
@@ -410,7 +415,11 @@ moeca_status moeca_ddpm_schedule(int32_t n_steps, int32_t n_train, double beta_s
  * `stream` (the current device).  x_prev may alias x_t; x_next (optional)
  * receives x_prev in eps_dtype, the next denoiser input.  n must be a
  * multiple of 8 and every pointer 16-byte aligned (INVALID_ARG otherwise);
- * z may be NULL only when sigma == 0.  The noise z is the caller's draw. */
+ * z may be NULL only when sigma == 0.  The noise z is the caller's draw.
+ * Every buffer is caller-owned device memory and must stay valid until the
+ * stream has run the update.  Errors: INVALID_ARG (checked on the host,
+ * nothing launched), CUDA (the launch failed); the message is in
+ * moeca_last_error(NULL). */
 typedef struct {
   int64_t n;             /* elements                                   */
   int32_t eps_dtype;     /* moeca_dtype of eps and x_next              */
