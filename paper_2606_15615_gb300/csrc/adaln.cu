@@ -101,6 +101,14 @@ __device__ __forceinline__ void load8f(const float* p, float* v) {
   v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 
+// Plain (coherent) loads, for a buffer the same kernel writes: the read-only
+// path above requires the data to stay unchanged for the kernel's duration.
+__device__ __forceinline__ void load8f_rw(const float* p, float* v) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0];
+  const float4 b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
 __device__ __forceinline__ uint4 pack8(const float* f) {
   uint4 v;
   __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&v);
@@ -252,7 +260,7 @@ __global__ void __launch_bounds__(kDdpmThreads) ddpm_kernel(DdpmArgs a) {
   for (long long c = static_cast<long long>(blockIdx.x) * kDdpmThreads + threadIdx.x; c < nv;
        c += static_cast<long long>(gridDim.x) * kDdpmThreads) {
     float x[8], e[8], z[8];
-    load8f(a.x_t + 8 * c, x);
+    load8f_rw(a.x_t + 8 * c, x);  // x_prev may alias x_t
     if constexpr (BF) {
       unpack_vec(__ldg(reinterpret_cast<const uint4*>(a.eps) + c), e, static_cast<__nv_bfloat16*>(nullptr));
     } else {
@@ -318,8 +326,13 @@ cudaError_t launch_adaln_rows(const AdaLnArgs& a, cudaStream_t s) {
 
 cudaError_t launch_ddpm(const DdpmArgs& a, cudaStream_t s) {
   if (a.n <= 0) return cudaSuccess;
+  int dev = 0, n_sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  // Grid-stride loop: eight 256-thread blocks per SM at most.
   long long blocks = (a.n / 8 + kDdpmThreads - 1) / kDdpmThreads;
-  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (blocks > 8LL * n_sms) blocks = 8LL * n_sms;
   if (a.bf16) return launch_pdl(ddpm_kernel<true>, dim3(static_cast<unsigned>(blocks)), dim3(kDdpmThreads), 0, s, a);
   return launch_pdl(ddpm_kernel<false>, dim3(static_cast<unsigned>(blocks)), dim3(kDdpmThreads), 0, s, a);
 }

@@ -4,7 +4,7 @@
 // bf16 operands, fp32 scores and accumulation, one pass over the keys with a
 // running maximum and sum (online softmax).
 //
-// One CTA per (128 query rows, sample, head), 6 warps:
+// One CTA per (128 query rows, sample, head), 10 warps (320 threads):
 //   warp 0    TMA producers: lane 0 loads the q tile once, then per block of
 //             128 keys the k block (K-major, 128-byte swizzle) into a ring of
 //             two or three, freed as soon as q k^T has read it; lane 1 loads
@@ -19,10 +19,10 @@
 //             two halves of a row exchange their maxima through shared
 //             memory and a bounded barrier.  Per thread:
 //             reads S_j from TMEM (tcgen05.ld), keeps the row maximum m in
-//             base 2, rescales the O row in TMEM only when m rises
-//             (tcgen05.ld / st), writes P_j = 2^(s - m) in bf16 into shared
-//             memory in the 128-byte-swizzle K-major layout the MMA reads as
-//             its A operand, and at the end writes o = O / l.
+//             base 2, rescales the O row in TMEM only when m rises by more
+//             than 2^8 (tcgen05.ld / st), writes P_j = 2^(s - m) in bf16 back
+//             into S_j's own TMEM columns (two values per column), where p v
+//             reads it as its A operand, and at the end writes o = O / l.
 // The row sum l comes from the tensor core: each v^T tile carries one more
 // channel row of ones (and 15 rows of zeros to keep N a multiple of 16), so
 // O's column DKP accumulates sum_k P[k], from the same rounded P as O and

@@ -16,6 +16,12 @@ enum StatIndex {
   kStNearRoute, kStNearScore, kStAttnRows, kStCount
 };
 
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize, bytes) for `func` on the
+// current device, once per (device, kernel) unless a larger value is asked
+// for: the attribute belongs to the kernel on each device, so a process that
+// uses several devices sets it on each.  Thread-safe.
+cudaError_t set_dyn_smem_on_device(const void* func, int bytes);
+
 constexpr int kMaxExperts = 64;
 constexpr int kMaxTopK = 8;
 constexpr int kRouterTokensPerBlock = 16;   // 8 warps x 2 tokens

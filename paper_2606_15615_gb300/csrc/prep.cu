@@ -1,5 +1,6 @@
-// Fused per-layer preparation of the branch-cached MoE layer, one cooperative
-// launch with two grid barriers:
+// Fused per-layer preparation of the branch-cached MoE layer, one launch
+// (programmatic dependent launch, every block co-resident) with two grid
+// barriers:
 //
 //   A  router (Eq. 7): gate logits on the tensor cores (mma.sync m16n8k16,
 //      bf16 in, fp32 accumulate) from the block's token rows and the gate
@@ -54,7 +55,7 @@ __device__ __forceinline__ float grp_sum(float v) {
   return v;
 }
 
-// Grid-wide barrier over co-resident blocks (cooperative launch).  *cnt only
+// Grid-wide barrier over co-resident blocks (see prep_launch).  *cnt only
 // grows: barrier b (0 or 1) of a launch is passed once it reaches
 // base + (b + 1) * nblocks arrivals, base being the arrivals of all earlier
 // launches (kept by the host).  Arrive is a release add, the wait an
@@ -675,13 +676,8 @@ size_t prep_smem(int D, int n_blocks, int G, bool attn) {  // G: groups of the c
 
 template <int TB, int EPAD, int KMAX>
 cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(prep_kernel<TB, EPAD, KMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kPrepSmemMax);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  cudaError_t e = set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX>), kPrepSmemMax);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(n_blocks);
   cfg.blockDim = dim3(kThreads);
@@ -705,14 +701,10 @@ cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream
 
 template <int TB, int EPAD, int KMAX>
 int prep_occupancy(size_t smem) {
-  static bool configured = false;
-  if (!configured) {
-    if (cudaFuncSetAttribute(prep_kernel<TB, EPAD, KMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPrepSmemMax) !=
-        cudaSuccess) {
-      cudaGetLastError();
-      return 0;
-    }
-    configured = true;
+  if (set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX>), kPrepSmemMax) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return 0;
   }
   int n = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD, KMAX>, kThreads, smem) != cudaSuccess) {

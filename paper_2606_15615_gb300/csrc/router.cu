@@ -373,17 +373,14 @@ constexpr size_t kSmemPerBlock = 227 * 1024;
 template <typename TI, int G, int EPL, int NT>
 cudaError_t launch_g(const RouterArgs& a, cudaStream_t s) {
   constexpr int TB = NT / G;
-  static size_t cap = 0;  // per instantiation, set on first use
-  if (cap == 0) {
-    cudaFuncAttributes attr;
-    cudaError_t e = cudaFuncGetAttributes(&attr, router_kernel<TI, G, EPL, NT>);
-    if (e != cudaSuccess) return e;
-    const size_t c = kSmemPerBlock - attr.sharedSizeBytes - 1024;
-    e = cudaFuncSetAttribute(router_kernel<TI, G, EPL, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(c));
-    if (e != cudaSuccess) return e;
-    cap = c;
-  }
+  // The staging cap depends on the kernel's static shared memory only; the
+  // attribute that allows it is set on every device the process uses.
+  cudaFuncAttributes attr;
+  cudaError_t e = cudaFuncGetAttributes(&attr, router_kernel<TI, G, EPL, NT>);
+  if (e != cudaSuccess) return e;
+  const size_t cap = kSmemPerBlock - attr.sharedSizeBytes - 1024;
+  e = set_dyn_smem_on_device(reinterpret_cast<const void*>(router_kernel<TI, G, EPL, NT>), static_cast<int>(cap));
+  if (e != cudaSuccess) return e;
   const int grid = (a.T + TB - 1) / TB;
   const size_t row = static_cast<size_t>(a.D / Elem<TI>::kVec + 1) * 16;
   const size_t epad = (a.E + 7) / 8 * 8;
