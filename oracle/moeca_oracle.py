@@ -42,6 +42,11 @@ Readings where the paper is silent (each is a switch in ``Params``):
     ("overwrite");
   * shared experts are recomputed on full-computation steps and for tokens
     with a non-empty recompute set ("sync"), or always ("always");
+  * Eq. 8 forms every token's output from its branches with the current
+    gate weights w^t ("current"); Sec. 4.1's other wording, that a token
+    with an empty recompute set reuses its cached state, is the "copy"
+    reading: such a token takes its last computed MoE output y^{t0}
+    unchanged (``token_reuse_policy``);
   * GELU is the tanh form ("tanh") or the erf form ("erf"); experts have no bias.
   * a DiT block (n_heads > 0) is x -> u = x + Attn(x) -> u + MoE(u), without
     normalisation or modulation; attention is multi-head self-attention over
@@ -101,6 +106,7 @@ class Params:
     act_store: str = "f64"             # or "bf16": storage rounding of the block's a and u
     adaln: bool = False                # DiT block with AdaLN modulation of both sub-layers (Sec. 3)
     ln_eps: float = 1e-6               # layer-normalisation epsilon of the AdaLN block
+    token_reuse_policy: str = "current"  # or "copy": R_i empty => y_i = y_i^{t0} (Sec. 4.1)
 
 
 # ---------------------------------------------------------------------------
@@ -383,6 +389,7 @@ class LayerState:
     C: np.ndarray              # [E, T] float64 C_{e,i}
     valid: bool = False
     attn_a: np.ndarray | None = None  # [T, D] float64 a_i^{t0} of a DiT block (Sec. 4.1)
+    cache_y: np.ndarray | None = None  # [T, D] float64 y_i^{t0}, the token's last MoE output (ungated)
 
     @staticmethod
     def empty(T: int, D: int, E: int, k: int, n_shared: int, attention: bool = False) -> "LayerState":
@@ -390,12 +397,13 @@ class LayerState:
             cache_e=np.full((T, k), -1, np.int32), cache_w=np.zeros((T, k)),
             cache_norm=np.zeros((T, k)), cache_h=np.zeros((T, k, D)),
             shared_h=np.zeros((T, D)) if n_shared else None, C=np.zeros((E, T)), valid=False,
-            attn_a=np.zeros((T, D)) if attention else None)
+            attn_a=np.zeros((T, D)) if attention else None, cache_y=np.zeros((T, D)))
 
     def copy(self) -> "LayerState":
         return LayerState(self.cache_e.copy(), self.cache_w.copy(), self.cache_norm.copy(),
                           self.cache_h.copy(), None if self.shared_h is None else self.shared_h.copy(),
-                          self.C.copy(), self.valid, None if self.attn_a is None else self.attn_a.copy())
+                          self.C.copy(), self.valid, None if self.attn_a is None else self.attn_a.copy(),
+                          None if self.cache_y is None else self.cache_y.copy())
 
 
 def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, slot, weights: dict,
@@ -410,6 +418,11 @@ def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, s
 
     ``resid`` and ``gate`` ([T, D], or None) give the AdaLN block's output
     resid + gate * y (Sec. 3 residual form) instead of u + y.
+
+    Under ``token_reuse_policy`` "copy", a token with an empty recompute set
+    on a cache step takes y_i = y_i^{t0}, its MoE output of the last step it
+    computed one (Sec. 4.1, "reuse cached states"), in place of Eq. 8 with
+    the current weights.  The new state keeps every token's y (ungated).
     """
     u = np.asarray(u, np.float64)
     T, D = u.shape
@@ -447,6 +460,14 @@ def recompute_and_combine(state: LayerState, u: np.ndarray, e_cur, w_cur, rec, s
         y += np.asarray(w_cur, np.float64)[:, p:p + 1] * new.cache_h[np.arange(T), slot[:, p]]
     if new.shared_h is not None:
         y += new.shared_h
+    if prm.token_reuse_policy == "copy" and not refresh:
+        if state.cache_y is None:
+            raise ValueError("the copy reading needs the cached outputs y^{t0}")
+        keep = ~token_any
+        y[keep] = state.cache_y[keep]
+    elif prm.token_reuse_policy not in ("current", "copy"):
+        raise ValueError(prm.token_reuse_policy)
+    new.cache_y = y.copy()
     if gate is not None:
         y = np.asarray(gate, np.float64) * y
     out = (u if resid is None else np.asarray(resid, np.float64)) + y

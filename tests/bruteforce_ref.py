@@ -152,6 +152,8 @@ def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool, ffn_input=No
                     hs = _ffn(u[i], wts["ws1"][s], wts["ws2"][s], prm["gelu"])
                     sh[i] = [a + b for a, b in zip(sh[i], hs)]
     out = []
+    ys = []
+    copy = prm.get("token_reuse_policy", "current") == "copy" and not refresh
     for i in range(T):
         y = [0.0] * D
         for p in range(k):
@@ -161,11 +163,15 @@ def layer_step(state: dict, x, wts: dict, prm: dict, refresh: bool, ffn_input=No
         if sh is not None:
             for d in range(D):
                 y[d] += sh[i][d]
+        if copy and not any(rec[i]):
+            # Sec. 4.1 "reuse cached states": the token's last MoE output.
+            y = list(state["cache_y"][i])
+        ys.append(y)
         base = u[i] if resid is None else resid[i]
         g = [1.0] * D if gate is None else gate[i]
         out.append([base[d] + g[d] * y[d] for d in range(D)])
     cn = [[math.sqrt(sum(v * v for v in ch[i][q])) for q in range(k)] for i in range(T)]
-    new = dict(cache_e=ce, cache_w=cw, cache_norm=cn, cache_h=ch, shared_h=sh, C=C)
+    new = dict(cache_e=ce, cache_w=cw, cache_norm=cn, cache_h=ch, shared_h=sh, C=C, cache_y=ys)
     dec = dict(e=e_cur, w=w_cur, recompute=rec, slot=slot, tau=tau)
     return out, new, dec
 
@@ -175,7 +181,7 @@ def empty_state(T, D, E, k, n_shared):
                 cache_norm=[[0.0] * k for _ in range(T)],
                 cache_h=[[[0.0] * D for _ in range(k)] for _ in range(T)],
                 shared_h=[[0.0] * D for _ in range(T)] if n_shared else None,
-                C=[[0.0] * T for _ in range(E)])
+                C=[[0.0] * T for _ in range(E)], cache_y=[[0.0] * D for _ in range(T)])
 
 
 # ---------------------------------------------------------------------------

@@ -32,6 +32,10 @@ CASES = [
     (15, 8, 6, 4, 2, 5, 0, False, {"score_terms": 6, "tau0": 0.3}),
     (16, 8, 6, 4, 2, 5, 1, False, {"granularity": "token", "tau0": 1.1}),
     (17, 8, 5, 4, 3, 4, 0, True, {"granularity": "token", "score_terms": 3, "tau0": 0.9}),
+    # Sec. 4.1's "reuse cached states" reading: R_i empty => y_i^{t0} copied
+    (19, 8, 6, 4, 2, 5, 0, False, {"token_reuse_policy": "copy", "tau0": 1.1}),
+    (20, 8, 5, 4, 2, 4, 1, True, {"token_reuse_policy": "copy", "tau0": 1.3}),
+    (21, 8, 6, 4, 2, 5, 0, False, {"token_reuse_policy": "copy", "granularity": "token", "tau0": 1.2}),
 ]
 
 
@@ -40,7 +44,7 @@ def _bf_params(prm: O.Params) -> dict:
                 alpha=prm.alpha, beta=prm.beta, renorm_topk=prm.renorm_topk,
                 entropy_norm=prm.entropy_norm, shared_policy=prm.shared_policy,
                 reused_meta_policy=prm.reused_meta_policy, gelu=prm.gelu, score_terms=prm.score_terms,
-                granularity=prm.granularity)
+                granularity=prm.granularity, token_reuse_policy=prm.token_reuse_policy)
 
 
 @pytest.mark.parametrize("case", CASES, ids=[f"case{c[0]}" for c in CASES])
@@ -75,11 +79,15 @@ def test_oracle_equals_bruteforce(case):
         np.testing.assert_allclose(s.cache_h, bstate["cache_h"], rtol=1e-11, atol=1e-13)
         if S:
             np.testing.assert_allclose(s.shared_h, bstate["shared_h"], rtol=1e-11, atol=1e-13)
+        np.testing.assert_allclose(s.cache_y, bstate["cache_y"], rtol=1e-11, atol=1e-13)
         if not refresh:
             kinds |= {("reuse", bool(b)) for b in (~inf["recompute"]).ravel()}
             kinds |= {("unmatched", bool(b)) for b in (~inf["matched"]).ravel()}
+            kinds |= {("token_reused", bool(b)) for b in (~inf["recompute"].any(axis=1))}
     if T > 1 and k < E:
         assert ("reuse", True) in kinds and ("unmatched", True) in kinds, kinds
+    if prm.token_reuse_policy == "copy":
+        assert ("token_reused", True) in kinds and ("token_reused", False) in kinds, kinds
 
 
 ADALN_CASES = [
@@ -88,6 +96,7 @@ ADALN_CASES = [
     (32, 8, 4, 8, 2, 4, 2, 5, 1, "sync", 0.9),
     (33, 6, 3, 6, 3, 3, 1, 4, 0, "stale", 1.4),  # k = 1: a matched score is 1 + lambda2
     (34, 8, 8, 8, 2, 4, 2, 5, 0, "full", 0.75),
+    (35, 8, 4, 8, 2, 4, 2, 5, 1, "sync", 1.2, "copy"),  # Sec. 4.1 "reuse cached states" reading
 ]
 
 
@@ -98,11 +107,13 @@ def test_adaln_block_equals_bruteforce(case):
     sync rule's attention update and the gated combine, over 6 steps with the
     conditioning changing every step."""
     from paper_2606_15615_gb300.workloads import conditioning, tiny_adaln, tiny_attn
-    seed, T, S, D, H, E, k, F, n_sh, policy, tau0 = case
+    seed, T, S, D, H, E, k, F, n_sh, policy, tau0 = case[:11]
+    reuse = case[11] if len(case) > 11 else "current"
     w, x0, rng = tiny_layer(seed, T, D, E, k, F, n_shared=n_sh, bias=True, wscale=0.6)
     w.update(tiny_attn(seed, D, wscale=0.5))
     w.update(tiny_adaln(seed, D, wscale=0.4))
-    prm = O.Params(top_k=k, tau0=tau0, refresh_period=4, n_heads=H, seq_len=S, attn_policy=policy, adaln=True)
+    prm = O.Params(top_k=k, tau0=tau0, refresh_period=4, n_heads=H, seq_len=S, attn_policy=policy, adaln=True,
+                   token_reuse_policy=reuse)
     st = O.Stack([w], prm, D, E, n_sh)
     bprm = dict(_bf_params(prm), n_heads=H, seq_len=S, attn_policy=policy, ln_eps=prm.ln_eps)
     bstate = BF.empty_state(T, D, E, k, n_sh)
@@ -132,6 +143,9 @@ def test_adaln_block_equals_bruteforce(case):
             kinds |= {("reuse", bool(b)) for b in (~inf["recompute"]).ravel()}
             if policy == "sync":
                 kinds.add(("partial_attention", 0 < len(dec["attn_rows"]) < T))
+            kinds |= {("token_reused", not any(r)) for r in dec["recompute"]}
     assert ("reuse", True) in kinds and ("reuse", False) in kinds, kinds
+    if reuse == "copy":
+        assert ("token_reused", True) in kinds, kinds
     if policy == "sync":
         assert ("partial_attention", True) in kinds, kinds

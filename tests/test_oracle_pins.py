@@ -336,3 +336,65 @@ def test_token_granularity_never_reuses_more_than_branch_granularity():
                                granularity="token")
         assert tk["recompute"].sum() >= br["recompute"].sum()
         assert np.all(tk["recompute"] | ~br["recompute"])
+
+
+# --- Token-level reuse reading of Sec. 4.1 ("reuse cached states") ----------
+
+def _textbook_y(x, w, k):
+    return textbook_moe(x, w, k) - x.astype(np.float64)
+
+
+def test_copy_reading_returns_the_last_computed_output_exactly():
+    """Under the "copy" reading a token with an empty recompute set returns
+    y^{t0}: its MoE output of the last step it computed one, here the full
+    step, which is the textbook Eq. 5 value.  The default reading (Eq. 8)
+    instead recombines the cached branches with the current weights."""
+    w, x0, rng = tiny_layer(40, T=48, D=16, E=5, k=2, F=10, n_shared=1, bias=True)
+    x1 = (x0 + 0.3 * rng.standard_normal(x0.shape)).astype(np.float32)
+    x2 = (x1 + 0.1 * rng.standard_normal(x0.shape)).astype(np.float32)
+    y0 = _textbook_y(x0, w, 2)
+    cur = O.Params(top_k=2, tau0=math.inf)
+    cpy = O.Params(top_k=2, tau0=math.inf, token_reuse_policy="copy")
+    outs_c, infos_c, _ = _run(w, cpy, [x0, x1, x2], n_shared=1)
+    outs_d, infos_d, _ = _run(w, cur, [x0, x1, x2], n_shared=1)
+    for t in (1, 2):
+        assert np.array_equal(infos_c[t]["recompute"], infos_d[t]["recompute"]), "decisions do not depend on it"
+    kept1 = ~infos_c[1]["recompute"].any(axis=1)
+    kept12 = kept1 & ~infos_c[2]["recompute"].any(axis=1)
+    assert kept1.sum() >= 10 and kept12.sum() >= 5 and (~kept1).sum() >= 3
+    # Reused for one and for two steps: still the full step's y, bit for bit
+    # the oracle's, and equal to the textbook value.
+    np.testing.assert_allclose(outs_c[1][kept1] - x1[kept1], y0[kept1], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(outs_c[2][kept12] - x2[kept12], y0[kept12], rtol=1e-12, atol=1e-12)
+    # The current-weight reading differs on those tokens (the weights moved).
+    assert np.abs((outs_d[1] - outs_c[1])[kept1]).max() > 1e-6
+    # Tokens that computed on step 1 agree under both readings.
+    np.testing.assert_array_equal(outs_c[1][~kept1], outs_d[1][~kept1])
+
+
+def test_copy_reading_after_a_recompute_keeps_the_new_output():
+    """A token that recomputes at step 1 and is reused at step 2 returns its
+    step-1 output, not the full step's: y^{t0} follows the last computation."""
+    w, x0, rng = tiny_layer(41, T=64, D=12, E=4, k=2, F=8)
+    prm = O.Params(top_k=2, tau0=0.62, token_reuse_policy="copy")
+    xs = [x0]
+    for _ in range(2):
+        xs.append((xs[-1] + 0.2 * rng.standard_normal(x0.shape)).astype(np.float32))
+    outs, infos, _ = _run(w, prm, xs)
+    comp1 = infos[1]["recompute"].any(axis=1)
+    kept2 = ~infos[2]["recompute"].any(axis=1)
+    both = comp1 & kept2
+    assert both.sum() >= 3
+    y1 = outs[1] - xs[1].astype(np.float64)
+    np.testing.assert_allclose((outs[2] - xs[2].astype(np.float64))[both], y1[both], rtol=1e-12, atol=1e-15)
+    assert np.abs(y1[both] - _textbook_y(xs[0], w, 2)[both]).max() > 1e-9
+
+
+def test_copy_reading_equals_default_when_nothing_is_reused():
+    w, x0, rng = tiny_layer(42, T=32, D=8, E=4, k=2, F=6)
+    xs = [x0, (x0 + 0.3 * rng.standard_normal(x0.shape)).astype(np.float32)]
+    a, _, _ = _run(w, O.Params(top_k=2, tau0=-math.inf, token_reuse_policy="copy"), xs)
+    b, _, _ = _run(w, O.Params(top_k=2, tau0=-math.inf), xs)
+    for oa, ob, x in zip(a, b, xs):
+        np.testing.assert_array_equal(oa, ob)
+        np.testing.assert_allclose(oa, textbook_moe(x, w, 2), rtol=1e-12, atol=1e-12)
