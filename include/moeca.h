@@ -127,6 +127,13 @@ typedef struct {
   int32_t keep_route_in;      /* 1: keep each AdaLN block's router input (m' on sync cache steps)
                                  for moeca_get_layer_trace, one more [T, D] write per layer;
                                  0 (default) */
+  int32_t token_reuse_policy; /* what a token whose recompute set R_i is empty returns on a cache
+                                 step: 0 (default) = Eq. 8, its cached branch outputs combined with
+                                 the current gate weights w^t; 1 = Sec. 4.1's "reuse cached states"
+                                 read at token level: its last computed MoE output y^{t0} (routed
+                                 branches and shared expert, before the AdaLN gate) unchanged.
+                                 1 keeps y for every token: one [T, D] fp32 buffer per layer
+                                 (moeca_layer_state.cache_y), written by every token that computes */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters
@@ -195,14 +202,17 @@ typedef struct {
 
 /* Caller-owned DEVICE buffers for one layer's cached state, T rows each.
  * Any pointer may be NULL in moeca_get_layer_state (that field is skipped);
- * moeca_set_layer_state needs all of them (shared_h only when n_shared == 1).
+ * moeca_set_layer_state needs all of them (shared_h only when n_shared == 1,
+ * attn_a only when n_heads > 0, cache_y only when token_reuse_policy == 1).
  *   cache_e [T, k] int32   cached expert ids e^{t0}        (Eq. 7)
  *   cache_w [T, k] fp32    cached gate weights w^{t0}      (Eq. 7)
  *   cache_norm [T, k] fp32 ||h^{t0}|| over D                (Eq. 9, o)
  *   cache_h [T, k, D] dtype cached branch outputs h^{t0}    (Eq. 7)
  *   shared_h [T, D] dtype  cached shared-expert output      (Eq. 6)
  *   ema [T, E] fp32        C_{e,i} stored at [i * E + e]     (Eq. 10)
- *   attn_a [T, D] dtype    cached attention output a^{t0}   (Sec. 4.1; n_heads > 0) */
+ *   attn_a [T, D] dtype    cached attention output a^{t0}   (Sec. 4.1; n_heads > 0)
+ *   cache_y [T, D] fp32    each token's last computed MoE output y^{t0}, before the AdaLN
+ *                          gate (token_reuse_policy = 1; ignored otherwise) */
 typedef struct {
   int32_t* cache_e;
   float* cache_w;
@@ -211,6 +221,7 @@ typedef struct {
   void* shared_h;
   float* ema;
   void* attn_a;
+  float* cache_y;
 } moeca_layer_state;
 
 /* Caller-owned DEVICE buffers for what one layer computed on the last step.
@@ -293,6 +304,31 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
  * CUDA (launch failure). */
 moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out,
                         const moeca_step_args* args, void* stream);
+
+/* One step from and to HOST buffers: the serving form of moeca_step.
+ * x_in_host [T, D] and x_out_host [T, D] are host memory in the config dtype
+ * (page-locked memory makes the copies asynchronous; pageable memory works
+ * but each copy then blocks the calling thread); args->cond, when the stack
+ * is AdaLN, is a HOST pointer to [T / seq_len, D] fp32 here.  The library
+ * uploads the input (and cond) into one of two device staging buffers on its
+ * own upload stream, runs moeca_step on `stream`, and reads the output back
+ * on its own read-back stream, so the upload of the next call and the
+ * read-back of this one overlap the neighbouring steps' compute.
+ * Asynchronous: x_out_host is written once the read-back has run; call
+ * moeca_host_join(h, stream) and then synchronise `stream` (or an event
+ * recorded on it after the join) before reading it.  The caller keeps
+ * x_in_host and cond unchanged, and x_out_host alive, until then.
+ * The first call allocates the staging buffers (4 x max_tokens x D elements,
+ * plus the conditioning) and the two copy streams: make it before any stream
+ * capture.  Errors: as moeca_step, plus OOM / CUDA from that first call. */
+moeca_status moeca_step_host(moeca_handle* h, const void* x_in_host, void* x_out_host,
+                             const moeca_step_args* args, void* stream);
+
+/* Make `stream` wait for every upload and read-back that earlier
+ * moeca_step_host calls enqueued: work enqueued on `stream` afterwards (an
+ * event, a synchronisation) comes after the last output reached host memory.
+ * No-op when moeca_step_host was never called. */
+moeca_status moeca_host_join(moeca_handle* h, void* stream);
 
 /* Copy the counters of `layer` (or the sum over layers for layer = -1) into
  * *out.  Synchronises the device. */

@@ -7,6 +7,10 @@
 //   out_i = x_i + g_i * y_i      in an AdaLN block (g the sample's MoE gate, Sec. 3)
 //   cache_norm[i, q] = ||cache_h[i, q]||_2 for every slot q (slot is a
 //   permutation of 0..k-1, so the k rows read are all of the token's slots).
+// Under the token-level reading of Sec. 4.1 (token_reuse_policy 1) every
+// computing token also stores its y in fp32, and on a cache step a token
+// whose recompute set is empty takes y from there instead (its cache rows
+// and norms are unchanged, so they are not read).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -17,7 +21,7 @@ constexpr int kWarps = 8;
 
 // CG 16-byte chunks per lane are in flight at once (all k cache rows, the
 // shared row and x loaded before any arithmetic).
-template <typename TI, int KMAX, int CG, bool GATED>
+template <typename TI, int KMAX, int CG, bool GATED, bool YC>
 __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -61,10 +65,37 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
     const int c = g * 32 + lane;
     if (c < nvec) x_first[g] = x4[c];
   }
+  // token_any comes from the preparation kernel, which completed before the
+  // previous kernel passed its own dependency wait.
+  const bool copy_tok = YC && a.copy_y && !a.token_any[i];
   pdl_entry();
   if (bad) {
     if (lane == 0) report_status(a.status, kStatusBadIndex, 3000000 + i);
     return;
+  }
+  if constexpr (YC) {
+    if (copy_tok) {
+      // Sec. 4.1, token level: y = y^{t0}, read back in fp32.
+      const float4* yc = reinterpret_cast<const float4*>(a.cache_y + static_cast<size_t>(i) * D);
+      for (int c = lane; c < nvec; c += 32) {
+        float xs[V], y[V];
+#pragma unroll
+        for (int j = 0; j < V / 4; ++j) {
+          const float4 v = yc[static_cast<size_t>(c) * (V / 4) + j];
+          y[4 * j] = v.x; y[4 * j + 1] = v.y; y[4 * j + 2] = v.z; y[4 * j + 3] = v.w;
+        }
+        unpack_vec(x4[c], xs, static_cast<TI*>(nullptr));
+        if constexpr (GATED) {
+#pragma unroll
+          for (int j = 0; j < V; ++j) xs[j] = fmaf(gr[c * V + j], y[j], xs[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < V; ++j) xs[j] += y[j];
+        }
+        store_vec(out + c * V, xs);
+      }
+      return;
+    }
   }
   float ss[KMAX];
 #pragma unroll
@@ -115,6 +146,11 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
 #pragma unroll
           for (int j = 0; j < V; ++j) y[j] += hv[j];
         }
+        if constexpr (YC) {
+          float4* yo = reinterpret_cast<float4*>(a.cache_y + static_cast<size_t>(i) * D) + static_cast<size_t>(c) * (V / 4);
+#pragma unroll
+          for (int j = 0; j < V / 4; ++j) yo[j] = make_float4(y[4 * j], y[4 * j + 1], y[4 * j + 2], y[4 * j + 3]);
+        }
         float xs[V];
         unpack_vec(xr[g], xs, static_cast<TI*>(nullptr));
         if constexpr (GATED) {
@@ -138,22 +174,29 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   }
 }
 
-template <typename TI, bool GATED>
+template <typename TI, bool GATED, bool YC>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
   // The gated form holds the gate values with the rows: half the chunks in flight keeps it near 128 registers.
-  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, GATED ? 2 : 4, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else launch_pdl(combine_kernel<TI, 8, 1, GATED>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, GATED ? 2 : 4, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else launch_pdl(combine_kernel<TI, 8, 1, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+}
+
+template <bool YC>
+void launch_y(const CombineArgs& a, bool bf16, cudaStream_t s) {
+  if (bf16 && a.gate) launch_t<__nv_bfloat16, true, YC>(a, s);
+  else if (bf16) launch_t<__nv_bfloat16, false, YC>(a, s);
+  else launch_t<float, false, YC>(a, s);
 }
 
 }  // namespace
 
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s) {
   if (a.gate && !bf16) return cudaErrorInvalidValue;  // AdaLN blocks are bf16 only
-  if (bf16 && a.gate) launch_t<__nv_bfloat16, true>(a, s);
-  else if (bf16) launch_t<__nv_bfloat16, false>(a, s);
-  else launch_t<float, false>(a, s);
+  if (a.cache_y && (!a.token_any || reinterpret_cast<uintptr_t>(a.cache_y) % 16)) return cudaErrorInvalidValue;
+  if (a.cache_y) launch_y<true>(a, bf16, s);
+  else launch_y<false>(a, bf16, s);
   return cudaGetLastError();
 }
 

@@ -209,6 +209,10 @@ struct CombineArgs {
                           // ticket), set to 0 after the dependency wait, or null
   const float* gate;      // AdaLN block (bf16): out = x + gate * y, gate row of token i at
   int gate_ld, seq;       //   gate + (i / seq) * gate_ld; null: out = x + y
+  float* cache_y;         // [T, D] fp32 last computed y per token (token_reuse_policy 1), or null
+  const uint8_t* token_any;  // [T] recompute set non-empty (with cache_y)
+  int copy_y;             // 1: a token with token_any 0 takes y = cache_y (a cache step under
+                          //   token_reuse_policy 1); 0: every token computes y (and stores it)
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);

@@ -96,6 +96,7 @@ struct LayerBuf {
   void* attn_u = nullptr;    // [T, D] MoE sub-layer input u of the last step (AdaLN: the residual u)
   void* attn_m = nullptr;    // [T, D] AdaLN block: the MoE input m of the last step
   void* route_m = nullptr;   // [T, D] AdaLN block: its router input (keep_route_in)
+  float* cache_y = nullptr;  // [T, D] fp32 each token's last computed MoE output (token_reuse_policy 1)
   TcPlan* tc = nullptr;
   bool valid = false;
 };
@@ -151,6 +152,17 @@ struct moeca_handle {
   const void* last_x_in = nullptr;
   std::string last_error;
   std::vector<void*> allocs;
+  // moeca_step_host: double-buffered device staging, an upload and a
+  // read-back stream, and the events that order them against the steps.
+  struct HostIo {
+    bool ready = false;
+    void* in[2] = {nullptr, nullptr};
+    void* out[2] = {nullptr, nullptr};
+    float* cond[2] = {nullptr, nullptr};
+    cudaStream_t up_stream = nullptr, back_stream = nullptr;
+    cudaEvent_t up[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr}, back[2] = {nullptr, nullptr};
+    long long calls = 0;
+  } hio;
   bool timing = false;
   std::vector<cudaEvent_t> event_pool;
   std::vector<PendingTiming> pending;
@@ -185,6 +197,17 @@ bool dev_alloc(moeca_handle* h, void** p, size_t bytes) {
 void free_all(moeca_handle* h) {
   for (auto& L : h->layers)
     if (L.tc) tc_plan_destroy(L.tc);
+  auto& io = h->hio;
+  for (int b = 0; b < 2; ++b) {
+    if (io.up[b]) cudaEventDestroy(io.up[b]);
+    if (io.done[b]) cudaEventDestroy(io.done[b]);
+    if (io.back[b]) cudaEventDestroy(io.back[b]);
+    io.up[b] = io.done[b] = io.back[b] = nullptr;
+  }
+  if (io.up_stream) cudaStreamDestroy(io.up_stream);
+  if (io.back_stream) cudaStreamDestroy(io.back_stream);
+  io.up_stream = io.back_stream = nullptr;
+  io.ready = false;
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   if (h->status_host) cudaFreeHost(h->status_host);
@@ -281,6 +304,7 @@ void moeca_config_default(moeca_config* c) {
   c->adaln = 0;
   c->ln_eps = 1e-6f;
   c->keep_route_in = 0;
+  c->token_reuse_policy = 0;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -324,6 +348,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (c.score_terms < 1 || c.score_terms > 7 || (c.granularity != 0 && c.granularity != 1))
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "score_terms must be 1..7 and granularity 0 or 1");
   if (c.refresh_period < 0) return fail(nullptr, MOECA_ERR_INVALID_ARG, "refresh_period < 0");
+  if (c.token_reuse_policy != 0 && c.token_reuse_policy != 1)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "token_reuse_policy must be 0 or 1");
   if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
   if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&
@@ -413,6 +439,7 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
       A(&L.attn_m, T * D * es);
       if (c.keep_route_in) A(&L.route_m, T * D * es);
     }
+    if (c.token_reuse_policy) A((void**)&L.cache_y, T * D * 4);
   }
   if (ada) {
     A(&h->ada_h, T * D * es);
@@ -771,6 +798,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       cb.gate = mod_l + 5 * c.hidden; cb.gate_ld = static_cast<int>(mod_ld); cb.seq = seq;
     }
     cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
+    if (L.cache_y) {
+      // Sec. 4.1, token level: a token with an empty recompute set returns y^{t0}.
+      cb.cache_y = L.cache_y; cb.token_any = L.token_any; cb.copy_y = refresh ? 0 : 1;
+    }
     cb.rearm = use_tc ? h->tc_work : nullptr;
     if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
     L.valid = true;
@@ -784,6 +815,84 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
   h->last_x_in = x_in;
   h->inject_stall = false;
   return MOECA_OK;
+}
+
+moeca_status moeca_step_host(moeca_handle* h, const void* x_in_host, void* x_out_host, const moeca_step_args* args,
+                             void* stream) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  if (!args) return fail(h, MOECA_ERR_INVALID_ARG, "args is NULL");
+  const moeca_config& c = h->cfg;
+  const int T = args->n_tokens;
+  if (T < 0 || T > c.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of [0, max_tokens]");
+  if (T == 0) return moeca_step(h, nullptr, nullptr, args, stream);
+  if (!x_in_host || !x_out_host) return fail(h, MOECA_ERR_INVALID_ARG, "x_in_host or x_out_host is NULL");
+  const bool ada = c.adaln != 0;
+  if (ada && !args->cond) return fail(h, MOECA_ERR_INVALID_ARG, "an AdaLN stack needs cond");
+  cudaSetDevice(h->device);
+  auto& io = h->hio;
+  cudaError_t e = cudaSuccess;
+  if (!io.ready) {
+    const size_t xb = static_cast<size_t>(c.max_tokens) * c.hidden * h->es;
+    const size_t cb = ada ? static_cast<size_t>(std::max(1, c.seq_len ? c.max_tokens / c.seq_len : 1)) * c.hidden * 4 : 0;
+    bool ok = true;
+    for (int b = 0; b < 2 && ok; ++b) {
+      ok = dev_alloc(h, &io.in[b], xb) && dev_alloc(h, &io.out[b], xb);
+      if (ok && cb) ok = dev_alloc(h, reinterpret_cast<void**>(&io.cond[b]), cb);
+    }
+    if (!ok) return fail(h, MOECA_ERR_OOM, "host staging buffers");
+    if ((e = cudaStreamCreateWithFlags(&io.up_stream, cudaStreamNonBlocking)) != cudaSuccess ||
+        (e = cudaStreamCreateWithFlags(&io.back_stream, cudaStreamNonBlocking)) != cudaSuccess)
+      return cuda_fail(h, e, "host copy streams");
+    for (int b = 0; b < 2; ++b)
+      if ((e = cudaEventCreateWithFlags(&io.up[b], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&io.done[b], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&io.back[b], cudaEventDisableTiming)) != cudaSuccess)
+        return cuda_fail(h, e, "host copy events");
+    io.ready = true;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int b = static_cast<int>(io.calls & 1);
+  const size_t xbytes = static_cast<size_t>(T) * c.hidden * h->es;
+  const bool reused = io.calls >= 2;  // buffers b were used by the call before the last
+  // Upload: staging input b is free once the step two calls back has run.
+  if (reused && (e = cudaStreamWaitEvent(io.up_stream, io.done[b], 0)) != cudaSuccess) return cuda_fail(h, e, "wait");
+  if ((e = cudaMemcpyAsync(io.in[b], x_in_host, xbytes, cudaMemcpyHostToDevice, io.up_stream)) != cudaSuccess)
+    return cuda_fail(h, e, "upload");
+  moeca_step_args a = *args;
+  if (ada) {
+    const int seq = c.seq_len ? c.seq_len : T;
+    const size_t cbytes = static_cast<size_t>(T / seq) * c.hidden * 4;
+    if ((e = cudaMemcpyAsync(io.cond[b], args->cond, cbytes, cudaMemcpyHostToDevice, io.up_stream)) != cudaSuccess)
+      return cuda_fail(h, e, "upload cond");
+    a.cond = io.cond[b];
+  }
+  if ((e = cudaEventRecord(io.up[b], io.up_stream)) != cudaSuccess) return cuda_fail(h, e, "record");
+  // The step waits for its upload and for the read-back that last used output b.
+  if ((e = cudaStreamWaitEvent(s, io.up[b], 0)) != cudaSuccess) return cuda_fail(h, e, "wait");
+  if (reused && (e = cudaStreamWaitEvent(s, io.back[b], 0)) != cudaSuccess) return cuda_fail(h, e, "wait");
+  moeca_status st = moeca_step(h, io.in[b], io.out[b], &a, stream);
+  if (st != MOECA_OK) return st;
+  if ((e = cudaEventRecord(io.done[b], s)) != cudaSuccess) return cuda_fail(h, e, "record");
+  // Read-back once the step has run.
+  if ((e = cudaStreamWaitEvent(io.back_stream, io.done[b], 0)) != cudaSuccess) return cuda_fail(h, e, "wait");
+  if ((e = cudaMemcpyAsync(x_out_host, io.out[b], xbytes, cudaMemcpyDeviceToHost, io.back_stream)) != cudaSuccess)
+    return cuda_fail(h, e, "read back");
+  if ((e = cudaEventRecord(io.back[b], io.back_stream)) != cudaSuccess) return cuda_fail(h, e, "record");
+  ++io.calls;
+  return MOECA_OK;
+}
+
+moeca_status moeca_host_join(moeca_handle* h, void* stream) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  auto& io = h->hio;
+  if (!io.ready || io.calls == 0) return MOECA_OK;
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // The read-back stream runs the read-backs in call order: its last event covers all of them.
+  const int last = static_cast<int>((io.calls - 1) & 1);
+  cudaError_t e = cudaStreamWaitEvent(s, io.back[last], 0);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, io.up[last], 0);
+  return e == cudaSuccess ? MOECA_OK : cuda_fail(h, e, "join");
 }
 
 moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out) {
@@ -842,7 +951,7 @@ moeca_status moeca_get_layer_state(moeca_handle* h, int32_t layer, const moeca_l
       {dst->cache_e, L.cache_e, T * k * 4},      {dst->cache_w, L.cache_w, T * k * 4},
       {dst->cache_norm, L.cache_norm, T * k * 4}, {dst->cache_h, L.cache_h, T * k * D * h->es},
       {dst->shared_h, L.shared_h, T * D * h->es}, {dst->ema, L.ema, T * E * 4},
-      {dst->attn_a, L.attn_a, T * D * h->es}};
+      {dst->attn_a, L.attn_a, T * D * h->es},     {dst->cache_y, L.cache_y, T * D * 4}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);
@@ -857,7 +966,8 @@ moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_l
   if (layer < 0 || layer >= h->cfg.n_layers) return fail(h, MOECA_ERR_INVALID_ARG, "layer out of range");
   if (n_tokens < 1 || n_tokens > h->cfg.max_tokens) return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens out of range");
   if (!src->cache_e || !src->cache_w || !src->cache_norm || !src->cache_h || !src->ema ||
-      (h->cfg.n_shared && !src->shared_h) || (h->cfg.n_heads && !src->attn_a))
+      (h->cfg.n_shared && !src->shared_h) || (h->cfg.n_heads && !src->attn_a) ||
+      (h->cfg.token_reuse_policy && !src->cache_y))
     return fail(h, MOECA_ERR_INVALID_ARG, "every state buffer is required");
   LayerBuf& L = h->layers[layer];
   const size_t T = n_tokens, k = h->cfg.top_k, D = h->cfg.hidden, E = h->cfg.n_experts;
@@ -867,7 +977,7 @@ moeca_status moeca_set_layer_state(moeca_handle* h, int32_t layer, const moeca_l
       {L.cache_e, src->cache_e, T * k * 4},      {L.cache_w, src->cache_w, T * k * 4},
       {L.cache_norm, src->cache_norm, T * k * 4}, {L.cache_h, src->cache_h, T * k * D * h->es},
       {L.shared_h, src->shared_h, T * D * h->es}, {L.ema, src->ema, T * E * 4},
-      {L.attn_a, src->attn_a, T * D * h->es}};
+      {L.attn_a, src->attn_a, T * D * h->es},     {L.cache_y, src->cache_y, T * D * 4}};
   for (auto& x : cp) {
     if (!x.d || !x.s) continue;
     cudaError_t e = cudaMemcpyAsync(x.d, x.s, x.n, cudaMemcpyDeviceToDevice, s);

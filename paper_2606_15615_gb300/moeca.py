@@ -15,7 +15,8 @@ import re
 
 PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(PKG, "libmoeca.so")
-HEADER = os.path.join(os.path.dirname(PKG), "include", "moeca.h")
+INCLUDE = os.path.join(os.path.dirname(PKG), "include")
+HEADER = os.path.join(INCLUDE, "moeca.h")
 
 MOECA_OK = 0
 MOECA_ERR_INVALID_ARG, MOECA_ERR_UNSUPPORTED, MOECA_ERR_CUDA, MOECA_ERR_OOM = -1, -2, -3, -4
@@ -41,7 +42,7 @@ class moeca_config(C.Structure):
                 ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32),
                 ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32),
                 ("attn_impl", C.c_int32), ("adaln", C.c_int32), ("ln_eps", C.c_float),
-                ("keep_route_in", C.c_int32)]
+                ("keep_route_in", C.c_int32), ("token_reuse_policy", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):
@@ -70,7 +71,7 @@ class moeca_stats(C.Structure):
 
 class moeca_layer_state(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema",
-                                            "attn_a")]
+                                            "attn_a", "cache_y")]
 
 
 class moeca_layer_trace(C.Structure):
@@ -113,6 +114,8 @@ def _load():
         "moeca_create": (C.c_int, [C.POINTER(moeca_config), C.POINTER(moeca_layer_weights), C.c_int32,
                                    C.POINTER(H)]),
         "moeca_step": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args), C.c_void_p]),
+        "moeca_step_host": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args), C.c_void_p]),
+        "moeca_host_join": (C.c_int, [H, C.c_void_p]),
         "moeca_get_stats": (C.c_int, [H, C.c_int32, C.POINTER(moeca_stats)]),
         "moeca_reset_stats": (C.c_int, [H]),
         "moeca_get_layer_state": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_state),
@@ -131,6 +134,7 @@ def _load():
         "moeca_ddpm_schedule": (C.c_int, [C.c_int32, C.c_int32, C.c_double, C.c_double, C.POINTER(C.c_int32),
                                           C.POINTER(C.c_double), C.POINTER(C.c_double), C.POINTER(C.c_double)]),
         "moeca_ddpm_step": (C.c_int, [C.POINTER(moeca_ddpm_args), C.c_void_p]),
+        "moeca_probe_ffma": (C.c_int32, [C.c_int32, C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -143,11 +147,14 @@ LIB = _load()
 
 
 def header_functions() -> list:
-    """Names of the functions include/moeca.h declares."""
-    with open(HEADER) as f:
-        text = f.read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(moeca_[a-z_]+)\s*\(", text)))
+    """Names of the functions the headers under include/ declare."""
+    names = set()
+    for fn in sorted(os.listdir(INCLUDE)):
+        if fn.endswith(".h"):
+            with open(os.path.join(INCLUDE, fn)) as f:
+                text = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
+            names |= set(re.findall(r"\b(moeca_[a-z_]+)\s*\(", text))
+    return sorted(names)
 
 
 def _check(status: int, handle=None):
@@ -178,6 +185,19 @@ def moeca_step(h, x_in_ptr: int, x_out_ptr: int, n_tokens: int, step_index: int,
                cond_ptr: int | None = None):
     args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override, cond_ptr)
     _check(LIB.moeca_step(h, x_in_ptr, x_out_ptr, C.byref(args), stream or None), h)
+
+
+def moeca_step_host(h, x_in_host_ptr: int, x_out_host_ptr: int, n_tokens: int, step_index: int,
+                    force_refresh: bool = False, tau0_override: float = math.nan, stream: int = 0,
+                    cond_host_ptr: int | None = None):
+    """One step from and to host buffers (see include/moeca.h); asynchronous."""
+    args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override, cond_host_ptr)
+    _check(LIB.moeca_step_host(h, x_in_host_ptr, x_out_host_ptr, C.byref(args), stream or None), h)
+
+
+def moeca_host_join(h, stream: int = 0):
+    """Order ``stream`` after every upload and read-back of moeca_step_host."""
+    _check(LIB.moeca_host_join(h, stream or None), h)
 
 
 def moeca_get_stats(h, layer: int = -1) -> dict:
@@ -253,6 +273,15 @@ def moeca_ddpm_step(args: moeca_ddpm_args, stream: int = 0):
     st = LIB.moeca_ddpm_step(C.byref(args), stream or None)
     if st != MOECA_OK:
         _check(st, None)
+
+
+def moeca_probe_ffma(device: int = 0, iterations: int = 1 << 16) -> tuple:
+    """Measured fp32 FFMA throughput of ``device``: (TFLOP/s, ms) (include/moeca_probe.h)."""
+    tf, ms = C.c_double(), C.c_double()
+    st = LIB.moeca_probe_ffma(device, iterations, C.byref(tf), C.byref(ms))
+    if st != 0:
+        raise MoecaError(st, "moeca_probe_ffma")
+    return tf.value, ms.value
 
 
 def moeca_status_string(status: int) -> str:
@@ -356,7 +385,8 @@ class Stack:
                  cache_h=self._empty((T, c.top_k, c.hidden), self.dtype),
                  shared_h=self._empty((T, c.hidden), self.dtype) if c.n_shared else None,
                  ema=self._empty((T, c.n_experts), torch.float32),
-                 attn_a=self._empty((T, c.hidden), self.dtype) if c.n_heads else None)
+                 attn_a=self._empty((T, c.hidden), self.dtype) if c.n_heads else None,
+                 cache_y=self._empty((T, c.hidden), torch.float32) if c.token_reuse_policy else None)
         st = moeca_layer_state(**{k: (v.data_ptr() if v is not None else None) for k, v in t.items()})
         n = moeca_get_layer_state(self.handle, layer, st, self.stream_ptr())
         return {k: (v[:n] if v is not None else None) for k, v in t.items()} | {"n_tokens": n}
@@ -366,7 +396,7 @@ class Stack:
         keep = {k: v.contiguous() for k, v in state.items() if k != "n_tokens" and v is not None}
         st = moeca_layer_state(**{k: keep[k].data_ptr() if k in keep else None
                                   for k in ("cache_e", "cache_w", "cache_norm", "cache_h", "shared_h", "ema",
-                                            "attn_a")})
+                                            "attn_a", "cache_y")})
         moeca_set_layer_state(self.handle, layer, st, n, self.stream_ptr())
         self.torch.cuda.current_stream(self.device).synchronize()
 

@@ -94,6 +94,20 @@ def test_shared_expert_block(M):
     st.close()
 
 
+def test_token_reuse_copy_block(M):
+    """Sec. 4.1's token-level reading in the AdaLN block: a token with an
+    empty recompute set returns its stored ungated y^{t0}, and the current
+    step's gate g_m applies to it (the conditioning changes every step)."""
+    T, D, H, S = 256, 256, 4, 128
+    st, cfg, ws = make_adaln_stack(M, T, D, H, 4, 2, 256, L=2, S=S, n_shared=1, seed=12, tau0=0.95,
+                                   token_reuse_policy=1)
+    rng = np.random.default_rng(120)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.03)
+    rep, _ = run_trajectory(st, cfg, ws, xs, conds=W.conditioning(12, T // S, D, 4))
+    assert rep.tokens_copied > 0 and rep.recomputed > 0, rep.summary()
+    st.close()
+
+
 def test_wide_block(M):
     """D 2560 (20 heads of 128 channels), the widest row the AdaLN row kernel
     holds in registers (ten 16-byte chunks per lane)."""

@@ -193,9 +193,9 @@ def test_sixteen_token_prep_blocks(M):
     st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 256, L=1, S=S, n_shared=1, seed=13, tau0=0.7)
     rng = np.random.default_rng(130)
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 3, 0.08)
-    # Outputs of magnitude ~40 here: the per-row relative bounds apply, not
-    # the absolute one.
-    rep, _ = run_trajectory(st, cfg, ws, xs, out_tol=(1e-2, None))
+    # Outputs of magnitude ~40 here: the max-abs bound follows the bf16
+    # step of the value (see output_abs_bound).
+    rep, _ = run_trajectory(st, cfg, ws, xs)
     assert rep.reused > 0 and rep.attn_rows > T
     st.close()
 
@@ -231,6 +231,6 @@ def test_wide_block_separate_path(M):
     st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 512, L=1, S=S, n_shared=1, seed=15, wscale=0.02, tau0=0.7)
     rng = np.random.default_rng(150)
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 3, 0.08)
-    rep, _ = run_trajectory(st, cfg, ws, xs, out_tol=(1e-2, None))
+    rep, _ = run_trajectory(st, cfg, ws, xs)
     assert rep.reused > 0 and rep.attn_rows > T
     st.close()

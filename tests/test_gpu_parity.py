@@ -108,7 +108,10 @@ def test_bf16_fine_grained_64_experts_top8(M):
     # Table 5's score-signal subsets and token-level granularity (Sec. 3)
     dict(score_terms=1, tau0=0.55), dict(score_terms=2, tau0=0.05), dict(score_terms=4, tau0=0.25),
     dict(score_terms=3, tau0=0.6), dict(score_terms=6, tau0=0.3), dict(granularity=1, tau0=0.9),
-    dict(granularity=1, score_terms=5, tau0=0.8)])
+    dict(granularity=1, score_terms=5, tau0=0.8),
+    # Sec. 4.1's token-level reading: R_i empty => y^{t0} returned unchanged
+    dict(token_reuse_policy=1, tau0=0.9), dict(token_reuse_policy=1, n_shared=1, tau0=1.0),
+    dict(token_reuse_policy=1, granularity=1, tau0=0.95)])
 def test_reading_switches(M, switch):
     sw = dict(switch)
     S = sw.pop("n_shared", 0)
@@ -116,7 +119,24 @@ def test_reading_switches(M, switch):
     st, cfg, ws = make_stack(M, T, D, E, k, F, L=1, S=S, seed=4, **({"tau0": 0.75} | sw))
     rng = np.random.default_rng(14)
     xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05, True)
-    run_trajectory(st, cfg, ws, xs)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    if sw.get("token_reuse_policy"):
+        assert rep.tokens_copied > 0 and rep.recomputed > 0, rep.summary()
+    st.close()
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_token_reuse_copy_multi_layer(M, bf16):
+    """The copy reading on the fp32 separate-kernel path and on the bf16
+    fused path, three layers, tokens reused for several steps in a row: the
+    returned y must be the one stored when the token last computed."""
+    T, D, E, k, F = 193, 128, 8, 2, 256
+    st, cfg, ws = make_stack(M, T, D, E, k, F, L=3, bf16=bf16, seed=9, tau0=0.95, token_reuse_policy=1,
+                             refresh_period=5)
+    rng = np.random.default_rng(19)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 6, 0.03, bf16)
+    rep, out = run_trajectory(st, cfg, ws, xs, bf16=bf16)
+    assert rep.tokens_copied > T and rep.recomputed > 0, rep.summary()
     st.close()
 
 
