@@ -2,13 +2,17 @@
 """Benchmark of the GB300 branch-cached MoE layer stack (MoECa).
 
 A step is one denoising step of the whole stack (every layer: router, select,
-compact, grouped FFN x2, combine) over one batch of synthetic tokens.  The
-default workload is the 12-layer stack D 768, E 16, top-2, F 3072, T 2048
-(8 x 256 tokens) in bf16, driven along its seeded drift trajectory.  The
-headline value is tokens/s at the 60% branch-reuse point (tau0 calibrated on
-the GPU path itself); the same line carries the sweep over reuse 0/30/60/90%,
-end-to-end numbers with host buffers, a roofline entry for the dominant kernel,
-the oracle's CPU baseline, and the SM clocks sampled during the timed region.
+compact, grouped FFN, combine) over one batch of synthetic tokens.  The
+headline workload is the 12-layer stack D 768, E 16, top-2, F 3072, T 2048
+(8 x 256 tokens) in bf16, driven along its seeded drift trajectory, at the
+60% branch-reuse point: tau0 calibrated on the oracle (oracle/calibrate_tau0.py,
+stored in paper_2606_15615_gb300/headline_points.json) so that this GPU arm
+and the reference arm (the oracle) time the same configuration.  The line
+carries the sweep over reuse 0/30/60/90%, end-to-end numbers through the
+host-buffer C call, a roofline entry for the dominant kernel, the oracle's CPU
+baseline, the SM clocks sampled during the timed region, and one row per
+other workload (the fp32 layer, the 28-layer and 16-layer stacks at 60%
+reuse, the 64-expert layer over reuse 0-95% in 5% steps).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -37,6 +41,23 @@ DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn", "qkv", "attn", "oproj", "attn_aux",
          "adaln"]
+# Reuse points per workload index (BASELINE's sweeps) and the point each row's kernels are timed at.
+CONFIG_POINTS = {1: (0.5,), 2: (0.0, 0.3, 0.6, 0.9), 3: (0.6,), 4: (0.6,),
+                 5: tuple(round(0.05 * j, 2) for j in range(20))}
+MAIN_POINT = {1: 0.5, 2: 0.6, 3: 0.6, 4: 0.6, 5: 0.6}
+HEADLINE_POINTS = os.path.join(ROOT, "paper_2606_15615_gb300", "headline_points.json")
+
+
+def headline_point(wl, reuse: float):
+    """The stored oracle-calibrated tau0 of ``wl`` at ``reuse``, or None."""
+    if not os.path.exists(HEADLINE_POINTS):
+        return None
+    with open(HEADLINE_POINTS) as f:
+        pts = json.load(f)
+    p = pts.get(wl.name)
+    if p and abs(p.get("reuse_target", -1) - reuse) < 1e-9:
+        return p
+    return None
 
 
 # ---------------------------------------------------------------------------
@@ -220,13 +241,9 @@ class Runner:
         T, D = wl.n_tokens, wl.hidden
         self.out = torch.empty((T, D), dtype=dt, device=self.dev)
         self.stream = torch.cuda.current_stream(self.dev)
-        # End to end: two input and two output buffers, so the upload of step
-        # t + 1 and the read-back of step t run on a copy stream while the
-        # neighbouring steps compute (every step still moves its own bytes).
-        self.in_bufs = [torch.empty((T, D), dtype=dt, device=self.dev) for _ in range(2)]
-        self.out_bufs = [torch.empty((T, D), dtype=dt, device=self.dev) for _ in range(2)]
+        # End to end through moeca_step_host: pinned host outputs, two of them
+        # so that a step's read-back never waits for the one before.
         self.out_host = [torch.empty((T, D), dtype=dt).pin_memory() for _ in range(2)]
-        self.copy_stream = torch.cuda.Stream(device=self.dev)
         # AdaLN workloads: a conditioning vector per sample and step, and the
         # Eq. 1 update of each step's output (x_t kept in float32; the noise
         # draw z is one fixed buffer, an input of the update).
@@ -235,12 +252,18 @@ class Runner:
             c = torch.from_numpy(W.workload_conditioning(wl, n_steps))
             self.cond_host = c.pin_memory()
             self.cond_dev = c.to(self.dev)
-            self.cond_bufs = [torch.empty_like(self.cond_dev[0]) for _ in range(2)]
             g = torch.Generator(device=self.dev)
             g.manual_seed(3000 + wl.index)
             self.x_state = torch.empty((T, D), dtype=torch.float32, device=self.dev).normal_(generator=g)
             self.z = torch.empty((T, D), dtype=torch.float32, device=self.dev).normal_(generator=g)
             _, self.alpha, self.abar, self.beta = M.moeca_ddpm_schedule(max(wl.n_steps, n_steps, 2))
+
+    def close(self):
+        self.stack.close()
+        self.weights = self.x_dev = self.x_host = self.out = self.out_host = None
+        self.cond_dev = self.cond_host = None
+        self.torch.cuda.synchronize(self.dev)
+        self.torch.cuda.empty_cache()
 
     def _sampler_update(self, t, eps):
         """Eq. 1: x_{t-1} from x_t and this step's output; run step t visits schedule step n - 1 - t."""
@@ -263,7 +286,6 @@ class Runner:
         M.moeca_reset(h)
         M.moeca_set_kernel_timing(h, False)
         sp = self.stream.cuda_stream
-        T = self.wl.n_tokens
         for t in range(W_):
             self._step(h, self.x_dev[t].data_ptr(), self.out, t, tau0, sp)
         torch.cuda.synchronize(self.dev)
@@ -290,46 +312,56 @@ class Runner:
         return ms, st, kt
 
     def _e2e_steps(self, tau0, W_, K):
-        """Steps W_ .. W_ + K - 1 from pinned host inputs to pinned host outputs.
+        """Steps W_ .. W_ + K - 1 through the host-buffer C call: each step's
+        input is uploaded from pinned host memory and its output read back
+        into pinned host memory by the library (moeca_step_host), which
+        overlaps them with the neighbouring steps' compute; the join orders
+        the end event after the last read-back."""
+        M, h, sp = self.M, self.stack.handle, self.stream.cuda_stream
+        if self.wl.adaln:
+            return self._e2e_steps_sampler(tau0, W_, K)
+        for t in range(W_, W_ + K):
+            M.moeca_step_host(h, self.x_host[t].data_ptr(), self.out_host[t % 2].data_ptr(), self.wl.n_tokens, t,
+                              False, tau0, sp)
+        M.moeca_host_join(h, sp)
 
-        Step t reads in_bufs[t % 2] and writes out_bufs[t % 2].  The copy
-        stream uploads step t + 1's input once step t - 1 (its buffer's last
-        reader) is done, then reads step t's output back once step t is done;
-        the compute stream starts step t after its upload and, for t >= 2,
-        after step t - 2's read-back (its output buffer's last reader).
-        """
-        torch, M = self.torch, self.M
-        h, T, sp, cs = self.stack.handle, self.wl.n_tokens, self.stream.cuda_stream, self.copy_stream
+    def _e2e_steps_sampler(self, tau0, W_, K):
+        """AdaLN workloads, whose step ends with the Eq. 1 update of the
+        device output: the inputs and conditioning are uploaded and the
+        outputs read back by torch copies on a side stream, double-buffered
+        against the neighbouring steps (step t reads in_bufs[t % 2])."""
+        torch = self.torch
+        h, T, D, sp = self.stack.handle, self.wl.n_tokens, self.wl.hidden, self.stream.cuda_stream
+        in_bufs = [torch.empty((T, D), dtype=self.dt, device=self.dev) for _ in range(2)]
+        out_bufs = [torch.empty((T, D), dtype=self.dt, device=self.dev) for _ in range(2)]
+        cond_bufs = [torch.empty_like(self.cond_dev[0]) for _ in range(2)]
+        cs = torch.cuda.Stream(device=self.dev)
         ev = lambda: torch.cuda.Event()  # noqa: E731
         up, done, back = [ev(), ev()], [ev(), ev()], [ev(), ev()]
         cs.wait_stream(self.stream)
-        ada = self.wl.adaln
         with torch.cuda.stream(cs):
-            self.in_bufs[W_ % 2].copy_(self.x_host[W_], non_blocking=True)
-            if ada:
-                self.cond_bufs[W_ % 2].copy_(self.cond_host[W_], non_blocking=True)
+            in_bufs[W_ % 2].copy_(self.x_host[W_], non_blocking=True)
+            cond_bufs[W_ % 2].copy_(self.cond_host[W_], non_blocking=True)
             up[W_ % 2].record(cs)
         for t in range(W_, W_ + K):
             b = t % 2
             self.stream.wait_event(up[b])
             if t - 2 >= W_:
                 self.stream.wait_event(back[b])
-            self._step(h, self.in_bufs[b].data_ptr(), self.out_bufs[b], t, tau0, sp,
-                       cond=self.cond_bufs[b] if ada else None)
+            self._step(h, in_bufs[b].data_ptr(), out_bufs[b], t, tau0, sp, cond=cond_bufs[b])
             done[b].record(self.stream)
             with torch.cuda.stream(cs):
                 if t + 1 < W_ + K:
                     nb = (t + 1) % 2
                     if t - 1 >= W_:
                         cs.wait_event(done[nb])
-                    self.in_bufs[nb].copy_(self.x_host[t + 1], non_blocking=True)
-                    if ada:
-                        self.cond_bufs[nb].copy_(self.cond_host[t + 1], non_blocking=True)
+                    in_bufs[nb].copy_(self.x_host[t + 1], non_blocking=True)
+                    cond_bufs[nb].copy_(self.cond_host[t + 1], non_blocking=True)
                     up[nb].record(cs)
                 cs.wait_event(done[b])
-                self.out_host[b].copy_(self.out_bufs[b], non_blocking=True)
+                self.out_host[b].copy_(out_bufs[b], non_blocking=True)
                 back[b].record(cs)
-        self.stream.wait_stream(cs)  # the last read-back is inside the timed region
+        self.stream.wait_stream(cs)
 
     def reuse_of(self, st) -> float:
         return st["reused"] / max(st["branches"], 1)
@@ -360,8 +392,12 @@ class Runner:
 def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float, attn_rows: float = 0.0):
     """Algorithmic (bytes, flops) of one launch of a kernel kind for this workload.
 
-    ``attn_rows`` is the mean number of token rows one attention launch
-    computes (every token on a full step, the recomputing tokens otherwise)."""
+    ``rows_per_launch`` is the mean number of recomputed branch rows (plus
+    shared-expert rows) of one layer step; ``attn_rows`` the mean number of
+    token rows one attention launch computes (every token on a full step, the
+    recomputing tokens otherwise).  The FFN's bf16 hidden activations are
+    an implementation intermediate, not algorithmic: its bytes are the active
+    experts' weights, the gathered input rows and the scattered output rows."""
     T, D, E, k, F, S = wl.n_tokens, wl.hidden, wl.n_experts, wl.top_k, wl.ffn, wl.n_shared
     es = 2 if wl.dtype == "bf16" else 4
     if kind == "qkv":      # x [T, D] and W_qkv [3D, D] in, q | k | v [T, 3D] out
@@ -387,10 +423,10 @@ def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float, att
         return T * k * (8 + 12 + 8 + 3) + T, 0.0
     if kind == "compact":
         return T * k * 6 + T + rows_per_launch * (4 + 2 * D * es), 0.0
-    if kind == "ffn1":
-        return active_groups * F * D * es + rows_per_launch * (D + F) * es, 2.0 * rows_per_launch * D * F
-    if kind == "ffn2":
-        return active_groups * F * D * es + rows_per_launch * (F + D) * es, 2.0 * rows_per_launch * D * F
+    if kind == "ffn1":     # W1 of the active experts, gathered input rows
+        return active_groups * F * D * es + rows_per_launch * D * es, 2.0 * rows_per_launch * D * F
+    if kind == "ffn2":     # W2 of the active experts, output rows scattered into the cache
+        return active_groups * F * D * es + rows_per_launch * D * es, 2.0 * rows_per_launch * D * F
     if kind == "ffn":
         b1, f1 = algorithmic("ffn1", wl, rows_per_launch, active_groups)
         b2, f2 = algorithmic("ffn2", wl, rows_per_launch, active_groups)
@@ -405,11 +441,108 @@ def algorithmic(kind: str, wl, rows_per_launch: float, active_groups: float, att
     raise KeyError(kind)
 
 
+def kernel_table(wl, kt, st_k, K):
+    """Per-kernel-kind mean event time, algorithmic bytes / flops and achieved rates."""
+    rows_per_launch = (st_k["recomputed"] + st_k["shared_recomputed"]) / (K * wl.n_layers)
+    attn_rows = st_k["attn_recomputed"] / max(kt["attn"][1], 1)
+    total = max(sum(v[0] for v in kt.values()), 1e-12)
+    kernels = {}
+    for kind in KINDS:
+        tot, n = kt[kind]
+        if not n:
+            continue
+        nb, nf = algorithmic(kind, wl, rows_per_launch, wl.n_experts + wl.n_shared, attn_rows)
+        avg = tot / n
+        kernels[kind] = {"launches": n, "avg_us": avg * 1e3, "share": tot / total, "alg_bytes": nb, "alg_flops": nf,
+                         "gbs": nb / (avg * 1e-3) / 1e9 if avg > 0 else None,
+                         "tflops": nf / (avg * 1e-3) / 1e12 if avg > 0 and nf else None}
+    return kernels
+
+
+def roofline(kind: str, kd: dict, wl, pk: dict, pk_src: str, ffma_peak):
+    """Roofline entry of one kernel kind from its event-timed mean.
+
+    Peaks are MEASURED_PEAKS.json's burst figures (the kernels are timed one
+    launch at a time): HBM copy GB/s and cuBLAS bf16 TFLOP/s.  A bf16 kernel
+    whose algorithmic intensity is above the ridge is tensor-bound; the fp32
+    path's FFN is FFMA-bound, against the measured FFMA rate.  Both fractions
+    are given for the FFN."""
+    src = "of measured (MEASURED_PEAKS.json, burst)" if pk_src == "measured" else "of fallback"
+    ridge = pk["bf16_tflops"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+    hbm = {"achieved": kd["gbs"], "peak": pk["hbm_gbs"], "unit": "GB/s",
+           "frac": kd["gbs"] / pk["hbm_gbs"] if kd["gbs"] else None}
+    r = {"kernel": kind, "alg_bytes_per_launch": kd["alg_bytes"], "alg_flops_per_launch": kd["alg_flops"],
+         "avg_us": kd["avg_us"]}
+    if wl.dtype != "bf16" and kind in ("ffn1", "ffn2") and ffma_peak:
+        tf = kd["tflops"]
+        r.update(bound="fp32", achieved=tf, peak=ffma_peak, unit="TFLOP/s", frac=tf / ffma_peak if tf else None,
+                 peak_source="measured on this GPU (moeca_probe_ffma)", hbm=hbm)
+    elif kd["alg_flops"] and kd["alg_flops"] / kd["alg_bytes"] > ridge:
+        tf = kd["tflops"]
+        r.update(bound="tensor", achieved=tf, peak=pk["bf16_tflops"], unit="TFLOP/s",
+                 frac=tf / pk["bf16_tflops"] if tf else None, peak_source=src, hbm=hbm)
+    else:
+        r.update(bound="hbm", achieved=hbm["achieved"], peak=hbm["peak"], unit="GB/s", frac=hbm["frac"],
+                 peak_source=src)
+        if kd["alg_flops"] and kd["tflops"]:
+            r["tensor"] = {"achieved": kd["tflops"], "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+                           "frac": kd["tflops"] / pk["bf16_tflops"]}
+    return r
+
+
+def point_row(runner, wl, tgt, tau0, ms, st, K, world):
+    tokens_all = wl.n_tokens * K * world
+    executed = (st["recomputed"] + st["shared_recomputed"]) * 4.0 * wl.hidden * wl.ffn
+    dense = wl.dense_flops_per_layer() * wl.n_layers * K
+    if wl.n_heads:
+        D, T = wl.hidden, wl.n_tokens
+        executed += (2.0 * T * D * 3 * D * wl.n_layers * K
+                     + st["attn_recomputed"] * (4.0 * wl.seq * D + 2.0 * D * D))
+        dense += (2.0 * T * D * 3 * D + T * (4.0 * wl.seq * D + 2.0 * D * D)) * wl.n_layers * K
+    return {"reuse_target": tgt, "reuse_achieved": round(runner.reuse_of(st), 4),
+            "tau0": None if not math.isfinite(tau0) else round(tau0, 5), "tokens_per_s": tokens_all / (ms / 1e3),
+            "ms_per_step": ms / K, "effective_tflops": dense * world / (ms / 1e3) / 1e12,
+            "executed_tflops": executed * world / (ms / 1e3) / 1e12}
+
+
+def config_row(wl, local: int, W_: int, K: int, pk, pk_src, ffma_peak):
+    """One BASELINE workload at its reuse points: tokens/s, effective TFLOP/s
+    per point, and at the main point the per-kernel times with the dominant
+    kernel's roofline."""
+    runner = Runner(wl, local, W_ + K)
+    try:
+        pts, main = CONFIG_POINTS[wl.index], MAIN_POINT[wl.index]
+        rows, main_tau = [], None
+        for tgt in pts:
+            tau0, _ = runner.calibrate(tgt, W_, K)
+            reps = [runner._run(tau0, W_, K) for _ in range(2)]
+            ms = statistics.median(r[0] for r in reps)
+            rows.append(point_row(runner, wl, tgt, tau0, ms, reps[-1][1], K, 1))
+            if abs(tgt - main) < 1e-9:
+                main_tau = tau0
+        _, st_k, kt = runner._run(main_tau, W_, K, kernel_timing=True)
+        kernels = kernel_table(wl, kt, st_k, K)
+        dom = max(kernels, key=lambda k_: kernels[k_]["avg_us"] * kernels[k_]["launches"])
+        row = {"workload": wl.name, "dtype": wl.dtype, "tokens": wl.n_tokens, "layers": wl.n_layers,
+               **next(r for r in rows if abs(r["reuse_target"] - main) < 1e-9),
+               "roofline": roofline(dom, kernels[dom], wl, pk, pk_src, ffma_peak),
+               "kernels": {k_: {kk: (round(v, 3) if isinstance(v, float) else v) for kk, v in d.items()
+                                if kk in ("launches", "avg_us", "share", "gbs", "tflops")}
+                           for k_, d in kernels.items()}}
+        for kind in ("ffn", "ffn2", "combine", "prep", "router"):
+            if kind in kernels and kind != dom:
+                row[f"roofline_{kind}"] = roofline(kind, kernels[kind], wl, pk, pk_src, ffma_peak)
+        if len(rows) > 1:
+            row["sweep"] = rows
+        return row
+    finally:
+        runner.close()
+
+
 def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
     """The oracle on this host's cores: full-T cache steps of layer 0, extrapolated to L layers."""
     import numpy as np
     from oracle import moeca_oracle as O
-    torch = runner.torch
     w = {k: (None if v is None else v.float().cpu().numpy().astype(np.float64)) for k, v in runner.weights[0].items()}
     if w["ws1"] is None:
         w["ws1"] = w["ws2"] = None
@@ -432,16 +565,19 @@ def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
         if time.perf_counter() - t_all > budget_s:
             break
     per_layer = statistics.mean(times)
-    try:
-        from threadpoolctl import threadpool_info
-        cores = max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
-    except Exception:
-        cores = os.cpu_count()
-    return {"value": wl.n_tokens / (per_layer * wl.n_layers), "unit": "tokens/s", "cores": cores,
+    return {"value": wl.n_tokens / (per_layer * wl.n_layers), "unit": "tokens/s", "cores": host_threads(),
             "kind": "oracle",
             "sample": (f"{len(times)} cache steps of layer 0 at full T={wl.n_tokens} (tau0 of the headline point), "
                        f"{per_layer * 1e3:.0f} ms per layer step, extrapolated to {wl.n_layers} layers; "
                        f"numpy float64, host cores {os.cpu_count()}")}
+
+
+def host_threads() -> int:
+    try:
+        from threadpoolctl import threadpool_info
+        return max([i.get("num_threads", 1) for i in threadpool_info()] or [1])
+    except Exception:
+        return os.cpu_count()
 
 
 # ---------------------------------------------------------------------------
@@ -449,42 +585,58 @@ def cpu_oracle_baseline(wl, runner, tau0: float, budget_s: float = 12.0):
 # ---------------------------------------------------------------------------
 
 def reference_arm(args, wl):
+    """The oracle (plain numpy float64) on the host cores: the whole L-layer
+    stack on consecutive steps of the same seeded trajectory, with the same
+    weights (torch's seeded CUDA generator, copied to host memory) and the
+    same headline tau0 as the GPU arm; W untimed steps, then K timed ones."""
     import numpy as np
+    import torch
     from oracle import moeca_oracle as O
     from paper_2606_15615_gb300 import workloads as W
-    rng_layers = min(wl.n_layers, 2)
-    ws = [W.make_layer_weights(wl, l) for l in range(rng_layers)]
-    if wl.n_heads:
-        for l in range(rng_layers):
-            ws[l].update(W.make_attn_weights(wl, l))
+    pt = headline_point(wl, args.reuse)
+    tau0 = args.tau0 if args.tau0 is not None else (pt["tau0"] if pt else args.ref_tau0)
+    dev = torch.device("cuda", 0) if torch.cuda.is_available() else None
+    ws = []
+    for l in range(wl.n_layers):
+        if dev is not None:
+            w = W.make_layer_weights_device(wl, l, dev)
+            w = {k: (None if v is None else v.float().cpu().numpy().astype(np.float64)) for k, v in w.items()}
+        else:
+            w = W.make_layer_weights(wl, l)
+        if wl.n_heads:
+            w.update(W.make_attn_weights(wl, l))
             if wl.adaln:
-                ws[l].update(W.make_adaln_weights(wl, l))
-    xs = list(W.trajectory(wl, args.warmup + args.steps + 1))
+                w.update(W.make_adaln_weights(wl, l))
+        ws.append(w)
+    xs = list(W.trajectory(wl, args.warmup + args.steps))
     conds = W.workload_conditioning(wl, len(xs)) if wl.adaln else [None] * len(xs)
-    prm = O.Params(top_k=wl.top_k, tau0=args.ref_tau0, refresh_period=wl.refresh_period,
+    prm = O.Params(top_k=wl.top_k, tau0=tau0, refresh_period=wl.refresh_period,
                    n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0, adaln=wl.adaln,
                    act_store="bf16" if wl.adaln else "f64")
-    stacks = [O.Stack([ws[l]], prm, wl.hidden, wl.n_experts, wl.n_shared) for l in range(rng_layers)]
+    stack = O.Stack(ws, prm, wl.hidden, wl.n_experts, wl.n_shared)
     for t in range(args.warmup):
-        stacks[t % rng_layers].step(xs[t], t, cond=conds[t])
-    times = []
-    for j in range(args.steps):
-        t = args.warmup + j
-        s = stacks[t % rng_layers]
-        t0 = time.perf_counter()
-        s.step(xs[t], t, cond=conds[t])
-        times.append(time.perf_counter() - t0)
-    per_layer = statistics.mean(times)
-    value = wl.n_tokens / (per_layer * wl.n_layers)
-    cores = os.cpu_count()
+        stack.step(xs[t], t, cond=conds[t])
+    reused = routed = 0
+    t0 = time.perf_counter()
+    for t in range(args.warmup, args.warmup + args.steps):
+        _, infos = stack.step(xs[t], t, cond=conds[t])
+        for inf in infos:
+            reused += int((~inf["recompute"]).sum())
+            routed += inf["recompute"].size
+    elapsed = time.perf_counter() - t0
+    value = wl.n_tokens * args.steps / elapsed
+    cores = host_threads()
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * wl.n_layers * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "tau0": args.ref_tau0},
+        "config": {"workload": wl.name, "reuse_target": args.reuse},
+        "point": {"tau0": tau0, "tau0_source": "oracle-calibrated (headline_points.json)" if pt and args.tau0 is None
+                  else "command line", "reuse_achieved": round(reused / max(routed, 1), 4)},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                         "sample": (f"each step is one full-T layer step of the CPU oracle (layers 0-{rng_layers - 1} "
-                                    f"alternating, numpy weights), time extrapolated to {wl.n_layers} layers")},
+                         "sample": (f"the whole {wl.n_layers}-layer stack, {args.steps} consecutive timed steps "
+                                    f"after {args.warmup} untimed ones, at full T={wl.n_tokens}; numpy float64 on "
+                                    f"{os.cpu_count()} host cores; no extrapolation")},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -502,12 +654,15 @@ def main():
     ap.add_argument("--reuse", type=float, default=0.6, help="headline reuse target")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--configs", default="auto",
+                    help="other workloads to add as rows: 'all', 'none', or indices like '1,3' "
+                         "(auto: all with the default workload, none otherwise)")
     ap.add_argument("--reps", type=int, default=5)
-    ap.add_argument("--ref-tau0", type=float, default=0.8)
+    ap.add_argument("--ref-tau0", type=float, default=0.665, help="reference arm tau0 without a stored point")
     ap.add_argument("--ffn-tile-n", type=int, default=0, help="force the tensor-core FFN tile width (0: auto)")
     ap.add_argument("--ffn-split-k", type=int, default=0, help="force the tensor-core FFN K splits (0: auto)")
     ap.add_argument("--tau0", type=float, default=None,
-                    help="use this tau0 for the headline point instead of calibrating it (profiling runs)")
+                    help="use this tau0 for the headline point instead of the stored / calibrated one")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first N layers of the workload (small ncu captures; not a bench line)")
     args = ap.parse_args()
@@ -530,17 +685,19 @@ def main():
     dev = runner.dev
     W_, K = args.warmup, args.steps
     targets = [args.reuse] if args.no_sweep else sorted(set(wl.reuse_targets) | {args.reuse})
-    if wl.reuse_targets == (0.5,) and args.no_sweep is False:
-        targets = sorted(set(wl.reuse_targets) | {args.reuse})
+    pk, pk_src = peaks()
+    stored = headline_point(wl, args.reuse) if not args.layers else None
     sweep = []
     head = None
-    pk, pk_src = peaks()
     for tgt in targets:
-        if args.tau0 is not None and abs(tgt - args.reuse) < 1e-9:
-            tau0 = args.tau0
-        else:
-            tau0, achieved = runner.calibrate(tgt, W_, K)
         is_head = abs(tgt - args.reuse) < 1e-9
+        if is_head and args.tau0 is not None:
+            tau0, src = args.tau0, "command line"
+        elif is_head and stored is not None:
+            tau0, src = stored["tau0"], "oracle-calibrated (headline_points.json)"
+        else:
+            tau0, _ = runner.calibrate(tgt, W_, K)
+            src = "calibrated on this GPU"
         sampler = None
         if is_head and rank == 0:
             sampler = ClockSampler(gpu_smi_id(local))
@@ -552,59 +709,28 @@ def main():
                 dist.barrier()
             torch.cuda.synchronize(dev)
             ms, st, _ = runner._run(tau0, W_, K)
-            ms, tokens = aggregate(ms, wl.n_tokens * K, dist, dev)
+            ms, _ = aggregate(ms, wl.n_tokens * K, dist, dev)
             reps.append(ms)
         clocks = sampler.stop() if sampler else None
-        ms = statistics.median(reps)
-        tokens_all = wl.n_tokens * K * world
-        tps = tokens_all / (ms / 1e3)
-        executed = (st["recomputed"] + st["shared_recomputed"]) * 4.0 * wl.hidden * wl.ffn  # per rank, K steps
-        dense = wl.dense_flops_per_layer() * wl.n_layers * K
-        if wl.n_heads:
-            D, T = wl.hidden, wl.n_tokens
-            executed += (2.0 * T * D * 3 * D * wl.n_layers * K
-                         + st["attn_recomputed"] * (4.0 * wl.seq * D + 2.0 * D * D))
-            dense += (2.0 * T * D * 3 * D + T * (4.0 * wl.seq * D + 2.0 * D * D)) * wl.n_layers * K
-        row = {"reuse_target": tgt, "reuse_achieved": round(runner.reuse_of(st), 4),
-               "tau0": None if not math.isfinite(tau0) else round(tau0, 5), "tokens_per_s": tps,
-               "ms_per_step": ms / K, "effective_tflops": dense * world / (ms / 1e3) / 1e12,
-               "executed_tflops": executed * world / (ms / 1e3) / 1e12}
+        row = point_row(runner, wl, tgt, tau0, statistics.median(reps), st, K, world)
         sweep.append(row)
         if is_head:
-            head = dict(row, clocks=clocks, stats=st, tau0_raw=tau0)
+            head = dict(row, clocks=clocks, stats=st, tau0_raw=tau0, tau0_source=src)
 
     # Per-kernel CUDA-event durations on the launching stream, same steps as the headline.
     _, st_k, kt = runner._run(head["tau0_raw"], W_, K, kernel_timing=True)
-    # End to end through the C ABI with host buffers.
+    # End to end through the host-buffer C call.
     if dist is not None:
         dist.barrier()
     e2e_reps = [runner._run(head["tau0_raw"], W_, K, e2e=True)[0] for _ in range(max(1, args.reps))]
     e2e_ms, _ = aggregate(statistics.median(e2e_reps), 0, dist, dev)
-    rows_per_launch = (st_k["recomputed"] + st_k["shared_recomputed"]) / (K * wl.n_layers)
-    attn_rows = st_k["attn_recomputed"] / max(kt["attn"][1], 1)
-    kernels = {}
-    for kind in KINDS:
-        tot, n = kt[kind]
-        nb, nf = algorithmic(kind, wl, rows_per_launch, wl.n_experts + wl.n_shared, attn_rows)
-        avg = tot / max(n, 1)
-        kernels[kind] = {"launches": n, "avg_us": avg * 1e3, "share": tot / max(sum(v[0] for v in kt.values()), 1e-12),
-                         "alg_bytes": nb, "alg_flops": nf,
-                         "gbs": nb / (avg * 1e-3) / 1e9 if avg > 0 else None,
-                         "tflops": nf / (avg * 1e-3) / 1e12 if avg > 0 and nf else None}
-    dom = max(KINDS, key=lambda k_: kt[k_][0])
-    kd = kernels[dom]
-    ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)
-    if kd["alg_flops"] and kd["alg_flops"] / kd["alg_bytes"] > ridge:
-        roof = {"bound": "tensor", "achieved": kd["tflops"], "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s"}
-    else:
-        roof = {"bound": "hbm", "achieved": kd["gbs"], "peak": pk["hbm_gbs"], "unit": "GB/s"}
-    roof["frac"] = roof["achieved"] / roof["peak"] if roof["achieved"] else None
-    tr = recorded_traffic(dom, wl.name, args.reuse)
-    roof["traffic"] = tr
-    roof["kernel"] = dom
-    roof["peak_source"] = f"{pk_src} (MEASURED_PEAKS.json)" if pk_src == "measured" else "fallback"
-    roof["alg_bytes_per_launch"] = kd["alg_bytes"]
-    roof["alg_flops_per_launch"] = kd["alg_flops"]
+    kernels = kernel_table(wl, kt, st_k, K)
+    ffma_peak = None
+    if wl.dtype != "bf16" or args.configs != "none":
+        ffma_peak = runner.M.moeca_probe_ffma(local)[0]
+    dom = max(kernels, key=lambda k_: kernels[k_]["avg_us"] * kernels[k_]["launches"])
+    roof = roofline(dom, kernels[dom], wl, pk, pk_src, ffma_peak)
+    roof["traffic"] = recorded_traffic(dom, wl.name, args.reuse)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -612,45 +738,64 @@ def main():
     es = 2 if wl.dtype == "bf16" else 4
     io_bytes = wl.n_tokens * wl.hidden * es
     cond_bytes = wl.batch * wl.hidden * 4 if wl.adaln else 0
+    runner.close()
+
+    # The other workloads, one row each (rank 0 of a single-GPU run).
+    rows = []
+    want = args.configs
+    if want == "auto":
+        want = "all" if (args.workload == DEFAULT_WORKLOAD and world == 1 and not args.layers) else "none"
+    if want != "none" and rank == 0:
+        idx = [1, 2, 3, 4, 5] if want == "all" else [int(v) for v in want.split(",") if v]
+        for i in idx:
+            if i == wl.index and not wl.n_heads:
+                continue
+            rows.append(config_row(W.workload(i), local, W_, K, pk, pk_src, ffma_peak))
+
     line = {
         "metric": METRIC, "value": head["tokens_per_s"], "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": W_, "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": {"workload": wl.name, "tokens": wl.n_tokens, "hidden": wl.hidden, "experts": wl.n_experts,
-                   "shared_experts": wl.n_shared, "top_k": wl.top_k, "ffn": wl.ffn, "layers": wl.n_layers,
-                   "refresh_period": wl.refresh_period, "reuse_target": args.reuse,
-                   **({"attn_heads": wl.n_heads, "seq_len": wl.seq,
-                       "attn_rows_recomputed_per_step": head["stats"]["attn_recomputed"] / K}
-                      if wl.n_heads else {}),
-                   **({"adaln": True,
-                       "step": "AdaLN modulation of every block from the step's conditioning, the L blocks, "
-                               "then the Eq. 1 update of the step's output (x_t in float32); the blocks' "
-                               "inputs follow the synthetic drift trajectory, not the update, so the reuse "
-                               "ratio is controlled as for the other workloads"}
-                      if wl.adaln else {}),
-                   "reuse_achieved": head["reuse_achieved"], "tau0": head["tau0"],
-                   "effective_tflops": head["effective_tflops"], "executed_tflops": head["executed_tflops"],
-                   "timed": f"median of {args.reps} reps of {K} steps after {W_} warm-up steps (step 0 full)",
-                   "l2": "no flush: each step streams the active experts' weights "
-                         f"({wl.n_layers} x {2 * wl.n_experts * wl.hidden * wl.ffn * es / 1e6:.0f} MB) > 129 MB L2",
-                   "parallelism": f"replicas x{world}"},
+        "config": {"workload": wl.name, "reuse_target": args.reuse},
+        "point": {"tau0": head["tau0"], "tau0_source": head["tau0_source"], "reuse_achieved": head["reuse_achieved"],
+                  "effective_tflops": head["effective_tflops"], "executed_tflops": head["executed_tflops"]},
+        "shape": {"tokens": wl.n_tokens, "hidden": wl.hidden, "experts": wl.n_experts,
+                  "shared_experts": wl.n_shared, "top_k": wl.top_k, "ffn": wl.ffn, "layers": wl.n_layers,
+                  "refresh_period": wl.refresh_period,
+                  **({"attn_heads": wl.n_heads, "seq_len": wl.seq,
+                      "attn_rows_recomputed_per_step": head["stats"]["attn_recomputed"] / K}
+                     if wl.n_heads else {}),
+                  **({"adaln": True,
+                      "step": "AdaLN modulation of every block from the step's conditioning, the L blocks, "
+                              "then the Eq. 1 update of the step's output (x_t in float32); the blocks' "
+                              "inputs follow the synthetic drift trajectory, not the update, so the reuse "
+                              "ratio is controlled as for the other workloads"}
+                     if wl.adaln else {}),
+                  "timed": f"median of {args.reps} reps of {K} steps after {W_} warm-up steps (step 0 full)",
+                  "l2": "no flush: each step streams the active experts' weights "
+                        f"({wl.n_layers} x {2 * wl.n_experts * wl.hidden * wl.ffn * es / 1e6:.0f} MB) > 129 MB L2",
+                  "parallelism": f"replicas x{world}"},
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": {"value": wl.n_tokens * K * world / (e2e_ms / 1e3), "unit": "tokens/s",
                 "h2d_bytes_per_step": io_bytes + cond_bytes, "d2h_bytes_per_step": io_bytes,
-                "pipelining": "each step's upload and read-back run on a copy stream, overlapping the "
-                              "neighbouring steps' compute (double-buffered input and output)"},
+                "how": ("torch copies on a side stream, double-buffered (the AdaLN step ends with the Eq. 1 "
+                        "update of the device output)" if wl.adaln else
+                        "moeca_step_host per step from pinned host input to pinned host output: the library "
+                        "uploads on its own stream into double-buffered staging and reads back on another, so "
+                        "the copies overlap the neighbouring steps' compute; moeca_host_join before the end event")},
         "gpu_launches": sum(kt[k_][1] for k_ in KINDS) + (K if wl.adaln else 0),
         "clocks": head["clocks"],
         "sweep": sweep,
         "kernels": kernels,
+        "fp32_ffma_tflops": ffma_peak,
+        "configs": rows,
     }
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
-    runner.stack.close()
 
 
 if __name__ == "__main__":

@@ -48,3 +48,35 @@ def test_single_rank_needs_no_group():
     import bench
     assert bench.init_group(1, "gloo") is None
     assert bench.aggregate(3.5, 77, None) == (3.5, 77)
+
+
+def test_ffn_algorithmic_bytes_exclude_the_hidden_activations():
+    """The grouped FFN's algorithmic bytes are the active experts' weights,
+    the gathered input rows and the scattered output rows; its bf16 hidden
+    activations are an implementation intermediate (not counted)."""
+    import bench
+    from paper_2606_15615_gb300 import workloads as W
+    wl = W.workload(2)
+    rows, G = 1638.4, 16
+    b, f = bench.algorithmic("ffn", wl, rows, G)
+    D, F = wl.hidden, wl.ffn
+    assert b == 2 * G * F * D * 2 + 2 * rows * D * 2
+    assert f == 4.0 * rows * D * F
+    # 16 experts x 2 x 3072 x 768 x 2 B = 151.0 MB of weights, plus 2 x 1638.4 rows x 768 x 2 B.
+    assert abs(b / 1e6 - 156.03) < 0.05
+
+
+def test_roofline_uses_burst_peaks_and_bounds():
+    import bench
+    from paper_2606_15615_gb300 import workloads as W
+    pk = {"hbm_gbs": 6694.5, "bf16_tflops": 1918.9, "bf16_tflops_sustained": 1733.4}
+    wl = W.workload(2)
+    kd = {"alg_bytes": 156.0e6, "alg_flops": 15.46e9, "avg_us": 50.0, "gbs": 3120.0, "tflops": 309.2}
+    r = bench.roofline("ffn", kd, wl, pk, "measured", None)
+    assert r["bound"] == "hbm" and r["peak"] == 6694.5 and abs(r["frac"] - 3120.0 / 6694.5) < 1e-12
+    kd4 = {"alg_bytes": 400e6, "alg_flops": 350e12 * 1e-3, "avg_us": 300.0, "gbs": 1333.0, "tflops": 1166.7}
+    r4 = bench.roofline("ffn", kd4, W.workload(4), pk, "measured", None)
+    assert r4["bound"] == "tensor" and r4["peak"] == 1918.9  # burst, not sustained
+    kd1 = {"alg_bytes": 20e6, "alg_flops": 1.2e9, "avg_us": 60.0, "gbs": 333.0, "tflops": 20.0}
+    r1 = bench.roofline("ffn2", kd1, W.workload(1), pk, "measured", 75.0)
+    assert r1["bound"] == "fp32" and abs(r1["frac"] - 20.0 / 75.0) < 1e-12
