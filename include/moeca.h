@@ -361,8 +361,9 @@ moeca_status moeca_reset(moeca_handle* h);
 
 /* Host-side fault injection for tests of failure detection (no counterpart
  * in the paper).  MOECA_FAULT_BARRIER_STALL: the next step's fused
- * preparation kernels wait at their grid barriers for an arrival count that
- * never comes; every block gives up after about one second of %globaltimer,
+ * preparation kernels wait at their grid-wide exchanges for values tagged
+ * with a launch number that no launch writes, as if a block never arrived;
+ * every block gives up after about one second of %globaltimer,
  * records MOECA_ERR_TIMEOUT in the device status and skips its later phases,
  * so the step's outputs are garbage and the next call that checks the device
  * status returns MOECA_ERR_TIMEOUT until moeca_reset.  Nothing faults or

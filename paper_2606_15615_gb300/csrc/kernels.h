@@ -149,10 +149,12 @@ struct PrepArgs {
   int32_t* route_e;       // [T, k]
   float* route_w;         // [T, k]
   float* ema;             // [T, E]
-  float* partials;        // [blocks, E, 2]
+  unsigned long long* part_words;   // [blocks, E, 2] tagged (sum C, sum C ln C) per block (exchange 1)
+  unsigned long long* count_words;  // [blocks, groups] tagged recomputed rows per group (exchange 2)
+  unsigned epoch;         // this launch's tag (never 0, never reused before a reset)
+  unsigned wait_epoch;    // the tag the exchanges wait for (epoch, unless a stall is injected)
   float* tau;             // [E] (written by block 0)
   SelectArgs sel;         // decision inputs and outputs (its tau is replaced in-kernel)
-  int32_t* block_counts;  // [blocks, G]
   int32_t* counts;        // [G]
   int32_t* offsets;       // [G + 1]
   int32_t* list;          // [rows]
@@ -170,9 +172,6 @@ struct PrepArgs {
   int32_t* attn_inv;      //   [T] each token's place (-1 if absent),
   int32_t* sample_lo;     //   [T / seq + 1] where each sample's tokens start
   int seq;                //   tokens per sample
-  int region_groups;      // groups the counts region was sized for: prep_region_groups(E, attn)
-  unsigned* gbar;         // grid barrier arrival counter (zeroed once, only grows)
-  unsigned bar_base;      // arrivals on gbar from earlier launches (mod 2^32)
   unsigned long long* stats;
   int* status;
 };
@@ -190,9 +189,6 @@ PrepShape prep_plan_plain(int D, int E, int k, int max_tokens, int n_sms);
 PrepShape prep_plan_attn(int D, int E, int k, int max_tokens, int n_sms);
 cudaError_t launch_prep_plain(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 cudaError_t launch_prep_attn(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
-// Groups of the fused kernel's count scan: E routed + a shared one (sized for
-// always), + the recomputing-token list of a DiT-MoE block.
-inline int prep_region_groups(int E, bool attn) { return E + 1 + (attn ? 1 : 0); }
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 
 // Eq. 8 combine + residual + cached branch norms.

@@ -129,10 +129,11 @@ struct moeca_handle {
   int* tc_work = nullptr;       // GEMM unit tickets {next, CTAs done}, left at 0
   int tc_dep_pairs_n = 0;
   PrepShape prep{0, 0, 0, 0, false};  // fused router + select + compact, when it fits
-  unsigned prep_arrivals = 0;   // grid-barrier arrivals of all fused launches so far (mod 2^32)
-  bool inject_stall = false;    // moeca_inject_fault: next step's barrier targets unreachable
-  int32_t* prep_counts = nullptr;
-  unsigned* prep_bar = nullptr;
+  unsigned prep_epoch = 0;      // tag of the last fused launch (its exchanges' words)
+  bool inject_stall = false;    // moeca_inject_fault: next step's exchanges wait for a tag nobody writes
+  unsigned long long* prep_words = nullptr;  // tagged exchange words: partials, then row counts
+  size_t prep_words_n = 0;
+  size_t prep_count_off = 0;    // where the row-count words start
   void* qkv = nullptr;          // attention workspace: q [T, D] (list order), k [T, D], v^T [D, T]
   int32_t* attn_inv = nullptr;  // [T] each token's place in attn_rows (-1: absent)
   void* attn_o = nullptr;       // [T, D] attention rows before the output projection
@@ -485,8 +486,9 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     h->prep = prep_plan(c.hidden, c.n_experts, c.top_k, c.max_tokens, h->n_sms, attn && !ada);
     if (h->prep.tokens_per_block) {
       const size_t nb = (T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block;
-      A((void**)&h->prep_counts, nb * (G + 1) * 4);
-      A((void**)&h->prep_bar, 2 * sizeof(unsigned));
+      h->prep_count_off = nb * E * 2;
+      h->prep_words_n = h->prep_count_off + nb * (G + 1);
+      A((void**)&h->prep_words, h->prep_words_n * 8);
     }
   }
   h->act.assign(c.n_layers, nullptr);
@@ -702,7 +704,6 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       PrepArgs pa{};
       pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
       pa.n_shared = c.n_shared;
-      pa.region_groups = prep_region_groups(c.n_experts, attn && !ada);
       if (attn && !ada && !attn_full) {
         pa.x = in;
         pa.attn_a = L.attn_a;
@@ -727,14 +728,15 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
       pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
       pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
-      pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.partials = h->partials; pa.tau = L.tau;
+      pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.tau = L.tau;
       pa.sel = sa;
-      pa.block_counts = h->prep_counts; pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
-      pa.xg = xg_now; pa.gbar = h->prep_bar; pa.stats = L.stats; pa.status = h->status_dev;
-      pa.bar_base = h->prep_arrivals;
-      if (h->inject_stall) pa.bar_base += 0x40000000u;  // targets no launch will reach
+      pa.part_words = h->prep_words; pa.count_words = h->prep_words + h->prep_count_off;
+      if (++h->prep_epoch == 0) h->prep_epoch = 1;  // 0 marks words never written
+      pa.epoch = pa.wait_epoch = h->prep_epoch;
+      if (h->inject_stall) pa.wait_epoch = h->prep_epoch ^ 0x80000000u;  // a tag no launch writes
+      pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
+      pa.xg = xg_now; pa.stats = L.stats; pa.status = h->status_dev;
       if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
-      h->prep_arrivals += 2u * static_cast<unsigned>((T + h->prep.tokens_per_block - 1) / h->prep.tokens_per_block);
     } else {
       if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
       if ((e = timed(h, MOECA_K_SELECT, s, [&] { return launch_select(sa, s); })) != cudaSuccess) break;
@@ -1034,10 +1036,10 @@ moeca_status moeca_reset(moeca_handle* h) {
     h->status_host[0] = 0;
     h->status_host[1] = 0;
   }
-  if (h->prep_bar) {
-    cudaError_t e = cudaMemset(h->prep_bar, 0, 2 * sizeof(unsigned));
-    if (e != cudaSuccess) return cuda_fail(h, e, "reset barrier");
-    h->prep_arrivals = 0;
+  if (h->prep_words) {
+    cudaError_t e = cudaMemset(h->prep_words, 0, h->prep_words_n * 8);
+    if (e != cudaSuccess) return cuda_fail(h, e, "reset exchange words");
+    h->prep_epoch = 0;
   }
   // Counters that kernels leave at zero, unless a launch was cut short.
   if (h->tc_dep) {

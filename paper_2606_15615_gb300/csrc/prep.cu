@@ -1,26 +1,35 @@
 // Fused per-layer preparation of the branch-cached MoE layer, one launch
-// (programmatic dependent launch, every block co-resident) with two grid
-// barriers:
+// (programmatic dependent launch, every block co-resident) with two
+// grid-wide exchanges:
 //
 //   A  router (Eq. 7): gate logits on the tensor cores (mma.sync m16n8k16,
-//      bf16 in, fp32 accumulate) from the block's token rows and the gate
-//      matrix staged in shared memory by bulk async copies; fp32 softmax and
-//      top-k with ties to the lower expert id; the EMA statistic (Eq. 10) and
-//      the block's entropy partial sums.
-//   -- grid barrier --
-//   B  every block reduces all blocks' partials in block order to the same
-//      thresholds tau_e (Eq. 11-12), then decides its tokens' branches
-//      (Sec. 4.2, Eq. 9) and counts recomputed rows per expert group.
-//   -- grid barrier --
-//   C  every block scans the per-block counts into group offsets and its own
-//      prefix, writes its rows into the per-group lists (ascending token
-//      order) and gathers their inputs for the grouped FFN.
+//      bf16 in, fp32 accumulate; the warps of a 16-token group split D) from
+//      the block's token rows and the gate matrix staged in shared memory by
+//      bulk async copies; fp32 softmax and top-k with ties to the lower
+//      expert id; the EMA statistic (Eq. 10) and the block's entropy partial
+//      sums, published; then the threshold-free half of each token's
+//      decision (matching, slots, scores; Sec. 4.2, Eq. 9).
+//   -- exchange 1: every block reads all blocks' partials --
+//   B  every block reduces the partials in block order to the same
+//      thresholds tau_e (Eq. 11-12), finishes its tokens' decisions and
+//      publishes its recomputed rows per expert group.
+//   -- exchange 2: every block reads all blocks' row counts --
+//   C  every block forms the group offsets and its own prefix, writes its
+//      rows into the per-group lists (ascending token order) and gathers
+//      their inputs for the grouped FFN.
+//
+// An exchange is data-carrying: each published value is a 64-bit word whose
+// high half is the launch's epoch (a number the host never reuses before a
+// reset), stored and loaded with relaxed GPU-scope accesses (each word is
+// single-copy atomic).  A reader polls the words it needs until every one
+// carries the epoch, so a value and its readiness arrive in the same load:
+// no fence, no arrival counter, one round trip.  The poll is bounded by one
+// second of %globaltimer; on timeout it records MOECA's timeout status and
+// the block skips its later phases.
 //
 // The results are those of router_kernel + select_kernel + compact_kernel,
 // which remain the path for fp32, for shapes whose staging does not fit in
-// shared memory, and for grids that cannot be co-resident.  The grid barrier
-// spins with a one-second bound; on timeout it records MOECA's timeout status
-// and later phases are skipped.
+// shared memory, and for grids that cannot be co-resident.
 #include "common.cuh"
 #include "kernels.h"
 #include "select_token.cuh"
@@ -55,41 +64,56 @@ __device__ __forceinline__ float grp_sum(float v) {
   return v;
 }
 
-// Grid-wide barrier over co-resident blocks (see prep_launch).  *cnt only
-// grows: barrier b (0 or 1) of a launch is passed once it reaches
-// base + (b + 1) * nblocks arrivals, base being the arrivals of all earlier
-// launches (kept by the host).  Arrive is a release add, the wait an
-// acquire poll bounded by one second.  Returns false after a timeout.
-__device__ bool grid_sync(unsigned* cnt, unsigned target, int* status) {
-  __shared__ int ok_sh;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
-    bool ok = true;
-    const unsigned long long t0 = globaltimer();
+// Tagged words of the grid-wide exchanges: payload in the low 32 bits, the
+// launch's epoch in the high 32.
+__device__ __forceinline__ unsigned long long tag_word(uint32_t payload, unsigned epoch) {
+  return (static_cast<unsigned long long>(epoch) << 32) | payload;
+}
+__device__ __forceinline__ void st_word(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_word(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Read n tagged words p[idx(0)] .. p[idx(n - 1)] and hand their payloads to
+// f(j, payload) in order j = 0..n-1.  Words are fetched kB at a time; while
+// any word of a batch still carries another epoch, the batch's stale words
+// are fetched again (one round trip per retry).  Returns false once
+// `deadline` (%globaltimer) has passed.
+template <int kB, typename Idx, typename F>
+__device__ __forceinline__ bool read_tagged(const unsigned long long* p, int n, Idx idx, unsigned epoch,
+                                            unsigned long long deadline, F&& f) {
+  for (int j0 = 0; j0 < n; j0 += kB) {
+    unsigned long long v[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) v[u] = 0ull;  // epoch 0 is never used: every word starts stale
     for (;;) {
-      unsigned v;
-      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(cnt) : "memory");
-      if (static_cast<int>(v - target) >= 0) break;
-      if (globaltimer() - t0 > kBarrierNs) {
-        ok = false;
-        report_status(status, kStatusWaitTimeout, 600);
-        break;
-      }
+#pragma unroll
+      for (int u = 0; u < kB; ++u)
+        if (j0 + u < n && static_cast<unsigned>(v[u] >> 32) != epoch) v[u] = ld_word(p + idx(j0 + u));
+      bool all = true;
+#pragma unroll
+      for (int u = 0; u < kB; ++u) all &= j0 + u >= n || static_cast<unsigned>(v[u] >> 32) == epoch;
+      if (all) break;
+      if (globaltimer() > deadline) return false;
     }
-    ok_sh = ok;
+#pragma unroll
+    for (int u = 0; u < kB; ++u)
+      if (j0 + u < n) f(j0 + u, static_cast<uint32_t>(v[u]));
   }
-  __syncthreads();
-  return ok_sh != 0;
+  return true;
 }
 
 // TB tokens per block (16 or 32); EPAD experts padded to a multiple of 8.
-// Bytes of the region holding the logits (phase A) and, later, the per-block
-// group counts (phase C), rounded up to 16.
-__host__ __device__ constexpr size_t prep_region_bytes(int TB, int EPAD, int n_blocks, int G) {
-  const size_t logits = static_cast<size_t>(TB) * (EPAD + 1) * 4;
-  const size_t counts = static_cast<size_t>(n_blocks) * G * 4;
-  return ((logits > counts ? logits : counts) + 15) / 16 * 16;
+// Bytes of the region holding the partial logits of phase A, one
+// [TB][EPAD + 1] table per warp of a 16-token group (each sums its own range
+// of D), rounded up to 16.
+__host__ __device__ constexpr int prep_wpg(int TB) { return 4 / (TB / 16); }
+__host__ __device__ constexpr size_t prep_region_bytes(int TB, int EPAD) {
+  return (static_cast<size_t>(prep_wpg(TB)) * TB * (EPAD + 1) * 4 + 15) / 16 * 16;
 }
 
 // DiT-MoE block work kept out of line, so the MoE-only path's code (phases
@@ -150,7 +174,6 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   constexpr int NTILE = EPAD / 8;        // mma n-tiles
   constexpr int TOKG = TB / 16;          // 16-token mma groups
   constexpr int WPG = 4 / TOKG;          // warps per token group
-  constexpr int NPW = (NTILE + WPG - 1) / WPG;  // n-tiles per warp
   static_assert(EPL >= 1 && EPL * G == EPAD, "experts per lane");
   extern __shared__ __align__(128) uint8_t dyn[];
   __shared__ float sm_S[TB * EPAD];
@@ -170,6 +193,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __shared__ int sm_rows[TB * (KMAX + 1)][2];
   __shared__ bool sm_any[kAttn ? TB : 1];
   __shared__ int sm_nrows;
+  __shared__ int sm_fail;
   __shared__ __align__(8) uint64_t sm_bar;
   // Per-token inputs of the decision, fetched at the start and kept here.
   __shared__ int32_t sm_re[TB * KMAX];
@@ -184,14 +208,14 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   const int ldw = D + 8;  // padded row, in bf16
   __nv_bfloat16* s_w = reinterpret_cast<__nv_bfloat16*>(dyn);
   __nv_bfloat16* s_x = s_w + EPAD * ldw;
-  float* s_logit = reinterpret_cast<float*>(s_x + TB * ldw);  // [TB][EPAD + 1]
+  float* s_logit = reinterpret_cast<float*>(s_x + TB * ldw);  // [WPG][TB][EPAD + 1]
   const int tok0 = blockIdx.x * TB;
   const int ntok = min(TB, T - tok0);
   // DiT-MoE block on a cache step: the cached attention rows, after the
-  // logits / counts region (sized as prep_smem sizes it for this grid).
+  // logits region.
   const bool add_a = kAttn && a.attn_a != nullptr;
-  __nv_bfloat16* s_a = reinterpret_cast<__nv_bfloat16*>(
-      reinterpret_cast<uint8_t*>(s_logit) + prep_region_bytes(TB, EPAD, gridDim.x, a.region_groups));
+  __nv_bfloat16* s_a = reinterpret_cast<__nv_bfloat16*>(reinterpret_cast<uint8_t*>(s_logit) +
+                                                        prep_region_bytes(TB, EPAD));
 
   // ---- A0: stage gate rows and token rows ----
   // Before the programmatic-dependency wait: everything that the previous
@@ -202,6 +226,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   if (t == 0) {
     sm_near = 0;
     sm_nrows = 0;
+    sm_fail = 0;
     mbar_init(smem_u32(&sm_bar), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -255,39 +280,53 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
 
   // ---- A1: logits on the tensor cores ----
+  // The WPG warps of a 16-token group each take a contiguous range of the
+  // D / 16 k-steps and every n-tile over it, with two interleaved
+  // accumulator chains and the next step's fragments loaded ahead; each
+  // warp's partial logits go to its own table, added in range order below.
   {
-    const int tg = warp / WPG;               // token group of this warp
-    const int nt0 = (warp % WPG) * NPW;      // first n-tile of this warp
-    float acc[NPW][4];
+    const int tg = warp / WPG, h = warp % WPG;
+    const int KS = D / 16;
+    const int ks0 = h * KS / WPG, ks1 = (h + 1) * KS / WPG;
+    float acc[2][NTILE][4];
 #pragma unroll
-    for (int j = 0; j < NPW; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
-    if (tg < TOKG && nt0 < NTILE) {
+    for (int c = 0; c < 2; ++c)
+#pragma unroll
+      for (int j = 0; j < NTILE; ++j) acc[c][j][0] = acc[c][j][1] = acc[c][j][2] = acc[c][j][3] = 0.f;
+    if (tg < TOKG) {
       const uint32_t a_addr = smem_u32(s_x + (tg * 16 + (lane & 15)) * ldw + (lane >> 4) * 8);
       const int bl = lane & 15;
-      for (int k0 = 0; k0 < D; k0 += 16) {
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
+      uint32_t b_addr[NTILE];
 #pragma unroll
-        for (int j = 0; j < NPW; ++j) {
-          const int nt = nt0 + j;
-          if (nt < NTILE) {
-            uint32_t b0, b1;
-            ldsm_x2(smem_u32(s_w + (nt * 8 + (bl & 7)) * ldw + k0 + (bl >> 3) * 8), b0, b1);
-            mma_16816(acc[j], a0, a1, a2, a3, b0, b1);
-          }
+      for (int j = 0; j < NTILE; ++j) b_addr[j] = smem_u32(s_w + (j * 8 + (bl & 7)) * ldw + (bl >> 3) * 8);
+      uint32_t A[4], B[NTILE][2];
+      auto load = [&](int ks, uint32_t* Ar, uint32_t (*Br)[2]) {
+        ldsm_x4(a_addr + ks * 32, Ar[0], Ar[1], Ar[2], Ar[3]);
+#pragma unroll
+        for (int j = 0; j < NTILE; ++j) ldsm_x2(b_addr[j] + ks * 32, Br[j][0], Br[j][1]);
+      };
+      if (ks0 < ks1) load(ks0, A, B);
+      for (int ks = ks0; ks < ks1; ks += 2) {
+        uint32_t A1[4], B1[NTILE][2];
+        const bool two = ks + 1 < ks1;
+        if (two) load(ks + 1, A1, B1);
+#pragma unroll
+        for (int j = 0; j < NTILE; ++j) mma_16816(acc[0][j], A[0], A[1], A[2], A[3], B[j][0], B[j][1]);
+        if (two) {
+          if (ks + 2 < ks1) load(ks + 2, A, B);
+#pragma unroll
+          for (int j = 0; j < NTILE; ++j) mma_16816(acc[1][j], A1[0], A1[1], A1[2], A1[3], B1[j][0], B1[j][1]);
         }
       }
       const int g = lane >> 2, c2 = (lane & 3) * 2;
+      float* tab = s_logit + h * TB * (EPAD + 1);
 #pragma unroll
-      for (int j = 0; j < NPW; ++j) {
-        const int nt = nt0 + j;
-        if (nt < NTILE) {
-          const int r0 = tg * 16 + g, e0 = nt * 8 + c2;
-          s_logit[r0 * (EPAD + 1) + e0] = acc[j][0];
-          s_logit[r0 * (EPAD + 1) + e0 + 1] = acc[j][1];
-          s_logit[(r0 + 8) * (EPAD + 1) + e0] = acc[j][2];
-          s_logit[(r0 + 8) * (EPAD + 1) + e0 + 1] = acc[j][3];
-        }
+      for (int j = 0; j < NTILE; ++j) {
+        const int r0 = tg * 16 + g, e0 = j * 8 + c2;
+        tab[r0 * (EPAD + 1) + e0] = acc[0][j][0] + acc[1][j][0];
+        tab[r0 * (EPAD + 1) + e0 + 1] = acc[0][j][1] + acc[1][j][1];
+        tab[(r0 + 8) * (EPAD + 1) + e0] = acc[0][j][2] + acc[1][j][2];
+        tab[(r0 + 8) * (EPAD + 1) + e0 + 1] = acc[0][j][3] + acc[1][j][3];
       }
     }
   }
@@ -304,7 +343,10 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     for (int j = 0; j < EPL; ++j) {
       const int e = g + G * j;
       if (e < E) {
-        zl[j] = s_logit[tok * (EPAD + 1) + e] + (a.b_gate ? a.b_gate[e] : 0.f);
+        float z = 0.f;
+#pragma unroll
+        for (int hh = 0; hh < WPG; ++hh) z += s_logit[(hh * TB + tok) * (EPAD + 1) + e];
+        zl[j] = z + (a.b_gate ? a.b_gate[e] : 0.f);
         lmax = fmaxf(lmax, zl[j]);
         labs = fmaxf(labs, fabsf(zl[j]));
       } else {
@@ -394,9 +436,10 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     }
   }
   __syncthreads();
+  const unsigned epoch = a.epoch;
   {
     // Block partials per expert: J interleaved runs over the block's tokens,
-    // added in run order.
+    // added in run order, then published.
     const int J = kThreads / E;
     const int e = t % E, jr = t / E;
     float S = 0.f, U = 0.f;
@@ -414,30 +457,47 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         Ss += sm_rs[q * E + t][0];
         Us += sm_rs[q * E + t][1];
       }
-      reinterpret_cast<float2*>(a.partials)[static_cast<size_t>(blockIdx.x) * E + t] = make_float2(Ss, Us);
+      unsigned long long* pw = a.part_words + (static_cast<size_t>(blockIdx.x) * E + t) * 2;
+      st_word(pw, tag_word(__float_as_uint(Ss), epoch));
+      st_word(pw + 1, tag_word(__float_as_uint(Us), epoch));
     }
     if (t == 0 && sm_near) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(sm_near));
   }
-  __threadfence();
-  if (!grid_sync(a.gbar, a.bar_base + gridDim.x, a.status)) return;
 
-  // ---- B: thresholds from every block's partials (same order in every block) ----
+  // The threshold-free half of the decisions (warp 0, one token per lane),
+  // while the other blocks publish their partials.
+  TokenPrepT<KMAX> tp;
+  if (warp == 0) {
+    const bool valid = lane < ntok;
+    const int q = valid ? lane * k : 0;
+    prepare_token(a.sel, tok0 + lane, valid, sm_re + q, sm_rw + q, sm_ce + q, sm_cw + q, sm_cn + q, tp);
+  }
+
+  // ---- exchange 1, B: thresholds from every block's partials (same order in every block) ----
+  __syncthreads();  // sm_rs is rewritten below: the block-partial reads above are done
   {
     const int J = kThreads / E;
     const int e = t % E, j = t / E;
+    const int nb = gridDim.x;
     float S = 0.f, U = 0.f;
+    bool ok = true;
     if (j < J) {
-      const float2* part = reinterpret_cast<const float2*>(a.partials);
-#pragma unroll 8
-      for (unsigned b = j; b < gridDim.x; b += J) {
-        const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
-        S += v.x;
-        U += v.y;
-      }
+      const int n = 2 * ((nb - j + J - 1) / J);  // (S, U) of blocks j, j + J, ...
+      ok = read_tagged<8>(
+          a.part_words, n, [&](int q) { return (static_cast<size_t>(j + (q >> 1) * J) * E + e) * 2 + (q & 1); },
+          a.wait_epoch, globaltimer() + kBarrierNs, [&](int q, uint32_t v) {
+            if (q & 1) U += __uint_as_float(v);
+            else S += __uint_as_float(v);
+          });
+    }
+    if (!ok) {
+      report_status(a.status, kStatusWaitTimeout, 600);
+      sm_fail = 1;
     }
     sm_rs[t][0] = S;
     sm_rs[t][1] = U;
     __syncthreads();
+    if (sm_fail) return;
     if (t < E) {
       float Ss = 0.f, Us = 0.f;
       for (int jj = 0; jj < J; ++jj) {
@@ -477,32 +537,28 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     __syncthreads();
   }
 
-  // ---- B: branch decisions of the block's tokens (warp 0, one token per lane) ----
+  // ---- B: finish the block's decisions (warp 0), publish its rows per group ----
   const int GG = a.G + ((kAttn && a.attn_list) ? 1 : 0);  // the attention list is group G, after the FFN groups
   TokenDecisionT<KMAX> d;
   if (warp == 0) {
-    SelectArgs sa = a.sel;
-    sa.tau = sm_tau;
     const bool valid = lane < ntok;
-    const int q = valid ? lane * k : 0;
-    decide_token(sa, tok0 + lane, valid, sm_re + q, sm_rw + q, sm_ce + q, sm_cw + q, sm_cn + q, d);
+    finish_token(a.sel, tok0 + lane, tp, sm_tau, d);
     int n_full = (valid && !d.bad && !d.any) ? 1 : 0;
-    for (int g = 0; g < GG; ++g) {
-      bool has = false;
-      if (g < E) {
+    // The groups this lane's token has a row in: its recomputed experts, the
+    // shared expert, and (DiT-MoE block) the list of recomputing tokens.
+    uint32_t gm[3] = {0u, 0u, 0u};
 #pragma unroll
-        for (int p = 0; p < KMAX; ++p) has |= (d.rec[p] && d.e[p] == g);
-      } else if (g < a.G) {
-        has = d.shared_row;
-      } else {
-        has = valid && d.any;  // recomputes its attention (Sec. 4.1)
-      }
-      const unsigned b = __ballot_sync(0xffffffffu, has);
-      if (lane == 0) {
-        sm_bal[g] = b;
-        a.block_counts[static_cast<size_t>(blockIdx.x) * GG + g] = __popc(b);
-      }
+    for (int p = 0; p < KMAX; ++p)
+      if (d.rec[p]) gm[d.e[p] >> 5] |= 1u << (d.e[p] & 31);
+    if (d.shared_row) gm[E >> 5] |= 1u << (E & 31);
+    if ((kAttn && a.attn_list) && valid && d.any) gm[a.G >> 5] |= 1u << (a.G & 31);
+    for (int g = 0; g < GG; ++g) {
+      const unsigned b = __ballot_sync(0xffffffffu, (gm[g >> 5] >> (g & 31)) & 1u);
+      if (lane == (g & 31)) sm_bal[g] = b;
     }
+    __syncwarp();
+    for (int g = lane; g < GG; g += 32)
+      st_word(a.count_words + static_cast<size_t>(blockIdx.x) * GG + g, tag_word(__popc(sm_bal[g]), epoch));
     const int c_matched = warp_sum_i(d.n_matched), c_rec = warp_sum_i(d.n_rec), c_near = warp_sum_i(d.n_near);
     const int c_full = warp_sum_i(n_full), c_shared = warp_sum_i(d.shared_row ? 1 : 0);
     if (lane == 0) {
@@ -510,7 +566,7 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       atomicAdd(st + kStRecomputed, static_cast<unsigned long long>(c_rec));
       atomicAdd(st + kStReused, static_cast<unsigned long long>(ntok * k - c_rec));
       if (c_shared) atomicAdd(st + kStSharedRecomputed, static_cast<unsigned long long>(c_shared));
-      if (!sa.refresh) {
+      if (!a.sel.refresh) {
         atomicAdd(st + kStMatched, static_cast<unsigned long long>(c_matched));
         atomicAdd(st + kStTokensFullyReused, static_cast<unsigned long long>(c_full));
         if (c_near) atomicAdd(st + kStNearScore, static_cast<unsigned long long>(c_near));
@@ -519,67 +575,47 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         const unsigned long long br = static_cast<unsigned long long>(T) * k;
         atomicAdd(st + kStLayerSteps, 1ull);
         atomicAdd(st + kStBranches, br);
-        if (sa.refresh) atomicAdd(st + kStRefreshSteps, 1ull);
+        if (a.sel.refresh) atomicAdd(st + kStRefreshSteps, 1ull);
         else atomicAdd(st + kStCacheBranches, br);
       }
     }
   }
-  __threadfence();
-  if (!grid_sync(a.gbar, a.bar_base + 2 * gridDim.x, a.status)) return;
 
-  // ---- C: group offsets, this block's prefix, row lists and row gather ----
+  // ---- exchange 2, C: group offsets, this block's prefix, row lists and row gather ----
   {
     const int nb = gridDim.x;
-    int* s_cnt = reinterpret_cast<int*>(s_logit);  // [nb][GG], after the staged rows (the logits are done)
-    {
-      // All loads in flight before any store.
-      constexpr int kU = 8;
-      for (int base = 0; base < nb * GG; base += kThreads * kU) {
-        int v[kU];
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int idx = base + u * kThreads + t;
-          v[u] = idx < nb * GG ? __ldcg(a.block_counts + idx) : 0;
-        }
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int idx = base + u * kThreads + t;
-          if (idx < nb * GG) s_cnt[idx] = v[u];
-        }
-      }
-    }
-    __syncthreads();
     // Per group: rows of the blocks before this one and of all blocks.  Each
-    // group's sum is split over kThreads / GG threads (block ranges), whose
-    // parts are then added in range order.
+    // group's blocks are split over kThreads / GG threads (block ranges),
+    // whose parts are then added in range order.
     {
-      const int R = GG <= kThreads ? kThreads / GG : 1;
+      const int R = kThreads / GG;
       const int g = t % GG, j = t / GG;
       int pre = 0, tot = 0;
-      if (j < R && t < R * GG) {
+      bool ok = true;
+      if (j < R) {
         const int b0 = j * nb / R, b1 = (j + 1) * nb / R;
-        for (int b = b0; b < b1; ++b) {
-          const int c = s_cnt[b * GG + g];
-          if (b < static_cast<int>(blockIdx.x)) pre += c;
-          tot += c;
-        }
+        const int me = static_cast<int>(blockIdx.x);
+        ok = read_tagged<8>(
+            a.count_words, b1 - b0, [&](int q) { return static_cast<size_t>(b0 + q) * GG + g; }, a.wait_epoch,
+            globaltimer() + kBarrierNs, [&](int q, uint32_t v) {
+              const int c = static_cast<int>(v);
+              if (b0 + q < me) pre += c;
+              tot += c;
+            });
+      }
+      if (!ok) {
+        report_status(a.status, kStatusWaitTimeout, 601);
+        sm_fail = 1;
       }
       sm_rs[t][0] = __int_as_float(pre);
       sm_rs[t][1] = __int_as_float(tot);
       __syncthreads();
+      if (sm_fail) return;
       for (int gg = t; gg < GG; gg += kThreads) {
         int p2 = 0, t2 = 0;
-        if (R * GG <= kThreads) {
-          for (int jj = 0; jj < R; ++jj) {
-            p2 += __float_as_int(sm_rs[jj * GG + gg][0]);
-            t2 += __float_as_int(sm_rs[jj * GG + gg][1]);
-          }
-        } else {  // more groups than threads: plain loop over blocks
-          for (int b = 0; b < nb; ++b) {
-            const int c = s_cnt[b * GG + gg];
-            if (b < static_cast<int>(blockIdx.x)) p2 += c;
-            t2 += c;
-          }
+        for (int jj = 0; jj < R; ++jj) {
+          p2 += __float_as_int(sm_rs[jj * GG + gg][0]);
+          t2 += __float_as_int(sm_rs[jj * GG + gg][1]);
         }
         sm_pre[gg] = p2;
         sm_tot[gg] = t2;
@@ -618,6 +654,18 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       const bool track = kAttn && a.row_of != nullptr;  // DiT-MoE block, sync rule: record the FFN rows
       int pos_of[KMAX];
       int shared_pos = -1;
+      // This lane's slots in the block's row table: after the rows of lower lanes.
+      int nr = d.shared_row ? 1 : 0;
+#pragma unroll
+      for (int p = 0; p < KMAX; ++p) nr += d.rec[p] ? 1 : 0;
+      int r = nr;
+#pragma unroll
+      for (int dd = 1; dd < 32; dd <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, r, dd);
+        if (lane >= dd) r += u;
+      }
+      if (lane == 31) sm_nrows = r;
+      r -= nr;
 #pragma unroll
       for (int p = 0; p < KMAX; ++p) {
         if (track) pos_of[p] = -1;
@@ -626,16 +674,15 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
           const int pos = sm_off[g] + sm_pre[g] + __popc(sm_bal[g] & lt);
           a.list[pos] = i * k + d.sl[p];
           if (track) pos_of[p] = pos;
-          const int r = atomicAdd(&sm_nrows, 1);
           sm_rows[r][0] = pos;
           sm_rows[r][1] = i;
+          ++r;
         }
       }
       if (d.shared_row) {
         const int pos = sm_off[E] + sm_pre[E] + __popc(sm_bal[E] & lt);
         a.list[pos] = i;
         shared_pos = pos;
-        const int r = atomicAdd(&sm_nrows, 1);
         sm_rows[r][0] = pos;
         sm_rows[r][1] = i;
       }
@@ -667,11 +714,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
 }
 
 template <int TB, int EPAD>
-size_t prep_smem(int D, int n_blocks, int G, bool attn) {  // G: groups of the counts region
+size_t prep_smem(int D, bool attn) {
   const size_t ldw = static_cast<size_t>(D) + 8;
   const size_t rows = (EPAD + TB) * ldw * 2;                        // gate rows, token rows
   const size_t a_rows = attn ? TB * ldw * 2 : 0;                    // cached attention rows
-  return rows + prep_region_bytes(TB, EPAD, n_blocks, G) + a_rows;
+  return rows + prep_region_bytes(TB, EPAD) + a_rows;
 }
 
 template <int TB, int EPAD, int KMAX>
@@ -748,7 +795,7 @@ PrepShape prep_plan_plain(int D, int E, int k, int max_tokens, int n_sms) {
     const int nb = (max_tokens + TB - 1) / TB;
     const size_t smem = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> size_t {
       if constexpr (tb == 0) return 0;
-      else return prep_smem<tb, ep>(D, nb, prep_region_groups(E, attn), attn);
+      else return prep_smem<tb, ep>(D, attn);
     });
     if (smem == 0 || smem > kPrepSmemMax) continue;
     const int occ = with_shape(TB, epad, km, [&]<int tb, int ep, int kk>() -> int {
