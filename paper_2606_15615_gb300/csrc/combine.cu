@@ -1,7 +1,8 @@
 // Combine of fresh and cached branch outputs (Eq. 8) with the residual of
 // Eq. 5 / Eq. 6, and the cached-norm refresh that Eq. 9's o reads next step.
 //
-// One warp per token, 16-byte vectors over D:
+// Two forms: a staged one (combine_staged_kernel, the default, below) and a
+// direct one (combine_kernel: one warp per token, 16-byte vectors over D):
 //   y_i = sum_{p=1..k} w_{i,p}^t cache_h[i, slot(p)]  (+ shared_h[i])
 //   out_i = x_i + y_i            (fp32 accumulation in p order, rounded once)
 //   out_i = x_i + g_i * y_i      in an AdaLN block (g the sample's MoE gate, Sec. 3)
@@ -174,6 +175,180 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   }
 }
 
+// Staged form (the default): each warp walks its tokens i = w, w + W, ...
+// (w its global warp index, W the grid's warps) and stages a token's rows in
+// shared memory with bulk copies, lane 0 issuing them onto one mbarrier per
+// buffer: the token's k cache rows (one contiguous [k, D] block; slot is a
+// permutation of 0..k-1, so these are all the rows Eq. 8 and the norms read),
+// its shared-expert row and its residual row.  Two buffers per warp: the next
+// token's rows are in flight while this one is combined, so every warp keeps
+// a whole token's bytes in flight and no lane waits on more than one round
+// trip per token.  Arithmetic and its order are those of combine_kernel.
+constexpr int kStagedWarps = 4;
+
+template <typename TI>
+__host__ __device__ inline size_t staged_buf_bytes(int k, int n_shared, int D) {
+  return (static_cast<size_t>(k + n_shared + 1) * D * sizeof(TI) + 127) / 128 * 128;
+}
+
+template <typename TI, int KMAX, bool GATED>
+__global__ void __launch_bounds__(kStagedWarps * 32) combine_staged_kernel(CombineArgs a) {
+  constexpr int V = Elem<TI>::kVec;
+  extern __shared__ __align__(128) uint8_t dyn[];
+  __shared__ __align__(8) uint64_t bars[kStagedWarps][2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = a.k, D = a.D, nvec = D / V, T = a.T;
+  const bool has_sh = a.shared_h != nullptr;
+  const size_t row_bytes = static_cast<size_t>(D) * sizeof(TI);
+  const size_t buf_bytes = staged_buf_bytes<TI>(k, has_sh ? 1 : 0, D);
+  uint8_t* wbuf = dyn + static_cast<size_t>(warp) * 2 * buf_bytes;
+  const uint32_t bar0 = smem_u32(&bars[warp][0]), bar1 = smem_u32(&bars[warp][1]);
+  const int nw = gridDim.x * kStagedWarps;
+  int i = blockIdx.x * kStagedWarps + warp;
+  if (lane == 0) {
+    mbar_init(bar0, 1);
+    mbar_init(bar1, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  const TI* ch = static_cast<const TI*>(a.cache_h);
+  const TI* sh = static_cast<const TI*>(a.shared_h);
+  const TI* xin = static_cast<const TI*>(a.x);
+  const uint32_t tx = static_cast<uint32_t>(row_bytes) * (k + (has_sh ? 1 : 0) + 1);
+  // Lane 0 stages token t into buffer b; the residual row (an earlier
+  // kernel's output) may go before the dependency wait, the cache and shared
+  // rows (the previous kernel's output) only after it.
+  auto issue_rows = [&](int t, int b) {
+    const uint32_t dst = smem_u32(wbuf + b * buf_bytes), bar = b ? bar1 : bar0;
+    bulk_g2s(dst, ch + static_cast<size_t>(t) * k * D, static_cast<uint32_t>(row_bytes) * k, bar);
+    if (has_sh) bulk_g2s(dst + static_cast<uint32_t>(row_bytes) * k, sh + static_cast<size_t>(t) * D,
+                         static_cast<uint32_t>(row_bytes), bar);
+  };
+  auto issue_x = [&](int t, int b) {
+    const uint32_t dst = smem_u32(wbuf + b * buf_bytes), bar = b ? bar1 : bar0;
+    mbar_expect_tx(bar, tx);
+    bulk_g2s(dst + static_cast<uint32_t>(row_bytes) * (k + (has_sh ? 1 : 0)), xin + static_cast<size_t>(t) * D,
+             static_cast<uint32_t>(row_bytes), bar);
+  };
+  if (lane == 0 && i < T) issue_x(i, 0);
+  pdl_entry();
+  if (a.rearm && blockIdx.x == 0 && threadIdx.x == 0) *a.rearm = 0;  // the grouped GEMM before has ended
+  if (lane == 0 && i < T) issue_rows(i, 0);
+  uint32_t phase = 0u;  // bit b: parity of buffer b's next completion
+  for (int b = 0; i < T; i += nw, b ^= 1) {
+    const int nx = i + nw;
+    if (lane == 0 && nx < T) {
+      issue_x(nx, b ^ 1);
+      issue_rows(nx, b ^ 1);
+    }
+    float w[KMAX];
+    int q[KMAX];
+    bool bad = false;
+#pragma unroll
+    for (int p = 0; p < KMAX; ++p) {
+      w[p] = 0.f;
+      q[p] = 0;
+      if (p < k) {
+        w[p] = a.route_w[static_cast<size_t>(i) * k + p];
+        q[p] = a.slot[static_cast<size_t>(i) * k + p];
+        if (q[p] < 0 || q[p] >= k) bad = true;
+      }
+    }
+    const bool ok = mbar_wait_for(b ? bar1 : bar0, (phase >> b) & 1u, 1000000000ull);
+    phase ^= 1u << b;
+    if (!ok) {
+      // The copies never completed: record it, let the next token's copies
+      // (if issued) land before this warp leaves its shared memory, stop.
+      if (lane == 0) {
+        report_status(a.status, kStatusWaitTimeout, 3100000 + i);
+        if (nx < T) mbar_wait_for(b ? bar0 : bar1, (phase >> (b ^ 1)) & 1u, 1000000000ull);
+      }
+      __syncwarp();
+      return;
+    }
+    if (bad) {
+      if (lane == 0) report_status(a.status, kStatusBadIndex, 3000000 + i);
+      __syncwarp();
+      continue;
+    }
+    const uint8_t* buf = wbuf + b * buf_bytes;
+    const uint4* hrow = reinterpret_cast<const uint4*>(buf);
+    const uint4* srow = reinterpret_cast<const uint4*>(buf + row_bytes * k);
+    const uint4* xrow = reinterpret_cast<const uint4*>(buf + row_bytes * (k + (has_sh ? 1 : 0)));
+    const float* gr = GATED ? a.gate + static_cast<size_t>(i / a.seq) * a.gate_ld : nullptr;
+    TI* out = static_cast<TI*>(a.out) + static_cast<size_t>(i) * D;
+    float ss[KMAX];
+#pragma unroll
+    for (int p = 0; p < KMAX; ++p) ss[p] = 0.f;
+    for (int c = lane; c < nvec; c += 32) {
+      float y[V];
+#pragma unroll
+      for (int j = 0; j < V; ++j) y[j] = 0.f;
+#pragma unroll
+      for (int p = 0; p < KMAX; ++p) {
+        if (p < k) {
+          float hv[V];
+          unpack_vec(hrow[static_cast<size_t>(q[p]) * nvec + c], hv, static_cast<TI*>(nullptr));
+#pragma unroll
+          for (int j = 0; j < V; ++j) {
+            y[j] = fmaf(w[p], hv[j], y[j]);
+            ss[p] = fmaf(hv[j], hv[j], ss[p]);
+          }
+        }
+      }
+      if (has_sh) {
+        float hv[V];
+        unpack_vec(srow[c], hv, static_cast<TI*>(nullptr));
+#pragma unroll
+        for (int j = 0; j < V; ++j) y[j] += hv[j];
+      }
+      float xs[V];
+      unpack_vec(xrow[c], xs, static_cast<TI*>(nullptr));
+      if constexpr (GATED) {
+        float gv[V];
+#pragma unroll
+        for (int j = 0; j < V / 4; ++j) {
+          const float4 g4 = __ldg(reinterpret_cast<const float4*>(gr + c * V) + j);
+          gv[4 * j] = g4.x; gv[4 * j + 1] = g4.y; gv[4 * j + 2] = g4.z; gv[4 * j + 3] = g4.w;
+        }
+#pragma unroll
+        for (int j = 0; j < V; ++j) xs[j] = fmaf(gv[j], y[j], xs[j]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < V; ++j) xs[j] += y[j];
+      }
+      store_vec(out + c * V, xs);
+    }
+#pragma unroll
+    for (int p = 0; p < KMAX; ++p) {
+      if (p < k) {
+        const float s2 = warp_sum(ss[p]);
+        if (lane == 0) a.cache_norm[static_cast<size_t>(i) * k + q[p]] = sqrtf(s2);
+      }
+    }
+    __syncwarp();  // every lane is done with buffer b before lane 0 refills it
+  }
+}
+
+template <typename TI, bool GATED>
+cudaError_t launch_staged(const CombineArgs& a, cudaStream_t s) {
+  const size_t smem = static_cast<size_t>(kStagedWarps) * 2 * staged_buf_bytes<TI>(a.k, a.shared_h ? 1 : 0, a.D);
+  auto run = [&](auto kern) -> cudaError_t {
+    cudaError_t e = set_dyn_smem_on_device(reinterpret_cast<const void*>(kern), static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kStagedWarps * 32, smem)) != cudaSuccess)
+      return e;
+    long long grid = (a.T + kStagedWarps - 1) / kStagedWarps;
+    const long long cap = static_cast<long long>(a.n_sms > 0 ? a.n_sms : 1) * (per_sm > 0 ? per_sm : 1);
+    if (grid > cap) grid = cap;
+    return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(kStagedWarps * 32), smem, s, a);
+  };
+  if (a.k <= 2) return run(combine_staged_kernel<TI, 2, GATED>);
+  if (a.k <= 4) return run(combine_staged_kernel<TI, 4, GATED>);
+  return run(combine_staged_kernel<TI, 8, GATED>);
+}
+
 template <typename TI, bool GATED, bool YC>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
@@ -195,6 +370,21 @@ void launch_y(const CombineArgs& a, bool bf16, cudaStream_t s) {
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s) {
   if (a.gate && !bf16) return cudaErrorInvalidValue;  // AdaLN blocks are bf16 only
   if (a.cache_y && (!a.token_any || reinterpret_cast<uintptr_t>(a.cache_y) % 16)) return cudaErrorInvalidValue;
+  if (a.T <= 0) return cudaSuccess;
+  // The staged form while a warp's two buffers take at most 24 KB, so that
+  // two blocks (8 warps) fit an SM: with larger tokens (D 2560 with a shared
+  // expert, top-8 at D 1152: about 41 KB a warp) a block of 4 warps per SM
+  // measured slower than the direct form's 24 warps (31 vs 26 us, 40 vs 27 us
+  // per launch).  The 16-byte alignment of every staged row holds for D a
+  // multiple of the vector width.  The token-level reading of Sec. 4.1
+  // (cache_y) keeps the direct form.
+  const size_t per_warp = 2 * (bf16 ? staged_buf_bytes<__nv_bfloat16>(a.k, a.shared_h ? 1 : 0, a.D)
+                                    : staged_buf_bytes<float>(a.k, a.shared_h ? 1 : 0, a.D));
+  if (!a.cache_y && !a.direct && per_warp <= 24 * 1024 && reinterpret_cast<uintptr_t>(a.x) % 16 == 0) {
+    if (bf16 && a.gate) return launch_staged<__nv_bfloat16, true>(a, s);
+    if (bf16) return launch_staged<__nv_bfloat16, false>(a, s);
+    return launch_staged<float, false>(a, s);
+  }
   if (a.cache_y) launch_y<true>(a, bf16, s);
   else launch_y<false>(a, bf16, s);
   return cudaGetLastError();

@@ -209,6 +209,8 @@ struct CombineArgs {
   const uint8_t* token_any;  // [T] recompute set non-empty (with cache_y)
   int copy_y;             // 1: a token with token_any 0 takes y = cache_y (a cache step under
                           //   token_reuse_policy 1); 0: every token computes y (and stores it)
+  int n_sms;              // the device's SM count (the staged form's persistent grid)
+  int direct;             // 1: force the direct form (one warp per token, rows loaded by the lanes)
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);

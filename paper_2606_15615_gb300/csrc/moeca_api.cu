@@ -306,6 +306,7 @@ void moeca_config_default(moeca_config* c) {
   c->ln_eps = 1e-6f;
   c->keep_route_in = 0;
   c->token_reuse_policy = 0;
+  c->combine_direct = 0;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -351,6 +352,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   if (c.refresh_period < 0) return fail(nullptr, MOECA_ERR_INVALID_ARG, "refresh_period < 0");
   if (c.token_reuse_policy != 0 && c.token_reuse_policy != 1)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "token_reuse_policy must be 0 or 1");
+  if (c.combine_direct != 0 && c.combine_direct != 1)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "combine_direct must be 0 or 1");
   if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
   if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&
@@ -800,6 +803,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       cb.gate = mod_l + 5 * c.hidden; cb.gate_ld = static_cast<int>(mod_ld); cb.seq = seq;
     }
     cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
+    cb.n_sms = h->n_sms; cb.direct = c.combine_direct;
     if (L.cache_y) {
       // Sec. 4.1, token level: a token with an empty recompute set returns y^{t0}.
       cb.cache_y = L.cache_y; cb.token_any = L.token_any; cb.copy_y = refresh ? 0 : 1;

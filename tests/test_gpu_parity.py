@@ -224,3 +224,33 @@ def test_tc_and_simt_agree(M):
         res.append(np_of(st.step(x, 0)))
         st.close()
     assert rel_l2(res[0], res[1]) < 5e-3
+
+
+@pytest.mark.parametrize("shape", [
+    dict(T=300, D=256, E=8, k=2, F=256, S=1, bf16=True),
+    dict(T=257, D=128, E=16, k=8, F=128, S=0, bf16=True),
+    dict(T=190, D=128, E=8, k=2, F=128, S=0, bf16=False)])
+def test_staged_and_direct_combine_agree(M, shape):
+    """The staged combine (rows brought into shared memory by bulk copies,
+    two tokens in flight per warp) and the direct one give the same bits:
+    outputs, cached norms and cache rows, over cache steps with reuse."""
+    sh = dict(shape)
+    bf16 = sh.pop("bf16")
+    outs, states = [], []
+    for direct in (0, 1):
+        st, cfg, ws = make_stack(M, sh["T"], sh["D"], sh["E"], sh["k"], sh["F"], L=2, S=sh["S"], bf16=bf16,
+                                 seed=31, bias=sh["S"] > 0, tau0=0.75 if sh["k"] == 2 else 0.25, combine_direct=direct)
+        rng = np.random.default_rng(310)
+        xs = drift(rng.standard_normal((sh["T"], sh["D"])).astype(np.float32), rng, 4, 0.05, bf16)
+        dt = torch.bfloat16 if bf16 else torch.float32
+        o = [st.step(torch.from_numpy(x).cuda().to(dt), t).clone() for t, x in enumerate(xs)]
+        torch.cuda.synchronize()
+        outs.append(o)
+        states.append([st.get_state(l) for l in range(2)])
+        assert st.stats()["reused"] > 0
+        st.close()
+    for a, b in zip(outs[0], outs[1]):
+        assert torch.equal(a, b)
+    for sa, sb in zip(states[0], states[1]):
+        for key in ("cache_norm", "cache_h", "cache_e", "cache_w"):
+            assert torch.equal(sa[key], sb[key]), key
