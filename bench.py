@@ -213,7 +213,11 @@ def recorded_traffic(kind: str, workload: str, reuse_target: float):
 # ---------------------------------------------------------------------------
 
 class Runner:
-    def __init__(self, wl, device_index: int, n_steps: int, tile_n: int = 0, split_k: int = 0):
+    """One workload on one GPU.  With ``shard = (rank, world)`` the handle
+    holds this rank's contiguous slice of the batch and every step is a
+    token-sharded step whose per-layer exchange is an NCCL all-gather."""
+
+    def __init__(self, wl, device_index: int, n_steps: int, tile_n: int = 0, split_k: int = 0, shard=None):
         import numpy as np
         import torch
         from paper_2606_15615_gb300 import build
@@ -222,12 +226,14 @@ class Runner:
         from paper_2606_15615_gb300 import workloads as W
         self.torch, self.M, self.W, self.np = torch, M, W, np
         self.wl = wl
+        self.shard = shard
+        self.n_local = wl.n_tokens // shard[1] if shard else wl.n_tokens
         self.dev = torch.device("cuda", device_index)
         torch.cuda.set_device(self.dev)
         self.weights = [W.make_layer_weights_device(wl, l, self.dev) for l in range(wl.n_layers)]
         cfg = M.moeca_config_default(
             n_layers=wl.n_layers, hidden=wl.hidden, ffn=wl.ffn, n_experts=wl.n_experts, top_k=wl.top_k,
-            n_shared=wl.n_shared, max_tokens=wl.n_tokens,
+            n_shared=wl.n_shared, max_tokens=self.n_local,
             dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period,
             ffn_tile_n=tile_n, ffn_split_k=split_k, n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0,
             adaln=int(wl.adaln))
@@ -236,9 +242,12 @@ class Runner:
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
         self.dt = dt
         xs = [torch.from_numpy(x) for x in W.trajectory(wl, n_steps)]
+        if shard:  # this rank's rows of every step's batch
+            xs = [x[shard[0] * self.n_local:(shard[0] + 1) * self.n_local] for x in xs]
+            self.exchange = M.torch_allgather()
         self.x_host = torch.stack(xs).to(dt).pin_memory()
         self.x_dev = self.x_host.to(self.dev)
-        T, D = wl.n_tokens, wl.hidden
+        T, D = self.n_local, wl.hidden
         self.out = torch.empty((T, D), dtype=dt, device=self.dev)
         self.stream = torch.cuda.current_stream(self.dev)
         # End to end through moeca_step_host: pinned host outputs, two of them
@@ -273,10 +282,15 @@ class Runner:
                          x_prev=self.x_state, stream=self.stream.cuda_stream)
 
     def _step(self, h, x_ptr, out, t, tau0, sp, cond=None):
+        if self.shard:
+            x = self.x_dev[t] if x_ptr == self.x_dev[t].data_ptr() else None
+            assert x is not None, "token-sharded steps read the device trajectory"
+            self.stack.step_sharded(x, t, self.shard[0], self.shard[1], self.exchange, tau0=tau0, out=out)
+            return
         cp = None
         if self.wl.adaln:
             cp = (self.cond_dev[t] if cond is None else cond).data_ptr()
-        self.M.moeca_step(h, x_ptr, out.data_ptr(), self.wl.n_tokens, t, False, tau0, sp, cp)
+        self.M.moeca_step(h, x_ptr, out.data_ptr(), self.n_local, t, False, tau0, sp, cp)
         if self.wl.adaln:
             self._sampler_update(t, out)
 
@@ -643,6 +657,50 @@ def reference_arm(args, wl):
 
 
 # ---------------------------------------------------------------------------
+# token-sharded stacks across ranks
+# ---------------------------------------------------------------------------
+
+def sharded_main(args, wl, world, rank, local, dist):
+    """The workload's batch split by tokens over the ranks: every step runs
+    the token-sharded step, each layer exchanging its entropy partials with an
+    NCCL all-gather; the time is the max over ranks of K steps of the one
+    batch (strong scaling: the work is fixed as N grows)."""
+    import torch
+    if wl.n_tokens % (32 * world):
+        raise SystemExit(f"{wl.n_tokens} tokens do not split into {world} slices of whole 32-token blocks")
+    runner = Runner(wl, local, args.warmup + args.steps, args.ffn_tile_n, args.ffn_split_k, shard=(rank, world))
+    pt = headline_point(wl, args.reuse)
+    tau0 = args.tau0 if args.tau0 is not None else (pt["tau0"] if pt else args.ref_tau0)
+    W_, K = args.warmup, args.steps
+    reps = []
+    st = None
+    for _ in range(args.reps):
+        dist.barrier()
+        torch.cuda.synchronize(runner.dev)
+        ms, st, _ = runner._run(tau0, W_, K)
+        ms, _ = aggregate(ms, 0, dist, runner.dev)
+        reps.append(ms)
+    ms = statistics.median(reps)
+    n = torch.tensor([float(st["reused"]), float(st["branches"])], dtype=torch.float64, device=runner.dev)
+    dist.all_reduce(n)
+    line = {
+        "metric": METRIC, "value": wl.n_tokens * K / (ms / 1e3), "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W_, "ms_per_step": ms / K, "higher_is_better": True, "scaling": "strong", "vs_baseline": None,
+        "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "reuse_target": args.reuse, "parallelism": f"token-sharded x{world}"},
+        "point": {"tau0": tau0, "reuse_achieved": round(float(n[0] / max(n[1], 1)), 4)},
+        "exchange": f"one NCCL all-gather per layer per step of {world} x "
+                    f"{runner.M.moeca_shard_exchange_bytes(runner.stack.handle, runner.n_local)} bytes "
+                    "(per-block entropy partials)",
+    }
+    if rank == 0:
+        print(json.dumps(line))
+    dist.barrier()
+    dist.destroy_process_group()
+    runner.close()
+
+
+# ---------------------------------------------------------------------------
 
 def main():
     ap = argparse.ArgumentParser()
@@ -665,6 +723,9 @@ def main():
                     help="use this tau0 for the headline point instead of the stored / calibrated one")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first N layers of the workload (small ncu captures; not a bench line)")
+    ap.add_argument("--shard", action="store_true",
+                    help="under torchrun: split each step's batch over the ranks by tokens (one NCCL all-gather of "
+                         "the entropy partials per layer) instead of running one replica per rank")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -681,6 +742,8 @@ def main():
 
     import torch
     dist = init_group(world, "nccl")
+    if args.shard and world > 1:
+        return sharded_main(args, wl, world, rank, local, dist)
     runner = Runner(wl, local, args.warmup + args.steps, args.ffn_tile_n, args.ffn_split_k)
     dev = runner.dev
     W_, K = args.warmup, args.steps

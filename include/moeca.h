@@ -335,6 +335,51 @@ moeca_status moeca_step_host(moeca_handle* h, const void* x_in_host, void* x_out
  * No-op when moeca_step_host was never called. */
 moeca_status moeca_host_join(moeca_handle* h, void* stream);
 
+/* ---- Token-sharded stacks --------------------------------------------------
+ * Tokens are independent in every step of the layer except one: Eq. 11's
+ * per-expert sums S_e = sum_i C_{e,i} and U_e = sum_i C ln C run over all T
+ * token rows of the batch.  A stack can therefore be split by tokens over
+ * `world` ranks (processes or GPUs), each holding a contiguous slice of
+ * n_tokens rows (rank r: global rows [r n_tokens, (r + 1) n_tokens)) with
+ * the weights replicated, exchanging only the per-block partial sums of
+ * S_e and U_e once per layer per step.  Every rank then reduces every
+ * rank's partials in the same global block order as a single-rank step
+ * over the whole batch, so thresholds, decisions, row lists and outputs are
+ * bit-identical to that step's.
+ *
+ *   moeca_shard_exchange_bytes(h, n_tokens, &bytes);     // per rank
+ *   (send: bytes, recv: world x bytes, caller-owned device buffers)
+ *   moeca_shard_begin(h, x_in, x_out, args, shard, send, recv, stream);  // layer 0 routed
+ *   do {
+ *     all-gather `bytes` from every rank's send into recv in rank order, on
+ *       `stream` (e.g. ncclAllGather);
+ *     moeca_shard_next(h, stream, &done);   // finish this layer, route the next
+ *   } while (!done);
+ *
+ * Supported for the bf16 MoE layer stack run by the fused preparation kernel
+ * (n_heads 0, ffn_impl AUTO, token_reuse_policy 0); n_tokens must be a
+ * multiple of that kernel's token block (32 or 16) and equal on every rank;
+ * total_tokens = world x n_tokens (else INVALID_ARG / UNSUPPORTED).  The
+ * refresh schedule and state are as moeca_step's.  send and recv are
+ * 16-byte aligned device buffers the caller keeps until the step is done;
+ * each layer's partials are written to send by the kernels before the
+ * exchange and read from recv by those after it.  Asynchronous on `stream`
+ * like moeca_step; a started step must be finished with moeca_shard_next
+ * before another step (MOECA_ERR_STATE otherwise; moeca_reset abandons it). */
+typedef struct {
+  int32_t rank;          /* this rank, 0 .. world - 1                        */
+  int32_t world;         /* ranks holding a slice of the batch               */
+  int32_t total_tokens;  /* token rows of the whole batch (world x n_tokens) */
+} moeca_shard;
+/* Bytes one rank contributes to each layer's exchange for n_tokens rows. */
+moeca_status moeca_shard_exchange_bytes(moeca_handle* h, int32_t n_tokens, int64_t* bytes_per_rank);
+moeca_status moeca_shard_begin(moeca_handle* h, const void* x_in, void* x_out, const moeca_step_args* args,
+                               const moeca_shard* shard, void* send, const void* recv, void* stream);
+/* Finish the layer in progress from the gathered partials in recv and route
+ * the next one into send; *done = 1 after the last layer (x_out then holds
+ * the output). */
+moeca_status moeca_shard_next(moeca_handle* h, void* stream, int32_t* done);
+
 /* Copy the counters of `layer` (or the sum over layers for layer = -1) into
  * *out.  Synchronises the device. */
 moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out);

@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmoeca.so")
 
 SOURCES = ["moeca_api.cu", "router.cu", "select.cu", "prep.cu", "ffn_simt.cu", "ffn_tc.cu", "combine.cu",
-           "proj_tc.cu", "attention.cu", "attn_tc.cu", "prep_attn.cu", "adaln.cu", "probe.cu"]
+           "proj_tc.cu", "attention.cu", "attn_tc.cu", "prep_attn.cu", "prep_shard.cu", "adaln.cu", "probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++20", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

@@ -153,6 +153,10 @@ struct PrepArgs {
   unsigned long long* count_words;  // [blocks, groups] tagged recomputed rows per group (exchange 2)
   unsigned epoch;         // this launch's tag (never 0, never reused before a reset)
   unsigned wait_epoch;    // the tag the exchanges wait for (epoch, unless a stall is injected)
+  float* shard_send;      // token-sharded MODE 1: [blocks, E] float2 block partials (sum C, sum C ln C)
+  const float* shard_recv;  // MODE 2: [shard_blocks, E] float2, every rank's partials in rank order
+  int shard_blocks;       // MODE 2: blocks of all ranks
+  int shard_tokens;       // MODE 2: tokens of all ranks (T of Eq. 11's normalisation)
   float* tau;             // [E] (written by block 0)
   SelectArgs sel;         // decision inputs and outputs (its tau is replaced in-kernel)
   int32_t* counts;        // [G]
@@ -190,6 +194,9 @@ PrepShape prep_plan_attn(int D, int E, int k, int max_tokens, int n_sms);
 cudaError_t launch_prep_plain(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 cudaError_t launch_prep_attn(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
 cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s);
+// Token-sharded launches of the plain build: mode 1 routes and writes the
+// block partials to shard_send, mode 2 reduces shard_recv and decides.
+cudaError_t launch_prep_shard(const PrepArgs& a, const PrepShape& p, int mode, cudaStream_t s);
 
 // Eq. 8 combine + residual + cached branch norms.
 struct CombineArgs {

@@ -164,6 +164,17 @@ struct moeca_handle {
     cudaEvent_t up[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr}, back[2] = {nullptr, nullptr};
     long long calls = 0;
   } hio;
+  // Token-sharded step in progress (moeca_shard_begin / moeca_shard_next).
+  struct ShardRun {
+    bool active = false;
+    int layer = 0, T = 0, world = 1, total = 0;
+    bool refresh = false;
+    float tau0 = 0.f;
+    const void* x_in = nullptr;
+    void* x_out = nullptr;
+  } sh;
+  float* shard_send = nullptr;  // caller's [blocks, E] float2: this rank's block partials
+  float* shard_recv = nullptr;  // caller's [world x blocks, E] float2: every rank's, in rank order
   bool timing = false;
   std::vector<cudaEvent_t> event_pool;
   std::vector<PendingTiming> pending;
@@ -271,6 +282,72 @@ bool overlaps(const void* a, const void* b, size_t n) {
   const char* x = static_cast<const char*>(a);
   const char* y = static_cast<const char*>(b);
   return x < y + n && y < x + n;
+}
+
+// Launch arguments shared by the whole-step path and the token-sharded one.
+SelectArgs select_args(const moeca_handle* h, const LayerBuf& L, int T, bool refresh) {
+  const moeca_config& c = h->cfg;
+  SelectArgs sa{};
+  sa.T = T; sa.k = c.top_k; sa.E = c.n_experts; sa.G = h->G; sa.refresh = refresh;
+  sa.lambda1 = c.lambda1; sa.lambda2 = c.lambda2;
+  sa.score_terms = c.score_terms; sa.token_level = c.granularity;
+  sa.reused_meta_policy = c.reused_meta_policy; sa.shared_policy = c.shared_policy; sa.n_shared = c.n_shared;
+  sa.route_e = L.route_e; sa.route_w = L.route_w; sa.tau = L.tau;
+  sa.cache_e = L.cache_e; sa.cache_w = L.cache_w; sa.cache_norm = L.cache_norm;
+  sa.recompute = L.recompute; sa.slot = L.slot; sa.matched = L.matched; sa.token_any = L.token_any;
+  sa.block_counts = h->block_counts; sa.block_offsets = h->block_offsets;
+  sa.counts = L.counts; sa.offsets = L.offsets; sa.done = h->done + 1;
+  sa.stats = L.stats; sa.status = h->status_dev;
+  return sa;
+}
+
+// The fused preparation kernel's arguments for the MoE layer alone (no
+// attention sub-layer); the epoch is taken by the caller.
+PrepArgs prep_args_plain(const moeca_handle* h, const LayerBuf& L, const void* moe_in, int T, float tau0,
+                         const SelectArgs& sa, void* xg) {
+  const moeca_config& c = h->cfg;
+  PrepArgs pa{};
+  pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
+  pa.n_shared = c.n_shared;
+  pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
+  pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
+  pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
+  pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.tau = L.tau;
+  pa.sel = sa;
+  pa.part_words = h->prep_words; pa.count_words = h->prep_words + h->prep_count_off;
+  pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
+  pa.xg = xg; pa.stats = L.stats; pa.status = h->status_dev;
+  return pa;
+}
+
+FfnArgs ffn_args(const moeca_handle* h, const LayerBuf& L, int T, const void* moe_in) {
+  const moeca_config& c = h->cfg;
+  FfnArgs fa{};
+  fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;
+  fa.max_rows = T * (c.top_k + c.n_shared);
+  fa.counts = L.counts; fa.offsets = L.offsets; fa.list = L.list;
+  fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? moe_in : nullptr;
+  fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
+  fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
+  fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
+  fa.dep = h->tc_dep; fa.max_mtiles = h->tc_dep_pairs_n; fa.work = h->tc_work;
+  return fa;
+}
+
+CombineArgs combine_args(const moeca_handle* h, const LayerBuf& L, int T, const void* resid, void* out, bool refresh,
+                         bool use_tc) {
+  const moeca_config& c = h->cfg;
+  CombineArgs cb{};
+  cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
+  cb.x = resid; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+  cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
+  cb.n_sms = h->n_sms; cb.direct = c.combine_direct;
+  if (L.cache_y) {
+    // Sec. 4.1, token level: a token with an empty recompute set returns y^{t0}.
+    cb.cache_y = L.cache_y; cb.token_any = L.token_any; cb.copy_y = refresh ? 0 : 1;
+  }
+  cb.rearm = use_tc ? h->tc_work : nullptr;
+  return cb;
 }
 
 }  // namespace
@@ -685,17 +762,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ra.partials = h->partials; ra.done = h->done; ra.tau = L.tau; ra.stats = L.stats;
     ra.status = h->status_dev;
 
-    SelectArgs sa{};
-    sa.T = T; sa.k = c.top_k; sa.E = c.n_experts; sa.G = h->G; sa.refresh = refresh;
-    sa.lambda1 = c.lambda1; sa.lambda2 = c.lambda2;
-    sa.score_terms = c.score_terms; sa.token_level = c.granularity;
-    sa.reused_meta_policy = c.reused_meta_policy; sa.shared_policy = c.shared_policy; sa.n_shared = c.n_shared;
-    sa.route_e = L.route_e; sa.route_w = L.route_w; sa.tau = L.tau;
-    sa.cache_e = L.cache_e; sa.cache_w = L.cache_w; sa.cache_norm = L.cache_norm;
-    sa.recompute = L.recompute; sa.slot = L.slot; sa.matched = L.matched; sa.token_any = L.token_any;
-    sa.block_counts = h->block_counts; sa.block_offsets = h->block_offsets;
-    sa.counts = L.counts; sa.offsets = L.offsets; sa.done = h->done + 1;
-    sa.stats = L.stats; sa.status = h->status_dev;
+    SelectArgs sa = select_args(h, L, T, refresh);
 
     CompactArgs ca{};
     ca.T = T; ca.k = c.top_k; ca.E = c.n_experts; ca.G = h->G; ca.D = c.hidden; ca.n_shared = c.n_shared;
@@ -704,9 +771,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     ca.block_offsets = h->block_offsets; ca.offsets = L.offsets; ca.list = L.list;
     ca.x = moe_in; ca.xg = xg_now; ca.status = h->status_dev;
     if (fused) {
-      PrepArgs pa{};
-      pa.x = moe_in; pa.w_gate = L.w.w_gate; pa.b_gate = L.w.b_gate;
-      pa.n_shared = c.n_shared;
+      PrepArgs pa = prep_args_plain(h, L, moe_in, T, tau0, sa, xg_now);
       if (attn && !ada && !attn_full) {
         pa.x = in;
         pa.attn_a = L.attn_a;
@@ -728,17 +793,9 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
         oa.row_w = c.top_k + c.n_shared;
         oa.xg = h->xg;
       }
-      pa.T = T; pa.D = c.hidden; pa.E = c.n_experts; pa.k = c.top_k; pa.G = h->G;
-      pa.renorm = c.renorm_topk; pa.entropy_norm = c.entropy_norm;
-      pa.beta = c.beta; pa.tau0 = tau0; pa.alpha = c.alpha;
-      pa.route_e = L.route_e; pa.route_w = L.route_w; pa.ema = L.ema; pa.tau = L.tau;
-      pa.sel = sa;
-      pa.part_words = h->prep_words; pa.count_words = h->prep_words + h->prep_count_off;
       if (++h->prep_epoch == 0) h->prep_epoch = 1;  // 0 marks words never written
       pa.epoch = pa.wait_epoch = h->prep_epoch;
       if (h->inject_stall) pa.wait_epoch = h->prep_epoch ^ 0x80000000u;  // a tag no launch writes
-      pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
-      pa.xg = xg_now; pa.stats = L.stats; pa.status = h->status_dev;
       if ((e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep(pa, h->prep, s); })) != cudaSuccess) break;
     } else {
       if ((e = timed(h, MOECA_K_ROUTER, s, [&] { return launch_router(ra, h->bf16, s); })) != cudaSuccess) break;
@@ -773,15 +830,7 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
       }
     }
 
-    FfnArgs fa{};
-    fa.G = h->G; fa.E = c.n_experts; fa.D = c.hidden; fa.F = c.ffn; fa.k = c.top_k; fa.T = T;
-    fa.max_rows = T * (c.top_k + c.n_shared);
-    fa.counts = L.counts; fa.offsets = L.offsets; fa.list = L.list;
-    fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? moe_in : nullptr;
-    fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
-    fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
-    fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
-    fa.dep = h->tc_dep; fa.max_mtiles = h->tc_dep_pairs_n; fa.work = h->tc_work;
+    FfnArgs fa = ffn_args(h, L, T, moe_in);
     if (use_tc) {
       // Both GEMMs in one persistent launch: phase-2 tiles start as soon as
       // the phase-1 tiles of their rows are stored.
@@ -796,19 +845,10 @@ moeca_status moeca_step(moeca_handle* h, const void* x_in, void* x_out, const mo
     }
     if (e != cudaSuccess) break;
 
-    CombineArgs cb{};
-    cb.T = T; cb.D = c.hidden; cb.k = c.top_k; cb.n_shared = c.n_shared;
-    cb.x = resid; cb.out = out; cb.cache_h = L.cache_h; cb.shared_h = L.shared_h;
+    CombineArgs cb = combine_args(h, L, T, resid, out, refresh, use_tc);
     if (ada) {
       cb.gate = mod_l + 5 * c.hidden; cb.gate_ld = static_cast<int>(mod_ld); cb.seq = seq;
     }
-    cb.route_w = L.route_w; cb.slot = L.slot; cb.cache_norm = L.cache_norm; cb.status = h->status_dev;
-    cb.n_sms = h->n_sms; cb.direct = c.combine_direct;
-    if (L.cache_y) {
-      // Sec. 4.1, token level: a token with an empty recompute set returns y^{t0}.
-      cb.cache_y = L.cache_y; cb.token_any = L.token_any; cb.copy_y = refresh ? 0 : 1;
-    }
-    cb.rearm = use_tc ? h->tc_work : nullptr;
     if ((e = timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); })) != cudaSuccess) break;
     L.valid = true;
   }
@@ -899,6 +939,139 @@ moeca_status moeca_host_join(moeca_handle* h, void* stream) {
   cudaError_t e = cudaStreamWaitEvent(s, io.back[last], 0);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(s, io.up[last], 0);
   return e == cudaSuccess ? MOECA_OK : cuda_fail(h, e, "join");
+}
+
+namespace {
+
+// Layer l's routing and block partials (the fused preparation kernel, MODE 1)
+// on layer input `in`, into the exchange buffer.
+cudaError_t shard_route(moeca_handle* h, int l, const void* in, cudaStream_t s) {
+  LayerBuf& L = h->layers[l];
+  const SelectArgs sa = select_args(h, L, h->sh.T, h->sh.refresh);
+  PrepArgs pa = prep_args_plain(h, L, in, h->sh.T, h->sh.tau0, sa, nullptr);
+  pa.shard_send = h->shard_send;
+  return timed(h, MOECA_K_PREP, s, [&] { return launch_prep_shard(pa, h->prep, 1, s); });
+}
+
+// Layer l from the gathered partials on: decisions and compaction (MODE 2),
+// grouped FFN, combine.
+cudaError_t shard_finish(moeca_handle* h, int l, const void* in, void* out, cudaStream_t s) {
+  LayerBuf& L = h->layers[l];
+  const int T = h->sh.T;
+  const SelectArgs sa = select_args(h, L, T, h->sh.refresh);
+  PrepArgs pa = prep_args_plain(h, L, in, T, h->sh.tau0, sa, h->xg);
+  pa.shard_recv = h->shard_recv;
+  pa.shard_blocks = h->sh.world * (T / h->prep.tokens_per_block);
+  pa.shard_tokens = h->sh.total;
+  if (++h->prep_epoch == 0) h->prep_epoch = 1;
+  pa.epoch = pa.wait_epoch = h->prep_epoch;
+  cudaError_t e = timed(h, MOECA_K_PREP, s, [&] { return launch_prep_shard(pa, h->prep, 2, s); });
+  if (e != cudaSuccess) return e;
+  FfnArgs fa = ffn_args(h, L, T, in);
+  if ((e = timed(h, MOECA_K_FFN, s, [&] { return launch_ffn_tc(L.tc, fa, 0, s); })) != cudaSuccess) return e;
+  const CombineArgs cb = combine_args(h, L, T, in, out, h->sh.refresh, true);
+  return timed(h, MOECA_K_COMBINE, s, [&] { return launch_combine(cb, h->bf16, s); });
+}
+
+}  // namespace
+
+moeca_status moeca_shard_exchange_bytes(moeca_handle* h, int32_t n_tokens, int64_t* bytes_per_rank) {
+  if (!h || !bytes_per_rank) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  const int TB = h->prep.tokens_per_block;
+  if (!TB) return fail(h, MOECA_ERR_UNSUPPORTED, "no fused preparation kernel on this handle");
+  if (n_tokens < 1 || n_tokens > h->cfg.max_tokens || n_tokens % TB)
+    return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens must be in [1, max_tokens] and a multiple of the block size");
+  *bytes_per_rank = static_cast<int64_t>(n_tokens / TB) * h->cfg.n_experts * 2 * static_cast<int64_t>(sizeof(float));
+  return MOECA_OK;
+}
+
+moeca_status moeca_shard_begin(moeca_handle* h, const void* x_in, void* x_out, const moeca_step_args* args,
+                               const moeca_shard* shard, void* send, const void* recv, void* stream) {
+  if (!h) return fail(nullptr, MOECA_ERR_INVALID_ARG, "handle is NULL");
+  if (!args || !shard) return fail(h, MOECA_ERR_INVALID_ARG, "args or shard is NULL");
+  const moeca_config& c = h->cfg;
+  const int TB = h->prep.tokens_per_block;
+  if (!TB || c.n_heads || !h->bf16 || c.ffn_impl != MOECA_FFN_AUTO || c.token_reuse_policy)
+    return fail(h, MOECA_ERR_UNSUPPORTED,
+                "token-sharded steps run the bf16 MoE layer stack on the fused preparation kernel "
+                "(n_heads 0, tensor-core FFN, token_reuse_policy 0, a shape the fused kernel fits)");
+  if (h->sh.active) return fail(h, MOECA_ERR_STATE, "a sharded step is in progress: call moeca_shard_next");
+  const int T = args->n_tokens;
+  if (T < 1 || T > c.max_tokens || T % TB)
+    return fail(h, MOECA_ERR_INVALID_ARG, "n_tokens must be in [1, max_tokens] and a multiple of the block size");
+  if (shard->world < 1 || shard->rank < 0 || shard->rank >= shard->world ||
+      static_cast<long long>(shard->total_tokens) != static_cast<long long>(shard->world) * T)
+    return fail(h, MOECA_ERR_INVALID_ARG, "0 <= rank < world and total_tokens = world x n_tokens");
+  if (!send || !recv || reinterpret_cast<uintptr_t>(send) % 16 || reinterpret_cast<uintptr_t>(recv) % 16)
+    return fail(h, MOECA_ERR_INVALID_ARG, "send and recv must be 16-byte aligned device buffers");
+  moeca_status st = check_device_status(h);
+  if (st != MOECA_OK) return st;
+  if (!x_in || !x_out) return fail(h, MOECA_ERR_INVALID_ARG, "x_in or x_out is NULL");
+  const size_t xbytes = static_cast<size_t>(T) * c.hidden * h->es;
+  if (overlaps(x_in, x_out, xbytes)) return fail(h, MOECA_ERR_INVALID_ARG, "x_in and x_out overlap");
+  if (reinterpret_cast<uintptr_t>(x_in) % 16 || reinterpret_cast<uintptr_t>(x_out) % 16)
+    return fail(h, MOECA_ERR_INVALID_ARG, "x_in and x_out must be 16-byte aligned");
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  bool all_valid = h->state_T == T;
+  for (auto& L : h->layers) all_valid = all_valid && L.valid;
+  const int N = c.refresh_period;
+  const bool refresh = args->force_refresh || !all_valid || (N > 0 && args->step_index % N == 0);
+  if (h->state_T != T) {
+    for (auto& L : h->layers) {
+      cudaError_t e = cudaMemsetAsync(L.ema, 0, static_cast<size_t>(c.max_tokens) * c.n_experts * 4, s);
+      if (e != cudaSuccess) return cuda_fail(h, e, "reset EMA");
+      L.valid = false;
+    }
+  }
+  h->shard_send = static_cast<float*>(send);
+  h->shard_recv = static_cast<float*>(const_cast<void*>(recv));
+  h->sh.layer = 0;
+  h->sh.T = T;
+  h->sh.world = shard->world;
+  h->sh.total = shard->total_tokens;
+  h->sh.refresh = refresh;
+  h->sh.tau0 = std::isnan(args->tau0_override) ? c.tau0 : args->tau0_override;
+  h->sh.x_in = x_in;
+  h->sh.x_out = x_out;
+  cudaError_t e = shard_route(h, 0, x_in, s);
+  if (e != cudaSuccess) {
+    for (auto& L : h->layers) L.valid = false;
+    return cuda_fail(h, e, "kernel launch");
+  }
+  h->sh.active = true;
+  return MOECA_OK;
+}
+
+moeca_status moeca_shard_next(moeca_handle* h, void* stream, int32_t* done) {
+  if (!h || !done) return fail(h, MOECA_ERR_INVALID_ARG, "NULL argument");
+  if (!h->sh.active) return fail(h, MOECA_ERR_STATE, "no sharded step in progress");
+  cudaSetDevice(h->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int l = h->sh.layer, nL = h->cfg.n_layers;
+  const void* in = l == 0 ? h->sh.x_in : h->act[l];
+  void* out = l + 1 == nL ? h->sh.x_out : h->act[l + 1];
+  NvtxRange range("moeca_shard_next");
+  cudaError_t e = shard_finish(h, l, in, out, s);
+  if (e == cudaSuccess) {
+    h->layers[l].valid = true;
+    if (l + 1 < nL) e = shard_route(h, l + 1, out, s);
+  }
+  if (e != cudaSuccess) {
+    for (auto& L : h->layers) L.valid = false;
+    h->sh.active = false;
+    return cuda_fail(h, e, "kernel launch");
+  }
+  if (l + 1 < nL) {
+    h->sh.layer = l + 1;
+    *done = 0;
+  } else {
+    h->state_T = h->sh.T;
+    h->last_x_in = h->sh.x_in;
+    h->sh.active = false;
+    *done = 1;
+  }
+  return MOECA_OK;
 }
 
 moeca_status moeca_get_stats(moeca_handle* h, int32_t layer, moeca_stats* out) {
@@ -1058,6 +1231,7 @@ moeca_status moeca_reset(moeca_handle* h) {
     if (e != cudaSuccess) return cuda_fail(h, e, "reset EMA");
   }
   h->state_T = 0;
+  h->sh.active = false;
   return MOECA_OK;
 }
 

@@ -42,6 +42,9 @@
 #ifndef MOECA_PREP_ATTN
 #define MOECA_PREP_ATTN 0
 #endif
+#ifndef MOECA_PREP_SHARD
+#define MOECA_PREP_SHARD 0
+#endif
 
 namespace moeca {
 namespace {
@@ -167,7 +170,14 @@ static __device__ __noinline__ void attn_bookkeeping(const PrepArgs& a, int i, i
   }
 }
 
-template <int TB, int EPAD, int KMAX>
+// MODE 0: the whole preparation of a layer (the default).  A token-sharded
+// stack (each rank holds a block-aligned slice of the batch) runs it in two
+// launches around an all-gather of the entropy partials, Eq. 11's per-expert
+// sums being the only coupling between tokens: MODE 1 routes its blocks'
+// tokens and writes the block partials (plain floats) for the exchange;
+// MODE 2 reads every rank's partials, in the global block order MODE 0 uses,
+// and decides and compacts.
+template <int TB, int EPAD, int KMAX, int MODE>
 __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   constexpr int G = kThreads / TB;       // lanes per token in the routing epilogue (4 or 8)
   constexpr int EPL = EPAD / G;          // experts per lane (>= 1)
@@ -233,10 +243,12 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   __syncthreads();
   const uint32_t bar = smem_u32(&sm_bar);
   const uint32_t row_bytes = static_cast<uint32_t>(D) * 2;
+  constexpr bool kRoute = MODE != 2;  // MODE 2 reads the routing MODE 1 wrote
   if (t == 0) {
-    mbar_expect_tx(bar, row_bytes * (E + ntok + (add_a ? ntok : 0)));
+    mbar_expect_tx(bar, row_bytes * ((kRoute ? E : 0) + ntok + (add_a ? ntok : 0)));
     const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
-    for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
+    if (kRoute)
+      for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
     if constexpr (kAttn) {
       if (add_a) issue_attn_rows(a, s_a, ldw, tok0, ntok, row_bytes, bar);  // written on an earlier step
     }
@@ -251,10 +263,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         sm_cn[idx] = a.sel.cache_norm[cb + idx];
       }
     const size_t eb = static_cast<size_t>(tok0) * E;
-    for (int idx = t; idx < ntok * E; idx += kThreads) sm_ema[(idx / E) * EPAD + idx % E] = a.ema[eb + idx];
+    if (kRoute)
+      for (int idx = t; idx < ntok * E; idx += kThreads) sm_ema[(idx / E) * EPAD + idx % E] = a.ema[eb + idx];
   }
   // Zero the padding rows the tensor cores read (experts past E, tokens past T).
-  for (int idx = t; idx < (EPAD - E) * (D / 8); idx += kThreads) {
+  for (int idx = t; kRoute && idx < (EPAD - E) * (D / 8); idx += kThreads) {
     const int r = E + idx / (D / 8), c = idx % (D / 8);
     reinterpret_cast<uint4*>(s_w + r * ldw)[c] = make_uint4(0, 0, 0, 0);
   }
@@ -279,6 +292,14 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     }
   }
 
+  if constexpr (!kRoute) {
+    // The routing of the block's tokens, written by MODE 1.
+    for (int idx = t; idx < ntok * k; idx += kThreads) {
+      sm_re[idx] = a.route_e[static_cast<size_t>(tok0) * k + idx];
+      sm_rw[idx] = a.route_w[static_cast<size_t>(tok0) * k + idx];
+    }
+    __syncthreads();
+  } else {
   // ---- A1: logits on the tensor cores ----
   // The WPG warps of a 16-token group each take a contiguous range of the
   // D / 16 k-steps and every n-tile over it, with two interleaved
@@ -436,8 +457,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     }
   }
   __syncthreads();
+  }  // kRoute
   const unsigned epoch = a.epoch;
-  {
+  if constexpr (kRoute) {
     // Block partials per expert: J interleaved runs over the block's tokens,
     // added in run order, then published.
     const int J = kThreads / E;
@@ -457,12 +479,17 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
         Ss += sm_rs[q * E + t][0];
         Us += sm_rs[q * E + t][1];
       }
-      unsigned long long* pw = a.part_words + (static_cast<size_t>(blockIdx.x) * E + t) * 2;
-      st_word(pw, tag_word(__float_as_uint(Ss), epoch));
-      st_word(pw + 1, tag_word(__float_as_uint(Us), epoch));
+      if constexpr (MODE == 1) {
+        reinterpret_cast<float2*>(a.shard_send)[static_cast<size_t>(blockIdx.x) * E + t] = make_float2(Ss, Us);
+      } else {
+        unsigned long long* pw = a.part_words + (static_cast<size_t>(blockIdx.x) * E + t) * 2;
+        st_word(pw, tag_word(__float_as_uint(Ss), epoch));
+        st_word(pw + 1, tag_word(__float_as_uint(Us), epoch));
+      }
     }
     if (t == 0 && sm_near) atomicAdd(a.stats + kStNearRoute, static_cast<unsigned long long>(sm_near));
   }
+  if constexpr (MODE == 1) return;  // the exchange and the rest run in MODE 2
 
   // The threshold-free half of the decisions (warp 0, one token per lane),
   // while the other blocks publish their partials.
@@ -478,10 +505,18 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   {
     const int J = kThreads / E;
     const int e = t % E, j = t / E;
-    const int nb = gridDim.x;
+    const int nb = MODE == 2 ? a.shard_blocks : static_cast<int>(gridDim.x);
     float S = 0.f, U = 0.f;
     bool ok = true;
-    if (j < J) {
+    if (MODE == 2 && j < J) {
+      // Every rank's blocks, gathered in rank order = global block order.
+      const float2* part = reinterpret_cast<const float2*>(a.shard_recv);
+      for (int b = j; b < nb; b += J) {
+        const float2 v = __ldcg(part + static_cast<size_t>(b) * E + e);
+        S += v.x;
+        U += v.y;
+      }
+    } else if (j < J) {
       const int n = 2 * ((nb - j + J - 1) / J);  // (S, U) of blocks j, j + J, ...
       ok = read_tagged<8>(
           a.part_words, n, [&](int q) { return (static_cast<size_t>(j + (q >> 1) * J) * E + e) * 2 + (q & 1); },
@@ -525,7 +560,8 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
       float hb = 0.5f;
       if (sm_live[t]) {
         if (a.entropy_norm == 0) {
-          if (T > 1) hb = fminf(1.f, fmaxf(0.f, sm_H[t] / logf(static_cast<float>(T))));
+          const int Te = MODE == 2 ? a.shard_tokens : T;  // every rank's tokens (Eq. 11's i)
+          if (Te > 1) hb = fminf(1.f, fmaxf(0.f, sm_H[t] / logf(static_cast<float>(Te))));
         } else if (sm_hi > sm_lo) {
           hb = (sm_H[t] - sm_lo) / (sm_hi - sm_lo);
         }
@@ -721,9 +757,10 @@ size_t prep_smem(int D, bool attn) {
   return rows + prep_region_bytes(TB, EPAD) + a_rows;
 }
 
-template <int TB, int EPAD, int KMAX>
+template <int TB, int EPAD, int KMAX, int MODE = 0>
 cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream_t s) {
-  cudaError_t e = set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX>), kPrepSmemMax);
+  cudaError_t e =
+      set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX, MODE>), kPrepSmemMax);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(n_blocks);
@@ -743,18 +780,19 @@ cudaError_t prep_launch(const PrepArgs& a, int n_blocks, size_t smem, cudaStream
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD, KMAX>, a);
+  return cudaLaunchKernelEx(&cfg, prep_kernel<TB, EPAD, KMAX, MODE>, a);
 }
 
 template <int TB, int EPAD, int KMAX>
 int prep_occupancy(size_t smem) {
-  if (set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX>), kPrepSmemMax) !=
+  if (set_dyn_smem_on_device(reinterpret_cast<const void*>(prep_kernel<TB, EPAD, KMAX, 0>), kPrepSmemMax) !=
       cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD, KMAX>, kThreads, smem) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, prep_kernel<TB, EPAD, KMAX, 0>, kThreads, smem) !=
+      cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -779,6 +817,17 @@ int kmax_of(int k) { return k <= 2 ? 2 : (k <= 4 ? 4 : 8); }
 
 }  // namespace
 
+#if MOECA_PREP_SHARD
+// The token-sharded launches (MODE 1, MODE 2) of the plain build, compiled in
+// their own translation unit (prep_shard.cu) beside the plain one.
+cudaError_t launch_prep_shard(const PrepArgs& a, const PrepShape& p, int mode, cudaStream_t s) {
+  const int nb = (a.T + p.tokens_per_block - 1) / p.tokens_per_block;
+  return with_shape(p.tokens_per_block, p.epad, p.kmax, [&]<int tb, int ep, int kk>() -> cudaError_t {
+    if constexpr (tb == 0) return cudaErrorInvalidValue;
+    else return mode == 1 ? prep_launch<tb, ep, kk, 1>(a, nb, p.smem, s) : prep_launch<tb, ep, kk, 2>(a, nb, p.smem, s);
+  });
+}
+#else
 #if MOECA_PREP_ATTN
 PrepShape prep_plan_attn(int D, int E, int k, int max_tokens, int n_sms) {
   const bool attn = true;
@@ -834,5 +883,7 @@ cudaError_t launch_prep(const PrepArgs& a, const PrepShape& p, cudaStream_t s) {
   return p.attn ? launch_prep_attn(a, p, s) : launch_prep_plain(a, p, s);
 }
 #endif
+
+#endif  // MOECA_PREP_SHARD
 
 }  // namespace moeca

@@ -80,6 +80,10 @@ class moeca_layer_trace(C.Structure):
                                             "block_in", "route_in", "resid", "mod")]
 
 
+class moeca_shard(C.Structure):
+    _fields_ = [("rank", C.c_int32), ("world", C.c_int32), ("total_tokens", C.c_int32)]
+
+
 class moeca_kernel_times(C.Structure):
     _fields_ = [("total_ms", C.c_double * 13), ("launches", C.c_int64 * 13)]
 
@@ -116,6 +120,10 @@ def _load():
         "moeca_step": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args), C.c_void_p]),
         "moeca_step_host": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args), C.c_void_p]),
         "moeca_host_join": (C.c_int, [H, C.c_void_p]),
+        "moeca_shard_exchange_bytes": (C.c_int, [H, C.c_int32, C.POINTER(C.c_int64)]),
+        "moeca_shard_begin": (C.c_int, [H, C.c_void_p, C.c_void_p, C.POINTER(moeca_step_args),
+                                        C.POINTER(moeca_shard), C.c_void_p, C.c_void_p, C.c_void_p]),
+        "moeca_shard_next": (C.c_int, [H, C.c_void_p, C.POINTER(C.c_int32)]),
         "moeca_get_stats": (C.c_int, [H, C.c_int32, C.POINTER(moeca_stats)]),
         "moeca_reset_stats": (C.c_int, [H]),
         "moeca_get_layer_state": (C.c_int, [H, C.c_int32, C.POINTER(moeca_layer_state),
@@ -198,6 +206,41 @@ def moeca_step_host(h, x_in_host_ptr: int, x_out_host_ptr: int, n_tokens: int, s
 def moeca_host_join(h, stream: int = 0):
     """Order ``stream`` after every upload and read-back of moeca_step_host."""
     _check(LIB.moeca_host_join(h, stream or None), h)
+
+
+def moeca_shard_exchange_bytes(h, n_tokens: int) -> int:
+    """Bytes one rank contributes to each layer's exchange (see include/moeca.h)."""
+    n = C.c_int64()
+    _check(LIB.moeca_shard_exchange_bytes(h, n_tokens, C.byref(n)), h)
+    return n.value
+
+
+def moeca_shard_begin(h, x_in_ptr: int, x_out_ptr: int, n_tokens: int, step_index: int, rank: int, world: int,
+                      send_ptr: int, recv_ptr: int, force_refresh: bool = False, tau0_override: float = math.nan,
+                      stream: int = 0):
+    args = moeca_step_args(n_tokens, step_index, int(force_refresh), tau0_override, None)
+    sh = moeca_shard(rank, world, world * n_tokens)
+    _check(LIB.moeca_shard_begin(h, x_in_ptr, x_out_ptr, C.byref(args), C.byref(sh), send_ptr, recv_ptr,
+                                 stream or None), h)
+
+
+def moeca_shard_next(h, stream: int = 0) -> bool:
+    done = C.c_int32()
+    _check(LIB.moeca_shard_next(h, stream or None, C.byref(done)), h)
+    return bool(done.value)
+
+
+def torch_allgather(group=None):
+    """The exchange of a token-sharded step over torch.distributed: every
+    rank's send bytes into recv in rank order (NCCL on the current stream)."""
+    import torch.distributed as dist
+
+    def exchange(send, recv):
+        if dist.get_backend(group) == "nccl":
+            dist.all_gather_into_tensor(recv, send, group=group)
+        else:  # gloo: the list form, into views of recv in rank order
+            dist.all_gather(list(recv.chunk(dist.get_world_size(group))), send, group=group)
+    return exchange
 
 
 def moeca_get_stats(h, layer: int = -1) -> dict:
@@ -372,6 +415,30 @@ class Stack:
         moeca_step(self.handle, x.data_ptr(), out.data_ptr(), T, step_index, force_refresh, tau0,
                    self.stream_ptr(), cond.data_ptr() if cond is not None else None)
         return out
+
+    def step_sharded(self, x, step_index: int, rank: int, world: int, exchange, force_refresh: bool = False,
+                     tau0=math.nan, out=None):
+        """One denoising step of this rank's slice ``x`` [n_tokens, D] of a
+        token-sharded batch (include/moeca.h): each layer's entropy partials
+        are exchanged with ``exchange(send, recv)`` (uint8 CUDA tensors:
+        ``send`` this rank's bytes, ``recv`` world x that, filled in rank
+        order), e.g. ``torch_allgather()``."""
+        torch = self.torch
+        T = x.shape[0]
+        if out is None:
+            out = torch.empty_like(x)
+        nbytes = moeca_shard_exchange_bytes(self.handle, T)
+        if getattr(self, "_xbuf", None) is None or self._xbuf[0].numel() < nbytes or \
+                self._xbuf[1].numel() < world * nbytes:
+            self._xbuf = (self._empty((nbytes,), torch.uint8), self._empty((world * nbytes,), torch.uint8))
+        send, recv = self._xbuf[0][:nbytes], self._xbuf[1][:world * nbytes]
+        sp = self.stream_ptr()
+        moeca_shard_begin(self.handle, x.data_ptr(), out.data_ptr(), T, step_index, rank, world, send.data_ptr(),
+                          recv.data_ptr(), force_refresh, tau0, sp)
+        while True:
+            exchange(send, recv)
+            if moeca_shard_next(self.handle, sp):
+                return out
 
     def _empty(self, shape, dtype):
         return self.torch.empty(shape, dtype=dtype, device=self.device)

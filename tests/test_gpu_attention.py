@@ -98,6 +98,20 @@ def test_one_sample_shared_expert(M):
     st.close()
 
 
+def test_sync_block_shared_expert_always(M):
+    """A shared expert recomputed for every token (shared_policy 1) under the
+    sync rule: a token that keeps its attention (empty recompute set) still
+    has a shared-expert row, whose input the preparation kernel gathers."""
+    T, D, H, S = 256, 256, 4, 128
+    st, cfg, ws = make_block_stack(M, T, D, H, 4, 2, 192, L=2, S=S, n_shared=1, seed=9, tau0=0.8, shared_policy=1)
+    rng = np.random.default_rng(90)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.03)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    stats = st.stats()
+    assert stats["tokens_fully_reused"] > 0 and stats["shared_recomputed"] == 2 * 4 * T
+    st.close()
+
+
 def test_block_full_size_d768_12_heads(M):
     """The 12-head block of the D 768 stack at full size (T 2048 = 8 samples
     of 256, E 16, top-2, F 3072), two of its layers, three steps."""
