@@ -134,11 +134,12 @@ typedef struct {
                                  branches and shared expert, before the AdaLN gate) unchanged.
                                  1 keeps y for every token: one [T, D] fp32 buffer per layer
                                  (moeca_layer_state.cache_y), written by every token that computes */
-  int32_t combine_direct;     /* Eq. 8 combine kernel form: 0 (default) = staged, each warp stages
-                                 a token's rows in shared memory with bulk copies while it combines
-                                 the previous one; 1 = direct, the lanes load the rows themselves
-                                 (the cross-check; the token-level reading above always uses it).
-                                 Both give the same bits */
+  int32_t combine_direct;     /* Eq. 8 combine kernel form: 1 (default) = direct, one warp per
+                                 token, the lanes load the rows themselves; 0 = staged where a
+                                 warp's two token buffers take at most 24 KB, each warp bringing a
+                                 token's rows into shared memory with bulk copies while it combines
+                                 the previous one (the direct form otherwise, and always under the
+                                 token-level reading above).  Both give the same bits */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters

@@ -1,8 +1,8 @@
 // Combine of fresh and cached branch outputs (Eq. 8) with the residual of
 // Eq. 5 / Eq. 6, and the cached-norm refresh that Eq. 9's o reads next step.
 //
-// Two forms: a staged one (combine_staged_kernel, the default, below) and a
-// direct one (combine_kernel: one warp per token, 16-byte vectors over D):
+// Two forms: a direct one (combine_kernel, the default: one warp per token,
+// 16-byte vectors over D) and a staged one (combine_staged_kernel, below):
 //   y_i = sum_{p=1..k} w_{i,p}^t cache_h[i, slot(p)]  (+ shared_h[i])
 //   out_i = x_i + y_i            (fp32 accumulation in p order, rounded once)
 //   out_i = x_i + g_i * y_i      in an AdaLN block (g the sample's MoE gate, Sec. 3)
@@ -21,9 +21,10 @@ namespace {
 constexpr int kWarps = 8;
 
 // CG 16-byte chunks per lane are in flight at once (all k cache rows, the
-// shared row and x loaded before any arithmetic).
-template <typename TI, int KMAX, int CG, bool GATED, bool YC>
-__global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
+// shared row and x loaded before any arithmetic).  MINB is the launch's
+// minimum of resident blocks per SM (see direct_min_blocks).
+template <typename TI, int KMAX, int CG, bool GATED, bool YC, int MINB>
+__global__ void __launch_bounds__(kWarps * 32, MINB) combine_kernel(CombineArgs a) {
   constexpr int V = Elem<TI>::kVec;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * kWarps + warp;
@@ -175,7 +176,7 @@ __global__ void __launch_bounds__(kWarps * 32) combine_kernel(CombineArgs a) {
   }
 }
 
-// Staged form (the default): each warp walks its tokens i = w, w + W, ...
+// Staged form: each warp walks its tokens i = w, w + W, ...
 // (w its global warp index, W the grid's warps) and stages a token's rows in
 // shared memory with bulk copies, lane 0 issuing them onto one mbarrier per
 // buffer: the token's k cache rows (one contiguous [k, D] block; slot is a
@@ -349,13 +350,29 @@ cudaError_t launch_staged(const CombineArgs& a, cudaStream_t s) {
   return run(combine_staged_kernel<TI, 8, GATED>);
 }
 
+// Resident blocks per SM that the direct form asks of the compiler, with one
+// 16-byte chunk per row and lane in flight.  Top-2 tokens fit four blocks
+// (64 registers a thread): every token of a 4096-token batch is then in
+// flight at once, which measured 37.5 -> 20.8 us per launch at D 2560 with a
+// shared expert against two blocks with four chunks in flight.  Top-4 takes
+// three, top-8 two (with the AdaLN gate values one block fewer, and fp32 top-8
+// one): under a tighter cap the compiler spills, or moves row loads next to
+// their use, one round trip each (top-8 at D 1152: 25 us per launch with two
+// blocks, 30 to 60 us with three in the spill-free variants tried).
+template <typename TI, int KMAX, bool GATED>
+constexpr int direct_min_blocks() {
+  return KMAX <= 2 ? (GATED ? 3 : 4) : KMAX <= 4 ? (GATED ? 2 : 3) : sizeof(TI) == 4 ? 1 : 2;
+}
+
 template <typename TI, bool GATED, bool YC>
 void launch_t(const CombineArgs& a, cudaStream_t s) {
   const int grid = (a.T + kWarps - 1) / kWarps;
-  // The gated form holds the gate values with the rows: half the chunks in flight keeps it near 128 registers.
-  if (a.k <= 2) launch_pdl(combine_kernel<TI, 2, GATED ? 2 : 4, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else if (a.k <= 4) launch_pdl(combine_kernel<TI, 4, 2, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
-  else launch_pdl(combine_kernel<TI, 8, 1, GATED, YC>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  if (a.k <= 2)
+    launch_pdl(combine_kernel<TI, 2, 1, GATED, YC, direct_min_blocks<TI, 2, GATED>()>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else if (a.k <= 4)
+    launch_pdl(combine_kernel<TI, 4, 1, GATED, YC, direct_min_blocks<TI, 4, GATED>()>, dim3(grid), dim3(kWarps * 32), 0, s, a);
+  else
+    launch_pdl(combine_kernel<TI, 8, 1, GATED, YC, direct_min_blocks<TI, 8, GATED>()>, dim3(grid), dim3(kWarps * 32), 0, s, a);
 }
 
 template <bool YC>
@@ -371,13 +388,16 @@ cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s) {
   if (a.gate && !bf16) return cudaErrorInvalidValue;  // AdaLN blocks are bf16 only
   if (a.cache_y && (!a.token_any || reinterpret_cast<uintptr_t>(a.cache_y) % 16)) return cudaErrorInvalidValue;
   if (a.T <= 0) return cudaSuccess;
-  // The staged form while a warp's two buffers take at most 24 KB, so that
-  // two blocks (8 warps) fit an SM: with larger tokens (D 2560 with a shared
-  // expert, top-8 at D 1152: about 41 KB a warp) a block of 4 warps per SM
-  // measured slower than the direct form's 24 warps (31 vs 26 us, 40 vs 27 us
-  // per launch).  The 16-byte alignment of every staged row holds for D a
-  // multiple of the vector width.  The token-level reading of Sec. 4.1
-  // (cache_y) keeps the direct form.
+  // The direct form by default: inside the launch pipeline it measured the
+  // shorter step (12-layer D 768: 0.7785 -> 0.774 ms; 28-layer D 1152: 4.150
+  // -> 4.108 ms) although the staged form is the faster launch when timed
+  // alone at D 768 (8.5 vs 10.4 us).  The staged form, on request, while a
+  // warp's two buffers take at most 24 KB, so that two blocks (8 warps) fit
+  // an SM: with larger tokens (D 2560 with a shared expert, top-8 at D 1152:
+  // about 41 KB a warp) a block of 4 warps per SM measured slower than the
+  // direct form (31 vs 26 us, 40 vs 27 us per launch).  The 16-byte alignment
+  // of every staged row holds for D a multiple of the vector width.  The
+  // token-level reading of Sec. 4.1 (cache_y) keeps the direct form.
   const size_t per_warp = 2 * (bf16 ? staged_buf_bytes<__nv_bfloat16>(a.k, a.shared_h ? 1 : 0, a.D)
                                     : staged_buf_bytes<float>(a.k, a.shared_h ? 1 : 0, a.D));
   if (!a.cache_y && !a.direct && per_warp <= 24 * 1024 && reinterpret_cast<uintptr_t>(a.x) % 16 == 0) {

@@ -383,7 +383,7 @@ void moeca_config_default(moeca_config* c) {
   c->ln_eps = 1e-6f;
   c->keep_route_in = 0;
   c->token_reuse_policy = 0;
-  c->combine_direct = 0;
+  c->combine_direct = 1;
 }
 
 const char* moeca_status_string(moeca_status s) {
