@@ -505,6 +505,19 @@ def roofline(kind: str, kd: dict, wl, pk: dict, pk_src: str, ffma_peak):
     return r
 
 
+def stream_ceiling(M, wl, device: int, kd, pk: dict) -> dict:
+    """What a plain streaming kernel reaches at the combine's size and shape
+    (moeca_probe_stream: a token's k + shared + 1 rows read, one written, one
+    warp per token, clean L2), beside the combine's event-timed rate: at tens
+    of MB a launch's ramp and drain keep any kernel below the large-copy peak."""
+    es = 2 if wl.dtype == "bf16" else 4
+    rows = wl.top_k + wl.n_shared + 1
+    gbs, us = M.moeca_probe_stream(device, wl.n_tokens, rows, wl.hidden * es)
+    return {"shape": f"{wl.n_tokens} tokens x {rows} rows of {wl.hidden * es} B read, one row written",
+            "stream_gbs": gbs, "stream_us": us, "stream_frac_of_peak": gbs / pk["hbm_gbs"],
+            "combine_gbs": kd["gbs"], "combine_frac_of_stream": kd["gbs"] / gbs if kd["gbs"] else None}
+
+
 def point_row(runner, wl, tgt, tau0, ms, st, K, world):
     tokens_all = wl.n_tokens * K * world
     executed = (st["recomputed"] + st["shared_recomputed"]) * 4.0 * wl.hidden * wl.ffn
@@ -547,6 +560,8 @@ def config_row(wl, local: int, W_: int, K: int, pk, pk_src, ffma_peak):
         for kind in ("ffn", "ffn2", "combine", "prep", "router"):
             if kind in kernels and kind != dom:
                 row[f"roofline_{kind}"] = roofline(kind, kernels[kind], wl, pk, pk_src, ffma_peak)
+        if "combine" in kernels:
+            row["combine_size_ceiling"] = stream_ceiling(runner.M, wl, local, kernels["combine"], pk)
         if len(rows) > 1:
             row["sweep"] = rows
         return row
@@ -799,6 +814,7 @@ def main():
     dom = max(kernels, key=lambda k_: kernels[k_]["avg_us"] * kernels[k_]["launches"])
     roof = roofline(dom, kernels[dom], wl, pk, pk_src, ffma_peak)
     roof["traffic"] = recorded_traffic(dom, wl.name, args.reuse)
+    ceiling = stream_ceiling(runner.M, wl, local, kernels["combine"], pk) if "combine" in kernels else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -844,6 +860,7 @@ def main():
                         f"({wl.n_layers} x {2 * wl.n_experts * wl.hidden * wl.ffn * es / 1e6:.0f} MB) > 129 MB L2",
                   "parallelism": f"replicas x{world}"},
         "roofline": roof,
+        "combine_size_ceiling": ceiling,
         "cpu_baseline": cpu,
         "e2e": {"value": wl.n_tokens * K * world / (e2e_ms / 1e3), "unit": "tokens/s",
                 "h2d_bytes_per_step": io_bytes + cond_bytes, "d2h_bytes_per_step": io_bytes,

@@ -1,6 +1,10 @@
-// fp32 FMA-throughput probe (include/moeca_probe.h): the roofline of the fp32
-// debug path's SIMT expert FFN.
+// Measurement probes (include/moeca_probe.h): the fp32 FMA throughput (the
+// roofline of the fp32 debug path's SIMT expert FFN) and the rate a plain
+// streaming kernel reaches at the combine's size and shape.
 #include <cuda_runtime.h>
+
+#include <algorithm>
+#include <vector>
 
 #include "moeca_probe.h"
 
@@ -25,7 +29,117 @@ __global__ void __launch_bounds__(kThreads) ffma_probe_kernel(float* out, int it
   if (s == -1.2345e30f) out[0] = s;
 }
 
+// One warp per token: the token's ROWS rows, chunk by chunk (all rows of a
+// lane's chunk loaded before use), summed as integers into one output row.
+template <int ROWS>
+__global__ void __launch_bounds__(256, 4) stream_probe_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst,
+                                                              long long n_tokens, int nvec) {
+  const long long t = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (t >= n_tokens) return;
+  const uint4* s = src + static_cast<size_t>(t) * ROWS * nvec;
+#pragma unroll 1
+  for (int c = threadIdx.x & 31; c < nvec; c += 32) {
+    uint4 v[ROWS];
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r) v[r] = s[static_cast<size_t>(r) * nvec + c];
+    uint4 a = v[0];
+#pragma unroll
+    for (int r = 1; r < ROWS; ++r) {
+      a.x += v[r].x;
+      a.y += v[r].y;
+      a.z += v[r].z;
+      a.w += v[r].w;
+    }
+    dst[static_cast<size_t>(t) * nvec + c] = a;
+  }
+}
+
+// Reads a buffer through L2 (evicting what was there for clean lines).
+__global__ void l2_read_kernel(const uint4* __restrict__ p, size_t n, uint4* sink) {
+  uint32_t a = 0;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const uint4 v = p[i];
+    a ^= v.x ^ v.y ^ v.z ^ v.w;
+  }
+  if (a == 0x9e3779b9u) sink->x = a;  // never true for the zeroed buffer; keeps the loads
+}
+
+template <int ROWS>
+void launch_stream(const uint4* src, uint4* dst, long long n_tokens, int nvec) {
+  const unsigned grid = static_cast<unsigned>((n_tokens + 7) / 8);
+  stream_probe_kernel<ROWS><<<grid, 256>>>(src, dst, n_tokens, nvec);
+}
+
+void launch_stream_rows(int rows, const uint4* src, uint4* dst, long long n_tokens, int nvec) {
+  switch (rows) {
+    case 1: launch_stream<1>(src, dst, n_tokens, nvec); break;
+    case 2: launch_stream<2>(src, dst, n_tokens, nvec); break;
+    case 3: launch_stream<3>(src, dst, n_tokens, nvec); break;
+    case 4: launch_stream<4>(src, dst, n_tokens, nvec); break;
+    case 5: launch_stream<5>(src, dst, n_tokens, nvec); break;
+    case 6: launch_stream<6>(src, dst, n_tokens, nvec); break;
+    case 7: launch_stream<7>(src, dst, n_tokens, nvec); break;
+    case 8: launch_stream<8>(src, dst, n_tokens, nvec); break;
+    case 9: launch_stream<9>(src, dst, n_tokens, nvec); break;
+    default: launch_stream<10>(src, dst, n_tokens, nvec); break;
+  }
+}
+
 }  // namespace
+
+extern "C" int32_t moeca_probe_stream(int32_t device, int64_t n_tokens, int32_t rows, int32_t row_bytes, int32_t reps,
+                                      double* gbs, double* us) {
+  if (!gbs || !us || rows < 1 || rows > 10 || row_bytes < 16 || row_bytes > 65536 || row_bytes % 16 ||
+      n_tokens < 1 || reps < 1 || reps > 1000)
+    return -1;
+  const size_t flush_bytes = size_t(512) << 20;
+  const double src_bytes = static_cast<double>(n_tokens) * rows * row_bytes;
+  const double dst_bytes = static_cast<double>(n_tokens) * row_bytes;
+  if (src_bytes + dst_bytes + static_cast<double>(flush_bytes) > 8.0 * (1ull << 30)) return -1;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+    cudaGetLastError();
+    return -1;
+  }
+  uint4 *src = nullptr, *dst = nullptr, *flush = nullptr;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  int n_sms = 0;
+  bool ok = cudaSetDevice(device) == cudaSuccess &&
+            cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, device) == cudaSuccess &&
+            cudaMalloc(&src, static_cast<size_t>(src_bytes)) == cudaSuccess &&
+            cudaMalloc(&dst, static_cast<size_t>(dst_bytes)) == cudaSuccess &&
+            cudaMalloc(&flush, flush_bytes) == cudaSuccess && cudaMemset(src, 1, static_cast<size_t>(src_bytes)) == cudaSuccess &&
+            cudaMemset(flush, 0, flush_bytes) == cudaSuccess && cudaEventCreate(&e0) == cudaSuccess &&
+            cudaEventCreate(&e1) == cudaSuccess;
+  const int nvec = row_bytes / 16;
+  std::vector<float> times;
+  for (int r = 0; ok && r < reps + 2; ++r) {
+    l2_read_kernel<<<8 * n_sms, 256>>>(flush, flush_bytes / 16, dst);
+    cudaEventRecord(e0);
+    launch_stream_rows(rows, src, dst, n_tokens, nvec);
+    cudaEventRecord(e1);
+    float t = 0.f;
+    ok = cudaEventSynchronize(e1) == cudaSuccess && cudaGetLastError() == cudaSuccess &&
+         cudaEventElapsedTime(&t, e0, e1) == cudaSuccess;
+    if (ok && r >= 2) times.push_back(t);
+  }
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  if (src) cudaFree(src);
+  if (dst) cudaFree(dst);
+  if (flush) cudaFree(flush);
+  if (!ok || times.empty()) {
+    cudaGetLastError();
+    return -3;
+  }
+  std::sort(times.begin(), times.end());
+  const double t_ms = times[times.size() / 2];
+  if (t_ms <= 0.0) return -3;
+  *us = t_ms * 1e3;
+  *gbs = (src_bytes + dst_bytes) / (t_ms * 1e-3) / 1e9;
+  return 0;
+}
 
 extern "C" int32_t moeca_probe_ffma(int32_t device, int32_t iterations, double* tflops, double* ms) {
   if (!tflops || !ms || iterations < 1) return -1;

@@ -143,6 +143,8 @@ def _load():
                                           C.POINTER(C.c_double), C.POINTER(C.c_double), C.POINTER(C.c_double)]),
         "moeca_ddpm_step": (C.c_int, [C.POINTER(moeca_ddpm_args), C.c_void_p]),
         "moeca_probe_ffma": (C.c_int32, [C.c_int32, C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+        "moeca_probe_stream": (C.c_int32, [C.c_int32, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
+                                           C.POINTER(C.c_double), C.POINTER(C.c_double)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -325,6 +327,17 @@ def moeca_probe_ffma(device: int = 0, iterations: int = 1 << 16) -> tuple:
     if st != 0:
         raise MoecaError(st, "moeca_probe_ffma")
     return tf.value, ms.value
+
+
+def moeca_probe_stream(device: int, n_tokens: int, rows: int, row_bytes: int, reps: int = 15) -> tuple:
+    """Streaming rate of ``device`` at one shape: (GB/s, median us) of a kernel
+    that reads ``rows`` rows of ``row_bytes`` per token and writes one
+    (include/moeca_probe.h)."""
+    gbs, us = C.c_double(), C.c_double()
+    st = LIB.moeca_probe_stream(device, n_tokens, rows, row_bytes, reps, C.byref(gbs), C.byref(us))
+    if st != 0:
+        raise MoecaError(st, "moeca_probe_stream")
+    return gbs.value, us.value
 
 
 def moeca_status_string(status: int) -> str:

@@ -1,5 +1,5 @@
 """The host-buffer step (moeca_step_host) against the device-buffer step, and
-the fp32 FFMA probe (marked gpu).
+the measurement probes (marked gpu).
 
 moeca_step_host uploads each input into double-buffered device staging on
 its own stream, runs the same step and reads the output back on another
@@ -90,3 +90,14 @@ def test_ffma_probe(M):
     tf, ms = M.moeca_probe_ffma(0)
     # 152 SMs x 128 FP32 lanes x 2 flops at up to 2.07 GHz is 80.5 TFLOP/s.
     assert 10.0 < tf < 100.0 and ms > 0.0, (tf, ms)
+
+
+def test_stream_probe(M):
+    # 4096 tokens x (2 rows read + 1 written) of 2304 B: 28 MB in, 9 MB out.
+    gbs, us = M.moeca_probe_stream(0, 4096, 2, 2304, reps=5)
+    assert 100.0 < gbs < 20000.0 and us > 0.0, (gbs, us)
+    assert abs(gbs - 4096 * 3 * 2304 / (us * 1e-6) / 1e9) < 1e-6 * gbs
+    with pytest.raises(M.MoecaError):
+        M.moeca_probe_stream(0, 4096, 11, 2304)
+    with pytest.raises(M.MoecaError):
+        M.moeca_probe_stream(0, 4096, 2, 2300)
