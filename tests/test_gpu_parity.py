@@ -226,6 +226,31 @@ def test_tc_and_simt_agree(M):
     assert rel_l2(res[0], res[1]) < 5e-3
 
 
+@pytest.mark.parametrize("split", [2, 3])
+def test_ffn_k_splits(M, split):
+    """The second GEMM split along K (forced; 600 tokens, 16 m-tiles, phase 2
+    in 64-wide tiles with 6 K stages): parity against the oracle over a
+    two-layer trajectory, and the same bits on a second handle.  Two splits
+    add the parked tile to the later split's accumulator, a sum whose value
+    does not depend on which split finishes first; three add in split order."""
+    T, D, E, k, F = 600, 256, 8, 2, 768
+    finals = []
+    for run in range(2):
+        st, cfg, ws = make_stack(M, T, D, E, k, F, L=2, seed=12, tau0=0.75, ffn_split_k=split)
+        rng = np.random.default_rng(120)
+        xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05, True)
+        if run == 0:
+            rep, out = run_trajectory(st, cfg, ws, xs)
+            assert rep.reused > 0 and rep.recomputed > 0, rep
+        else:
+            for t, x in enumerate(xs):
+                out = st.step(torch.from_numpy(x).cuda().to(torch.bfloat16), t)
+        torch.cuda.synchronize()
+        finals.append(out.clone())
+        st.close()
+    assert torch.equal(finals[0], finals[1])
+
+
 @pytest.mark.parametrize("shape", [
     dict(T=300, D=256, E=8, k=2, F=256, S=1, bf16=True),
     dict(T=257, D=128, E=16, k=8, F=128, S=0, bf16=True),
