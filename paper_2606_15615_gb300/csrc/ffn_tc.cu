@@ -709,75 +709,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.dep + 2 * (t.mi * kMaxSplit + t.n / gq))
                          : "memory");
         }
-      } else if (S == 2) {
-        // Two K splits: the first to arrive parks its fp32 tile and releases
-        // it; the second adds the parked tile to its own accumulator as it
-        // stores.  A sum of two values does not depend on their order, so
-        // the bits are the same whichever split arrives first.  tile_sem
-        // counts the two arrivals and the release (3); the second resets it.
-        // The second's wait ends once the first has stored 64-128 KB, which
-        // depends on nothing else.
-        if (leader) ep_last = atomicAdd(a.tile_sem + t.tile, 1);
-        asm volatile("bar.sync 1, 256;" ::: "memory");
-        const int order = ep_last;
-        asm volatile("bar.sync 1, 256;" ::: "memory");  // every thread has read ep_last
-        if (order == 0) {
-          float4* mine = reinterpret_cast<float4*>(a.partial + (static_cast<size_t>(t.tile) * 2 + t.sp) * kBM * BN);
-          for (int c = c_lo; c < c_hi; ++c) {
-            uint32_t v[32];
-            tmem_ld32(tbase + c * 32, v);
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              mine[(c * 8 + j) * kBM + r] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                                        __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
-          }
-          tc_fence_before();
-          mbar_arrive(smem_u32(&tempty_bar[acc]));
-          __threadfence();
-          asm volatile("bar.sync 1, 256;" ::: "memory");
-          if (leader) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.tile_sem + t.tile) : "memory");
-        } else {
-          if (leader) {
-            const unsigned long long t0 = globaltimer();
-            int v = 0;
-            for (;;) {
-              asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(a.tile_sem + t.tile) : "memory");
-              if (v == 3 || globaltimer() - t0 > kWaitNs) break;
-            }
-            if (v != 3) ep_abort = 1;
-          }
-          asm volatile("bar.sync 1, 256;" ::: "memory");
-          if (ep_abort) {
-            if (leader && !abort_flag) report_status(a.status, kStatusWaitTimeout, 350 + a.first);
-            abort_flag = 1;
-            break;
-          }
-          __threadfence();
-          const float4* other =
-              reinterpret_cast<const float4*>(a.partial + (static_cast<size_t>(t.tile) * 2 + (1 - t.sp)) * kBM * BN);
-          for (int c = c_lo; c < c_hi; ++c) {
-            float4 f[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) f[j] = __ldcg(other + (c * 8 + j) * kBM + r);
-            uint32_t v[32];
-            tmem_ld32(tbase + c * 32, v);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              v[4 * j] = __float_as_uint(__uint_as_float(v[4 * j]) + f[j].x);
-              v[4 * j + 1] = __float_as_uint(__uint_as_float(v[4 * j + 1]) + f[j].y);
-              v[4 * j + 2] = __float_as_uint(__uint_as_float(v[4 * j + 2]) + f[j].z);
-              v[4 * j + 3] = __float_as_uint(__uint_as_float(v[4 * j + 3]) + f[j].w);
-            }
-            store_chunk(stage, dst ? dst + c * 32 : nullptr, v, t.p == 0, a.gelu_tanh, lane);
-          }
-          tc_fence_before();
-          mbar_arrive(smem_u32(&tempty_bar[acc]));
-          if (leader) a.tile_sem[t.tile] = 0;
-        }
       } else {
-        // Split K (three or four splits): park this split's fp32 tile, free
-        // TMEM, then the last split to arrive for the tile sums the splits in
-        // split order.  A parked
+        // Split K: park this split's fp32 tile, free TMEM, then the last split
+        // to arrive for the tile sums the splits in split order.  A parked
         // tile is laid out [32-column chunk][4-column group][row][4], so each
         // warp access covers 512 contiguous bytes.
         float4* mine = reinterpret_cast<float4*>(a.partial + (static_cast<size_t>(t.tile) * S + t.sp) * kBM * BN);

@@ -230,9 +230,9 @@ def test_tc_and_simt_agree(M):
 def test_ffn_k_splits(M, split):
     """The second GEMM split along K (forced; 600 tokens, 16 m-tiles, phase 2
     in 64-wide tiles with 6 K stages): parity against the oracle over a
-    two-layer trajectory, and the same bits on a second handle.  Two splits
-    add the parked tile to the later split's accumulator, a sum whose value
-    does not depend on which split finishes first; three add in split order."""
+    two-layer trajectory, and the same bits on a second handle (the last
+    split to arrive adds the parked tiles in split order, whichever arrives
+    first)."""
     T, D, E, k, F = 600, 256, 8, 2, 768
     finals = []
     for run in range(2):
