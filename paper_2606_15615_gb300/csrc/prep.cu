@@ -244,13 +244,16 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   const uint32_t bar = smem_u32(&sm_bar);
   const uint32_t row_bytes = static_cast<uint32_t>(D) * 2;
   constexpr bool kRoute = MODE != 2;  // MODE 2 reads the routing MODE 1 wrote
-  if (t == 0) {
-    mbar_expect_tx(bar, row_bytes * ((kRoute ? E : 0) + ntok + (add_a ? ntok : 0)));
+  // The copies are issued by the lanes of warp 0 (one row each), after lane
+  // 0's expect-tx, which carries the barrier's only arrival.
+  if (t == 0) mbar_expect_tx(bar, row_bytes * ((kRoute ? E : 0) + ntok + (add_a ? ntok : 0)));
+  if (warp == 0) {
+    __syncwarp();
     const __nv_bfloat16* wg = static_cast<const __nv_bfloat16*>(a.w_gate);
     if (kRoute)
-      for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
+      for (int e = lane; e < E; e += 32) bulk_g2s(smem_u32(s_w + e * ldw), wg + static_cast<size_t>(e) * D, row_bytes, bar);
     if constexpr (kAttn) {
-      if (add_a) issue_attn_rows(a, s_a, ldw, tok0, ntok, row_bytes, bar);  // written on an earlier step
+      if (add_a && lane == 0) issue_attn_rows(a, s_a, ldw, tok0, ntok, row_bytes, bar);  // written on an earlier step
     }
   }
   // Prefetch what later phases read: cached metadata and EMA rows.
@@ -276,9 +279,9 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
     reinterpret_cast<uint4*>(s_x + r * ldw)[c] = make_uint4(0, 0, 0, 0);
   }
   pdl_entry();
-  if (t == 0) {
+  if (warp == 0) {
     const __nv_bfloat16* x = static_cast<const __nv_bfloat16*>(a.x);
-    for (int q = 0; q < ntok; ++q)
+    for (int q = lane; q < ntok; q += 32)
       bulk_g2s(smem_u32(s_x + q * ldw), x + static_cast<size_t>(tok0 + q) * D, row_bytes, bar);
   }
   if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);

@@ -66,6 +66,16 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   const int i = blockIdx.x * TB + tok;
   const bool valid = i < a.T;
   const int ntok = min(TB, a.T - static_cast<int>(blockIdx.x) * TB);
+  // Loaded before the dependency wait: the gate bias (a weight) and this
+  // token's EMA values (this layer's state, last written one step earlier by
+  // this kernel, which completed before the previous kernel could start).
+  float bias_pre[EPL], ema_pre[EPL];
+#pragma unroll
+  for (int j = 0; j < EPL; ++j) {
+    const int e = g + G * j;
+    bias_pre[j] = (e < E && a.b_gate) ? a.b_gate[e] : 0.f;
+    ema_pre[j] = (valid && e < E) ? a.ema[static_cast<size_t>(i) * E + e] : 0.f;
+  }
   pdl_entry();
   const uint4* wsrc = static_cast<const uint4*>(a.w_gate);
   int wstride = rowv;
@@ -86,12 +96,15 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   if (stage_wg || stage_x) {
     const uint32_t bar = smem_u32(&sm_bar);
     const uint32_t row_bytes = static_cast<uint32_t>(rowv) * 16;
-    if (t == 0) {
-      mbar_expect_tx(bar, row_bytes * ((stage_wg ? E : 0) + (stage_x ? ntok : 0)));
+    // Lane 0's expect-tx carries the barrier's only arrival; the lanes of
+    // warp 0 then issue one row copy each.
+    if (t == 0) mbar_expect_tx(bar, row_bytes * ((stage_wg ? E : 0) + (stage_x ? ntok : 0)));
+    if (t < 32) {
+      __syncwarp();
       if (stage_wg)
-        for (int e = 0; e < E; ++e) bulk_g2s(smem_u32(sm_wg + e * pstride), wsrc + e * rowv, row_bytes, bar);
+        for (int e = t; e < E; e += 32) bulk_g2s(smem_u32(sm_wg + e * pstride), wsrc + e * rowv, row_bytes, bar);
       if (stage_x)
-        for (int q = 0; q < ntok; ++q)
+        for (int q = t; q < ntok; q += 32)
           bulk_g2s(smem_u32(sm_x + q * pstride),
                    static_cast<const uint4*>(a.x) + static_cast<size_t>(blockIdx.x * TB + q) * rowv, row_bytes, bar);
     }
@@ -170,7 +183,7 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   for (int j = 0; j < EPL; ++j) {
     const int e = g + G * j;
     if (e < E) {
-      zl[j] = z[j] + (a.b_gate ? a.b_gate[e] : 0.f);
+      zl[j] = z[j] + bias_pre[j];
       lmax = fmaxf(lmax, zl[j]);
       labs = fmaxf(labs, fabsf(zl[j]));
     } else {
@@ -250,10 +263,9 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
     if (e < EMAXB) {
       float c = 0.f, u = 0.f;
       if (valid && e < E) {
-        float* cp = a.ema + static_cast<size_t>(i) * E + e;
         const float ind = ((topk_mask >> e) & 1ull) ? 1.f : 0.f;
-        c = a.beta * (*cp) + (1.f - a.beta) * ind;
-        *cp = c;
+        c = a.beta * ema_pre[j] + (1.f - a.beta) * ind;
+        a.ema[static_cast<size_t>(i) * E + e] = c;
         if (c > 0.f) u = c * logf(c);
       }
       sm_S[tok * EMAXB + e] = c;
@@ -307,17 +319,17 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
     const int e = t % E, j = t / E;
     float S = 0.f, U = 0.f;
     if (j < J) {
-      // 16 loads in flight per thread, then added in block order.
+      // 32 loads in flight per thread, then added in block order.
       const float2* part = reinterpret_cast<const float2*>(a.partials);
-      for (unsigned b0 = j; b0 < gridDim.x; b0 += 16u * J) {
-        float2 v[16];
+      for (unsigned b0 = j; b0 < gridDim.x; b0 += 32u * J) {
+        float2 v[32];
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
+        for (int u = 0; u < 32; ++u) {
           const unsigned b = b0 + u * J;
           v[u] = b < gridDim.x ? __ldcg(part + static_cast<size_t>(b) * E + e) : make_float2(0.f, 0.f);
         }
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
+        for (int u = 0; u < 32; ++u) {
           S += v[u].x;
           U += v[u].y;
         }
@@ -337,18 +349,25 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
     }
   }
   __syncthreads();
-  if (t == 0) {
-    float lo = 0.f, hi = 0.f;
-    bool any = false;
-    for (int e = 0; e < E; ++e) {
+  if (t < 32) {
+    // Range of the live experts' entropies (min and max are exact in any order).
+    float lo = INFINITY, hi = -INFINITY;
+    for (int e = t; e < E; e += 32) {
       if (!sm_live[e]) continue;
-      if (!any || sm_H[e] < lo) lo = sm_H[e];
-      if (!any || sm_H[e] > hi) hi = sm_H[e];
-      any = true;
+      lo = fminf(lo, sm_H[e]);
+      hi = fmaxf(hi, sm_H[e]);
     }
-    sm_lo = lo;
-    sm_hi = hi;
-    *a.done = 0u;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    if (t == 0) {
+      const bool any = lo <= hi;
+      sm_lo = any ? lo : 0.f;
+      sm_hi = any ? hi : 0.f;
+      *a.done = 0u;
+    }
   }
   __syncthreads();
   if (t < E) {
