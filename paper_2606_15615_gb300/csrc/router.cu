@@ -54,9 +54,16 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   constexpr int EMAXB = G * EPL;              // experts covered by a group
   constexpr int kThreads = NT;
   constexpr bool kTensor = std::is_same_v<TI, __nv_bfloat16> && TB % 16 == 0 && TB / 16 <= NT / 32;
+  // 32-token blocks for wide gates (256 threads): the logit table and the
+  // entropy terms take the gate rows' shared memory once the tensor cores
+  // are done with it, so the gate matrix and 32 token rows fit beside each
+  // other (the host launches this form only with both staged).
+  constexpr bool kAlias = kTensor && NT == 256;
   extern __shared__ uint4 sm_dyn[];           // [EPAD][rowv + 1] gate rows, [TB][rowv + 1] token rows, logits
-  __shared__ float sm_S[TB * EMAXB];
-  __shared__ float sm_U[TB * EMAXB];
+  __shared__ float sm_S_st[kAlias ? 1 : TB * EMAXB];
+  __shared__ float sm_U_st[kAlias ? 1 : TB * EMAXB];
+  float* sm_S = sm_S_st;
+  float* sm_U = sm_U_st;
   __shared__ int sm_near;
   __shared__ __align__(8) uint64_t sm_bar;
   const int t = threadIdx.x;
@@ -84,7 +91,12 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
   uint4* sm_wg = sm_dyn;
   uint4* sm_x = sm_dyn + (stage_wg ? epad * pstride : 0);
   const bool tensor = kTensor && stage_x && stage_wg;
-  float* sm_logit = reinterpret_cast<float*>(sm_x + TB * pstride);  // [TB][epad + 1], tensor path
+  float* sm_logit = kAlias ? reinterpret_cast<float*>(sm_wg)
+                           : reinterpret_cast<float*>(sm_x + TB * pstride);  // [TB][epad + 1], tensor path
+  if constexpr (kAlias) {
+    sm_S = sm_logit + TB * (epad + 1);
+    sm_U = sm_S + TB * EMAXB;
+  }
   if (t == 0) {
     sm_near = 0;
     if (stage_wg || stage_x) {
@@ -136,20 +148,53 @@ __global__ void __launch_bounds__(NT) router_kernel(RouterArgs a, int stage_x, i
       const __nv_bfloat16* wb = reinterpret_cast<const __nv_bfloat16*>(sm_wg);
       const uint32_t a_addr = smem_u32(xb + (tg * 16 + (lane & 15)) * ldw + (lane >> 4) * 8);
       const int bl = lane & 15;
-      for (int nt = warp % WPG; nt < ntile; nt += WPG) {
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        const uint32_t b_addr = smem_u32(wb + (nt * 8 + (bl & 7)) * ldw + (bl >> 3) * 8);
-        for (int k0 = 0; k0 < a.D; k0 += 16) {
-          uint32_t a0, a1, a2, a3, b0, b1;
-          ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
-          ldsm_x2(b_addr + k0 * 2, b0, b1);
-          mma_16816(acc, a0, a1, a2, a3, b0, b1);
+      if constexpr (kAlias) {
+        // Every warp's n-tiles stay in registers until all warps are done
+        // reading the gate rows; then the table overwrites them.
+        constexpr int NTW = (kMaxExperts / 8 + WPG - 1) / WPG;
+        float acc[NTW][4];
+#pragma unroll
+        for (int q = 0; q < NTW; ++q) {
+          acc[q][0] = acc[q][1] = acc[q][2] = acc[q][3] = 0.f;
+          const int nt = warp % WPG + q * WPG;
+          if (nt < ntile) {
+            const uint32_t b_addr = smem_u32(wb + (nt * 8 + (bl & 7)) * ldw + (bl >> 3) * 8);
+            for (int k0 = 0; k0 < a.D; k0 += 16) {
+              uint32_t a0, a1, a2, a3, b0, b1;
+              ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
+              ldsm_x2(b_addr + k0 * 2, b0, b1);
+              mma_16816(acc[q], a0, a1, a2, a3, b0, b1);
+            }
+          }
         }
-        const int r0 = tg * 16 + (lane >> 2), e0 = nt * 8 + (lane & 3) * 2;
-        sm_logit[r0 * (epad + 1) + e0] = acc[0];
-        sm_logit[r0 * (epad + 1) + e0 + 1] = acc[1];
-        sm_logit[(r0 + 8) * (epad + 1) + e0] = acc[2];
-        sm_logit[(r0 + 8) * (epad + 1) + e0 + 1] = acc[3];
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < NTW; ++q) {
+          const int nt = warp % WPG + q * WPG;
+          if (nt < ntile) {
+            const int r0 = tg * 16 + (lane >> 2), e0 = nt * 8 + (lane & 3) * 2;
+            sm_logit[r0 * (epad + 1) + e0] = acc[q][0];
+            sm_logit[r0 * (epad + 1) + e0 + 1] = acc[q][1];
+            sm_logit[(r0 + 8) * (epad + 1) + e0] = acc[q][2];
+            sm_logit[(r0 + 8) * (epad + 1) + e0 + 1] = acc[q][3];
+          }
+        }
+      } else {
+        for (int nt = warp % WPG; nt < ntile; nt += WPG) {
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+          const uint32_t b_addr = smem_u32(wb + (nt * 8 + (bl & 7)) * ldw + (bl >> 3) * 8);
+          for (int k0 = 0; k0 < a.D; k0 += 16) {
+            uint32_t a0, a1, a2, a3, b0, b1;
+            ldsm_x4(a_addr + k0 * 2, a0, a1, a2, a3);
+            ldsm_x2(b_addr + k0 * 2, b0, b1);
+            mma_16816(acc, a0, a1, a2, a3, b0, b1);
+          }
+          const int r0 = tg * 16 + (lane >> 2), e0 = nt * 8 + (lane & 3) * 2;
+          sm_logit[r0 * (epad + 1) + e0] = acc[0];
+          sm_logit[r0 * (epad + 1) + e0 + 1] = acc[1];
+          sm_logit[(r0 + 8) * (epad + 1) + e0] = acc[2];
+          sm_logit[(r0 + 8) * (epad + 1) + e0 + 1] = acc[3];
+        }
       }
       __syncthreads();
 #pragma unroll
@@ -392,6 +437,7 @@ constexpr size_t kSmemPerBlock = 227 * 1024;
 template <typename TI, int G, int EPL, int NT>
 cudaError_t launch_g(const RouterArgs& a, cudaStream_t s) {
   constexpr int TB = NT / G;
+  constexpr bool kAlias = std::is_same_v<TI, __nv_bfloat16> && NT == 256;
   // The staging cap depends on the kernel's static shared memory only; the
   // attribute that allows it is set on every device the process uses.
   cudaFuncAttributes attr;
@@ -404,6 +450,13 @@ cudaError_t launch_g(const RouterArgs& a, cudaStream_t s) {
   const size_t row = static_cast<size_t>(a.D / Elem<TI>::kVec + 1) * 16;
   const size_t epad = (a.E + 7) / 8 * 8;
   const size_t wg_bytes = epad * row, x_bytes = TB * row, logit_bytes = TB * (epad + 1) * 4;
+  if constexpr (kAlias) {
+    // The logit table and the entropy terms must fit in the gate rows' space,
+    // and both the gate rows and the token rows must be staged.
+    const size_t alias_bytes = logit_bytes + 2 * static_cast<size_t>(TB) * G * EPL * 4;
+    if (wg_bytes + x_bytes > cap || alias_bytes > wg_bytes) return cudaErrorNotSupported;
+    return launch_pdl(router_kernel<TI, G, EPL, NT>, dim3(grid), dim3(NT), wg_bytes + x_bytes, s, a, 1, 1);
+  }
   const int stage_wg = wg_bytes <= cap;
   const int stage_x = stage_wg && wg_bytes + x_bytes + logit_bytes <= cap;
   const size_t smem = (stage_wg ? wg_bytes : 0) + (stage_x ? x_bytes + logit_bytes : 0);
@@ -421,6 +474,12 @@ cudaError_t launch_t(const RouterArgs& a, cudaStream_t s) {
   // 16 tokens per block for wide gates, so the token rows and the logit
   // table fit beside the staged gate matrix (the tensor-core path).
   if (E <= 32) return launch_g<TI, 8, 4, 128>(a, s);
+  if constexpr (std::is_same_v<TI, __nv_bfloat16>) {
+    // 32-token blocks (one wave of 128 blocks at 4096 tokens) when the gate
+    // matrix and the token rows fit in shared memory together.
+    const cudaError_t e = launch_g<TI, 8, 8, 256>(a, s);
+    if (e != cudaErrorNotSupported) return e;
+  }
   return launch_g<TI, 8, 8, 128>(a, s);
 }
 
