@@ -8,6 +8,8 @@
 // (group, m-tile) from them; blocks past the last tile exit.  fp32 FFMA with
 // fp32 accumulation: the fp32 debug-precision path, and a cross-check of the
 // tensor-core kernel on bf16.
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -108,6 +110,136 @@ __global__ void __launch_bounds__(256) ffn_simt_kernel(FfnArgs a) {
   }
 }
 
+// fp32 form with the operand tiles brought into shared memory by cp.async,
+// three stages in flight, so a block's K loop does not wait one memory
+// round trip per tile.  Tiles keep K contiguous (rows padded to 36 floats);
+// thread (ty, tx) owns outputs (ty + 16 r, tx + 16 c), so the 16-byte shared
+// loads of a quarter warp fall in distinct banks.  Every output still sums
+// its K terms in increasing order with one fmaf each, starting from zero, as
+// the plain form does, so both give the same bits.
+constexpr int PBM = 64, PBN = 64, PBK = 32, PST = 3, PLD = PBK + 4;
+constexpr size_t kPipeSmem = static_cast<size_t>(PST) * (PBM + PBN) * PLD * sizeof(float);
+
+__device__ __forceinline__ void cp_async16_zf(uint32_t dst, const void* src, bool valid) {
+  const int n = valid ? 16 : 0;  // 0: the 16 bytes are zero-filled
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
+}
+
+template <int PHASE>
+__global__ void __launch_bounds__(256) ffn_simt_pipe_kernel(FfnArgs a) {
+  pdl_entry();
+  const int N = PHASE == 1 ? a.F : a.D;
+  const int K = PHASE == 1 ? a.D : a.F;
+  int mt = blockIdx.y, g = -1, m0 = 0;
+  for (int gg = 0; gg < a.G; ++gg) {
+    const int tiles = (a.counts[gg] + PBM - 1) / PBM;
+    if (mt < tiles) {
+      g = gg;
+      m0 = mt * PBM;
+      break;
+    }
+    mt -= tiles;
+  }
+  if (g < 0) return;
+  const int rows = a.counts[g];
+  const int row0 = a.offsets[g];
+  const int n0 = blockIdx.x * PBN;
+  const float* A = static_cast<const float*>(PHASE == 1 ? a.xg : a.hmid);
+  const float* B;
+  if (g < a.E) {
+    B = static_cast<const float*>(PHASE == 1 ? a.w1 : a.w2) + static_cast<size_t>(g) * a.F * a.D;
+  } else {
+    B = static_cast<const float*>(PHASE == 1 ? a.ws1 : a.ws2);
+  }
+  extern __shared__ __align__(16) float sm_pipe[];
+  float* As = sm_pipe;                    // [PST][PBM][PLD]
+  float* Bs = sm_pipe + PST * PBM * PLD;  // [PST][PBN][PLD]
+  const int t = threadIdx.x, ty = t >> 4, tx = t & 15;
+  const int KT = (K + PBK - 1) / PBK;
+  // Stage st <- K tile kt: 64 rows x 8 chunks of 4 floats per operand, two
+  // chunks of each per thread; chunks past K or past the rows are zeros.
+  auto load = [&](int kt, int st) {
+    const int k0 = kt * PBK;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = t + h * 256, r = c >> 3, kc = (c & 7) * 4;
+      const bool in_k = k0 + kc < K;
+      const bool va = in_k && m0 + r < rows;
+      const bool vb = in_k && n0 + r < N;
+      cp_async16_zf(smem_u32(As + (st * PBM + r) * PLD + kc),
+                    va ? A + static_cast<size_t>(row0 + m0 + r) * K + k0 + kc : A, va);
+      cp_async16_zf(smem_u32(Bs + (st * PBN + r) * PLD + kc),
+                    vb ? B + static_cast<size_t>(n0 + r) * K + k0 + kc : B, vb);
+    }
+  };
+  float acc[4][4];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+#pragma unroll
+  for (int st = 0; st < PST - 1; ++st) {
+    if (st < KT) load(st, st);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+  for (int kt = 0; kt < KT; ++kt) {
+    asm volatile("cp.async.wait_group %0;" ::"n"(PST - 2) : "memory");
+    __syncthreads();  // tile kt is in; every thread is done with tile kt - 1
+    const int st = kt % PST;
+    const float* as = As + st * PBM * PLD;
+    const float* bs = Bs + st * PBN * PLD;
+#pragma unroll
+    for (int kk = 0; kk < PBK; kk += 4) {
+      float4 av[4], bv[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) av[r] = *reinterpret_cast<const float4*>(as + (ty + 16 * r) * PLD + kk);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) bv[c] = *reinterpret_cast<const float4*>(bs + (tx + 16 * c) * PLD + kk);
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          acc[r][c] = fmaf(av[r].x, bv[c].x, acc[r][c]);
+          acc[r][c] = fmaf(av[r].y, bv[c].y, acc[r][c]);
+          acc[r][c] = fmaf(av[r].z, bv[c].z, acc[r][c]);
+          acc[r][c] = fmaf(av[r].w, bv[c].w, acc[r][c]);
+        }
+    }
+    // Refill the stage tile kt - 1 used.
+    const int nk = kt + PST - 1;
+    if (nk < KT) load(nk, nk % PST);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int m = m0 + ty + 16 * r;
+    if (m >= rows) continue;
+    const size_t row = static_cast<size_t>(row0 + m);
+    if (PHASE == 1) {
+      float* H = static_cast<float*>(a.hmid);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int n = n0 + tx + 16 * c;
+        if (n < N) H[row * a.F + n] = gelu_f(acc[r][c], a.gelu_tanh);
+      }
+    } else {
+      const int dr = a.list[row];
+      const int lim = g < a.E ? a.T * a.k : a.T;
+      if (dr < 0 || dr >= lim) {
+        report_status(a.status, kStatusBadIndex, 2000000 + static_cast<int>(row));
+        continue;
+      }
+      float* dst = static_cast<float*>(g < a.E ? a.cache_h : a.shared_h);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int n = n0 + tx + 16 * c;
+        if (n < N) dst[static_cast<size_t>(dr) * a.D + n] = acc[r][c];
+      }
+    }
+  }
+}
+
 // Plain launches: the grid covers the worst case, and its blocks launched
 // early under a programmatic dependency would sit resident beside the
 // previous kernel's blocks and slow them (measured: 455 vs 209 us per step
@@ -115,6 +247,17 @@ __global__ void __launch_bounds__(256) ffn_simt_kernel(FfnArgs a) {
 template <typename TI>
 cudaError_t launch_t(const FfnArgs& a, int phase, cudaStream_t s) {
   const int N = phase == 1 ? a.F : a.D;
+  auto al16 = [](const void* p) { return reinterpret_cast<uintptr_t>(p) % 16 == 0; };
+  if (std::is_same_v<TI, float> && a.D % 4 == 0 && a.F % 4 == 0 && al16(a.xg) && al16(a.hmid) && al16(a.w1) &&
+      al16(a.w2) && al16(a.ws1) && al16(a.ws2)) {
+    // The pipelined form (16-byte row chunks: K a multiple of 4 floats, aligned operands).
+    auto kern = phase == 1 ? ffn_simt_pipe_kernel<1> : ffn_simt_pipe_kernel<2>;
+    const cudaError_t e = set_dyn_smem_on_device(reinterpret_cast<const void*>(kern), static_cast<int>(kPipeSmem));
+    if (e != cudaSuccess) return e;
+    const dim3 grid((N + PBN - 1) / PBN, (a.max_rows + PBM - 1) / PBM + a.G);
+    kern<<<grid, 256, kPipeSmem, s>>>(a);
+    return cudaGetLastError();
+  }
   const dim3 grid((N + BN - 1) / BN, (a.max_rows + BM - 1) / BM + a.G);
   if (phase == 1) ffn_simt_kernel<TI, 1><<<grid, 256, 0, s>>>(a);
   else ffn_simt_kernel<TI, 2><<<grid, 256, 0, s>>>(a);
