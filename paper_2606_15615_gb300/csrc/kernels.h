@@ -116,7 +116,8 @@ struct FfnArgs {
   int gelu_tanh;
   int tile_n;            // tensor-core tile width to force (0: chosen per launch)
   int split_k;           // tensor-core K splits to force (0: chosen per launch)
-  float* partial;        // split-K workspace of the tensor-core path (or null: no split)
+  float* partial;        // split-K workspace: tensor-core path, or the fp32 path's [simt_split, max_rows, D]
+  int simt_split;        // fp32 path: K splits of the second GEMM (1: none)
   int* tile_sem;         // split-K arrival counters, zeroed once
   int* dep;              // tensor-core fused launch: per m-tile counter pairs, zeroed once (or null)
   int max_mtiles;        // capacity of dep, tc_dep_pairs(max_rows, G)

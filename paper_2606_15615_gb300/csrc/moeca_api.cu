@@ -124,6 +124,8 @@ struct moeca_handle {
   void* xg = nullptr;
   void* hmid = nullptr;
   float* tc_partial = nullptr;
+  float* simt_partial = nullptr;  // fp32 path: second-GEMM K-split partials [simt_split, max_rows, D]
+  int simt_split = 1;
   int* tc_sem = nullptr;
   int* tc_dep = nullptr;        // fused GEMM launch: m-tile dependency counters, left at 0
   int* tc_work = nullptr;       // GEMM unit tickets {next, CTAs done}, left at 0
@@ -329,7 +331,8 @@ FfnArgs ffn_args(const moeca_handle* h, const LayerBuf& L, int T, const void* mo
   fa.xg = h->xg; fa.hmid = h->hmid; fa.x = kGemmGathersRows ? moe_in : nullptr;
   fa.w1 = L.w.w1; fa.w2 = L.w.w2; fa.ws1 = L.w.ws1; fa.ws2 = L.w.ws2;
   fa.cache_h = L.cache_h; fa.shared_h = L.shared_h; fa.gelu_tanh = c.gelu_tanh; fa.status = h->status_dev;
-  fa.partial = h->tc_partial; fa.tile_sem = h->tc_sem;
+  fa.partial = h->simt_partial ? h->simt_partial : h->tc_partial; fa.tile_sem = h->tc_sem;
+  fa.simt_split = h->simt_split;
   fa.dep = h->tc_dep; fa.max_mtiles = h->tc_dep_pairs_n; fa.work = h->tc_work;
   return fa;
 }
@@ -555,6 +558,18 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
   A((void**)&h->block_offsets, nblk_sel * G * 4);
   A(&h->xg, static_cast<size_t>(h->max_rows) * D * es);
   A(&h->hmid, static_cast<size_t>(h->max_rows) * F * es);
+  if (!use_tc && !bf16) {
+    // fp32: the second GEMM (few outputs, long K) in K splits, their partials
+    // added in split order by a second pass; four splits while the workspace
+    // stays within 512 MB.
+    for (int sk = 4; sk > 1; sk /= 2) {
+      if (static_cast<size_t>(sk) * h->max_rows * D * 4 <= (size_t(512) << 20)) {
+        h->simt_split = sk;
+        break;
+      }
+    }
+    if (h->simt_split > 1) A((void**)&h->simt_partial, static_cast<size_t>(h->simt_split) * h->max_rows * D * 4);
+  }
   if (use_tc) {
     A((void**)&h->tc_partial, tc_partial_bytes(h->n_sms));
     A((void**)&h->tc_sem, tc_split_units(h->n_sms) * sizeof(int));
