@@ -833,21 +833,30 @@ TcShape make_shape(int N, int K, int BN) {
   return t;
 }
 
-// Tile-width choice: the widest candidate that still yields at least half
-// a wave of tiles (wider tiles re-read the 128 activation rows fewer times
-// per weight byte; too few tiles leave SMs idle), else the narrowest.
-// Measured on the 12-layer D768 stack at ~60% reuse (16 m-tiles, one
-// fused launch): phase-2 width 128 took 51 us, 64 took 59 us, and 256
-// (48 tiles) 56 us with two K splits.  K splits are used only when forced:
-// their parked partials and reductions cost 4-9 us of epilogue per unit.
+// Tile-width choice.  A unit moves (128 + BN) x K bf16 through its SM's
+// ring, whose fill rate bounds it, and units run in waves of one per CTA:
+// the width with the fewest waves x bytes per unit, the wider on a tie.
+// Measured on the 12-layer D768 stack at ~60% reuse (16 m-tiles, one fused
+// launch): phase-2 width 128 took 51 us, 64 took 59 us, and 256 (48 tiles)
+// 56 us with two K splits; on the 28-layer D1152 stack (32 m-tiles) phase-2
+// width 128 (288 tiles, 2 waves of 2.4 MB) beat 192 (192 tiles, 2 waves of
+// 2.9 MB).  K splits are used only when forced: their parked partials and
+// reductions cost 4-9 us of epilogue per unit.
 int pick_width(const TcShape* shp, int mt, int grid, int force_bn) {
-  int last = -1;
+  int best = -1;
+  double best_cost = 0.0;
   for (int i = 0; i < 3; ++i) {
     if (!shp[i].BN || (force_bn && shp[i].BN != force_bn)) continue;
-    if (2 * mt * shp[i].nt >= grid) return i;
-    last = i;
+    const long long units = static_cast<long long>(mt) * shp[i].nt;
+    const long long waves = (units + grid - 1) / grid;
+    const double K = static_cast<double>(shp[i].KB) * shp[i].sub * kBK;
+    const double cost = static_cast<double>(waves) * (kBM + shp[i].BN) * K;
+    if (best < 0 || cost < best_cost) {
+      best = i;
+      best_cost = cost;
+    }
   }
-  return last < 0 ? 0 : last;  // forced width absent: the widest
+  return best < 0 ? 0 : best;  // forced width absent: the widest
 }
 
 // Plan for `mt` m-tiles: fused (section 0) or one phase alone (section 1 + p).
