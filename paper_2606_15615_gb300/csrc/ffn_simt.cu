@@ -269,13 +269,16 @@ __global__ void __launch_bounds__(256) ffn_split_sum_kernel(FfnArgs a) {
   pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G, E = a.E, S = a.simt_split;
-  const int rows = a.offsets[G];
+  __shared__ int off_sm[kMaxExperts + 2];  // group offsets, read once
+  for (int g = threadIdx.x; g <= G; g += blockDim.x) off_sm[g] = a.offsets[g];
+  __syncthreads();
+  const int rows = off_sm[G];
   const int nv = a.D / 4;
   for (int r = blockIdx.x * 8 + warp; r < rows; r += gridDim.x * 8) {
     int lo = 0, hi = G - 1;  // group of row r: the last g with offsets[g] <= r
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (a.offsets[mid] <= r) lo = mid;
+      if (off_sm[mid] <= r) lo = mid;
       else hi = mid - 1;
     }
     const int dr = a.list[r];

@@ -212,7 +212,10 @@ __global__ void __launch_bounds__(256) gather_kernel(CompactArgs a) {
   pdl_entry();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = a.G, E = a.E;
-  const int rows = a.offsets[G];
+  __shared__ int off_sm[kMaxGroups + 1];  // group offsets, read once
+  for (int g = threadIdx.x; g <= G; g += blockDim.x) off_sm[g] = a.offsets[g];
+  __syncthreads();
+  const int rows = off_sm[G];
   const int nv = a.D * static_cast<int>(sizeof(TI)) / 16;
   const uint4* x = static_cast<const uint4*>(a.x);
   uint4* xg = static_cast<uint4*>(a.xg);
@@ -221,7 +224,7 @@ __global__ void __launch_bounds__(256) gather_kernel(CompactArgs a) {
     int lo = 0, hi = G - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (a.offsets[mid] <= r) lo = mid;
+      if (off_sm[mid] <= r) lo = mid;
       else hi = mid - 1;
     }
     const int ent = a.list[r];
