@@ -17,7 +17,9 @@ import pytest
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-from gpu_harness import np_of  # noqa: E402
+from gpu_harness import (Report, assert_margins, check_gate_weights, count_route_margins, np_of,  # noqa: E402
+                         oracle_weights, params_of)
+from oracle import moeca_oracle as O  # noqa: E402
 from paper_2606_15615_gb300 import workloads as W  # noqa: E402
 
 
@@ -71,6 +73,49 @@ def test_noalloc_router_matches_moeca_step_twice(M, bf16):
         assert np.allclose(np_of(ema), np_of(st["ema"]), rtol=2e-6, atol=1e-7)
         assert np.allclose(np_of(tau), np_of(tr["tau"]), rtol=1e-5, atol=1e-6)
     stack.close()
+
+
+@pytest.mark.parametrize("D,bf16", [(1152, True), (1536, True), (1152, False)])
+def test_noalloc_wide_gate_router_against_oracle(M, D, bf16):
+    """64 experts, top-8, 300 tokens (a ragged last block), two calls in a row,
+    against the oracle: the ids outside near ties, the gate weights, the EMA
+    statistic (Eq. 10) and the thresholds (Eq. 11-12).  The shapes take the
+    router's wide-gate forms: 32-token blocks with the gate matrix and the
+    token rows in shared memory together (D 1152, bf16), 16-token blocks with
+    the token rows read through L1 (D 1536), and the fp32 form."""
+    T, E, k = 300, 64, 8
+    w, x0, rng = W.tiny_layer(41, T, D, E, k, 64, dtype="bf16" if bf16 else "f32", bias=True, wscale=0.05)
+    cfg = M.moeca_config_default(n_layers=1, hidden=D, ffn=64, n_experts=E, top_k=k, max_tokens=T,
+                                 dtype=M.MOECA_BF16 if bf16 else M.MOECA_F32, tau0=0.75)
+    prm = params_of(cfg)
+    dt = torch.bfloat16 if bf16 else torch.float32
+    wg = torch.from_numpy(w["w_gate"]).cuda().to(dt)
+    bg = torch.from_numpy(w["b_gate"]).cuda()
+    wo = oracle_weights({"w_gate": w["w_gate"], "b_gate": w["b_gate"]})
+    ema = torch.zeros((T, E), dtype=torch.float32, device="cuda")
+    rep = Report()
+    C_pre = np.zeros((E, T))
+    x1 = x0 + 0.05 * rng.standard_normal(x0.shape).astype(np.float32)
+    for xn in (x0, x1):
+        if bf16:
+            xn = W.round_to_bf16(xn)
+        x = torch.from_numpy(np.ascontiguousarray(xn, np.float32)).cuda().to(dt)
+        e, rw, tau = _noalloc(M, cfg, x, wg, bg, ema, T)
+        torch.cuda.synchronize()
+        e_g = np_of(e).astype(np.int64)
+        w_g = np_of(rw).astype(np.float64)
+        e_o, w_o, ok, cond = count_route_margins(rep, np_of(x).astype(np.float64), wo, k, bool(cfg.renorm_topk), e_g)
+        bad = np.nonzero(ok & (e_o != e_g).any(axis=1))[0]
+        assert len(bad) == 0, f"top-k ids differ on {len(bad)} tokens, e.g. {bad[:5]}"
+        check_gate_weights(w_g[ok], w_o[ok], cond[ok])
+        C_g = np_of(ema).astype(np.float64).T
+        C_o = O.ema_update(C_pre, e_g, prm.beta)
+        assert np.allclose(C_g, C_o, rtol=2e-6, atol=1e-7), f"EMA: max err {np.abs(C_g - C_o).max()}"
+        tau_o = O.expert_threshold(O.normalized_entropy(C_g, prm.entropy_norm), prm.tau0, prm.alpha)
+        tau_g = np_of(tau).astype(np.float64)
+        assert np.allclose(tau_g, tau_o, rtol=1e-5, atol=1e-6), f"tau: max err {np.abs(tau_g - tau_o).max()}"
+        C_pre = C_g
+    assert_margins(rep)
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch(M):
