@@ -70,7 +70,9 @@ __global__ void __launch_bounds__(kWarps * 32, MINB) combine_kernel(CombineArgs 
   // token_any comes from the preparation kernel, which completed before the
   // previous kernel passed its own dependency wait.
   const bool copy_tok = YC && a.copy_y && !a.token_any[i];
-  pdl_entry();
+  // A token whose branches are all reused (its shared row too) reads nothing
+  // the grouped GEMM before this kernel writes, so it does not wait for it.
+  if (!(a.early && !a.token_any[i])) pdl_entry();
   if (bad) {
     if (lane == 0) report_status(a.status, kStatusBadIndex, 3000000 + i);
     return;

@@ -219,6 +219,9 @@ struct CombineArgs {
                           //   token_reuse_policy 1); 0: every token computes y (and stores it)
   int n_sms;              // the device's SM count (the staged form's persistent grid)
   int direct;             // 1: force the direct form (one warp per token, rows loaded by the lanes)
+  int early;              // 1: in the direct form, a token with token_any 0 is combined without
+                          //   waiting for the previous kernel (a cache step, no token-level copy,
+                          //   the shared row, if any, recomputed only for tokens with token_any)
   int* status;
 };
 cudaError_t launch_combine(const CombineArgs& a, bool bf16, cudaStream_t s);

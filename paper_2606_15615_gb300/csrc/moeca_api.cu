@@ -350,6 +350,9 @@ CombineArgs combine_args(const moeca_handle* h, const LayerBuf& L, int T, const 
     cb.cache_y = L.cache_y; cb.token_any = L.token_any; cb.copy_y = refresh ? 0 : 1;
   }
   cb.rearm = use_tc ? h->tc_work : nullptr;
+  // A fully reused token's rows are not written by this layer's GEMM.
+  cb.token_any = L.token_any;
+  cb.early = !refresh && !L.cache_y && (c.n_shared == 0 || c.shared_policy == 0) ? 1 : 0;
   return cb;
 }
 
