@@ -28,15 +28,17 @@ constexpr int kThreads = kSelectTokensPerBlock;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxGroups = kMaxExperts + 1;
 
+// KMAX >= k bounds the per-token loops at compile time.
+template <int KMAX>
 __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
   pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int i = blockIdx.x * kThreads + t;
   const bool valid = i < a.T;
   const int k = a.k, E = a.E, G = a.G;
-  TokenDecision d;
+  TokenDecisionT<KMAX> d;
   const size_t b0 = static_cast<size_t>(valid ? i : 0) * a.k;
-  decide_token<kMaxTopK>(a, i, valid, a.route_e + b0, a.route_w + b0, a.cache_e + b0, a.cache_w + b0, a.cache_norm + b0, d);
+  decide_token<KMAX>(a, i, valid, a.route_e + b0, a.route_w + b0, a.cache_e + b0, a.cache_w + b0, a.cache_norm + b0, d);
   const int* e = d.e;
   const bool* rec = d.rec;
   const bool any = d.any, bad = d.bad, shared_row = d.shared_row;
@@ -48,7 +50,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
     bool has = false;
     if (g < E) {
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) has |= (rec[p] && e[p] == g);
+      for (int p = 0; p < KMAX; ++p) has |= (rec[p] && e[p] == g);
     } else {
       has = shared_row;
     }
@@ -139,18 +141,18 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
   }
 }
 
-template <typename TI>
+template <typename TI, int KMAX>
 __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
   pdl_entry();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int i = blockIdx.x * kThreads + t;
   const bool valid = i < a.T;
   const int k = a.k, E = a.E, G = a.G;
-  int e[kMaxTopK], sl[kMaxTopK];
-  bool rec[kMaxTopK];
+  int e[KMAX], sl[KMAX];
+  bool rec[KMAX];
   bool any = false;
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) {
+  for (int p = 0; p < KMAX; ++p) {
     e[p] = -1;
     sl[p] = 0;
     rec[p] = false;
@@ -171,7 +173,7 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
     bool has = false;
     if (g < E) {
 #pragma unroll
-      for (int p = 0; p < kMaxTopK; ++p) has |= (rec[p] && e[p] == g);
+      for (int p = 0; p < KMAX; ++p) has |= (rec[p] && e[p] == g);
     } else {
       has = shared_row;
     }
@@ -190,7 +192,7 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(CompactArgs a) {
   __syncthreads();
   const unsigned lt = (1u << lane) - 1u;
 #pragma unroll
-  for (int p = 0; p < kMaxTopK; ++p) {
+  for (int p = 0; p < KMAX; ++p) {
     if (rec[p]) {
       const int g = e[p];
       const int pos = sm_pre[warp][g] + __popc(sm_bal[warp][g] & lt);
@@ -243,13 +245,19 @@ __global__ void __launch_bounds__(256) gather_kernel(CompactArgs a) {
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t s) {
   const int grid = (a.T + kThreads - 1) / kThreads;
-  return launch_pdl(select_kernel, dim3(grid), dim3(kThreads), 0, s, a);
+  if (a.k <= 2) return launch_pdl(select_kernel<2>, dim3(grid), dim3(kThreads), 0, s, a);
+  if (a.k <= 4) return launch_pdl(select_kernel<4>, dim3(grid), dim3(kThreads), 0, s, a);
+  return launch_pdl(select_kernel<kMaxTopK>, dim3(grid), dim3(kThreads), 0, s, a);
 }
 
 cudaError_t launch_compact(const CompactArgs& a, bool bf16, cudaStream_t s) {
   const int grid = (a.T + kThreads - 1) / kThreads;
-  cudaError_t e = bf16 ? launch_pdl(compact_kernel<__nv_bfloat16>, dim3(grid), dim3(kThreads), 0, s, a)
-                       : launch_pdl(compact_kernel<float>, dim3(grid), dim3(kThreads), 0, s, a);
+  auto run = [&](auto kern) { return launch_pdl(kern, dim3(grid), dim3(kThreads), 0, s, a); };
+  cudaError_t e;
+  if (bf16) e = a.k <= 2 ? run(compact_kernel<__nv_bfloat16, 2>) : a.k <= 4 ? run(compact_kernel<__nv_bfloat16, 4>)
+                                                                            : run(compact_kernel<__nv_bfloat16, kMaxTopK>);
+  else e = a.k <= 2 ? run(compact_kernel<float, 2>) : a.k <= 4 ? run(compact_kernel<float, 4>)
+                                                             : run(compact_kernel<float, kMaxTopK>);
   if (e != cudaSuccess || a.xg == nullptr) return e;
   // The row gather runs over the whole list, one warp per row.
   const int rows = a.T * (a.k + a.n_shared);
