@@ -218,7 +218,7 @@ class Runner:
     token-sharded step whose per-layer exchange is an NCCL all-gather."""
 
     def __init__(self, wl, device_index: int, n_steps: int, tile_n: int = 0, split_k: int = 0, shard=None,
-                 combine_staged: bool = False):
+                 combine_staged: bool = False, prefetch_mb=None):
         import numpy as np
         import torch
         from paper_2606_15615_gb300 import build
@@ -238,6 +238,8 @@ class Runner:
             dtype=M.MOECA_BF16 if wl.dtype == "bf16" else M.MOECA_F32, refresh_period=wl.refresh_period,
             ffn_tile_n=tile_n, ffn_split_k=split_k, n_heads=wl.n_heads, seq_len=wl.seq if wl.n_heads else 0,
             adaln=int(wl.adaln), combine_direct=0 if combine_staged else 1)
+        if prefetch_mb is not None:
+            cfg.weight_prefetch_mb = prefetch_mb
         self.cfg = cfg
         self.stack = M.Stack(cfg, self.weights, device=device_index)
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -685,7 +687,7 @@ def sharded_main(args, wl, world, rank, local, dist):
     if wl.n_tokens % (32 * world):
         raise SystemExit(f"{wl.n_tokens} tokens do not split into {world} slices of whole 32-token blocks")
     runner = Runner(wl, local, args.warmup + args.steps, args.ffn_tile_n, args.ffn_split_k, shard=(rank, world),
-                    combine_staged=args.combine_staged)
+                    combine_staged=args.combine_staged, prefetch_mb=args.weight_prefetch_mb)
     pt = headline_point(wl, args.reuse)
     tau0 = args.tau0 if args.tau0 is not None else (pt["tau0"] if pt else args.ref_tau0)
     W_, K = args.warmup, args.steps
@@ -738,6 +740,8 @@ def main():
     ap.add_argument("--combine-staged", action="store_true",
                     help="stage the combine's rows in shared memory where they fit (default: the direct form)")
     ap.add_argument("--ffn-split-k", type=int, default=0, help="force the tensor-core FFN K splits (0: auto)")
+    ap.add_argument("--weight-prefetch-mb", type=int, default=None,
+                    help="MB of each layer's routed W1 the preparation kernel brings into L2 (default: the library's)")
     ap.add_argument("--tau0", type=float, default=None,
                     help="use this tau0 for the headline point instead of the stored / calibrated one")
     ap.add_argument("--layers", type=int, default=0,
@@ -764,7 +768,7 @@ def main():
     if args.shard and world > 1:
         return sharded_main(args, wl, world, rank, local, dist)
     runner = Runner(wl, local, args.warmup + args.steps, args.ffn_tile_n, args.ffn_split_k,
-                    combine_staged=args.combine_staged)
+                    combine_staged=args.combine_staged, prefetch_mb=args.weight_prefetch_mb)
     dev = runner.dev
     W_, K = args.warmup, args.steps
     targets = [args.reuse] if args.no_sweep else sorted(set(wl.reuse_targets) | {args.reuse})

@@ -140,6 +140,12 @@ typedef struct {
                                  token's rows into shared memory with bulk copies while it combines
                                  the previous one (the direct form otherwise, and always under the
                                  token-level reading above).  Both give the same bits */
+  int32_t weight_prefetch_mb; /* bf16 layers run by the fused preparation kernel: while that kernel
+                                 routes and decides, its blocks bring up to this many MB of the
+                                 layer's routed first-GEMM weights (W1, from expert 0 on, the order
+                                 in which the grouped GEMM takes them) into L2, so that the GEMM's
+                                 first phase reads them from L2 instead of HBM.  A cache hint: the
+                                 results do not depend on it.  0 = none; default 16; at most 4096 */
 } moeca_config;
 
 /* Fill `cfg` with the defaults above and the paper's hyper-parameters

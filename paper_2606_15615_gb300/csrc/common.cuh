@@ -183,6 +183,23 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                : "memory");
 }
 
+// L2 prefetch hint over [base, base + bytes) in 32 KB pieces, without waiting:
+// part `part` of `parts` takes pieces part, part + parts, ..., one per lane
+// of the calling warp at a time, so that all parts together cover the range
+// from its start.  base is 16-byte aligned and bytes a multiple of 16.
+constexpr uint32_t kL2PrefetchPiece = 32768;
+__device__ __forceinline__ void l2_prefetch_share(const void* base, size_t bytes, int part, int parts, int lane) {
+  const size_t pieces = (bytes + kL2PrefetchPiece - 1) / kL2PrefetchPiece;
+  const size_t step = static_cast<size_t>(parts) * 32;
+  for (size_t p = static_cast<size_t>(part) + static_cast<size_t>(parts) * lane; p < pieces; p += step) {
+    const size_t off = p * kL2PrefetchPiece;
+    const size_t rest = bytes - off;
+    const uint32_t n = rest < kL2PrefetchPiece ? static_cast<uint32_t>(rest) : kL2PrefetchPiece;
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(base) + off), "r"(n)
+                 : "memory");
+  }
+}
+
 __device__ __forceinline__ float gelu_f(float z, int tanh_form) {
   if (tanh_form) {
     const float c = 0.7978845608028654f;  // sqrt(2 / pi)

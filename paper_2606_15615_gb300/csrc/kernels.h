@@ -177,6 +177,8 @@ struct PrepArgs {
   int32_t* attn_inv;      //   [T] each token's place (-1 if absent),
   int32_t* sample_lo;     //   [T / seq + 1] where each sample's tokens start
   int seq;                //   tokens per sample
+  const void* l2_pf;      // or null: [l2_pf_bytes] brought into L2 while the block routes (a hint)
+  size_t l2_pf_bytes;     // a multiple of 16; l2_pf 16-byte aligned
   unsigned long long* stats;
   int* status;
 };

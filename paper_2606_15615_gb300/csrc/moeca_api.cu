@@ -319,6 +319,10 @@ PrepArgs prep_args_plain(const moeca_handle* h, const LayerBuf& L, const void* m
   pa.part_words = h->prep_words; pa.count_words = h->prep_words + h->prep_count_off;
   pa.counts = L.counts; pa.offsets = L.offsets; pa.list = L.list;
   pa.xg = xg; pa.stats = L.stats; pa.status = h->status_dev;
+  // The head of the routed W1, in the GEMM's expert order (a whole number of 16-byte units).
+  const size_t w1_bytes = static_cast<size_t>(c.n_experts) * c.ffn * c.hidden * h->es;
+  pa.l2_pf = L.w.w1;
+  pa.l2_pf_bytes = std::min(w1_bytes, static_cast<size_t>(c.weight_prefetch_mb) << 20) & ~size_t(15);
   return pa;
 }
 
@@ -390,6 +394,7 @@ void moeca_config_default(moeca_config* c) {
   c->keep_route_in = 0;
   c->token_reuse_policy = 0;
   c->combine_direct = 1;
+  c->weight_prefetch_mb = 16;
 }
 
 const char* moeca_status_string(moeca_status s) {
@@ -437,6 +442,8 @@ moeca_status moeca_create(const moeca_config* cfg, const moeca_layer_weights* la
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "token_reuse_policy must be 0 or 1");
   if (c.combine_direct != 0 && c.combine_direct != 1)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "combine_direct must be 0 or 1");
+  if (c.weight_prefetch_mb < 0 || c.weight_prefetch_mb > 4096)
+    return fail(nullptr, MOECA_ERR_INVALID_ARG, "weight_prefetch_mb must be in [0, 4096]");
   if (c.ffn_impl != MOECA_FFN_AUTO && c.ffn_impl != MOECA_FFN_SIMT)
     return fail(nullptr, MOECA_ERR_INVALID_ARG, "ffn_impl");
   if ((c.ffn_tile_n != 0 && c.ffn_tile_n != 64 && c.ffn_tile_n != 128 && c.ffn_tile_n != 192 &&

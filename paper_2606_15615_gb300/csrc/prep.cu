@@ -286,6 +286,11 @@ __global__ void __launch_bounds__(kThreads) prep_kernel(PrepArgs a) {
   }
   if (!mbar_wait_for(bar, 0, kBarrierNs) && t == 0) report_status(a.status, kStatusWaitTimeout, 610);
   __syncthreads();
+  // The grouped GEMM after this kernel reads the routed W1 first, expert by
+  // expert.  HBM is nearly idle while the routing, the exchanges and the
+  // decisions run, so the blocks bring its head into L2 now (a hint, issued
+  // once the block's own rows have landed so as not to delay them).
+  if (warp == 0 && a.l2_pf_bytes) l2_prefetch_share(a.l2_pf, a.l2_pf_bytes, blockIdx.x, gridDim.x, lane);
   if constexpr (kAttn) {
     if (add_a) {
       // u = x + a^{t0}: the router input, the rows the FFN gathers, and the

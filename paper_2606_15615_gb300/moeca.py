@@ -42,7 +42,8 @@ class moeca_config(C.Structure):
                 ("ffn_split_k", C.c_int32), ("score_terms", C.c_int32), ("granularity", C.c_int32),
                 ("n_heads", C.c_int32), ("seq_len", C.c_int32), ("attn_policy", C.c_int32),
                 ("attn_impl", C.c_int32), ("adaln", C.c_int32), ("ln_eps", C.c_float),
-                ("keep_route_in", C.c_int32), ("token_reuse_policy", C.c_int32), ("combine_direct", C.c_int32)]
+                ("keep_route_in", C.c_int32), ("token_reuse_policy", C.c_int32), ("combine_direct", C.c_int32),
+                ("weight_prefetch_mb", C.c_int32)]
 
 
 class moeca_layer_weights(C.Structure):
