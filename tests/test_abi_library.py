@@ -31,6 +31,9 @@ def test_status_strings_and_defaults(lib):
     assert cfg.renorm_topk == 1 and cfg.gelu_tanh == 1 and cfg.dtype == lib.MOECA_BF16
     assert cfg.score_terms == 7 and cfg.granularity == 0
     assert (cfg.n_heads, cfg.seq_len, cfg.attn_policy) == (0, 0, lib.ATTN_SYNC)
+    assert cfg.combine_direct == 1 and cfg.weight_prefetch_mb == 16
+    # The Python mirror of moeca_config ends at the header's last field.
+    assert ctypes.sizeof(lib.moeca_config) == lib.moeca_config.weight_prefetch_mb.offset + 4
 
 
 def test_host_validation_needs_no_gpu(lib):
@@ -49,6 +52,11 @@ def test_host_validation_needs_no_gpu(lib):
         c2 = lib.moeca_config_default(n_layers=1, hidden=64, ffn=64, n_experts=4, top_k=2, max_tokens=8, **bad)
         assert L.moeca_create(ctypes.byref(c2), w, 0, ctypes.byref(h)) == -1
         assert b"score_terms" in L.moeca_last_error(None)
+    for bad in (-1, 4097):
+        c2 = lib.moeca_config_default(n_layers=1, hidden=64, ffn=64, n_experts=4, top_k=2, max_tokens=8,
+                                      weight_prefetch_mb=bad)
+        assert L.moeca_create(ctypes.byref(c2), w, 0, ctypes.byref(h)) == -1
+        assert b"weight_prefetch_mb" in L.moeca_last_error(None)
     assert L.moeca_create(ctypes.byref(cfg), w, 0, ctypes.byref(h)) == -1  # NULL weights
     cfg.hidden = 60
     w[0].w_gate = w[0].w1 = w[0].w2 = 4096
