@@ -1,6 +1,6 @@
-"""The binding's ctypes mirrors of the C-ABI structs against the header itself.
+"""The binding's ctypes mirrors of the C-ABI structs against the headers themselves.
 
-A C program compiled from ``include/moeca.h`` prints ``sizeof`` and the
+A C program compiled from the headers in ``include/`` prints ``sizeof`` and the
 ``offsetof`` of every field the Python mirror names; a field added on one side
 only, or in a different place, changes an offset or the size.
 """
@@ -14,7 +14,9 @@ import pytest
 from paper_2606_15615_gb300 import moeca as M
 
 ROOT = Path(__file__).resolve().parents[1]
-STRUCTS = [("moeca_config", M.moeca_config), ("moeca_layer_weights", M.moeca_layer_weights)]
+STRUCTS = [(n, getattr(M, n)) for n in (
+    "moeca_config", "moeca_layer_weights", "moeca_step_args", "moeca_stats", "moeca_layer_state",
+    "moeca_layer_trace", "moeca_shard", "moeca_kernel_times", "moeca_route_args", "moeca_ddpm_args")]
 
 
 def test_struct_layouts_match_the_header(tmp_path):
