@@ -41,7 +41,8 @@ DEFAULT_WORKLOAD = "moe_d768_e16_k2_f3072_t2048_l12_bf16"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KINDS = ["router", "select", "compact", "ffn1", "ffn2", "combine", "prep", "ffn", "qkv", "attn", "oproj", "attn_aux",
          "adaln"]
-# Reuse points per workload index (BASELINE's sweeps) and the point each row's kernels are timed at.
+# Reuse points per workload index (the measured reuse sweep of each workload) and the point each
+# row's kernels are timed at.
 CONFIG_POINTS = {1: (0.5,), 2: (0.0, 0.3, 0.6, 0.9), 3: (0.6,), 4: (0.6,),
                  5: tuple(round(0.05 * j, 2) for j in range(20))}
 MAIN_POINT = {1: 0.5, 2: 0.6, 3: 0.6, 4: 0.6, 5: 0.6}
@@ -536,7 +537,7 @@ def point_row(runner, wl, tgt, tau0, ms, st, K, world):
 
 
 def config_row(wl, local: int, W_: int, K: int, pk, pk_src, ffma_peak):
-    """One BASELINE workload at its reuse points: tokens/s, effective TFLOP/s
+    """One benchmark workload at its reuse points: tokens/s, effective TFLOP/s
     per point, and at the main point the per-kernel times with the dominant
     kernel's roofline."""
     runner = Runner(wl, local, W_ + K)
