@@ -102,6 +102,22 @@ def test_bf16_fine_grained_64_experts_top8(M):
     st.close()
 
 
+@pytest.mark.parametrize("k,impl", [(3, "simt"), (4, "simt"), (4, "tc")])
+def test_bf16_top3_top4(M, k, impl):
+    """The kernels' middle top-k bound (k <= 4): the separate router / select /
+    compact launches (the SIMT FFN takes them), and the fused preparation
+    kernel.  The tau0 values give both reused and recomputed branches in the
+    oracle on these inputs."""
+    T, D, E, F = 233, 128, 16, 192
+    kw = {"ffn_impl": M.MOECA_FFN_SIMT} if impl == "simt" else {}
+    st, cfg, ws = make_stack(M, T, D, E, k, F, L=2, seed=21 + k, tau0={3: 0.4, 4: 0.3}[k], **kw)
+    rng = np.random.default_rng(60 + k)
+    xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05, True)
+    rep, _ = run_trajectory(st, cfg, ws, xs)
+    assert rep.reused > 0 and rep.recomputed > 0
+    st.close()
+
+
 @pytest.mark.parametrize("switch", [
     dict(entropy_norm=1), dict(reused_meta_policy=1), dict(shared_policy=1, n_shared=1),
     dict(gelu_tanh=0), dict(renorm_topk=0, tau0=0.45),
