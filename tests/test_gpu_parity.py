@@ -295,3 +295,28 @@ def test_staged_and_direct_combine_agree(M, shape):
     for sa, sb in zip(states[0], states[1]):
         for key in ("cache_norm", "cache_h", "cache_e", "cache_w"):
             assert torch.equal(sa[key], sb[key]), key
+
+
+def test_weight_prefetch_is_only_a_hint(M):
+    """The preparation kernel's L2 prefetch of the routed W1 (none, the first
+    1 MB of the 4 MB W1, and a cap above the whole W1) leaves every result
+    bit unchanged: outputs, cached norms and cache rows, over cache steps
+    with reuse."""
+    T, D, E, k, F = 300, 256, 8, 2, 1024
+    outs, states = [], []
+    for mb in (0, 1, 4096):
+        st, cfg, ws = make_stack(M, T, D, E, k, F, L=2, seed=33, tau0=0.75, weight_prefetch_mb=mb)
+        rng = np.random.default_rng(330)
+        xs = drift(rng.standard_normal((T, D)).astype(np.float32), rng, 4, 0.05, True)
+        o = [st.step(torch.from_numpy(x).cuda().to(torch.bfloat16), t).clone() for t, x in enumerate(xs)]
+        torch.cuda.synchronize()
+        outs.append(o)
+        states.append([st.get_state(l) for l in range(2)])
+        assert st.stats()["reused"] > 0
+        st.close()
+    for other in (1, 2):
+        for a, b in zip(outs[0], outs[other]):
+            assert torch.equal(a, b)
+        for sa, sb in zip(states[0], states[other]):
+            for key in ("cache_norm", "cache_h", "cache_e", "cache_w"):
+                assert torch.equal(sa[key], sb[key]), key
